@@ -1,0 +1,6 @@
+"""CPU oracle of the hot path (test infrastructure only; never imported by the product path)."""
+from .hg_oracle import *  # noqa: F401,F403
+from .hg_oracle import (  # noqa: F401
+    align_backward, align_forward, build_csr, layer_backward, layer_backward_rows, layer_forward,
+    layer_forward_rows, mean_aggregate, overlap_intersect, standardise, step, valid_edges,
+)
