@@ -1,0 +1,378 @@
+#!/usr/bin/env python
+"""Benchmark of the hot path: GNN layer forward+backward edges/s on one GB300.
+
+One step = one pass of the whole hot path over one overlapping subgraph (relation-typed CSR/CSC
+build, L layers forward, overlap intersection, alignment loss and gradient, L layers backward,
+dL/dX included).  value = L * E * steps * ranks / (max over ranks of the device time of the timed
+steps).  Inputs are seeded synthetic graphs of the named workload (default: 1M nodes, 20M edges,
+bf16 d=128, 2 layers), resident in HBM before timing; they are larger than L2, which is not
+flushed.  Multi-GPU (torchrun): every rank runs its own subgraph (weak scaling), no collective on
+the data path.  `--impl reference` times the CPU oracle on a bounded sample of the same workload.
+
+Prints one JSON line (rank 0).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import hgsynth  # noqa: E402
+
+METRIC = "GNN layer fwd+bwd edges/sec on 1 GB300; achieved HBM GB/s vs roofline"
+UNIT = "edges/s"
+ORACLE_SCALE = 40        # the CPU baseline runs the oracle on a 1/40-size instance of the workload
+REFERENCE_SCALE = 100    # each reference-arm step runs the oracle on a 1/100-size instance
+FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "sm_max_mhz": 2070.0}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="sub-1m", choices=sorted(hgsynth.WORKLOADS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--oracle-sample", type=int, default=0, help=argparse.SUPPRESS)  # internal: child process
+    return ap.parse_args()
+
+
+def scaled(spec, k: int):
+    return hgsynth.spec(spec.name, n_user=max(1, spec.n_user // k), n_risk=max(1, spec.n_risk // k),
+                        num_edges=spec.num_edges // k, n_overlap=max(2, spec.n_overlap // k))
+
+
+def workload_desc(sp) -> str:
+    return (f"{sp.name}: {sp.num_nodes:,} nodes ({sp.n_user:,} user / {sp.n_risk:,} risk), {sp.num_rels} relations, "
+            f"{sp.num_edges:,} edges, Zipf s={sp.zipf_s}, d={sp.d} {sp.dtype}, {sp.layers} layers, "
+            f"{sp.n_overlap:,} overlap rows ({sp.overlap}), second view: {sp.view_b}")
+
+
+# ------------------------------------------------------------------------------------------------
+# oracle timing (CPU baseline / reference arm); runs in a child process with one thread
+# ------------------------------------------------------------------------------------------------
+def oracle_sample_main(name: str, k: int):
+    import oracle
+    sp = scaled(hgsynth.spec(name), k)
+    w = hgsynth.make_workload(sp)
+    vb = {"idx": w.overlap_local, "X_b": w.X_b} if sp.view_b == "perturbed" else \
+        {"H_b": w.H_b, "gid_a": w.gid_a, "gid_b": w.gid_b}
+    t0 = time.perf_counter()
+    oracle.step(w.graph, w.X, w.params, w.dH_top, vb)
+    dt = time.perf_counter() - t0
+    print(json.dumps({"seconds": dt, "edges": sp.num_edges, "layers": sp.layers,
+                      "value": sp.layers * sp.num_edges / dt}))
+
+
+def time_oracle(name: str, k: int) -> dict:
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               CUDA_VISIBLE_DEVICES="")
+    r = subprocess.run([sys.executable, os.path.abspath(__file__), "--workload", name, "--oracle-sample", str(k)],
+                       capture_output=True, text=True, env=env)
+    if r.returncode != 0:
+        raise RuntimeError(f"oracle sample failed: {r.stderr[-2000:]}")
+    return json.loads(r.stdout.strip().splitlines()[-1])
+
+
+# ------------------------------------------------------------------------------------------------
+# clocks during the timed region
+# ------------------------------------------------------------------------------------------------
+class Clocks:
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.3)
+        self.proc.terminate()
+        out, _ = self.proc.communicate(timeout=10)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------------------------
+# algorithmic bytes / flops per step for each kernel (from the graph's own statistics)
+# ------------------------------------------------------------------------------------------------
+HUB, CHUNK = 512, 512
+
+
+def graph_stats(w) -> dict:
+    g = w.graph
+    sp = w.spec
+    offs = g["type_offsets"]
+    N = int(offs[-1])
+    src, dst, rel = g["src"].astype(np.int64), g["dst"].astype(np.int64), g["rel"]
+    st = dict(N=N, E=len(src), RR=0, CC=0, fwd=dict(E_nh=0, E_h=0, U_nh=0, U_h=0, chunks=0),
+              bwd=dict(E_nh=0, E_h=0, U_nh=0, U_h=0, chunks=0), types=[], rels=[])
+    for t in range(len(offs) - 1):
+        st["types"].append(dict(n=int(offs[t + 1] - offs[t]), R=sum(1 for r in g["rels"] if r[1] == t)))
+    for r, (ts, tt) in enumerate(g["rels"]):
+        m = rel == r
+        s_r, d_r = src[m], dst[m]
+        n_t, n_s = int(offs[tt + 1] - offs[tt]), int(offs[ts + 1] - offs[ts])
+        st["RR"] += n_t
+        st["CC"] += n_s
+        st["rels"].append(dict(n_t=n_t, n_s=n_s, E=int(m.sum())))
+        for key, rows, other, nrow in (("fwd", d_r, s_r, N), ("bwd", s_r, d_r, N)):
+            deg = np.bincount(rows, minlength=N)
+            hub_edge = deg[rows] > HUB
+            a = st[key]
+            a["E_h"] += int(hub_edge.sum())
+            a["E_nh"] += int((~hub_edge).sum())
+            a["U_h"] += int(np.count_nonzero(np.bincount(other[hub_edge], minlength=nrow)))
+            a["U_nh"] += int(np.count_nonzero(np.bincount(other[~hub_edge], minlength=nrow)))
+            hd = deg[deg > HUB]
+            a["chunks"] += int(((hd + CHUNK - 1) // CHUNK).sum())
+    return st
+
+
+def kernel_models(st: dict, sp) -> dict:
+    """{kernel: (bytes per step, flops per step)}: compulsory traffic (each distinct row read once,
+    every output written once, index arrays read once) and the arithmetic of the definition."""
+    b, d, L, N, RR, CC = (4 if sp.dtype == "f32" else 2), sp.d, sp.layers, st["N"], st["RR"], st["CC"]
+    f, bw = st["fwd"], st["bwd"]
+    row = d * b
+    m = {}
+    m["agg_fwd_rows"] = (L * (4 * (RR + 1) + 4 * f["E_nh"] + row * f["U_nh"] + row * RR + 4 * d * f["chunks"]), 0)
+    m["agg_fwd_chunks"] = (L * (4 * f["E_h"] + row * f["U_h"] + 4 * d * f["chunks"]), 0)
+    m["agg_bwd_nodes"] = (L * (4 * (CC + 1) + 4 * bw["E_nh"] + row * bw["U_nh"] + 2 * row * N + 4 * d * bw["chunks"]), 0)
+    m["agg_bwd_chunks"] = (L * (4 * bw["E_h"] + row * bw["U_h"] + 4 * d * bw["chunks"]), 0)
+    fb = ff = bb = bf = 0
+    for t in st["types"]:
+        n, R = t["n"], t["R"]
+        fb += n * row * (R + 4) + 8 * n
+        ff += 2 * n * d * (R * d + d)
+        bb += n * row * (6 + R) + 8 * n
+        bf += 2 * n * d * (d + R * d)
+    m["proj_fwd_simt"] = (L * fb, L * ff)
+    m["proj_bwd_simt"] = (L * bb, L * bf)
+    m["wgrad_partial"] = (L * 2 * row * (N + RR), L * 2 * d * d * (N + RR))
+    m["radix_scatter"] = (2 * 3 * 4 * 4 * st["E"], 0)  # 2 layouts x 3 passes x (read+write of key+value)
+    return m
+
+
+def load_peaks() -> tuple:
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as fh:
+            return json.load(fh), "measured"
+    return dict(FALLBACK), "fallback"
+
+
+def roofline(report: dict, models: dict, steps: int, peaks: dict, src: str) -> tuple:
+    total = sum(ms for _, ms in report.values()) or 1.0
+    shares = {k: round(ms / total, 4) for k, (_, ms) in sorted(report.items(), key=lambda kv: -kv[1][1])}
+    dom = max(report, key=lambda k: report[k][1])
+    n, ms = report[dom]
+    by, fl = models.get(dom, (0, 0))
+    secs = ms / 1e3
+    alu_peak = 152 * 128 * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12  # fp32 FMA, TFLOP/s
+    if dom.endswith("_simt") or dom == "wgrad_partial":
+        ach = fl * steps / secs / 1e12 if secs > 0 else 0.0
+        rf = dict(bound="alu", achieved=round(ach, 3), peak=round(alu_peak, 1), unit="TFLOP/s",
+                  peak_source="derived: 152 SMs x 128 fp32 lanes x 2 flop x max SM clock")
+    else:
+        ach = by * steps / secs / 1e9 if secs > 0 else 0.0
+        rf = dict(bound="hbm", achieved=round(ach, 1), peak=peaks["hbm_gbs"], unit="GB/s",
+                  peak_source=f"{src} hbm_gbs")
+    rf["frac"] = round(rf["achieved"] / rf["peak"], 4) if rf["peak"] else None
+    rf["traffic"] = None
+    rf.update(kernel=dom, launches=n, avg_launch_ms=round(ms / max(n, 1), 4),
+              algorithmic_bytes_per_launch=int(by * steps / max(n, 1)), flops_per_launch=int(fl * steps / max(n, 1)))
+    return rf, shares
+
+
+# ------------------------------------------------------------------------------------------------
+def main():
+    args = parse()
+    if args.oracle_sample:
+        oracle_sample_main(args.workload, args.oracle_sample)
+        return
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    sp = hgsynth.spec(args.workload)
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        run_reference(args, sp)
+        return
+    run_ours(args, sp, rank, world)
+
+
+def run_reference(args, sp):
+    for _ in range(args.warmup):
+        time_oracle(sp.name, REFERENCE_SCALE)
+    vals = [time_oracle(sp.name, REFERENCE_SCALE) for _ in range(args.steps)]
+    secs = sum(v["seconds"] for v in vals)
+    edges = sum(v["edges"] * v["layers"] for v in vals)
+    value = edges / secs
+    sample = (f"1/{REFERENCE_SCALE}-size instance of the workload per step "
+              f"({vals[0]['edges']:,} edges, same recipe), fp64 numpy oracle, one thread")
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": workload_desc(sp)},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+def run_ours(args, sp, rank, world):
+    import torch
+    if world > 1:
+        import torch.distributed as dist
+        local = int(os.environ.get("LOCAL_RANK", "0"))
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    from paper_2608_02168_gb300 import build as hbuild
+    hbuild.build()
+    from paper_2608_02168_gb300 import hg
+    from paper_2608_02168_gb300.step import HotPath
+
+    dev = torch.device("cuda", torch.cuda.current_device())
+    w = hgsynth.make_workload(sp, sub=rank)
+    g = w.graph
+    td = torch.float32 if sp.dtype == "f32" else torch.bfloat16
+    path = HotPath(g["type_offsets"], g["rels"], len(g["src"]), sp.d, sp.dtype, w.params, view=sp.view_b,
+                   n_overlap_max=len(w.overlap_local), n_gid_a=0 if w.gid_a is None else len(w.gid_a),
+                   n_gid_b=0 if w.gid_b is None else len(w.gid_b), device=dev)
+    host = {"src": torch.from_numpy(g["src"]), "dst": torch.from_numpy(g["dst"]), "rel": torch.from_numpy(g["rel"]),
+            "X": torch.from_numpy(w.X).to(td), "dH_top": torch.from_numpy(w.dH_top).to(td)}
+    if sp.view_b == "perturbed":
+        host.update(X_b=torch.from_numpy(w.X_b).to(td), overlap_idx=torch.from_numpy(w.overlap_local))
+    else:
+        host.update(gid_a=torch.from_numpy(w.gid_a), gid_b=torch.from_numpy(w.gid_b), H_bank=torch.from_numpy(w.H_b).to(td))
+    devin = {k: v.to(dev) for k, v in host.items()}
+    stream = torch.cuda.current_stream()
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+
+    def max_over_ranks(x: float) -> float:
+        if world == 1:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        return float(t.item())
+
+    def step(inp):
+        kw = {k: inp[k] for k in ("X_b", "overlap_idx", "gid_a", "gid_b", "H_bank") if k in inp}
+        path.step(inp["src"], inp["dst"], inp["rel"], inp["X"], inp["dH_top"], **kw)
+
+    for _ in range(max(args.warmup, 0)):
+        step(devin)
+    torch.cuda.synchronize()
+    stats = graph_stats(w)
+    models = kernel_models(stats, sp)
+    clocks = Clocks(dev.index if dev.index is not None else 0)
+    hg.hg_timing_enable(True)
+    hg.hg_timing_report()  # clear
+    clocks.start()
+    barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step(devin)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop()
+    hg.hg_timing_enable(False)
+    report = hg.hg_timing_report()
+    t = max_over_ranks(e0.elapsed_time(e1) / 1e3)
+    edges_per_step = sp.layers * sp.num_edges
+    value = world * edges_per_step * args.steps / t
+
+    # end to end: pinned host inputs copied in, the step, the loss read back, every step
+    e2e = None
+    if not args.no_e2e:
+        pinned = {k: v.pin_memory() for k, v in host.items()}
+        h2d = sum(v.numel() * v.element_size() for v in pinned.values())
+        loss_host = torch.empty(3, dtype=torch.float32).pin_memory()
+        barrier()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            for k, v in pinned.items():
+                devin[k].copy_(v, non_blocking=True)
+            step(devin)
+            loss_host.copy_(path.loss, non_blocking=True)
+            torch.cuda.synchronize()
+        te = max_over_ranks(time.perf_counter() - t0)
+        e2e = {"value": world * edges_per_step * args.steps / te, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+               "d2h_bytes_per_step": int(loss_host.numel() * 4)}
+
+    if rank != 0:
+        if world > 1:
+            torch.distributed.destroy_process_group()
+        return
+    peaks, psrc = load_peaks()
+    rf, shares = roofline(report, models, args.steps, peaks, psrc)
+    cpu = None
+    if not args.no_cpu_baseline:
+        o = time_oracle(sp.name, ORACLE_SCALE)
+        cpu = {"value": o["value"], "unit": UNIT, "cores": 1, "kind": "oracle",
+               "sample": f"1/{ORACLE_SCALE}-size instance of the workload ({o['edges']:,} edges, same recipe), one "
+                         f"full step of the fp64 numpy oracle, one thread, {o['seconds']:.1f} s"}
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * t / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": sp.dtype, "data": "synthetic",
+        "config": {"workload": workload_desc(sp), "l2": "inputs larger than L2 (not flushed)",
+                   "parallelism": f"{world} independent subgraph(s), one per GPU"},
+        "roofline": rf, "kernel_time_share": dict(list(shares.items())[:8]),
+        "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+        "gpu_launches": int(sum(n for n, _ in report.values())),
+        "loss": [float(x) for x in path.loss.cpu()],
+    }
+    print(json.dumps(out))
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

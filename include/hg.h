@@ -1,0 +1,237 @@
+/*
+ * hg.h -- C ABI of the GB300 hot path of risk-aware overlapping-subgraph GNN training.
+ *
+ * The library computes, on one GPU and on the caller's stream:
+ *   - the relation-typed adjacency of one overlapping subgraph as CSR (by destination) and CSC
+ *     (by source) per relation (Section 2.2: node types, relations, meta-relation triplets;
+ *     Section 3.1, Eq. 5 and Algorithm 1: the induced overlapping subgraph);
+ *   - the forward and backward pass of one heterogeneous message-passing layer (Eq. 7 with one
+ *     message matrix W_r per relation, Eq. 10 with the mean over each relation's neighbours,
+ *     per-relation means summed into the target, Eq. 11: per-type Linear_agg, activation,
+ *     residual; optional LayerNorm per node type after the residual);
+ *   - the overlap batch B between two subgraphs as pairs of local rows (Section 3.3);
+ *   - the cross-subgraph CCA alignment loss on B (Eq. 14-17) and its gradient.
+ *
+ * Conventions for every entry point:
+ *   - Pointers named *_dev, H_*, dH_*, idx_*, gid_*, workspace, saved, scratch, and the edge
+ *     arrays are DEVICE pointers; everything else (type_offsets, rels, sizes) is HOST memory.
+ *   - The library allocates no device memory.  All device buffers are owned by the caller; the
+ *     *_size queries give the bytes each call needs.  Buffers must be 256-byte aligned.
+ *   - Work is enqueued on `stream` (a cudaStream_t; NULL = legacy default stream).  No entry point
+ *     synchronises except hg_graph_check and hg_timing_report, which say so.
+ *   - Arguments are validated on the host before any launch.  A failed check returns a status
+ *     (never traps or aborts) and leaves a message in hg_last_error().  Device-side input
+ *     problems (an edge id out of range, unsorted global ids) never cause out-of-bounds
+ *     accesses: the offending items are dropped or flagged as documented per call.
+ *   - Node ids are local to the subgraph and contiguous per node type: type t owns ids
+ *     [type_offsets[t], type_offsets[t+1]).  Features are row-major N x d.
+ *   - Supported feature widths: d in {64, 128, 256}; dtypes HG_F32 and HG_BF16 (storage type of
+ *     features, weights and activations; arithmetic accumulates in fp32).  Edge counts < 2^31.
+ */
+#ifndef HG_H_
+#define HG_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* hg_stream; /* identical to cudaStream_t */
+
+typedef enum {
+  HG_OK = 0,
+  HG_ERR_INVALID_ARG = 1,  /* null pointer, bad size, mismatched shapes */
+  HG_ERR_UNSUPPORTED = 2,  /* valid request outside what the kernels handle (d, dtype, > 2^31 edges) */
+  HG_ERR_WORKSPACE = 3,    /* caller buffer smaller than the matching *_size query */
+  HG_ERR_CUDA = 4,         /* a CUDA runtime call or launch failed */
+  HG_ERR_DEVICE_CHECK = 5, /* a device-side input check failed (reported by hg_graph_check) */
+  HG_ERR_TIMEOUT = 6       /* reserved for bounded waits; no kernel of this library waits */
+} hg_status;
+
+typedef enum { HG_F32 = 0, HG_BF16 = 1 } hg_dtype;
+typedef enum { HG_ACT_RELU = 0, HG_ACT_GELU_TANH = 1, HG_ACT_NONE = 2 } hg_act;
+
+/* Relation r connects a source node of type src_type to a destination node of type dst_type
+ * (the meta-relation triplet <tau(i), phi(e), tau(j)> of Section 2.2). */
+typedef struct {
+  int32_t src_type;
+  int32_t dst_type;
+} hg_rel_desc;
+
+typedef struct hg_graph hg_graph; /* opaque host handle; its arrays live in the caller's workspace */
+
+/* Static description of a status code. */
+const char* hg_status_string(hg_status status);
+/* Detail of the last failure on the calling thread ("" if none).  Valid until the next call. */
+const char* hg_last_error(void);
+/* Version of this ABI (bumped on any incompatible change). */
+int32_t hg_abi_version(void);
+
+/* ------------------------------------------------------------------------------------------- */
+/* Graph layout (Section 2.2, Section 3.1 / Eq. 5: the adjacency of one overlapping subgraph)   */
+/* ------------------------------------------------------------------------------------------- */
+
+/* Bytes of device workspace hg_build_csr needs for this many edges and these types/relations. */
+hg_status hg_graph_workspace_size(int64_t num_edges, const int64_t* type_offsets, int32_t num_types,
+                                  const hg_rel_desc* rels, int32_t num_rels, size_t* bytes);
+
+/* Builds, on the device, per relation r: CSR by destination (rows = destination nodes of type
+ * rels[r].dst_type in local order; each row lists its in-edges in ascending input edge id) and CSC
+ * by source (rows = source nodes of type rels[r].src_type; out-edges in ascending edge id), plus
+ * the per-CSC-edge coefficient 1/deg_r(destination) as an IEEE fp32 quotient, and the split tables
+ * the aggregation kernels use for high-degree rows.
+ *   src, dst, rel : device int32 arrays of num_edges entries (COO, any order).
+ *   type_offsets  : host int64 [num_types + 1], type_offsets[0] = 0, non-decreasing.
+ *   rels          : host [num_rels].
+ *   workspace     : device buffer of at least hg_graph_workspace_size bytes, owned by the caller
+ *                   and kept alive (and unmodified) for the lifetime of the graph.
+ *   out           : receives a host handle; release it with hg_graph_destroy.
+ * Edges with an id out of range, a relation out of range, or endpoint types that differ from their
+ * relation are dropped (never dereferenced out of bounds); hg_graph_check reports how many.
+ * The src/dst/rel arrays may be freed once the work on `stream` has completed. */
+hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const int32_t* rel, int64_t num_edges,
+                       const int64_t* type_offsets, int32_t num_types, const hg_rel_desc* rels,
+                       int32_t num_rels, void* workspace, size_t workspace_bytes, hg_stream stream,
+                       hg_graph** out);
+
+/* Releases the host handle (the workspace stays with the caller).  NULL is accepted. */
+hg_status hg_graph_destroy(hg_graph* graph);
+
+/* SYNCHRONISES the graph's build stream.  Writes the number of dropped (invalid) edges; returns
+ * HG_ERR_DEVICE_CHECK if it is non-zero, HG_OK otherwise. */
+hg_status hg_graph_check(const hg_graph* graph, int64_t* num_invalid_edges);
+
+/* Read-only device views of one relation's layout (for tests and for callers that want the CSR).
+ * row_ptr has n_dst + 1 entries and csc_ptr n_src + 1 entries; their values index the col/eid and
+ * csc_col/csc_eid/csc_coef arrays directly (relations are stored one after another).
+ * col holds source node ids, csc_col destination node ids, eid/csc_eid input edge ids. */
+typedef struct {
+  int64_t n_dst, n_src, num_edges;
+  const int32_t* row_ptr;
+  const int32_t* col;
+  const int32_t* eid;
+  const int32_t* csc_ptr;
+  const int32_t* csc_col;
+  const int32_t* csc_eid;
+  const float* csc_coef;
+} hg_graph_arrays;
+hg_status hg_graph_view(const hg_graph* graph, int32_t rel, hg_graph_arrays* out);
+
+/* ------------------------------------------------------------------------------------------- */
+/* Layer (Eq. 7, Eq. 10 with mean aggregation, Eq. 11, optional LayerNorm)                      */
+/* ------------------------------------------------------------------------------------------- */
+
+/* Layer parameters, packed device arrays in `dtype`:
+ *   W_rel    [num_rels  x d x d]  message matrix of relation r, row-major (d_in x d_out)
+ *   W_agg    [num_types x d x d]  Linear_agg of the target type, row-major (d_in x d_out)
+ *   b_agg    [num_types x d]
+ *   ln_gamma [num_types x d], ln_beta [num_types x d]  (read only when layernorm != 0)
+ * For destination node j of type t:
+ *   Z[j]     = sum over relations r into t of M_r[j] W_rel[r],
+ *   M_r[j]   = mean of H_in over j's in-neighbours under r (0 when j has none),
+ *   U[j]     = Z[j] W_agg[t] + b_agg[t],
+ *   Y[j]     = act(U[j]) + H_in[j],
+ *   H_out[j] = layernorm ? (Y[j] - mean) / sqrt(var + ln_eps) * ln_gamma[t] + ln_beta[t] : Y[j]
+ * (population variance over the d features of the row). */
+typedef struct {
+  int32_t d;
+  hg_dtype dtype;
+  hg_act act;
+  int32_t layernorm;
+  float ln_eps;
+  const void* W_rel;
+  const void* W_agg;
+  const void* b_agg;
+  const void* ln_gamma;
+  const void* ln_beta;
+} hg_layer_params;
+
+/* Gradients, fp32 device arrays with the shapes of the parameters; OVERWRITTEN by hg_layer_bwd.
+ * dln_gamma / dln_beta may be NULL when layernorm == 0. */
+typedef struct {
+  float* dW_rel;
+  float* dW_agg;
+  float* db_agg;
+  float* dln_gamma;
+  float* dln_beta;
+} hg_layer_grads;
+
+/* Bytes of the `saved` buffer (written by hg_layer_fwd, read by hg_layer_bwd) and of the `scratch`
+ * buffer (contents undefined between calls) one layer of this graph needs. */
+hg_status hg_layer_workspace_size(const hg_graph* graph, const hg_layer_params* params,
+                                  size_t* saved_bytes, size_t* scratch_bytes);
+
+/* Forward pass.  H_in, H_out: N x d in params->dtype (N = type_offsets[num_types]); they must not
+ * overlap.  saved: keeps what the backward pass needs (per-relation means, Z, U, row statistics). */
+hg_status hg_layer_fwd(const hg_graph* graph, const hg_layer_params* params, const void* H_in,
+                       void* H_out, void* saved, void* scratch, hg_stream stream);
+
+/* Backward pass of the layer whose forward wrote `saved` from the same H_in and params.
+ *   dH_out : N x d upstream gradient (dtype).
+ *   dH_in  : N x d, OVERWRITTEN with dL/dH_in (residual path plus the transposed aggregation);
+ *            NULL skips that part (then only the weight gradients are produced).
+ *   grads  : weight gradients, OVERWRITTEN. */
+hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* params, const void* H_in,
+                       const void* saved, const void* dH_out, void* dH_in, const hg_layer_grads* grads,
+                       void* scratch, hg_stream stream);
+
+/* ------------------------------------------------------------------------------------------- */
+/* Overlap batch (Section 3.3) and CCA alignment (Eq. 14-17)                                     */
+/* ------------------------------------------------------------------------------------------- */
+
+hg_status hg_overlap_intersect_workspace_size(int64_t n_a, int64_t n_b, size_t* bytes);
+
+/* B = the nodes present in both subgraphs.  gid_a [n_a], gid_b [n_b]: device int64 global ids of
+ * each subgraph's local rows, STRICTLY ASCENDING (local ids follow global-id order).  Writes, for
+ * k < *n_out, idx_a[k] / idx_b[k] = local rows of the k-th common node in ascending global id;
+ * idx_a and idx_b need min(n_a, n_b) entries.  n_out: device int64 scalar; it is set to -1 if
+ * either list is not strictly ascending (then idx_* are unspecified). */
+hg_status hg_overlap_intersect(const int64_t* gid_a, int64_t n_a, const int64_t* gid_b, int64_t n_b,
+                               int32_t* idx_a, int32_t* idx_b, int64_t* n_out, void* scratch,
+                               size_t scratch_bytes, hg_stream stream);
+
+/* Buffer sizes for the alignment calls with at most n_max overlap rows of width d. */
+hg_status hg_overlap_align_workspace_size(int64_t n_max, int32_t d, size_t* saved_bytes,
+                                          size_t* scratch_bytes);
+
+/* Alignment loss between rows H_a[idx_a[k]] and H_b[idx_b[k]], k < n (H_a has rows_a rows,
+ * H_b rows_b rows):
+ *   Z = (X - mean) / (sqrt(var + var_eps) * sqrt(n)) per column (population variance, Eq. 14),
+ *   loss_out[1] = L_inv = ||Z_a - Z_b||_F^2                                         (Eq. 15)
+ *   loss_out[2] = L_dec = ||Z_a^T Z_a - I||_F^2 + ||Z_b^T Z_b - I||_F^2              (Eq. 16)
+ *   loss_out[0] = L_inv + lambda_n * L_dec                                           (Eq. 17)
+ * H_a, H_b: row-major, d columns, dtype.  idx_a, idx_b: device int32 [n_max]; each list must
+ * hold distinct rows.  An index outside [0, rows) is never dereferenced: it is clamped, the loss
+ * becomes NaN and hg_overlap_align_bwd then writes no gradient.  n_dev: optional device int64 with the actual n (<= n_max), e.g. the n_out
+ * of hg_overlap_intersect, so no host round trip is needed; NULL means n = n_max.  n < 2 gives a
+ * zero loss.  loss_out: device fp32 [3].  saved: kept for hg_overlap_align_bwd. */
+hg_status hg_overlap_align_loss(const void* H_a, int64_t rows_a, const int32_t* idx_a, const void* H_b,
+                                int64_t rows_b, const int32_t* idx_b, int64_t n_max, const int64_t* n_dev,
+                                int32_t d, hg_dtype dtype, float lambda_n, float var_eps, float* loss_out,
+                                void* saved, void* scratch, hg_stream stream);
+
+/* Gradient of dloss * L (dloss = lambda_CCA of Eq. 20 in training) with respect to the overlap
+ * rows, ACCUMULATED into dH_a[idx_a[k]] and dH_b[idx_b[k]] (dtype, same layout as H_a / H_b).
+ * dH_b may be NULL (a detached view, e.g. embeddings received from another subgraph); dH_a may be
+ * NULL too.  `saved` must come from hg_overlap_align_loss on the same inputs. */
+hg_status hg_overlap_align_bwd(const void* H_a, int64_t rows_a, const int32_t* idx_a, const void* H_b,
+                               int64_t rows_b, const int32_t* idx_b, int64_t n_max, const int64_t* n_dev,
+                               int32_t d, hg_dtype dtype, float lambda_n, float var_eps, float dloss,
+                               const void* saved, void* dH_a, void* dH_b, void* scratch, hg_stream stream);
+
+/* ------------------------------------------------------------------------------------------- */
+/* Kernel timing (measurement support; off by default)                                          */
+/* ------------------------------------------------------------------------------------------- */
+
+/* When on, every kernel launch of this library is bracketed by CUDA events on its stream. */
+hg_status hg_timing_enable(int32_t on);
+/* SYNCHRONISES on the recorded events, then writes one line per kernel name,
+ * "name launches total_ms\n", into buf (truncated to len) and clears the record. */
+hg_status hg_timing_report(char* buf, size_t len);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* HG_H_ */

@@ -1,0 +1,254 @@
+// Per-relation mean aggregation (Eq. 10 with the mean as the aggregation operator) and its
+// transpose for the backward pass.
+//
+// Forward:  M_r[j] = (1/deg_r(j)) * sum_{(i -> j) in r} H[i]          (CSR row j of relation r)
+// Backward: dH[i]  = dY[i] + sum_r sum_{(i -> j) in r} dMs_r[j]         (CSC row i of relation r)
+//           where dMs_r[j] = dM_r[j] / deg_r(j) is produced, already scaled, by the projection
+//           backward kernel, and dY[i] is the residual-path gradient of Eq. 11.
+//
+// Mapping: one group of G lanes per row, each lane owning 16-byte slices of the feature row
+// (G = d * sizeof(T) / 16, at most 32), gathers with 128-bit loads and four neighbour rows in
+// flight, fp32 accumulation.  Rows above kHubDegree edges are split into kChunkEdges-edge chunks:
+// a whole CTA reduces one chunk (its groups interleave over the chunk's edges, then combine in
+// group order), writes an fp32 partial, and the row kernel adds the partials in chunk order.
+// Every sum has a fixed order, so results are bitwise reproducible run to run.
+#include <algorithm>
+
+#include "layer_kernels.cuh"
+
+namespace hg {
+
+template <typename T, int D>
+struct AggShape {
+  static constexpr int kVec = VecTraits<T>::kElems;  // elements per 16 bytes
+  static constexpr int kRowVecs = D / kVec;          // 16-byte vectors per row
+  static constexpr int G = kRowVecs < 32 ? kRowVecs : 32;
+  static constexpr int V = kRowVecs / G;  // vectors per lane
+  static constexpr int F = V * kVec;      // fp32 accumulators per lane
+  static constexpr int kThreads = 256;
+  static constexpr int kGroups = kThreads / G;
+};
+
+// acc += sum of rows src[col[e] + delta] for e = beg, beg + stride, ... < end
+template <typename T, int D>
+__device__ __forceinline__ void gather_sum(const int32_t* __restrict__ col, int64_t beg, int64_t end,
+                                           int stride, int64_t delta, const T* __restrict__ src,
+                                           int lane, float* acc) {
+  using S = AggShape<T, D>;
+  int64_t e = beg;
+  for (; e + 3 * (int64_t)stride < end; e += 4 * (int64_t)stride) {
+    int64_t c[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) c[u] = (int64_t)__ldg(col + e + u * stride) + delta;
+    uint4 x[4][S::V];
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+      for (int v = 0; v < S::V; ++v) x[u][v] = ldg16(src + c[u] * D + (lane + v * S::G) * S::kVec);
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+      for (int v = 0; v < S::V; ++v) {
+        float f[S::kVec];
+        unpack(x[u][v], f, T());
+#pragma unroll
+        for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] += f[q];
+      }
+  }
+  for (; e < end; e += stride) {
+    const int64_t c = (int64_t)__ldg(col + e) + delta;
+#pragma unroll
+    for (int v = 0; v < S::V; ++v) {
+      float f[S::kVec];
+      unpack(ldg16(src + c * D + (lane + v * S::G) * S::kVec), f, T());
+#pragma unroll
+      for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] += f[q];
+    }
+  }
+}
+
+template <typename T, int D>
+__device__ __forceinline__ void add_partials(const float* __restrict__ partials, int c0, int c1, int lane,
+                                             float* acc) {
+  using S = AggShape<T, D>;
+  for (int c = c0; c < c1; ++c) {
+#pragma unroll
+    for (int v = 0; v < S::V; ++v) {
+      const float4* p = reinterpret_cast<const float4*>(partials + (int64_t)c * D + (lane + v * S::G) * S::kVec);
+#pragma unroll
+      for (int q = 0; q < S::kVec / 4; ++q) {
+        float4 x = p[q];
+        acc[v * S::kVec + 4 * q + 0] += x.x;
+        acc[v * S::kVec + 4 * q + 1] += x.y;
+        acc[v * S::kVec + 4 * q + 2] += x.z;
+        acc[v * S::kVec + 4 * q + 3] += x.w;
+      }
+    }
+  }
+}
+
+template <typename T, int D>
+__device__ __forceinline__ void store_row(T* __restrict__ dst, int lane, const float* acc, float scale) {
+  using S = AggShape<T, D>;
+#pragma unroll
+  for (int v = 0; v < S::V; ++v) {
+    float f[S::kVec];
+#pragma unroll
+    for (int q = 0; q < S::kVec; ++q) f[q] = acc[v * S::kVec + q] * scale;
+    st16(dst + (lane + v * S::G) * S::kVec, pack(f, T()));
+  }
+}
+
+// One CTA per chunk (grid-stride over the chunk list): fp32 partial sum of the chunk's rows.
+// rel_of_row: for CSC chunks the relation decides the index shift applied to csc_col.
+template <typename T, int D>
+__global__ void __launch_bounds__(256) agg_chunks(const int32_t* __restrict__ ptr, const int32_t* __restrict__ col,
+                                                  const T* __restrict__ src, const int32_t* __restrict__ chunk_row,
+                                                  const int32_t* __restrict__ chunk_ofs, int64_t rows,
+                                                  GraphMeta m, int transposed, float* __restrict__ partials) {
+  using S = AggShape<T, D>;
+  __shared__ float red[S::kGroups][D];
+  const int grp = threadIdx.x / S::G, lane = threadIdx.x % S::G;
+  const int nchunks = chunk_ofs[rows];
+  for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
+    const int row = chunk_row[c];
+    const int64_t beg = (int64_t)ptr[row] + (int64_t)(c - chunk_ofs[row]) * kChunkEdges;
+    const int64_t end = min((int64_t)ptr[row + 1], beg + kChunkEdges);
+    int64_t delta = 0;
+    if (transposed) {
+      int r = 0;
+#pragma unroll
+      for (int k = 1; k < kMaxRels; ++k)
+        if (k < m.num_rels && row >= m.csc_base[k]) r = k;
+      delta = m.row_base[r] - m.type_off[m.rel_dst[r]];
+    }
+    float acc[S::F];
+#pragma unroll
+    for (int q = 0; q < S::F; ++q) acc[q] = 0.f;
+    gather_sum<T, D>(col, beg + grp, end, S::kGroups, delta, src, lane, acc);
+#pragma unroll
+    for (int v = 0; v < S::V; ++v)
+#pragma unroll
+      for (int q = 0; q < S::kVec; ++q) red[grp][(lane + v * S::G) * S::kVec + q] = acc[v * S::kVec + q];
+    __syncthreads();
+    for (int k = threadIdx.x; k < D; k += blockDim.x) {
+      float s = 0.f;
+#pragma unroll
+      for (int g = 0; g < S::kGroups; ++g) s += red[g][k];
+      partials[(int64_t)c * D + k] = s;
+    }
+    __syncthreads();
+  }
+}
+
+// Forward rows: M[row] = mean over the row's neighbours (concatenated CSR rows of all relations).
+template <typename T, int D>
+__global__ void __launch_bounds__(256) agg_fwd_rows(const int32_t* __restrict__ ptr, const int32_t* __restrict__ col,
+                                                    const T* __restrict__ H, T* __restrict__ M, int64_t rows,
+                                                    const int32_t* __restrict__ chunk_ofs,
+                                                    const float* __restrict__ partials) {
+  using S = AggShape<T, D>;
+  const int grp = threadIdx.x / S::G, lane = threadIdx.x % S::G;
+  const int64_t row = (int64_t)blockIdx.x * S::kGroups + grp;
+  if (row >= rows) return;
+  const int beg = ptr[row], end = ptr[row + 1], deg = end - beg;
+  float acc[S::F];
+#pragma unroll
+  for (int q = 0; q < S::F; ++q) acc[q] = 0.f;
+  if (deg > kHubDegree)
+    add_partials<T, D>(partials, chunk_ofs[row], chunk_ofs[row + 1], lane, acc);
+  else
+    gather_sum<T, D>(col, beg, end, 1, 0, H, lane, acc);
+  const float scale = deg > 0 ? __fdiv_rn(1.0f, (float)deg) : 0.f;
+  store_row<T, D>(M + row * D, lane, acc, scale);
+}
+
+// Backward nodes: dH[i] = dY[i] + sum over relations with source type tau(i) of the CSC row sums.
+template <typename T, int D>
+__global__ void __launch_bounds__(256) agg_bwd_nodes(GraphMeta m, const int32_t* __restrict__ cptr,
+                                                     const int32_t* __restrict__ ccol, const T* __restrict__ dMs,
+                                                     const T* __restrict__ dY, T* __restrict__ dH,
+                                                     const int32_t* __restrict__ chunk_ofs,
+                                                     const float* __restrict__ partials) {
+  using S = AggShape<T, D>;
+  const int grp = threadIdx.x / S::G, lane = threadIdx.x % S::G;
+  const int64_t node = (int64_t)blockIdx.x * S::kGroups + grp;
+  if (node >= m.type_off[m.num_types]) return;
+  const int t = node_type_of(m, node);
+  float acc[S::F];
+#pragma unroll
+  for (int v = 0; v < S::V; ++v) {
+    float f[S::kVec];
+    unpack(ldg16(dY + node * D + (lane + v * S::G) * S::kVec), f, T());
+#pragma unroll
+    for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] = f[q];
+  }
+  for (int r = 0; r < m.num_rels; ++r) {
+    if (m.rel_src[r] != t) continue;
+    const int64_t crow = m.csc_base[r] + (node - m.type_off[t]);
+    const int beg = cptr[crow], end = cptr[crow + 1];
+    if (end - beg > kHubDegree)
+      add_partials<T, D>(partials, chunk_ofs[crow], chunk_ofs[crow + 1], lane, acc);
+    else
+      gather_sum<T, D>(ccol, beg, end, 1, m.row_base[r] - m.type_off[m.rel_dst[r]], dMs, lane, acc);
+  }
+  store_row<T, D>(dH + node * D, lane, acc, 1.0f);
+}
+
+// ---------------------------------------------------------------------------------------------
+// host dispatch
+// ---------------------------------------------------------------------------------------------
+static unsigned chunk_grid(int64_t cap) { return (unsigned)std::max<int64_t>(1, std::min<int64_t>(cap, 152 * 8)); }
+
+template <typename T, int D>
+static hg_status agg_fwd_t(const hg_graph* g, const void* H, void* M, float* partials, cudaStream_t s) {
+  using S = AggShape<T, D>;
+  HG_TRY(launch("agg_fwd_chunks", agg_chunks<T, D>, dim3(chunk_grid(g->chunk_cap_csr)), dim3(256), 0, s,
+                (const int32_t*)g->csr_ptr, (const int32_t*)g->csr_col, (const T*)H,
+                (const int32_t*)g->csr_chunk_row, (const int32_t*)g->csr_chunk_ofs, g->csr_rows, g->meta, 0,
+                partials));
+  return launch("agg_fwd_rows", agg_fwd_rows<T, D>, dim3((unsigned)ceil_div(g->csr_rows, S::kGroups)), dim3(256),
+                0, s, (const int32_t*)g->csr_ptr, (const int32_t*)g->csr_col, (const T*)H, (T*)M, g->csr_rows,
+                (const int32_t*)g->csr_chunk_ofs, (const float*)partials);
+}
+
+template <typename T, int D>
+static hg_status agg_bwd_t(const hg_graph* g, const void* dMs, const void* dY, void* dH, float* partials,
+                           cudaStream_t s) {
+  using S = AggShape<T, D>;
+  HG_TRY(launch("agg_bwd_chunks", agg_chunks<T, D>, dim3(chunk_grid(g->chunk_cap_csc)), dim3(256), 0, s,
+                (const int32_t*)g->csc_ptr, (const int32_t*)g->csc_col, (const T*)dMs,
+                (const int32_t*)g->csc_chunk_row, (const int32_t*)g->csc_chunk_ofs, g->csc_rows, g->meta, 1,
+                partials));
+  const int64_t N = g->meta.type_off[g->meta.num_types];
+  return launch("agg_bwd_nodes", agg_bwd_nodes<T, D>, dim3((unsigned)ceil_div(N, S::kGroups)), dim3(256), 0, s,
+                g->meta, (const int32_t*)g->csc_ptr, (const int32_t*)g->csc_col, (const T*)dMs, (const T*)dY,
+                (T*)dH, (const int32_t*)g->csc_chunk_ofs, (const float*)partials);
+}
+
+#define HG_DISPATCH_TD(dtype, d, FN, ...)                                                   \
+  do {                                                                                      \
+    if (dtype == HG_F32) {                                                                  \
+      if (d == 64) return FN<float, 64>(__VA_ARGS__);                                       \
+      if (d == 128) return FN<float, 128>(__VA_ARGS__);                                     \
+      if (d == 256) return FN<float, 256>(__VA_ARGS__);                                     \
+    } else {                                                                                \
+      if (d == 64) return FN<__nv_bfloat16, 64>(__VA_ARGS__);                               \
+      if (d == 128) return FN<__nv_bfloat16, 128>(__VA_ARGS__);                             \
+      if (d == 256) return FN<__nv_bfloat16, 256>(__VA_ARGS__);                             \
+    }                                                                                       \
+    set_error("unsupported feature width %d", d);                                           \
+    return HG_ERR_UNSUPPORTED;                                                              \
+  } while (0)
+
+hg_status aggregate_forward(const hg_graph* g, hg_dtype dt, int d, const void* H, void* M, float* partials,
+                            cudaStream_t s) {
+  HG_DISPATCH_TD(dt, d, agg_fwd_t, g, H, M, partials, s);
+}
+
+hg_status aggregate_backward(const hg_graph* g, hg_dtype dt, int d, const void* dMs, const void* dY, void* dH,
+                             float* partials, cudaStream_t s) {
+  HG_DISPATCH_TD(dt, d, agg_bwd_t, g, dMs, dY, dH, partials, s);
+}
+
+}  // namespace hg

@@ -1,0 +1,531 @@
+// Relation-typed CSR / CSC construction on the device.
+//
+// The adjacency of one overlapping subgraph (Section 2.2 typed relations; Section 3.1, Eq. 5 and
+// Algorithm 1: the induced subgraph of V_k extended by the sampled candidates) is laid out per
+// relation twice: by destination (CSR, forward aggregation of Eq. 10) and by source (CSC, its
+// transpose in the backward pass).  Rows of all relations are concatenated: relation r owns CSR
+// rows [row_base[r], row_base[r+1]) = its destination type's nodes in local order, and CSC rows
+// [csc_base[r], csc_base[r+1]) = its source type's nodes.
+//
+// Construction: each edge gets a row key (or a sentinel key past the last row when invalid), the
+// row degrees are counted with integer atomics (order-free) and scanned into row pointers, and a
+// STABLE least-significant-digit radix sort of (key, edge id) places every edge in its row with
+// ascending edge ids.  The layout is therefore unique and bit-reproducible.
+#include <algorithm>
+
+#include "hg_internal.cuh"
+
+namespace hg {
+
+// ---------------------------------------------------------------------------------------------
+// exclusive scan (int32), three phases: tile sums -> scan of tile sums (recursive) -> tile scan
+// ---------------------------------------------------------------------------------------------
+constexpr int kScanThreads = 256;
+constexpr int kScanItems = 8;
+constexpr int kScanTile = kScanThreads * kScanItems;
+
+__device__ __forceinline__ int warp_inclusive_scan(int v) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    int y = __shfl_up_sync(0xffffffffu, v, o);
+    if (lane >= o) v += y;
+  }
+  return v;
+}
+
+// Exclusive block scan of one value per thread; *total receives the block total.
+__device__ __forceinline__ int block_exclusive_scan(int v, int* total) {
+  __shared__ int warp_tot[33];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  int incl = warp_inclusive_scan(v);
+  if (lane == 31) warp_tot[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    int x = lane < nwarps ? warp_tot[lane] : 0;
+    int xi = warp_inclusive_scan(x);
+    if (lane < nwarps) warp_tot[lane] = xi - x;
+    if (lane == 31) warp_tot[32] = xi;
+  }
+  __syncthreads();
+  int r = warp_tot[warp] + incl - v;
+  *total = warp_tot[32];
+  __syncthreads();
+  return r;
+}
+
+__global__ void scan_tile_sums(const int32_t* __restrict__ in, int64_t n, int32_t* __restrict__ sums) {
+  const int64_t base = (int64_t)blockIdx.x * kScanTile + (int64_t)threadIdx.x * kScanItems;
+  int s = 0;
+#pragma unroll
+  for (int i = 0; i < kScanItems; ++i)
+    if (base + i < n) s += in[base + i];
+  int total;
+  block_exclusive_scan(s, &total);
+  if (threadIdx.x == 0) sums[blockIdx.x] = total;
+}
+
+// tile_off == nullptr: a single tile starting at 0.  Writes out[n] = grand total from the last tile.
+__global__ void scan_tiles(const int32_t* in, int32_t* out, int64_t n, const int32_t* __restrict__ tile_off) {
+  const int64_t base = (int64_t)blockIdx.x * kScanTile + (int64_t)threadIdx.x * kScanItems;
+  int v[kScanItems];
+  int s = 0;
+#pragma unroll
+  for (int i = 0; i < kScanItems; ++i) {
+    v[i] = base + i < n ? in[base + i] : 0;
+    s += v[i];
+  }
+  int total;
+  int run = block_exclusive_scan(s, &total) + (tile_off ? tile_off[blockIdx.x] : 0);
+#pragma unroll
+  for (int i = 0; i < kScanItems; ++i) {
+    if (base + i < n) out[base + i] = run;
+    run += v[i];
+  }
+  if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0)
+    out[n] = (tile_off ? tile_off[blockIdx.x] : 0) + total;
+}
+
+size_t scan_scratch_bytes(int64_t n) {
+  size_t b = 0;
+  while (n > kScanTile) {
+    n = ceil_div(n, kScanTile);
+    b += align_up((size_t)(n + 1) * sizeof(int32_t));
+  }
+  return b + 256;
+}
+
+hg_status exclusive_scan(const int32_t* in, int32_t* out, int64_t n, void* scratch, cudaStream_t s) {
+  if (n <= 0) {
+    if (n == 0) HG_CUDA(cudaMemsetAsync(out, 0, sizeof(int32_t), s));
+    return HG_OK;
+  }
+  if (n <= kScanTile)
+    return launch("scan_tiles", scan_tiles, dim3(1), dim3(kScanThreads), 0, s, in, out, n,
+                  (const int32_t*)nullptr);
+  const int64_t tiles = ceil_div(n, kScanTile);
+  int32_t* sums = static_cast<int32_t*>(scratch);
+  char* rest = static_cast<char*>(scratch) + align_up((size_t)(tiles + 1) * sizeof(int32_t));
+  HG_TRY(launch("scan_tile_sums", scan_tile_sums, dim3((unsigned)tiles), dim3(kScanThreads), 0, s,
+                in, n, sums));
+  HG_TRY(exclusive_scan(sums, sums, tiles, rest, s));
+  return launch("scan_tiles", scan_tiles, dim3((unsigned)tiles), dim3(kScanThreads), 0, s, in, out,
+                n, (const int32_t*)sums);
+}
+
+// ---------------------------------------------------------------------------------------------
+// stable LSD radix sort of (uint32 key, uint32 value) pairs, 8-bit digits
+// ---------------------------------------------------------------------------------------------
+constexpr int kSortThreads = 256;
+constexpr int kSortWarps = kSortThreads / 32;
+constexpr int kSortItems = 16;                          // per thread
+constexpr int kSortTile = kSortThreads * kSortItems;    // 4096 per block
+constexpr int kRadix = 256;
+
+__global__ void __launch_bounds__(kSortThreads) radix_hist(const uint32_t* __restrict__ keys, int64_t n,
+                                                           int shift, int32_t* __restrict__ hist,
+                                                           int64_t tiles) {
+  __shared__ int h[kRadix];
+  h[threadIdx.x] = 0;
+  __syncthreads();
+  const int64_t base = (int64_t)blockIdx.x * kSortTile;
+#pragma unroll 4
+  for (int i = 0; i < kSortItems; ++i) {
+    int64_t idx = base + (int64_t)i * kSortThreads + threadIdx.x;
+    if (idx < n) atomicAdd(&h[(keys[idx] >> shift) & (kRadix - 1)], 1);
+  }
+  __syncthreads();
+  hist[(int64_t)threadIdx.x * tiles + blockIdx.x] = h[threadIdx.x];
+}
+
+// Each warp owns a contiguous 512-item slice of the tile and walks it 32 items at a time, so the
+// item order inside the tile is (warp, round, lane).  Ranks among equal digits come from
+// __match_any_sync within a round plus per-warp running counts, then an exclusive prefix over
+// warps, then the tile's global base per digit: equal keys keep their input order (stable).
+__global__ void __launch_bounds__(kSortThreads) radix_scatter(
+    const uint32_t* __restrict__ keys_in, const uint32_t* __restrict__ vals_in,
+    uint32_t* __restrict__ keys_out, uint32_t* __restrict__ vals_out, int64_t n, int shift,
+    const int32_t* __restrict__ offs, int64_t tiles) {
+  __shared__ int whist[kSortWarps][kRadix];
+  __shared__ int base[kRadix];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  for (int i = threadIdx.x; i < kSortWarps * kRadix; i += kSortThreads) (&whist[0][0])[i] = 0;
+  base[threadIdx.x] = offs[(int64_t)threadIdx.x * tiles + blockIdx.x];
+  __syncthreads();
+  const unsigned lt_mask = (1u << lane) - 1u;
+  const int64_t slice = (int64_t)blockIdx.x * kSortTile + (int64_t)warp * (kSortItems * 32);
+  uint32_t k[kSortItems], v[kSortItems];
+  int rank[kSortItems], dg[kSortItems];
+#pragma unroll
+  for (int it = 0; it < kSortItems; ++it) {
+    const int64_t idx = slice + it * 32 + lane;
+    const bool ok = idx < n;
+    k[it] = ok ? keys_in[idx] : 0u;
+    v[it] = ok ? vals_in[idx] : 0u;
+    const int d = ok ? (int)((k[it] >> shift) & (kRadix - 1)) : kRadix;
+    const unsigned peers = __match_any_sync(0xffffffffu, d);
+    const int cnt = d < kRadix ? whist[warp][d] : 0;
+    __syncwarp();
+    if (d < kRadix && lane == __ffs(peers) - 1) whist[warp][d] = cnt + __popc(peers);
+    __syncwarp();
+    rank[it] = cnt + __popc(peers & lt_mask);
+    dg[it] = d;
+  }
+  __syncthreads();
+  {
+    int run = 0;
+#pragma unroll
+    for (int w = 0; w < kSortWarps; ++w) {
+      int c = whist[w][threadIdx.x];
+      whist[w][threadIdx.x] = run;
+      run += c;
+    }
+  }
+  __syncthreads();
+#pragma unroll
+  for (int it = 0; it < kSortItems; ++it) {
+    if (dg[it] < kRadix) {
+      const int64_t pos = (int64_t)base[dg[it]] + whist[warp][dg[it]] + rank[it];
+      keys_out[pos] = k[it];
+      vals_out[pos] = v[it];
+    }
+  }
+}
+
+struct SortBuffers {
+  uint32_t* keys[2];
+  uint32_t* vals[2];
+  int32_t* hist;
+  void* scan_scratch;
+};
+
+static int64_t sort_tiles(int64_t n) { return std::max<int64_t>(1, ceil_div(n, kSortTile)); }
+
+// Sorts keys[0]/vals[0] by the low `bits` key bits; returns the buffer index holding the result.
+static hg_status radix_sort(SortBuffers& b, int64_t n, int bits, cudaStream_t s, int* result) {
+  int cur = 0;
+  const int64_t tiles = sort_tiles(n);
+  for (int shift = 0; shift < bits; shift += 8) {
+    HG_TRY(launch("radix_hist", radix_hist, dim3((unsigned)tiles), dim3(kSortThreads), 0, s,
+                  (const uint32_t*)b.keys[cur], n, shift, b.hist, tiles));
+    HG_TRY(exclusive_scan(b.hist, b.hist, tiles * kRadix, b.scan_scratch, s));
+    HG_TRY(launch("radix_scatter", radix_scatter, dim3((unsigned)tiles), dim3(kSortThreads), 0, s,
+                  (const uint32_t*)b.keys[cur], (const uint32_t*)b.vals[cur], b.keys[cur ^ 1],
+                  b.vals[cur ^ 1], n, shift, (const int32_t*)b.hist, tiles));
+    cur ^= 1;
+  }
+  *result = cur;
+  return HG_OK;
+}
+
+// ---------------------------------------------------------------------------------------------
+// CSR / CSC kernels
+// ---------------------------------------------------------------------------------------------
+__global__ void edge_keys(const int32_t* __restrict__ src, const int32_t* __restrict__ dst,
+                          const int32_t* __restrict__ rel, int64_t E, GraphMeta m, int by_dst,
+                          int64_t rows, uint32_t* __restrict__ keys, uint32_t* __restrict__ vals,
+                          int32_t* __restrict__ deg, int32_t* __restrict__ invalid) {
+  const int64_t N = m.type_off[m.num_types];
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < E;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int r = rel[e];
+    const int64_t s = src[e], t = dst[e];
+    bool ok = r >= 0 && r < m.num_rels && s >= 0 && s < N && t >= 0 && t < N;
+    int64_t key = rows;
+    if (ok) {
+      ok = node_type_of(m, s) == m.rel_src[r] && node_type_of(m, t) == m.rel_dst[r];
+      if (ok)
+        key = by_dst ? m.row_base[r] + (t - m.type_off[m.rel_dst[r]])
+                     : m.csc_base[r] + (s - m.type_off[m.rel_src[r]]);
+    }
+    keys[e] = (uint32_t)key;
+    vals[e] = (uint32_t)e;
+    if (ok)
+      atomicAdd(&deg[key], 1);
+    else if (invalid)
+      atomicAdd(invalid, 1);
+  }
+}
+
+__global__ void csr_finish(const uint32_t* __restrict__ eid_sorted, const int32_t* __restrict__ ptr,
+                           int64_t rows, int64_t E, const int32_t* __restrict__ src,
+                           int32_t* __restrict__ col, int32_t* __restrict__ eid) {
+  const int64_t nv = ptr[rows];
+  for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < nv;
+       p += (int64_t)gridDim.x * blockDim.x) {
+    const uint32_t e = eid_sorted[p];
+    eid[p] = (int32_t)e;
+    col[p] = src[e];
+  }
+}
+
+__global__ void csc_finish(const uint32_t* __restrict__ eid_sorted, const int32_t* __restrict__ cptr,
+                           int64_t crows, const int32_t* __restrict__ dst, const int32_t* __restrict__ rel,
+                           GraphMeta m, const int32_t* __restrict__ csr_ptr, int32_t* __restrict__ ccol,
+                           int32_t* __restrict__ ceid, float* __restrict__ coef) {
+  const int64_t nv = cptr[crows];
+  for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < nv;
+       p += (int64_t)gridDim.x * blockDim.x) {
+    const uint32_t e = eid_sorted[p];
+    const int r = rel[e];
+    const int32_t j = dst[e];
+    const int64_t row = m.row_base[r] + (j - m.type_off[m.rel_dst[r]]);
+    const int deg = csr_ptr[row + 1] - csr_ptr[row];
+    ceid[p] = (int32_t)e;
+    ccol[p] = j;
+    coef[p] = __fdiv_rn(1.0f, (float)deg);
+  }
+}
+
+__global__ void chunk_counts(const int32_t* __restrict__ ptr, int64_t rows, int32_t* __restrict__ cnt) {
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < rows;
+       r += (int64_t)gridDim.x * blockDim.x) {
+    const int deg = ptr[r + 1] - ptr[r];
+    cnt[r] = deg > kHubDegree ? (deg + kChunkEdges - 1) / kChunkEdges : 0;
+  }
+}
+
+__global__ void chunk_fill(const int32_t* __restrict__ ofs, int64_t rows, int32_t* __restrict__ chunk_row) {
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < rows;
+       r += (int64_t)gridDim.x * blockDim.x) {
+    for (int c = ofs[r]; c < ofs[r + 1]; ++c) chunk_row[c] = (int32_t)r;
+  }
+}
+
+// Rows above kHubDegree hold sum ceil(deg / kChunkEdges) <= E / kChunkEdges + E / (kHubDegree + 1)
+// chunks (each such row adds at most one partial chunk); +2 covers the integer floors.
+static int64_t chunk_cap(int64_t E) { return E / kChunkEdges + E / (kHubDegree + 1) + 2; }
+
+struct GraphLayout {
+  int32_t *csr_ptr, *csr_col, *csr_eid, *csc_ptr, *csc_col, *csc_eid;
+  float* csc_coef;
+  int32_t *csr_chunk_ofs, *csr_chunk_row, *csc_chunk_ofs, *csc_chunk_row, *invalid, *cnt;
+  SortBuffers sort;
+};
+
+static size_t carve_graph(void* ws, int64_t E, int64_t rows, int64_t crows, GraphLayout* L) {
+  Carve c(ws);
+  const int64_t Ea = std::max<int64_t>(E, 1);
+  L->csr_ptr = c.take<int32_t>(rows + 1);
+  L->csr_col = c.take<int32_t>(Ea);
+  L->csr_eid = c.take<int32_t>(Ea);
+  L->csc_ptr = c.take<int32_t>(crows + 1);
+  L->csc_col = c.take<int32_t>(Ea);
+  L->csc_eid = c.take<int32_t>(Ea);
+  L->csc_coef = c.take<float>(Ea);
+  L->csr_chunk_ofs = c.take<int32_t>(rows + 1);
+  L->csr_chunk_row = c.take<int32_t>(chunk_cap(E));
+  L->csc_chunk_ofs = c.take<int32_t>(crows + 1);
+  L->csc_chunk_row = c.take<int32_t>(chunk_cap(E));
+  L->invalid = c.take<int32_t>(1);
+  L->cnt = c.take<int32_t>(std::max(rows, crows) + 1);
+  for (int i = 0; i < 2; ++i) {
+    L->sort.keys[i] = c.take<uint32_t>(Ea);
+    L->sort.vals[i] = c.take<uint32_t>(Ea);
+  }
+  const int64_t hist_n = sort_tiles(E) * kRadix;
+  L->sort.hist = c.take<int32_t>(hist_n + 1);
+  L->sort.scan_scratch = c.take<char>(scan_scratch_bytes(std::max(std::max(hist_n, rows), crows)));
+  return c.used;
+}
+
+static hg_status make_meta(const int64_t* type_offsets, int32_t num_types, const hg_rel_desc* rels,
+                           int32_t num_rels, GraphMeta* m) {
+  HG_REQUIRE(type_offsets != nullptr && rels != nullptr, "type_offsets and rels must be non-null");
+  if (num_types < 1 || num_types > kMaxTypes || num_rels < 1 || num_rels > kMaxRels) {
+    set_error("need 1 <= num_types <= %d and 1 <= num_rels <= %d (got %d, %d)", kMaxTypes, kMaxRels,
+              num_types, num_rels);
+    return HG_ERR_UNSUPPORTED;
+  }
+  HG_REQUIRE(type_offsets[0] == 0, "type_offsets[0] must be 0");
+  for (int t = 0; t < num_types; ++t)
+    HG_REQUIRE(type_offsets[t + 1] >= type_offsets[t], "type_offsets must be non-decreasing");
+  if (type_offsets[num_types] >= (int64_t(1) << 31)) {
+    set_error("more than 2^31 - 1 nodes");
+    return HG_ERR_UNSUPPORTED;
+  }
+  *m = GraphMeta{};
+  m->num_types = num_types;
+  m->num_rels = num_rels;
+  for (int t = 0; t <= num_types; ++t) m->type_off[t] = type_offsets[t];
+  for (int t = num_types + 1; t <= kMaxTypes; ++t) m->type_off[t] = type_offsets[num_types];
+  m->row_base[0] = m->csc_base[0] = 0;
+  for (int r = 0; r < num_rels; ++r) {
+    const int s = rels[r].src_type, d = rels[r].dst_type;
+    HG_REQUIRE(s >= 0 && s < num_types && d >= 0 && d < num_types,
+               "relation %d has a node type out of range", r);
+    m->rel_src[r] = s;
+    m->rel_dst[r] = d;
+    m->row_base[r + 1] = m->row_base[r] + (type_offsets[d + 1] - type_offsets[d]);
+    m->csc_base[r + 1] = m->csc_base[r] + (type_offsets[s + 1] - type_offsets[s]);
+  }
+  if (m->row_base[num_rels] >= (int64_t(1) << 31) - 1 || m->csc_base[num_rels] >= (int64_t(1) << 31) - 1) {
+    set_error("more than 2^31 - 2 relation rows");
+    return HG_ERR_UNSUPPORTED;
+  }
+  return HG_OK;
+}
+
+static int bit_width(uint64_t x) {
+  int b = 0;
+  while (x) {
+    ++b;
+    x >>= 1;
+  }
+  return b;
+}
+
+static unsigned grid_for(int64_t n, int threads = 256) {
+  return (unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(n, threads), 152 * 16));
+}
+
+}  // namespace hg
+
+using namespace hg;
+
+extern "C" hg_status hg_graph_workspace_size(int64_t num_edges, const int64_t* type_offsets,
+                                             int32_t num_types, const hg_rel_desc* rels,
+                                             int32_t num_rels, size_t* bytes) {
+  clear_error();
+  HG_REQUIRE(bytes != nullptr, "bytes must be non-null");
+  HG_REQUIRE(num_edges >= 0, "num_edges must be >= 0");
+  if (num_edges >= (int64_t(1) << 31)) {
+    set_error("num_edges >= 2^31 is not supported");
+    return HG_ERR_UNSUPPORTED;
+  }
+  GraphMeta m;
+  HG_TRY(make_meta(type_offsets, num_types, rels, num_rels, &m));
+  GraphLayout L;
+  *bytes = carve_graph(nullptr, num_edges, m.row_base[num_rels], m.csc_base[num_rels], &L);
+  return HG_OK;
+}
+
+extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const int32_t* rel,
+                                  int64_t num_edges, const int64_t* type_offsets, int32_t num_types,
+                                  const hg_rel_desc* rels, int32_t num_rels, void* workspace,
+                                  size_t workspace_bytes, hg_stream stream, hg_graph** out) {
+  clear_error();
+  HG_REQUIRE(out != nullptr, "out must be non-null");
+  *out = nullptr;
+  HG_REQUIRE(num_edges >= 0, "num_edges must be >= 0");
+  if (num_edges >= (int64_t(1) << 31)) {
+    set_error("num_edges >= 2^31 is not supported");
+    return HG_ERR_UNSUPPORTED;
+  }
+  HG_REQUIRE(num_edges == 0 || (src && dst && rel), "src, dst and rel must be non-null");
+  HG_REQUIRE(workspace != nullptr, "workspace must be non-null");
+  HG_REQUIRE(((uintptr_t)workspace & 255) == 0, "workspace must be 256-byte aligned");
+  GraphMeta m;
+  HG_TRY(make_meta(type_offsets, num_types, rels, num_rels, &m));
+  const int64_t E = num_edges, rows = m.row_base[num_rels], crows = m.csc_base[num_rels];
+  GraphLayout L;
+  const size_t need = carve_graph(nullptr, E, rows, crows, &L);
+  if (workspace_bytes < need) {
+    set_error("workspace has %zu bytes, %zu needed", workspace_bytes, need);
+    return HG_ERR_WORKSPACE;
+  }
+  carve_graph(workspace, E, rows, crows, &L);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+
+  HG_CUDA(cudaMemsetAsync(L.csr_ptr, 0, (rows + 1) * sizeof(int32_t), s));
+  HG_CUDA(cudaMemsetAsync(L.csc_ptr, 0, (crows + 1) * sizeof(int32_t), s));
+  HG_CUDA(cudaMemsetAsync(L.invalid, 0, sizeof(int32_t), s));
+  const unsigned g = grid_for(E);
+  int res = 0;
+  // CSR by destination
+  if (E > 0) {
+    HG_TRY(launch("edge_keys", edge_keys, dim3(g), dim3(256), 0, s, src, dst, rel, E, m, 1, rows,
+                  L.sort.keys[0], L.sort.vals[0], L.csr_ptr, L.invalid));
+  }
+  HG_TRY(exclusive_scan(L.csr_ptr, L.csr_ptr, rows, L.sort.scan_scratch, s));
+  if (E > 0) {
+    HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)rows), s, &res));
+    HG_TRY(launch("csr_finish", csr_finish, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.vals[res],
+                  (const int32_t*)L.csr_ptr, rows, E, src, L.csr_col, L.csr_eid));
+  }
+  // CSC by source
+  if (E > 0) {
+    HG_TRY(launch("edge_keys", edge_keys, dim3(g), dim3(256), 0, s, src, dst, rel, E, m, 0, crows,
+                  L.sort.keys[0], L.sort.vals[0], L.csc_ptr, (int32_t*)nullptr));
+  }
+  HG_TRY(exclusive_scan(L.csc_ptr, L.csc_ptr, crows, L.sort.scan_scratch, s));
+  if (E > 0) {
+    HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)crows), s, &res));
+    HG_TRY(launch("csc_finish", csc_finish, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.vals[res],
+                  (const int32_t*)L.csc_ptr, crows, dst, rel, m, (const int32_t*)L.csr_ptr, L.csc_col,
+                  L.csc_eid, L.csc_coef));
+  }
+  // chunk tables for rows above the hub degree
+  HG_TRY(launch("chunk_counts", chunk_counts, dim3(grid_for(rows)), dim3(256), 0, s,
+                (const int32_t*)L.csr_ptr, rows, L.cnt));
+  HG_TRY(exclusive_scan(L.cnt, L.csr_chunk_ofs, rows, L.sort.scan_scratch, s));
+  HG_TRY(launch("chunk_fill", chunk_fill, dim3(grid_for(rows)), dim3(256), 0, s,
+                (const int32_t*)L.csr_chunk_ofs, rows, L.csr_chunk_row));
+  HG_TRY(launch("chunk_counts", chunk_counts, dim3(grid_for(crows)), dim3(256), 0, s,
+                (const int32_t*)L.csc_ptr, crows, L.cnt));
+  HG_TRY(exclusive_scan(L.cnt, L.csc_chunk_ofs, crows, L.sort.scan_scratch, s));
+  HG_TRY(launch("chunk_fill", chunk_fill, dim3(grid_for(crows)), dim3(256), 0, s,
+                (const int32_t*)L.csc_chunk_ofs, crows, L.csc_chunk_row));
+
+  hg_graph* gh = new hg_graph{};
+  gh->meta = m;
+  gh->num_edges = E;
+  gh->csr_rows = rows;
+  gh->csc_rows = crows;
+  gh->chunk_cap_csr = chunk_cap(E);
+  gh->chunk_cap_csc = chunk_cap(E);
+  gh->stream = s;
+  gh->csr_ptr = L.csr_ptr;
+  gh->csr_col = L.csr_col;
+  gh->csr_eid = L.csr_eid;
+  gh->csc_ptr = L.csc_ptr;
+  gh->csc_col = L.csc_col;
+  gh->csc_eid = L.csc_eid;
+  gh->csc_coef = L.csc_coef;
+  gh->csr_chunk_ofs = L.csr_chunk_ofs;
+  gh->csr_chunk_row = L.csr_chunk_row;
+  gh->csc_chunk_ofs = L.csc_chunk_ofs;
+  gh->csc_chunk_row = L.csc_chunk_row;
+  gh->invalid_count = L.invalid;
+  *out = gh;
+  return HG_OK;
+}
+
+extern "C" hg_status hg_graph_destroy(hg_graph* graph) {
+  delete graph;
+  return HG_OK;
+}
+
+extern "C" hg_status hg_graph_check(const hg_graph* graph, int64_t* num_invalid_edges) {
+  clear_error();
+  HG_REQUIRE(graph != nullptr, "graph must be non-null");
+  int32_t bad = 0;
+  HG_CUDA(cudaMemcpyAsync(&bad, graph->invalid_count, sizeof(int32_t), cudaMemcpyDeviceToHost,
+                          graph->stream));
+  HG_CUDA(cudaStreamSynchronize(graph->stream));
+  if (num_invalid_edges) *num_invalid_edges = bad;
+  if (bad != 0) {
+    set_error("%d edges were dropped (id out of range, relation out of range, or endpoint types "
+              "that do not match the relation)", bad);
+    return HG_ERR_DEVICE_CHECK;
+  }
+  return HG_OK;
+}
+
+extern "C" hg_status hg_graph_view(const hg_graph* graph, int32_t rel, hg_graph_arrays* out) {
+  clear_error();
+  HG_REQUIRE(graph != nullptr && out != nullptr, "graph and out must be non-null");
+  const GraphMeta& m = graph->meta;
+  HG_REQUIRE(rel >= 0 && rel < m.num_rels, "relation %d out of range", rel);
+  out->n_dst = m.row_base[rel + 1] - m.row_base[rel];
+  out->n_src = m.csc_base[rel + 1] - m.csc_base[rel];
+  out->num_edges = graph->num_edges;
+  out->row_ptr = graph->csr_ptr + m.row_base[rel];
+  out->col = graph->csr_col;
+  out->eid = graph->csr_eid;
+  out->csc_ptr = graph->csc_ptr + m.csc_base[rel];
+  out->csc_col = graph->csc_col;
+  out->csc_eid = graph->csc_eid;
+  out->csc_coef = graph->csc_coef;
+  return HG_OK;
+}

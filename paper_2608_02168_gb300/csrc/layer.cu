@@ -1,0 +1,323 @@
+// Layer entry points (Eq. 7, Eq. 10 with mean aggregation, Eq. 11, optional LayerNorm), status
+// strings, thread-local error text and the optional per-kernel event timing.
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <algorithm>
+#include <map>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "layer_kernels.cuh"
+
+namespace hg {
+
+
+// ---------------------------------------------------------------------------------------------
+// errors
+// ---------------------------------------------------------------------------------------------
+static thread_local char g_err[1024];
+
+void set_error(const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+}
+void clear_error() { g_err[0] = 0; }
+
+// ---------------------------------------------------------------------------------------------
+// timing
+// ---------------------------------------------------------------------------------------------
+struct TimingRec {
+  const char* name;
+  cudaEvent_t a, b;
+};
+static std::mutex g_tmu;
+static bool g_timing = false;
+static std::vector<TimingRec> g_recs;
+static std::vector<cudaEvent_t> g_pool;
+
+static cudaEvent_t take_event() {
+  if (!g_pool.empty()) {
+    cudaEvent_t e = g_pool.back();
+    g_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+int timing_begin(const char* name, cudaStream_t s) {
+  if (!g_timing) return -1;
+  std::lock_guard<std::mutex> lk(g_tmu);
+  TimingRec r{name, take_event(), take_event()};
+  cudaEventRecord(r.a, s);
+  g_recs.push_back(r);
+  return (int)g_recs.size() - 1;
+}
+
+void timing_end(int slot, cudaStream_t s) {
+  if (slot < 0) return;
+  std::lock_guard<std::mutex> lk(g_tmu);
+  cudaEventRecord(g_recs[slot].b, s);
+}
+
+// ---------------------------------------------------------------------------------------------
+// layer workspace layout
+// ---------------------------------------------------------------------------------------------
+struct LayerLayout {
+  void* M;        // saved: csr_rows x d
+  void* Z;        // saved: N x d
+  void* U;        // saved: N x d
+  float2* stats;  // saved: N
+  float* agg_part;  // scratch: chunk partials
+  void* dY;       // scratch: N x d
+  void* dU;
+  void* dZ;
+  void* dMs;      // scratch: csr_rows x d
+  float* cpart;   // scratch: row blocks x 3 x d
+  float* wpart;   // scratch: splits x d x d
+  void* WrelT;    // scratch: R x d x d
+  void* WaggT;    // scratch: T x d x d
+};
+
+static size_t elem_size(hg_dtype dt) { return dt == HG_F32 ? 4 : 2; }
+
+static void carve_layer(const hg_graph* g, int d, hg_dtype dt, void* saved, void* scratch, LayerLayout* L,
+                        size_t* saved_bytes, size_t* scratch_bytes) {
+  const GraphMeta& m = g->meta;
+  const int64_t N = m.type_off[m.num_types];
+  const size_t b = elem_size(dt);
+  Carve s(saved), k(scratch);
+  L->M = s.take<char>((size_t)g->csr_rows * d * b);
+  L->Z = s.take<char>((size_t)N * d * b);
+  L->U = s.take<char>((size_t)N * d * b);
+  L->stats = s.take<float2>(std::max<int64_t>(N, 1));
+  L->agg_part = k.take<float>((size_t)std::max(g->chunk_cap_csr, g->chunk_cap_csc) * d);
+  L->dY = k.take<char>((size_t)N * d * b);
+  L->dU = k.take<char>((size_t)N * d * b);
+  L->dZ = k.take<char>((size_t)N * d * b);
+  L->dMs = k.take<char>((size_t)g->csr_rows * d * b);
+  int64_t max_rows = 1;
+  for (int t = 0; t < m.num_types; ++t) max_rows = std::max(max_rows, m.type_off[t + 1] - m.type_off[t]);
+  L->cpart = k.take<float>((size_t)ceil_div(max_rows, 64) * 3 * d);
+  L->wpart = k.take<float>((size_t)wgrad_splits(max_rows) * d * d);
+  L->WrelT = k.take<char>((size_t)m.num_rels * d * d * b);
+  L->WaggT = k.take<char>((size_t)m.num_types * d * d * b);
+  if (saved_bytes) *saved_bytes = s.used;
+  if (scratch_bytes) *scratch_bytes = k.used;
+}
+
+static hg_status check_params(const hg_graph* g, const hg_layer_params* p) {
+  HG_REQUIRE(g != nullptr && p != nullptr, "graph and params must be non-null");
+  if (!(p->d == 64 || p->d == 128 || p->d == 256)) {
+    set_error("d=%d not supported (64, 128, 256)", p->d);
+    return HG_ERR_UNSUPPORTED;
+  }
+  if (!(p->dtype == HG_F32 || p->dtype == HG_BF16)) {
+    set_error("dtype %d not supported", (int)p->dtype);
+    return HG_ERR_UNSUPPORTED;
+  }
+  HG_REQUIRE(p->act == HG_ACT_RELU || p->act == HG_ACT_GELU_TANH || p->act == HG_ACT_NONE, "unknown activation %d",
+             (int)p->act);
+  HG_REQUIRE(p->W_rel && p->W_agg && p->b_agg, "W_rel, W_agg and b_agg must be non-null");
+  HG_REQUIRE(!p->layernorm || (p->ln_gamma && p->ln_beta), "layernorm needs ln_gamma and ln_beta");
+  HG_REQUIRE(!p->layernorm || p->ln_eps > 0.f, "ln_eps must be > 0");
+  return HG_OK;
+}
+
+static hg_status check_buf(const void* p, const char* name) {
+  HG_REQUIRE(p != nullptr, "%s must be non-null", name);
+  HG_REQUIRE(((uintptr_t)p & 255) == 0, "%s must be 256-byte aligned", name);
+  return HG_OK;
+}
+
+}  // namespace hg
+
+using namespace hg;
+
+extern "C" const char* hg_status_string(hg_status s) {
+  switch (s) {
+    case HG_OK: return "ok";
+    case HG_ERR_INVALID_ARG: return "invalid argument";
+    case HG_ERR_UNSUPPORTED: return "unsupported";
+    case HG_ERR_WORKSPACE: return "workspace too small";
+    case HG_ERR_CUDA: return "CUDA error";
+    case HG_ERR_DEVICE_CHECK: return "device-side input check failed";
+    case HG_ERR_TIMEOUT: return "timeout";
+  }
+  return "unknown status";
+}
+
+extern "C" const char* hg_last_error(void) { return g_err; }
+extern "C" int32_t hg_abi_version(void) { return 1; }
+
+extern "C" hg_status hg_timing_enable(int32_t on) {
+  std::lock_guard<std::mutex> lk(g_tmu);
+  g_timing = on != 0;
+  return HG_OK;
+}
+
+extern "C" hg_status hg_timing_report(char* buf, size_t len) {
+  clear_error();
+  std::lock_guard<std::mutex> lk(g_tmu);
+  std::map<std::string, std::pair<long, double>> acc;
+  hg_status st = HG_OK;
+  for (auto& r : g_recs) {
+    float ms = 0.f;
+    if (cudaEventSynchronize(r.b) != cudaSuccess || cudaEventElapsedTime(&ms, r.a, r.b) != cudaSuccess) {
+      set_error("event timing failed: %s", cudaGetErrorString(cudaGetLastError()));
+      st = HG_ERR_CUDA;
+    }
+    auto& e = acc[r.name];
+    e.first += 1;
+    e.second += ms;
+    g_pool.push_back(r.a);
+    g_pool.push_back(r.b);
+  }
+  g_recs.clear();
+  std::string out;
+  char line[256];
+  for (auto& kv : acc) {
+    snprintf(line, sizeof(line), "%s %ld %.6f\n", kv.first.c_str(), kv.second.first, kv.second.second);
+    out += line;
+  }
+  if (buf && len) {
+    size_t n = std::min(len - 1, out.size());
+    memcpy(buf, out.data(), n);
+    buf[n] = 0;
+  }
+  return st;
+}
+
+extern "C" hg_status hg_layer_workspace_size(const hg_graph* graph, const hg_layer_params* params,
+                                             size_t* saved_bytes, size_t* scratch_bytes) {
+  clear_error();
+  HG_TRY(check_params(graph, params));
+  HG_REQUIRE(saved_bytes && scratch_bytes, "saved_bytes and scratch_bytes must be non-null");
+  LayerLayout L;
+  carve_layer(graph, params->d, params->dtype, nullptr, nullptr, &L, saved_bytes, scratch_bytes);
+  return HG_OK;
+}
+
+extern "C" hg_status hg_layer_fwd(const hg_graph* graph, const hg_layer_params* p, const void* H_in, void* H_out,
+                                  void* saved, void* scratch, hg_stream stream) {
+  clear_error();
+  HG_TRY(check_params(graph, p));
+  HG_TRY(check_buf(H_in, "H_in"));
+  HG_TRY(check_buf(H_out, "H_out"));
+  HG_TRY(check_buf(saved, "saved"));
+  HG_TRY(check_buf(scratch, "scratch"));
+  HG_REQUIRE(H_in != H_out, "H_in and H_out must not alias");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const GraphMeta& m = graph->meta;
+  const int d = p->d;
+  const size_t b = elem_size(p->dtype);
+  LayerLayout L;
+  carve_layer(graph, d, p->dtype, saved, scratch, &L, nullptr, nullptr);
+  HG_TRY(aggregate_forward(graph, p->dtype, d, H_in, L.M, L.agg_part, s));
+  for (int t = 0; t < m.num_types; ++t) {
+    FwdArgs a{};
+    a.M = L.M;
+    for (int r = 0; r < m.num_rels; ++r) {
+      if (m.rel_dst[r] != t) continue;
+      a.mrow0[a.nrel] = m.row_base[r];
+      a.W_rel[a.nrel] = (const char*)p->W_rel + (size_t)r * d * d * b;
+      ++a.nrel;
+    }
+    a.W_agg = (const char*)p->W_agg + (size_t)t * d * d * b;
+    a.b = (const char*)p->b_agg + (size_t)t * d * b;
+    a.gamma = p->layernorm ? (const char*)p->ln_gamma + (size_t)t * d * b : nullptr;
+    a.beta = p->layernorm ? (const char*)p->ln_beta + (size_t)t * d * b : nullptr;
+    a.H_in = H_in;
+    a.H_out = H_out;
+    a.Z = L.Z;
+    a.U = L.U;
+    a.stats = L.stats;
+    a.off = m.type_off[t];
+    a.n = m.type_off[t + 1] - m.type_off[t];
+    a.act = p->act;
+    a.ln = p->layernorm;
+    a.eps = p->ln_eps;
+    if (a.n > 0) HG_TRY(proj_forward(p->dtype, d, a, s));
+  }
+  return HG_OK;
+}
+
+extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* p, const void* H_in, const void* saved,
+                                  const void* dH_out, void* dH_in, const hg_layer_grads* grads, void* scratch,
+                                  hg_stream stream) {
+  clear_error();
+  HG_TRY(check_params(graph, p));
+  HG_TRY(check_buf(H_in, "H_in"));
+  HG_TRY(check_buf(saved, "saved"));
+  HG_TRY(check_buf(dH_out, "dH_out"));
+  HG_TRY(check_buf(scratch, "scratch"));
+  HG_REQUIRE(dH_in == nullptr || ((uintptr_t)dH_in & 255) == 0, "dH_in must be 256-byte aligned");
+  HG_REQUIRE(grads && grads->dW_rel && grads->dW_agg && grads->db_agg, "grads and its dW_rel, dW_agg, db_agg must be non-null");
+  HG_REQUIRE(!p->layernorm || (grads->dln_gamma && grads->dln_beta), "layernorm needs dln_gamma and dln_beta");
+  HG_REQUIRE(dH_in != dH_out, "dH_in and dH_out must not alias");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const GraphMeta& m = graph->meta;
+  const int d = p->d;
+  const size_t b = elem_size(p->dtype);
+  LayerLayout L;
+  carve_layer(graph, d, p->dtype, const_cast<void*>(saved), scratch, &L, nullptr, nullptr);
+  HG_TRY(transpose_weights(p->dtype, d, p->W_rel, L.WrelT, m.num_rels, s));
+  HG_TRY(transpose_weights(p->dtype, d, p->W_agg, L.WaggT, m.num_types, s));
+  for (int t = 0; t < m.num_types; ++t) {
+    const int64_t n = m.type_off[t + 1] - m.type_off[t];
+    float* db = grads->db_agg + (size_t)t * d;
+    if (n == 0) {
+      HG_CUDA(cudaMemsetAsync(db, 0, d * sizeof(float), s));
+      if (p->layernorm) {
+        HG_CUDA(cudaMemsetAsync(grads->dln_gamma + (size_t)t * d, 0, d * sizeof(float), s));
+        HG_CUDA(cudaMemsetAsync(grads->dln_beta + (size_t)t * d, 0, d * sizeof(float), s));
+      }
+      continue;
+    }
+    BwdArgs a{};
+    a.dH_out = dH_out;
+    a.H_in = H_in;
+    a.U = L.U;
+    a.stats = L.stats;
+    a.gamma = p->layernorm ? (const char*)p->ln_gamma + (size_t)t * d * b : nullptr;
+    a.W_aggT = (const char*)L.WaggT + (size_t)t * d * d * b;
+    for (int r = 0; r < m.num_rels; ++r) {
+      if (m.rel_dst[r] != t) continue;
+      a.mrow0[a.nrel] = m.row_base[r];
+      a.W_relT[a.nrel] = (const char*)L.WrelT + (size_t)r * d * d * b;
+      ++a.nrel;
+    }
+    a.csr_ptr = graph->csr_ptr;
+    a.dY = L.dY;
+    a.dU = L.dU;
+    a.dZ = L.dZ;
+    a.dMs = L.dMs;
+    a.part = L.cpart;
+    a.off = m.type_off[t];
+    a.n = n;
+    a.act = p->act;
+    a.ln = p->layernorm;
+    HG_TRY(proj_backward(p->dtype, d, a, s));
+    const int blocks = (int)ceil_div(n, 64);
+    HG_TRY(reduce_partials(L.cpart, 3LL * d, blocks, d, db, s));
+    if (p->layernorm) {
+      HG_TRY(reduce_partials(L.cpart + d, 3LL * d, blocks, d, grads->dln_gamma + (size_t)t * d, s));
+      HG_TRY(reduce_partials(L.cpart + 2 * d, 3LL * d, blocks, d, grads->dln_beta + (size_t)t * d, s));
+    }
+    HG_TRY(weight_grad(p->dtype, d, L.Z, a.off, L.dU, a.off, n, L.wpart, grads->dW_agg + (size_t)t * d * d, s));
+  }
+  for (int r = 0; r < m.num_rels; ++r) {
+    const int t = m.rel_dst[r];
+    const int64_t n = m.type_off[t + 1] - m.type_off[t];
+    HG_TRY(weight_grad(p->dtype, d, L.M, m.row_base[r], L.dZ, m.type_off[t], n, L.wpart,
+                       grads->dW_rel + (size_t)r * d * d, s));
+  }
+  if (dH_in) HG_TRY(aggregate_backward(graph, p->dtype, d, L.dMs, L.dY, dH_in, L.agg_part, s));
+  return HG_OK;
+}

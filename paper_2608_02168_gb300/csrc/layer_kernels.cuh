@@ -1,0 +1,60 @@
+// Argument blocks and internal entry points of the layer kernels (shared by the translation
+// units; not part of the public ABI).
+#pragma once
+
+#include "hg_internal.cuh"
+
+namespace hg {
+
+struct FwdArgs {
+  const void* M;                 // saved relation means, concatenated CSR rows
+  int nrel;
+  int64_t mrow0[kMaxRels];       // first CSR row of each relation into this type
+  const void* W_rel[kMaxRels];   // its D x D message matrix (d_in x d_out)
+  const void* W_agg;
+  const void* b;
+  const void* gamma;
+  const void* beta;
+  const void* H_in;
+  void* H_out;
+  void* Z;                       // saved, node rows
+  void* U;                       // saved, node rows
+  float2* stats;                 // saved (mean, rstd) per node row
+  int64_t off, n;                // node rows [off, off + n) of this type
+  int act, ln;
+  float eps;
+};
+
+struct BwdArgs {
+  const void* dH_out;
+  const void* H_in;
+  const void* U;
+  const float2* stats;
+  const void* gamma;
+  const void* W_aggT;            // W_agg^T, D x D row-major
+  int nrel;
+  int64_t mrow0[kMaxRels];
+  const void* W_relT[kMaxRels];  // W_r^T
+  const int32_t* csr_ptr;        // degrees of the relation rows
+  void* dY;                      // node rows
+  void* dU;                      // node rows
+  void* dZ;                      // node rows
+  void* dMs;                     // concatenated CSR rows (scaled by 1/deg)
+  float* part;                   // [blocks][3][D]: db, dgamma, dbeta partials
+  int64_t off, n;
+  int act, ln;
+};
+
+hg_status aggregate_forward(const hg_graph* g, hg_dtype dt, int d, const void* H, void* M, float* partials,
+                            cudaStream_t s);
+hg_status aggregate_backward(const hg_graph* g, hg_dtype dt, int d, const void* dMs, const void* dY, void* dH,
+                             float* partials, cudaStream_t s);
+hg_status proj_forward(hg_dtype dt, int d, const FwdArgs& a, cudaStream_t s);
+hg_status proj_backward(hg_dtype dt, int d, const BwdArgs& a, cudaStream_t s);
+hg_status weight_grad(hg_dtype dt, int d, const void* X, int64_t x0, const void* Y, int64_t y0, int64_t n, float* part,
+                      float* out, cudaStream_t s);
+hg_status transpose_weights(hg_dtype dt, int d, const void* W, void* Wt, int count, cudaStream_t s);
+hg_status reduce_partials(const float* part, int64_t stride, int splits, int64_t count, float* out, cudaStream_t s);
+int wgrad_splits(int64_t n);
+
+}  // namespace hg

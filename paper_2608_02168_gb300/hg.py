@@ -1,0 +1,302 @@
+"""Python binding of libhg (include/hg.h): same entry-point names, argument marshalling only.
+
+Device buffers are torch CUDA tensors (their data pointers are passed through); streams are torch
+streams.  Every computation happens inside libhg's CUDA kernels.  A missing library raises
+ImportError: there is no fallback path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from ctypes import POINTER, Structure, byref, c_char_p, c_float, c_int32, c_int64, c_size_t, c_void_p
+
+import torch
+
+from . import build as _build
+
+HG_F32, HG_BF16 = 0, 1
+HG_ACT_RELU, HG_ACT_GELU_TANH, HG_ACT_NONE = 0, 1, 2
+DTYPES = {"f32": HG_F32, "bf16": HG_BF16}
+TORCH_DTYPES = {HG_F32: torch.float32, HG_BF16: torch.bfloat16}
+ACTS = {"relu": HG_ACT_RELU, "gelu_tanh": HG_ACT_GELU_TANH, "none": HG_ACT_NONE}
+
+
+class hg_rel_desc(Structure):
+    _fields_ = [("src_type", c_int32), ("dst_type", c_int32)]
+
+
+class hg_graph_arrays(Structure):
+    _fields_ = [("n_dst", c_int64), ("n_src", c_int64), ("num_edges", c_int64), ("row_ptr", c_void_p),
+                ("col", c_void_p), ("eid", c_void_p), ("csc_ptr", c_void_p), ("csc_col", c_void_p),
+                ("csc_eid", c_void_p), ("csc_coef", c_void_p)]
+
+
+class hg_layer_params(Structure):
+    _fields_ = [("d", c_int32), ("dtype", c_int32), ("act", c_int32), ("layernorm", c_int32), ("ln_eps", c_float),
+                ("W_rel", c_void_p), ("W_agg", c_void_p), ("b_agg", c_void_p), ("ln_gamma", c_void_p),
+                ("ln_beta", c_void_p)]
+
+
+class hg_layer_grads(Structure):
+    _fields_ = [("dW_rel", c_void_p), ("dW_agg", c_void_p), ("db_agg", c_void_p), ("dln_gamma", c_void_p),
+                ("dln_beta", c_void_p)]
+
+
+EXPORTS = {
+    # name: (restype, argtypes)
+    "hg_status_string": (c_char_p, [c_int32]),
+    "hg_last_error": (c_char_p, []),
+    "hg_abi_version": (c_int32, []),
+    "hg_graph_workspace_size": (c_int32, [c_int64, POINTER(c_int64), c_int32, POINTER(hg_rel_desc), c_int32,
+                                          POINTER(c_size_t)]),
+    "hg_build_csr": (c_int32, [c_void_p, c_void_p, c_void_p, c_int64, POINTER(c_int64), c_int32,
+                               POINTER(hg_rel_desc), c_int32, c_void_p, c_size_t, c_void_p, POINTER(c_void_p)]),
+    "hg_graph_destroy": (c_int32, [c_void_p]),
+    "hg_graph_check": (c_int32, [c_void_p, POINTER(c_int64)]),
+    "hg_graph_view": (c_int32, [c_void_p, c_int32, POINTER(hg_graph_arrays)]),
+    "hg_layer_workspace_size": (c_int32, [c_void_p, POINTER(hg_layer_params), POINTER(c_size_t), POINTER(c_size_t)]),
+    "hg_layer_fwd": (c_int32, [c_void_p, POINTER(hg_layer_params), c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),
+    "hg_layer_bwd": (c_int32, [c_void_p, POINTER(hg_layer_params), c_void_p, c_void_p, c_void_p, c_void_p,
+                               POINTER(hg_layer_grads), c_void_p, c_void_p]),
+    "hg_overlap_intersect_workspace_size": (c_int32, [c_int64, c_int64, POINTER(c_size_t)]),
+    "hg_overlap_intersect": (c_int32, [c_void_p, c_int64, c_void_p, c_int64, c_void_p, c_void_p, c_void_p, c_void_p,
+                                       c_size_t, c_void_p]),
+    "hg_overlap_align_workspace_size": (c_int32, [c_int64, c_int32, POINTER(c_size_t), POINTER(c_size_t)]),
+    "hg_overlap_align_loss": (c_int32, [c_void_p, c_int64, c_void_p, c_void_p, c_int64, c_void_p, c_int64, c_void_p,
+                                        c_int32, c_int32, c_float, c_float, c_void_p, c_void_p, c_void_p, c_void_p]),
+    "hg_overlap_align_bwd": (c_int32, [c_void_p, c_int64, c_void_p, c_void_p, c_int64, c_void_p, c_int64, c_void_p,
+                                       c_int32, c_int32, c_float, c_float, c_float, c_void_p, c_void_p, c_void_p,
+                                       c_void_p, c_void_p]),
+    "hg_timing_enable": (c_int32, [c_int32]),
+    "hg_timing_report": (c_int32, [c_char_p, c_size_t]),
+}
+
+_lib = None
+
+
+class HGError(RuntimeError):
+    def __init__(self, status: int, where: str, detail: str):
+        super().__init__(f"{where}: status {status} ({_lib.hg_status_string(status).decode()}): {detail}")
+        self.status = status
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded libhg.so (ImportError if it has not been built)."""
+    global _lib
+    if _lib is None:
+        path = _build.library_path()
+        if not os.path.exists(path):
+            raise ImportError(f"{path} is missing: build it with __graft_entry__.build() or "
+                              "`python -m paper_2608_02168_gb300.build`")
+        so = ctypes.CDLL(path)
+        for name, (res, args) in EXPORTS.items():
+            fn = getattr(so, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = so
+    return _lib
+
+
+def _check(status: int, where: str):
+    if status != 0:
+        raise HGError(status, where, lib().hg_last_error().decode())
+
+
+def _ptr(t) -> int | None:
+    if t is None:
+        return None
+    return t.data_ptr()
+
+
+def _stream(stream) -> int | None:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream
+
+
+def _offsets(type_offsets):
+    arr = (c_int64 * len(type_offsets))(*[int(x) for x in type_offsets])
+    return arr
+
+
+def _rels(rels):
+    arr = (hg_rel_desc * len(rels))(*[hg_rel_desc(int(s), int(t)) for s, t in rels])
+    return arr
+
+
+# ------------------------------------------------------------------------------------------------
+# graph
+# ------------------------------------------------------------------------------------------------
+def hg_graph_workspace_size(num_edges: int, type_offsets, rels) -> int:
+    n = c_size_t(0)
+    _check(lib().hg_graph_workspace_size(int(num_edges), _offsets(type_offsets), len(type_offsets) - 1, _rels(rels),
+                                         len(rels), byref(n)), "hg_graph_workspace_size")
+    return n.value
+
+
+class Graph:
+    """Host handle of a built graph; keeps the workspace tensor alive."""
+
+    def __init__(self, handle: c_void_p, workspace: torch.Tensor, type_offsets, rels):
+        self.handle = handle
+        self.workspace = workspace
+        self.type_offsets = [int(x) for x in type_offsets]
+        self.rels = [tuple(r) for r in rels]
+
+    @property
+    def num_nodes(self) -> int:
+        return self.type_offsets[-1]
+
+    def __del__(self):
+        if getattr(self, "handle", None) and _lib is not None:
+            _lib.hg_graph_destroy(self.handle)
+            self.handle = None
+
+
+def hg_build_csr(src, dst, rel, type_offsets, rels, workspace: torch.Tensor | None = None, stream=None) -> Graph:
+    E = int(src.numel())
+    need = hg_graph_workspace_size(E, type_offsets, rels)
+    if workspace is None:
+        workspace = torch.empty(need, dtype=torch.uint8, device=src.device)
+    h = c_void_p()
+    _check(lib().hg_build_csr(_ptr(src), _ptr(dst), _ptr(rel), E, _offsets(type_offsets), len(type_offsets) - 1,
+                              _rels(rels), len(rels), _ptr(workspace), workspace.numel(), _stream(stream), byref(h)),
+           "hg_build_csr")
+    return Graph(h, workspace, type_offsets, rels)
+
+
+def hg_graph_destroy(g: Graph):
+    if g.handle:
+        _check(lib().hg_graph_destroy(g.handle), "hg_graph_destroy")
+        g.handle = None
+
+
+def hg_graph_check(g: Graph) -> int:
+    """Synchronises the build stream; returns the number of dropped (invalid) edges."""
+    n = c_int64(0)
+    st = lib().hg_graph_check(g.handle, byref(n))
+    if st not in (0, 5):
+        _check(st, "hg_graph_check")
+    return n.value
+
+
+def hg_graph_view(g: Graph, rel: int) -> dict:
+    """Device views (torch tensors sharing the workspace) of one relation's CSR / CSC arrays."""
+    a = hg_graph_arrays()
+    _check(lib().hg_graph_view(g.handle, int(rel), byref(a)), "hg_graph_view")
+    ws = g.workspace
+    base = ws.data_ptr()
+
+    def view(ptr, n, dtype):
+        off = ptr - base
+        return ws[off:off + n * 4].view(dtype)
+
+    E = a.num_edges
+    return dict(n_dst=a.n_dst, n_src=a.n_src, row_ptr=view(a.row_ptr, a.n_dst + 1, torch.int32),
+                col=view(a.col, E, torch.int32), eid=view(a.eid, E, torch.int32),
+                csc_ptr=view(a.csc_ptr, a.n_src + 1, torch.int32), csc_col=view(a.csc_col, E, torch.int32),
+                csc_eid=view(a.csc_eid, E, torch.int32), csc_coef=view(a.csc_coef, E, torch.float32))
+
+
+# ------------------------------------------------------------------------------------------------
+# layer
+# ------------------------------------------------------------------------------------------------
+class LayerParams:
+    """Packed device parameters of one layer (see hg_layer_params)."""
+
+    def __init__(self, W_rel, W_agg, b_agg, ln_gamma=None, ln_beta=None, act: str = "relu", layernorm: bool = True,
+                 ln_eps: float = 1e-5):
+        self.W_rel, self.W_agg, self.b_agg = W_rel.contiguous(), W_agg.contiguous(), b_agg.contiguous()
+        self.ln_gamma = ln_gamma.contiguous() if ln_gamma is not None else None
+        self.ln_beta = ln_beta.contiguous() if ln_beta is not None else None
+        self.act, self.layernorm, self.ln_eps = act, layernorm, ln_eps
+        self.d = int(W_rel.shape[-1])
+        self.dtype = HG_F32 if W_rel.dtype == torch.float32 else HG_BF16
+
+    def c(self) -> hg_layer_params:
+        return hg_layer_params(self.d, self.dtype, ACTS[self.act], 1 if self.layernorm else 0, self.ln_eps,
+                               _ptr(self.W_rel), _ptr(self.W_agg), _ptr(self.b_agg), _ptr(self.ln_gamma),
+                               _ptr(self.ln_beta))
+
+
+def hg_layer_workspace_size(g: Graph, params: LayerParams) -> tuple:
+    s, k = c_size_t(0), c_size_t(0)
+    p = params.c()
+    _check(lib().hg_layer_workspace_size(g.handle, byref(p), byref(s), byref(k)), "hg_layer_workspace_size")
+    return s.value, k.value
+
+
+def hg_layer_fwd(g: Graph, params: LayerParams, H_in, H_out, saved, scratch, stream=None):
+    p = params.c()
+    _check(lib().hg_layer_fwd(g.handle, byref(p), _ptr(H_in), _ptr(H_out), _ptr(saved), _ptr(scratch),
+                              _stream(stream)), "hg_layer_fwd")
+
+
+def hg_layer_bwd(g: Graph, params: LayerParams, H_in, saved, dH_out, dH_in, grads: dict, scratch, stream=None):
+    p = params.c()
+    gr = hg_layer_grads(_ptr(grads["W_rel"]), _ptr(grads["W_agg"]), _ptr(grads["b_agg"]), _ptr(grads.get("ln_gamma")),
+                        _ptr(grads.get("ln_beta")))
+    _check(lib().hg_layer_bwd(g.handle, byref(p), _ptr(H_in), _ptr(saved), _ptr(dH_out), _ptr(dH_in), byref(gr),
+                              _ptr(scratch), _stream(stream)), "hg_layer_bwd")
+
+
+# ------------------------------------------------------------------------------------------------
+# overlap + alignment
+# ------------------------------------------------------------------------------------------------
+def hg_overlap_intersect_workspace_size(n_a: int, n_b: int) -> int:
+    n = c_size_t(0)
+    _check(lib().hg_overlap_intersect_workspace_size(int(n_a), int(n_b), byref(n)), "hg_overlap_intersect_workspace_size")
+    return n.value
+
+
+def hg_overlap_intersect(gid_a, gid_b, idx_a, idx_b, n_out, scratch, stream=None):
+    _check(lib().hg_overlap_intersect(_ptr(gid_a), gid_a.numel(), _ptr(gid_b), gid_b.numel(), _ptr(idx_a), _ptr(idx_b),
+                                      _ptr(n_out), _ptr(scratch), scratch.numel(), _stream(stream)),
+           "hg_overlap_intersect")
+
+
+def hg_overlap_align_workspace_size(n_max: int, d: int) -> tuple:
+    s, k = c_size_t(0), c_size_t(0)
+    _check(lib().hg_overlap_align_workspace_size(int(n_max), int(d), byref(s), byref(k)),
+           "hg_overlap_align_workspace_size")
+    return s.value, k.value
+
+
+def _dtype_of(t) -> int:
+    return HG_F32 if t.dtype == torch.float32 else HG_BF16
+
+
+def hg_overlap_align_loss(H_a, idx_a, H_b, idx_b, n_max: int, n_dev, lambda_n: float, var_eps: float, loss_out, saved,
+                          scratch, stream=None):
+    _check(lib().hg_overlap_align_loss(_ptr(H_a), H_a.shape[0], _ptr(idx_a), _ptr(H_b), H_b.shape[0], _ptr(idx_b),
+                                       int(n_max), _ptr(n_dev),
+                                       int(H_a.shape[-1]), _dtype_of(H_a), float(lambda_n), float(var_eps),
+                                       _ptr(loss_out), _ptr(saved), _ptr(scratch), _stream(stream)),
+           "hg_overlap_align_loss")
+
+
+def hg_overlap_align_bwd(H_a, idx_a, H_b, idx_b, n_max: int, n_dev, lambda_n: float, var_eps: float, dloss: float,
+                         saved, dH_a, dH_b, scratch, stream=None):
+    _check(lib().hg_overlap_align_bwd(_ptr(H_a), H_a.shape[0], _ptr(idx_a), _ptr(H_b), H_b.shape[0], _ptr(idx_b),
+                                      int(n_max), _ptr(n_dev),
+                                      int(H_a.shape[-1]), _dtype_of(H_a), float(lambda_n), float(var_eps),
+                                      float(dloss), _ptr(saved), _ptr(dH_a), _ptr(dH_b), _ptr(scratch),
+                                      _stream(stream)), "hg_overlap_align_bwd")
+
+
+# ------------------------------------------------------------------------------------------------
+# timing
+# ------------------------------------------------------------------------------------------------
+def hg_timing_enable(on: bool):
+    _check(lib().hg_timing_enable(1 if on else 0), "hg_timing_enable")
+
+
+def hg_timing_report() -> dict:
+    """Synchronises; returns {kernel name: (launches, total ms)} since the last report."""
+    buf = ctypes.create_string_buffer(1 << 16)
+    _check(lib().hg_timing_report(buf, len(buf)), "hg_timing_report")
+    out = {}
+    for line in buf.value.decode().splitlines():
+        name, n, ms = line.split()
+        out[name] = (int(n), float(ms))
+    return out

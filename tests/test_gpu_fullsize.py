@@ -1,0 +1,135 @@
+"""The 1M-node / 20M-edge bf16 workload at full size, in the launch configuration the benchmark
+times: the CSR layout is checked by the invariants that determine it uniquely, the layer on
+sampled rows the oracle computes one by one, and the weight gradients exactly by giving the
+upstream gradient a sampled support (only those rows contribute)."""
+import numpy as np
+import pytest
+import torch
+
+import hgsynth
+import oracle
+from tests.gpu_util import TOL, dev, grad_bufs, host, layer_params, lib, need_gpu, relerr, tdtype
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def full():
+    need_gpu()
+    hg = lib()
+    sp = hgsynth.spec("sub-1m")
+    w = hgsynth.make_workload(sp, random_affine=True, with_ids=True)
+    g = w.graph
+    G = hg.hg_build_csr(dev(g["src"]), dev(g["dst"]), dev(g["rel"]), g["type_offsets"], g["rels"])
+    assert hg.hg_graph_check(G) == 0
+    return hg, sp, w, G
+
+
+def test_full_csr_invariants(full):
+    hg, sp, w, G = full
+    g = w.graph
+    src, dst, rel = g["src"].astype(np.int64), g["dst"].astype(np.int64), g["rel"]
+    offs = g["type_offsets"]
+    seen = np.zeros(len(src), bool)
+    for r, (ts, tt) in enumerate(g["rels"]):
+        v = hg.hg_graph_view(G, r)
+        rp = v["row_ptr"].cpu().numpy().astype(np.int64)
+        a, b = rp[0], rp[-1]
+        eid = v["eid"][a:b].cpu().numpy().astype(np.int64)
+        col = v["col"][a:b].cpu().numpy()
+        deg = np.diff(rp)
+        rows = np.repeat(np.arange(len(deg)), deg)
+        assert np.all(deg >= 0) and b - a == int((rel == r).sum())
+        assert np.all(rel[eid] == r) and np.all(dst[eid] - offs[tt] == rows) and np.array_equal(src[eid], col)
+        same = rows[1:] == rows[:-1]
+        assert np.all(np.diff(eid)[same] > 0)  # ascending edge id within a row
+        assert not seen[eid].any()
+        seen[eid] = True
+        cp = v["csc_ptr"].cpu().numpy().astype(np.int64)
+        ca, cb = cp[0], cp[-1]
+        ceid = v["csc_eid"][ca:cb].cpu().numpy().astype(np.int64)
+        crow = np.repeat(np.arange(len(cp) - 1), np.diff(cp))
+        assert np.all(src[ceid] - offs[ts] == crow) and np.all(rel[ceid] == r)
+        assert np.all(np.diff(ceid)[crow[1:] == crow[:-1]] > 0)
+        coef = v["csc_coef"][ca:cb].cpu().numpy()
+        want = np.float32(1) / deg[dst[ceid] - offs[tt]].astype(np.float32)
+        assert np.array_equal(coef.view(np.uint32), want.view(np.uint32))
+    assert seen.all()
+
+
+def sample_rows(w, k, seed):
+    """Random rows of both types plus the largest in-degree hubs and some rows with no in-edges."""
+    g = w.graph
+    n = int(g["type_offsets"][-1])
+    rng = np.random.default_rng(seed)
+    indeg = np.bincount(g["dst"], minlength=n)
+    hubs = np.argsort(-indeg, kind="stable")[:8]
+    isolated = np.flatnonzero(indeg == 0)[:8]
+    risk = int(g["type_offsets"][1]) + rng.choice(n - int(g["type_offsets"][1]), k // 4, replace=False)
+    return np.unique(np.concatenate([rng.choice(n, k, replace=False), hubs, isolated, risk]))
+
+
+def test_full_layer_sampled_rows(full):
+    hg, sp, w, G = full
+    g = w.graph
+    td = tdtype(sp.dtype)
+    p = w.params[0]
+    P = layer_params(hg, p, sp.dtype)
+    sb, kb = hg.hg_layer_workspace_size(G, P)
+    saved = torch.empty(sb, dtype=torch.uint8, device="cuda")
+    scratch = torch.empty(kb, dtype=torch.uint8, device="cuda")
+    X = dev(w.X, td)
+    out = torch.empty_like(X)
+    hg.hg_layer_fwd(G, P, X, out, saved, scratch)
+    rows = sample_rows(w, 3000, 1)
+    ref, _ = oracle.layer_forward_rows(g["src"], g["dst"], g["rel"], g["type_offsets"], g["rels"], p, w.X, rows)
+    assert relerr(host(out[torch.from_numpy(rows).cuda()]), ref) <= TOL[sp.dtype]
+    # backward with an upstream gradient supported on a row sample S
+    S = sample_rows(w, 2000, 2)
+    dH_out = torch.zeros_like(X)
+    dH_out[torch.from_numpy(S).cuda()] = dev(w.dH_top[S], td)
+    dH_in = torch.empty_like(X)
+    grads = grad_bufs(len(g["rels"]), 2, sp.d)
+    hg.hg_layer_bwd(G, P, X, saved, dH_out, dH_in, grads, scratch)
+    # query rows: S itself, sources of edges into S (they receive the transposed gather) and others
+    into_S = np.unique(g["src"][np.isin(g["dst"], S)])
+    rng = np.random.default_rng(3)
+    q = np.unique(np.concatenate([S[:500], rng.choice(into_S, min(1500, len(into_S)), replace=False),
+                                  rng.choice(int(g["type_offsets"][-1]), 500, replace=False)]))
+    dq, gref = oracle.layer_backward_rows(g["src"], g["dst"], g["rel"], g["type_offsets"], g["rels"], p, w.X, S,
+                                          w.dH_top[S], q)
+    tol = TOL[sp.dtype]
+    assert relerr(host(dH_in[torch.from_numpy(q).cuda()]), dq) <= tol
+    for k, v in gref.items():
+        assert relerr(host(grads[k]), v) <= tol, (k, relerr(host(grads[k]), v))
+
+
+def test_full_overlap_and_alignment(full):
+    hg, sp, w, G = full
+    td = tdtype(sp.dtype)
+    n_a, n_b = len(w.gid_a), len(w.gid_b)
+    cap = min(n_a, n_b)
+    idx_a = torch.empty(cap, dtype=torch.int32, device="cuda")
+    idx_b = torch.empty(cap, dtype=torch.int32, device="cuda")
+    n_dev = torch.zeros(1, dtype=torch.int64, device="cuda")
+    scr = torch.empty(hg.hg_overlap_intersect_workspace_size(n_a, n_b), dtype=torch.uint8, device="cuda")
+    hg.hg_overlap_intersect(dev(w.gid_a), dev(w.gid_b), idx_a, idx_b, n_dev, scr)
+    ia, ib = oracle.overlap_intersect(w.gid_a, w.gid_b)
+    n = int(n_dev.item())
+    assert n == len(ia) == sp.n_overlap
+    assert np.array_equal(idx_a[:n].cpu().numpy(), ia) and np.array_equal(idx_b[:n].cpu().numpy(), ib)
+    # the overlap rows are long-tail nodes (total degree <= 2, hence h-index <= 2)
+    deg = np.bincount(w.graph["src"], minlength=sp.num_nodes) + np.bincount(w.graph["dst"], minlength=sp.num_nodes)
+    assert deg[ia].max() <= 2
+    s, k = hg.hg_overlap_align_workspace_size(cap, sp.d)
+    saved = torch.empty(s, dtype=torch.uint8, device="cuda")
+    scratch = torch.empty(k, dtype=torch.uint8, device="cuda")
+    loss = torch.empty(3, dtype=torch.float32, device="cuda")
+    A, B = dev(w.X, td), dev(w.H_b, td)
+    hg.hg_overlap_align_loss(A, idx_a, B, idx_b, cap, n_dev, 2e-4, 1e-8, loss, saved, scratch)
+    dA = torch.zeros_like(A)
+    hg.hg_overlap_align_bwd(A, idx_a, B, idx_b, cap, n_dev, 2e-4, 1e-8, 0.1, saved, dA, None, scratch)
+    ref = oracle.align_forward(w.X, ia, w.H_b, ib, 2e-4, 1e-8)
+    assert relerr(host(loss), np.array(ref)) <= 1e-4
+    rA, _ = oracle.align_backward(w.X, ia, w.H_b, ib, 2e-4, 1e-8, 0.1)
+    assert relerr(host(dA)[ia], rA[ia]) <= TOL[sp.dtype]

@@ -1,0 +1,90 @@
+"""The C-ABI library loads, exports every entry point include/hg.h declares, and rejects bad
+arguments on the host before touching the GPU (CPU only: no compute call is made)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def hg():
+    from paper_2608_02168_gb300 import build
+    build.build()
+    from paper_2608_02168_gb300 import hg as binding
+    return binding
+
+
+def declared_functions():
+    text = open(os.path.join(ROOT, "include", "hg.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\*?\s+(hg_\w+)\s*\(", text, flags=re.M)))
+
+
+def test_every_declared_symbol_is_exported(hg):
+    names = declared_functions()
+    assert len(names) >= 17, names
+    so = hg.lib()
+    for n in names:
+        assert hasattr(so, n), n
+    assert set(names) == set(hg.EXPORTS), "binding and header disagree"
+
+
+def test_status_strings_and_version(hg):
+    so = hg.lib()
+    assert so.hg_abi_version() == 1
+    assert so.hg_status_string(0) == b"ok"
+    assert so.hg_status_string(3) == b"workspace too small"
+
+
+def test_workspace_queries_are_host_only(hg):
+    n = hg.hg_graph_workspace_size(1000, [0, 80, 100], [(0, 0), (0, 1), (1, 0)])
+    assert n > 1000 * 4 * 7
+    s, k = hg.hg_overlap_align_workspace_size(500, 64)
+    assert s >= 4 * 64 * 4 + 2 * 64 * 64 * 4 and k > 2 * 500 * 64 * 4
+    assert hg.hg_overlap_intersect_workspace_size(10, 20) > 0
+
+
+def test_host_argument_checks(hg):
+    so = hg.lib()
+    offs = (ctypes.c_int64 * 3)(0, 8, 10)
+    rels = (hg.hg_rel_desc * 1)(hg.hg_rel_desc(0, 1))
+    out = ctypes.c_void_p()
+    # null edge arrays with edges
+    assert so.hg_build_csr(None, None, None, 5, offs, 2, rels, 1, 256, 1 << 20, None, ctypes.byref(out)) == 1
+    # too many relation types
+    assert so.hg_graph_workspace_size(5, offs, 2, rels, 9, ctypes.byref(ctypes.c_size_t())) == 2
+    # edge count beyond int32
+    assert so.hg_graph_workspace_size(1 << 31, offs, 2, rels, 1, ctypes.byref(ctypes.c_size_t())) == 2
+    # a relation pointing at a type that does not exist
+    bad = (hg.hg_rel_desc * 1)(hg.hg_rel_desc(0, 2))
+    assert so.hg_graph_workspace_size(5, offs, 2, bad, 1, ctypes.byref(ctypes.c_size_t())) == 1
+    assert b"type out of range" in so.hg_last_error()
+    # workspace smaller than the query (fake aligned address: rejected before any device access)
+    assert so.hg_build_csr(256, 256, 256, 5, offs, 2, rels, 1, 256, 16, None, ctypes.byref(out)) == 3
+    # unsupported feature width for the alignment
+    assert so.hg_overlap_align_loss(256, 10, 256, 256, 10, 256, 4, None, 96, 0, 0.0, 0.0, 256, 256, 256, None) == 2
+    # negative overlap size; empty tables with a non-empty overlap
+    assert so.hg_overlap_align_loss(256, 10, 256, 256, 10, 256, -1, None, 64, 0, 0.0, 0.0, 256, 256, 256, None) == 1
+    assert so.hg_overlap_align_bwd(256, 0, 256, 256, 10, 256, 4, None, 64, 0, 0.0, 0.0, 1.0, 256, 256, None, 256,
+                                   None) == 1
+    # unsorted ids are a device-side condition; a null n_out is a host one
+    assert so.hg_overlap_intersect(256, 4, 256, 4, 256, 256, None, 256, 1 << 20, None) == 1
+
+
+def test_timing_report_empty(hg):
+    hg.hg_timing_enable(True)
+    assert hg.hg_timing_report() == {}
+    hg.hg_timing_enable(False)
+
+
+def test_product_path_has_no_fallback():
+    """The binding and step driver import neither the oracle nor any CPU implementation."""
+    pkg = os.path.join(ROOT, "paper_2608_02168_gb300")
+    for f in os.listdir(pkg):
+        if f.endswith(".py"):
+            src = open(os.path.join(pkg, f)).read()
+            assert "oracle" not in src.replace("oracle.", ""), f
+            assert "import numpy" not in src, f
