@@ -32,6 +32,15 @@ Readings where the paper is silent or ambiguous (listed again in the design note
   alignment standardisation uses the population standard deviation with eps added to the
   variance; both loss terms are plain sums (squared Frobenius norms); lambda_n = 2e-4.
 
+Storage precision of intermediates (store="bf16").  For bf16 workloads the kernels store the
+relation means M_r, the first product Z and the pre-activation U in bf16, and the activation and
+its derivative are taken at the stored U.  The ReLU mask is an integer decision made by floating
+point, and the paper fixes no precision, so the oracle takes that decision in the kernel's
+precision: with store="bf16" it rounds M_r, Z and U to bf16 (round to nearest, ties to even; its
+own rounding routine) and keeps every other operation in fp64.  store="f64" (default)
+is the plain definition.  Without this, pre-activations within a bf16 rounding of zero flip their
+mask, and the long transposed sums of hub rows amplify those flips far beyond the bf16 tolerance.
+
 Functions that no independent pin covers are marked "parity unpinned" in their docstring; every
 function here has pins in tests/test_oracle_*.py.
 """
@@ -41,6 +50,23 @@ import numpy as np
 
 F64 = np.float64
 GELU_K = float(np.sqrt(2.0 / np.pi))
+
+
+def round_bf16(x: np.ndarray) -> np.ndarray:
+    """Round to the nearest bfloat16 (ties to even) via fp32: keep the top 16 bits of the fp32
+    pattern after adding 0x7FFF plus the lowest kept bit.  Returns fp64 values."""
+    f = np.ascontiguousarray(np.asarray(x, np.float64).astype(np.float32))
+    u = f.view(np.uint32).astype(np.uint64)
+    r = ((u + 0x7FFF + ((u >> 16) & 1)) & 0xFFFF0000).astype(np.uint32)
+    return r.view(np.float32).astype(np.float64).reshape(f.shape)
+
+
+def _stored(x: np.ndarray, store: str) -> np.ndarray:
+    if store == "f64":
+        return x
+    if store == "bf16":
+        return round_bf16(x)
+    raise ValueError(store)
 
 
 # ----------------------------------------------------------------------------------------------
@@ -133,7 +159,7 @@ def _p64(params: dict) -> dict:
 
 
 def layer_forward(csr: list, type_offsets, rels, params: dict, H, act: str = "relu",
-                  layernorm: bool = True, ln_eps: float = 1e-5) -> tuple:
+                  layernorm: bool = True, ln_eps: float = 1e-5, store: str = "f64") -> tuple:
     """H_out[j] = LN_tau(act(Z[j] W_agg[tau] + b[tau]) + H[j]),  Z[j] = sum_{r: t_r = tau} M_r[j] W_r.
     Eq. 7 (one W_r per relation), Eq. 10 (mean), Eq. 11 (update + residual), LayerNorm optional.
     Returns (H_out, cache) with the intermediates per type."""
@@ -148,10 +174,11 @@ def layer_forward(csr: list, type_offsets, rels, params: dict, H, act: str = "re
         for r, (_, tt) in enumerate(rels):
             if tt != t:
                 continue
-            M = mean_aggregate(csr[r], H)
+            M = _stored(mean_aggregate(csr[r], H), store)
             cache["M"][r] = M
             Z += M @ p["W_rel"][r]
-        U = Z @ p["W_agg"][t] + p["b_agg"][t]
+        Z = _stored(Z, store)
+        U = _stored(Z @ p["W_agg"][t] + p["b_agg"][t], store)
         Y = act_fwd(U, act) + H[lo:hi]
         c = {"Z": Z, "U": U, "Y": Y}
         if layernorm:
@@ -168,14 +195,14 @@ def layer_forward(csr: list, type_offsets, rels, params: dict, H, act: str = "re
 
 
 def layer_backward(csr: list, type_offsets, rels, params: dict, H, dH_out, act: str = "relu",
-                   layernorm: bool = True, ln_eps: float = 1e-5) -> tuple:
+                   layernorm: bool = True, ln_eps: float = 1e-5, store: str = "f64") -> tuple:
     """Gradients of layer_forward: returns (dH_in, grads) with grads = dict(W_rel, W_agg, b_agg,
     ln_gamma, ln_beta).  dH_in = residual path + transpose of the mean aggregation."""
     p = _p64(params)
     H = np.asarray(H, F64)
     dH_out = np.asarray(dH_out, F64)
     offs = np.asarray(type_offsets, np.int64)
-    _, cache = layer_forward(csr, type_offsets, rels, params, H, act, layernorm, ln_eps)
+    _, cache = layer_forward(csr, type_offsets, rels, params, H, act, layernorm, ln_eps, store)
     d = H.shape[1]
     R, T = len(rels), len(offs) - 1
     g = dict(W_rel=np.zeros((R, d, d)), W_agg=np.zeros((T, d, d)), b_agg=np.zeros((T, d)),
@@ -233,7 +260,7 @@ def _row_aggregates(src, dst, rel, valid, rows_sorted, H, R, chunk=1 << 20):
 
 
 def layer_forward_rows(src, dst, rel, type_offsets, rels, params, H, rows, act="relu",
-                       layernorm=True, ln_eps=1e-5) -> tuple:
+                       layernorm=True, ln_eps=1e-5, store="f64") -> tuple:
     """layer_forward evaluated only at node ids `rows` (sorted, unique), straight from the COO list.
     Returns (H_out[rows], cache) with per-row M (n x R x d), Z, U, deg, Xh, rstd."""
     src = np.asarray(src, np.int64)
@@ -244,7 +271,7 @@ def layer_forward_rows(src, dst, rel, type_offsets, rels, params, H, rows, act="
     valid = valid_edges(src, dst, rel, type_offsets, rels)
     R = len(rels)
     S, deg = _row_aggregates(src, dst, rel, valid, rows, H, R)
-    M = np.where(deg[:, :, None] > 0, S / np.maximum(deg, 1)[:, :, None], 0.0)
+    M = _stored(np.where(deg[:, :, None] > 0, S / np.maximum(deg, 1)[:, :, None], 0.0), store)
     ty = node_type(rows, type_offsets)
     d = H.shape[1]
     Z = np.zeros((rows.shape[0], d), F64)
@@ -252,7 +279,8 @@ def layer_forward_rows(src, dst, rel, type_offsets, rels, params, H, rows, act="
     for r in range(R):
         m = ty == rt[r]
         Z[m] += M[m, r] @ p["W_rel"][r]
-    U = np.einsum("nk,nkj->nj", Z, p["W_agg"][ty]) + p["b_agg"][ty]
+    Z = _stored(Z, store)
+    U = _stored(np.einsum("nk,nkj->nj", Z, p["W_agg"][ty]) + p["b_agg"][ty], store)
     Y = act_fwd(U, act) + np.asarray(H, F64)[rows]
     cache = dict(M=M, Z=Z, U=U, Y=Y, deg=deg, ty=ty)
     if layernorm:
@@ -266,7 +294,7 @@ def layer_forward_rows(src, dst, rel, type_offsets, rels, params, H, rows, act="
 
 
 def layer_backward_rows(src, dst, rel, type_offsets, rels, params, H, S_rows, dH_S, query_rows,
-                        act="relu", layernorm=True, ln_eps=1e-5) -> tuple:
+                        act="relu", layernorm=True, ln_eps=1e-5, store="f64") -> tuple:
     """layer_backward for an upstream gradient that is zero except on the sorted node ids S_rows
     (values dH_S).  Returns (dH_in[query_rows], grads); the weight gradients are complete because
     only rows in S_rows contribute to them."""
@@ -276,7 +304,7 @@ def layer_backward_rows(src, dst, rel, type_offsets, rels, params, H, S_rows, dH
     p = _p64(params)
     S_rows = np.asarray(S_rows, np.int64)
     query_rows = np.asarray(query_rows, np.int64)
-    _, c = layer_forward_rows(src, dst, rel, type_offsets, rels, params, H, S_rows, act, layernorm, ln_eps)
+    _, c = layer_forward_rows(src, dst, rel, type_offsets, rels, params, H, S_rows, act, layernorm, ln_eps, store)
     ty = c["ty"]
     dout = np.asarray(dH_S, F64)
     d = dout.shape[1]
@@ -392,25 +420,30 @@ def overlap_intersect(gid_a, gid_b) -> tuple:
 # one whole step of the hot path (used for the CPU baseline and small end-to-end checks)
 # ----------------------------------------------------------------------------------------------
 def step(graph: dict, X, params: list, dH_top, view_b: dict, act="relu", layernorm=True,
-         ln_eps=1e-5, lambda_n=2e-4, var_eps=1e-8, dloss=0.1) -> dict:
+         ln_eps=1e-5, lambda_n=2e-4, var_eps=1e-8, dloss=0.1, store="f64") -> dict:
     """CSR build -> L layers forward -> overlap rows -> alignment loss and gradient -> L layers
-    backward.  `view_b` is either {"H_b": bank rows, "gid_a", "gid_b"} (a detached neighbour view)
+    backward.  With store="bf16" the tensors handed from layer to layer (outputs, their gradients)
+    are rounded to bf16 as well, like every bf16 tensor the layer interface exchanges.  `view_b` is either {"H_b": bank rows, "gid_a", "gid_b"} (a detached neighbour view)
     or {"idx": overlap rows, "X_b": second input} (a second live stack on the same graph).
     The last layer's upstream gradient is dH_top plus the alignment gradient."""
     offs, rels = graph["type_offsets"], graph["rels"]
     csr = build_csr(graph["src"], graph["dst"], graph["rel"], offs, rels)
 
+    # layer outputs and gradients passed between layers are tensors of the storage type
+    io = (lambda x: x) if store == "f64" else round_bf16
+
     def run_stack(H0):
         hs = [np.asarray(H0, F64)]
         for p in params:
-            hs.append(layer_forward(csr, offs, rels, p, hs[-1], act, layernorm, ln_eps)[0])
+            hs.append(io(layer_forward(csr, offs, rels, p, hs[-1], act, layernorm, ln_eps, store)[0]))
         return hs
 
     def back_stack(hs, dtop):
         grads = [None] * len(params)
-        dh = dtop
+        dh = io(dtop)
         for l in range(len(params) - 1, -1, -1):
-            dh, grads[l] = layer_backward(csr, offs, rels, params[l], hs[l], dh, act, layernorm, ln_eps)
+            dh, grads[l] = layer_backward(csr, offs, rels, params[l], hs[l], dh, act, layernorm, ln_eps, store)
+            dh = io(dh)
         return dh, grads
 
     hs = run_stack(X)

@@ -7,10 +7,10 @@
 // rows [row_base[r], row_base[r+1]) = its destination type's nodes in local order, and CSC rows
 // [csc_base[r], csc_base[r+1]) = its source type's nodes.
 //
-// Construction: each edge gets a row key (or a sentinel key past the last row when invalid), the
-// row degrees are counted with integer atomics (order-free) and scanned into row pointers, and a
+// Construction: each edge gets a row key (or a sentinel key past the last row when invalid), a
 // STABLE least-significant-digit radix sort of (key, edge id) places every edge in its row with
-// ascending edge ids.  The layout is therefore unique and bit-reproducible.
+// ascending edge ids, and the row pointers are read off the sorted keys (no atomics, so hub rows
+// cost nothing extra).  The layout is therefore unique and bit-reproducible.
 #include <algorithm>
 
 #include "hg_internal.cuh"
@@ -223,15 +223,14 @@ static hg_status radix_sort(SortBuffers& b, int64_t n, int bits, cudaStream_t s,
 // ---------------------------------------------------------------------------------------------
 __global__ void edge_keys(const int32_t* __restrict__ src, const int32_t* __restrict__ dst,
                           const int32_t* __restrict__ rel, int64_t E, GraphMeta m, int by_dst,
-                          int64_t rows, uint32_t* __restrict__ keys, uint32_t* __restrict__ vals,
-                          int32_t* __restrict__ deg, int32_t* __restrict__ invalid) {
+                          int64_t rows, uint32_t* __restrict__ keys, uint32_t* __restrict__ vals) {
   const int64_t N = m.type_off[m.num_types];
   for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < E;
        e += (int64_t)gridDim.x * blockDim.x) {
     const int r = rel[e];
     const int64_t s = src[e], t = dst[e];
     bool ok = r >= 0 && r < m.num_rels && s >= 0 && s < N && t >= 0 && t < N;
-    int64_t key = rows;
+    int64_t key = rows;  // invalid edges sort after every row
     if (ok) {
       ok = node_type_of(m, s) == m.rel_src[r] && node_type_of(m, t) == m.rel_dst[r];
       if (ok)
@@ -240,17 +239,27 @@ __global__ void edge_keys(const int32_t* __restrict__ src, const int32_t* __rest
     }
     keys[e] = (uint32_t)key;
     vals[e] = (uint32_t)e;
-    if (ok)
-      atomicAdd(&deg[key], 1);
-    else if (invalid)
-      atomicAdd(invalid, 1);
+  }
+}
+
+// Row pointers from the sorted keys: ptr[k] = first position whose key is >= k, k in [0, rows].
+// Position p owns the rows k with key[p-1] < k <= key[p] (key[-1] = -1, key[n] = rows), so every
+// entry is written exactly once and empty rows get the position of the next non-empty one.
+__global__ void row_ptr_from_keys(const uint32_t* __restrict__ keys, int64_t n, int64_t rows,
+                                  int32_t* __restrict__ ptr) {
+  for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p <= n;
+       p += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t lo = p == 0 ? 0 : (int64_t)keys[p - 1] + 1;
+    const int64_t hi = p == n ? rows : min((int64_t)keys[p], rows);
+    for (int64_t k = lo; k <= hi; ++k) ptr[k] = (int32_t)p;
   }
 }
 
 __global__ void csr_finish(const uint32_t* __restrict__ eid_sorted, const int32_t* __restrict__ ptr,
                            int64_t rows, int64_t E, const int32_t* __restrict__ src,
-                           int32_t* __restrict__ col, int32_t* __restrict__ eid) {
+                           int32_t* __restrict__ col, int32_t* __restrict__ eid, int32_t* __restrict__ invalid) {
   const int64_t nv = ptr[rows];
+  if (blockIdx.x == 0 && threadIdx.x == 0) *invalid = (int32_t)(E - nv);
   for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < nv;
        p += (int64_t)gridDim.x * blockDim.x) {
     const uint32_t e = eid_sorted[p];
@@ -427,33 +436,30 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
   carve_graph(workspace, E, rows, crows, &L);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
 
-  HG_CUDA(cudaMemsetAsync(L.csr_ptr, 0, (rows + 1) * sizeof(int32_t), s));
-  HG_CUDA(cudaMemsetAsync(L.csc_ptr, 0, (crows + 1) * sizeof(int32_t), s));
-  HG_CUDA(cudaMemsetAsync(L.invalid, 0, sizeof(int32_t), s));
-  const unsigned g = grid_for(E);
+  const unsigned g = grid_for(E + 1);
   int res = 0;
-  // CSR by destination
-  if (E > 0) {
-    HG_TRY(launch("edge_keys", edge_keys, dim3(g), dim3(256), 0, s, src, dst, rel, E, m, 1, rows,
-                  L.sort.keys[0], L.sort.vals[0], L.csr_ptr, L.invalid));
-  }
-  HG_TRY(exclusive_scan(L.csr_ptr, L.csr_ptr, rows, L.sort.scan_scratch, s));
-  if (E > 0) {
+  if (E == 0) {
+    HG_CUDA(cudaMemsetAsync(L.csr_ptr, 0, (rows + 1) * sizeof(int32_t), s));
+    HG_CUDA(cudaMemsetAsync(L.csc_ptr, 0, (crows + 1) * sizeof(int32_t), s));
+    HG_CUDA(cudaMemsetAsync(L.invalid, 0, sizeof(int32_t), s));
+  } else {
+    // CSR by destination
+    HG_TRY(launch("edge_keys", edge_keys, dim3(g), dim3(256), 0, s, src, dst, rel, E, m, 1, rows, L.sort.keys[0],
+                  L.sort.vals[0]));
     HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)rows), s, &res));
+    HG_TRY(launch("row_ptr_from_keys", row_ptr_from_keys, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[res],
+                  E, rows, L.csr_ptr));
     HG_TRY(launch("csr_finish", csr_finish, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.vals[res],
-                  (const int32_t*)L.csr_ptr, rows, E, src, L.csr_col, L.csr_eid));
-  }
-  // CSC by source
-  if (E > 0) {
-    HG_TRY(launch("edge_keys", edge_keys, dim3(g), dim3(256), 0, s, src, dst, rel, E, m, 0, crows,
-                  L.sort.keys[0], L.sort.vals[0], L.csc_ptr, (int32_t*)nullptr));
-  }
-  HG_TRY(exclusive_scan(L.csc_ptr, L.csc_ptr, crows, L.sort.scan_scratch, s));
-  if (E > 0) {
+                  (const int32_t*)L.csr_ptr, rows, E, src, L.csr_col, L.csr_eid, L.invalid));
+    // CSC by source
+    HG_TRY(launch("edge_keys", edge_keys, dim3(g), dim3(256), 0, s, src, dst, rel, E, m, 0, crows, L.sort.keys[0],
+                  L.sort.vals[0]));
     HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)crows), s, &res));
+    HG_TRY(launch("row_ptr_from_keys", row_ptr_from_keys, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[res],
+                  E, crows, L.csc_ptr));
     HG_TRY(launch("csc_finish", csc_finish, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.vals[res],
-                  (const int32_t*)L.csc_ptr, crows, dst, rel, m, (const int32_t*)L.csr_ptr, L.csc_col,
-                  L.csc_eid, L.csc_coef));
+                  (const int32_t*)L.csc_ptr, crows, dst, rel, m, (const int32_t*)L.csr_ptr, L.csc_col, L.csc_eid,
+                  L.csc_coef));
   }
   // chunk tables for rows above the hub degree
   HG_TRY(launch("chunk_counts", chunk_counts, dim3(grid_for(rows)), dim3(256), 0, s,

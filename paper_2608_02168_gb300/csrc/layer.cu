@@ -81,6 +81,7 @@ struct LayerLayout {
   void* dMs;      // scratch: csr_rows x d
   float* cpart;   // scratch: row blocks x 3 x d
   float* wpart;   // scratch: splits x d x d
+  float* rtmp;    // scratch: levels of the fixed-order reductions
   void* WrelT;    // scratch: R x d x d
   void* WaggT;    // scratch: T x d x d
 };
@@ -106,6 +107,8 @@ static void carve_layer(const hg_graph* g, int d, hg_dtype dt, void* saved, void
   for (int t = 0; t < m.num_types; ++t) max_rows = std::max(max_rows, m.type_off[t + 1] - m.type_off[t]);
   L->cpart = k.take<float>((size_t)ceil_div(max_rows, 64) * 3 * d);
   L->wpart = k.take<float>((size_t)wgrad_splits(max_rows) * d * d);
+  L->rtmp = k.take<float>(std::max(reduce_tmp_floats((int)ceil_div(max_rows, 64), d),
+                                   reduce_tmp_floats(wgrad_splits(max_rows), (int64_t)d * d)));
   L->WrelT = k.take<char>((size_t)m.num_rels * d * d * b);
   L->WaggT = k.take<char>((size_t)m.num_types * d * d * b);
   if (saved_bytes) *saved_bytes = s.used;
@@ -305,18 +308,19 @@ extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* 
     a.ln = p->layernorm;
     HG_TRY(proj_backward(p->dtype, d, a, s));
     const int blocks = (int)ceil_div(n, 64);
-    HG_TRY(reduce_partials(L.cpart, 3LL * d, blocks, d, db, s));
+    HG_TRY(reduce_partials(L.cpart, 3LL * d, blocks, d, db, L.rtmp, s));
     if (p->layernorm) {
-      HG_TRY(reduce_partials(L.cpart + d, 3LL * d, blocks, d, grads->dln_gamma + (size_t)t * d, s));
-      HG_TRY(reduce_partials(L.cpart + 2 * d, 3LL * d, blocks, d, grads->dln_beta + (size_t)t * d, s));
+      HG_TRY(reduce_partials(L.cpart + d, 3LL * d, blocks, d, grads->dln_gamma + (size_t)t * d, L.rtmp, s));
+      HG_TRY(reduce_partials(L.cpart + 2 * d, 3LL * d, blocks, d, grads->dln_beta + (size_t)t * d, L.rtmp, s));
     }
-    HG_TRY(weight_grad(p->dtype, d, L.Z, a.off, L.dU, a.off, n, L.wpart, grads->dW_agg + (size_t)t * d * d, s));
+    HG_TRY(weight_grad(p->dtype, d, L.Z, a.off, L.dU, a.off, n, L.wpart, grads->dW_agg + (size_t)t * d * d, L.rtmp,
+                       s));
   }
   for (int r = 0; r < m.num_rels; ++r) {
     const int t = m.rel_dst[r];
     const int64_t n = m.type_off[t + 1] - m.type_off[t];
     HG_TRY(weight_grad(p->dtype, d, L.M, m.row_base[r], L.dZ, m.type_off[t], n, L.wpart,
-                       grads->dW_rel + (size_t)r * d * d, s));
+                       grads->dW_rel + (size_t)r * d * d, L.rtmp, s));
   }
   if (dH_in) HG_TRY(aggregate_backward(graph, p->dtype, d, L.dMs, L.dY, dH_in, L.agg_part, s));
   return HG_OK;

@@ -52,9 +52,12 @@ hg_status aggregate_backward(const hg_graph* g, hg_dtype dt, int d, const void* 
 hg_status proj_forward(hg_dtype dt, int d, const FwdArgs& a, cudaStream_t s);
 hg_status proj_backward(hg_dtype dt, int d, const BwdArgs& a, cudaStream_t s);
 hg_status weight_grad(hg_dtype dt, int d, const void* X, int64_t x0, const void* Y, int64_t y0, int64_t n, float* part,
-                      float* out, cudaStream_t s);
+                      float* out, float* tmp, cudaStream_t s);
 hg_status transpose_weights(hg_dtype dt, int d, const void* W, void* Wt, int count, cudaStream_t s);
-hg_status reduce_partials(const float* part, int64_t stride, int splits, int64_t count, float* out, cudaStream_t s);
+// fixed-order sum of `splits` partial arrays (tmp: reduce_tmp_floats(splits, count) floats)
+hg_status reduce_partials(const float* part, int64_t stride, int splits, int64_t count, float* out, float* tmp,
+                          cudaStream_t s);
+size_t reduce_tmp_floats(int splits, int64_t count);
 int wgrad_splits(int64_t n);
 
 }  // namespace hg

@@ -308,13 +308,46 @@ __global__ void __launch_bounds__(256) wgrad_partial(const T* __restrict__ X, in
   }
 }
 
-// out[i] = sum_{s < splits} part[s * stride + i], in split order
+// out[i] = sum_{s < splits} part[s * stride + i], added in split order; the loads of eight splits
+// are issued together so the chain of dependent adds does not wait on memory latency.
 __global__ void reduce_splits(const float* __restrict__ part, int64_t stride, int splits, int64_t count,
                               float* __restrict__ out) {
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < count; i += (int64_t)gridDim.x * blockDim.x) {
     float s = 0.f;
-    for (int k = 0; k < splits; ++k) s += part[(int64_t)k * stride + i];
+    int k = 0;
+    for (; k + 8 <= splits; k += 8) {
+      float v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) v[u] = __ldg(part + (int64_t)(k + u) * stride + i);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) s += v[u];
+    }
+    for (; k < splits; ++k) s += __ldg(part + (int64_t)k * stride + i);
     out[i] = s;
+  }
+}
+
+// out[g * count + i] = sum over splits [g * kRedGroup, (g + 1) * kRedGroup) of part, in order.
+constexpr int kRedGroup = 64;
+__global__ void reduce_groups(const float* __restrict__ part, int64_t stride, int splits, int64_t count,
+                              float* __restrict__ out) {
+  const int groups = (splits + kRedGroup - 1) / kRedGroup;
+  const int64_t total = (int64_t)groups * count;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+    const int g = (int)(e / count);
+    const int64_t i = e % count;
+    const int k0 = g * kRedGroup, k1 = min(splits, k0 + kRedGroup);
+    float s = 0.f;
+    int k = k0;
+    for (; k + 8 <= k1; k += 8) {
+      float v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) v[u] = __ldg(part + (int64_t)(k + u) * stride + i);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) s += v[u];
+    }
+    for (; k < k1; ++k) s += __ldg(part + (int64_t)k * stride + i);
+    out[e] = s;
   }
 }
 
@@ -363,17 +396,19 @@ int wgrad_splits(int64_t n) {
   return (int)std::max<int64_t>(1, std::min<int64_t>(304, ceil_div(n, 256)));
 }
 
+hg_status reduce_partials(const float* part, int64_t stride, int splits, int64_t count, float* out, float* tmp,
+                          cudaStream_t s);
+
 template <typename T, int D>
 static hg_status wgrad_t(const void* X, int64_t x0, const void* Y, int64_t y0, int64_t n, float* part, float* out,
-                         cudaStream_t s) {
+                         float* tmp, cudaStream_t s) {
   const int splits = wgrad_splits(n);
   const int64_t rps = ceil_div(std::max<int64_t>(n, 1), splits);
   constexpr int TW = D < kWT ? D : kWT;
   const int tiles = (D / TW) * (D / TW);
   HG_TRY(launch("wgrad_partial", wgrad_partial<T, D>, dim3(tiles, splits), dim3(256), 0, s, (const T*)X, x0,
                 (const T*)Y, y0, n, rps, part));
-  return launch("reduce_splits", reduce_splits, dim3((unsigned)std::min<int64_t>(ceil_div((int64_t)D * D, 256), 1024)),
-                dim3(256), 0, s, (const float*)part, (int64_t)D * D, splits, (int64_t)D * D, out);
+  return reduce_partials(part, (int64_t)D * D, splits, (int64_t)D * D, out, tmp, s);
 }
 
 template <typename T, int D>
@@ -400,13 +435,34 @@ static hg_status transpose_t(const void* W, void* Wt, int count, cudaStream_t s)
 hg_status proj_forward(hg_dtype dt, int d, const FwdArgs& a, cudaStream_t s) { HG_DISPATCH_TD2(dt, d, proj_fwd_t, a, s); }
 hg_status proj_backward(hg_dtype dt, int d, const BwdArgs& a, cudaStream_t s) { HG_DISPATCH_TD2(dt, d, proj_bwd_t, a, s); }
 hg_status weight_grad(hg_dtype dt, int d, const void* X, int64_t x0, const void* Y, int64_t y0, int64_t n, float* part,
-                      float* out, cudaStream_t s) {
-  HG_DISPATCH_TD2(dt, d, wgrad_t, X, x0, Y, y0, n, part, out, s);
+                      float* out, float* tmp, cudaStream_t s) {
+  HG_DISPATCH_TD2(dt, d, wgrad_t, X, x0, Y, y0, n, part, out, tmp, s);
 }
 hg_status transpose_weights(hg_dtype dt, int d, const void* W, void* Wt, int count, cudaStream_t s) {
   HG_DISPATCH_TD2(dt, d, transpose_t, W, Wt, count, s);
 }
-hg_status reduce_partials(const float* part, int64_t stride, int splits, int64_t count, float* out, cudaStream_t s) {
+size_t reduce_tmp_floats(int splits, int64_t count) {
+  const int64_t g1 = (splits + kRedGroup - 1) / kRedGroup;
+  const int64_t g2 = (g1 + kRedGroup - 1) / kRedGroup;
+  return (size_t)(g1 + g2 + 2) * count;
+}
+
+// Fixed-order sum over `splits` partial arrays: groups of kRedGroup are summed level by level (each
+// level fully parallel) until at most kRedGroup remain, then the last level writes `out`.
+hg_status reduce_partials(const float* part, int64_t stride, int splits, int64_t count, float* out, float* tmp,
+                          cudaStream_t s) {
+  const int64_t g1 = (splits + kRedGroup - 1) / kRedGroup;
+  float* buf[2] = {tmp, tmp + (g1 + 1) * count};
+  int which = 0;
+  while (splits > kRedGroup) {
+    const int groups = (splits + kRedGroup - 1) / kRedGroup;
+    HG_TRY(launch("reduce_groups", reduce_groups, dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div((int64_t)groups * count, 256), 152 * 16))),
+                  dim3(256), 0, s, part, stride, splits, count, buf[which]));
+    part = buf[which];
+    stride = count;
+    splits = groups;
+    which ^= 1;
+  }
   return launch("reduce_splits", reduce_splits, dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(count, 256), 1024))),
                 dim3(256), 0, s, part, stride, splits, count, out);
 }

@@ -82,7 +82,8 @@ def test_full_layer_sampled_rows(full):
     out = torch.empty_like(X)
     hg.hg_layer_fwd(G, P, X, out, saved, scratch)
     rows = sample_rows(w, 3000, 1)
-    ref, _ = oracle.layer_forward_rows(g["src"], g["dst"], g["rel"], g["type_offsets"], g["rels"], p, w.X, rows)
+    ref, _ = oracle.layer_forward_rows(g["src"], g["dst"], g["rel"], g["type_offsets"], g["rels"], p, w.X, rows,
+                                       store="bf16")
     assert relerr(host(out[torch.from_numpy(rows).cuda()]), ref) <= TOL[sp.dtype]
     # backward with an upstream gradient supported on a row sample S
     S = sample_rows(w, 2000, 2)
@@ -97,7 +98,7 @@ def test_full_layer_sampled_rows(full):
     q = np.unique(np.concatenate([S[:500], rng.choice(into_S, min(1500, len(into_S)), replace=False),
                                   rng.choice(int(g["type_offsets"][-1]), 500, replace=False)]))
     dq, gref = oracle.layer_backward_rows(g["src"], g["dst"], g["rel"], g["type_offsets"], g["rels"], p, w.X, S,
-                                          w.dH_top[S], q)
+                                          w.dH_top[S], q, store="bf16")
     tol = TOL[sp.dtype]
     assert relerr(host(dH_in[torch.from_numpy(q).cuda()]), dq) <= tol
     for k, v in gref.items():

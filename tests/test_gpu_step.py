@@ -43,7 +43,7 @@ def test_step_matches_oracle(variant):
     run(path, w)
     vb = {"idx": w.overlap_local, "X_b": w.X_b} if sp.view_b == "perturbed" else \
         {"H_b": w.H_b, "gid_a": w.gid_a, "gid_b": w.gid_b}
-    ref = oracle.step(w.graph, w.X, w.params, w.dH_top, vb)
+    ref = oracle.step(w.graph, w.X, w.params, w.dH_top, vb, store="bf16" if sp.dtype == "bf16" else "f64")
     tol = TOL[sp.dtype]
     assert relerr(host(path.loss), np.array(ref["loss"])) <= (1e-4 if sp.dtype == "f32" else 2e-2)
     for l in range(1, sp.layers + 1):

@@ -260,3 +260,39 @@ def test_planted_layer_mistakes_are_caught(mistake):
         p2["ln_gamma"] = np.ones_like(params["ln_gamma"])  # gain forgotten in dX_hat = dout * gamma
         dH, _ = O.layer_backward(csr, offs, rels, p2, H, dout)
         assert np.abs(dH - Ht.grad.numpy()).max() > 1e-3
+
+
+# ---------------------------------------------------------------------------------------------
+# bf16 storage mode: the oracle's rounding and its use at the two storage points
+# ---------------------------------------------------------------------------------------------
+def test_round_bf16_matches_torch():
+    rng = np.random.default_rng(21)
+    x = np.concatenate([rng.standard_normal(100_000) * 10.0 ** rng.integers(-30, 30, 100_000),
+                        [0.0, -0.0, 1.0, 1.00390625, 1.01171875, 3.0e38, -1e-38]])
+    want = torch.tensor(x, dtype=torch.float64).to(torch.float32).to(torch.bfloat16).to(torch.float64).numpy()
+    assert np.array_equal(O.round_bf16(x), want)
+
+
+def test_bf16_store_mode_matches_torch_with_bf16_casts():
+    """store='bf16' = the dense torch formulation with M_r, Z and U cast through torch.bfloat16."""
+    src, dst, rel, offs, rels, H, params = small_graph(13, d=8)
+    csr = oracle.build_csr(src, dst, rel, offs, rels)
+    out, _ = oracle.layer_forward(csr, offs, rels, params, H, store="bf16")
+    P = {k: torch.tensor(v, dtype=torch.float64) for k, v in params.items()}
+    Ht = torch.tensor(H)
+    bf = lambda t: t.to(torch.float32).to(torch.bfloat16).to(torch.float64)  # noqa: E731
+    outs = []
+    for t in range(2):
+        lo, hi = int(offs[t]), int(offs[t + 1])
+        Z = torch.zeros(hi - lo, H.shape[1], dtype=torch.float64)
+        for r, (_, tt) in enumerate(rels):
+            if tt == t:
+                A = torch.tensor(dense_mean_matrix(src, dst, rel, offs, rels, r))
+                Z = Z + bf(A @ Ht) @ P["W_rel"][r]
+        U = bf(bf(Z) @ P["W_agg"][t] + P["b_agg"][t])
+        Y = torch.relu(U) + Ht[lo:hi]
+        outs.append(torch.nn.functional.layer_norm(Y, (H.shape[1],), P["ln_gamma"][t], P["ln_beta"][t], 1e-5))
+    assert np.allclose(out, torch.cat(outs).numpy(), rtol=0, atol=1e-12)
+    # and the two modes differ (the rounding is really applied)
+    out64, _ = oracle.layer_forward(csr, offs, rels, params, H)
+    assert np.abs(out - out64).max() > 1e-6
