@@ -206,8 +206,11 @@ def make_features(sp: GraphSpec, sub: int = 0) -> np.ndarray:
     return _store(rng.standard_normal((sp.num_nodes, sp.d), dtype=np.float32), sp.dtype)
 
 
-def make_layer_params(sp: GraphSpec, layer: int, random_affine: bool = False) -> dict:
-    """Per-layer weights: W_rel[r] (d_in x d_out), W_agg[t], b_agg[t], ln_gamma[t], ln_beta[t]."""
+def make_layer_params(sp: GraphSpec, layer: int, random_affine: bool = False, bias_margin: float | None = None) -> dict:
+    """Per-layer weights: W_rel[r] (d_in x d_out), W_agg[t], b_agg[t], ln_gamma[t], ln_beta[t].
+
+    bias_margin: biases of +-margin per column (seeded signs), which keep pre-activations away from
+    the activation's kink so that the ReLU decisions of two implementations cannot differ."""
     rng = _rng(sp.seed + 100 + layer)
     d = sp.d
     a = math.sqrt(6.0 / (2 * d))
@@ -221,6 +224,8 @@ def make_layer_params(sp: GraphSpec, layer: int, random_affine: bool = False) ->
         b = np.zeros((2, d), np.float32)
         gamma = np.ones((2, d), np.float32)
         beta = np.zeros((2, d), np.float32)
+    if bias_margin is not None:
+        b = (bias_margin * rng.choice([-1.0, 1.0], size=(2, d))).astype(np.float32)
     return {k: _store(v, sp.dtype) for k, v in
             dict(W_rel=W_rel, W_agg=W_agg, b_agg=b, ln_gamma=gamma, ln_beta=beta).items()}
 
@@ -279,10 +284,11 @@ class Workload:
     dH_top: np.ndarray  # upstream gradient of the last layer's output (stands in for the prediction head)
 
 
-def make_workload(sp: GraphSpec, sub: int = 0, random_affine: bool = False, with_ids: bool = True) -> Workload:
+def make_workload(sp: GraphSpec, sub: int = 0, random_affine: bool = False, with_ids: bool = True,
+                  bias_margin: float | None = None) -> Workload:
     g = make_graph(sp, sub)
     X = make_features(sp, sub)
-    params = [make_layer_params(sp, l, random_affine) for l in range(sp.layers)]
+    params = [make_layer_params(sp, l, random_affine, bias_margin) for l in range(sp.layers)]
     ov = overlap_nodes(sp, g, sub)
     rng3 = _rng(sp.seed + 3, sub)
     X_b = H_b = None

@@ -47,7 +47,7 @@ typedef enum {
   HG_ERR_WORKSPACE = 3,    /* caller buffer smaller than the matching *_size query */
   HG_ERR_CUDA = 4,         /* a CUDA runtime call or launch failed */
   HG_ERR_DEVICE_CHECK = 5, /* a device-side input check failed (reported by hg_graph_check) */
-  HG_ERR_TIMEOUT = 6       /* reserved for bounded waits; no kernel of this library waits */
+  HG_ERR_TIMEOUT = 6       /* a bounded wait inside a kernel gave up (see hg_device_status) */
 } hg_status;
 
 typedef enum { HG_F32 = 0, HG_BF16 = 1 } hg_dtype;
@@ -68,6 +68,10 @@ const char* hg_status_string(hg_status status);
 const char* hg_last_error(void);
 /* Version of this ABI (bumped on any incompatible change). */
 int32_t hg_abi_version(void);
+/* SYNCHRONISES the device, then reports and clears the library's device status word.  Every wait
+ * inside a kernel of this library is bounded; a wait that gave up sets a flag here (its kernel's
+ * results are then invalid) and this call returns HG_ERR_TIMEOUT.  flags may be NULL. */
+hg_status hg_device_status(int32_t* flags);
 
 /* ------------------------------------------------------------------------------------------- */
 /* Graph layout (Section 2.2, Section 3.1 / Eq. 5: the adjacency of one overlapping subgraph)   */

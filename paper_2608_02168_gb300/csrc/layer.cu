@@ -106,9 +106,10 @@ static void carve_layer(const hg_graph* g, int d, hg_dtype dt, void* saved, void
   int64_t max_rows = 1;
   for (int t = 0; t < m.num_types; ++t) max_rows = std::max(max_rows, m.type_off[t + 1] - m.type_off[t]);
   L->cpart = k.take<float>((size_t)ceil_div(max_rows, 64) * 3 * d);
-  L->wpart = k.take<float>((size_t)wgrad_splits(max_rows) * d * d);
+  const int wsplits = std::max(wgrad_splits(max_rows), wgrad_tc_splits(max_rows, d));
+  L->wpart = k.take<float>((size_t)wsplits * d * d);
   L->rtmp = k.take<float>(std::max(reduce_tmp_floats((int)ceil_div(max_rows, 64), d),
-                                   reduce_tmp_floats(wgrad_splits(max_rows), (int64_t)d * d)));
+                                   reduce_tmp_floats(wsplits, (int64_t)d * d)));
   L->WrelT = k.take<char>((size_t)m.num_rels * d * d * b);
   L->WaggT = k.take<char>((size_t)m.num_types * d * d * b);
   if (saved_bytes) *saved_bytes = s.used;
@@ -158,6 +159,23 @@ extern "C" const char* hg_status_string(hg_status s) {
 
 extern "C" const char* hg_last_error(void) { return g_err; }
 extern "C" int32_t hg_abi_version(void) { return 1; }
+
+extern "C" hg_status hg_device_status(int32_t* flags) {
+  clear_error();
+  int* p = device_status_ptr();
+  HG_REQUIRE(p != nullptr, "device status word unavailable");
+  int v = 0;
+  HG_CUDA(cudaDeviceSynchronize());
+  HG_CUDA(cudaMemcpy(&v, p, sizeof(int), cudaMemcpyDeviceToHost));
+  if (flags) *flags = v;
+  if (v != 0) {
+    const int zero = 0;
+    HG_CUDA(cudaMemcpy(p, &zero, sizeof(int), cudaMemcpyHostToDevice));
+    set_error("a bounded wait in a tensor-core kernel gave up (flags %d); its results are invalid", v);
+    return HG_ERR_TIMEOUT;
+  }
+  return HG_OK;
+}
 
 extern "C" hg_status hg_timing_enable(int32_t on) {
   std::lock_guard<std::mutex> lk(g_tmu);
@@ -223,6 +241,37 @@ extern "C" hg_status hg_layer_fwd(const hg_graph* graph, const hg_layer_params* 
   LayerLayout L;
   carve_layer(graph, d, p->dtype, saved, scratch, &L, nullptr, nullptr);
   HG_TRY(aggregate_forward(graph, p->dtype, d, H_in, L.M, L.agg_part, s));
+  if (p->dtype == HG_BF16) {
+    // tensor-core path: B operands are the transposed weights (K-major)
+    HG_TRY(transpose_weights(p->dtype, d, p->W_rel, L.WrelT, m.num_rels, s));
+    HG_TRY(transpose_weights(p->dtype, d, p->W_agg, L.WaggT, m.num_types, s));
+    for (int t = 0; t < m.num_types; ++t) {
+      TcFwdArgs a{};
+      for (int r = 0; r < m.num_rels; ++r) {
+        if (m.rel_dst[r] != t) continue;
+        a.rel[a.nrel] = r;
+        a.mrow0[a.nrel] = m.row_base[r];
+        ++a.nrel;
+      }
+      a.type = t;
+      a.b = (const __nv_bfloat16*)p->b_agg + (size_t)t * d;
+      a.gamma = p->layernorm ? (const __nv_bfloat16*)p->ln_gamma + (size_t)t * d : nullptr;
+      a.beta = p->layernorm ? (const __nv_bfloat16*)p->ln_beta + (size_t)t * d : nullptr;
+      a.H_in = (const __nv_bfloat16*)H_in;
+      a.H_out = (__nv_bfloat16*)H_out;
+      a.Z = (__nv_bfloat16*)L.Z;
+      a.U = (__nv_bfloat16*)L.U;
+      a.stats = L.stats;
+      a.off = m.type_off[t];
+      a.n = m.type_off[t + 1] - m.type_off[t];
+      a.act = p->act;
+      a.ln = p->layernorm;
+      a.eps = p->ln_eps;
+      a.status = device_status_ptr();
+      if (a.n > 0) HG_TRY(tc_proj_forward(d, a, L.M, graph->csr_rows, L.WrelT, m.num_rels, L.WaggT, m.num_types, s));
+    }
+    return HG_OK;
+  }
   for (int t = 0; t < m.num_types; ++t) {
     FwdArgs a{};
     a.M = L.M;
@@ -270,8 +319,11 @@ extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* 
   const size_t b = elem_size(p->dtype);
   LayerLayout L;
   carve_layer(graph, d, p->dtype, const_cast<void*>(saved), scratch, &L, nullptr, nullptr);
-  HG_TRY(transpose_weights(p->dtype, d, p->W_rel, L.WrelT, m.num_rels, s));
-  HG_TRY(transpose_weights(p->dtype, d, p->W_agg, L.WaggT, m.num_types, s));
+  const bool tc = p->dtype == HG_BF16;
+  if (!tc) {
+    HG_TRY(transpose_weights(p->dtype, d, p->W_rel, L.WrelT, m.num_rels, s));
+    HG_TRY(transpose_weights(p->dtype, d, p->W_agg, L.WaggT, m.num_types, s));
+  }
   for (int t = 0; t < m.num_types; ++t) {
     const int64_t n = m.type_off[t + 1] - m.type_off[t];
     float* db = grads->db_agg + (size_t)t * d;
@@ -281,46 +333,83 @@ extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* 
         HG_CUDA(cudaMemsetAsync(grads->dln_gamma + (size_t)t * d, 0, d * sizeof(float), s));
         HG_CUDA(cudaMemsetAsync(grads->dln_beta + (size_t)t * d, 0, d * sizeof(float), s));
       }
+      HG_CUDA(cudaMemsetAsync(grads->dW_agg + (size_t)t * d * d, 0, (size_t)d * d * sizeof(float), s));
       continue;
     }
-    BwdArgs a{};
-    a.dH_out = dH_out;
-    a.H_in = H_in;
-    a.U = L.U;
-    a.stats = L.stats;
-    a.gamma = p->layernorm ? (const char*)p->ln_gamma + (size_t)t * d * b : nullptr;
-    a.W_aggT = (const char*)L.WaggT + (size_t)t * d * d * b;
-    for (int r = 0; r < m.num_rels; ++r) {
-      if (m.rel_dst[r] != t) continue;
-      a.mrow0[a.nrel] = m.row_base[r];
-      a.W_relT[a.nrel] = (const char*)L.WrelT + (size_t)r * d * d * b;
-      ++a.nrel;
+    int blocks;
+    if (tc) {
+      TcBwdArgs a{};
+      for (int r = 0; r < m.num_rels; ++r) {
+        if (m.rel_dst[r] != t) continue;
+        a.rel[a.nrel] = r;
+        a.mrow0[a.nrel] = m.row_base[r];
+        ++a.nrel;
+      }
+      a.type = t;
+      a.dH_out = (const __nv_bfloat16*)dH_out;
+      a.H_in = (const __nv_bfloat16*)H_in;
+      a.U = (const __nv_bfloat16*)L.U;
+      a.stats = L.stats;
+      a.gamma = p->layernorm ? (const __nv_bfloat16*)p->ln_gamma + (size_t)t * d : nullptr;
+      a.csr_ptr = graph->csr_ptr;
+      a.dY = (__nv_bfloat16*)L.dY;
+      a.dU = (__nv_bfloat16*)L.dU;
+      a.dZ = (__nv_bfloat16*)L.dZ;
+      a.dMs = (__nv_bfloat16*)L.dMs;
+      a.part = L.cpart;
+      a.off = m.type_off[t];
+      a.n = n;
+      a.act = p->act;
+      a.ln = p->layernorm;
+      a.status = device_status_ptr();
+      HG_TRY(tc_proj_backward(d, a, p->W_agg, m.num_types, p->W_rel, m.num_rels, s));
+      blocks = (int)ceil_div(n, 128);
+    } else {
+      BwdArgs a{};
+      a.dH_out = dH_out;
+      a.H_in = H_in;
+      a.U = L.U;
+      a.stats = L.stats;
+      a.gamma = p->layernorm ? (const char*)p->ln_gamma + (size_t)t * d * b : nullptr;
+      a.W_aggT = (const char*)L.WaggT + (size_t)t * d * d * b;
+      for (int r = 0; r < m.num_rels; ++r) {
+        if (m.rel_dst[r] != t) continue;
+        a.mrow0[a.nrel] = m.row_base[r];
+        a.W_relT[a.nrel] = (const char*)L.WrelT + (size_t)r * d * d * b;
+        ++a.nrel;
+      }
+      a.csr_ptr = graph->csr_ptr;
+      a.dY = L.dY;
+      a.dU = L.dU;
+      a.dZ = L.dZ;
+      a.dMs = L.dMs;
+      a.part = L.cpart;
+      a.off = m.type_off[t];
+      a.n = n;
+      a.act = p->act;
+      a.ln = p->layernorm;
+      HG_TRY(proj_backward(p->dtype, d, a, s));
+      blocks = (int)ceil_div(n, 64);
     }
-    a.csr_ptr = graph->csr_ptr;
-    a.dY = L.dY;
-    a.dU = L.dU;
-    a.dZ = L.dZ;
-    a.dMs = L.dMs;
-    a.part = L.cpart;
-    a.off = m.type_off[t];
-    a.n = n;
-    a.act = p->act;
-    a.ln = p->layernorm;
-    HG_TRY(proj_backward(p->dtype, d, a, s));
-    const int blocks = (int)ceil_div(n, 64);
     HG_TRY(reduce_partials(L.cpart, 3LL * d, blocks, d, db, L.rtmp, s));
     if (p->layernorm) {
       HG_TRY(reduce_partials(L.cpart + d, 3LL * d, blocks, d, grads->dln_gamma + (size_t)t * d, L.rtmp, s));
       HG_TRY(reduce_partials(L.cpart + 2 * d, 3LL * d, blocks, d, grads->dln_beta + (size_t)t * d, L.rtmp, s));
     }
-    HG_TRY(weight_grad(p->dtype, d, L.Z, a.off, L.dU, a.off, n, L.wpart, grads->dW_agg + (size_t)t * d * d, L.rtmp,
-                       s));
+    const int64_t off = m.type_off[t];
+    if (tc)
+      HG_TRY(tc_weight_grad(d, L.Z, off, L.dU, off, n, L.wpart, grads->dW_agg + (size_t)t * d * d, L.rtmp, s));
+    else
+      HG_TRY(weight_grad(p->dtype, d, L.Z, off, L.dU, off, n, L.wpart, grads->dW_agg + (size_t)t * d * d, L.rtmp, s));
   }
   for (int r = 0; r < m.num_rels; ++r) {
     const int t = m.rel_dst[r];
     const int64_t n = m.type_off[t + 1] - m.type_off[t];
-    HG_TRY(weight_grad(p->dtype, d, L.M, m.row_base[r], L.dZ, m.type_off[t], n, L.wpart,
-                       grads->dW_rel + (size_t)r * d * d, L.rtmp, s));
+    float* out = grads->dW_rel + (size_t)r * d * d;
+    if (tc)
+      HG_TRY(tc_weight_grad(d, L.M, m.row_base[r], L.dZ, m.type_off[t], n, L.wpart, out, L.rtmp, s));
+    else
+      HG_TRY(weight_grad(p->dtype, d, L.M, m.row_base[r], L.dZ, m.type_off[t], n, L.wpart, out, L.rtmp, s));
   }
   if (dH_in) HG_TRY(aggregate_backward(graph, p->dtype, d, L.dMs, L.dY, dH_in, L.agg_part, s));
   return HG_OK;

@@ -2,6 +2,8 @@
 // units; not part of the public ABI).
 #pragma once
 
+#include <cuda_bf16.h>
+
 #include "hg_internal.cuh"
 
 namespace hg {
@@ -44,6 +46,56 @@ struct BwdArgs {
   int64_t off, n;
   int act, ln;
 };
+
+// tensor-core kernels (bf16 storage)
+struct TcFwdArgs {
+  int nrel;
+  int rel[kMaxRels];          // relation ids into this type (row block of W_rel^T)
+  int64_t mrow0[kMaxRels];    // first CSR row of each
+  int type;
+  const __nv_bfloat16* b;
+  const __nv_bfloat16* gamma;
+  const __nv_bfloat16* beta;
+  const __nv_bfloat16* H_in;
+  __nv_bfloat16* H_out;
+  __nv_bfloat16* Z;
+  __nv_bfloat16* U;
+  float2* stats;
+  int64_t off, n;
+  int act, ln;
+  float eps;
+  int* status;  // library status word (timeouts of bounded waits)
+};
+
+struct TcBwdArgs {
+  int nrel;
+  int rel[kMaxRels];
+  int64_t mrow0[kMaxRels];
+  int type;
+  const __nv_bfloat16* dH_out;
+  const __nv_bfloat16* H_in;
+  const __nv_bfloat16* U;
+  const float2* stats;
+  const __nv_bfloat16* gamma;
+  const int32_t* csr_ptr;
+  __nv_bfloat16* dY;
+  __nv_bfloat16* dU;
+  __nv_bfloat16* dZ;
+  __nv_bfloat16* dMs;
+  float* part;  // [gridDim.x][3][D]
+  int64_t off, n;
+  int act, ln;
+  int* status;
+};
+
+hg_status tc_proj_forward(int d, const TcFwdArgs& a, const void* M, int64_t m_rows, const void* WrelT, int num_rels,
+                          const void* WaggT, int num_types, cudaStream_t s);
+hg_status tc_proj_backward(int d, const TcBwdArgs& a, const void* Wagg, int num_types, const void* Wrel, int num_rels,
+                           cudaStream_t s);
+hg_status tc_weight_grad(int d, const void* X, int64_t x0, const void* Y, int64_t y0, int64_t n, float* part,
+                         float* out, float* tmp, cudaStream_t s);
+int wgrad_tc_splits(int64_t n, int d);
+int* device_status_ptr();  // device address of the library status word
 
 hg_status aggregate_forward(const hg_graph* g, hg_dtype dt, int d, const void* H, void* M, float* partials,
                             cudaStream_t s);

@@ -45,10 +45,14 @@ hg_status make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint
   return HG_OK;
 }
 
+// Resolved once per process on the current device (the library drives one GPU per process).
 int* device_status_ptr() {
-  void* p = nullptr;
-  if (cudaGetSymbolAddress(&p, g_device_status) != cudaSuccess) return nullptr;
-  return static_cast<int*>(p);
+  static int* addr = nullptr;
+  if (!addr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_device_status) == cudaSuccess) addr = static_cast<int*>(p);
+  }
+  return addr;
 }
 
 }  // namespace hg

@@ -47,6 +47,7 @@ EXPORTS = {
     "hg_status_string": (c_char_p, [c_int32]),
     "hg_last_error": (c_char_p, []),
     "hg_abi_version": (c_int32, []),
+    "hg_device_status": (c_int32, [POINTER(c_int32)]),
     "hg_graph_workspace_size": (c_int32, [c_int64, POINTER(c_int64), c_int32, POINTER(hg_rel_desc), c_int32,
                                           POINTER(c_size_t)]),
     "hg_build_csr": (c_int32, [c_void_p, c_void_p, c_void_p, c_int64, POINTER(c_int64), c_int32,
@@ -282,6 +283,15 @@ def hg_overlap_align_bwd(H_a, idx_a, H_b, idx_b, n_max: int, n_dev, lambda_n: fl
                                       int(H_a.shape[-1]), _dtype_of(H_a), float(lambda_n), float(var_eps),
                                       float(dloss), _ptr(saved), _ptr(dH_a), _ptr(dH_b), _ptr(scratch),
                                       _stream(stream)), "hg_overlap_align_bwd")
+
+
+def hg_device_status() -> int:
+    """Synchronises; returns the device status flags (0 = no bounded wait gave up) and clears them."""
+    f = c_int32(0)
+    st = lib().hg_device_status(byref(f))
+    if st not in (0, 6):
+        _check(st, "hg_device_status")
+    return f.value
 
 
 # ------------------------------------------------------------------------------------------------

@@ -18,7 +18,8 @@ def full():
     need_gpu()
     hg = lib()
     sp = hgsynth.spec("sub-1m")
-    w = hgsynth.make_workload(sp, random_affine=True, with_ids=True)
+    # biases of +-3 keep the ReLU decisions unambiguous (see test_gpu_layer)
+    w = hgsynth.make_workload(sp, random_affine=True, with_ids=True, bias_margin=3.0)
     g = w.graph
     G = hg.hg_build_csr(dev(g["src"]), dev(g["dst"]), dev(g["rel"]), g["type_offsets"], g["rels"])
     assert hg.hg_graph_check(G) == 0
