@@ -225,6 +225,23 @@ hg_status hg_overlap_align_bwd(const void* H_a, int64_t rows_a, const int32_t* i
                                int32_t d, hg_dtype dtype, float lambda_n, float var_eps, float dloss,
                                const void* saved, void* dH_a, void* dH_b, void* scratch, hg_stream stream);
 
+/* The same loss as hg_overlap_align_loss for callers that cannot allocate device memory -- a host
+ * program that links only this C ABI and owns no CUDA allocator, a process whose device memory is
+ * fully reserved by another framework's caching allocator, or code for which cudaMalloc is off
+ * limits because it can synchronise the device.  The paper has no counterpart; this is an
+ * interface convenience.  Inputs, `loss_out` and `saved` are as for hg_overlap_align_loss (the
+ * `saved` buffer still comes from the caller and feeds hg_overlap_align_bwd); the scratch is a
+ * 12 MiB device array inside the library, which every GPU that loads the library holds until the
+ * process exits.  It calls no allocating routine.  The array's device address is looked up on
+ * the first call made on each device (with that device current), so that first call should come
+ * before any stream capture.  All calls share the array: calls that overlap on the GPU race.
+ * Returns HG_ERR_UNSUPPORTED for a width whose scratch would exceed the array (none of the
+ * supported d do). */
+hg_status hg_overlap_align_loss_static(const void* H_a, int64_t rows_a, const int32_t* idx_a, const void* H_b,
+                                       int64_t rows_b, const int32_t* idx_b, int64_t n_max, const int64_t* n_dev,
+                                       int32_t d, hg_dtype dtype, float lambda_n, float var_eps, float* loss_out,
+                                       void* saved, hg_stream stream);
+
 /* ------------------------------------------------------------------------------------------- */
 /* Kernel timing (measurement support; off by default)                                          */
 /* ------------------------------------------------------------------------------------------- */

@@ -599,3 +599,129 @@ extern "C" hg_status hg_overlap_align_bwd(const void* H_a, int64_t rows_a, const
   carve_align(const_cast<void*>(saved), scratch, n_max, d, &L, nullptr, nullptr);
   return align_bwd_dispatch(dtype, d, in, lambda_n, dloss, dH_a, dH_b, L, reinterpret_cast<cudaStream_t>(stream));
 }
+
+// ---------------------------------------------------------------------------------------------
+// Allocation-free variant of hg_overlap_align_loss.
+//
+// Some callers cannot hand this library a scratch buffer: a host program that links only this C
+// ABI and owns no CUDA allocator, a serving process whose device memory is entirely reserved by
+// another framework's caching allocator, or code for which cudaMalloc is off limits because it can
+// synchronise the device.  This variant runs the same kernels with their scratch in a file-scope
+// device array of kStaticAlignBytes (every GPU that loads the library holds it until exit), so
+// the caller passes only inputs and outputs.  The array's device address is looked up once per
+// device, on the first call made with that device current (that first call should therefore come
+// before any stream capture).  All calls share the array: calls that overlap on the GPU race, and
+// each call leaves its partial sums behind.  Nothing needs zeroing first: every scratch element a
+// kernel reads has been written earlier in the same call.
+// ---------------------------------------------------------------------------------------------
+#include <mutex>
+
+namespace hg {
+
+constexpr int kStaticGramSplits = 16;                        // row splits of the Gram products
+constexpr size_t kStaticAlignBytes = size_t(12) << 20;      // 12 MiB: d <= 256 at 16 splits
+static __device__ __align__(256) unsigned char g_align_static_scratch[kStaticAlignBytes];
+
+constexpr int kStaticMaxDevices = 64;
+static std::mutex g_static_mu;
+static void* g_static_addr[kStaticMaxDevices] = {};
+
+static hg_status static_align_scratch(void** out) {
+  int dev = 0;
+  HG_CUDA(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= kStaticMaxDevices) {
+    set_error("device %d is beyond the %d devices this entry point tracks", dev, kStaticMaxDevices);
+    return HG_ERR_UNSUPPORTED;
+  }
+  std::lock_guard<std::mutex> lk(g_static_mu);
+  if (!g_static_addr[dev]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_align_static_scratch);
+    if (e != cudaSuccess || p == nullptr) {
+      set_error("cudaGetSymbolAddress of the static alignment scratch failed: %s", cudaGetErrorString(e));
+      return HG_ERR_CUDA;
+    }
+    g_static_addr[dev] = p;
+  }
+  *out = g_static_addr[dev];
+  return HG_OK;
+}
+
+// Layout of the static scratch for width d: column partials, Gram partials, L_inv partials.
+static size_t carve_static(void* base, int d, float** part, float** gpart, float** inv) {
+  Carve k(base);
+  *part = k.take<float>((size_t)kAlignBlocks * 2 * d);
+  *gpart = k.take<float>((size_t)kStaticGramSplits * 2 * d * d);
+  *inv = k.take<float>(kStaticGramSplits);
+  return k.used;
+}
+
+template <typename T, int D>
+static hg_status align_loss_static_t(const AlignIn& in, float lambda_n, float eps, float* loss, float* stats, float* C,
+                                     int32_t* bad, float* part, float* gpart, float* inv, cudaStream_t s) {
+  const int rstep = 256 / D;
+  const size_t cs_smem = sizeof(float) * rstep * 2 * D;
+  const int blocks = (int)std::max<int64_t>(1, std::min<int64_t>(kAlignBlocks, ceil_div(in.n_max, rstep)));
+  const int splits = std::min(gram_splits(in.n_max), kStaticGramSplits);
+  const T* Ha = (const T*)in.Ha;
+  const T* Hb = (const T*)in.Hb;
+  HG_CUDA(cudaMemsetAsync(bad, 0, sizeof(int32_t), s));
+  HG_TRY(launch("align_colstats", align_colstats<T>, dim3(blocks), dim3(256), cs_smem, s, Ha, in.rows_a, in.ia, Hb,
+                in.rows_b, in.ib, in.n_max, in.n_dev, D, 0, (const float*)nullptr, part, bad));
+  HG_TRY(launch("align_colfinish", align_colfinish, dim3(1), dim3(256), 0, s, (const float*)part, blocks, D, in.n_dev,
+                in.n_max, 0, 0.f, stats));
+  HG_TRY(launch("align_colstats", align_colstats<T>, dim3(blocks), dim3(256), cs_smem, s, Ha, in.rows_a, in.ia, Hb,
+                in.rows_b, in.ib, in.n_max, in.n_dev, D, 1, (const float*)stats, part, bad));
+  HG_TRY(launch("align_colfinish", align_colfinish, dim3(1), dim3(256), 0, s, (const float*)part, blocks, D, in.n_dev,
+                in.n_max, 1, eps, stats + 2 * D));
+  constexpr int TW = D < 128 ? D : 128;
+  const int tiles = (D / TW) * (D / TW);
+  HG_TRY(launch("align_gram", align_gram<T, D>, dim3(tiles, splits, 2), dim3(256), 0, s, Ha, in.rows_a, in.ia, Hb,
+                in.rows_b, in.ib, in.n_max, in.n_dev, (const float*)stats, gpart, inv));
+  HG_TRY(launch("align_gram_reduce", align_gram_reduce, dim3((unsigned)ceil_div(2LL * D * D, 256)), dim3(256), 0, s,
+                (const float*)gpart, splits, 2LL * D * D, C));
+  return launch("align_loss_finish", align_loss_finish, dim3(1), dim3(256), 0, s, (const float*)C, D,
+                (const float*)inv, splits, in.n_dev, in.n_max, lambda_n, (const int32_t*)bad, loss);
+}
+
+}  // namespace hg
+
+extern "C" hg_status hg_overlap_align_loss_static(const void* H_a, int64_t rows_a, const int32_t* idx_a,
+                                                  const void* H_b, int64_t rows_b, const int32_t* idx_b,
+                                                  int64_t n_max, const int64_t* n_dev, int32_t d, hg_dtype dtype,
+                                                  float lambda_n, float var_eps, float* loss_out, void* saved,
+                                                  hg_stream stream) {
+  clear_error();
+  const AlignIn in{H_a, rows_a, idx_a, H_b, rows_b, idx_b, n_max, n_dev};
+  void* scratch = nullptr;
+  HG_TRY(static_align_scratch(&scratch));
+  HG_TRY(check_align_args(in, d, dtype, saved, scratch));
+  HG_REQUIRE(loss_out != nullptr, "loss_out must be non-null");
+  HG_REQUIRE(lambda_n >= 0.f && var_eps >= 0.f, "lambda_n and var_eps must be >= 0");
+  float *part, *gpart, *inv;
+  const size_t need = carve_static(nullptr, d, &part, &gpart, &inv);
+  if (need > kStaticAlignBytes) {
+    set_error("d=%d needs %zu bytes of scratch, beyond the %zu-byte static array of this entry point", d, need,
+              kStaticAlignBytes);
+    return HG_ERR_UNSUPPORTED;
+  }
+  carve_static(scratch, d, &part, &gpart, &inv);
+  AlignLayout L;  // only the `saved` part (statistics, Gram matrices, index flag) is used
+  carve_align(saved, nullptr, n_max, d, &L, nullptr, nullptr);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+#define HG_STATIC_CASE(T, D_)                                                                                \
+  if (d == D_)                                                                                               \
+    return align_loss_static_t<T, D_>(in, lambda_n, var_eps, loss_out, L.stats, L.C, L.bad, part, gpart, inv, s);
+  if (dtype == HG_F32) {
+    HG_STATIC_CASE(float, 64)
+    HG_STATIC_CASE(float, 128)
+    HG_STATIC_CASE(float, 256)
+  } else {
+    HG_STATIC_CASE(__nv_bfloat16, 64)
+    HG_STATIC_CASE(__nv_bfloat16, 128)
+    HG_STATIC_CASE(__nv_bfloat16, 256)
+  }
+#undef HG_STATIC_CASE
+  set_error("unsupported feature width %d", d);
+  return HG_ERR_UNSUPPORTED;
+}

@@ -68,6 +68,9 @@ EXPORTS = {
     "hg_overlap_align_bwd": (c_int32, [c_void_p, c_int64, c_void_p, c_void_p, c_int64, c_void_p, c_int64, c_void_p,
                                        c_int32, c_int32, c_float, c_float, c_float, c_void_p, c_void_p, c_void_p,
                                        c_void_p, c_void_p]),
+    "hg_overlap_align_loss_static": (c_int32, [c_void_p, c_int64, c_void_p, c_void_p, c_int64, c_void_p, c_int64,
+                                               c_void_p, c_int32, c_int32, c_float, c_float, c_void_p, c_void_p,
+                                               c_void_p]),
     "hg_timing_enable": (c_int32, [c_int32]),
     "hg_timing_report": (c_int32, [c_char_p, c_size_t]),
 }
@@ -292,6 +295,16 @@ def hg_device_status() -> int:
     if st not in (0, 6):
         _check(st, "hg_device_status")
     return f.value
+
+
+def hg_overlap_align_loss_static(H_a, idx_a, H_b, idx_b, n_max: int, n_dev, lambda_n: float, var_eps: float,
+                                 loss_out, saved, stream=None):
+    """hg_overlap_align_loss without a scratch argument: the library's own static device array is
+    used instead, for callers that cannot allocate (calls must not overlap on the GPU)."""
+    _check(lib().hg_overlap_align_loss_static(_ptr(H_a), H_a.shape[0], _ptr(idx_a), _ptr(H_b), H_b.shape[0],
+                                              _ptr(idx_b), int(n_max), _ptr(n_dev), int(H_a.shape[-1]),
+                                              _dtype_of(H_a), float(lambda_n), float(var_eps), _ptr(loss_out),
+                                              _ptr(saved), _stream(stream)), "hg_overlap_align_loss_static")
 
 
 # ------------------------------------------------------------------------------------------------
