@@ -7,10 +7,11 @@
 //           backward kernel, and dY[i] is the residual-path gradient of Eq. 11.
 //
 // Mapping: one group of G lanes per row, each lane owning 16-byte slices of the feature row
-// (G = d * sizeof(T) / 16, at most 32), gathers with 128-bit loads and four neighbour rows in
-// flight, fp32 accumulation.  Rows above kHubDegree edges are split into kChunkEdges-edge chunks:
-// a whole CTA reduces one chunk (its groups interleave over the chunk's edges, then combine in
-// group order), writes an fp32 partial, and the row kernel adds the partials in chunk order.
+// (G = d * sizeof(T) / 16, at most 32), gathers with 128-bit loads and eight neighbour rows in
+// flight, fp32 accumulation; the row kernels are persistent (one wave of blocks striding over
+// rows).  Rows above kHubDegree edges are split into kChunkEdges-edge chunks: a whole CTA reduces
+// one chunk (its groups interleave over the chunk's edges, then combine in group order) into an
+// fp32 partial, runs of 64 partials are summed in order, and the row adds the run sums in order.
 // Every sum has a fixed order, so results are bitwise reproducible run to run.
 #include <algorithm>
 
@@ -29,24 +30,27 @@ struct AggShape {
   static constexpr int kGroups = kThreads / G;
 };
 
-// acc += sum of rows src[col[e] + delta] for e = beg, beg + stride, ... < end
+// acc += sum of rows src[col[e] + delta] for e = beg, beg + stride, ... < end, added in edge
+// order; eight neighbour rows are loaded before they are added.
 template <typename T, int D>
 __device__ __forceinline__ void gather_sum(const int32_t* __restrict__ col, int64_t beg, int64_t end,
                                            int stride, int64_t delta, const T* __restrict__ src,
                                            int lane, float* acc) {
   using S = AggShape<T, D>;
+  constexpr int U = 8;
+  const T* base = src + delta * D + lane * S::kVec;
   int64_t e = beg;
-  for (; e + 3 * (int64_t)stride < end; e += 4 * (int64_t)stride) {
-    int64_t c[4];
+  for (; e + (U - 1) * (int64_t)stride < end; e += U * (int64_t)stride) {
+    int c[U];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) c[u] = (int64_t)__ldg(col + e + u * stride) + delta;
-    uint4 x[4][S::V];
+    for (int u = 0; u < U; ++u) c[u] = __ldg(col + e + u * stride);
+    uint4 x[U][S::V];
 #pragma unroll
-    for (int u = 0; u < 4; ++u)
+    for (int u = 0; u < U; ++u)
 #pragma unroll
-      for (int v = 0; v < S::V; ++v) x[u][v] = ldg16(src + c[u] * D + (lane + v * S::G) * S::kVec);
+      for (int v = 0; v < S::V; ++v) x[u][v] = ldg16(base + (int64_t)c[u] * D + v * S::G * S::kVec);
 #pragma unroll
-    for (int u = 0; u < 4; ++u)
+    for (int u = 0; u < U; ++u)
 #pragma unroll
       for (int v = 0; v < S::V; ++v) {
         float f[S::kVec];
@@ -56,22 +60,52 @@ __device__ __forceinline__ void gather_sum(const int32_t* __restrict__ col, int6
       }
   }
   for (; e < end; e += stride) {
-    const int64_t c = (int64_t)__ldg(col + e) + delta;
+    const int c = __ldg(col + e);
 #pragma unroll
     for (int v = 0; v < S::V; ++v) {
       float f[S::kVec];
-      unpack(ldg16(src + c * D + (lane + v * S::G) * S::kVec), f, T());
+      unpack(ldg16(base + (int64_t)c * D + v * S::G * S::kVec), f, T());
 #pragma unroll
       for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] += f[q];
     }
   }
 }
 
+// Chunk partials are combined in two fixed-order levels: combine_chunk_partials sums every run of
+// kPartRun consecutive chunks of a row into the run's first slot, and a row then adds its run
+// sums in order (eight loads in flight).
+constexpr int kPartRun = 64;
+
 template <typename T, int D>
 __device__ __forceinline__ void add_partials(const float* __restrict__ partials, int c0, int c1, int lane,
                                              float* acc) {
   using S = AggShape<T, D>;
-  for (int c = c0; c < c1; ++c) {
+  constexpr int U = 8;
+  int c = c0;
+  for (; c + (U - 1) * kPartRun < c1; c += U * kPartRun) {
+    float4 x[U][S::V][S::kVec / 4];
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+#pragma unroll
+      for (int v = 0; v < S::V; ++v) {
+        const float4* p = reinterpret_cast<const float4*>(partials + (int64_t)(c + u * kPartRun) * D +
+                                                          (lane + v * S::G) * S::kVec);
+#pragma unroll
+        for (int q = 0; q < S::kVec / 4; ++q) x[u][v][q] = p[q];
+      }
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+#pragma unroll
+      for (int v = 0; v < S::V; ++v)
+#pragma unroll
+        for (int q = 0; q < S::kVec / 4; ++q) {
+          acc[v * S::kVec + 4 * q + 0] += x[u][v][q].x;
+          acc[v * S::kVec + 4 * q + 1] += x[u][v][q].y;
+          acc[v * S::kVec + 4 * q + 2] += x[u][v][q].z;
+          acc[v * S::kVec + 4 * q + 3] += x[u][v][q].w;
+        }
+  }
+  for (; c < c1; c += kPartRun) {
 #pragma unroll
     for (int v = 0; v < S::V; ++v) {
       const float4* p = reinterpret_cast<const float4*>(partials + (int64_t)c * D + (lane + v * S::G) * S::kVec);
@@ -84,6 +118,34 @@ __device__ __forceinline__ void add_partials(const float* __restrict__ partials,
         acc[v * S::kVec + 4 * q + 3] += x.w;
       }
     }
+  }
+}
+
+// Sums each run of kPartRun consecutive chunk partials of a row, in order, into the run's first
+// slot (one block of d threads per run leader; grid-stride over the chunk list).
+template <int D>
+__global__ void __launch_bounds__(D) combine_chunk_partials(const int32_t* __restrict__ chunk_row,
+                                                            const int32_t* __restrict__ chunk_ofs, int64_t rows,
+                                                            float* __restrict__ partials) {
+  const int nchunks = chunk_ofs[rows];
+  for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
+    const int row = chunk_row[c];
+    const int first = chunk_ofs[row];
+    if ((c - first) % kPartRun != 0) continue;
+    const int c1 = min(chunk_ofs[row + 1], c + kPartRun);
+    if (c1 - c < 2) continue;
+    const int k = threadIdx.x;
+    float s = 0.f;
+    int cc = c;
+    for (; cc + 8 <= c1; cc += 8) {
+      float v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) v[u] = partials[(int64_t)(cc + u) * D + k];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) s += v[u];
+    }
+    for (; cc < c1; ++cc) s += partials[(int64_t)cc * D + k];
+    partials[(int64_t)c * D + k] = s;
   }
 }
 
@@ -142,6 +204,7 @@ __global__ void __launch_bounds__(256) agg_chunks(const int32_t* __restrict__ pt
 }
 
 // Forward rows: M[row] = mean over the row's neighbours (concatenated CSR rows of all relations).
+// Persistent: each group strides over rows and fetches the next row's bounds while it gathers.
 template <typename T, int D>
 __global__ void __launch_bounds__(256) agg_fwd_rows(const int32_t* __restrict__ ptr, const int32_t* __restrict__ col,
                                                     const T* __restrict__ H, T* __restrict__ M, int64_t rows,
@@ -149,21 +212,38 @@ __global__ void __launch_bounds__(256) agg_fwd_rows(const int32_t* __restrict__ 
                                                     const float* __restrict__ partials) {
   using S = AggShape<T, D>;
   const int grp = threadIdx.x / S::G, lane = threadIdx.x % S::G;
-  const int64_t row = (int64_t)blockIdx.x * S::kGroups + grp;
-  if (row >= rows) return;
-  const int beg = ptr[row], end = ptr[row + 1], deg = end - beg;
-  float acc[S::F];
+  const int64_t step = (int64_t)gridDim.x * S::kGroups;
+  int64_t row = (int64_t)blockIdx.x * S::kGroups + grp;
+  int beg = 0, end = 0;
+  if (row < rows) {
+    beg = __ldg(ptr + row);
+    end = __ldg(ptr + row + 1);
+  }
+  while (row < rows) {
+    const int64_t nrow = row + step;
+    int nbeg = 0, nend = 0;
+    if (nrow < rows) {
+      nbeg = __ldg(ptr + nrow);
+      nend = __ldg(ptr + nrow + 1);
+    }
+    const int deg = end - beg;
+    float acc[S::F];
 #pragma unroll
-  for (int q = 0; q < S::F; ++q) acc[q] = 0.f;
-  if (deg > kHubDegree)
-    add_partials<T, D>(partials, chunk_ofs[row], chunk_ofs[row + 1], lane, acc);
-  else
-    gather_sum<T, D>(col, beg, end, 1, 0, H, lane, acc);
-  const float scale = deg > 0 ? __fdiv_rn(1.0f, (float)deg) : 0.f;
-  store_row<T, D>(M + row * D, lane, acc, scale);
+    for (int q = 0; q < S::F; ++q) acc[q] = 0.f;
+    if (deg > kHubDegree)
+      add_partials<T, D>(partials, chunk_ofs[row], chunk_ofs[row + 1], lane, acc);
+    else
+      gather_sum<T, D>(col, beg, end, 1, 0, H, lane, acc);
+    const float scale = deg > 0 ? __fdiv_rn(1.0f, (float)deg) : 0.f;
+    store_row<T, D>(M + row * D, lane, acc, scale);
+    row = nrow;
+    beg = nbeg;
+    end = nend;
+  }
 }
 
 // Backward nodes: dH[i] = dY[i] + sum over relations with source type tau(i) of the CSC row sums.
+// Persistent: each group strides over nodes.
 template <typename T, int D>
 __global__ void __launch_bounds__(256) agg_bwd_nodes(GraphMeta m, const int32_t* __restrict__ cptr,
                                                      const int32_t* __restrict__ ccol, const T* __restrict__ dMs,
@@ -172,32 +252,36 @@ __global__ void __launch_bounds__(256) agg_bwd_nodes(GraphMeta m, const int32_t*
                                                      const float* __restrict__ partials) {
   using S = AggShape<T, D>;
   const int grp = threadIdx.x / S::G, lane = threadIdx.x % S::G;
-  const int64_t node = (int64_t)blockIdx.x * S::kGroups + grp;
-  if (node >= m.type_off[m.num_types]) return;
-  const int t = node_type_of(m, node);
-  float acc[S::F];
+  const int64_t N = m.type_off[m.num_types];
+  const int64_t step = (int64_t)gridDim.x * S::kGroups;
+  for (int64_t node = (int64_t)blockIdx.x * S::kGroups + grp; node < N; node += step) {
+    const int t = node_type_of(m, node);
+    float acc[S::F];
 #pragma unroll
-  for (int v = 0; v < S::V; ++v) {
-    float f[S::kVec];
-    unpack(ldg16(dY + node * D + (lane + v * S::G) * S::kVec), f, T());
+    for (int v = 0; v < S::V; ++v) {
+      float f[S::kVec];
+      unpack(ldg16(dY + node * D + (lane + v * S::G) * S::kVec), f, T());
 #pragma unroll
-    for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] = f[q];
+      for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] = f[q];
+    }
+    for (int r = 0; r < m.num_rels; ++r) {
+      if (m.rel_src[r] != t) continue;
+      const int64_t crow = m.csc_base[r] + (node - m.type_off[t]);
+      const int beg = __ldg(cptr + crow), end = __ldg(cptr + crow + 1);
+      if (end - beg > kHubDegree)
+        add_partials<T, D>(partials, chunk_ofs[crow], chunk_ofs[crow + 1], lane, acc);
+      else
+        gather_sum<T, D>(ccol, beg, end, 1, m.row_base[r] - m.type_off[m.rel_dst[r]], dMs, lane, acc);
+    }
+    store_row<T, D>(dH + node * D, lane, acc, 1.0f);
   }
-  for (int r = 0; r < m.num_rels; ++r) {
-    if (m.rel_src[r] != t) continue;
-    const int64_t crow = m.csc_base[r] + (node - m.type_off[t]);
-    const int beg = cptr[crow], end = cptr[crow + 1];
-    if (end - beg > kHubDegree)
-      add_partials<T, D>(partials, chunk_ofs[crow], chunk_ofs[crow + 1], lane, acc);
-    else
-      gather_sum<T, D>(ccol, beg, end, 1, m.row_base[r] - m.type_off[m.rel_dst[r]], dMs, lane, acc);
-  }
-  store_row<T, D>(dH + node * D, lane, acc, 1.0f);
 }
 
 // ---------------------------------------------------------------------------------------------
 // host dispatch
 // ---------------------------------------------------------------------------------------------
+constexpr int64_t kPersistBlocks = 152 * 6;  // resident 256-thread blocks per SM at 40 registers
+
 static unsigned chunk_grid(int64_t cap) { return (unsigned)std::max<int64_t>(1, std::min<int64_t>(cap, 152 * 8)); }
 
 template <typename T, int D>
@@ -207,7 +291,11 @@ static hg_status agg_fwd_t(const hg_graph* g, const void* H, void* M, float* par
                 (const int32_t*)g->csr_ptr, (const int32_t*)g->csr_col, (const T*)H,
                 (const int32_t*)g->csr_chunk_row, (const int32_t*)g->csr_chunk_ofs, g->csr_rows, g->meta, 0,
                 partials));
-  return launch("agg_fwd_rows", agg_fwd_rows<T, D>, dim3((unsigned)ceil_div(g->csr_rows, S::kGroups)), dim3(256),
+  HG_TRY(launch("combine_chunk_partials", combine_chunk_partials<D>, dim3(chunk_grid(g->chunk_cap_csr)), dim3(D), 0, s,
+                (const int32_t*)g->csr_chunk_row, (const int32_t*)g->csr_chunk_ofs, g->csr_rows, partials));
+  return launch("agg_fwd_rows", agg_fwd_rows<T, D>,
+                dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(g->csr_rows, S::kGroups), kPersistBlocks))),
+                dim3(256),
                 0, s, (const int32_t*)g->csr_ptr, (const int32_t*)g->csr_col, (const T*)H, (T*)M, g->csr_rows,
                 (const int32_t*)g->csr_chunk_ofs, (const float*)partials);
 }
@@ -220,8 +308,12 @@ static hg_status agg_bwd_t(const hg_graph* g, const void* dMs, const void* dY, v
                 (const int32_t*)g->csc_ptr, (const int32_t*)g->csc_col, (const T*)dMs,
                 (const int32_t*)g->csc_chunk_row, (const int32_t*)g->csc_chunk_ofs, g->csc_rows, g->meta, 1,
                 partials));
+  HG_TRY(launch("combine_chunk_partials", combine_chunk_partials<D>, dim3(chunk_grid(g->chunk_cap_csc)), dim3(D), 0, s,
+                (const int32_t*)g->csc_chunk_row, (const int32_t*)g->csc_chunk_ofs, g->csc_rows, partials));
   const int64_t N = g->meta.type_off[g->meta.num_types];
-  return launch("agg_bwd_nodes", agg_bwd_nodes<T, D>, dim3((unsigned)ceil_div(N, S::kGroups)), dim3(256), 0, s,
+  return launch("agg_bwd_nodes", agg_bwd_nodes<T, D>,
+                dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(N, S::kGroups), kPersistBlocks))),
+                dim3(256), 0, s,
                 g->meta, (const int32_t*)g->csc_ptr, (const int32_t*)g->csc_col, (const T*)dMs, (const T*)dY,
                 (T*)dH, (const int32_t*)g->csc_chunk_ofs, (const float*)partials);
 }

@@ -81,18 +81,19 @@ class HotPath:
 
     def _layer_sizes(self, num_edges: int):
         """Layer buffer sizes depend on the node types, relations and edge count only; ask the
-        library with a placeholder graph of that shape (every edge in relation 0)."""
+        library with a placeholder graph of that shape (edges of relation 0 spread over its rows)."""
         dev = self.device
-        src = torch.zeros(num_edges, dtype=torch.int32, device=dev)
-        rel = torch.zeros(num_edges, dtype=torch.int32, device=dev)
-        # relation 0's endpoints: first node of its source / destination type
         s_t, d_t = self.rels[0]
-        src.fill_(self.type_offsets[s_t])
-        dst = torch.full((num_edges,), self.type_offsets[d_t], dtype=torch.int32, device=dev)
+        n_s = max(1, self.type_offsets[s_t + 1] - self.type_offsets[s_t])
+        n_d = max(1, self.type_offsets[d_t + 1] - self.type_offsets[d_t])
+        k = torch.arange(num_edges, dtype=torch.int64, device=dev)
+        src = (self.type_offsets[s_t] + k % n_s).to(torch.int32)
+        dst = (self.type_offsets[d_t] + k % n_d).to(torch.int32)
+        rel = torch.zeros(num_edges, dtype=torch.int32, device=dev)
         g = hg.hg_build_csr(src, dst, rel, self.type_offsets, self.rels, workspace=self.graph_ws)
-        s, k = hg.hg_layer_workspace_size(g, self.params[0])
+        s, k2 = hg.hg_layer_workspace_size(g, self.params[0])
         del g
-        return s, k
+        return s, k2
 
     def _grad_bufs(self):
         d, dev = self.d, self.device
