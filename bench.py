@@ -188,6 +188,10 @@ def kernel_models(st: dict, sp) -> dict:
     m["proj_fwd_simt"] = (L * fb, L * ff)
     m["proj_bwd_simt"] = (L * bb, L * bf)
     m["wgrad_partial"] = (L * 2 * row * (N + RR), L * 2 * d * d * (N + RR))
+    # tensor-core kernels: the same traffic and arithmetic, bound by HBM at these shapes
+    m["proj_fwd_tc"] = m["proj_fwd_simt"]
+    m["proj_bwd_tc"] = m["proj_bwd_simt"]
+    m["wgrad_tc"] = m["wgrad_partial"]
     m["radix_scatter"] = (2 * 3 * 4 * 4 * st["E"], 0)  # 2 layouts x 3 passes x (read+write of key+value)
     return m
 
@@ -208,7 +212,7 @@ def roofline(report: dict, models: dict, steps: int, peaks: dict, src: str) -> t
     by, fl = models.get(dom, (0, 0))
     secs = ms / 1e3
     alu_peak = 152 * 128 * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12  # fp32 FMA, TFLOP/s
-    if dom.endswith("_simt") or dom == "wgrad_partial":
+    if dom.endswith("_simt") or dom == "wgrad_partial":  # CUDA-core kernels: fp32 FMA bound
         ach = fl * steps / secs / 1e12 if secs > 0 else 0.0
         rf = dict(bound="alu", achieved=round(ach, 3), peak=round(alu_peak, 1), unit="TFLOP/s",
                   peak_source="derived: 152 SMs x 128 fp32 lanes x 2 flop x max SM clock")

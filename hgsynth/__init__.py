@@ -17,6 +17,8 @@ from .graphs import (  # noqa: F401
     bf16_round,
     make_graph,
     make_layer_params,
+    make_ring_part,
     make_workload,
+    ring_ids,
     spec,
 )

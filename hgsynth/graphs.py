@@ -302,3 +302,50 @@ def make_workload(sp: GraphSpec, sub: int = 0, random_affine: bool = False, with
     rng4 = _rng(sp.seed + 4, sub)
     dH_top = _store(rng4.standard_normal((sp.num_nodes, sp.d), dtype=np.float32), sp.dtype)
     return Workload(sp, g, X, params, ov, gid_a, gid_b, X_b, H_b, dH_top)
+
+
+# ------------------------------------------------------------------------------------------------
+# ring of overlapping subgraphs: subgraph k shares its first n_overlap nodes (split between the
+# types in proportion to their sizes) with subgraph k-1 and its last ones with subgraph k+1
+# ------------------------------------------------------------------------------------------------
+FEATURE_BLOCK = 1 << 16
+
+
+def _global_features(sp: GraphSpec, gids: np.ndarray) -> np.ndarray:
+    """Feature rows keyed by global id (blocks of 65,536 ids share one seeded draw), so a node
+    shared by two subgraphs has the same row in both."""
+    out = np.empty((gids.shape[0], sp.d), np.float32)
+    blocks = gids // FEATURE_BLOCK
+    for b in np.unique(blocks):
+        sel = np.flatnonzero(blocks == b)
+        rows = _rng(sp.seed + 1, int(b), 7).standard_normal((FEATURE_BLOCK, sp.d), dtype=np.float32)
+        out[sel] = rows[gids[sel] - b * FEATURE_BLOCK]
+    return _store(out, sp.dtype)
+
+
+def ring_ids(sp: GraphSpec, k: int) -> np.ndarray:
+    """Sorted global ids of subgraph k of the ring (users below risk events)."""
+    ov_u = round(sp.n_overlap * sp.n_user / sp.num_nodes)
+    ov_r = sp.n_overlap - ov_u
+    span_u = sp.num_subgraphs * (sp.n_user - ov_u) + ov_u
+    u = k * (sp.n_user - ov_u) + np.arange(sp.n_user, dtype=np.int64)
+    r = span_u + k * (sp.n_risk - ov_r) + np.arange(sp.n_risk, dtype=np.int64)
+    return np.concatenate([u, r])
+
+
+@dataclasses.dataclass
+class RingPart:
+    k: int
+    graph: dict
+    X: np.ndarray
+    gid: np.ndarray
+    dH_top: np.ndarray
+
+
+def make_ring_part(sp: GraphSpec, k: int) -> RingPart:
+    """Subgraph k of the ring: its own edges (seeded by k), features of its global ids."""
+    g = make_graph(sp, sub=k)
+    gid = ring_ids(sp, k)
+    X = _global_features(sp, gid)
+    dH_top = _store(_rng(sp.seed + 4, k).standard_normal((sp.num_nodes, sp.d), dtype=np.float32), sp.dtype)
+    return RingPart(k, g, X, gid, dH_top)

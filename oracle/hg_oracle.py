@@ -422,7 +422,7 @@ def overlap_intersect(gid_a, gid_b) -> tuple:
 def step(graph: dict, X, params: list, dH_top, view_b: dict, act="relu", layernorm=True,
          ln_eps=1e-5, lambda_n=2e-4, var_eps=1e-8, dloss=0.1, store="f64") -> dict:
     """CSR build -> L layers forward -> overlap rows -> alignment loss and gradient -> L layers
-    backward.  With store="bf16" the tensors handed from layer to layer (outputs, their gradients)
+    backward (view_b None: no alignment term, as for the first subgraph of a sequence).  With store="bf16" the tensors handed from layer to layer (outputs, their gradients)
     are rounded to bf16 as well, like every bf16 tensor the layer interface exchanges.  `view_b` is either {"H_b": bank rows, "gid_a", "gid_b"} (a detached neighbour view)
     or {"idx": overlap rows, "X_b": second input} (a second live stack on the same graph).
     The last layer's upstream gradient is dH_top plus the alignment gradient."""
@@ -447,6 +447,10 @@ def step(graph: dict, X, params: list, dH_top, view_b: dict, act="relu", layerno
         return dh, grads
 
     hs = run_stack(X)
+    if view_b is None:  # first subgraph of a sequence: no alignment term
+        dX, grads = back_stack(hs, np.asarray(dH_top, F64))
+        return dict(H=hs, loss=(0.0, 0.0, 0.0), idx_a=np.zeros(0, np.int64), idx_b=np.zeros(0, np.int64), dX=dX,
+                    grads=grads)
     if "H_b" in view_b:
         ia, ib = overlap_intersect(view_b["gid_a"], view_b["gid_b"])
         Hb = view_b["H_b"]

@@ -118,6 +118,13 @@ class HotPath:
                 hg.hg_layer_fwd(g, self.params[l], self.H[s][l], self.H[s][l + 1], self.saved[s][l], self.scratch, stream)
         top = self.H[0][self.L]
         self.dH[0][self.L].copy_(dH_top)
+        if self.view == "bank" and H_bank is None:
+            # first subgraph of a sequence: no neighbour view yet, no alignment term
+            self.loss.zero_()
+            for l in range(self.L - 1, -1, -1):
+                hg.hg_layer_bwd(g, self.params[l], self.H[0][l], self.saved[0][l], self.dH[0][l + 1], self.dH[0][l],
+                                self.grads[0][l], self.scratch, stream)
+            return
         if self.view == "bank":
             hg.hg_overlap_intersect(gid_a, gid_b, self.idx_a, self.idx_b, self.n_dev, self.isect_scratch, stream)
             n_max = self.n_overlap_max
@@ -136,3 +143,30 @@ class HotPath:
             for l in range(self.L - 1, -1, -1):
                 hg.hg_layer_bwd(g, self.params[l], self.H[s][l], self.saved[s][l], self.dH[s][l + 1], self.dH[s][l],
                                 self.grads[s][l], self.scratch, stream)
+
+
+class Ring:
+    """Overlapping subgraphs processed one after another on one GPU (the per-worker step of
+    Algorithm 1 for each subgraph in turn).  Subgraph k aligns its overlap rows with the final
+    embeddings of subgraph k-1, held as a detached view (no gradient flows into them); the first
+    subgraph has no alignment term.  All subgraphs share the layer weights and sizes."""
+
+    def __init__(self, type_offsets, rels, num_edges: int, d: int, dtype: str, layer_params: list, device="cuda"):
+        n = int(type_offsets[-1])
+        self.path = HotPath(type_offsets, rels, num_edges, d, dtype, layer_params, view="bank", n_overlap_max=n,
+                            n_gid_a=n, n_gid_b=n, device=device)
+        self.bank = torch.empty(n, d, dtype=self.path.td, device=self.path.device)
+        self.bank_gid = torch.empty(n, dtype=torch.int64, device=self.path.device)
+        self.have_bank = False
+
+    def step(self, src, dst, rel, X, dH_top, gid, stream=None):
+        p = self.path
+        if self.have_bank:
+            p.step(src, dst, rel, X, dH_top, gid_a=gid, gid_b=self.bank_gid, H_bank=self.bank, stream=stream)
+        else:
+            p.step(src, dst, rel, X, dH_top, stream=stream)
+        # keep this subgraph's embeddings as the next one's view: swap buffers instead of copying
+        p.H[0][p.L], self.bank = self.bank, p.H[0][p.L]
+        self.bank_gid.copy_(gid)
+        self.have_bank = True
+        return self.bank
