@@ -70,20 +70,23 @@ void timing_end(int slot, cudaStream_t s) {
 // layer workspace layout
 // ---------------------------------------------------------------------------------------------
 struct LayerLayout {
-  void* M;        // saved: csr_rows x d
-  void* Z;        // saved: N x d
-  void* U;        // saved: N x d
-  float2* stats;  // saved: N
+  void* M;        // saved: csr_rows x d relation means
+  void* Z;        // saved (fp32 storage only): N x d
+  void* U;        // saved: N x d pre-activation
+  float2* stats;  // saved: N row statistics
+  void* V;        // saved (bf16 only): R x d x d fused weights W_r W_agg
+  void* Vt;       // saved (bf16 only): their transposes
   float* agg_part;  // scratch: chunk partials
   void* dY;       // scratch: N x d
   void* dU;
-  void* dZ;
+  void* dZ;       // scratch (fp32 storage only)
   void* dMs;      // scratch: csr_rows x d
-  float* cpart;   // scratch: row blocks x 3 x d
+  float* cpart;   // scratch: column partials (blocks x 3 x d)
   float* wpart;   // scratch: splits x d x d
   float* rtmp;    // scratch: levels of the fixed-order reductions
-  void* WrelT;    // scratch: R x d x d
-  void* WaggT;    // scratch: T x d x d
+  float* G;       // scratch (bf16 only): R x d x d products M_r^T dU
+  void* WrelT;    // scratch (fp32 storage only): R x d x d
+  void* WaggT;    // scratch (fp32 storage only): T x d x d
 };
 
 static size_t elem_size(hg_dtype dt) { return dt == HG_F32 ? 4 : 2; }
@@ -93,27 +96,44 @@ static void carve_layer(const hg_graph* g, int d, hg_dtype dt, void* saved, void
   const GraphMeta& m = g->meta;
   const int64_t N = m.type_off[m.num_types];
   const size_t b = elem_size(dt);
+  const bool tc = dt == HG_BF16;
+  const size_t dd = (size_t)d * d;
   Carve s(saved), k(scratch);
+  *L = LayerLayout{};
   L->M = s.take<char>((size_t)g->csr_rows * d * b);
-  L->Z = s.take<char>((size_t)N * d * b);
+  if (!tc) L->Z = s.take<char>((size_t)N * d * b);
   L->U = s.take<char>((size_t)N * d * b);
   L->stats = s.take<float2>(std::max<int64_t>(N, 1));
+  if (tc) {
+    L->V = s.take<char>(m.num_rels * dd * b);
+    L->Vt = s.take<char>(m.num_rels * dd * b);
+  }
   L->agg_part = k.take<float>((size_t)std::max(g->chunk_cap_csr, g->chunk_cap_csc) * d);
   L->dY = k.take<char>((size_t)N * d * b);
   L->dU = k.take<char>((size_t)N * d * b);
-  L->dZ = k.take<char>((size_t)N * d * b);
+  if (!tc) L->dZ = k.take<char>((size_t)N * d * b);
   L->dMs = k.take<char>((size_t)g->csr_rows * d * b);
   int64_t max_rows = 1;
   for (int t = 0; t < m.num_types; ++t) max_rows = std::max(max_rows, m.type_off[t + 1] - m.type_off[t]);
-  L->cpart = k.take<float>((size_t)ceil_div(max_rows, 64) * 3 * d);
+  const int cblocks = (int)std::max<int64_t>(ceil_div(max_rows, 64), std::min<int64_t>(ceil_div(max_rows, 8), 152 * 8));
+  L->cpart = k.take<float>((size_t)cblocks * 3 * d);
   const int wsplits = std::max(wgrad_splits(max_rows), wgrad_tc_splits(max_rows, d));
-  L->wpart = k.take<float>((size_t)wsplits * d * d);
-  L->rtmp = k.take<float>(std::max(reduce_tmp_floats((int)ceil_div(max_rows, 64), d),
-                                   reduce_tmp_floats(wsplits, (int64_t)d * d)));
-  L->WrelT = k.take<char>((size_t)m.num_rels * d * d * b);
-  L->WaggT = k.take<char>((size_t)m.num_types * d * d * b);
+  L->wpart = k.take<float>((size_t)wsplits * dd);
+  L->rtmp = k.take<float>(std::max(reduce_tmp_floats(cblocks, d), reduce_tmp_floats(wsplits, (int64_t)dd)));
+  if (tc) {
+    L->G = k.take<float>(m.num_rels * dd);
+  } else {
+    L->WrelT = k.take<char>(m.num_rels * dd * b);
+    L->WaggT = k.take<char>(m.num_types * dd * b);
+  }
   if (saved_bytes) *saved_bytes = s.used;
   if (scratch_bytes) *scratch_bytes = k.used;
+}
+
+static RelDst rel_dst_of(const GraphMeta& m) {
+  RelDst rd{};
+  for (int r = 0; r < m.num_rels; ++r) rd.v[r] = m.rel_dst[r];
+  return rd;
 }
 
 static hg_status check_params(const hg_graph* g, const hg_layer_params* p) {
@@ -242,9 +262,8 @@ extern "C" hg_status hg_layer_fwd(const hg_graph* graph, const hg_layer_params* 
   carve_layer(graph, d, p->dtype, saved, scratch, &L, nullptr, nullptr);
   HG_TRY(aggregate_forward(graph, p->dtype, d, H_in, L.M, L.agg_part, s));
   if (p->dtype == HG_BF16) {
-    // tensor-core path: B operands are the transposed weights (K-major)
-    HG_TRY(transpose_weights(p->dtype, d, p->W_rel, L.WrelT, m.num_rels, s));
-    HG_TRY(transpose_weights(p->dtype, d, p->W_agg, L.WaggT, m.num_types, s));
+    // tensor-core path: U = sum_r M_r V_r with the fused weights V_r = W_r W_agg[t_r]
+    HG_TRY(tc_fuse_weights(d, p->W_rel, p->W_agg, rel_dst_of(m), m.num_rels, L.V, L.Vt, s));
     for (int t = 0; t < m.num_types; ++t) {
       TcFwdArgs a{};
       for (int r = 0; r < m.num_rels; ++r) {
@@ -259,7 +278,6 @@ extern "C" hg_status hg_layer_fwd(const hg_graph* graph, const hg_layer_params* 
       a.beta = p->layernorm ? (const __nv_bfloat16*)p->ln_beta + (size_t)t * d : nullptr;
       a.H_in = (const __nv_bfloat16*)H_in;
       a.H_out = (__nv_bfloat16*)H_out;
-      a.Z = (__nv_bfloat16*)L.Z;
       a.U = (__nv_bfloat16*)L.U;
       a.stats = L.stats;
       a.off = m.type_off[t];
@@ -268,7 +286,7 @@ extern "C" hg_status hg_layer_fwd(const hg_graph* graph, const hg_layer_params* 
       a.ln = p->layernorm;
       a.eps = p->ln_eps;
       a.status = device_status_ptr();
-      if (a.n > 0) HG_TRY(tc_proj_forward(d, a, L.M, graph->csr_rows, L.WrelT, m.num_rels, L.WaggT, m.num_types, s));
+      if (a.n > 0) HG_TRY(tc_proj_forward(d, a, L.M, graph->csr_rows, L.Vt, m.num_rels, s));
     }
     return HG_OK;
   }
@@ -354,7 +372,6 @@ extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* 
       a.csr_ptr = graph->csr_ptr;
       a.dY = (__nv_bfloat16*)L.dY;
       a.dU = (__nv_bfloat16*)L.dU;
-      a.dZ = (__nv_bfloat16*)L.dZ;
       a.dMs = (__nv_bfloat16*)L.dMs;
       a.part = L.cpart;
       a.off = m.type_off[t];
@@ -362,8 +379,8 @@ extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* 
       a.act = p->act;
       a.ln = p->layernorm;
       a.status = device_status_ptr();
-      HG_TRY(tc_proj_backward(d, a, p->W_agg, m.num_types, p->W_rel, m.num_rels, s));
-      blocks = (int)ceil_div(n, 128);
+      HG_TRY(tc_ln_act_backward(d, a, &blocks, s));
+      HG_TRY(tc_proj_backward(d, a, L.V, m.num_rels, s));
     } else {
       BwdArgs a{};
       a.dH_out = dH_out;
@@ -397,20 +414,22 @@ extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* 
       HG_TRY(reduce_partials(L.cpart + 2 * d, 3LL * d, blocks, d, grads->dln_beta + (size_t)t * d, L.rtmp, s));
     }
     const int64_t off = m.type_off[t];
-    if (tc)
-      HG_TRY(tc_weight_grad(d, L.Z, off, L.dU, off, n, L.wpart, grads->dW_agg + (size_t)t * d * d, L.rtmp, s));
-    else
+    if (!tc)
       HG_TRY(weight_grad(p->dtype, d, L.Z, off, L.dU, off, n, L.wpart, grads->dW_agg + (size_t)t * d * d, L.rtmp, s));
   }
   for (int r = 0; r < m.num_rels; ++r) {
     const int t = m.rel_dst[r];
     const int64_t n = m.type_off[t + 1] - m.type_off[t];
-    float* out = grads->dW_rel + (size_t)r * d * d;
-    if (tc)
-      HG_TRY(tc_weight_grad(d, L.M, m.row_base[r], L.dZ, m.type_off[t], n, L.wpart, out, L.rtmp, s));
+    if (tc)  // G_r = M_r^T dU
+      HG_TRY(tc_weight_grad(d, L.M, m.row_base[r], L.dU, m.type_off[t], n, L.wpart, L.G + (size_t)r * d * d, L.rtmp,
+                            s));
     else
-      HG_TRY(weight_grad(p->dtype, d, L.M, m.row_base[r], L.dZ, m.type_off[t], n, L.wpart, out, L.rtmp, s));
+      HG_TRY(weight_grad(p->dtype, d, L.M, m.row_base[r], L.dZ, m.type_off[t], n, L.wpart,
+                         grads->dW_rel + (size_t)r * d * d, L.rtmp, s));
   }
+  if (tc)  // dW_r = G_r W_agg^T, dW_agg[t] = sum_{r -> t} W_r^T G_r
+    HG_TRY(tc_wgrad_finish(d, L.G, p->W_rel, p->W_agg, rel_dst_of(m), m.num_rels, m.num_types, grads->dW_rel,
+                           grads->dW_agg, s));
   if (dH_in) HG_TRY(aggregate_backward(graph, p->dtype, d, L.dMs, L.dY, dH_in, L.agg_part, s));
   return HG_OK;
 }

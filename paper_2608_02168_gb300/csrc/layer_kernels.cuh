@@ -58,7 +58,6 @@ struct TcFwdArgs {
   const __nv_bfloat16* beta;
   const __nv_bfloat16* H_in;
   __nv_bfloat16* H_out;
-  __nv_bfloat16* Z;
   __nv_bfloat16* U;
   float2* stats;
   int64_t off, n;
@@ -80,7 +79,6 @@ struct TcBwdArgs {
   const int32_t* csr_ptr;
   __nv_bfloat16* dY;
   __nv_bfloat16* dU;
-  __nv_bfloat16* dZ;
   __nv_bfloat16* dMs;
   float* part;  // [gridDim.x][3][D]
   int64_t off, n;
@@ -88,12 +86,20 @@ struct TcBwdArgs {
   int* status;
 };
 
-hg_status tc_proj_forward(int d, const TcFwdArgs& a, const void* M, int64_t m_rows, const void* WrelT, int num_rels,
-                          const void* WaggT, int num_types, cudaStream_t s);
-hg_status tc_proj_backward(int d, const TcBwdArgs& a, const void* Wagg, int num_types, const void* Wrel, int num_rels,
-                           cudaStream_t s);
+// destination type of each relation, passed by value to kernels
+struct RelDst {
+  int v[kMaxRels];
+};
+hg_status tc_fuse_weights(int d, const void* W_rel, const void* W_agg, RelDst rd, int num_rels, void* V, void* Vt,
+                          cudaStream_t s);
+hg_status tc_proj_forward(int d, const TcFwdArgs& a, const void* M, int64_t m_rows, const void* Vt, int num_rels,
+                          cudaStream_t s);
+hg_status tc_ln_act_backward(int d, const TcBwdArgs& a, int* blocks, cudaStream_t s);
+hg_status tc_proj_backward(int d, const TcBwdArgs& a, const void* V, int num_rels, cudaStream_t s);
 hg_status tc_weight_grad(int d, const void* X, int64_t x0, const void* Y, int64_t y0, int64_t n, float* part,
                          float* out, float* tmp, cudaStream_t s);
+hg_status tc_wgrad_finish(int d, const float* G, const void* W_rel, const void* W_agg, RelDst rd, int num_rels,
+                          int num_types, float* dW_rel, float* dW_agg, cudaStream_t s);
 int wgrad_tc_splits(int64_t n, int d);
 int* device_status_ptr();  // device address of the library status word
 

@@ -1,20 +1,23 @@
 // Dense projections of the layer on the 5th-generation tensor cores (tcgen05, bf16 operands,
 // fp32 accumulation in tensor memory).  Used for bf16 storage; fp32 storage stays on CUDA cores.
 //
-// Forward, one CTA per 128 destination rows of type t (Eq. 7 with one W_r per relation, Eq. 11):
-//   phase 1  Z = sum_{r -> t} M_r W_r      A = relation means (TMA, 128 x 64 tiles), B = W_r^T chunks
-//   phase 2  U = Z W_agg[t]                A = Z (written to shared memory by the epilogue), B = W_agg^T
-//   epilogue U += b, stored; Y = act(U) + H_in; H_out = LayerNorm(Y); row statistics saved.
-// Backward, one CTA per 128 rows of type t:
-//   prologue dY = LayerNorm backward, dU = dY act'(U) -> shared memory; column partials of the
-//            bias / gain / shift gradients
-//   dZ = dU W_agg^T  (B = W_agg as stored: rows d_in, K = d_out)
-//   dMs_r = (dZ W_r^T) / deg_r per relation r into t (B = W_r as stored)
-// Weight gradients, split over rows (K = rows): dW = X^T Y with MN-major operands loaded by TMA,
-// fp32 partials per split, reduced in a fixed order afterwards.
+// The two products of Eq. 7 and Eq. 11 are associated as U = sum_r M_r V_r + b with the fused
+// weights V_r = W_r W_agg[t_r] (computed once per layer in fp64, stored in bf16): the same value
+// as (sum_r M_r W_r) W_agg up to rounding, with one GEMM instead of two and no intermediate Z.
 //
-// Thread layout: 128 threads; thread (warp w, lane l) owns accumulator row 32 w + l (its TMEM
-// lane).  Thread 0 issues every TMA load and MMA.  All waits are bounded (tc::kSpinLimit).
+// Forward, one CTA per 128 destination rows of type t:
+//   U = sum_{r -> t} M_r V_r      A = relation means (TMA, 128 x 64 tiles), B = V_r^T chunks
+//   epilogue: U += b, stored; Y = act(U) + H_in; H_out = LayerNorm(Y); row statistics saved.
+// Backward:
+//   ln_act_bwd   (warp per row)  dY = LayerNorm backward, dU = dY act'(U); column partials of the
+//                                bias / gain / shift gradients
+//   proj_bwd_tc  (CTA per 128 rows)  dMs_r = (dU V_r^T) / deg_r   (A = dU by TMA, B = V_r chunks)
+//   weight gradients: G_r = M_r^T dU (split-K GEMM, MN-major TMA operands), then
+//                     dW_r = G_r W_agg^T and dW_agg[t] = sum_{r -> t} W_r^T G_r (wgrad_finish).
+//
+// Thread layout of the tensor-core kernels: 128 threads; thread (warp w, lane l) owns accumulator
+// row 32 w + l (its TMEM lane).  Thread 0 issues every TMA load and MMA.  All waits are bounded
+// (tc::kSpinLimit) and report through the library status word.
 #include <algorithm>
 
 #include "layer_kernels.cuh"
@@ -33,38 +36,20 @@ constexpr int kATile = kTileRows * 128;  // 128 rows x 64 bf16
 
 template <int D>
 struct FwdCfg {
-  static constexpr int kStages = D == 64 ? 4 : (D == 128 ? 2 : 3);
+  static constexpr int kStages = D == 64 ? 4 : 3;
   static constexpr int kB = D * 128;  // D rows x 64 bf16
   static constexpr int kStage = kATile + kB;
-  static constexpr int kZ = kTileRows * D * 2;
-  static constexpr int kSmem = kStages * kStage + kZ + 256 + 1024;
+  static constexpr int kSmem = kStages * kStage + 256 + 1024;
   static constexpr int kTmemCols = D < 32 ? 32 : D;
 };
-
-__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
-  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
-}
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
-// 16 fp32 values -> bf16, stored as two 16-byte pieces into a K-major swizzled tile row.
-__device__ __forceinline__ void put_tile16(uint8_t* tile, int row, int col, const float* v) {
-  // col is a multiple of 16 elements; chunk of 64 columns -> separate 16 KB tile
-  uint8_t* t = tile + (col >> 6) * kATile;
-  const uint32_t cb = (uint32_t)(col & 63) * 2;
-  uint4 lo = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
-  uint4 hi = make_uint4(pack_bf16x2(v[8], v[9]), pack_bf16x2(v[10], v[11]), pack_bf16x2(v[12], v[13]),
-                        pack_bf16x2(v[14], v[15]));
-  *reinterpret_cast<uint4*>(t + sw128_offset(row, cb)) = lo;
-  *reinterpret_cast<uint4*>(t + sw128_offset(row, cb + 16)) = hi;
-}
-
-__device__ __forceinline__ void round16(float* v) {
-#pragma unroll
-  for (int i = 0; i < 16; ++i) v[i] = __bfloat162float(__float2bfloat16_rn(v[i]));
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
 }
 
 __device__ __forceinline__ void load16_bf16(const __nv_bfloat16* p, float* v) {
@@ -76,23 +61,6 @@ __device__ __forceinline__ void store16_bf16(__nv_bfloat16* p, const float* v) {
   st16(p + 8, pack(v + 8, __nv_bfloat16()));
 }
 
-// Butterfly reduction of 32 per-lane values: afterwards lane l holds the warp-wide sum of v[l]
-// (fixed order, deterministic).
-__device__ __forceinline__ float warp_transpose_sum(float* v) {
-  const int lane = threadIdx.x & 31;
-#pragma unroll
-  for (int w = 16; w >= 1; w >>= 1) {
-    const bool upper = (lane & w) != 0;
-#pragma unroll
-    for (int i = 0; i < w; ++i) {
-      const float send = upper ? v[i] : v[i + w];
-      const float keep = upper ? v[i + w] : v[i];
-      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, w);
-    }
-  }
-  return v[0];
-}
-
 }  // namespace
 
 // ---------------------------------------------------------------------------------------------
@@ -101,20 +69,17 @@ __device__ __forceinline__ float warp_transpose_sum(float* v) {
 
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1) proj_fwd_tc(const __grid_constant__ CUtensorMap tm_M,
-                                                          const __grid_constant__ CUtensorMap tm_WrelT,
-                                                          const __grid_constant__ CUtensorMap tm_WaggT, TcFwdArgs a) {
+                                                          const __grid_constant__ CUtensorMap tm_Vt, TcFwdArgs a) {
   using C = FwdCfg<D>;
   constexpr int S = C::kStages;
   constexpr int KC = D / 64;  // 64-wide K chunks per D
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  uint8_t* stage = smem;                               // S x (A | B)
-  uint8_t* ztile = smem + S * C::kStage;               // KC x 16 KB
-  uint64_t* full = reinterpret_cast<uint64_t*>(ztile + C::kZ);
+  uint8_t* stage = smem;  // S x (A | B)
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S * C::kStage);
   uint64_t* empty = full + S;
   uint64_t* accb = empty + S;
   uint32_t* tslot = reinterpret_cast<uint32_t*>(accb + 1);
-  int* abort_flag = reinterpret_cast<int*>(tslot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t m0 = (int64_t)blockIdx.x * kTileRows;
@@ -124,69 +89,49 @@ __global__ void __launch_bounds__(kThreads, 1) proj_fwd_tc(const __grid_constant
       mbar_init(&empty[s], 1);
     }
     mbar_init(accb, 1);
-    *abort_flag = 0;
     fence_mbar_init();
     prefetch_tmap(&tm_M);
-    prefetch_tmap(&tm_WrelT);
-    prefetch_tmap(&tm_WaggT);
+    prefetch_tmap(&tm_Vt);
   }
   if (warp == 0) tmem_alloc(tslot, C::kTmemCols);
   fence_before_sync();
   __syncthreads();
   fence_after_sync();
   const uint32_t tmem = *tslot;
-  const int C1 = a.nrel * KC, CT = C1 + KC;
+  const int CT = a.nrel * KC;
   const uint32_t idesc = idesc_bf16(128, D, false, false);
 
-  auto issue_load = [&](int g) {
-    const int s = g % S;
-    uint8_t* A = stage + s * C::kStage;
-    uint8_t* B = A + kATile;
-    if (g < C1) {
-      const int r = g / KC, kc = g % KC;
-      mbar_expect_tx(&full[s], kATile + C::kB);
-      tma_load_2d(A, &tm_M, kc * 64, (int)(a.mrow0[r] + m0), &full[s]);
-      tma_load_2d(B, &tm_WrelT, kc * 64, a.rel[r] * D, &full[s]);
-    } else {
-      mbar_expect_tx(&full[s], C::kB);
-      tma_load_2d(B, &tm_WaggT, (g - C1) * 64, a.type * D, &full[s]);
-    }
-  };
-  // consumes chunks [g0, g1): MMAs into the accumulator, refills freed stages
-  auto run_chunks = [&](int g0, int g1) {
-    bool ok = *abort_flag == 0;
-    for (int g = g0; g < g1 && ok; ++g) {
-      const int s = g % S;
-      ok = mbar_wait(&full[s], (g / S) & 1);
-      if (!ok) break;
-      fence_after_sync();
-      const uint8_t* A = g < C1 ? stage + s * C::kStage : ztile + (g - C1) * kATile;
-      const uint8_t* B = stage + s * C::kStage + kATile;
-#pragma unroll
-      for (int ks = 0; ks < 4; ++ks) {
-        const uint64_t ad = desc_sw128(smem_u32(A) + ks * 32, 16, 1024);
-        const uint64_t bd = desc_sw128(smem_u32(B) + ks * 32, 16, 1024);
-        mma_bf16(tmem, ad, bd, idesc, (g > g0 || ks > 0) ? 1u : 0u);
-      }
-      mma_commit(&empty[s]);
-      if (g + S < CT) {
-        ok = mbar_wait(&empty[s], (g / S) & 1);
-        if (ok) issue_load(g + S);
-      }
-    }
-    if (!ok) {
-      *abort_flag = 1;
-      atomicOr(a.status, kErrTimeout);
-    }
-    mma_commit(accb);
-  };
-
-  // ---- phase 1: Z = sum_r M_r W_r
+  // ---- U = sum_r M_r V_r
   if (warp == 0) {
     if (lane == 0) {
+      auto issue_load = [&](int g) {
+        const int s = g % S;
+        uint8_t* A = stage + s * C::kStage;
+        const int r = g / KC, kc = g % KC;
+        mbar_expect_tx(&full[s], kATile + C::kB);
+        tma_load_2d(A, &tm_M, kc * 64, (int)(a.mrow0[r] + m0), &full[s]);
+        tma_load_2d(A + kATile, &tm_Vt, kc * 64, a.rel[r] * D, &full[s]);
+      };
+      bool ok = true;
       for (int g = 0; g < S && g < CT; ++g) issue_load(g);
-      if (C1 > 0) run_chunks(0, C1);
-      else mma_commit(accb);
+      for (int g = 0; g < CT && ok; ++g) {
+        const int s = g % S;
+        ok = mbar_wait(&full[s], (g / S) & 1);
+        if (!ok) break;
+        fence_after_sync();
+        const uint32_t A = smem_u32(stage + s * C::kStage);
+#pragma unroll
+        for (int ks = 0; ks < 4; ++ks)
+          mma_bf16(tmem, desc_sw128(A + ks * 32, 16, 1024), desc_sw128(A + kATile + ks * 32, 16, 1024), idesc,
+                   (g > 0 || ks > 0) ? 1u : 0u);
+        mma_commit(&empty[s]);
+        if (g + S < CT) {
+          ok = mbar_wait(&empty[s], (g / S) & 1);
+          if (ok) issue_load(g + S);
+        }
+      }
+      if (!ok) atomicOr(a.status, kErrTimeout);
+      mma_commit(accb);
     }
     __syncwarp();
   }
@@ -197,44 +142,28 @@ __global__ void __launch_bounds__(kThreads, 1) proj_fwd_tc(const __grid_constant
   const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
   if (!mbar_wait(accb, 0)) atomicOr(a.status, kErrTimeout);
   fence_after_sync();
-  // ---- epilogue 1: Z -> bf16 -> saved + shared-memory operand (zero when no relation)
-#pragma unroll 1
-  for (int c = 0; c < D; c += 16) {
-    float v[16];
-    if (C1 > 0) {
-      tmem_ld16(trow + c, v);
-      round16(v);
+  // ---- epilogue: bias, activation, residual, LayerNorm
+  auto u16 = [&](int c, float* u) {  // stored pre-activation of columns c .. c+15
+    float bb[16];
+    if (CT > 0) {
+      tmem_ld16(trow + c, u);
     } else {
 #pragma unroll
-      for (int i = 0; i < 16; ++i) v[i] = 0.f;
+      for (int i = 0; i < 16; ++i) u[i] = 0.f;
     }
-    if (live) store16_bf16(a.Z + node * D + c, v);
-    put_tile16(ztile, row, c, v);
-  }
-  fence_async_smem();
-  fence_before_sync();
-  __syncthreads();
-  fence_after_sync();
-  // ---- phase 2: U = Z W_agg
-  if (warp == 0) {
-    if (lane == 0) run_chunks(C1, CT);
-    __syncwarp();
-  }
-  if (!mbar_wait(accb, 1)) atomicOr(a.status, kErrTimeout);
-  fence_after_sync();
-  // ---- epilogue 2: bias, activation, residual, LayerNorm
+    load16_bf16(a.b + c, bb);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) u[i] = __bfloat162float(__float2bfloat16_rn(u[i] + bb[i]));
+  };
   const __nv_bfloat16* hrow = a.H_in + node * D;
   float sum = 0.f;
   if constexpr (D <= 128) {
     float y[D];
 #pragma unroll
     for (int c = 0; c < D; c += 16) {
-      float u[16], h[16], bb[16];
-      tmem_ld16(trow + c, u);
-      load16_bf16(a.b + c, bb);
+      float u[16], h[16];
+      u16(c, u);
       load16_bf16(hrow + c, h);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) u[i] = __bfloat162float(__float2bfloat16_rn(u[i] + bb[i]));
       if (live) store16_bf16(a.U + node * D + c, u);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
@@ -265,26 +194,19 @@ __global__ void __launch_bounds__(kThreads, 1) proj_fwd_tc(const __grid_constant
   } else {
     // wide rows: three passes over TMEM / H_in instead of holding the row in registers
     auto y16 = [&](int c, float* y) {
-      float u[16], h[16], bb[16];
-      tmem_ld16(trow + c, u);
-      load16_bf16(a.b + c, bb);
+      float u[16], h[16];
+      u16(c, u);
       load16_bf16(hrow + c, h);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        u[i] = __bfloat162float(__float2bfloat16_rn(u[i] + bb[i]));
-        y[i] = act_apply(u[i], a.act) + h[i];
-      }
-      return;
+      for (int i = 0; i < 16; ++i) y[i] = act_apply(u[i], a.act) + h[i];
     };
 #pragma unroll 1
     for (int c = 0; c < D; c += 16) {
-      float u[16], h[16], bb[16], y[16];
-      tmem_ld16(trow + c, u);
-      load16_bf16(a.b + c, bb);
+      float u[16], h[16], y[16];
+      u16(c, u);
       load16_bf16(hrow + c, h);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
-        u[i] = __bfloat162float(__float2bfloat16_rn(u[i] + bb[i]));
         y[i] = act_apply(u[i], a.act) + h[i];
         sum += y[i];
       }
@@ -320,69 +242,213 @@ __global__ void __launch_bounds__(kThreads, 1) proj_fwd_tc(const __grid_constant
   if (warp == 0) tmem_dealloc(tmem, C::kTmemCols);
 }
 
+// Fused weights V_r = W_r W_agg[t_r] accumulated in fp64 (exact for bf16 factors of these sizes),
+// rounded once to bf16; both V_r and its transpose are written.
+template <int D>
+__global__ void fuse_weights(const __nv_bfloat16* __restrict__ W_rel, const __nv_bfloat16* __restrict__ W_agg,
+                             RelDst rel_dst, int num_rels, __nv_bfloat16* __restrict__ V,
+                             __nv_bfloat16* __restrict__ Vt) {
+  const int64_t total = (int64_t)num_rels * D * D;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+    const int r = (int)(e / (D * D));
+    const int i = (int)((e / D) % D), j = (int)(e % D);
+    const __nv_bfloat16* w = W_rel + (int64_t)r * D * D + (int64_t)i * D;
+    const __nv_bfloat16* g = W_agg + (int64_t)rel_dst.v[r] * D * D + j;
+    double acc = 0.0;
+    for (int k = 0; k < D; ++k) acc += (double)__bfloat162float(w[k]) * (double)__bfloat162float(g[(int64_t)k * D]);
+    const __nv_bfloat16 v = __float2bfloat16_rn(__double2float_rn(acc));
+    V[e] = v;
+    Vt[(int64_t)r * D * D + (int64_t)j * D + i] = v;
+  }
+}
+
+// dW_r = G_r W_agg[t_r]^T and dW_agg[t] = sum over r -> t (ascending) of W_r^T G_r, fp32, where
+// G_r = M_r^T dU_{t_r}; types without relations get zero.
+template <int D>
+__global__ void wgrad_finish(const float* __restrict__ G, const __nv_bfloat16* __restrict__ W_rel,
+                             const __nv_bfloat16* __restrict__ W_agg, RelDst rel_dst, int num_rels, int num_types,
+                             float* __restrict__ dW_rel, float* __restrict__ dW_agg) {
+  const int64_t n_rel = (int64_t)num_rels * D * D, total = n_rel + (int64_t)num_types * D * D;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+    if (e < n_rel) {
+      const int r = (int)(e / (D * D));
+      const int i = (int)((e / D) % D), j = (int)(e % D);
+      const float* g = G + (int64_t)r * D * D + (int64_t)i * D;
+      const __nv_bfloat16* w = W_agg + (int64_t)rel_dst.v[r] * D * D + (int64_t)j * D;
+      float acc = 0.f;
+      for (int k = 0; k < D; ++k) acc = fmaf(g[k], __bfloat162float(w[k]), acc);
+      dW_rel[e] = acc;
+    } else {
+      const int64_t f = e - n_rel;
+      const int t = (int)(f / (D * D));
+      const int i = (int)((f / D) % D), j = (int)(f % D);
+      float acc = 0.f;
+      for (int r = 0; r < num_rels; ++r) {
+        if (rel_dst.v[r] != t) continue;
+        const __nv_bfloat16* w = W_rel + (int64_t)r * D * D + i;
+        const float* g = G + (int64_t)r * D * D + j;
+        for (int k = 0; k < D; ++k) acc = fmaf(__bfloat162float(w[(int64_t)k * D]), g[(int64_t)k * D], acc);
+      }
+      dW_agg[f] = acc;
+    }
+  }
+}
+
+// LayerNorm / activation backward, one warp per row (coalesced rows, D / 32 columns per lane):
+// dY = rstd (dXh - mean(dXh) - Xh mean(dXh Xh)), dXh = dH_out gamma, dU = dY act'(U); per-block
+// column partials part[block] = {sum dU, sum dH_out Xh, sum dH_out} over the block's rows.
+template <int D>
+__global__ void __launch_bounds__(256) ln_act_bwd(TcBwdArgs a) {
+  constexpr int E = D / 32;
+  __shared__ float red[8][3][D];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int c0 = lane * E;
+  float g[E];
+#pragma unroll
+  for (int i = 0; i < E; ++i) g[i] = a.ln ? __bfloat162float(a.gamma[c0 + i]) : 1.f;
+  float pdb[E], pdg[E], pdbe[E];
+#pragma unroll
+  for (int i = 0; i < E; ++i) pdb[i] = pdg[i] = pdbe[i] = 0.f;
+  auto load = [&](const __nv_bfloat16* p, float* v) {
+    if constexpr (E == 2) {
+      const uint32_t w = *reinterpret_cast<const uint32_t*>(p);
+      v[0] = __uint_as_float(w << 16);
+      v[1] = __uint_as_float(w & 0xFFFF0000u);
+    } else if constexpr (E == 4) {
+      const uint2 w = *reinterpret_cast<const uint2*>(p);
+      v[0] = __uint_as_float(w.x << 16);
+      v[1] = __uint_as_float(w.x & 0xFFFF0000u);
+      v[2] = __uint_as_float(w.y << 16);
+      v[3] = __uint_as_float(w.y & 0xFFFF0000u);
+    } else {
+      unpack(ld16(p), v, __nv_bfloat16());
+    }
+  };
+  auto store = [&](__nv_bfloat16* p, const float* v) {
+    if constexpr (E == 2) {
+      *reinterpret_cast<uint32_t*>(p) = pack_bf16x2(v[0], v[1]);
+    } else if constexpr (E == 4) {
+      *reinterpret_cast<uint2*>(p) = make_uint2(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]));
+    } else {
+      st16(p, pack(v, __nv_bfloat16()));
+    }
+  };
+  for (int64_t row = (int64_t)blockIdx.x * 8 + warp; row < a.n; row += (int64_t)gridDim.x * 8) {
+    const int64_t node = a.off + row;
+    float dv[E], uv[E], hv[E], dy[E], du[E], xh[E];
+    load(a.dH_out + node * D + c0, dv);
+    load(a.U + node * D + c0, uv);
+    load(a.H_in + node * D + c0, hv);
+    if (a.ln) {
+      const float2 st = a.stats[node];
+      float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+      for (int i = 0; i < E; ++i) {
+        xh[i] = (act_apply(uv[i], a.act) + hv[i] - st.x) * st.y;
+        const float dxh = dv[i] * g[i];
+        s1 += dxh;
+        s2 += dxh * xh[i];
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        s1 += __shfl_xor_sync(0xffffffffu, s1, o);
+        s2 += __shfl_xor_sync(0xffffffffu, s2, o);
+      }
+      const float mean1 = s1 * (1.f / D), mean2 = s2 * (1.f / D);
+#pragma unroll
+      for (int i = 0; i < E; ++i) dy[i] = st.y * (dv[i] * g[i] - mean1 - xh[i] * mean2);
+    } else {
+#pragma unroll
+      for (int i = 0; i < E; ++i) {
+        dy[i] = dv[i];
+        xh[i] = 0.f;
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < E; ++i) {
+      du[i] = __bfloat162float(__float2bfloat16_rn(dy[i] * act_grad(uv[i], a.act)));
+      pdb[i] += du[i];
+      pdg[i] += dv[i] * xh[i];
+      pdbe[i] += dv[i];
+    }
+    store(a.dY + node * D + c0, dy);
+    store(a.dU + node * D + c0, du);
+  }
+#pragma unroll
+  for (int i = 0; i < E; ++i) {
+    red[warp][0][c0 + i] = pdb[i];
+    red[warp][1][c0 + i] = pdg[i];
+    red[warp][2][c0 + i] = pdbe[i];
+  }
+  __syncthreads();
+  for (int k = threadIdx.x; k < 3 * D; k += blockDim.x) {
+    const int q = k / D, c = k % D;
+    float s = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) s += red[w][q][c];
+    a.part[((int64_t)blockIdx.x * 3 + q) * D + c] = s;
+  }
+}
+
 // ---------------------------------------------------------------------------------------------
 // backward, row side
 // ---------------------------------------------------------------------------------------------
 template <int D>
 struct BwdCfg {
-  static constexpr int kStages = D == 256 ? 3 : 2;
+  static constexpr int kStages = 2;
   static constexpr int kB = D * 128;
-  static constexpr int kT = kTileRows * D * 2;  // dU / dZ operand tile
-  static constexpr int kRed = 4 * 3 * D * 4;    // per-warp column partials
-  static constexpr int kSmem = kStages * kB + kT + kRed + 256 + 1024;
+  static constexpr int kT = kTileRows * D * 2;  // dU operand tile (KC x 16 KB)
+  static constexpr int kSmem = kStages * kB + kT + 256 + 1024;
   static constexpr int kTmemCols = D < 32 ? 32 : D;
 };
 
-
+// dMs_r = (dU V_r^T) / deg_r for every relation r into this type; dU loaded by TMA.
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1) proj_bwd_tc(const __grid_constant__ CUtensorMap tm_Wagg,
-                                                          const __grid_constant__ CUtensorMap tm_Wrel, TcBwdArgs a) {
+__global__ void __launch_bounds__(kThreads, 1) proj_bwd_tc(const __grid_constant__ CUtensorMap tm_dU,
+                                                          const __grid_constant__ CUtensorMap tm_V, TcBwdArgs a) {
   using C = BwdCfg<D>;
   constexpr int S = C::kStages;
   constexpr int KC = D / 64;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  uint8_t* bstage = smem;                       // S x B chunk
-  uint8_t* tile = smem + S * C::kB;             // KC x 16 KB
-  float* red = reinterpret_cast<float*>(tile + C::kT);
-  uint64_t* full = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(red) + C::kRed);
+  uint8_t* bstage = smem;            // S x B chunk
+  uint8_t* tile = smem + S * C::kB;  // KC x 16 KB
+  uint64_t* full = reinterpret_cast<uint64_t*>(tile + C::kT);
   uint64_t* empty = full + S;
   uint64_t* accb = empty + S;
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(accb + 1);
+  uint64_t* tileb = accb + 1;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(tileb + 1);
   int* abort_flag = reinterpret_cast<int*>(tslot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t m0 = (int64_t)blockIdx.x * kTileRows;
+  const int CT = KC * a.nrel;
+  auto issue_load = [&](int g) {
+    const int s = g % S;
+    mbar_expect_tx(&full[s], C::kB);
+    tma_load_2d(bstage + s * C::kB, &tm_V, (g % KC) * 64, a.rel[g / KC] * D, &full[s]);
+  };
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
     mbar_init(accb, 1);
+    mbar_init(tileb, 1);
     *abort_flag = 0;
     fence_mbar_init();
-    prefetch_tmap(&tm_Wagg);
-    prefetch_tmap(&tm_Wrel);
+    prefetch_tmap(&tm_dU);
+    prefetch_tmap(&tm_V);
+    mbar_expect_tx(tileb, C::kT);
+    for (int kc = 0; kc < KC; ++kc) tma_load_2d(tile + kc * kATile, &tm_dU, kc * 64, (int)m0, tileb);
+    for (int g = 0; g < S && g < CT; ++g) issue_load(g);
   }
   if (warp == 0) tmem_alloc(tslot, C::kTmemCols);
   fence_before_sync();
   __syncthreads();
   fence_after_sync();
   const uint32_t tmem = *tslot;
-  // B chunks: [0, KC) = W_agg[t], then KC per relation
-  const int CT = KC * (1 + a.nrel);
-  auto issue_load = [&](int g) {
-    const int s = g % S;
-    mbar_expect_tx(&full[s], C::kB);
-    if (g < KC)
-      tma_load_2d(bstage + s * C::kB, &tm_Wagg, g * 64, a.type * D, &full[s]);
-    else
-      tma_load_2d(bstage + s * C::kB, &tm_Wrel, (g % KC) * 64, a.rel[g / KC - 1] * D, &full[s]);
-  };
-  if (threadIdx.x == 0)
-    for (int g = 0; g < S && g < CT; ++g) issue_load(g);
   const uint32_t idesc = idesc_bf16(128, D, false, false);
-  // one product: accumulator = tile (128 x D) x chunks [g0, g0 + KC)
   auto product = [&](int g0) {
     bool ok = *abort_flag == 0;
     for (int g = g0; g < g0 + KC && ok; ++g) {
@@ -390,11 +456,11 @@ __global__ void __launch_bounds__(kThreads, 1) proj_bwd_tc(const __grid_constant
       ok = mbar_wait(&full[s], (g / S) & 1);
       if (!ok) break;
       fence_after_sync();
-      const uint8_t* A = tile + (g - g0) * kATile;
-      const uint8_t* B = bstage + s * C::kB;
+      const uint32_t A = smem_u32(tile + (g - g0) * kATile);
+      const uint32_t B = smem_u32(bstage + s * C::kB);
 #pragma unroll
       for (int ks = 0; ks < 4; ++ks)
-        mma_bf16(tmem, desc_sw128(smem_u32(A) + ks * 32, 16, 1024), desc_sw128(smem_u32(B) + ks * 32, 16, 1024), idesc,
+        mma_bf16(tmem, desc_sw128(A + ks * 32, 16, 1024), desc_sw128(B + ks * 32, 16, 1024), idesc,
                  (g > g0 || ks > 0) ? 1u : 0u);
       mma_commit(&empty[s]);
       if (g + S < CT) {
@@ -408,109 +474,18 @@ __global__ void __launch_bounds__(kThreads, 1) proj_bwd_tc(const __grid_constant
     }
     mma_commit(accb);
   };
-
+  if (threadIdx.x == 0 && !mbar_wait(tileb, 0)) {
+    *abort_flag = 1;
+    atomicOr(a.status, kErrTimeout);
+  }
   const int row = warp * 32 + lane;
   const int64_t m = m0 + row;
   const bool live = m < a.n;
-  const int64_t node = a.off + (live ? m : 0);
   const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
-  // ---- prologue: LayerNorm / activation backward, dU -> tile; column partials
-  {
-    const __nv_bfloat16* dor = a.dH_out + node * D;
-    const __nv_bfloat16* ur = a.U + node * D;
-    const __nv_bfloat16* hr = a.H_in + node * D;
-    const float2 st = (live && a.ln) ? a.stats[node] : make_float2(0.f, 1.f);
-    float s1 = 0.f, s2 = 0.f;
-    if (a.ln) {
-#pragma unroll 1
-      for (int c = 0; c < D; c += 16) {
-        float dv[16], uv[16], hv[16], g[16];
-        load16_bf16(dor + c, dv);
-        load16_bf16(ur + c, uv);
-        load16_bf16(hr + c, hv);
-        load16_bf16(a.gamma + c, g);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const float xh = (act_apply(uv[i], a.act) + hv[i] - st.x) * st.y;
-          const float dxh = dv[i] * g[i];
-          s1 += dxh;
-          s2 += dxh * xh;
-        }
-      }
-    }
-    const float mean1 = s1 * (1.f / D), mean2 = s2 * (1.f / D);
-#pragma unroll 1
-    for (int c = 0; c < D; c += 32) {
-      float pdb[32], pdg[32], pdb2[32];
-#pragma unroll
-      for (int h = 0; h < 32; h += 16) {
-        float dv[16], uv[16], hv[16], g[16], dy[16], du[16];
-        load16_bf16(dor + c + h, dv);
-        load16_bf16(ur + c + h, uv);
-        load16_bf16(hr + c + h, hv);
-        if (a.ln) load16_bf16(a.gamma + c + h, g);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          float xh = 0.f;
-          if (a.ln) {
-            xh = (act_apply(uv[i], a.act) + hv[i] - st.x) * st.y;
-            dy[i] = st.y * (dv[i] * g[i] - mean1 - xh * mean2);
-          } else {
-            dy[i] = dv[i];
-          }
-          du[i] = __bfloat162float(__float2bfloat16_rn(dy[i] * act_grad(uv[i], a.act)));
-          if (!live) du[i] = dy[i] = dv[i] = xh = 0.f;
-          pdb[h + i] = du[i];
-          pdg[h + i] = dv[i] * xh;
-          pdb2[h + i] = dv[i];
-        }
-        if (live) {
-          store16_bf16(a.dY + node * D + c + h, dy);
-          store16_bf16(a.dU + node * D + c + h, du);
-        }
-        put_tile16(tile, row, c + h, du);
-      }
-      const float vdb = warp_transpose_sum(pdb);
-      const float vdg = warp_transpose_sum(pdg);
-      const float vdb2 = warp_transpose_sum(pdb2);
-      red[(warp * 3 + 0) * D + c + lane] = vdb;
-      red[(warp * 3 + 1) * D + c + lane] = vdg;
-      red[(warp * 3 + 2) * D + c + lane] = vdb2;
-    }
-  }
-  fence_async_smem();
-  __syncthreads();
-  for (int k = threadIdx.x; k < 3 * D; k += kThreads) {
-    const int q = k / D, c = k % D;
-    a.part[((int64_t)blockIdx.x * 3 + q) * D + c] =
-        ((red[(0 * 3 + q) * D + c] + red[(1 * 3 + q) * D + c]) + red[(2 * 3 + q) * D + c]) + red[(3 * 3 + q) * D + c];
-  }
-  fence_after_sync();
-  // ---- dZ = dU W_agg^T
-  if (warp == 0) {
-    if (lane == 0) product(0);
-    __syncwarp();
-  }
   uint32_t phase = 0;
-  if (!mbar_wait(accb, phase)) atomicOr(a.status, kErrTimeout);
-  phase ^= 1;
-  fence_after_sync();
-#pragma unroll 1
-  for (int c = 0; c < D; c += 16) {
-    float v[16];
-    tmem_ld16(trow + c, v);
-    round16(v);
-    if (live) store16_bf16(a.dZ + node * D + c, v);
-    put_tile16(tile, row, c, v);
-  }
-  fence_async_smem();
-  fence_before_sync();
-  __syncthreads();
-  fence_after_sync();
-  // ---- dMs_r = (dZ W_r^T) / deg_r
   for (int r = 0; r < a.nrel; ++r) {
     if (warp == 0) {
-      if (lane == 0) product(KC * (1 + r));
+      if (lane == 0) product(KC * r);
       __syncwarp();
     }
     if (!mbar_wait(accb, phase)) atomicOr(a.status, kErrTimeout);
@@ -660,27 +635,45 @@ static hg_status smem_attr_once() {
   return HG_OK;
 }
 
-template <int D>
-static hg_status tc_fwd_t(const TcFwdArgs& a, const void* M, int64_t m_rows, const void* WrelT, int num_rels,
-                          const void* WaggT, int num_types, cudaStream_t s) {
-  HG_TRY(smem_attr_once<D>());
-  CUtensorMap tm_M, tm_W, tm_A;
-  HG_TRY(make_tmap_bf16(&tm_M, M, (uint64_t)std::max<int64_t>(m_rows, 1), D, kTileRows));
-  HG_TRY(make_tmap_bf16(&tm_W, WrelT, (uint64_t)num_rels * D, D, D));
-  HG_TRY(make_tmap_bf16(&tm_A, WaggT, (uint64_t)num_types * D, D, D));
-  return launch("proj_fwd_tc", proj_fwd_tc<D>, dim3((unsigned)ceil_div(a.n, kTileRows)), dim3(kThreads),
-                FwdCfg<D>::kSmem, s, tm_M, tm_W, tm_A, a);
+static unsigned flat_grid(int64_t n) {
+  return (unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(n, 256), 152 * 8));
 }
 
 template <int D>
-static hg_status tc_bwd_t(const TcBwdArgs& a, const void* Wagg, int num_types, const void* Wrel, int num_rels,
+static hg_status tc_fuse_t(const void* W_rel, const void* W_agg, RelDst rd, int num_rels, void* V, void* Vt,
+                           cudaStream_t s) {
+  return launch("fuse_weights", fuse_weights<D>, dim3(flat_grid((int64_t)num_rels * D * D)), dim3(256), 0, s,
+                (const __nv_bfloat16*)W_rel, (const __nv_bfloat16*)W_agg, rd, num_rels, (__nv_bfloat16*)V,
+                (__nv_bfloat16*)Vt);
+}
+
+template <int D>
+static hg_status tc_fwd_t(const TcFwdArgs& a, const void* M, int64_t m_rows, const void* Vt, int num_rels,
                           cudaStream_t s) {
   HG_TRY(smem_attr_once<D>());
-  CUtensorMap tm_A, tm_W;
-  HG_TRY(make_tmap_bf16(&tm_A, Wagg, (uint64_t)num_types * D, D, D));
-  HG_TRY(make_tmap_bf16(&tm_W, Wrel, (uint64_t)num_rels * D, D, D));
+  CUtensorMap tm_M, tm_V;
+  HG_TRY(make_tmap_bf16(&tm_M, M, (uint64_t)std::max<int64_t>(m_rows, 1), D, kTileRows));
+  HG_TRY(make_tmap_bf16(&tm_V, Vt, (uint64_t)num_rels * D, D, D));
+  return launch("proj_fwd_tc", proj_fwd_tc<D>, dim3((unsigned)ceil_div(a.n, kTileRows)), dim3(kThreads),
+                FwdCfg<D>::kSmem, s, tm_M, tm_V, a);
+}
+
+template <int D>
+static hg_status tc_ln_act_t(const TcBwdArgs& a, int* blocks, cudaStream_t s) {
+  const int g = (int)std::max<int64_t>(1, std::min<int64_t>(ceil_div(a.n, 8), 152 * 8));
+  *blocks = g;
+  return launch("ln_act_bwd", ln_act_bwd<D>, dim3(g), dim3(256), 0, s, a);
+}
+
+template <int D>
+static hg_status tc_bwd_t(const TcBwdArgs& a, const void* V, int num_rels, cudaStream_t s) {
+  HG_TRY(smem_attr_once<D>());
+  if (a.nrel == 0) return HG_OK;
+  CUtensorMap tm_dU, tm_V;
+  HG_TRY(make_tmap_bf16(&tm_dU, a.dU + a.off * D, (uint64_t)a.n, D, kTileRows));
+  HG_TRY(make_tmap_bf16(&tm_V, V, (uint64_t)num_rels * D, D, D));
   return launch("proj_bwd_tc", proj_bwd_tc<D>, dim3((unsigned)ceil_div(a.n, kTileRows)), dim3(kThreads),
-                BwdCfg<D>::kSmem, s, tm_A, tm_W, a);
+                BwdCfg<D>::kSmem, s, tm_dU, tm_V, a);
 }
 
 int wgrad_tc_splits(int64_t n, int d) {
@@ -709,31 +702,44 @@ static hg_status tc_wgrad_t(const void* X, int64_t x0, const void* Y, int64_t y0
   return reduce_partials(part, (int64_t)D * D, splits, (int64_t)D * D, out, tmp, s);
 }
 
-hg_status tc_proj_forward(int d, const TcFwdArgs& a, const void* M, int64_t m_rows, const void* WrelT, int num_rels,
-                          const void* WaggT, int num_types, cudaStream_t s) {
-  if (d == 64) return tc_fwd_t<64>(a, M, m_rows, WrelT, num_rels, WaggT, num_types, s);
-  if (d == 128) return tc_fwd_t<128>(a, M, m_rows, WrelT, num_rels, WaggT, num_types, s);
-  if (d == 256) return tc_fwd_t<256>(a, M, m_rows, WrelT, num_rels, WaggT, num_types, s);
-  set_error("unsupported feature width %d", d);
-  return HG_ERR_UNSUPPORTED;
+template <int D>
+static hg_status tc_finish_t(const float* G, const void* W_rel, const void* W_agg, RelDst rd, int num_rels,
+                             int num_types, float* dW_rel, float* dW_agg, cudaStream_t s) {
+  return launch("wgrad_finish", wgrad_finish<D>, dim3(flat_grid((int64_t)(num_rels + num_types) * D * D)), dim3(256),
+                0, s, G, (const __nv_bfloat16*)W_rel, (const __nv_bfloat16*)W_agg, rd, num_rels, num_types, dW_rel,
+                dW_agg);
 }
 
-hg_status tc_proj_backward(int d, const TcBwdArgs& a, const void* Wagg, int num_types, const void* Wrel, int num_rels,
-                           cudaStream_t s) {
-  if (d == 64) return tc_bwd_t<64>(a, Wagg, num_types, Wrel, num_rels, s);
-  if (d == 128) return tc_bwd_t<128>(a, Wagg, num_types, Wrel, num_rels, s);
-  if (d == 256) return tc_bwd_t<256>(a, Wagg, num_types, Wrel, num_rels, s);
-  set_error("unsupported feature width %d", d);
-  return HG_ERR_UNSUPPORTED;
-}
+#define HG_TC_DISPATCH(d, FN, ...)                  \
+  do {                                              \
+    if (d == 64) return FN<64>(__VA_ARGS__);        \
+    if (d == 128) return FN<128>(__VA_ARGS__);      \
+    if (d == 256) return FN<256>(__VA_ARGS__);      \
+    set_error("unsupported feature width %d", d);   \
+    return HG_ERR_UNSUPPORTED;                      \
+  } while (0)
 
+hg_status tc_fuse_weights(int d, const void* W_rel, const void* W_agg, RelDst rd, int num_rels, void* V, void* Vt,
+                          cudaStream_t s) {
+  HG_TC_DISPATCH(d, tc_fuse_t, W_rel, W_agg, rd, num_rels, V, Vt, s);
+}
+hg_status tc_proj_forward(int d, const TcFwdArgs& a, const void* M, int64_t m_rows, const void* Vt, int num_rels,
+                          cudaStream_t s) {
+  HG_TC_DISPATCH(d, tc_fwd_t, a, M, m_rows, Vt, num_rels, s);
+}
+hg_status tc_ln_act_backward(int d, const TcBwdArgs& a, int* blocks, cudaStream_t s) {
+  HG_TC_DISPATCH(d, tc_ln_act_t, a, blocks, s);
+}
+hg_status tc_proj_backward(int d, const TcBwdArgs& a, const void* V, int num_rels, cudaStream_t s) {
+  HG_TC_DISPATCH(d, tc_bwd_t, a, V, num_rels, s);
+}
 hg_status tc_weight_grad(int d, const void* X, int64_t x0, const void* Y, int64_t y0, int64_t n, float* part,
                          float* out, float* tmp, cudaStream_t s) {
-  if (d == 64) return tc_wgrad_t<64>(X, x0, Y, y0, n, part, out, tmp, s);
-  if (d == 128) return tc_wgrad_t<128>(X, x0, Y, y0, n, part, out, tmp, s);
-  if (d == 256) return tc_wgrad_t<256>(X, x0, Y, y0, n, part, out, tmp, s);
-  set_error("unsupported feature width %d", d);
-  return HG_ERR_UNSUPPORTED;
+  HG_TC_DISPATCH(d, tc_wgrad_t, X, x0, Y, y0, n, part, out, tmp, s);
+}
+hg_status tc_wgrad_finish(int d, const float* G, const void* W_rel, const void* W_agg, RelDst rd, int num_rels,
+                          int num_types, float* dW_rel, float* dW_agg, cudaStream_t s) {
+  HG_TC_DISPATCH(d, tc_finish_t, G, W_rel, W_agg, rd, num_rels, num_types, dW_rel, dW_agg, s);
 }
 
 }  // namespace hg
