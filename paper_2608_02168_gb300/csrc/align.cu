@@ -15,7 +15,10 @@
 //   dX = (g - mean(g) - x_hat mean(g x_hat)) / s, added into dH at the overlap rows.
 // All reductions run in a fixed order (per-block partials, then a serial sum over blocks).
 #include <algorithm>
+#include <type_traits>
 
+#include "align_kernels.cuh"
+#include "layer_kernels.cuh"
 #include "simt_tile.cuh"
 
 namespace hg {
@@ -59,84 +62,153 @@ __global__ void intersect_write(const int32_t* __restrict__ flag, const int32_t*
 // ---------------------------------------------------------------------------------------------
 constexpr int kAlignBlocks = 304;  // row blocks of the column reductions (2 per SM)
 
-// Row r of an overlap list, clamped into [0, rows) so that a bad index can never address memory
-// outside the embedding table; bad indices are reported through the flag in `saved` instead.
-__device__ __forceinline__ int64_t safe_row(const int32_t* __restrict__ idx, int64_t r, int64_t rows) {
-  const int64_t x = idx[r];
-  return x < 0 ? 0 : (x >= rows ? rows - 1 : x);
-}
-
-__device__ __forceinline__ int64_t count_of(const int64_t* n_dev, int64_t n_max) {
-  if (!n_dev) return n_max;
-  const int64_t n = *n_dev;
-  return n < 0 ? 0 : (n > n_max ? n_max : n);
-}
-
-// Per-block column partials over rows owned by the block (grid-stride in 8-row steps, fixed
-// order).  mode 0: sum x; mode 1: sum (x - mu)^2.  Both views in one pass:
-// part[block][view][c].
-template <typename T>
-__global__ void align_colstats(const T* __restrict__ Ha, int64_t rows_a, const int32_t* __restrict__ ia,
-                               const T* __restrict__ Hb, int64_t rows_b, const int32_t* __restrict__ ib, int64_t n_max,
-                               const int64_t* __restrict__ n_dev, int d, int mode, const float* __restrict__ mu,
-                               float* __restrict__ part, int32_t* __restrict__ bad) {
-  extern __shared__ float red[];  // [rows_per_pass][2][d]
+// Column sums over the overlap rows of both views, per block (fixed order within the block):
+//   MODE 0: x_a, x_b                               part[block][2][d]
+//   MODE 1: (x_a - mu_a)^2, (x_b - mu_b)^2          part[block][2][d]
+//   MODE 2: the kNumCross sums of z (CrossSum)      part[block][6][d]
+// A thread owns one 16-byte piece (VEC columns) of a row and keeps four rows in flight.
+template <typename T, int D, int MODE>
+__global__ void __launch_bounds__(256, 2) align_colstats(const T* __restrict__ Ha, int64_t rows_a,
+                                                      const int32_t* __restrict__ ia, const T* __restrict__ Hb,
+                                                      int64_t rows_b, const int32_t* __restrict__ ib, int64_t n_max,
+                                                      const int64_t* __restrict__ n_dev,
+                                                      const float* __restrict__ stats, float* __restrict__ part,
+                                                      int32_t* __restrict__ bad) {
+  constexpr int VEC = VecTraits<T>::kElems;
+  constexpr int TPR = D / VEC;                // threads per row
+  constexpr int RPP = 256 / TPR;              // rows per block pass
+  constexpr int Q = MODE == 2 ? kNumCross : 2;
+  constexpr int U = MODE == 2 ? 2 : 4;        // rows in flight per thread
+  constexpr int SLOTS = TPR < 32 ? 8 : RPP;   // partial rows left after the warp-level sums
+  __shared__ float red[SLOTS][D];
   const int64_t n = count_of(n_dev, n_max);
-  const int c = threadIdx.x % d;
-  const int rsub = threadIdx.x / d, rstep = blockDim.x / d;
-  float sa = 0.f, sb = 0.f;
-  const float ma = mode ? mu[c] : 0.f, mb = mode ? mu[d + c] : 0.f;
-  for (int64_t r = (int64_t)blockIdx.x * rstep + rsub; r < n; r += (int64_t)gridDim.x * rstep) {
-    if (mode == 0 && c == 0) {
-      const int64_t xa = ia[r], xb = ib[r];
-      if (xa < 0 || xa >= rows_a || xb < 0 || xb >= rows_b) atomicOr(bad, 1);
-    }
-    const float xa = to_f32(Ha[safe_row(ia, r, rows_a) * d + c]) - ma;
-    const float xb = to_f32(Hb[safe_row(ib, r, rows_b) * d + c]) - mb;
-    sa += mode ? xa * xa : xa;
-    sb += mode ? xb * xb : xb;
+  const int g = threadIdx.x % TPR, sub = threadIdx.x / TPR;
+  const int c0 = g * VEC;
+  float ma[VEC], mb[VEC], ka[VEC], kb[VEC];
+  const float rsn = n > 0 ? rsqrtf((float)n) : 0.f;
+#pragma unroll
+  for (int i = 0; i < VEC; ++i) {
+    ma[i] = MODE ? stats[c0 + i] : 0.f;
+    mb[i] = MODE ? stats[D + c0 + i] : 0.f;
+    ka[i] = MODE == 2 ? rsn / stats[2 * D + c0 + i] : 1.f;  // z = (x - mu) / (s sqrt(n))
+    kb[i] = MODE == 2 ? rsn / stats[3 * D + c0 + i] : 1.f;
   }
-  red[(rsub * 2 + 0) * d + c] = sa;
-  red[(rsub * 2 + 1) * d + c] = sb;
-  __syncthreads();
-  if (rsub == 0) {
-    float ta = 0.f, tb = 0.f;
-    for (int k = 0; k < rstep; ++k) {
-      ta += red[(k * 2 + 0) * d + c];
-      tb += red[(k * 2 + 1) * d + c];
+  float acc[Q][VEC];
+#pragma unroll
+  for (int q = 0; q < Q; ++q)
+#pragma unroll
+    for (int i = 0; i < VEC; ++i) acc[q][i] = 0.f;
+  const int64_t step = (int64_t)gridDim.x * RPP;
+  for (int64_t r0 = (int64_t)blockIdx.x * RPP + sub; r0 < n; r0 += U * step) {
+    float xa[U][VEC], xb[U][VEC];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int64_t r = r0 + u * step;
+      if (r < n) {
+        if (MODE == 0 && g == 0) {
+          const int64_t va = ia[r], vb = ib[r];
+          if (va < 0 || va >= rows_a || vb < 0 || vb >= rows_b) atomicOr(bad, 1);
+        }
+        unpack(ldg16(Ha + safe_row(ia, r, rows_a) * D + c0), xa[u], T());
+        unpack(ldg16(Hb + safe_row(ib, r, rows_b) * D + c0), xb[u], T());
+      }
     }
-    part[((int64_t)blockIdx.x * 2 + 0) * d + c] = ta;
-    part[((int64_t)blockIdx.x * 2 + 1) * d + c] = tb;
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (r0 + u * step >= n) break;
+#pragma unroll
+      for (int i = 0; i < VEC; ++i) {
+        if (MODE == 0) {
+          acc[0][i] += xa[u][i];
+          acc[1][i] += xb[u][i];
+        } else if (MODE == 1) {
+          const float da = xa[u][i] - ma[i], db = xb[u][i] - mb[i];
+          acc[0][i] += da * da;
+          acc[1][i] += db * db;
+        } else {
+          const float za = (xa[u][i] - ma[i]) * ka[i];
+          const float zb = (xb[u][i] - mb[i]) * kb[i];
+          acc[kSumZa][i] += za;
+          acc[kSumZb][i] += zb;
+          acc[kSumZaZb][i] += za * zb;
+          acc[kSumDiff2][i] += (za - zb) * (za - zb);
+          acc[kSumZa2][i] += za * za;
+          acc[kSumZb2][i] += zb * zb;
+        }
+      }
+    }
+  }
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int q = 0; q < Q; ++q) {
+#pragma unroll
+    for (int i = 0; i < VEC; ++i) {
+      float v = acc[q][i];
+      if (TPR < 32) {
+#pragma unroll
+        for (int off = TPR; off < 32; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+      }
+      acc[q][i] = v;
+    }
+    if (TPR < 32) {
+      if (lane < TPR)
+#pragma unroll
+        for (int i = 0; i < VEC; ++i) red[warp][c0 + i] = acc[q][i];
+    } else {
+#pragma unroll
+      for (int i = 0; i < VEC; ++i) red[sub][c0 + i] = acc[q][i];
+    }
+    __syncthreads();
+    for (int c = threadIdx.x; c < D; c += blockDim.x) {
+      float t = 0.f;
+#pragma unroll
+      for (int k = 0; k < SLOTS; ++k) t += red[k][c];
+      part[((int64_t)blockIdx.x * Q + q) * D + c] = t;
+    }
+    __syncthreads();
   }
 }
 
-// mode 0: mu = sum / n.  mode 1: s = sqrt(sum / n + eps).  out[view * d + c].
-__global__ void align_colfinish(const float* __restrict__ part, int blocks, int d, const int64_t* __restrict__ n_dev,
-                                int64_t n_max, int mode, float eps, float* __restrict__ out) {
+// out[q][c] from the block partials (summed in block order): MODE 0 -> mu = sum / n;
+// MODE 1 -> s = sqrt(sum / n + eps); MODE 2 -> the sums themselves.
+__global__ void align_colfinish(const float* __restrict__ part, int blocks, int q_count, int d,
+                                const int64_t* __restrict__ n_dev, int64_t n_max, int mode, float eps,
+                                float* __restrict__ out) {
   const int64_t n = count_of(n_dev, n_max);
-  for (int k = threadIdx.x; k < 2 * d; k += blockDim.x) {
-    float s = 0.f;
-    for (int b = 0; b < blocks; ++b) s += part[(int64_t)b * 2 * d + k];
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= q_count * d) return;
+  const int64_t stride = (int64_t)q_count * d;
+  float s = 0.f;
+  int b = 0;
+  for (; b + 4 <= blocks; b += 4) {
+    const float v0 = part[(b + 0) * stride + k], v1 = part[(b + 1) * stride + k];
+    const float v2 = part[(b + 2) * stride + k], v3 = part[(b + 3) * stride + k];
+    s += v0;
+    s += v1;
+    s += v2;
+    s += v3;
+  }
+  for (; b < blocks; ++b) s += part[b * stride + k];
+  if (mode == 2) {
+    out[k] = s;
+  } else {
     const float m = n > 0 ? s / (float)n : 0.f;
     out[k] = mode ? sqrtf(m + eps) : m;
   }
 }
 
-// Gram partials of the standardised rows: part[split][view][d][d].  Also the per-block L_inv
-// partial (view 0 blocks only, column tile 0): inv[split] = sum (z_a - z_b)^2 over its rows.
+// Gram partials of the standardised rows on the CUDA cores (fp32 storage): part[split][view][d][d].
 template <typename T, int D>
 __global__ void __launch_bounds__(256) align_gram(const T* __restrict__ Ha, int64_t rows_a,
                                                   const int32_t* __restrict__ ia, const T* __restrict__ Hb,
                                                   int64_t rows_b, const int32_t* __restrict__ ib,
                                                   int64_t n_max, const int64_t* __restrict__ n_dev,
-                                                  const float* __restrict__ stats, float* __restrict__ part,
-                                                  float* __restrict__ inv) {
+                                                  const float* __restrict__ stats, float* __restrict__ part) {
   constexpr int TW = D < 128 ? D : 128;
   constexpr int TPT = TW / 16;
   constexpr int KR = 32;
   __shared__ __align__(16) float Xs[KR][TW];
   __shared__ __align__(16) float Ys[KR][TW];
-  __shared__ float inv_red[256];
   const int64_t n = count_of(n_dev, n_max);
   const int view = blockIdx.z;
   const T* H = view ? Hb : Ha;
@@ -151,8 +223,6 @@ __global__ void __launch_bounds__(256) align_gram(const T* __restrict__ Ha, int6
   const int64_t rows_per_split = (n + gridDim.y - 1) / gridDim.y;
   const int64_t r0 = (int64_t)blockIdx.y * rows_per_split;
   const int64_t r1 = min(n, r0 + rows_per_split);
-  const bool do_inv = view == 0 && blockIdx.x == 0;
-  float inv_acc = 0.f;
   float acc[TPT][TPT];
 #pragma unroll
   for (int i = 0; i < TPT; ++i)
@@ -170,16 +240,6 @@ __global__ void __launch_bounds__(256) align_gram(const T* __restrict__ Ha, int6
       }
       Xs[k][c] = x;
       Ys[k][c] = y;
-    }
-    if (do_inv) {
-      for (int e = threadIdx.x; e < KR * D; e += blockDim.x) {
-        const int k = e / D, c = e % D;
-        if (rb + k < r1) {
-          const float za = (to_f32(Ha[safe_row(ia, rb + k, rows_a) * D + c]) - stats[c]) / stats[2 * D + c] * rsn;
-          const float zb = (to_f32(Hb[safe_row(ib, rb + k, rows_b) * D + c]) - stats[D + c]) / stats[3 * D + c] * rsn;
-          inv_acc += (za - zb) * (za - zb);
-        }
-      }
     }
     __syncthreads();
 #pragma unroll 4
@@ -202,15 +262,6 @@ __global__ void __launch_bounds__(256) align_gram(const T* __restrict__ Ha, int6
   for (int i = 0; i < TPT; ++i)
 #pragma unroll
     for (int j = 0; j < TPT; ++j) out[(int64_t)(ti * TW + ty * TPT + i) * D + tj * TW + tx * TPT + j] = acc[i][j];
-  if (do_inv) {
-    inv_red[threadIdx.x] = inv_acc;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      float s = 0.f;
-      for (int k = 0; k < 256; ++k) s += inv_red[k];
-      inv[blockIdx.y] = s;
-    }
-  }
 }
 
 // C[view] = sum of Gram partials in split order (count = 2 d^2 entries).
@@ -225,24 +276,27 @@ __global__ void align_gram_reduce(const float* __restrict__ part, int splits, in
   }
 }
 
-// One block: L_dec from C, L_inv from its partials, loss = [L, L_inv, L_dec].
-__global__ void align_loss_finish(const float* __restrict__ C, int d, const float* __restrict__ inv, int splits,
+// One block: L_dec from C, L_inv from the column sums of (z_a - z_b)^2, loss = [L, L_inv, L_dec].
+__global__ void align_loss_finish(const float* __restrict__ C, int d, const float* __restrict__ cross,
                                   const int64_t* __restrict__ n_dev, int64_t n_max, float lambda_n,
                                   const int32_t* __restrict__ bad, float* __restrict__ loss) {
   __shared__ float red[256];
+  __shared__ float red_inv[256];
   const int64_t n = count_of(n_dev, n_max);
-  float s = 0.f;
+  float s = 0.f, si = 0.f;
   for (int64_t k = threadIdx.x; k < 2LL * d * d; k += blockDim.x) {
     const int64_t e = k % ((int64_t)d * d);
     const float c = C[k] - ((e / d) == (e % d) ? 1.f : 0.f);
     s += c * c;
   }
+  for (int c = threadIdx.x; c < d; c += blockDim.x) si += cross[kSumDiff2 * d + c];
   red[threadIdx.x] = s;
+  red_inv[threadIdx.x] = si;
   __syncthreads();
   if (threadIdx.x == 0) {
     float dec = 0.f, iv = 0.f;
     for (int k = 0; k < (int)blockDim.x; ++k) dec += red[k];
-    for (int k = 0; k < splits; ++k) iv += inv[k];
+    for (int k = 0; k < (int)blockDim.x; ++k) iv += red_inv[k];
     if (n < 2) dec = iv = 0.f;
     if (*bad) dec = iv = __int_as_float(0x7fc00000);  // an overlap index outside its table: NaN loss
     loss[0] = iv + lambda_n * dec;
@@ -387,29 +441,40 @@ __global__ void align_bwd_apply(const T* __restrict__ Ha, int64_t rows_a, const 
 // host side
 // ---------------------------------------------------------------------------------------------
 static int gram_splits(int64_t n_max) { return (int)std::max<int64_t>(1, std::min<int64_t>(152, ceil_div(n_max, 512))); }
+static int max_gram_splits(int64_t n_max, int d) { return std::max(gram_splits(n_max), align_gram_tc_splits(n_max, d, 152)); }
 
 struct AlignLayout {
-  float* stats;  // saved: [mu_a, mu_b, s_a, s_b] (4 d)
-  float* C;      // saved: [C_a, C_b] (2 d^2)
-  int32_t* bad;  // saved: non-zero when an overlap index lies outside its table
-  float* part;   // scratch: column partials (kAlignBlocks x 2 x d) / bwd partials (row blocks x 4 d)
-  float* gpart;  // scratch: Gram partials (splits x 2 x d^2)
-  float* inv;    // scratch: L_inv partials (splits)
-  float* G;      // scratch: 2 x n_max x d
-  float* means;  // scratch: 4 d
+  float* stats;   // saved: [mu_a, mu_b, s_a, s_b] (4 d)
+  float* C;       // saved: [C_a, C_b] (2 d^2)
+  int32_t* bad;   // saved: non-zero when an overlap index lies outside its table
+  float* cross;   // saved: kNumCross column sums of z (CrossSum order, 6 d)
+  float* part;    // scratch: column partials (blocks x 6 d) / fp32 backward partials (row blocks x 4 d)
+  float* gpart;   // scratch: Gram partials (splits x 2 x d^2)
+  float* rtmp;    // scratch: reduction temporaries
+  float* G;       // scratch: fp32 backward, 2 x n_max x d
+  float* means;   // scratch: 4 d
+  void* cmi;      // scratch: bf16 backward operand C - I, 2 d^2 bf16
+  int max_splits;
 };
 
-static void carve_align(void* saved, void* scratch, int64_t n_max, int d, AlignLayout* L, size_t* sb, size_t* kb) {
-  Carve s(saved), k(scratch);
+static void carve_saved(Carve& s, int d, AlignLayout* L) {
   L->stats = s.take<float>(4 * d);
   L->C = s.take<float>(2 * (size_t)d * d);
   L->bad = s.take<int32_t>(1);
+  L->cross = s.take<float>((size_t)kNumCross * d);
+}
+
+static void carve_align(void* saved, void* scratch, int64_t n_max, int d, AlignLayout* L, size_t* sb, size_t* kb) {
+  Carve s(saved), k(scratch);
+  carve_saved(s, d, L);
   const int64_t rb = std::max<int64_t>(1, ceil_div(n_max, kBM));
-  L->part = k.take<float>(std::max<int64_t>(kAlignBlocks * 2 * d, std::min<int64_t>(rb, kAlignBlocks) * 4 * d));
-  L->gpart = k.take<float>((size_t)gram_splits(n_max) * 2 * d * d);
-  L->inv = k.take<float>(gram_splits(n_max));
+  L->max_splits = max_gram_splits(n_max, d);
+  L->part = k.take<float>(std::max<int64_t>((int64_t)kAlignBlocks * kNumCross * d, std::min<int64_t>(rb, kAlignBlocks) * 4 * d));
+  L->gpart = k.take<float>((size_t)L->max_splits * 2 * d * d);
+  L->rtmp = k.take<float>(reduce_tmp_floats(L->max_splits, (int64_t)d * d));
   L->G = k.take<float>(2 * std::max<int64_t>(n_max, 1) * d);
   L->means = k.take<float>(4 * d);
+  L->cmi = k.take<__nv_bfloat16>(2 * (size_t)d * d);
   if (sb) *sb = s.used;
   if (kb) *kb = k.used;
 }
@@ -439,56 +504,80 @@ static hg_status check_align_args(const AlignIn& in, int32_t d, hg_dtype dt, con
   return HG_OK;
 }
 
+// The loss (both entry points): three column passes (mean, variance, the sums of z), the Gram
+// partials of both views over `splits` row ranges, their fixed-order reduction and the loss.
+template <typename T, int D>
+static hg_status align_loss_run(const AlignIn& in, float lambda_n, float eps, float* loss, const AlignLayout& L,
+                                int splits, cudaStream_t s) {
+  constexpr int RPP = 256 / (D / VecTraits<T>::kElems);
+  const int blocks = (int)std::max<int64_t>(1, std::min<int64_t>(kAlignBlocks, ceil_div(in.n_max, RPP)));
+  const T* Ha = (const T*)in.Ha;
+  const T* Hb = (const T*)in.Hb;
+  const float* no_stats = nullptr;
+  HG_CUDA(cudaMemsetAsync(L.bad, 0, sizeof(int32_t), s));
+  HG_TRY(launch("align_colstats", align_colstats<T, D, 0>, dim3(blocks), dim3(256), 0, s, Ha, in.rows_a, in.ia, Hb,
+                in.rows_b, in.ib, in.n_max, in.n_dev, no_stats, L.part, L.bad));
+  HG_TRY(launch("align_colfinish", align_colfinish, dim3((unsigned)ceil_div(2 * D, 256)), dim3(256), 0, s,
+                (const float*)L.part, blocks, 2, D, in.n_dev, in.n_max, 0, 0.f, L.stats));
+  HG_TRY(launch("align_colstats", align_colstats<T, D, 1>, dim3(blocks), dim3(256), 0, s, Ha, in.rows_a, in.ia, Hb,
+                in.rows_b, in.ib, in.n_max, in.n_dev, (const float*)L.stats, L.part, L.bad));
+  HG_TRY(launch("align_colfinish", align_colfinish, dim3((unsigned)ceil_div(2 * D, 256)), dim3(256), 0, s,
+                (const float*)L.part, blocks, 2, D, in.n_dev, in.n_max, 1, eps, L.stats + 2 * D));
+  HG_TRY(launch("align_colstats", align_colstats<T, D, 2>, dim3(blocks), dim3(256), 0, s, Ha, in.rows_a, in.ia, Hb,
+                in.rows_b, in.ib, in.n_max, in.n_dev, (const float*)L.stats, L.part, L.bad));
+  HG_TRY(launch("align_colfinish", align_colfinish, dim3((unsigned)ceil_div(kNumCross * D, 256)), dim3(256), 0, s,
+                (const float*)L.part, blocks, (int)kNumCross, D, in.n_dev, in.n_max, 2, 0.f, L.cross));
+  if constexpr (std::is_same<T, __nv_bfloat16>::value) {
+    HG_TRY(align_gram_tc(D, in.Ha, in.rows_a, in.ia, in.Hb, in.rows_b, in.ib, in.n_max, in.n_dev, L.stats, splits,
+                         L.gpart, s));
+  } else {
+    constexpr int TW = D < 128 ? D : 128;
+    const int tiles = (D / TW) * (D / TW);
+    HG_TRY(launch("align_gram", align_gram<T, D>, dim3(tiles, splits, 2), dim3(256), 0, s, Ha, in.rows_a, in.ia, Hb,
+                  in.rows_b, in.ib, in.n_max, in.n_dev, (const float*)L.stats, L.gpart));
+  }
+  for (int v = 0; v < 2; ++v)
+    HG_TRY(reduce_partials(L.gpart + (size_t)v * D * D, 2LL * D * D, splits, (int64_t)D * D, L.C + (size_t)v * D * D,
+                           L.rtmp, s));
+  return launch("align_loss_finish", align_loss_finish, dim3(1), dim3(256), 0, s, (const float*)L.C, D,
+                (const float*)L.cross, in.n_dev, in.n_max, lambda_n, (const int32_t*)L.bad, loss);
+}
+
 template <typename T, int D>
 static hg_status align_loss_t(const AlignIn& in, float lambda_n, float eps, float* loss, AlignLayout& L,
                               cudaStream_t s) {
-  const int rstep = 256 / D;
-  const size_t cs_smem = sizeof(float) * rstep * 2 * D;
-  const int blocks = (int)std::max<int64_t>(1, std::min<int64_t>(kAlignBlocks, ceil_div(in.n_max, rstep)));
-  const T* Ha = (const T*)in.Ha;
-  const T* Hb = (const T*)in.Hb;
-  HG_CUDA(cudaMemsetAsync(L.bad, 0, sizeof(int32_t), s));
-  HG_TRY(launch("align_colstats", align_colstats<T>, dim3(blocks), dim3(256), cs_smem, s, Ha, in.rows_a, in.ia, Hb,
-                in.rows_b, in.ib, in.n_max, in.n_dev, D, 0, (const float*)nullptr, L.part, L.bad));
-  HG_TRY(launch("align_colfinish", align_colfinish, dim3(1), dim3(256), 0, s, (const float*)L.part, blocks, D,
-                in.n_dev, in.n_max, 0, 0.f, L.stats));
-  HG_TRY(launch("align_colstats", align_colstats<T>, dim3(blocks), dim3(256), cs_smem, s, Ha, in.rows_a, in.ia, Hb,
-                in.rows_b, in.ib, in.n_max, in.n_dev, D, 1, (const float*)L.stats, L.part, L.bad));
-  HG_TRY(launch("align_colfinish", align_colfinish, dim3(1), dim3(256), 0, s, (const float*)L.part, blocks, D,
-                in.n_dev, in.n_max, 1, eps, L.stats + 2 * D));
-  const int splits = gram_splits(in.n_max);
-  constexpr int TW = D < 128 ? D : 128;
-  const int tiles = (D / TW) * (D / TW);
-  HG_TRY(launch("align_gram", align_gram<T, D>, dim3(tiles, splits, 2), dim3(256), 0, s, Ha, in.rows_a, in.ia, Hb,
-                in.rows_b, in.ib, in.n_max, in.n_dev, (const float*)L.stats, L.gpart, L.inv));
-  HG_TRY(launch("align_gram_reduce", align_gram_reduce, dim3((unsigned)ceil_div(2LL * D * D, 256)), dim3(256), 0, s,
-                (const float*)L.gpart, splits, 2LL * D * D, L.C));
-  return launch("align_loss_finish", align_loss_finish, dim3(1), dim3(256), 0, s, (const float*)L.C, D,
-                (const float*)L.inv, splits, in.n_dev, in.n_max, lambda_n, (const int32_t*)L.bad, loss);
+  const int splits = std::is_same<T, __nv_bfloat16>::value ? align_gram_tc_splits(in.n_max, D, L.max_splits)
+                                                           : std::min(gram_splits(in.n_max), L.max_splits);
+  return align_loss_run<T, D>(in, lambda_n, eps, loss, L, splits, s);
 }
 
 template <typename T, int D>
 static hg_status align_bwd_t(const AlignIn& in, float lambda_n, float dloss, void* dHa, void* dHb, AlignLayout& L,
                              cudaStream_t s) {
   if (in.n_max == 0 || (!dHa && !dHb)) return HG_OK;
-  const size_t smem = sizeof(float) * (kBM * (D + 4) + kKC * D + 16 * 2 * D);
-  static bool attr = false;
-  if (!attr) {
-    HG_CUDA(cudaFuncSetAttribute(align_bwd_rows<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-    attr = true;
+  if constexpr (std::is_same<T, __nv_bfloat16>::value) {
+    return align_bwd_tc(D, in.Ha, in.rows_a, in.ia, in.Hb, in.rows_b, in.ib, in.n_max, in.n_dev, L.stats, L.C,
+                        L.cross, L.bad, lambda_n, dloss, L.cmi, L.means, dHa, dHb, s);
+  } else {
+    const size_t smem = sizeof(float) * (kBM * (D + 4) + kKC * D + 16 * 2 * D);
+    static bool attr = false;
+    if (!attr) {
+      HG_CUDA(cudaFuncSetAttribute(align_bwd_rows<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+      attr = true;
+    }
+    const T* Ha = (const T*)in.Ha;
+    const T* Hb = (const T*)in.Hb;
+    const int rblocks = (int)std::max<int64_t>(1, std::min<int64_t>(ceil_div(in.n_max, kBM), kAlignBlocks));
+    HG_TRY(launch("align_bwd_rows", align_bwd_rows<T, D>, dim3(rblocks, 2), dim3(256), smem, s, Ha, in.rows_a, in.ia,
+                  Hb, in.rows_b, in.ib, in.n_max, in.n_dev, (const float*)L.stats, (const float*)L.C, lambda_n, dloss,
+                  L.G, L.part));
+    HG_TRY(launch("align_bwd_means", align_bwd_means, dim3(1), dim3(256), 0, s, (const float*)L.part, rblocks, D,
+                  in.n_dev, in.n_max, L.means));
+    const unsigned g = (unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(2 * in.n_max * D, 256), 152 * 16));
+    return launch("align_bwd_apply", align_bwd_apply<T>, dim3(g), dim3(256), 0, s, Ha, in.rows_a, in.ia, Hb,
+                  in.rows_b, in.ib, in.n_max, in.n_dev, D, (const float*)L.stats, (const float*)L.G,
+                  (const float*)L.means, (const int32_t*)L.bad, (T*)dHa, (T*)dHb);
   }
-  const T* Ha = (const T*)in.Ha;
-  const T* Hb = (const T*)in.Hb;
-  const int rblocks = (int)std::max<int64_t>(1, std::min<int64_t>(ceil_div(in.n_max, kBM), kAlignBlocks));
-  HG_TRY(launch("align_bwd_rows", align_bwd_rows<T, D>, dim3(rblocks, 2), dim3(256), smem, s, Ha, in.rows_a, in.ia,
-                Hb, in.rows_b, in.ib, in.n_max, in.n_dev, (const float*)L.stats, (const float*)L.C, lambda_n, dloss,
-                L.G, L.part));
-  HG_TRY(launch("align_bwd_means", align_bwd_means, dim3(1), dim3(256), 0, s, (const float*)L.part, rblocks, D,
-                in.n_dev, in.n_max, L.means));
-  const unsigned g = (unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(2 * in.n_max * D, 256), 152 * 16));
-  return launch("align_bwd_apply", align_bwd_apply<T>, dim3(g), dim3(256), 0, s, Ha, in.rows_a, in.ia, Hb, in.rows_b,
-                in.ib, in.n_max, in.n_dev, D, (const float*)L.stats, (const float*)L.G, (const float*)L.means,
-                (const int32_t*)L.bad, (T*)dHa, (T*)dHb);
 }
 
 #define HG_DISPATCH_ALIGN(dtype, d, FN, ...)                                                \
@@ -647,41 +736,22 @@ static hg_status static_align_scratch(void** out) {
   return HG_OK;
 }
 
-// Layout of the static scratch for width d: column partials, Gram partials, L_inv partials.
-static size_t carve_static(void* base, int d, float** part, float** gpart, float** inv) {
+// Layout of the static scratch for width d: column partials, Gram partials, reduction temporaries.
+static size_t carve_static(void* base, int d, AlignLayout* L) {
   Carve k(base);
-  *part = k.take<float>((size_t)kAlignBlocks * 2 * d);
-  *gpart = k.take<float>((size_t)kStaticGramSplits * 2 * d * d);
-  *inv = k.take<float>(kStaticGramSplits);
+  L->part = k.take<float>((size_t)kAlignBlocks * kNumCross * d);
+  L->gpart = k.take<float>((size_t)kStaticGramSplits * 2 * d * d);
+  L->rtmp = k.take<float>(reduce_tmp_floats(kStaticGramSplits, (int64_t)d * d));
+  L->max_splits = kStaticGramSplits;
   return k.used;
 }
 
 template <typename T, int D>
-static hg_status align_loss_static_t(const AlignIn& in, float lambda_n, float eps, float* loss, float* stats, float* C,
-                                     int32_t* bad, float* part, float* gpart, float* inv, cudaStream_t s) {
-  const int rstep = 256 / D;
-  const size_t cs_smem = sizeof(float) * rstep * 2 * D;
-  const int blocks = (int)std::max<int64_t>(1, std::min<int64_t>(kAlignBlocks, ceil_div(in.n_max, rstep)));
-  const int splits = std::min(gram_splits(in.n_max), kStaticGramSplits);
-  const T* Ha = (const T*)in.Ha;
-  const T* Hb = (const T*)in.Hb;
-  HG_CUDA(cudaMemsetAsync(bad, 0, sizeof(int32_t), s));
-  HG_TRY(launch("align_colstats", align_colstats<T>, dim3(blocks), dim3(256), cs_smem, s, Ha, in.rows_a, in.ia, Hb,
-                in.rows_b, in.ib, in.n_max, in.n_dev, D, 0, (const float*)nullptr, part, bad));
-  HG_TRY(launch("align_colfinish", align_colfinish, dim3(1), dim3(256), 0, s, (const float*)part, blocks, D, in.n_dev,
-                in.n_max, 0, 0.f, stats));
-  HG_TRY(launch("align_colstats", align_colstats<T>, dim3(blocks), dim3(256), cs_smem, s, Ha, in.rows_a, in.ia, Hb,
-                in.rows_b, in.ib, in.n_max, in.n_dev, D, 1, (const float*)stats, part, bad));
-  HG_TRY(launch("align_colfinish", align_colfinish, dim3(1), dim3(256), 0, s, (const float*)part, blocks, D, in.n_dev,
-                in.n_max, 1, eps, stats + 2 * D));
-  constexpr int TW = D < 128 ? D : 128;
-  const int tiles = (D / TW) * (D / TW);
-  HG_TRY(launch("align_gram", align_gram<T, D>, dim3(tiles, splits, 2), dim3(256), 0, s, Ha, in.rows_a, in.ia, Hb,
-                in.rows_b, in.ib, in.n_max, in.n_dev, (const float*)stats, gpart, inv));
-  HG_TRY(launch("align_gram_reduce", align_gram_reduce, dim3((unsigned)ceil_div(2LL * D * D, 256)), dim3(256), 0, s,
-                (const float*)gpart, splits, 2LL * D * D, C));
-  return launch("align_loss_finish", align_loss_finish, dim3(1), dim3(256), 0, s, (const float*)C, D,
-                (const float*)inv, splits, in.n_dev, in.n_max, lambda_n, (const int32_t*)bad, loss);
+static hg_status align_loss_static_t(const AlignIn& in, float lambda_n, float eps, float* loss, const AlignLayout& L,
+                                     cudaStream_t s) {
+  const int splits = std::is_same<T, __nv_bfloat16>::value ? align_gram_tc_splits(in.n_max, D, kStaticGramSplits)
+                                                           : std::min(gram_splits(in.n_max), kStaticGramSplits);
+  return align_loss_run<T, D>(in, lambda_n, eps, loss, L, splits, s);
 }
 
 }  // namespace hg
@@ -698,20 +768,19 @@ extern "C" hg_status hg_overlap_align_loss_static(const void* H_a, int64_t rows_
   HG_TRY(check_align_args(in, d, dtype, saved, scratch));
   HG_REQUIRE(loss_out != nullptr, "loss_out must be non-null");
   HG_REQUIRE(lambda_n >= 0.f && var_eps >= 0.f, "lambda_n and var_eps must be >= 0");
-  float *part, *gpart, *inv;
-  const size_t need = carve_static(nullptr, d, &part, &gpart, &inv);
+  AlignLayout L{};
+  const size_t need = carve_static(nullptr, d, &L);
   if (need > kStaticAlignBytes) {
     set_error("d=%d needs %zu bytes of scratch, beyond the %zu-byte static array of this entry point", d, need,
               kStaticAlignBytes);
     return HG_ERR_UNSUPPORTED;
   }
-  carve_static(scratch, d, &part, &gpart, &inv);
-  AlignLayout L;  // only the `saved` part (statistics, Gram matrices, index flag) is used
-  carve_align(saved, nullptr, n_max, d, &L, nullptr, nullptr);
+  carve_static(scratch, d, &L);
+  Carve sv(saved);  // the `saved` part (statistics, Gram matrices, index flag, column sums)
+  carve_saved(sv, d, &L);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
 #define HG_STATIC_CASE(T, D_)                                                                                \
-  if (d == D_)                                                                                               \
-    return align_loss_static_t<T, D_>(in, lambda_n, var_eps, loss_out, L.stats, L.C, L.bad, part, gpart, inv, s);
+  if (d == D_) return align_loss_static_t<T, D_>(in, lambda_n, var_eps, loss_out, L, s);
   if (dtype == HG_F32) {
     HG_STATIC_CASE(float, 64)
     HG_STATIC_CASE(float, 128)

@@ -118,8 +118,9 @@ hg_status exclusive_scan(const int32_t* in, int32_t* out, int64_t n, void* scrat
 // ---------------------------------------------------------------------------------------------
 constexpr int kSortThreads = 256;
 constexpr int kSortWarps = kSortThreads / 32;
-constexpr int kSortItems = 16;                          // per thread
-constexpr int kSortTile = kSortThreads * kSortItems;    // 4096 per block
+constexpr int kSortItems = 8;                           // per thread
+constexpr int kSortTile = kSortThreads * kSortItems;    // 2048 per block
+constexpr int kWarpSlice = kSortTile / kSortWarps;      // 256 consecutive items per warp
 constexpr int kRadix = 256;
 
 __global__ void __launch_bounds__(kSortThreads) radix_hist(const uint32_t* __restrict__ keys, int64_t n,
@@ -129,7 +130,7 @@ __global__ void __launch_bounds__(kSortThreads) radix_hist(const uint32_t* __res
   h[threadIdx.x] = 0;
   __syncthreads();
   const int64_t base = (int64_t)blockIdx.x * kSortTile;
-#pragma unroll 4
+#pragma unroll
   for (int i = 0; i < kSortItems; ++i) {
     int64_t idx = base + (int64_t)i * kSortThreads + threadIdx.x;
     if (idx < n) atomicAdd(&h[(keys[idx] >> shift) & (kRadix - 1)], 1);
@@ -138,80 +139,129 @@ __global__ void __launch_bounds__(kSortThreads) radix_hist(const uint32_t* __res
   hist[(int64_t)threadIdx.x * tiles + blockIdx.x] = h[threadIdx.x];
 }
 
-// Each warp owns a contiguous 512-item slice of the tile and walks it 32 items at a time, so the
-// item order inside the tile is (warp, round, lane).  Ranks among equal digits come from
-// __match_any_sync within a round plus per-warp running counts, then an exclusive prefix over
-// warps, then the tile's global base per digit: equal keys keep their input order (stable).
+// Stable scatter of one 2048-item tile.  (1) The tile is staged in shared memory (coalesced).
+// (2) Warp w ranks its 256 consecutive items 32 at a time with __match_any_sync, keeping per-digit
+// running counts, so the item order inside the tile is (warp, round, lane).  (3) Per-digit
+// prefixes over warps and over digits give every item its position in the tile sorted by digit
+// (equal digits keep their order), where it is written in shared memory.  (4) Consecutive
+// threads write consecutive sorted items to base[digit] + (position - tile start of the digit):
+// runs of equal digits go out coalesced.
+template <bool kTwo>
 __global__ void __launch_bounds__(kSortThreads) radix_scatter(
     const uint32_t* __restrict__ keys_in, const uint32_t* __restrict__ vals_in,
-    uint32_t* __restrict__ keys_out, uint32_t* __restrict__ vals_out, int64_t n, int shift,
-    const int32_t* __restrict__ offs, int64_t tiles) {
+    const uint32_t* __restrict__ vals2_in, uint32_t* __restrict__ keys_out, uint32_t* __restrict__ vals_out,
+    uint32_t* __restrict__ vals2_out, int64_t n, int shift, const int32_t* __restrict__ offs, int64_t tiles) {
+  __shared__ uint32_t skey[kSortTile], sval[kSortTile];  // sorted tile
+  __shared__ uint32_t tkey[kSortTile], tval[kSortTile];  // staged tile
+  __shared__ uint32_t sval2[kTwo ? kSortTile : 1], tval2[kTwo ? kSortTile : 1];
+  __shared__ uint16_t srank[kSortTile];
   __shared__ int whist[kSortWarps][kRadix];
-  __shared__ int base[kRadix];
+  __shared__ int dstart[kRadix];  // tile position where each digit's run starts
+  __shared__ int gbase[kRadix];   // global position of the digit's run of this tile
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t t0 = (int64_t)blockIdx.x * kSortTile;
+  const int cnt = (int)min((int64_t)kSortTile, n - t0);
   for (int i = threadIdx.x; i < kSortWarps * kRadix; i += kSortThreads) (&whist[0][0])[i] = 0;
-  base[threadIdx.x] = offs[(int64_t)threadIdx.x * tiles + blockIdx.x];
-  __syncthreads();
-  const unsigned lt_mask = (1u << lane) - 1u;
-  const int64_t slice = (int64_t)blockIdx.x * kSortTile + (int64_t)warp * (kSortItems * 32);
-  uint32_t k[kSortItems], v[kSortItems];
-  int rank[kSortItems], dg[kSortItems];
+  gbase[threadIdx.x] = offs[(int64_t)threadIdx.x * tiles + blockIdx.x];
 #pragma unroll
-  for (int it = 0; it < kSortItems; ++it) {
-    const int64_t idx = slice + it * 32 + lane;
-    const bool ok = idx < n;
-    k[it] = ok ? keys_in[idx] : 0u;
-    v[it] = ok ? vals_in[idx] : 0u;
-    const int d = ok ? (int)((k[it] >> shift) & (kRadix - 1)) : kRadix;
-    const unsigned peers = __match_any_sync(0xffffffffu, d);
-    const int cnt = d < kRadix ? whist[warp][d] : 0;
-    __syncwarp();
-    if (d < kRadix && lane == __ffs(peers) - 1) whist[warp][d] = cnt + __popc(peers);
-    __syncwarp();
-    rank[it] = cnt + __popc(peers & lt_mask);
-    dg[it] = d;
+  for (int i = 0; i < kSortItems; ++i) {
+    const int j = i * kSortThreads + threadIdx.x;
+    if (j < cnt) {
+      tkey[j] = keys_in[t0 + j];
+      tval[j] = vals_in[t0 + j];
+      if (kTwo) tval2[j] = vals2_in[t0 + j];
+    }
   }
   __syncthreads();
-  {
+  const unsigned lt_mask = (1u << lane) - 1u;
+  for (int r = 0; r < kWarpSlice / 32; ++r) {
+    const int j = warp * kWarpSlice + r * 32 + lane;
+    const bool ok = j < cnt;
+    const int d = ok ? (int)((tkey[j] >> shift) & (kRadix - 1)) : kRadix;
+    const unsigned peers = __match_any_sync(0xffffffffu, d);
+    const int c = d < kRadix ? whist[warp][d] : 0;
+    __syncwarp();
+    if (d < kRadix && lane == __ffs(peers) - 1) whist[warp][d] = c + __popc(peers);
+    __syncwarp();
+    if (ok) srank[j] = (uint16_t)(c + __popc(peers & lt_mask));
+  }
+  __syncthreads();
+  {  // per digit: exclusive prefix over warps; tile total
     int run = 0;
 #pragma unroll
     for (int w = 0; w < kSortWarps; ++w) {
-      int c = whist[w][threadIdx.x];
+      const int c = whist[w][threadIdx.x];
       whist[w][threadIdx.x] = run;
       run += c;
     }
+    dstart[threadIdx.x] = run;
   }
   __syncthreads();
+  if (warp == 0) {  // exclusive scan of the 256 digit totals
+    int v[kRadix / 32], s = 0;
 #pragma unroll
-  for (int it = 0; it < kSortItems; ++it) {
-    if (dg[it] < kRadix) {
-      const int64_t pos = (int64_t)base[dg[it]] + whist[warp][dg[it]] + rank[it];
-      keys_out[pos] = k[it];
-      vals_out[pos] = v[it];
+    for (int i = 0; i < kRadix / 32; ++i) {
+      v[i] = dstart[lane * (kRadix / 32) + i];
+      s += v[i];
     }
+    int incl = s;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    int run = incl - s;
+#pragma unroll
+    for (int i = 0; i < kRadix / 32; ++i) {
+      dstart[lane * (kRadix / 32) + i] = run;
+      run += v[i];
+    }
+  }
+  __syncthreads();
+  for (int j = threadIdx.x; j < cnt; j += kSortThreads) {
+    const int w = j / kWarpSlice;
+    const int d = (int)((tkey[j] >> shift) & (kRadix - 1));
+    const int p = dstart[d] + whist[w][d] + srank[j];
+    skey[p] = tkey[j];
+    sval[p] = tval[j];
+    if (kTwo) sval2[p] = tval2[j];
+  }
+  __syncthreads();
+  for (int p = threadIdx.x; p < cnt; p += kSortThreads) {
+    const uint32_t k = skey[p];
+    const int d = (int)((k >> shift) & (kRadix - 1));
+    const int64_t pos = (int64_t)gbase[d] + (p - dstart[d]);
+    keys_out[pos] = k;
+    vals_out[pos] = sval[p];
+    if (kTwo) vals2_out[pos] = sval2[p];
   }
 }
 
 struct SortBuffers {
   uint32_t* keys[2];
   uint32_t* vals[2];
+  uint32_t* vals2[2];  // second payload (carried so the finish passes read sequentially)
   int32_t* hist;
   void* scan_scratch;
 };
 
 static int64_t sort_tiles(int64_t n) { return std::max<int64_t>(1, ceil_div(n, kSortTile)); }
 
-// Sorts keys[0]/vals[0] by the low `bits` key bits; returns the buffer index holding the result.
-static hg_status radix_sort(SortBuffers& b, int64_t n, int bits, cudaStream_t s, int* result) {
+// Sorts keys[0]/vals[0] (and the second payload, first read from vals2_src) by the low `bits` key
+// bits; returns the buffer index holding the result.
+static hg_status radix_sort(SortBuffers& b, int64_t n, int bits, const uint32_t* vals2_src, cudaStream_t s,
+                            int* result) {
   int cur = 0;
   const int64_t tiles = sort_tiles(n);
+  const uint32_t* v2 = vals2_src;
   for (int shift = 0; shift < bits; shift += 8) {
     HG_TRY(launch("radix_hist", radix_hist, dim3((unsigned)tiles), dim3(kSortThreads), 0, s,
                   (const uint32_t*)b.keys[cur], n, shift, b.hist, tiles));
     HG_TRY(exclusive_scan(b.hist, b.hist, tiles * kRadix, b.scan_scratch, s));
-    HG_TRY(launch("radix_scatter", radix_scatter, dim3((unsigned)tiles), dim3(kSortThreads), 0, s,
-                  (const uint32_t*)b.keys[cur], (const uint32_t*)b.vals[cur], b.keys[cur ^ 1],
-                  b.vals[cur ^ 1], n, shift, (const int32_t*)b.hist, tiles));
+    HG_TRY(launch("radix_scatter", radix_scatter<true>, dim3((unsigned)tiles), dim3(kSortThreads), 0, s,
+                  (const uint32_t*)b.keys[cur], (const uint32_t*)b.vals[cur], v2, b.keys[cur ^ 1], b.vals[cur ^ 1],
+                  b.vals2[cur ^ 1], n, shift, (const int32_t*)b.hist, tiles));
+    v2 = b.vals2[cur ^ 1];
     cur ^= 1;
   }
   *result = cur;
@@ -255,32 +305,37 @@ __global__ void row_ptr_from_keys(const uint32_t* __restrict__ keys, int64_t n, 
   }
 }
 
-__global__ void csr_finish(const uint32_t* __restrict__ eid_sorted, const int32_t* __restrict__ ptr,
-                           int64_t rows, int64_t E, const int32_t* __restrict__ src,
-                           int32_t* __restrict__ col, int32_t* __restrict__ eid, int32_t* __restrict__ invalid) {
+// CSR arrays from the sorted (row key, edge id, source id) triples.
+__global__ void csr_finish(const uint32_t* __restrict__ eid_sorted, const uint32_t* __restrict__ src_sorted,
+                           const int32_t* __restrict__ ptr, int64_t rows, int64_t E, int32_t* __restrict__ col,
+                           int32_t* __restrict__ eid, int32_t* __restrict__ invalid) {
   const int64_t nv = ptr[rows];
   if (blockIdx.x == 0 && threadIdx.x == 0) *invalid = (int32_t)(E - nv);
   for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < nv;
        p += (int64_t)gridDim.x * blockDim.x) {
-    const uint32_t e = eid_sorted[p];
-    eid[p] = (int32_t)e;
-    col[p] = src[e];
+    eid[p] = (int32_t)eid_sorted[p];
+    col[p] = (int32_t)src_sorted[p];
   }
 }
 
-__global__ void csc_finish(const uint32_t* __restrict__ eid_sorted, const int32_t* __restrict__ cptr,
-                           int64_t crows, const int32_t* __restrict__ dst, const int32_t* __restrict__ rel,
+// CSC arrays from the sorted (row key, edge id, destination id) triples; the relation is read off
+// the key, 1/deg_r(destination) from the CSR row pointers.
+__global__ void csc_finish(const uint32_t* __restrict__ key_sorted, const uint32_t* __restrict__ eid_sorted,
+                           const uint32_t* __restrict__ dst_sorted, const int32_t* __restrict__ cptr, int64_t crows,
                            GraphMeta m, const int32_t* __restrict__ csr_ptr, int32_t* __restrict__ ccol,
                            int32_t* __restrict__ ceid, float* __restrict__ coef) {
   const int64_t nv = cptr[crows];
   for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < nv;
        p += (int64_t)gridDim.x * blockDim.x) {
-    const uint32_t e = eid_sorted[p];
-    const int r = rel[e];
-    const int32_t j = dst[e];
+    const int64_t key = key_sorted[p];
+    int r = 0;
+#pragma unroll
+    for (int k = 1; k < kMaxRels; ++k)
+      if (k < m.num_rels && key >= m.csc_base[k]) r = k;
+    const int32_t j = (int32_t)dst_sorted[p];
     const int64_t row = m.row_base[r] + (j - m.type_off[m.rel_dst[r]]);
     const int deg = csr_ptr[row + 1] - csr_ptr[row];
-    ceid[p] = (int32_t)e;
+    ceid[p] = (int32_t)eid_sorted[p];
     ccol[p] = j;
     coef[p] = __fdiv_rn(1.0f, (float)deg);
   }
@@ -331,6 +386,7 @@ static size_t carve_graph(void* ws, int64_t E, int64_t rows, int64_t crows, Grap
   for (int i = 0; i < 2; ++i) {
     L->sort.keys[i] = c.take<uint32_t>(Ea);
     L->sort.vals[i] = c.take<uint32_t>(Ea);
+    L->sort.vals2[i] = c.take<uint32_t>(Ea);
   }
   const int64_t hist_n = sort_tiles(E) * kRadix;
   L->sort.hist = c.take<int32_t>(hist_n + 1);
@@ -446,20 +502,22 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
     // CSR by destination
     HG_TRY(launch("edge_keys", edge_keys, dim3(g), dim3(256), 0, s, src, dst, rel, E, m, 1, rows, L.sort.keys[0],
                   L.sort.vals[0]));
-    HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)rows), s, &res));
+    HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)rows), (const uint32_t*)src, s, &res));
     HG_TRY(launch("row_ptr_from_keys", row_ptr_from_keys, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[res],
                   E, rows, L.csr_ptr));
-    HG_TRY(launch("csr_finish", csr_finish, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.vals[res],
-                  (const int32_t*)L.csr_ptr, rows, E, src, L.csr_col, L.csr_eid, L.invalid));
+    const uint32_t* src_sorted = res == 0 && bit_width((uint64_t)rows) == 0 ? (const uint32_t*)src : L.sort.vals2[res];
+    HG_TRY(launch("csr_finish", csr_finish, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.vals[res], src_sorted,
+                  (const int32_t*)L.csr_ptr, rows, E, L.csr_col, L.csr_eid, L.invalid));
     // CSC by source
     HG_TRY(launch("edge_keys", edge_keys, dim3(g), dim3(256), 0, s, src, dst, rel, E, m, 0, crows, L.sort.keys[0],
                   L.sort.vals[0]));
-    HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)crows), s, &res));
+    HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)crows), (const uint32_t*)dst, s, &res));
     HG_TRY(launch("row_ptr_from_keys", row_ptr_from_keys, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[res],
                   E, crows, L.csc_ptr));
-    HG_TRY(launch("csc_finish", csc_finish, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.vals[res],
-                  (const int32_t*)L.csc_ptr, crows, dst, rel, m, (const int32_t*)L.csr_ptr, L.csc_col, L.csc_eid,
-                  L.csc_coef));
+    const uint32_t* dst_sorted = res == 0 && bit_width((uint64_t)crows) == 0 ? (const uint32_t*)dst : L.sort.vals2[res];
+    HG_TRY(launch("csc_finish", csc_finish, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[res],
+                  (const uint32_t*)L.sort.vals[res], dst_sorted, (const int32_t*)L.csc_ptr, crows, m,
+                  (const int32_t*)L.csr_ptr, L.csc_col, L.csc_eid, L.csc_coef));
   }
   // chunk tables for rows above the hub degree
   HG_TRY(launch("chunk_counts", chunk_counts, dim3(grid_for(rows)), dim3(256), 0, s,

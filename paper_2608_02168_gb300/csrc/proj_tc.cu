@@ -36,10 +36,14 @@ constexpr int kATile = kTileRows * 128;  // 128 rows x 64 bf16
 
 template <int D>
 struct FwdCfg {
-  static constexpr int kStages = D == 64 ? 4 : 3;
+  static constexpr int kStages = D == 64 ? 3 : 2;
   static constexpr int kB = D * 128;  // D rows x 64 bf16
   static constexpr int kStage = kATile + kB;
-  static constexpr int kSmem = kStages * kStage + 256 + 1024;
+  // The H_in tile (residual) is fetched by TMA at the start, in parallel with the main loop, where
+  // it still leaves room for two CTAs per SM; at D = 256 the epilogue reads H_in from global memory.
+  static constexpr bool kHTile = D <= 128;
+  static constexpr int kH = kHTile ? kTileRows * D * 2 : 0;
+  static constexpr int kSmem = kStages * kStage + kH + 256 + 1024;
   static constexpr int kTmemCols = D < 32 ? 32 : D;
 };
 
@@ -68,18 +72,21 @@ __device__ __forceinline__ void store16_bf16(__nv_bfloat16* p, const float* v) {
 // ---------------------------------------------------------------------------------------------
 
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1) proj_fwd_tc(const __grid_constant__ CUtensorMap tm_M,
-                                                          const __grid_constant__ CUtensorMap tm_Vt, TcFwdArgs a) {
+__global__ void __launch_bounds__(kThreads, 2) proj_fwd_tc(const __grid_constant__ CUtensorMap tm_M,
+                                                          const __grid_constant__ CUtensorMap tm_Vt,
+                                                          const __grid_constant__ CUtensorMap tm_H, TcFwdArgs a) {
   using C = FwdCfg<D>;
   constexpr int S = C::kStages;
   constexpr int KC = D / 64;  // 64-wide K chunks per D
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  uint8_t* stage = smem;  // S x (A | B)
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S * C::kStage);
+  uint8_t* stage = smem;                   // S x (A | B)
+  uint8_t* htile = smem + S * C::kStage;   // KC x 16 KB, 128B-swizzled rows
+  uint64_t* full = reinterpret_cast<uint64_t*>(htile + C::kH);
   uint64_t* empty = full + S;
   uint64_t* accb = empty + S;
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(accb + 1);
+  uint64_t* hbar = accb + 1;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(hbar + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t m0 = (int64_t)blockIdx.x * kTileRows;
@@ -89,9 +96,15 @@ __global__ void __launch_bounds__(kThreads, 1) proj_fwd_tc(const __grid_constant
       mbar_init(&empty[s], 1);
     }
     mbar_init(accb, 1);
+    mbar_init(hbar, 1);
     fence_mbar_init();
     prefetch_tmap(&tm_M);
     prefetch_tmap(&tm_Vt);
+    if constexpr (C::kHTile) {
+      prefetch_tmap(&tm_H);
+      mbar_expect_tx(hbar, C::kH);
+      for (int kc = 0; kc < KC; ++kc) tma_load_2d(htile + kc * kATile, &tm_H, kc * 64, (int)m0, hbar);
+    }
   }
   if (warp == 0) tmem_alloc(tslot, C::kTmemCols);
   fence_before_sync();
@@ -141,6 +154,9 @@ __global__ void __launch_bounds__(kThreads, 1) proj_fwd_tc(const __grid_constant
   const int64_t node = a.off + (live ? m : 0);
   const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
   if (!mbar_wait(accb, 0)) atomicOr(a.status, kErrTimeout);
+  if constexpr (C::kHTile) {
+    if (!mbar_wait(hbar, 0)) atomicOr(a.status, kErrTimeout);
+  }
   fence_after_sync();
   // ---- epilogue: bias, activation, residual, LayerNorm
   auto u16 = [&](int c, float* u) {  // stored pre-activation of columns c .. c+15
@@ -155,48 +171,23 @@ __global__ void __launch_bounds__(kThreads, 1) proj_fwd_tc(const __grid_constant
 #pragma unroll
     for (int i = 0; i < 16; ++i) u[i] = __bfloat162float(__float2bfloat16_rn(u[i] + bb[i]));
   };
-  const __nv_bfloat16* hrow = a.H_in + node * D;
+  // three passes over TMEM and the shared H_in tile (row sum, centred sum of squares, output)
+  auto h16 = [&](int c, float* h) {  // residual row, columns c .. c+15
+    if constexpr (C::kHTile) {  // from the 128B-swizzled tile
+      const uint8_t* t = htile + (c >> 6) * kATile;
+      const uint32_t cb = (uint32_t)(c & 63) * 2;
+      unpack(*reinterpret_cast<const uint4*>(t + sw128_offset(row, cb)), h, __nv_bfloat16());
+      unpack(*reinterpret_cast<const uint4*>(t + sw128_offset(row, cb + 16)), h + 8, __nv_bfloat16());
+    } else {
+      load16_bf16(a.H_in + node * D + c, h);
+    }
+  };
   float sum = 0.f;
-  if constexpr (D <= 128) {
-    float y[D];
-#pragma unroll
-    for (int c = 0; c < D; c += 16) {
-      float u[16], h[16];
-      u16(c, u);
-      load16_bf16(hrow + c, h);
-      if (live) store16_bf16(a.U + node * D + c, u);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        y[c + i] = act_apply(u[i], a.act) + h[i];
-        sum += y[c + i];
-      }
-    }
-    if (a.ln) {
-      const float mean = sum * (1.f / D);
-      float q = 0.f;
-#pragma unroll
-      for (int i = 0; i < D; ++i) q += (y[i] - mean) * (y[i] - mean);
-      const float rstd = rsqrtf(q * (1.f / D) + a.eps);
-#pragma unroll
-      for (int c = 0; c < D; c += 16) {
-        float g[16], be[16], o[16];
-        load16_bf16(a.gamma + c, g);
-        load16_bf16(a.beta + c, be);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) o[i] = (y[c + i] - mean) * rstd * g[i] + be[i];
-        if (live) store16_bf16(a.H_out + node * D + c, o);
-      }
-      if (live) a.stats[node] = make_float2(mean, rstd);
-    } else if (live) {
-#pragma unroll
-      for (int c = 0; c < D; c += 16) store16_bf16(a.H_out + node * D + c, y + c);
-    }
-  } else {
-    // wide rows: three passes over TMEM / H_in instead of holding the row in registers
+  {
     auto y16 = [&](int c, float* y) {
       float u[16], h[16];
       u16(c, u);
-      load16_bf16(hrow + c, h);
+      h16(c, h);
 #pragma unroll
       for (int i = 0; i < 16; ++i) y[i] = act_apply(u[i], a.act) + h[i];
     };
@@ -204,7 +195,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_fwd_tc(const __grid_constant
     for (int c = 0; c < D; c += 16) {
       float u[16], h[16], y[16];
       u16(c, u);
-      load16_bf16(hrow + c, h);
+      h16(c, h);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
         y[i] = act_apply(u[i], a.act) + h[i];
@@ -651,11 +642,16 @@ template <int D>
 static hg_status tc_fwd_t(const TcFwdArgs& a, const void* M, int64_t m_rows, const void* Vt, int num_rels,
                           cudaStream_t s) {
   HG_TRY(smem_attr_once<D>());
-  CUtensorMap tm_M, tm_V;
+  CUtensorMap tm_M, tm_V, tm_H;
   HG_TRY(make_tmap_bf16(&tm_M, M, (uint64_t)std::max<int64_t>(m_rows, 1), D, kTileRows));
   HG_TRY(make_tmap_bf16(&tm_V, Vt, (uint64_t)num_rels * D, D, D));
+  if (FwdCfg<D>::kHTile) {
+    HG_TRY(make_tmap_bf16(&tm_H, a.H_in + a.off * D, (uint64_t)a.n, D, kTileRows));
+  } else {
+    tm_H = tm_M;  // unused
+  }
   return launch("proj_fwd_tc", proj_fwd_tc<D>, dim3((unsigned)ceil_div(a.n, kTileRows)), dim3(kThreads),
-                FwdCfg<D>::kSmem, s, tm_M, tm_V, a);
+                FwdCfg<D>::kSmem, s, tm_M, tm_V, tm_H, a);
 }
 
 template <int D>

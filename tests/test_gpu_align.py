@@ -78,7 +78,7 @@ def align_gpu(hg, Ha, ia, Hb, ib, dt, lam, eps, dloss, n_dev_val=None, both=True
 
 
 @pytest.mark.parametrize("dt,d,n,N", [("f32", 64, 1000, 1300), ("bf16", 128, 5000, 7000), ("bf16", 256, 3000, 3100),
-                                      ("f32", 128, 70_001, 80_000)])
+                                      ("bf16", 64, 2001, 2600), ("f32", 128, 70_001, 80_000)])
 def test_align_matches_oracle(dt, d, n, N):
     need_gpu()
     hg = lib()
@@ -135,3 +135,25 @@ def test_align_device_count_detached_view_and_degenerate_sizes():
     # identical views: L_inv = 0
     loss, _, _, _, _ = align_gpu(hg, Ha, ia, Ha, ia, "f32", 2e-4, 1e-8, 1.0)
     assert abs(loss[1]) <= 1e-5 * 64
+
+
+@pytest.mark.parametrize("d", [64, 128, 256])
+def test_align_bf16_device_count_far_below_capacity(d):
+    """bf16 path with the live row count read from the device and far below the capacity (the
+    step passes one capacity for every subgraph): the row splits of the Gram products and the
+    persistent gradient CTAs follow the device count; strong decorrelation (lambda = 0.05) makes
+    the Z (C - I) term of the gradient visible."""
+    need_gpu()
+    hg = lib()
+    n_live = 13_001 if d < 256 else 4_001
+    Ha, ia, Hb, ib = views(300 + d, 3 * n_live, n_live, d, "bf16")
+    lam, eps, dloss = 0.05, 1e-8, 0.5
+    loss, gA, gB, _, _ = align_gpu(hg, Ha, ia, Hb, ib, "bf16", lam, eps, dloss, n_dev_val=n_live,
+                                   n_max=5 * n_live, base=0.0)
+    ref = oracle.align_forward(Ha, ia, Hb, ib, lam, eps)
+    assert relerr(loss, ref) <= 1e-3, (loss, ref)
+    rA, rB = oracle.align_backward(Ha, ia, Hb, ib, lam, eps, dloss)
+    assert relerr(gA[ia], rA[ia]) <= TOL["bf16"], relerr(gA[ia], rA[ia])
+    assert relerr(gB[ib], rB[ib]) <= TOL["bf16"], relerr(gB[ib], rB[ib])
+    assert np.abs(gA[np.setdiff1d(np.arange(len(Ha)), ia)]).max() == 0
+    assert hg.hg_device_status() == 0
