@@ -143,7 +143,8 @@ def graph_stats(w) -> dict:
     offs = g["type_offsets"]
     N = int(offs[-1])
     src, dst, rel = g["src"].astype(np.int64), g["dst"].astype(np.int64), g["rel"]
-    st = dict(N=N, E=len(src), RR=0, CC=0, fwd=dict(E_nh=0, E_h=0, U_nh=0, U_h=0, chunks=0),
+    st = dict(N=N, E=len(src), RR=0, CC=0, n_ov=int(len(w.overlap_local)),
+              fwd=dict(E_nh=0, E_h=0, U_nh=0, U_h=0, chunks=0),
               bwd=dict(E_nh=0, E_h=0, U_nh=0, U_h=0, chunks=0), types=[], rels=[])
     for t in range(len(offs) - 1):
         st["types"].append(dict(n=int(offs[t + 1] - offs[t]), R=sum(1 for r in g["rels"] if r[1] == t)))
@@ -188,11 +189,24 @@ def kernel_models(st: dict, sp) -> dict:
     m["proj_fwd_simt"] = (L * fb, L * ff)
     m["proj_bwd_simt"] = (L * bb, L * bf)
     m["wgrad_partial"] = (L * 2 * row * (N + RR), L * 2 * d * d * (N + RR))
-    # tensor-core kernels: the same traffic and arithmetic, bound by HBM at these shapes
-    m["proj_fwd_tc"] = m["proj_fwd_simt"]
-    m["proj_bwd_tc"] = m["proj_bwd_simt"]
-    m["wgrad_tc"] = m["wgrad_partial"]
+    # tensor-core path (fused weights V_r = W_r W_agg): per node of type t with R relations into t
+    tf = tfl = lb = pb = pfl = 0
+    for t in st["types"]:
+        n, R = t["n"], t["R"]
+        tf += n * row * (R + 3) + 8 * n      # read M_r (R rows), H_in; write U, H_out; row statistics
+        tfl += 2 * n * d * d * R
+        lb += n * (5 * row + 8)              # read dH_out, U, H_in, statistics; write dY, dU
+        pb += n * row * (R + 1) + 4 * n * R  # read dU, degrees; write dM_r (R rows)
+        pfl += 2 * n * d * d * R
+    m["proj_fwd_tc"] = (L * tf, L * tfl)
+    m["ln_act_bwd"] = (L * lb, 0)
+    m["proj_bwd_tc"] = (L * pb, L * pfl)
+    m["wgrad_tc"] = (L * 2 * row * RR, L * 2 * d * d * RR)  # G_r = M_r^T dU: read both operands once
     m["radix_scatter"] = (2 * 3 * 4 * 4 * st["E"], 0)  # 2 layouts x 3 passes x (read+write of key+value)
+    no = st["n_ov"]
+    m["align_colstats"] = (3 * 2 * no * (row + 4), 0)        # 3 passes over both gathered views
+    m["align_gram_tc"] = (2 * no * (row + 4), 2 * 2 * no * d * d)
+    m["align_bwd_tc"] = (2 * no * (4 * row + 8), 2 * 2 * no * d * d)  # per view: H_a, H_b, dH read, dH write
     return m
 
 

@@ -34,17 +34,23 @@ constexpr int kThreads = 128;
 constexpr int kTileRows = 128;
 constexpr int kATile = kTileRows * 128;  // 128 rows x 64 bf16
 
+// Persistent forward: one CTA per SM, warp 0 loads (TMA), warp 1 issues the MMAs, warps 2-5 run
+// the epilogue; two TMEM accumulators and two residual tiles let the epilogue of one 128-row tile
+// overlap the loads and MMAs of the next.
 template <int D>
 struct FwdCfg {
-  static constexpr int kStages = D == 64 ? 3 : 2;
+  static constexpr int kStages = D == 256 ? 3 : 4;
   static constexpr int kB = D * 128;  // D rows x 64 bf16
   static constexpr int kStage = kATile + kB;
-  // The H_in tile (residual) is fetched by TMA at the start, in parallel with the main loop, where
-  // it still leaves room for two CTAs per SM; at D = 256 the epilogue reads H_in from global memory.
+  // The H_in tile (residual) is fetched by TMA, double-buffered, where shared memory allows it; at
+  // D = 256 the epilogue reads H_in from global memory.
   static constexpr bool kHTile = D <= 128;
   static constexpr int kH = kHTile ? kTileRows * D * 2 : 0;
-  static constexpr int kSmem = kStages * kStage + kH + 256 + 1024;
-  static constexpr int kTmemCols = D < 32 ? 32 : D;
+  static constexpr int kParams = 3 * D * 4;  // bias, gamma, beta in fp32
+  static constexpr int kSmem = kStages * kStage + 2 * kH + kParams + 512 + 1024;
+  static constexpr int kAccCols = D < 32 ? 32 : D;
+  static constexpr int kTmemCols = 2 * kAccCols;
+  static constexpr int kThreads = 192;
 };
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
@@ -72,165 +78,239 @@ __device__ __forceinline__ void store16_bf16(__nv_bfloat16* p, const float* v) {
 // ---------------------------------------------------------------------------------------------
 
 template <int D>
-__global__ void __launch_bounds__(kThreads, 2) proj_fwd_tc(const __grid_constant__ CUtensorMap tm_M,
-                                                          const __grid_constant__ CUtensorMap tm_Vt,
-                                                          const __grid_constant__ CUtensorMap tm_H, TcFwdArgs a) {
+__global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
+    proj_fwd_tc(const __grid_constant__ CUtensorMap tm_M, const __grid_constant__ CUtensorMap tm_Vt,
+                const __grid_constant__ CUtensorMap tm_H, TcFwdArgs a) {
   using C = FwdCfg<D>;
   constexpr int S = C::kStages;
   constexpr int KC = D / 64;  // 64-wide K chunks per D
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  uint8_t* stage = smem;                   // S x (A | B)
-  uint8_t* htile = smem + S * C::kStage;   // KC x 16 KB, 128B-swizzled rows
-  uint64_t* full = reinterpret_cast<uint64_t*>(htile + C::kH);
+  uint8_t* stage = smem;                  // S x (A | B)
+  uint8_t* htile = smem + S * C::kStage;  // 2 x KC x 16 KB, 128B-swizzled rows
+  float* params = reinterpret_cast<float*>(htile + 2 * C::kH);  // [3][D]: b, gamma, beta
+  uint64_t* full = reinterpret_cast<uint64_t*>(params + 3 * D);
   uint64_t* empty = full + S;
-  uint64_t* accb = empty + S;
-  uint64_t* hbar = accb + 1;
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(hbar + 1);
+  uint64_t* acc_full = empty + S;   // [2] MMA -> epilogue
+  uint64_t* acc_empty = acc_full + 2;  // [2] epilogue -> MMA
+  uint64_t* h_full = acc_empty + 2;    // [2] TMA -> epilogue
+  uint64_t* h_empty = h_full + 2;      // [2] epilogue -> TMA
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(h_empty + 2);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t m0 = (int64_t)blockIdx.x * kTileRows;
+  const int64_t ntiles = (a.n + kTileRows - 1) / kTileRows;
+  const int CT = a.nrel * KC;
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    mbar_init(accb, 1);
-    mbar_init(hbar, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], kTileRows);
+      mbar_init(&h_full[b], 1);
+      mbar_init(&h_empty[b], kTileRows);
+    }
     fence_mbar_init();
     prefetch_tmap(&tm_M);
     prefetch_tmap(&tm_Vt);
-    if constexpr (C::kHTile) {
-      prefetch_tmap(&tm_H);
-      mbar_expect_tx(hbar, C::kH);
-      for (int kc = 0; kc < KC; ++kc) tma_load_2d(htile + kc * kATile, &tm_H, kc * 64, (int)m0, hbar);
-    }
+    if (C::kHTile) prefetch_tmap(&tm_H);
   }
-  if (warp == 0) tmem_alloc(tslot, C::kTmemCols);
+  if (warp == 1) tmem_alloc(tslot, C::kTmemCols);
   fence_before_sync();
   __syncthreads();
   fence_after_sync();
   const uint32_t tmem = *tslot;
-  const int CT = a.nrel * KC;
-  const uint32_t idesc = idesc_bf16(128, D, false, false);
 
-  // ---- U = sum_r M_r V_r
   if (warp == 0) {
+    // ---- TMA producer
     if (lane == 0) {
-      auto issue_load = [&](int g) {
-        const int s = g % S;
-        uint8_t* A = stage + s * C::kStage;
-        const int r = g / KC, kc = g % KC;
-        mbar_expect_tx(&full[s], kATile + C::kB);
-        tma_load_2d(A, &tm_M, kc * 64, (int)(a.mrow0[r] + m0), &full[s]);
-        tma_load_2d(A + kATile, &tm_Vt, kc * 64, a.rel[r] * D, &full[s]);
-      };
       bool ok = true;
-      for (int g = 0; g < S && g < CT; ++g) issue_load(g);
-      for (int g = 0; g < CT && ok; ++g) {
-        const int s = g % S;
-        ok = mbar_wait(&full[s], (g / S) & 1);
-        if (!ok) break;
-        fence_after_sync();
-        const uint32_t A = smem_u32(stage + s * C::kStage);
-#pragma unroll
-        for (int ks = 0; ks < 4; ++ks)
-          mma_bf16(tmem, desc_sw128(A + ks * 32, 16, 1024), desc_sw128(A + kATile + ks * 32, 16, 1024), idesc,
-                   (g > 0 || ks > 0) ? 1u : 0u);
-        mma_commit(&empty[s]);
-        if (g + S < CT) {
-          ok = mbar_wait(&empty[s], (g / S) & 1);
-          if (ok) issue_load(g + S);
+      uint32_t g = 0;
+      int it = 0;
+      for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
+        const int64_t m0 = tile * kTileRows;
+        const int b = it & 1;
+        if (C::kHTile) {
+          if (it >= 2) ok = mbar_wait(&h_empty[b], ((it >> 1) - 1) & 1);
+          if (!ok) break;
+          mbar_expect_tx(&h_full[b], C::kH);
+          for (int kc = 0; kc < KC; ++kc) tma_load_2d(htile + b * C::kH + kc * kATile, &tm_H, kc * 64, (int)m0, &h_full[b]);
+        }
+        for (int j = 0; j < CT && ok; ++j, ++g) {
+          const uint32_t s = g % S;
+          if (g >= (uint32_t)S) ok = mbar_wait(&empty[s], ((g / S) - 1) & 1);
+          if (!ok) break;
+          uint8_t* A = stage + s * C::kStage;
+          const int r = j / KC, kc = j % KC;
+          mbar_expect_tx(&full[s], kATile + C::kB);
+          tma_load_2d(A, &tm_M, kc * 64, (int)(a.mrow0[r] + m0), &full[s]);
+          tma_load_2d(A + kATile, &tm_Vt, kc * 64, a.rel[r] * D, &full[s]);
         }
       }
       if (!ok) atomicOr(a.status, kErrTimeout);
-      mma_commit(accb);
     }
     __syncwarp();
-  }
-  const int row = warp * 32 + lane;
-  const int64_t m = m0 + row;
-  const bool live = m < a.n;
-  const int64_t node = a.off + (live ? m : 0);
-  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
-  if (!mbar_wait(accb, 0)) atomicOr(a.status, kErrTimeout);
-  if constexpr (C::kHTile) {
-    if (!mbar_wait(hbar, 0)) atomicOr(a.status, kErrTimeout);
-  }
-  fence_after_sync();
-  // ---- epilogue: bias, activation, residual, LayerNorm
-  auto u16 = [&](int c, float* u) {  // stored pre-activation of columns c .. c+15
-    float bb[16];
-    if (CT > 0) {
-      tmem_ld16(trow + c, u);
-    } else {
+  } else if (warp == 1) {
+    // ---- MMA issuer: U_tile = sum_r M_r V_r into accumulator (it & 1)
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16(128, D, false, false);
+      bool ok = true;
+      uint32_t g = 0;
+      int it = 0;
+      for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
+        const int b = it & 1;
+        if (it >= 2) ok = mbar_wait(&acc_empty[b], ((it >> 1) - 1) & 1);
+        if (!ok) break;
+        fence_after_sync();
+        const uint32_t acc = tmem + b * C::kAccCols;
+        for (int j = 0; j < CT && ok; ++j, ++g) {
+          const uint32_t s = g % S;
+          ok = mbar_wait(&full[s], (g / S) & 1);
+          if (!ok) break;
+          fence_after_sync();
+          const uint32_t A = smem_u32(stage + s * C::kStage);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) u[i] = 0.f;
-    }
-    load16_bf16(a.b + c, bb);
-#pragma unroll
-    for (int i = 0; i < 16; ++i) u[i] = __bfloat162float(__float2bfloat16_rn(u[i] + bb[i]));
-  };
-  // three passes over TMEM and the shared H_in tile (row sum, centred sum of squares, output)
-  auto h16 = [&](int c, float* h) {  // residual row, columns c .. c+15
-    if constexpr (C::kHTile) {  // from the 128B-swizzled tile
-      const uint8_t* t = htile + (c >> 6) * kATile;
-      const uint32_t cb = (uint32_t)(c & 63) * 2;
-      unpack(*reinterpret_cast<const uint4*>(t + sw128_offset(row, cb)), h, __nv_bfloat16());
-      unpack(*reinterpret_cast<const uint4*>(t + sw128_offset(row, cb + 16)), h + 8, __nv_bfloat16());
-    } else {
-      load16_bf16(a.H_in + node * D + c, h);
-    }
-  };
-  float sum = 0.f;
-  {
-    auto y16 = [&](int c, float* y) {
-      float u[16], h[16];
-      u16(c, u);
-      h16(c, h);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) y[i] = act_apply(u[i], a.act) + h[i];
-    };
-#pragma unroll 1
-    for (int c = 0; c < D; c += 16) {
-      float u[16], h[16], y[16];
-      u16(c, u);
-      h16(c, h);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        y[i] = act_apply(u[i], a.act) + h[i];
-        sum += y[i];
+          for (int ks = 0; ks < 4; ++ks)
+            mma_bf16(acc, desc_sw128(A + ks * 32, 16, 1024), desc_sw128(A + kATile + ks * 32, 16, 1024), idesc,
+                     (j > 0 || ks > 0) ? 1u : 0u);
+          mma_commit(&empty[s]);
+        }
+        mma_commit(&acc_full[b]);
       }
-      if (live) store16_bf16(a.U + node * D + c, u);
-      if (!a.ln && live) store16_bf16(a.H_out + node * D + c, y);
+      if (!ok) atomicOr(a.status, kErrTimeout);
     }
-    if (a.ln) {
-      const float mean = sum * (1.f / D);
-      float q = 0.f;
-#pragma unroll 1
-      for (int c = 0; c < D; c += 16) {
-        float y[16];
-        y16(c, y);
+    __syncwarp();
+  } else {
+    // ---- epilogue: bias, activation, residual, LayerNorm; warp w owns TMEM lanes 32 (w % 4) ..
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    const float* pb = params;
+    const float* pgm = params + D;
+    const float* pbe = params + 2 * D;
+    for (int c = threadIdx.x - 64; c < D; c += kTileRows) {
+      params[c] = __bfloat162float(a.b[c]);
+      params[D + c] = a.ln ? __bfloat162float(a.gamma[c]) : 1.f;
+      params[2 * D + c] = a.ln ? __bfloat162float(a.beta[c]) : 0.f;
+    }
+    asm volatile("bar.sync 1, 128;" ::: "memory");  // the four epilogue warps
+    bool ok = true;
+    int it = 0;
+    for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
+      const int b = it & 1;
+      const int64_t m = tile * kTileRows + row;
+      const bool live = m < a.n;
+      const int64_t node = a.off + (live ? m : 0);
+      ok = mbar_wait(&acc_full[b], (it >> 1) & 1);
+      if (ok && C::kHTile) ok = mbar_wait(&h_full[b], (it >> 1) & 1);
+      if (!ok) break;
+      fence_after_sync();
+      const uint32_t trow = tmem + b * C::kAccCols + ((uint32_t)(q * 32) << 16);
+      const uint8_t* ht = htile + b * C::kH;
+      // U = bf16(acc + b) for columns c .. c+15, stored; returned unpacked in u
+      auto u16 = [&](int c, float* u, bool store) {
+        if (CT > 0) {
+          tmem_ld16(trow + c, u);
+        } else {
 #pragma unroll
-        for (int i = 0; i < 16; ++i) q += (y[i] - mean) * (y[i] - mean);
-      }
-      const float rstd = rsqrtf(q * (1.f / D) + a.eps);
-#pragma unroll 1
-      for (int c = 0; c < D; c += 16) {
-        float y[16], g[16], be[16], o[16];
-        y16(c, y);
-        load16_bf16(a.gamma + c, g);
-        load16_bf16(a.beta + c, be);
+          for (int i = 0; i < 16; ++i) u[i] = 0.f;
+        }
+        uint32_t up[8];
 #pragma unroll
-        for (int i = 0; i < 16; ++i) o[i] = (y[i] - mean) * rstd * g[i] + be[i];
+        for (int i = 0; i < 8; ++i) up[i] = pack_bf16x2(u[2 * i] + pb[c + 2 * i], u[2 * i + 1] + pb[c + 2 * i + 1]);
+        if (store && live) {
+          st16(a.U + node * D + c, make_uint4(up[0], up[1], up[2], up[3]));
+          st16(a.U + node * D + c + 8, make_uint4(up[4], up[5], up[6], up[7]));
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          u[2 * i] = __uint_as_float(up[i] << 16);
+          u[2 * i + 1] = __uint_as_float(up[i] & 0xFFFF0000u);
+        }
+      };
+      auto h16 = [&](int c, float* h) {  // residual row, columns c .. c+15
+        if constexpr (C::kHTile) {  // from the 128B-swizzled tile
+          const uint8_t* t = ht + (c >> 6) * kATile;
+          const uint32_t cb = (uint32_t)(c & 63) * 2;
+          unpack(*reinterpret_cast<const uint4*>(t + sw128_offset(row, cb)), h, __nv_bfloat16());
+          unpack(*reinterpret_cast<const uint4*>(t + sw128_offset(row, cb + 16)), h + 8, __nv_bfloat16());
+        } else {
+          load16_bf16(a.H_in + node * D + c, h);
+        }
+      };
+      auto out16 = [&](int c, const float* y, float mean, float rstd) {  // H_out columns c .. c+15
+        float o[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) o[i] = a.ln ? (y[i] - mean) * rstd * pgm[c + i] + pbe[c + i] : y[i];
         if (live) store16_bf16(a.H_out + node * D + c, o);
+      };
+      if constexpr (D <= 128) {
+        // the whole row in registers: one pass over TMEM
+        float y[D];
+        float sum = 0.f;
+#pragma unroll
+        for (int c = 0; c < D; c += 16) {
+          float u[16], h[16];
+          u16(c, u, true);
+          h16(c, h);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            y[c + i] = act_apply(u[i], a.act) + h[i];
+            sum += y[c + i];
+          }
+        }
+        const float mean = sum * (1.f / D);
+        float qq = 0.f;
+#pragma unroll
+        for (int i = 0; i < D; ++i) qq += (y[i] - mean) * (y[i] - mean);
+        const float rstd = rsqrtf(qq * (1.f / D) + a.eps);
+#pragma unroll
+        for (int c = 0; c < D; c += 16) out16(c, y + c, mean, rstd);
+        if (a.ln && live) a.stats[node] = make_float2(mean, rstd);
+      } else {
+        // three passes over TMEM and the residual (row sum, centred sum of squares, output)
+        auto y16 = [&](int c, float* y, bool store) {
+          float u[16], h[16];
+          u16(c, u, store);
+          h16(c, h);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) y[i] = act_apply(u[i], a.act) + h[i];
+        };
+        float sum = 0.f;
+#pragma unroll 1
+        for (int c = 0; c < D; c += 16) {
+          float y[16];
+          y16(c, y, true);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) sum += y[i];
+        }
+        const float mean = sum * (1.f / D);
+        float qq = 0.f;
+#pragma unroll 1
+        for (int c = 0; c < D; c += 16) {
+          float y[16];
+          y16(c, y, false);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) qq += (y[i] - mean) * (y[i] - mean);
+        }
+        const float rstd = rsqrtf(qq * (1.f / D) + a.eps);
+#pragma unroll 1
+        for (int c = 0; c < D; c += 16) {
+          float y[16];
+          y16(c, y, false);
+          out16(c, y, mean, rstd);
+        }
+        if (a.ln && live) a.stats[node] = make_float2(mean, rstd);
       }
-      if (live) a.stats[node] = make_float2(mean, rstd);
+      fence_before_sync();
+      mbar_arrive(&acc_empty[b]);
+      if (C::kHTile) mbar_arrive(&h_empty[b]);
     }
+    if (!ok) atomicOr(a.status, kErrTimeout);
   }
   fence_before_sync();
   __syncthreads();
-  if (warp == 0) tmem_dealloc(tmem, C::kTmemCols);
+  if (warp == 1) tmem_dealloc(tmem, C::kTmemCols);
 }
 
 // Fused weights V_r = W_r W_agg[t_r] accumulated in fp64 (exact for bf16 factors of these sizes),
@@ -650,8 +730,12 @@ static hg_status tc_fwd_t(const TcFwdArgs& a, const void* M, int64_t m_rows, con
   } else {
     tm_H = tm_M;  // unused
   }
-  return launch("proj_fwd_tc", proj_fwd_tc<D>, dim3((unsigned)ceil_div(a.n, kTileRows)), dim3(kThreads),
-                FwdCfg<D>::kSmem, s, tm_M, tm_V, tm_H, a);
+  int sms = 0, dev = 0;
+  HG_CUDA(cudaGetDevice(&dev));
+  HG_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(a.n, kTileRows), sms));
+  return launch("proj_fwd_tc", proj_fwd_tc<D>, dim3(grid), dim3(FwdCfg<D>::kThreads), FwdCfg<D>::kSmem, s, tm_M,
+                tm_V, tm_H, a);
 }
 
 template <int D>
