@@ -169,32 +169,15 @@ __global__ void __launch_bounds__(256, 2) align_colstats(const T* __restrict__ H
   }
 }
 
-// out[q][c] from the block partials (summed in block order): MODE 0 -> mu = sum / n;
-// MODE 1 -> s = sqrt(sum / n + eps); MODE 2 -> the sums themselves.
-__global__ void align_colfinish(const float* __restrict__ part, int blocks, int q_count, int d,
-                                const int64_t* __restrict__ n_dev, int64_t n_max, int mode, float eps,
-                                float* __restrict__ out) {
+// In place over the column sums (reduced from the block partials by reduce_partials):
+// mode 0 -> mu = sum / n;  mode 1 -> s = sqrt(sum / n + eps).
+__global__ void align_colscale(float* __restrict__ v, int count, const int64_t* __restrict__ n_dev, int64_t n_max,
+                               int mode, float eps) {
   const int64_t n = count_of(n_dev, n_max);
   const int k = blockIdx.x * blockDim.x + threadIdx.x;
-  if (k >= q_count * d) return;
-  const int64_t stride = (int64_t)q_count * d;
-  float s = 0.f;
-  int b = 0;
-  for (; b + 4 <= blocks; b += 4) {
-    const float v0 = part[(b + 0) * stride + k], v1 = part[(b + 1) * stride + k];
-    const float v2 = part[(b + 2) * stride + k], v3 = part[(b + 3) * stride + k];
-    s += v0;
-    s += v1;
-    s += v2;
-    s += v3;
-  }
-  for (; b < blocks; ++b) s += part[b * stride + k];
-  if (mode == 2) {
-    out[k] = s;
-  } else {
-    const float m = n > 0 ? s / (float)n : 0.f;
-    out[k] = mode ? sqrtf(m + eps) : m;
-  }
+  if (k >= count) return;
+  const float m = n > 0 ? v[k] / (float)n : 0.f;
+  v[k] = mode ? sqrtf(m + eps) : m;
 }
 
 // Gram partials of the standardised rows on the CUDA cores (fp32 storage): part[split][view][d][d].
@@ -276,27 +259,45 @@ __global__ void align_gram_reduce(const float* __restrict__ part, int splits, in
   }
 }
 
-// One block: L_dec from C, L_inv from the column sums of (z_a - z_b)^2, loss = [L, L_inv, L_dec].
-__global__ void align_loss_finish(const float* __restrict__ C, int d, const float* __restrict__ cross,
-                                  const int64_t* __restrict__ n_dev, int64_t n_max, float lambda_n,
-                                  const int32_t* __restrict__ bad, float* __restrict__ loss) {
-  __shared__ float red[256];
-  __shared__ float red_inv[256];
+// One block of 1024 threads: L_dec from C, L_inv from the column sums of (z_a - z_b)^2,
+// loss = [L, L_inv, L_dec]; fixed-order warp and block sums.
+__global__ void __launch_bounds__(1024) align_loss_finish(const float* __restrict__ C, int d,
+                                                          const float* __restrict__ cross,
+                                                          const int64_t* __restrict__ n_dev, int64_t n_max,
+                                                          float lambda_n, const int32_t* __restrict__ bad,
+                                                          float* __restrict__ loss) {
+  __shared__ float red[2][32];
   const int64_t n = count_of(n_dev, n_max);
+  const int64_t dd = (int64_t)d * d;
   float s = 0.f, si = 0.f;
-  for (int64_t k = threadIdx.x; k < 2LL * d * d; k += blockDim.x) {
-    const int64_t e = k % ((int64_t)d * d);
-    const float c = C[k] - ((e / d) == (e % d) ? 1.f : 0.f);
-    s += c * c;
+  for (int64_t k4 = threadIdx.x; k4 < 2 * dd / 4; k4 += blockDim.x) {
+    const float4 v = reinterpret_cast<const float4*>(C)[k4];
+    const float x[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int64_t e = (4 * k4 + u) % dd;
+      const float c = x[u] - ((e / d) == (e % d) ? 1.f : 0.f);
+      s += c * c;
+    }
   }
   for (int c = threadIdx.x; c < d; c += blockDim.x) si += cross[kSumDiff2 * d + c];
-  red[threadIdx.x] = s;
-  red_inv[threadIdx.x] = si;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    s += __shfl_xor_sync(0xffffffffu, s, o);
+    si += __shfl_xor_sync(0xffffffffu, si, o);
+  }
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  if (lane == 0) {
+    red[0][w] = s;
+    red[1][w] = si;
+  }
   __syncthreads();
   if (threadIdx.x == 0) {
     float dec = 0.f, iv = 0.f;
-    for (int k = 0; k < (int)blockDim.x; ++k) dec += red[k];
-    for (int k = 0; k < (int)blockDim.x; ++k) iv += red_inv[k];
+    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) {
+      dec += red[0][k];
+      iv += red[1][k];
+    }
     if (n < 2) dec = iv = 0.f;
     if (*bad) dec = iv = __int_as_float(0x7fc00000);  // an overlap index outside its table: NaN loss
     loss[0] = iv + lambda_n * dec;
@@ -517,16 +518,17 @@ static hg_status align_loss_run(const AlignIn& in, float lambda_n, float eps, fl
   HG_CUDA(cudaMemsetAsync(L.bad, 0, sizeof(int32_t), s));
   HG_TRY(launch("align_colstats", align_colstats<T, D, 0>, dim3(blocks), dim3(256), 0, s, Ha, in.rows_a, in.ia, Hb,
                 in.rows_b, in.ib, in.n_max, in.n_dev, no_stats, L.part, L.bad));
-  HG_TRY(launch("align_colfinish", align_colfinish, dim3((unsigned)ceil_div(2 * D, 256)), dim3(256), 0, s,
-                (const float*)L.part, blocks, 2, D, in.n_dev, in.n_max, 0, 0.f, L.stats));
+  HG_TRY(reduce_partials(L.part, 2LL * D, blocks, 2LL * D, L.stats, L.rtmp, s));
+  HG_TRY(launch("align_colscale", align_colscale, dim3((unsigned)ceil_div(2 * D, 256)), dim3(256), 0, s, L.stats,
+                2 * D, in.n_dev, in.n_max, 0, 0.f));
   HG_TRY(launch("align_colstats", align_colstats<T, D, 1>, dim3(blocks), dim3(256), 0, s, Ha, in.rows_a, in.ia, Hb,
                 in.rows_b, in.ib, in.n_max, in.n_dev, (const float*)L.stats, L.part, L.bad));
-  HG_TRY(launch("align_colfinish", align_colfinish, dim3((unsigned)ceil_div(2 * D, 256)), dim3(256), 0, s,
-                (const float*)L.part, blocks, 2, D, in.n_dev, in.n_max, 1, eps, L.stats + 2 * D));
+  HG_TRY(reduce_partials(L.part, 2LL * D, blocks, 2LL * D, L.stats + 2 * D, L.rtmp, s));
+  HG_TRY(launch("align_colscale", align_colscale, dim3((unsigned)ceil_div(2 * D, 256)), dim3(256), 0, s,
+                L.stats + 2 * D, 2 * D, in.n_dev, in.n_max, 1, eps));
   HG_TRY(launch("align_colstats", align_colstats<T, D, 2>, dim3(blocks), dim3(256), 0, s, Ha, in.rows_a, in.ia, Hb,
                 in.rows_b, in.ib, in.n_max, in.n_dev, (const float*)L.stats, L.part, L.bad));
-  HG_TRY(launch("align_colfinish", align_colfinish, dim3((unsigned)ceil_div(kNumCross * D, 256)), dim3(256), 0, s,
-                (const float*)L.part, blocks, (int)kNumCross, D, in.n_dev, in.n_max, 2, 0.f, L.cross));
+  HG_TRY(reduce_partials(L.part, (int64_t)kNumCross * D, blocks, (int64_t)kNumCross * D, L.cross, L.rtmp, s));
   if constexpr (std::is_same<T, __nv_bfloat16>::value) {
     HG_TRY(align_gram_tc(D, in.Ha, in.rows_a, in.ia, in.Hb, in.rows_b, in.ib, in.n_max, in.n_dev, L.stats, splits,
                          L.gpart, s));
@@ -539,7 +541,7 @@ static hg_status align_loss_run(const AlignIn& in, float lambda_n, float eps, fl
   for (int v = 0; v < 2; ++v)
     HG_TRY(reduce_partials(L.gpart + (size_t)v * D * D, 2LL * D * D, splits, (int64_t)D * D, L.C + (size_t)v * D * D,
                            L.rtmp, s));
-  return launch("align_loss_finish", align_loss_finish, dim3(1), dim3(256), 0, s, (const float*)L.C, D,
+  return launch("align_loss_finish", align_loss_finish, dim3(1), dim3(1024), 0, s, (const float*)L.C, D,
                 (const float*)L.cross, in.n_dev, in.n_max, lambda_n, (const int32_t*)L.bad, loss);
 }
 

@@ -175,33 +175,52 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) tmem_dealloc(tmem, C::kTmemCols);
 }
 
-// Per view (blockIdx.x), per column c (thread): the column means of g and g x_hat, and the bf16
-// operand cmi[v][c][k] = C_v[k][c] - [k == c] of the gradient's product.
+// Grid (2 views, D / 32 column slices), 256 threads: per column c the means of g and g x_hat (the
+// sums over k split over the eight warps, k = w, w + 8, ..., then added in warp order), and the
+// slice's rows of the bf16 operand cmi[v][c][k] = C_v[k][c] - [k == c] of the gradient's product.
 template <int D>
-__global__ void align_bwd_coef(const float* __restrict__ Cm, const float* __restrict__ cross,
-                               const int64_t* __restrict__ n_dev, int64_t n_max, float lambda_n, float dloss,
-                               __nv_bfloat16* __restrict__ cmi, float* __restrict__ means) {
-  const int view = blockIdx.x, c = threadIdx.x;
+__global__ void __launch_bounds__(256) align_bwd_coef(const float* __restrict__ Cm, const float* __restrict__ cross,
+                                                      const int64_t* __restrict__ n_dev, int64_t n_max,
+                                                      float lambda_n, float dloss, __nv_bfloat16* __restrict__ cmi,
+                                                      float* __restrict__ means) {
+  __shared__ float red[2][8][33];
+  const int view = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int c = blockIdx.y * 32 + lane;
   const int64_t n = count_of(n_dev, n_max);
   const float* Cv = Cm + (int64_t)view * D * D;
   const float* Sv = cross + (view ? kSumZb : kSumZa) * D;
   float sp = 0.f, spz = 0.f;
-  for (int kk = 0; kk < D; ++kk) {
-    const float cm = Cv[(int64_t)kk * D + c] - (kk == c ? 1.f : 0.f);
+  for (int kk = w; kk < D; kk += 8) {
+    const float cv = Cv[(int64_t)kk * D + c];
+    const float cm = cv - (kk == c ? 1.f : 0.f);
     sp += Sv[kk] * cm;
-    spz += cm * Cv[(int64_t)kk * D + c];
+    spz += cm * cv;
   }
-  const float sign = view ? -1.f : 1.f;
-  const float dz = cross[kSumZa * D + c] - cross[kSumZb * D + c];
-  const float dzz = view ? cross[kSumZaZb * D + c] - cross[kSumZb2 * D + c]
-                         : cross[kSumZa2 * D + c] - cross[kSumZaZb * D + c];
-  const float sum_g = dloss * (sign * 2.f * dz + 4.f * lambda_n * sp);
-  const float sum_gz = dloss * (sign * 2.f * dzz + 4.f * lambda_n * spz);
-  const float rn = n > 0 ? 1.f / (float)n : 0.f;
-  means[(view * 2 + 0) * D + c] = (n > 0 ? rsqrtf((float)n) : 0.f) * sum_g * rn;
-  means[(view * 2 + 1) * D + c] = sum_gz * rn;
-  __nv_bfloat16* row = cmi + ((int64_t)view * D + c) * D;
-  for (int kk = 0; kk < D; ++kk) row[kk] = __float2bfloat16_rn(Cv[(int64_t)kk * D + c] - (kk == c ? 1.f : 0.f));
+  red[0][w][lane] = sp;
+  red[1][w][lane] = spz;
+  __syncthreads();
+  if (w == 0) {
+    sp = spz = 0.f;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      sp += red[0][k][lane];
+      spz += red[1][k][lane];
+    }
+    const float sign = view ? -1.f : 1.f;
+    const float dz = cross[kSumZa * D + c] - cross[kSumZb * D + c];
+    const float dzz = view ? cross[kSumZaZb * D + c] - cross[kSumZb2 * D + c]
+                           : cross[kSumZa2 * D + c] - cross[kSumZaZb * D + c];
+    const float sum_g = dloss * (sign * 2.f * dz + 4.f * lambda_n * sp);
+    const float sum_gz = dloss * (sign * 2.f * dzz + 4.f * lambda_n * spz);
+    const float rn = n > 0 ? 1.f / (float)n : 0.f;
+    means[(view * 2 + 0) * D + c] = (n > 0 ? rsqrtf((float)n) : 0.f) * sum_g * rn;
+    means[(view * 2 + 1) * D + c] = sum_gz * rn;
+  }
+  for (int e = threadIdx.x; e < 32 * D; e += blockDim.x) {  // rows c0 .. c0+31 of cmi[view]
+    const int cl = e / D, kk = e % D;
+    const int cc = blockIdx.y * 32 + cl;
+    cmi[((int64_t)view * D + cc) * D + kk] = __float2bfloat16_rn(Cv[(int64_t)kk * D + cc] - (kk == cc ? 1.f : 0.f));
+  }
 }
 
 template <int D>
@@ -423,7 +442,7 @@ hg_status bwd_t(const void* Ha, int64_t rows_a, const int32_t* ia, const void* H
                                  ABwdCfg<D>::kSmem));
     attr = true;
   }
-  HG_TRY(launch("align_bwd_coef", align_bwd_coef<D>, dim3(2), dim3(D), 0, s, Cm, cross, n_dev, n_max, lambda_n,
+  HG_TRY(launch("align_bwd_coef", align_bwd_coef<D>, dim3(2, D / 32), dim3(256), 0, s, Cm, cross, n_dev, n_max, lambda_n,
                 dloss, (__nv_bfloat16*)cmi, means));
   CUtensorMap tm;
   HG_TRY(make_tmap_bf16(&tm, cmi, (uint64_t)2 * D, D, D));

@@ -308,48 +308,37 @@ __global__ void __launch_bounds__(256) wgrad_partial(const T* __restrict__ X, in
   }
 }
 
-// out[i] = sum_{s < splits} part[s * stride + i], added in split order; the loads of eight splits
-// are issued together so the chain of dependent adds does not wait on memory latency.
-__global__ void reduce_splits(const float* __restrict__ part, int64_t stride, int splits, int64_t count,
-                              float* __restrict__ out) {
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < count; i += (int64_t)gridDim.x * blockDim.x) {
-    float s = 0.f;
-    int k = 0;
-    for (; k + 8 <= splits; k += 8) {
-      float v[8];
+// out[i] = sum over splits k of part[k * stride + i] in a fixed order: a block owns 32 consecutive
+// outputs (one per lane); warp w sums the splits k = w, w + kRedLanes, ... in ascending order, and the
+// kRedLanes warp sums are added in warp order.
+constexpr int kRedLanes = 32;
+__global__ void __launch_bounds__(32 * kRedLanes) reduce_lanes(const float* __restrict__ part, int64_t stride,
+                                                             int splits, int64_t count, float* __restrict__ out) {
+  __shared__ float red[kRedLanes][33];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int64_t i = (int64_t)blockIdx.x * 32 + lane;
+  float s = 0.f;
+  if (i < count) {
+    int k = w;
+    for (; k + 3 * kRedLanes < splits; k += 4 * kRedLanes) {
+      float v[4];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) v[u] = __ldg(part + (int64_t)(k + u) * stride + i);
+      for (int u = 0; u < 4; ++u) v[u] = __ldg(part + (int64_t)(k + u * kRedLanes) * stride + i);
 #pragma unroll
-      for (int u = 0; u < 8; ++u) s += v[u];
+      for (int u = 0; u < 4; ++u) s += v[u];
     }
-    for (; k < splits; ++k) s += __ldg(part + (int64_t)k * stride + i);
-    out[i] = s;
+    for (; k < splits; k += kRedLanes) s += __ldg(part + (int64_t)k * stride + i);
+  }
+  red[w][lane] = s;
+  __syncthreads();
+  if (w == 0 && i < count) {
+    float t = 0.f;
+#pragma unroll
+    for (int k = 0; k < kRedLanes; ++k) t += red[k][lane];
+    out[i] = t;
   }
 }
 
-// out[g * count + i] = sum over splits [g * kRedGroup, (g + 1) * kRedGroup) of part, in order.
-constexpr int kRedGroup = 64;
-__global__ void reduce_groups(const float* __restrict__ part, int64_t stride, int splits, int64_t count,
-                              float* __restrict__ out) {
-  const int groups = (splits + kRedGroup - 1) / kRedGroup;
-  const int64_t total = (int64_t)groups * count;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
-    const int g = (int)(e / count);
-    const int64_t i = e % count;
-    const int k0 = g * kRedGroup, k1 = min(splits, k0 + kRedGroup);
-    float s = 0.f;
-    int k = k0;
-    for (; k + 8 <= k1; k += 8) {
-      float v[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) v[u] = __ldg(part + (int64_t)(k + u) * stride + i);
-#pragma unroll
-      for (int u = 0; u < 8; ++u) s += v[u];
-    }
-    for (; k < k1; ++k) s += __ldg(part + (int64_t)k * stride + i);
-    out[e] = s;
-  }
-}
 
 template <typename T>
 __global__ void transpose_square(const T* __restrict__ W, T* __restrict__ Wt, int d, int count) {
@@ -442,29 +431,17 @@ hg_status transpose_weights(hg_dtype dt, int d, const void* W, void* Wt, int cou
   HG_DISPATCH_TD2(dt, d, transpose_t, W, Wt, count, s);
 }
 size_t reduce_tmp_floats(int splits, int64_t count) {
-  const int64_t g1 = (splits + kRedGroup - 1) / kRedGroup;
-  const int64_t g2 = (g1 + kRedGroup - 1) / kRedGroup;
-  return (size_t)(g1 + g2 + 2) * count;
+  (void)splits;
+  return (size_t)count;  // reduce_partials needs no temporaries; one slot keeps callers' layouts valid
 }
 
-// Fixed-order sum over `splits` partial arrays: groups of kRedGroup are summed level by level (each
-// level fully parallel) until at most kRedGroup remain, then the last level writes `out`.
+// Fixed-order sum over `splits` partial arrays in one pass (reduce_lanes).
 hg_status reduce_partials(const float* part, int64_t stride, int splits, int64_t count, float* out, float* tmp,
                           cudaStream_t s) {
-  const int64_t g1 = (splits + kRedGroup - 1) / kRedGroup;
-  float* buf[2] = {tmp, tmp + (g1 + 1) * count};
-  int which = 0;
-  while (splits > kRedGroup) {
-    const int groups = (splits + kRedGroup - 1) / kRedGroup;
-    HG_TRY(launch("reduce_groups", reduce_groups, dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div((int64_t)groups * count, 256), 152 * 16))),
-                  dim3(256), 0, s, part, stride, splits, count, buf[which]));
-    part = buf[which];
-    stride = count;
-    splits = groups;
-    which ^= 1;
-  }
-  return launch("reduce_splits", reduce_splits, dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(count, 256), 1024))),
-                dim3(256), 0, s, part, stride, splits, count, out);
+  (void)tmp;
+  if (count <= 0) return HG_OK;
+  return launch("reduce_lanes", reduce_lanes, dim3((unsigned)ceil_div(count, 32)), dim3(32 * kRedLanes), 0, s, part,
+                stride, splits, count, out);
 }
 
 }  // namespace hg

@@ -207,13 +207,16 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
       fence_after_sync();
       const uint32_t trow = tmem + b * C::kAccCols + ((uint32_t)(q * 32) << 16);
       const uint8_t* ht = htile + b * C::kH;
-      // U = bf16(acc + b) for columns c .. c+15, stored; returned unpacked in u
-      auto u16 = [&](int c, float* u, bool store) {
-        if (CT > 0) {
-          tmem_ld16(trow + c, u);
-        } else {
+      // U = bf16(acc + b) for columns c .. c+15 (acc already in u when preloaded), stored;
+      // returned unpacked in u
+      auto u16 = [&](int c, float* u, bool store, bool preloaded = false) {
+        if (!preloaded) {
+          if (CT > 0) {
+            tmem_ld16(trow + c, u);
+          } else {
 #pragma unroll
-          for (int i = 0; i < 16; ++i) u[i] = 0.f;
+            for (int i = 0; i < 16; ++i) u[i] = 0.f;
+          }
         }
         uint32_t up[8];
 #pragma unroll
@@ -249,14 +252,24 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
         float y[D];
         float sum = 0.f;
 #pragma unroll
-        for (int c = 0; c < D; c += 16) {
-          float u[16], h[16];
-          u16(c, u, true);
-          h16(c, h);
+        for (int c = 0; c < D; c += 32) {
+          float u[32];
+          if (CT > 0) {
+            tmem_ld32(trow + c, u);
+          } else {
 #pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            y[c + i] = act_apply(u[i], a.act) + h[i];
-            sum += y[c + i];
+            for (int i = 0; i < 32; ++i) u[i] = 0.f;
+          }
+#pragma unroll
+          for (int hh = 0; hh < 32; hh += 16) {
+            float h[16];
+            u16(c + hh, u + hh, true, true);
+            h16(c + hh, h);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              y[c + hh + i] = act_apply(u[hh + i], a.act) + h[i];
+              sum += y[c + hh + i];
+            }
           }
         }
         const float mean = sum * (1.f / D);
@@ -314,54 +327,103 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
 }
 
 // Fused weights V_r = W_r W_agg[t_r] accumulated in fp64 (exact for bf16 factors of these sizes),
-// rounded once to bf16; both V_r and its transpose are written.
+// rounded once to bf16; both V_r and its transpose are written.  Grid (D/32, D/32, relations): a
+// block computes a 32 x 32 tile from 32-wide K slices staged in shared memory; thread (ty, tx)
+// owns rows ty, ty + 8, ty + 16, ty + 24 of column tx.
 template <int D>
-__global__ void fuse_weights(const __nv_bfloat16* __restrict__ W_rel, const __nv_bfloat16* __restrict__ W_agg,
-                             RelDst rel_dst, int num_rels, __nv_bfloat16* __restrict__ V,
-                             __nv_bfloat16* __restrict__ Vt) {
-  const int64_t total = (int64_t)num_rels * D * D;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
-    const int r = (int)(e / (D * D));
-    const int i = (int)((e / D) % D), j = (int)(e % D);
-    const __nv_bfloat16* w = W_rel + (int64_t)r * D * D + (int64_t)i * D;
-    const __nv_bfloat16* g = W_agg + (int64_t)rel_dst.v[r] * D * D + j;
-    double acc = 0.0;
-    for (int k = 0; k < D; ++k) acc += (double)__bfloat162float(w[k]) * (double)__bfloat162float(g[(int64_t)k * D]);
-    const __nv_bfloat16 v = __float2bfloat16_rn(__double2float_rn(acc));
-    V[e] = v;
+__global__ void __launch_bounds__(256) fuse_weights(const __nv_bfloat16* __restrict__ W_rel,
+                                                    const __nv_bfloat16* __restrict__ W_agg, RelDst rel_dst,
+                                                    int num_rels, __nv_bfloat16* __restrict__ V,
+                                                    __nv_bfloat16* __restrict__ Vt) {
+  __shared__ double As[32][33];
+  __shared__ double Bs[32][33];
+  const int r = blockIdx.z, i0 = blockIdx.y * 32, j0 = blockIdx.x * 32;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  const __nv_bfloat16* W = W_rel + (int64_t)r * D * D;
+  const __nv_bfloat16* G = W_agg + (int64_t)rel_dst.v[r] * D * D;
+  double acc[4] = {0.0, 0.0, 0.0, 0.0};
+  for (int k0 = 0; k0 < D; k0 += 32) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int rr = ty + 8 * q;
+      As[rr][tx] = (double)__bfloat162float(W[(int64_t)(i0 + rr) * D + k0 + tx]);
+      Bs[rr][tx] = (double)__bfloat162float(G[(int64_t)(k0 + rr) * D + j0 + tx]);
+    }
+    __syncthreads();
+#pragma unroll 8
+    for (int k = 0; k < 32; ++k) {
+      const double bv = Bs[k][tx];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) acc[q] = fma(As[ty + 8 * q][k], bv, acc[q]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int i = i0 + ty + 8 * q, j = j0 + tx;
+    const __nv_bfloat16 v = __float2bfloat16_rn(__double2float_rn(acc[q]));
+    V[(int64_t)r * D * D + (int64_t)i * D + j] = v;
     Vt[(int64_t)r * D * D + (int64_t)j * D + i] = v;
   }
 }
 
 // dW_r = G_r W_agg[t_r]^T and dW_agg[t] = sum over r -> t (ascending) of W_r^T G_r, fp32, where
-// G_r = M_r^T dU_{t_r}; types without relations get zero.
+// G_r = M_r^T dU_{t_r}; types without relations get zero.  Grid (D/32, D/32, relations + types),
+// 32 x 32 output tiles from 32-wide K slices in shared memory (thread layout as fuse_weights).
 template <int D>
-__global__ void wgrad_finish(const float* __restrict__ G, const __nv_bfloat16* __restrict__ W_rel,
-                             const __nv_bfloat16* __restrict__ W_agg, RelDst rel_dst, int num_rels, int num_types,
-                             float* __restrict__ dW_rel, float* __restrict__ dW_agg) {
-  const int64_t n_rel = (int64_t)num_rels * D * D, total = n_rel + (int64_t)num_types * D * D;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
-    if (e < n_rel) {
-      const int r = (int)(e / (D * D));
-      const int i = (int)((e / D) % D), j = (int)(e % D);
-      const float* g = G + (int64_t)r * D * D + (int64_t)i * D;
-      const __nv_bfloat16* w = W_agg + (int64_t)rel_dst.v[r] * D * D + (int64_t)j * D;
-      float acc = 0.f;
-      for (int k = 0; k < D; ++k) acc = fmaf(g[k], __bfloat162float(w[k]), acc);
-      dW_rel[e] = acc;
-    } else {
-      const int64_t f = e - n_rel;
-      const int t = (int)(f / (D * D));
-      const int i = (int)((f / D) % D), j = (int)(f % D);
-      float acc = 0.f;
-      for (int r = 0; r < num_rels; ++r) {
-        if (rel_dst.v[r] != t) continue;
-        const __nv_bfloat16* w = W_rel + (int64_t)r * D * D + i;
-        const float* g = G + (int64_t)r * D * D + j;
-        for (int k = 0; k < D; ++k) acc = fmaf(__bfloat162float(w[(int64_t)k * D]), g[(int64_t)k * D], acc);
-      }
-      dW_agg[f] = acc;
+__global__ void __launch_bounds__(256) wgrad_finish(const float* __restrict__ G, const __nv_bfloat16* __restrict__ W_rel,
+                                                    const __nv_bfloat16* __restrict__ W_agg, RelDst rel_dst,
+                                                    int num_rels, int num_types, float* __restrict__ dW_rel,
+                                                    float* __restrict__ dW_agg) {
+  __shared__ float As[32][33];
+  __shared__ float Bs[32][33];
+  const int z = blockIdx.z, i0 = blockIdx.y * 32, j0 = blockIdx.x * 32;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  auto mac = [&]() {
+#pragma unroll 8
+    for (int k = 0; k < 32; ++k) {
+      const float bv = Bs[k][tx];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) acc[q] = fmaf(As[ty + 8 * q][k], bv, acc[q]);
     }
+  };
+  if (z < num_rels) {  // dW_r[i][j] = sum_k G_r[i][k] W_agg[t][j][k]
+    const float* Gr = G + (int64_t)z * D * D;
+    const __nv_bfloat16* Wa = W_agg + (int64_t)rel_dst.v[z] * D * D;
+    for (int k0 = 0; k0 < D; k0 += 32) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int rr = ty + 8 * q;
+        As[rr][tx] = Gr[(int64_t)(i0 + rr) * D + k0 + tx];
+        Bs[tx][rr] = __bfloat162float(Wa[(int64_t)(j0 + rr) * D + k0 + tx]);
+      }
+      __syncthreads();
+      mac();
+      __syncthreads();
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) dW_rel[(int64_t)z * D * D + (int64_t)(i0 + ty + 8 * q) * D + j0 + tx] = acc[q];
+  } else {  // dW_agg[t][i][j] = sum_{r -> t} sum_k W_r[k][i] G_r[k][j]
+    const int t = z - num_rels;
+    for (int r = 0; r < num_rels; ++r) {
+      if (rel_dst.v[r] != t) continue;
+      const __nv_bfloat16* Wr = W_rel + (int64_t)r * D * D;
+      const float* Gr = G + (int64_t)r * D * D;
+      for (int k0 = 0; k0 < D; k0 += 32) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int rr = ty + 8 * q;
+          As[tx][rr] = __bfloat162float(Wr[(int64_t)(k0 + rr) * D + i0 + tx]);
+          Bs[rr][tx] = Gr[(int64_t)(k0 + rr) * D + j0 + tx];
+        }
+        __syncthreads();
+        mac();
+        __syncthreads();
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) dW_agg[(int64_t)t * D * D + (int64_t)(i0 + ty + 8 * q) * D + j0 + tx] = acc[q];
   }
 }
 
@@ -466,120 +528,166 @@ __global__ void __launch_bounds__(256) ln_act_bwd(TcBwdArgs a) {
 // ---------------------------------------------------------------------------------------------
 template <int D>
 struct BwdCfg {
-  static constexpr int kStages = 2;
+  static constexpr int kStages = D == 256 ? 2 : 4;     // ring of V_r chunks (D rows x 64 columns)
   static constexpr int kB = D * 128;
-  static constexpr int kT = kTileRows * D * 2;  // dU operand tile (KC x 16 KB)
-  static constexpr int kSmem = kStages * kB + kT + 256 + 1024;
-  static constexpr int kTmemCols = D < 32 ? 32 : D;
+  static constexpr int kT = kTileRows * D * 2;          // dU operand tile (KC x 16 KB), double-buffered
+  static constexpr int kAcc = D < 32 ? 32 : D;
+  static constexpr int kNumAcc = 512 / kAcc < 4 ? 512 / kAcc : 4;  // ring of TMEM accumulators
+  static constexpr int kTmemCols = kNumAcc * kAcc;
+  static constexpr int kSmem = kStages * kB + 2 * kT + 512 + 1024;
+  static constexpr int kEpiGroups = 2;  // epilogue warp groups, taking alternate accumulators
+  static constexpr int kThreads = 64 + kEpiGroups * 128;
 };
 
-// dMs_r = (dU V_r^T) / deg_r for every relation r into this type; dU loaded by TMA.
+// dMs_r = (dU V_r^T) / deg_r for every relation r into this type.  Persistent, one CTA per SM:
+// warp 0 loads dU tiles and V_r chunks (TMA), warp 1 issues one MMA chain per (tile, relation)
+// into a ring of TMEM accumulators, and two groups of four warps (2-5, 6-9) scale and store
+// alternate accumulators, so the stores of one relation overlap the products of the next.
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1) proj_bwd_tc(const __grid_constant__ CUtensorMap tm_dU,
-                                                          const __grid_constant__ CUtensorMap tm_V, TcBwdArgs a) {
+__global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
+    proj_bwd_tc(const __grid_constant__ CUtensorMap tm_dU, const __grid_constant__ CUtensorMap tm_V, TcBwdArgs a) {
   using C = BwdCfg<D>;
   constexpr int S = C::kStages;
+  constexpr int NB = C::kNumAcc;
   constexpr int KC = D / 64;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  uint8_t* bstage = smem;            // S x B chunk
-  uint8_t* tile = smem + S * C::kB;  // KC x 16 KB
-  uint64_t* full = reinterpret_cast<uint64_t*>(tile + C::kT);
-  uint64_t* empty = full + S;
-  uint64_t* accb = empty + S;
-  uint64_t* tileb = accb + 1;
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(tileb + 1);
-  int* abort_flag = reinterpret_cast<int*>(tslot + 1);
+  uint8_t* bstage = smem;                 // S x B chunk
+  uint8_t* tiles = smem + S * C::kB;      // 2 x (KC x 16 KB)
+  uint64_t* b_full = reinterpret_cast<uint64_t*>(tiles + 2 * C::kT);
+  uint64_t* b_empty = b_full + S;
+  uint64_t* a_full = b_empty + S;       // [2] dU tile loaded
+  uint64_t* a_empty = a_full + 2;       // [2] every product of the tile done
+  uint64_t* acc_full = a_empty + 2;     // [NB]
+  uint64_t* acc_empty = acc_full + NB;  // [NB]
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(acc_empty + NB);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t m0 = (int64_t)blockIdx.x * kTileRows;
-  const int CT = KC * a.nrel;
-  auto issue_load = [&](int g) {
-    const int s = g % S;
-    mbar_expect_tx(&full[s], C::kB);
-    tma_load_2d(bstage + s * C::kB, &tm_V, (g % KC) * 64, a.rel[g / KC] * D, &full[s]);
-  };
+  const int64_t ntiles = (a.n + kTileRows - 1) / kTileRows;
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&b_full[s], 1);
+      mbar_init(&b_empty[s], 1);
     }
-    mbar_init(accb, 1);
-    mbar_init(tileb, 1);
-    *abort_flag = 0;
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&a_full[b], 1);
+      mbar_init(&a_empty[b], 1);
+    }
+    for (int k = 0; k < NB; ++k) {
+      mbar_init(&acc_full[k], 1);
+      mbar_init(&acc_empty[k], kTileRows);
+    }
     fence_mbar_init();
     prefetch_tmap(&tm_dU);
     prefetch_tmap(&tm_V);
-    mbar_expect_tx(tileb, C::kT);
-    for (int kc = 0; kc < KC; ++kc) tma_load_2d(tile + kc * kATile, &tm_dU, kc * 64, (int)m0, tileb);
-    for (int g = 0; g < S && g < CT; ++g) issue_load(g);
   }
-  if (warp == 0) tmem_alloc(tslot, C::kTmemCols);
+  if (warp == 1) tmem_alloc(tslot, C::kTmemCols);
   fence_before_sync();
   __syncthreads();
   fence_after_sync();
   const uint32_t tmem = *tslot;
-  const uint32_t idesc = idesc_bf16(128, D, false, false);
-  auto product = [&](int g0) {
-    bool ok = *abort_flag == 0;
-    for (int g = g0; g < g0 + KC && ok; ++g) {
-      const int s = g % S;
-      ok = mbar_wait(&full[s], (g / S) & 1);
-      if (!ok) break;
-      fence_after_sync();
-      const uint32_t A = smem_u32(tile + (g - g0) * kATile);
-      const uint32_t B = smem_u32(bstage + s * C::kB);
+
+  if (warp == 0) {
+    if (lane == 0) {  // ---- TMA producer
+      bool ok = true;
+      uint32_t g = 0;
+      int it = 0;
+      for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
+        const int ab = it & 1;
+        if (it >= 2) ok = mbar_wait(&a_empty[ab], ((it >> 1) - 1) & 1);
+        if (!ok) break;
+        mbar_expect_tx(&a_full[ab], C::kT);
+        for (int kc = 0; kc < KC; ++kc)
+          tma_load_2d(tiles + ab * C::kT + kc * kATile, &tm_dU, kc * 64, (int)(tile * kTileRows), &a_full[ab]);
+        for (int j = 0; j < a.nrel * KC && ok; ++j, ++g) {
+          const uint32_t s = g % S;
+          if (g >= (uint32_t)S) ok = mbar_wait(&b_empty[s], ((g / S) - 1) & 1);
+          if (!ok) break;
+          mbar_expect_tx(&b_full[s], C::kB);
+          tma_load_2d(bstage + s * C::kB, &tm_V, (j % KC) * 64, a.rel[j / KC] * D, &b_full[s]);
+        }
+      }
+      if (!ok) atomicOr(a.status, kErrTimeout);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {  // ---- MMA issuer
+      const uint32_t idesc = idesc_bf16(128, D, false, false);
+      bool ok = true;
+      uint32_t g = 0, jb = 0;
+      int it = 0;
+      for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
+        const int ab = it & 1;
+        ok = mbar_wait(&a_full[ab], (it >> 1) & 1);
+        if (!ok) break;
+        const uint32_t A0 = smem_u32(tiles + ab * C::kT);
+        for (int r = 0; r < a.nrel && ok; ++r, ++jb) {
+          const uint32_t k = jb % NB;
+          if (jb >= (uint32_t)NB) ok = mbar_wait(&acc_empty[k], ((jb / NB) - 1) & 1);
+          if (!ok) break;
+          fence_after_sync();
+          const uint32_t acc = tmem + k * C::kAcc;
+          for (int kc = 0; kc < KC && ok; ++kc, ++g) {
+            const uint32_t s = g % S;
+            ok = mbar_wait(&b_full[s], (g / S) & 1);
+            if (!ok) break;
+            fence_after_sync();
+            const uint32_t A = A0 + kc * kATile;
+            const uint32_t B = smem_u32(bstage + s * C::kB);
 #pragma unroll
-      for (int ks = 0; ks < 4; ++ks)
-        mma_bf16(tmem, desc_sw128(A + ks * 32, 16, 1024), desc_sw128(B + ks * 32, 16, 1024), idesc,
-                 (g > g0 || ks > 0) ? 1u : 0u);
-      mma_commit(&empty[s]);
-      if (g + S < CT) {
-        ok = mbar_wait(&empty[s], (g / S) & 1);
-        if (ok) issue_load(g + S);
+            for (int ks = 0; ks < 4; ++ks)
+              mma_bf16(acc, desc_sw128(A + ks * 32, 16, 1024), desc_sw128(B + ks * 32, 16, 1024), idesc,
+                       (kc > 0 || ks > 0) ? 1u : 0u);
+            mma_commit(&b_empty[s]);
+          }
+          mma_commit(&acc_full[k]);
+        }
+        mma_commit(&a_empty[ab]);
+      }
+      if (!ok) atomicOr(a.status, kErrTimeout);
+    }
+    __syncwarp();
+  } else {  // ---- epilogue: scale by 1 / deg_r and store dMs_r rows
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    const uint32_t grp = (uint32_t)(warp - 2) / 4;  // this group takes jobs jb = grp mod kEpiGroups
+    bool ok = true;
+    uint32_t jb = 0;
+    for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+      const int64_t m = tile * kTileRows + row;
+      const bool live = m < a.n;
+      for (int r = 0; r < a.nrel && ok; ++r, ++jb) {
+        if (jb % C::kEpiGroups != grp) continue;
+        const uint32_t k = jb % NB;
+        const int64_t crow = a.mrow0[r] + (live ? m : 0);
+        const int deg = live ? a.csr_ptr[crow + 1] - a.csr_ptr[crow] : 0;
+        const float sc = deg > 0 ? __fdiv_rn(1.0f, (float)deg) : 0.f;
+        ok = mbar_wait(&acc_full[k], (jb / NB) & 1);
+        if (!ok) break;
+        fence_after_sync();
+        const uint32_t trow = tmem + k * C::kAcc + ((uint32_t)(q * 32) << 16);
+        if constexpr (D % 32 == 0) {
+#pragma unroll
+          for (int c = 0; c < D; c += 32) {
+            float v[32];
+            tmem_ld32(trow + c, v);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] *= sc;
+            if (live) {
+              store16_bf16(a.dMs + crow * D + c, v);
+              store16_bf16(a.dMs + crow * D + c + 16, v + 16);
+            }
+          }
+        }
+        fence_before_sync();
+        mbar_arrive(&acc_empty[k]);
       }
     }
-    if (!ok) {
-      *abort_flag = 1;
-      atomicOr(a.status, kErrTimeout);
-    }
-    mma_commit(accb);
-  };
-  if (threadIdx.x == 0 && !mbar_wait(tileb, 0)) {
-    *abort_flag = 1;
-    atomicOr(a.status, kErrTimeout);
-  }
-  const int row = warp * 32 + lane;
-  const int64_t m = m0 + row;
-  const bool live = m < a.n;
-  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
-  uint32_t phase = 0;
-  for (int r = 0; r < a.nrel; ++r) {
-    if (warp == 0) {
-      if (lane == 0) product(KC * r);
-      __syncwarp();
-    }
-    if (!mbar_wait(accb, phase)) atomicOr(a.status, kErrTimeout);
-    phase ^= 1;
-    fence_after_sync();
-    const int64_t crow = a.mrow0[r] + (live ? m : 0);
-    const int deg = live ? a.csr_ptr[crow + 1] - a.csr_ptr[crow] : 0;
-    const float sc = deg > 0 ? __fdiv_rn(1.0f, (float)deg) : 0.f;
-#pragma unroll 1
-    for (int c = 0; c < D; c += 16) {
-      float v[16];
-      tmem_ld16(trow + c, v);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) v[i] *= sc;
-      if (live) store16_bf16(a.dMs + crow * D + c, v);
-    }
-    fence_before_sync();
-    __syncthreads();
-    fence_after_sync();
+    if (!ok) atomicOr(a.status, kErrTimeout);
   }
   fence_before_sync();
   __syncthreads();
-  if (warp == 0) tmem_dealloc(tmem, C::kTmemCols);
+  if (warp == 1) tmem_dealloc(tmem, C::kTmemCols);
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -713,7 +821,8 @@ static unsigned flat_grid(int64_t n) {
 template <int D>
 static hg_status tc_fuse_t(const void* W_rel, const void* W_agg, RelDst rd, int num_rels, void* V, void* Vt,
                            cudaStream_t s) {
-  return launch("fuse_weights", fuse_weights<D>, dim3(flat_grid((int64_t)num_rels * D * D)), dim3(256), 0, s,
+  if (num_rels == 0) return HG_OK;
+  return launch("fuse_weights", fuse_weights<D>, dim3(D / 32, D / 32, num_rels), dim3(256), 0, s,
                 (const __nv_bfloat16*)W_rel, (const __nv_bfloat16*)W_agg, rd, num_rels, (__nv_bfloat16*)V,
                 (__nv_bfloat16*)Vt);
 }
@@ -752,14 +861,18 @@ static hg_status tc_bwd_t(const TcBwdArgs& a, const void* V, int num_rels, cudaS
   CUtensorMap tm_dU, tm_V;
   HG_TRY(make_tmap_bf16(&tm_dU, a.dU + a.off * D, (uint64_t)a.n, D, kTileRows));
   HG_TRY(make_tmap_bf16(&tm_V, V, (uint64_t)num_rels * D, D, D));
-  return launch("proj_bwd_tc", proj_bwd_tc<D>, dim3((unsigned)ceil_div(a.n, kTileRows)), dim3(kThreads),
-                BwdCfg<D>::kSmem, s, tm_dU, tm_V, a);
+  int sms = 0, dev = 0;
+  HG_CUDA(cudaGetDevice(&dev));
+  HG_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(a.n, kTileRows), sms));
+  return launch("proj_bwd_tc", proj_bwd_tc<D>, dim3(grid), dim3(BwdCfg<D>::kThreads), BwdCfg<D>::kSmem, s, tm_dU,
+                tm_V, a);
 }
 
 int wgrad_tc_splits(int64_t n, int d) {
   const int mtiles = d > 128 ? d / 128 : 1;
   const int64_t chunks = std::max<int64_t>(1, ceil_div(n, 64));
-  return (int)std::max<int64_t>(1, std::min<int64_t>(chunks, (2 * 152) / mtiles));
+  return (int)std::max<int64_t>(1, std::min<int64_t>(chunks, 152 / mtiles));  // one wave, one CTA per SM
 }
 
 template <int D>
@@ -785,7 +898,7 @@ static hg_status tc_wgrad_t(const void* X, int64_t x0, const void* Y, int64_t y0
 template <int D>
 static hg_status tc_finish_t(const float* G, const void* W_rel, const void* W_agg, RelDst rd, int num_rels,
                              int num_types, float* dW_rel, float* dW_agg, cudaStream_t s) {
-  return launch("wgrad_finish", wgrad_finish<D>, dim3(flat_grid((int64_t)(num_rels + num_types) * D * D)), dim3(256),
+  return launch("wgrad_finish", wgrad_finish<D>, dim3(D / 32, D / 32, num_rels + num_types), dim3(256),
                 0, s, G, (const __nv_bfloat16*)W_rel, (const __nv_bfloat16*)W_agg, rd, num_rels, num_types, dW_rel,
                 dW_agg);
 }
