@@ -202,7 +202,7 @@ def kernel_models(st: dict, sp) -> dict:
     m["ln_act_bwd"] = (L * lb, 0)
     m["proj_bwd_tc"] = (L * pb, L * pfl)
     m["wgrad_tc"] = (L * 2 * row * RR, L * 2 * d * d * RR)  # G_r = M_r^T dU: read both operands once
-    m["radix_scatter"] = (2 * 3 * 4 * 4 * st["E"], 0)  # 2 layouts x 3 passes x (read+write of key+value)
+    m["radix_scatter"] = (2 * 3 * 2 * 12 * st["E"], 0)  # 2 layouts x 3 passes x read+write of key, edge id, endpoint
     no = st["n_ov"]
     m["align_colstats"] = (3 * 2 * no * (row + 4), 0)        # 3 passes over both gathered views
     m["align_gram_tc"] = (2 * no * (row + 4), 2 * 2 * no * d * d)
@@ -216,6 +216,26 @@ def load_peaks() -> tuple:
         with open(p) as fh:
             return json.load(fh), "measured"
     return dict(FALLBACK), "fallback"
+
+
+def measured_traffic(kernel: str):
+    """DRAM bytes per launch of `kernel` from the committed ncu capture (profiles/traffic.json), or
+    None when there is none or the kernel's sources changed since it was taken."""
+    import glob
+    import hashlib
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as fh:
+        entry = json.load(fh).get(kernel)
+    if not entry:
+        return None
+    csrc = os.path.join(ROOT, "paper_2608_02168_gb300", "csrc")
+    h = hashlib.sha256()
+    for f in [os.path.join(csrc, entry["source"])] + sorted(glob.glob(os.path.join(csrc, "*.cuh"))):
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return int(entry["bytes_per_launch"]) if h.hexdigest() == entry["sha256"] else None
 
 
 def roofline(report: dict, models: dict, steps: int, peaks: dict, src: str) -> tuple:
@@ -235,7 +255,7 @@ def roofline(report: dict, models: dict, steps: int, peaks: dict, src: str) -> t
         rf = dict(bound="hbm", achieved=round(ach, 1), peak=peaks["hbm_gbs"], unit="GB/s",
                   peak_source=f"{src} hbm_gbs")
     rf["frac"] = round(rf["achieved"] / rf["peak"], 4) if rf["peak"] else None
-    rf["traffic"] = None
+    rf["traffic"] = measured_traffic(dom)
     rf.update(kernel=dom, launches=n, avg_launch_ms=round(ms / max(n, 1), 4),
               algorithmic_bytes_per_launch=int(by * steps / max(n, 1)), flops_per_launch=int(fl * steps / max(n, 1)))
     return rf, shares
