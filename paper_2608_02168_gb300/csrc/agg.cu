@@ -256,6 +256,17 @@ __global__ void __launch_bounds__(256) agg_bwd_nodes(GraphMeta m, const int32_t*
   const int64_t step = (int64_t)gridDim.x * S::kGroups;
   for (int64_t node = (int64_t)blockIdx.x * S::kGroups + grp; node < N; node += step) {
     const int t = node_type_of(m, node);
+    // the node's CSC bounds in every relation leaving its type, all loaded before any gather
+    int beg[kMaxRels], end[kMaxRels];
+#pragma unroll
+    for (int r = 0; r < kMaxRels; ++r) {
+      beg[r] = end[r] = 0;
+      if (r < m.num_rels && m.rel_src[r] == t) {
+        const int64_t crow = m.csc_base[r] + (node - m.type_off[t]);
+        beg[r] = __ldg(cptr + crow);
+        end[r] = __ldg(cptr + crow + 1);
+      }
+    }
     float acc[S::F];
 #pragma unroll
     for (int v = 0; v < S::V; ++v) {
@@ -264,14 +275,15 @@ __global__ void __launch_bounds__(256) agg_bwd_nodes(GraphMeta m, const int32_t*
 #pragma unroll
       for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] = f[q];
     }
-    for (int r = 0; r < m.num_rels; ++r) {
-      if (m.rel_src[r] != t) continue;
-      const int64_t crow = m.csc_base[r] + (node - m.type_off[t]);
-      const int beg = __ldg(cptr + crow), end = __ldg(cptr + crow + 1);
-      if (end - beg > kHubDegree)
+#pragma unroll
+    for (int r = 0; r < kMaxRels; ++r) {
+      if (end[r] == beg[r]) continue;
+      if (end[r] - beg[r] > kHubDegree) {
+        const int64_t crow = m.csc_base[r] + (node - m.type_off[t]);
         add_partials<T, D>(partials, chunk_ofs[crow], chunk_ofs[crow + 1], lane, acc);
-      else
-        gather_sum<T, D>(ccol, beg, end, 1, m.row_base[r] - m.type_off[m.rel_dst[r]], dMs, lane, acc);
+      } else {
+        gather_sum<T, D>(ccol, beg[r], end[r], 1, m.row_base[r] - m.type_off[m.rel_dst[r]], dMs, lane, acc);
+      }
     }
     store_row<T, D>(dH + node * D, lane, acc, 1.0f);
   }
@@ -280,7 +292,16 @@ __global__ void __launch_bounds__(256) agg_bwd_nodes(GraphMeta m, const int32_t*
 // ---------------------------------------------------------------------------------------------
 // host dispatch
 // ---------------------------------------------------------------------------------------------
-constexpr int64_t kPersistBlocks = 152 * 6;  // resident 256-thread blocks per SM at 40 registers
+// Persistent grids: as many 256-thread blocks as are resident at once (occupancy of the kernel).
+template <typename K>
+static hg_status persist_blocks(K kernel, int64_t* blocks) {
+  int dev = 0, sms = 0, per_sm = 0;
+  HG_CUDA(cudaGetDevice(&dev));
+  HG_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  HG_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, 256, 0));
+  *blocks = (int64_t)sms * std::max(1, per_sm);
+  return HG_OK;
+}
 
 static unsigned chunk_grid(int64_t cap) { return (unsigned)std::max<int64_t>(1, std::min<int64_t>(cap, 152 * 8)); }
 
@@ -293,8 +314,10 @@ static hg_status agg_fwd_t(const hg_graph* g, const void* H, void* M, float* par
                 partials));
   HG_TRY(launch("combine_chunk_partials", combine_chunk_partials<D>, dim3(chunk_grid(g->chunk_cap_csr)), dim3(D), 0, s,
                 (const int32_t*)g->csr_chunk_row, (const int32_t*)g->csr_chunk_ofs, g->csr_rows, partials));
+  static int64_t pb = 0;
+  if (pb == 0) HG_TRY(persist_blocks(agg_fwd_rows<T, D>, &pb));
   return launch("agg_fwd_rows", agg_fwd_rows<T, D>,
-                dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(g->csr_rows, S::kGroups), kPersistBlocks))),
+                dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(g->csr_rows, S::kGroups), pb))),
                 dim3(256),
                 0, s, (const int32_t*)g->csr_ptr, (const int32_t*)g->csr_col, (const T*)H, (T*)M, g->csr_rows,
                 (const int32_t*)g->csr_chunk_ofs, (const float*)partials);
@@ -311,8 +334,10 @@ static hg_status agg_bwd_t(const hg_graph* g, const void* dMs, const void* dY, v
   HG_TRY(launch("combine_chunk_partials", combine_chunk_partials<D>, dim3(chunk_grid(g->chunk_cap_csc)), dim3(D), 0, s,
                 (const int32_t*)g->csc_chunk_row, (const int32_t*)g->csc_chunk_ofs, g->csc_rows, partials));
   const int64_t N = g->meta.type_off[g->meta.num_types];
+  static int64_t pb = 0;
+  if (pb == 0) HG_TRY(persist_blocks(agg_bwd_nodes<T, D>, &pb));
   return launch("agg_bwd_nodes", agg_bwd_nodes<T, D>,
-                dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(N, S::kGroups), kPersistBlocks))),
+                dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(N, S::kGroups), pb))),
                 dim3(256), 0, s,
                 g->meta, (const int32_t*)g->csc_ptr, (const int32_t*)g->csc_col, (const T*)dMs, (const T*)dY,
                 (T*)dH, (const int32_t*)g->csc_chunk_ofs, (const float*)partials);

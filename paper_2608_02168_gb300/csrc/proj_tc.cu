@@ -466,46 +466,61 @@ __global__ void __launch_bounds__(256) ln_act_bwd(TcBwdArgs a) {
       st16(p, pack(v, __nv_bfloat16()));
     }
   };
-  for (int64_t row = (int64_t)blockIdx.x * 8 + warp; row < a.n; row += (int64_t)gridDim.x * 8) {
-    const int64_t node = a.off + row;
-    float dv[E], uv[E], hv[E], dy[E], du[E], xh[E];
-    load(a.dH_out + node * D + c0, dv);
-    load(a.U + node * D + c0, uv);
-    load(a.H_in + node * D + c0, hv);
-    if (a.ln) {
-      const float2 st = a.stats[node];
-      float s1 = 0.f, s2 = 0.f;
+  // two rows per iteration: both rows' loads are in flight before either is computed
+  const int64_t step = (int64_t)gridDim.x * 8;
+  for (int64_t row0 = (int64_t)blockIdx.x * 8 + warp; row0 < a.n; row0 += 2 * step) {
+    float dv[2][E], uv[2][E], hv[2][E];
+    float2 st[2];
+    bool has[2];
 #pragma unroll
-      for (int i = 0; i < E; ++i) {
-        xh[i] = (act_apply(uv[i], a.act) + hv[i] - st.x) * st.y;
-        const float dxh = dv[i] * g[i];
-        s1 += dxh;
-        s2 += dxh * xh[i];
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        s1 += __shfl_xor_sync(0xffffffffu, s1, o);
-        s2 += __shfl_xor_sync(0xffffffffu, s2, o);
-      }
-      const float mean1 = s1 * (1.f / D), mean2 = s2 * (1.f / D);
-#pragma unroll
-      for (int i = 0; i < E; ++i) dy[i] = st.y * (dv[i] * g[i] - mean1 - xh[i] * mean2);
-    } else {
-#pragma unroll
-      for (int i = 0; i < E; ++i) {
-        dy[i] = dv[i];
-        xh[i] = 0.f;
-      }
+    for (int k = 0; k < 2; ++k) {
+      const int64_t row = row0 + k * step;
+      has[k] = row < a.n;
+      const int64_t node = a.off + (has[k] ? row : row0);
+      load(a.dH_out + node * D + c0, dv[k]);
+      load(a.U + node * D + c0, uv[k]);
+      load(a.H_in + node * D + c0, hv[k]);
+      st[k] = a.ln ? a.stats[node] : make_float2(0.f, 1.f);
     }
 #pragma unroll
-    for (int i = 0; i < E; ++i) {
-      du[i] = __bfloat162float(__float2bfloat16_rn(dy[i] * act_grad(uv[i], a.act)));
-      pdb[i] += du[i];
-      pdg[i] += dv[i] * xh[i];
-      pdbe[i] += dv[i];
+    for (int k = 0; k < 2; ++k) {
+      if (!has[k]) continue;
+      const int64_t node = a.off + row0 + k * step;
+      float dy[E], du[E], xh[E];
+      if (a.ln) {
+        float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+        for (int i = 0; i < E; ++i) {
+          xh[i] = (act_apply(uv[k][i], a.act) + hv[k][i] - st[k].x) * st[k].y;
+          const float dxh = dv[k][i] * g[i];
+          s1 += dxh;
+          s2 += dxh * xh[i];
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          s1 += __shfl_xor_sync(0xffffffffu, s1, o);
+          s2 += __shfl_xor_sync(0xffffffffu, s2, o);
+        }
+        const float mean1 = s1 * (1.f / D), mean2 = s2 * (1.f / D);
+#pragma unroll
+        for (int i = 0; i < E; ++i) dy[i] = st[k].y * (dv[k][i] * g[i] - mean1 - xh[i] * mean2);
+      } else {
+#pragma unroll
+        for (int i = 0; i < E; ++i) {
+          dy[i] = dv[k][i];
+          xh[i] = 0.f;
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < E; ++i) {
+        du[i] = __bfloat162float(__float2bfloat16_rn(dy[i] * act_grad(uv[k][i], a.act)));
+        pdb[i] += du[i];
+        pdg[i] += dv[k][i] * xh[i];
+        pdbe[i] += dv[k][i];
+      }
+      store(a.dY + node * D + c0, dy);
+      store(a.dU + node * D + c0, du);
     }
-    store(a.dY + node * D + c0, dy);
-    store(a.dU + node * D + c0, du);
   }
 #pragma unroll
   for (int i = 0; i < E; ++i) {
@@ -814,9 +829,6 @@ static hg_status smem_attr_once() {
   return HG_OK;
 }
 
-static unsigned flat_grid(int64_t n) {
-  return (unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(n, 256), 152 * 8));
-}
 
 template <int D>
 static hg_status tc_fuse_t(const void* W_rel, const void* W_agg, RelDst rd, int num_rels, void* V, void* Vt,
