@@ -32,7 +32,7 @@ struct AggShape {
 
 // acc += sum of rows src[col[e] + delta] for e = beg, beg + stride, ... < end, added in edge
 // order; eight neighbour rows are loaded before they are added.
-template <typename T, int D>
+template <typename T, int D, bool kBatchTail = true>
 __device__ __forceinline__ void gather_sum(const int32_t* __restrict__ col, int64_t beg, int64_t end,
                                            int stride, int64_t delta, const T* __restrict__ src,
                                            int lane, float* acc) {
@@ -59,14 +59,37 @@ __device__ __forceinline__ void gather_sum(const int32_t* __restrict__ col, int6
         for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] += f[q];
       }
   }
-  for (; e < end; e += stride) {
-    const int c = __ldg(col + e);
+  if (!kBatchTail) {
+    for (; e < end; e += stride) {
+      const int c = __ldg(col + e);
 #pragma unroll
-    for (int v = 0; v < S::V; ++v) {
-      float f[S::kVec];
-      unpack(ldg16(base + (int64_t)c * D + v * S::G * S::kVec), f, T());
+      for (int v = 0; v < S::V; ++v) {
+        float f[S::kVec];
+        unpack(ldg16(base + (int64_t)c * D + v * S::G * S::kVec), f, T());
 #pragma unroll
-      for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] += f[q];
+        for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] += f[q];
+      }
+    }
+  } else if (e < end) {  // the last (fewer than U) rows as one predicated batch
+    int c[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) c[u] = e + u * (int64_t)stride < end ? __ldg(col + e + u * stride) : -1;
+    uint4 x[U][S::V];
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+#pragma unroll
+      for (int v = 0; v < S::V; ++v)
+        x[u][v] = c[u] >= 0 ? ldg16(base + (int64_t)c[u] * D + v * S::G * S::kVec) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (c[u] < 0) break;
+#pragma unroll
+      for (int v = 0; v < S::V; ++v) {
+        float f[S::kVec];
+        unpack(x[u][v], f, T());
+#pragma unroll
+        for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] += f[q];
+      }
     }
   }
 }
@@ -187,7 +210,7 @@ __global__ void __launch_bounds__(256) agg_chunks(const int32_t* __restrict__ pt
     float acc[S::F];
 #pragma unroll
     for (int q = 0; q < S::F; ++q) acc[q] = 0.f;
-    gather_sum<T, D>(col, beg + grp, end, S::kGroups, delta, src, lane, acc);
+    gather_sum<T, D, false>(col, beg + grp, end, S::kGroups, delta, src, lane, acc);
 #pragma unroll
     for (int v = 0; v < S::V; ++v)
 #pragma unroll
