@@ -139,22 +139,21 @@ __global__ void __launch_bounds__(kSortThreads) radix_hist(const uint32_t* __res
   hist[(int64_t)threadIdx.x * tiles + blockIdx.x] = h[threadIdx.x];
 }
 
-// Stable scatter of one 2048-item tile.  (1) The tile is staged in shared memory (coalesced).
-// (2) Warp w ranks its 256 consecutive items 32 at a time with __match_any_sync, keeping per-digit
-// running counts, so the item order inside the tile is (warp, round, lane).  (3) Per-digit
+// Stable scatter of one 2048-item tile.  (1) Warp w reads its 256 consecutive items, 32 at a time
+// (coalesced), into registers.  (2) It ranks them round by round with __match_any_sync, keeping
+// per-digit running counts, so the item order inside the tile is (warp, round, lane).  (3) Per-digit
 // prefixes over warps and over digits give every item its position in the tile sorted by digit
-// (equal digits keep their order), where it is written in shared memory.  (4) Consecutive
-// threads write consecutive sorted items to base[digit] + (position - tile start of the digit):
-// runs of equal digits go out coalesced.
+// (equal digits keep their order), where it is written in shared memory.  (4) Consecutive threads
+// write consecutive sorted items to base[digit] + (position - tile start of the digit): runs of
+// equal digits go out coalesced.
 template <bool kTwo>
 __global__ void __launch_bounds__(kSortThreads) radix_scatter(
     const uint32_t* __restrict__ keys_in, const uint32_t* __restrict__ vals_in,
     const uint32_t* __restrict__ vals2_in, uint32_t* __restrict__ keys_out, uint32_t* __restrict__ vals_out,
     uint32_t* __restrict__ vals2_out, int64_t n, int shift, const int32_t* __restrict__ offs, int64_t tiles) {
+  constexpr int R = kWarpSlice / 32;  // rounds (items per thread)
   __shared__ uint32_t skey[kSortTile], sval[kSortTile];  // sorted tile
-  __shared__ uint32_t tkey[kSortTile], tval[kSortTile];  // staged tile
-  __shared__ uint32_t sval2[kTwo ? kSortTile : 1], tval2[kTwo ? kSortTile : 1];
-  __shared__ uint16_t srank[kSortTile];
+  __shared__ uint32_t sval2[kTwo ? kSortTile : 1];
   __shared__ int whist[kSortWarps][kRadix];
   __shared__ int dstart[kRadix];  // tile position where each digit's run starts
   __shared__ int gbase[kRadix];   // global position of the digit's run of this tile
@@ -163,27 +162,29 @@ __global__ void __launch_bounds__(kSortThreads) radix_scatter(
   const int cnt = (int)min((int64_t)kSortTile, n - t0);
   for (int i = threadIdx.x; i < kSortWarps * kRadix; i += kSortThreads) (&whist[0][0])[i] = 0;
   gbase[threadIdx.x] = offs[(int64_t)threadIdx.x * tiles + blockIdx.x];
+  uint32_t k[R], v[R], v2[R];
+  int rank[R];
 #pragma unroll
-  for (int i = 0; i < kSortItems; ++i) {
-    const int j = i * kSortThreads + threadIdx.x;
+  for (int r = 0; r < R; ++r) {
+    const int j = warp * kWarpSlice + r * 32 + lane;
     if (j < cnt) {
-      tkey[j] = keys_in[t0 + j];
-      tval[j] = vals_in[t0 + j];
-      if (kTwo) tval2[j] = vals2_in[t0 + j];
+      k[r] = keys_in[t0 + j];
+      v[r] = vals_in[t0 + j];
+      if (kTwo) v2[r] = vals2_in[t0 + j];
     }
   }
   __syncthreads();
   const unsigned lt_mask = (1u << lane) - 1u;
-  for (int r = 0; r < kWarpSlice / 32; ++r) {
+#pragma unroll
+  for (int r = 0; r < R; ++r) {
     const int j = warp * kWarpSlice + r * 32 + lane;
-    const bool ok = j < cnt;
-    const int d = ok ? (int)((tkey[j] >> shift) & (kRadix - 1)) : kRadix;
+    const int d = j < cnt ? (int)((k[r] >> shift) & (kRadix - 1)) : kRadix;
     const unsigned peers = __match_any_sync(0xffffffffu, d);
     const int c = d < kRadix ? whist[warp][d] : 0;
     __syncwarp();
     if (d < kRadix && lane == __ffs(peers) - 1) whist[warp][d] = c + __popc(peers);
     __syncwarp();
-    if (ok) srank[j] = (uint16_t)(c + __popc(peers & lt_mask));
+    rank[r] = c + __popc(peers & lt_mask);
   }
   __syncthreads();
   {  // per digit: exclusive prefix over warps; tile total
@@ -198,40 +199,43 @@ __global__ void __launch_bounds__(kSortThreads) radix_scatter(
   }
   __syncthreads();
   if (warp == 0) {  // exclusive scan of the 256 digit totals
-    int v[kRadix / 32], s = 0;
+    int vv[kRadix / 32], sum = 0;
 #pragma unroll
     for (int i = 0; i < kRadix / 32; ++i) {
-      v[i] = dstart[lane * (kRadix / 32) + i];
-      s += v[i];
+      vv[i] = dstart[lane * (kRadix / 32) + i];
+      sum += vv[i];
     }
-    int incl = s;
+    int incl = sum;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const int y = __shfl_up_sync(0xffffffffu, incl, o);
       if (lane >= o) incl += y;
     }
-    int run = incl - s;
+    int run = incl - sum;
 #pragma unroll
     for (int i = 0; i < kRadix / 32; ++i) {
       dstart[lane * (kRadix / 32) + i] = run;
-      run += v[i];
+      run += vv[i];
     }
   }
   __syncthreads();
-  for (int j = threadIdx.x; j < cnt; j += kSortThreads) {
-    const int w = j / kWarpSlice;
-    const int d = (int)((tkey[j] >> shift) & (kRadix - 1));
-    const int p = dstart[d] + whist[w][d] + srank[j];
-    skey[p] = tkey[j];
-    sval[p] = tval[j];
-    if (kTwo) sval2[p] = tval2[j];
+#pragma unroll
+  for (int r = 0; r < R; ++r) {
+    const int j = warp * kWarpSlice + r * 32 + lane;
+    if (j < cnt) {
+      const int d = (int)((k[r] >> shift) & (kRadix - 1));
+      const int p = dstart[d] + whist[warp][d] + rank[r];
+      skey[p] = k[r];
+      sval[p] = v[r];
+      if (kTwo) sval2[p] = v2[r];
+    }
   }
   __syncthreads();
   for (int p = threadIdx.x; p < cnt; p += kSortThreads) {
-    const uint32_t k = skey[p];
-    const int d = (int)((k >> shift) & (kRadix - 1));
+    const uint32_t kk = skey[p];
+    const int d = (int)((kk >> shift) & (kRadix - 1));
     const int64_t pos = (int64_t)gbase[d] + (p - dstart[d]);
-    keys_out[pos] = k;
+    keys_out[pos] = kk;
     vals_out[pos] = sval[p];
     if (kTwo) vals2_out[pos] = sval2[p];
   }
