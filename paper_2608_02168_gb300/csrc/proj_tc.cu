@@ -19,6 +19,7 @@
 // row 32 w + l (its TMEM lane).  Thread 0 issues every TMA load and MMA.  All waits are bounded
 // (tc::kSpinLimit) and report through the library status word.
 #include <algorithm>
+#include <cstring>
 
 #include "layer_kernels.cuh"
 #include "simt_tile.cuh"
@@ -549,9 +550,19 @@ struct BwdCfg {
   static constexpr int kAcc = D < 32 ? 32 : D;
   static constexpr int kNumAcc = 512 / kAcc < 4 ? 512 / kAcc : 4;  // ring of TMEM accumulators
   static constexpr int kTmemCols = kNumAcc * kAcc;
-  static constexpr int kSmem = kStages * kB + 2 * kT + 512 + 1024;
   static constexpr int kEpiGroups = 2;  // epilogue warp groups, taking alternate accumulators
+  // Output tiles staged in shared memory (128B-swizzled, one per epilogue group) and written by
+  // TMA, where shared memory allows it; at D = 256 each thread stores its own row.
+  static constexpr bool kTmaOut = D <= 128;
+  static constexpr int kOut = kTmaOut ? kTileRows * D * 2 : 0;
+  static constexpr int kSmem = kStages * kB + 2 * kT + kEpiGroups * kOut + 512 + 1024;
   static constexpr int kThreads = 64 + kEpiGroups * 128;
+};
+
+// one tensor map per relation over its dMs rows [mrow0[r], mrow0[r] + n): a partial last tile is
+// clipped at the relation's end instead of running into the next relation's rows
+struct RelMaps {
+  CUtensorMap m[kMaxRels];
 };
 
 // dMs_r = (dU V_r^T) / deg_r for every relation r into this type.  Persistent, one CTA per SM:
@@ -560,7 +571,8 @@ struct BwdCfg {
 // alternate accumulators, so the stores of one relation overlap the products of the next.
 template <int D>
 __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
-    proj_bwd_tc(const __grid_constant__ CUtensorMap tm_dU, const __grid_constant__ CUtensorMap tm_V, TcBwdArgs a) {
+    proj_bwd_tc(const __grid_constant__ CUtensorMap tm_dU, const __grid_constant__ CUtensorMap tm_V,
+                const __grid_constant__ RelMaps tm_out, TcBwdArgs a) {
   using C = BwdCfg<D>;
   constexpr int S = C::kStages;
   constexpr int NB = C::kNumAcc;
@@ -569,7 +581,8 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
   uint8_t* smem = align1024(smem_raw);
   uint8_t* bstage = smem;                 // S x B chunk
   uint8_t* tiles = smem + S * C::kB;      // 2 x (KC x 16 KB)
-  uint64_t* b_full = reinterpret_cast<uint64_t*>(tiles + 2 * C::kT);
+  uint8_t* outs = tiles + 2 * C::kT;      // kEpiGroups x (KC x 16 KB) output staging
+  uint64_t* b_full = reinterpret_cast<uint64_t*>(outs + C::kEpiGroups * C::kOut);
   uint64_t* b_empty = b_full + S;
   uint64_t* a_full = b_empty + S;       // [2] dU tile loaded
   uint64_t* a_empty = a_full + 2;       // [2] every product of the tile done
@@ -666,6 +679,9 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
     const int q = warp & 3;
     const int row = q * 32 + lane;
     const uint32_t grp = (uint32_t)(warp - 2) / 4;  // this group takes jobs jb = grp mod kEpiGroups
+    const bool leader = (threadIdx.x & 127) == 0;   // issues the group's TMA stores
+    uint8_t* out = outs + grp * C::kOut;
+    auto group_sync = [&]() { asm volatile("bar.sync %0, 128;" ::"r"(1 + (int)grp) : "memory"); };
     bool ok = true;
     uint32_t jb = 0;
     for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
@@ -681,7 +697,31 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
         if (!ok) break;
         fence_after_sync();
         const uint32_t trow = tmem + k * C::kAcc + ((uint32_t)(q * 32) << 16);
-        if constexpr (D % 32 == 0) {
+        if constexpr (C::kTmaOut) {
+          if (leader) bulk_wait_read();  // the group's previous tile has left the staging buffer
+          group_sync();
+#pragma unroll
+          for (int c = 0; c < D; c += 32) {
+            float v[32];
+            tmem_ld32(trow + c, v);
+#pragma unroll
+            for (int h = 0; h < 32; h += 8) {
+              float w8[8];
+#pragma unroll
+              for (int i = 0; i < 8; ++i) w8[i] = v[h + i] * sc;
+              const int cc = c + h;
+              st16(out + (cc >> 6) * kATile + sw128_offset(row, (uint32_t)(cc & 63) * 2), pack(w8, __nv_bfloat16()));
+            }
+          }
+          fence_before_sync();
+          mbar_arrive(&acc_empty[k]);
+          fence_async_smem();
+          group_sync();
+          if (leader) {
+            for (int kc = 0; kc < KC; ++kc) tma_store_2d(&tm_out.m[r], out + kc * kATile, kc * 64, (int)(tile * kTileRows));
+            bulk_commit();
+          }
+        } else {
 #pragma unroll
           for (int c = 0; c < D; c += 32) {
             float v[32];
@@ -693,11 +733,12 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
               store16_bf16(a.dMs + crow * D + c + 16, v + 16);
             }
           }
+          fence_before_sync();
+          mbar_arrive(&acc_empty[k]);
         }
-        fence_before_sync();
-        mbar_arrive(&acc_empty[k]);
       }
     }
+    if (C::kTmaOut && leader) bulk_wait();
     if (!ok) atomicOr(a.status, kErrTimeout);
   }
   fence_before_sync();
@@ -877,8 +918,13 @@ static hg_status tc_bwd_t(const TcBwdArgs& a, const void* V, int num_rels, cudaS
   HG_CUDA(cudaGetDevice(&dev));
   HG_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
   const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(a.n, kTileRows), sms));
+  RelMaps outs;
+  std::memset(&outs, 0, sizeof(outs));
+  if (BwdCfg<D>::kTmaOut)
+    for (int r = 0; r < a.nrel; ++r)
+      HG_TRY(make_tmap_bf16(&outs.m[r], a.dMs + a.mrow0[r] * D, (uint64_t)a.n, D, kTileRows));
   return launch("proj_bwd_tc", proj_bwd_tc<D>, dim3(grid), dim3(BwdCfg<D>::kThreads), BwdCfg<D>::kSmem, s, tm_dU,
-                tm_V, a);
+                tm_V, outs, a);
 }
 
 int wgrad_tc_splits(int64_t n, int d) {
