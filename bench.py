@@ -370,18 +370,39 @@ def run_ours(args, sp, rank, world):
     # end to end: pinned host inputs copied in, the step, the loss read back, every step
     e2e = None
     if not args.no_e2e:
+        # every step copies its own inputs in from pinned host memory and reads its loss back; the
+        # copy of step i+1's inputs (second device buffer set, copy stream) overlaps step i
         pinned = {k: v.pin_memory() for k, v in host.items()}
         h2d = sum(v.numel() * v.element_size() for v in pinned.values())
         loss_host = torch.empty(3, dtype=torch.float32).pin_memory()
+        bufs = [devin, {k: torch.empty_like(v) for k, v in devin.items()}]
+        copy_stream = torch.cuda.Stream(device=dev)
+        copied = [torch.cuda.Event(), torch.cuda.Event()]
+        consumed = [torch.cuda.Event(), torch.cuda.Event()]
+
+        def copy_in(i):
+            b = i % 2
+            with torch.cuda.stream(copy_stream):
+                copy_stream.wait_event(consumed[b])  # the step that last read this buffer set is done
+                for k, v in pinned.items():
+                    bufs[b][k].copy_(v, non_blocking=True)
+                copied[b].record(copy_stream)
+
         barrier()
         torch.cuda.synchronize()
+        for ev in consumed:
+            ev.record(stream)
         t0 = time.perf_counter()
-        for _ in range(args.steps):
-            for k, v in pinned.items():
-                devin[k].copy_(v, non_blocking=True)
-            step(devin)
+        copy_in(0)
+        for i in range(args.steps):
+            if i + 1 < args.steps:
+                copy_in(i + 1)
+            stream.wait_event(copied[i % 2])
+            step(bufs[i % 2])
+            consumed[i % 2].record(stream)
             loss_host.copy_(path.loss, non_blocking=True)
-            torch.cuda.synchronize()
+            stream.synchronize()  # the loss of step i is on the host
+        torch.cuda.synchronize()
         te = max_over_ranks(time.perf_counter() - t0)
         e2e = {"value": world * edges_per_step * args.steps / te, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(loss_host.numel() * 4)}

@@ -132,7 +132,7 @@ __global__ void __launch_bounds__(kSortThreads) radix_hist(const uint32_t* __res
   const int64_t base = (int64_t)blockIdx.x * kSortTile;
 #pragma unroll
   for (int i = 0; i < kSortItems; ++i) {
-    int64_t idx = base + (int64_t)i * kSortThreads + threadIdx.x;
+    const int64_t idx = base + (int64_t)i * kSortThreads + threadIdx.x;
     if (idx < n) atomicAdd(&h[(keys[idx] >> shift) & (kRadix - 1)], 1);
   }
   __syncthreads();
@@ -169,7 +169,7 @@ __global__ void __launch_bounds__(kSortThreads) radix_scatter(
     const int j = warp * kWarpSlice + r * 32 + lane;
     if (j < cnt) {
       k[r] = keys_in[t0 + j];
-      v[r] = vals_in[t0 + j];
+      v[r] = vals_in ? vals_in[t0 + j] : (uint32_t)(t0 + j);  // first pass: the input position
       if (kTwo) v2[r] = vals2_in[t0 + j];
     }
   }
@@ -242,6 +242,7 @@ __global__ void __launch_bounds__(kSortThreads) radix_scatter(
 }
 
 struct SortBuffers {
+  uint32_t* ckeys;  // CSC keys, written together with the CSR keys
   uint32_t* keys[2];
   uint32_t* vals[2];
   uint32_t* vals2[2];  // second payload (carried so the finish passes read sequentially)
@@ -251,20 +252,24 @@ struct SortBuffers {
 
 static int64_t sort_tiles(int64_t n) { return std::max<int64_t>(1, ceil_div(n, kSortTile)); }
 
-// Sorts keys[0]/vals[0] (and the second payload, first read from vals2_src) by the low `bits` key
-// bits; returns the buffer index holding the result.
-static hg_status radix_sort(SortBuffers& b, int64_t n, int bits, const uint32_t* vals2_src, cudaStream_t s,
-                            int* result) {
+// Sorts (key, input position, second payload) by the low `bits` key bits (at least one pass), the
+// keys first read from keys_src and the payload from vals2_src; returns the buffer index holding
+// the result.
+static hg_status radix_sort(SortBuffers& b, int64_t n, int bits, const uint32_t* keys_src, const uint32_t* vals2_src,
+                            cudaStream_t s, int* result) {
   int cur = 0;
   const int64_t tiles = sort_tiles(n);
+  const uint32_t* k = keys_src;
+  const uint32_t* v = nullptr;  // first pass: values are the input positions
   const uint32_t* v2 = vals2_src;
-  for (int shift = 0; shift < bits; shift += 8) {
-    HG_TRY(launch("radix_hist", radix_hist, dim3((unsigned)tiles), dim3(kSortThreads), 0, s,
-                  (const uint32_t*)b.keys[cur], n, shift, b.hist, tiles));
+  for (int shift = 0; shift < std::max(bits, 1); shift += 8) {
+    HG_TRY(launch("radix_hist", radix_hist, dim3((unsigned)tiles), dim3(kSortThreads), 0, s, k, n, shift, b.hist,
+                  tiles));
     HG_TRY(exclusive_scan(b.hist, b.hist, tiles * kRadix, b.scan_scratch, s));
-    HG_TRY(launch("radix_scatter", radix_scatter<true>, dim3((unsigned)tiles), dim3(kSortThreads), 0, s,
-                  (const uint32_t*)b.keys[cur], (const uint32_t*)b.vals[cur], v2, b.keys[cur ^ 1], b.vals[cur ^ 1],
-                  b.vals2[cur ^ 1], n, shift, (const int32_t*)b.hist, tiles));
+    HG_TRY(launch("radix_scatter", radix_scatter<true>, dim3((unsigned)tiles), dim3(kSortThreads), 0, s, k, v, v2,
+                  b.keys[cur ^ 1], b.vals[cur ^ 1], b.vals2[cur ^ 1], n, shift, (const int32_t*)b.hist, tiles));
+    k = b.keys[cur ^ 1];
+    v = b.vals[cur ^ 1];
     v2 = b.vals2[cur ^ 1];
     cur ^= 1;
   }
@@ -275,24 +280,37 @@ static hg_status radix_sort(SortBuffers& b, int64_t n, int bits, const uint32_t*
 // ---------------------------------------------------------------------------------------------
 // CSR / CSC kernels
 // ---------------------------------------------------------------------------------------------
-__global__ void edge_keys(const int32_t* __restrict__ src, const int32_t* __restrict__ dst,
-                          const int32_t* __restrict__ rel, int64_t E, GraphMeta m, int by_dst,
-                          int64_t rows, uint32_t* __restrict__ keys, uint32_t* __restrict__ vals) {
+// Row keys of every edge in both layouts: CSR key = destination row, CSC key = source row;
+// invalid edges (relation or endpoint out of range, endpoint of the wrong type) get the sentinel
+// key past the last row.  The relation tables are read from shared memory.
+__global__ void __launch_bounds__(256) edge_keys(const int32_t* __restrict__ src, const int32_t* __restrict__ dst,
+                                                 const int32_t* __restrict__ rel, int64_t E, GraphMeta m,
+                                                 int64_t rows, int64_t crows, uint32_t* __restrict__ keys,
+                                                 uint32_t* __restrict__ ckeys) {
+  __shared__ int64_t row0[kMaxRels], crow0[kMaxRels];  // first row of relation r minus its type offset
+  __shared__ int32_t rsrc[kMaxRels], rdst[kMaxRels];
+  if (threadIdx.x < kMaxRels) {
+    const int r = threadIdx.x;
+    if (r < m.num_rels) {
+      rsrc[r] = m.rel_src[r];
+      rdst[r] = m.rel_dst[r];
+      row0[r] = m.row_base[r] - m.type_off[m.rel_dst[r]];
+      crow0[r] = m.csc_base[r] - m.type_off[m.rel_src[r]];
+    }
+  }
+  __syncthreads();
   const int64_t N = m.type_off[m.num_types];
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < E;
-       e += (int64_t)gridDim.x * blockDim.x) {
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < E; e += (int64_t)gridDim.x * blockDim.x) {
     const int r = rel[e];
-    const int64_t s = src[e], t = dst[e];
-    bool ok = r >= 0 && r < m.num_rels && s >= 0 && s < N && t >= 0 && t < N;
-    int64_t key = rows;  // invalid edges sort after every row
-    if (ok) {
-      ok = node_type_of(m, s) == m.rel_src[r] && node_type_of(m, t) == m.rel_dst[r];
-      if (ok)
-        key = by_dst ? m.row_base[r] + (t - m.type_off[m.rel_dst[r]])
-                     : m.csc_base[r] + (s - m.type_off[m.rel_src[r]]);
+    const int64_t sn = src[e], tn = dst[e];
+    bool ok = r >= 0 && r < m.num_rels && sn >= 0 && sn < N && tn >= 0 && tn < N;
+    int64_t key = rows, ckey = crows;  // invalid edges sort after every row
+    if (ok && node_type_of(m, sn) == rsrc[r] && node_type_of(m, tn) == rdst[r]) {
+      key = row0[r] + tn;
+      ckey = crow0[r] + sn;
     }
     keys[e] = (uint32_t)key;
-    vals[e] = (uint32_t)e;
+    ckeys[e] = (uint32_t)ckey;
   }
 }
 
@@ -387,6 +405,7 @@ static size_t carve_graph(void* ws, int64_t E, int64_t rows, int64_t crows, Grap
   L->csc_chunk_row = c.take<int32_t>(chunk_cap(E));
   L->invalid = c.take<int32_t>(1);
   L->cnt = c.take<int32_t>(std::max(rows, crows) + 1);
+  L->sort.ckeys = c.take<uint32_t>(Ea);
   for (int i = 0; i < 2; ++i) {
     L->sort.keys[i] = c.take<uint32_t>(Ea);
     L->sort.vals[i] = c.take<uint32_t>(Ea);
@@ -503,22 +522,24 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
     HG_CUDA(cudaMemsetAsync(L.csc_ptr, 0, (crows + 1) * sizeof(int32_t), s));
     HG_CUDA(cudaMemsetAsync(L.invalid, 0, sizeof(int32_t), s));
   } else {
+    // keys of both layouts in one pass (the CSR keys in keys[0], which the first sort pass reads
+    // while it writes keys[1]; the CSC keys wait in their own buffer)
+    HG_TRY(launch("edge_keys", edge_keys, dim3(g), dim3(256), 0, s, src, dst, rel, E, m, rows, crows,
+                  L.sort.keys[0], L.sort.ckeys));
     // CSR by destination
-    HG_TRY(launch("edge_keys", edge_keys, dim3(g), dim3(256), 0, s, src, dst, rel, E, m, 1, rows, L.sort.keys[0],
-                  L.sort.vals[0]));
-    HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)rows), (const uint32_t*)src, s, &res));
+    HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)rows), (const uint32_t*)L.sort.keys[0], (const uint32_t*)src, s,
+                      &res));
     HG_TRY(launch("row_ptr_from_keys", row_ptr_from_keys, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[res],
                   E, rows, L.csr_ptr));
-    const uint32_t* src_sorted = res == 0 && bit_width((uint64_t)rows) == 0 ? (const uint32_t*)src : L.sort.vals2[res];
+    const uint32_t* src_sorted = L.sort.vals2[res];
     HG_TRY(launch("csr_finish", csr_finish, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.vals[res], src_sorted,
                   (const int32_t*)L.csr_ptr, rows, E, L.csr_col, L.csr_eid, L.invalid));
     // CSC by source
-    HG_TRY(launch("edge_keys", edge_keys, dim3(g), dim3(256), 0, s, src, dst, rel, E, m, 0, crows, L.sort.keys[0],
-                  L.sort.vals[0]));
-    HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)crows), (const uint32_t*)dst, s, &res));
+    HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)crows), (const uint32_t*)L.sort.ckeys, (const uint32_t*)dst, s,
+                      &res));
     HG_TRY(launch("row_ptr_from_keys", row_ptr_from_keys, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[res],
                   E, crows, L.csc_ptr));
-    const uint32_t* dst_sorted = res == 0 && bit_width((uint64_t)crows) == 0 ? (const uint32_t*)dst : L.sort.vals2[res];
+    const uint32_t* dst_sorted = L.sort.vals2[res];
     HG_TRY(launch("csc_finish", csc_finish, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[res],
                   (const uint32_t*)L.sort.vals[res], dst_sorted, (const int32_t*)L.csc_ptr, crows, m,
                   (const int32_t*)L.csr_ptr, L.csc_col, L.csc_eid, L.csc_coef));
