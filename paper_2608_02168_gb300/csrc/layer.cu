@@ -118,7 +118,7 @@ static void carve_layer(const hg_graph* g, int d, hg_dtype dt, void* saved, void
   const int cblocks = (int)std::max<int64_t>(ceil_div(max_rows, 64), std::min<int64_t>(ceil_div(max_rows, 8), 152 * 8));
   L->cpart = k.take<float>((size_t)cblocks * 3 * d);
   const int wsplits = std::max(wgrad_splits(max_rows), wgrad_tc_splits(max_rows, d));
-  L->wpart = k.take<float>((size_t)wsplits * dd);
+  L->wpart = k.take<float>((size_t)wsplits * dd * (tc ? wgrad_tc_max_rels(d) : 1));
   L->rtmp = k.take<float>(std::max(reduce_tmp_floats(cblocks, d), reduce_tmp_floats(wsplits, (int64_t)dd)));
   if (tc) {
     L->G = k.take<float>(m.num_rels * dd);
@@ -417,15 +417,31 @@ extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* 
     if (!tc)
       HG_TRY(weight_grad(p->dtype, d, L.Z, off, L.dU, off, n, L.wpart, grads->dW_agg + (size_t)t * d * d, L.rtmp, s));
   }
-  for (int r = 0; r < m.num_rels; ++r) {
-    const int t = m.rel_dst[r];
-    const int64_t n = m.type_off[t + 1] - m.type_off[t];
-    if (tc)  // G_r = M_r^T dU
-      HG_TRY(tc_weight_grad(d, L.M, m.row_base[r], L.dU, m.type_off[t], n, L.wpart, L.G + (size_t)r * d * d, L.rtmp,
-                            s));
-    else
+  if (tc) {  // G_r = M_r^T dU, the relations into one type sharing the loads of dU
+    for (int t = 0; t < m.num_types; ++t) {
+      const int64_t n = m.type_off[t + 1] - m.type_off[t];
+      int64_t x0[kMaxRels];
+      float* outs[kMaxRels];
+      int R = 0;
+      for (int r = 0; r <= m.num_rels; ++r) {
+        if (r < m.num_rels && m.rel_dst[r] == t) {
+          x0[R] = m.row_base[r];
+          outs[R] = L.G + (size_t)r * d * d;
+          ++R;
+        }
+        if (R > 0 && (R == wgrad_tc_max_rels(d) || r == m.num_rels)) {
+          HG_TRY(tc_weight_grad(d, L.M, x0, R, L.dU, m.type_off[t], n, L.wpart, outs, L.rtmp, s));
+          R = 0;
+        }
+      }
+    }
+  } else {
+    for (int r = 0; r < m.num_rels; ++r) {
+      const int t = m.rel_dst[r];
+      const int64_t n = m.type_off[t + 1] - m.type_off[t];
       HG_TRY(weight_grad(p->dtype, d, L.M, m.row_base[r], L.dZ, m.type_off[t], n, L.wpart,
                          grads->dW_rel + (size_t)r * d * d, L.rtmp, s));
+    }
   }
   if (tc)  // dW_r = G_r W_agg^T, dW_agg[t] = sum_{r -> t} W_r^T G_r
     HG_TRY(tc_wgrad_finish(d, L.G, p->W_rel, p->W_agg, rel_dst_of(m), m.num_rels, m.num_types, grads->dW_rel,

@@ -96,8 +96,11 @@ hg_status tc_proj_forward(int d, const TcFwdArgs& a, const void* M, int64_t m_ro
                           cudaStream_t s);
 hg_status tc_ln_act_backward(int d, const TcBwdArgs& a, int* blocks, cudaStream_t s);
 hg_status tc_proj_backward(int d, const TcBwdArgs& a, const void* V, int num_rels, cudaStream_t s);
-hg_status tc_weight_grad(int d, const void* X, int64_t x0, const void* Y, int64_t y0, int64_t n, float* part,
-                         float* out, float* tmp, cudaStream_t s);
+// outs[r] = X[x0[r] .. x0[r]+n)^T Y[y0 .. y0+n) for r < R (R <= wgrad_tc_max_rels(d)); the R
+// products share the loads of Y.  part: R x wgrad_tc_splits(n, d) x d x d floats.
+hg_status tc_weight_grad(int d, const void* X, const int64_t* x0, int R, const void* Y, int64_t y0, int64_t n,
+                         float* part, float* const* outs, float* tmp, cudaStream_t s);
+int wgrad_tc_max_rels(int d);
 hg_status tc_wgrad_finish(int d, const float* G, const void* W_rel, const void* W_agg, RelDst rd, int num_rels,
                           int num_types, float* dW_rel, float* dW_agg, cudaStream_t s);
 int wgrad_tc_splits(int64_t n, int d);

@@ -31,7 +31,6 @@ using namespace tc;
 
 namespace {
 
-constexpr int kThreads = 128;
 constexpr int kTileRows = 128;
 constexpr int kATile = kTileRows * 128;  // 128 rows x 64 bf16
 
@@ -751,25 +750,28 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
 // ---------------------------------------------------------------------------------------------
 template <int D>
 struct WgCfg {
-  static constexpr int kStages = 4;
   static constexpr int kA = 2 * 8192;                  // 64 rows x 128 columns (two 64-wide blocks)
   static constexpr int kB = (D < 64 ? 64 : D) * 128;   // 64 rows x D columns
-  static constexpr int kStage = kA + kB;
-  static constexpr int kSmem = kStages * kStage + 256 + 1024;
-  static constexpr int kTmemCols = D < 32 ? 32 : D;
+  static constexpr int kAcc = D;                       // TMEM columns of one accumulator
+  static constexpr int kMaxR = D == 64 ? 5 : (D == 128 ? 4 : 2);  // relations per launch
+  static constexpr int kSmem = 227 * 1024;             // stages sized at run time within this
+  static constexpr int kThreads = 128;
 };
 
+// G_r = X_r^T Y for up to kMaxR relations r that share the operand Y (the dU rows of their common
+// destination type; X_r = the relation means M_r): each 64-row chunk of Y is loaded once and used
+// by the MMAs of every relation, each accumulating into its own TMEM region.  Grid (M tiles of 128
+// output rows, splits); part[r][split][D][D].
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1) wgrad_tc(const __grid_constant__ CUtensorMap tm_X,
-                                                       const __grid_constant__ CUtensorMap tm_Y, int64_t n,
-                                                       int chunks_per_split, float* __restrict__ part,
-                                                       int* __restrict__ status) {
+__global__ void __launch_bounds__(WgCfg<D>::kThreads, 1)
+    wgrad_tc(const __grid_constant__ RelMaps tm_X, const __grid_constant__ CUtensorMap tm_Y, int R, int S,
+             int64_t n, int chunks_per_split, float* __restrict__ part, int* __restrict__ status) {
   using C = WgCfg<D>;
-  constexpr int S = C::kStages;
   constexpr int NB = D / 64;  // 64-wide column blocks of Y
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S * C::kStage);
+  const int stage_bytes = R * C::kA + NB * 8192;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S * stage_bytes);
   uint64_t* empty = full + S;
   uint64_t* accb = empty + S;
   uint32_t* tslot = reinterpret_cast<uint32_t*>(accb + 1);
@@ -779,17 +781,19 @@ __global__ void __launch_bounds__(kThreads, 1) wgrad_tc(const __grid_constant__ 
   const int64_t c0 = (int64_t)blockIdx.y * chunks_per_split;
   const int64_t c1 = min(nchunks, c0 + chunks_per_split);
   const int CT = (int)max((int64_t)0, c1 - c0);
+  uint32_t ncols = 32;
+  while (ncols < (uint32_t)(R * C::kAcc)) ncols <<= 1;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < S; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+    for (int st = 0; st < S; ++st) {
+      mbar_init(&full[st], 1);
+      mbar_init(&empty[st], 1);
     }
     mbar_init(accb, 1);
     fence_mbar_init();
-    prefetch_tmap(&tm_X);
+    for (int r = 0; r < R; ++r) prefetch_tmap(&tm_X.m[r]);
     prefetch_tmap(&tm_Y);
   }
-  if (warp == 0) tmem_alloc(tslot, C::kTmemCols);
+  if (warp == 0) tmem_alloc(tslot, ncols);
   fence_before_sync();
   __syncthreads();
   fence_after_sync();
@@ -797,32 +801,36 @@ __global__ void __launch_bounds__(kThreads, 1) wgrad_tc(const __grid_constant__ 
   if (warp == 0) {
     if (lane == 0) {
       auto issue_load = [&](int g) {
-        const int s = g % S;
-        uint8_t* A = smem + s * C::kStage;
-        uint8_t* B = A + C::kA;
+        const int st = g % S;
+        uint8_t* stage = smem + st * stage_bytes;
+        uint8_t* B = stage + R * C::kA;
         const int y = (int)((c0 + g) * 64);
-        mbar_expect_tx(&full[s], C::kA + NB * 8192);
-        tma_load_2d(A, &tm_X, mt * 128, y, &full[s]);
-        tma_load_2d(A + 8192, &tm_X, mt * 128 + 64, y, &full[s]);
-        for (int j = 0; j < NB; ++j) tma_load_2d(B + j * 8192, &tm_Y, j * 64, y, &full[s]);
+        mbar_expect_tx(&full[st], stage_bytes);
+        for (int r = 0; r < R; ++r) {
+          tma_load_2d(stage + r * C::kA, &tm_X.m[r], mt * 128, y, &full[st]);
+          tma_load_2d(stage + r * C::kA + 8192, &tm_X.m[r], mt * 128 + 64, y, &full[st]);
+        }
+        for (int j = 0; j < NB; ++j) tma_load_2d(B + j * 8192, &tm_Y, j * 64, y, &full[st]);
       };
       const uint32_t idesc = idesc_bf16(128, D, true, true);
       bool ok = true;
       for (int g = 0; g < S && g < CT; ++g) issue_load(g);
       for (int g = 0; g < CT && ok; ++g) {
-        const int s = g % S;
-        ok = mbar_wait(&full[s], (g / S) & 1);
+        const int st = g % S;
+        ok = mbar_wait(&full[st], (g / S) & 1);
         if (!ok) break;
         fence_after_sync();
-        const uint32_t A = smem_u32(smem + s * C::kStage);
-        const uint32_t B = A + C::kA;
+        const uint32_t A0 = smem_u32(smem + st * stage_bytes);
+        const uint32_t B = A0 + R * C::kA;
+        for (int r = 0; r < R; ++r) {
 #pragma unroll
-        for (int ks = 0; ks < 4; ++ks)
-          mma_bf16(tmem, desc_sw128(A + ks * 2048, 8192, 1024), desc_sw128(B + ks * 2048, 8192, 1024), idesc,
-                   (g > 0 || ks > 0) ? 1u : 0u);
-        mma_commit(&empty[s]);
+          for (int ks = 0; ks < 4; ++ks)
+            mma_bf16(tmem + r * C::kAcc, desc_sw128(A0 + r * C::kA + ks * 2048, 8192, 1024),
+                     desc_sw128(B + ks * 2048, 8192, 1024), idesc, (g > 0 || ks > 0) ? 1u : 0u);
+        }
+        mma_commit(&empty[st]);
         if (g + S < CT) {
-          ok = mbar_wait(&empty[s], (g / S) & 1);
+          ok = mbar_wait(&empty[st], (g / S) & 1);
           if (ok) issue_load(g + S);
         }
       }
@@ -834,25 +842,27 @@ __global__ void __launch_bounds__(kThreads, 1) wgrad_tc(const __grid_constant__ 
   if (!mbar_wait(accb, 0)) atomicOr(status, kErrTimeout);
   fence_after_sync();
   const int orow = mt * 128 + warp * 32 + lane;  // output row i (column of X)
-  float* out = part + (int64_t)blockIdx.y * D * D;
+  for (int r = 0; r < R; ++r) {
+    float* out = part + ((int64_t)r * gridDim.y + blockIdx.y) * D * D;
 #pragma unroll 1
-  for (int c = 0; c < D; c += 16) {
-    float v[16];
-    if (CT > 0) {
-      tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + c, v);
-    } else {
+    for (int c = 0; c < D; c += 16) {
+      float v[16];
+      if (CT > 0) {
+        tmem_ld16(tmem + r * C::kAcc + ((uint32_t)(warp * 32) << 16) + c, v);
+      } else {
 #pragma unroll
-      for (int i = 0; i < 16; ++i) v[i] = 0.f;
-    }
-    if (orow < D) {
+        for (int i = 0; i < 16; ++i) v[i] = 0.f;
+      }
+      if (orow < D) {
 #pragma unroll
-      for (int i = 0; i < 16; i += 4)
-        *reinterpret_cast<float4*>(out + (int64_t)orow * D + c + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+        for (int i = 0; i < 16; i += 4)
+          *reinterpret_cast<float4*>(out + (int64_t)orow * D + c + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+      }
     }
   }
   fence_before_sync();
   __syncthreads();
-  if (warp == 0) tmem_dealloc(tmem, C::kTmemCols);
+  if (warp == 0) tmem_dealloc(tmem, ncols);
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -902,7 +912,16 @@ static hg_status tc_fwd_t(const TcFwdArgs& a, const void* M, int64_t m_rows, con
 
 template <int D>
 static hg_status tc_ln_act_t(const TcBwdArgs& a, int* blocks, cudaStream_t s) {
-  const int g = (int)std::max<int64_t>(1, std::min<int64_t>(ceil_div(a.n, 8), 152 * 8));
+  // one wave of resident blocks: fewer column partials to reduce afterwards
+  static int resident = 0;
+  if (resident == 0) {
+    int dev = 0, sms = 0, per_sm = 0;
+    HG_CUDA(cudaGetDevice(&dev));
+    HG_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    HG_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ln_act_bwd<D>, 256, 0));
+    resident = std::max(1, sms * per_sm);
+  }
+  const int g = (int)std::max<int64_t>(1, std::min<int64_t>(ceil_div(a.n, 8), std::min(resident, 152 * 8)));
   *blocks = g;
   return launch("ln_act_bwd", ln_act_bwd<D>, dim3(g), dim3(256), 0, s, a);
 }
@@ -934,23 +953,36 @@ int wgrad_tc_splits(int64_t n, int d) {
 }
 
 template <int D>
-static hg_status tc_wgrad_t(const void* X, int64_t x0, const void* Y, int64_t y0, int64_t n, float* part, float* out,
-                            float* tmp, cudaStream_t s) {
+static hg_status tc_wgrad_t(const void* X, const int64_t* x0, int R, const void* Y, int64_t y0, int64_t n,
+                            float* part, float* const* outs, float* tmp, cudaStream_t s) {
   HG_TRY(smem_attr_once<D>());
+  if (R < 1 || R > WgCfg<D>::kMaxR) {
+    set_error("tc_weight_grad: %d relations per launch (at most %d at d=%d)", R, WgCfg<D>::kMaxR, D);
+    return HG_ERR_UNSUPPORTED;
+  }
+  if (n == 0) {
+    for (int r = 0; r < R; ++r) HG_CUDA(cudaMemsetAsync(outs[r], 0, (size_t)D * D * sizeof(float), s));
+    return HG_OK;
+  }
   const int mtiles = D > 128 ? D / 128 : 1;
   const int splits = wgrad_tc_splits(n, D);
   const int64_t chunks = std::max<int64_t>(1, ceil_div(n, 64));
   const int cps = (int)ceil_div(chunks, splits);
-  if (n == 0) {
-    HG_CUDA(cudaMemsetAsync(out, 0, (size_t)D * D * sizeof(float), s));
-    return HG_OK;
-  }
-  CUtensorMap tm_X, tm_Y;
-  HG_TRY(make_tmap_bf16(&tm_X, (const __nv_bfloat16*)X + x0 * D, (uint64_t)n, D, 64));
+  const int stage_bytes = R * WgCfg<D>::kA + (D / 64) * 8192;
+  const int stages = std::min(4, (WgCfg<D>::kSmem - 1024 - 256) / stage_bytes);
+  RelMaps tm_X;
+  std::memset(&tm_X, 0, sizeof(tm_X));
+  for (int r = 0; r < R; ++r)
+    HG_TRY(make_tmap_bf16(&tm_X.m[r], (const __nv_bfloat16*)X + x0[r] * D, (uint64_t)n, D, 64));
+  CUtensorMap tm_Y;
   HG_TRY(make_tmap_bf16(&tm_Y, (const __nv_bfloat16*)Y + y0 * D, (uint64_t)n, D, 64));
-  HG_TRY(launch("wgrad_tc", wgrad_tc<D>, dim3(mtiles, splits), dim3(kThreads), WgCfg<D>::kSmem, s, tm_X, tm_Y, n, cps,
-                part, device_status_ptr()));
-  return reduce_partials(part, (int64_t)D * D, splits, (int64_t)D * D, out, tmp, s);
+  HG_TRY(launch("wgrad_tc", wgrad_tc<D>, dim3(mtiles, splits), dim3(WgCfg<D>::kThreads),
+                (size_t)stages * stage_bytes + 256 + 1024, s, tm_X, tm_Y, R, stages, n, cps, part,
+                device_status_ptr()));
+  for (int r = 0; r < R; ++r)
+    HG_TRY(reduce_partials(part + (size_t)r * splits * D * D, (int64_t)D * D, splits, (int64_t)D * D, outs[r], tmp,
+                           s));
+  return HG_OK;
 }
 
 template <int D>
@@ -984,10 +1016,11 @@ hg_status tc_ln_act_backward(int d, const TcBwdArgs& a, int* blocks, cudaStream_
 hg_status tc_proj_backward(int d, const TcBwdArgs& a, const void* V, int num_rels, cudaStream_t s) {
   HG_TC_DISPATCH(d, tc_bwd_t, a, V, num_rels, s);
 }
-hg_status tc_weight_grad(int d, const void* X, int64_t x0, const void* Y, int64_t y0, int64_t n, float* part,
-                         float* out, float* tmp, cudaStream_t s) {
-  HG_TC_DISPATCH(d, tc_wgrad_t, X, x0, Y, y0, n, part, out, tmp, s);
+hg_status tc_weight_grad(int d, const void* X, const int64_t* x0, int R, const void* Y, int64_t y0, int64_t n,
+                         float* part, float* const* outs, float* tmp, cudaStream_t s) {
+  HG_TC_DISPATCH(d, tc_wgrad_t, X, x0, R, Y, y0, n, part, outs, tmp, s);
 }
+int wgrad_tc_max_rels(int d) { return d == 64 ? WgCfg<64>::kMaxR : (d == 128 ? WgCfg<128>::kMaxR : WgCfg<256>::kMaxR); }
 hg_status tc_wgrad_finish(int d, const float* G, const void* W_rel, const void* W_agg, RelDst rd, int num_rels,
                           int num_types, float* dW_rel, float* dW_agg, cudaStream_t s) {
   HG_TC_DISPATCH(d, tc_finish_t, G, W_rel, W_agg, rd, num_rels, num_types, dW_rel, dW_agg, s);
