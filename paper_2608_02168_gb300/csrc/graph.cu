@@ -123,20 +123,26 @@ constexpr int kSortTile = kSortThreads * kSortItems;    // 2048 per block
 constexpr int kWarpSlice = kSortTile / kSortWarps;      // 256 consecutive items per warp
 constexpr int kRadix = 256;
 
+// Per-tile digit counts hist[digit * tiles + tile]; each warp counts into its own shared
+// histogram (atomics only contend within a warp), and the warp histograms are added at the end.
 __global__ void __launch_bounds__(kSortThreads) radix_hist(const uint32_t* __restrict__ keys, int64_t n,
                                                            int shift, int32_t* __restrict__ hist,
                                                            int64_t tiles) {
-  __shared__ int h[kRadix];
-  h[threadIdx.x] = 0;
+  __shared__ int h[kSortWarps][kRadix];
+  for (int i = threadIdx.x; i < kSortWarps * kRadix; i += kSortThreads) (&h[0][0])[i] = 0;
   __syncthreads();
+  const int warp = threadIdx.x >> 5;
   const int64_t base = (int64_t)blockIdx.x * kSortTile;
 #pragma unroll
   for (int i = 0; i < kSortItems; ++i) {
     const int64_t idx = base + (int64_t)i * kSortThreads + threadIdx.x;
-    if (idx < n) atomicAdd(&h[(keys[idx] >> shift) & (kRadix - 1)], 1);
+    if (idx < n) atomicAdd(&h[warp][(keys[idx] >> shift) & (kRadix - 1)], 1);
   }
   __syncthreads();
-  hist[(int64_t)threadIdx.x * tiles + blockIdx.x] = h[threadIdx.x];
+  int t = 0;
+#pragma unroll
+  for (int w = 0; w < kSortWarps; ++w) t += h[w][threadIdx.x];
+  hist[(int64_t)threadIdx.x * tiles + blockIdx.x] = t;
 }
 
 // Stable scatter of one 2048-item tile.  (1) Warp w reads its 256 consecutive items, 32 at a time
