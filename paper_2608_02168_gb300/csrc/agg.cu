@@ -256,7 +256,7 @@ __global__ void __launch_bounds__(256) agg_fwd_rows(const int32_t* __restrict__ 
     if (deg > kHubDegree)
       add_partials<T, D>(partials, chunk_ofs[row], chunk_ofs[row + 1], lane, acc);
     else
-      gather_sum<T, D>(col, beg, end, 1, 0, H, lane, acc);
+      gather_sum<T, D, false>(col, beg, end, 1, 0, H, lane, acc);
     const float scale = deg > 0 ? __fdiv_rn(1.0f, (float)deg) : 0.f;
     store_row<T, D>(M + row * D, lane, acc, scale);
     row = nrow;

@@ -132,12 +132,21 @@ __global__ void __launch_bounds__(kSortThreads) radix_hist(const uint32_t* __res
   for (int i = threadIdx.x; i < kSortWarps * kRadix; i += kSortThreads) (&h[0][0])[i] = 0;
   __syncthreads();
   const int warp = threadIdx.x >> 5;
-  const int64_t base = (int64_t)blockIdx.x * kSortTile;
+  // this thread's 8 consecutive keys, loaded before any of them is counted
+  const int64_t first = (int64_t)blockIdx.x * kSortTile + (int64_t)threadIdx.x * kSortItems;
+  uint32_t k[kSortItems];
+  if (first + kSortItems <= n) {
+    const uint4 a = *reinterpret_cast<const uint4*>(keys + first);
+    const uint4 b = *reinterpret_cast<const uint4*>(keys + first + 4);
+    k[0] = a.x; k[1] = a.y; k[2] = a.z; k[3] = a.w;
+    k[4] = b.x; k[5] = b.y; k[6] = b.z; k[7] = b.w;
+  } else {
 #pragma unroll
-  for (int i = 0; i < kSortItems; ++i) {
-    const int64_t idx = base + (int64_t)i * kSortThreads + threadIdx.x;
-    if (idx < n) atomicAdd(&h[warp][(keys[idx] >> shift) & (kRadix - 1)], 1);
+    for (int i = 0; i < kSortItems; ++i) k[i] = first + i < n ? keys[first + i] : 0u;
   }
+#pragma unroll
+  for (int i = 0; i < kSortItems; ++i)
+    if (first + i < n) atomicAdd(&h[warp][(k[i] >> shift) & (kRadix - 1)], 1);
   __syncthreads();
   int t = 0;
 #pragma unroll
