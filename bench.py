@@ -336,9 +336,9 @@ def run_ours(args, sp, rank, world):
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         return float(t.item())
 
-    def step(inp):
+    def step(inp, marks=None):
         kw = {k: inp[k] for k in ("X_b", "overlap_idx", "gid_a", "gid_b", "H_bank") if k in inp}
-        path.step(inp["src"], inp["dst"], inp["rel"], inp["X"], inp["dH_top"], **kw)
+        path.step(inp["src"], inp["dst"], inp["rel"], inp["X"], inp["dH_top"], marks=marks, **kw)
 
     for _ in range(max(args.warmup, 0)):
         step(devin)
@@ -360,6 +360,19 @@ def run_ours(args, sp, rank, world):
     barrier()
     clk = clocks.stop()
     t = max_over_ranks(e0.elapsed_time(e1) / 1e3)
+    # phases of the step (uninstrumented): graph build, forward layers, alignment (intersection,
+    # loss, gradient), backward layers
+    phase_ms = {}
+    for _ in range(args.steps):
+        marks = []
+        m0 = torch.cuda.Event(enable_timing=True)
+        m0.record(stream)
+        step(devin, marks)
+        torch.cuda.synchronize()
+        prev = m0
+        for name, ev in marks:
+            phase_ms[name] = phase_ms.get(name, 0.0) + prev.elapsed_time(ev) / args.steps
+            prev = ev
     # per-kernel durations (shares, roofline) from a second, instrumented run of the same steps: the
     # library records CUDA events around each of its launches, which the headline timing leaves out
     hg.hg_timing_enable(True)
@@ -431,6 +444,10 @@ def run_ours(args, sp, rank, world):
         "config": {"workload": workload_desc(sp), "l2": "inputs larger than L2 (not flushed)",
                    "parallelism": f"{world} independent subgraph(s), one per GPU"},
         "roofline": rf, "kernel_time_share": shares,
+        "phases_ms": {k: round(v, 4) for k, v in phase_ms.items()},
+        "layers_fwd_bwd_edges_per_s": edges_per_step / ((phase_ms.get("forward", 0) + phase_ms.get("backward", 0)) / 1e3)
+        if phase_ms else None,
+        "csr_build_edges_per_s": sp.num_edges / (phase_ms["graph"] / 1e3) if phase_ms.get("graph") else None,
         "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
         "gpu_launches": int(sum(n for n, _ in report.values())),
         "loss": [float(x) for x in path.loss.cpu()],

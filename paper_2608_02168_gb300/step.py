@@ -105,25 +105,37 @@ class HotPath:
 
     # --------------------------------------------------------------------------------------------
     def step(self, src, dst, rel, X, dH_top, X_b=None, overlap_idx=None, gid_a=None, gid_b=None, H_bank=None,
-             stream=None):
+             stream=None, marks=None):
         """Run one step; all inputs are device tensors.  Returns nothing (results stay in the buffers:
-        self.H, self.loss, self.grads, self.dH[s][0] = dL/dX)."""
+        self.H, self.loss, self.grads, self.dH[s][0] = dL/dX).  `marks`, if a list, receives
+        (phase, CUDA event) pairs recorded on the stream after the graph build, the forward layers,
+        the alignment and the backward layers."""
+        def mark(name):
+            if marks is not None:
+                ev = torch.cuda.Event(enable_timing=True)
+                ev.record(stream if stream is not None else torch.cuda.current_stream())
+                marks.append((name, ev))
+
         self.graph = hg.hg_build_csr(src, dst, rel, self.type_offsets, self.rels, workspace=self.graph_ws,
                                      stream=stream)
+        mark("graph")
         g = self.graph
         stacks = [X] if self.view == "bank" else [X, X_b]
         for s, x in enumerate(stacks):
             self.H[s][0] = x
             for l in range(self.L):
                 hg.hg_layer_fwd(g, self.params[l], self.H[s][l], self.H[s][l + 1], self.saved[s][l], self.scratch, stream)
+        mark("forward")
         top = self.H[0][self.L]
         self.dH[0][self.L].copy_(dH_top)
         if self.view == "bank" and H_bank is None:
             # first subgraph of a sequence: no neighbour view yet, no alignment term
             self.loss.zero_()
+            mark("alignment")
             for l in range(self.L - 1, -1, -1):
                 hg.hg_layer_bwd(g, self.params[l], self.H[0][l], self.saved[0][l], self.dH[0][l + 1], self.dH[0][l],
                                 self.grads[0][l], self.scratch, stream)
+            mark("backward")
             return
         if self.view == "bank":
             hg.hg_overlap_intersect(gid_a, gid_b, self.idx_a, self.idx_b, self.n_dev, self.isect_scratch, stream)
@@ -139,10 +151,12 @@ class HotPath:
                                  self.align_scratch, stream)
         hg.hg_overlap_align_bwd(top, ia, Hb, ib, n_max, n_dev, LAMBDA_N, VAR_EPS, LAMBDA_CCA, self.align_saved,
                                 self.dH[0][self.L], dHb, self.align_scratch, stream)
+        mark("alignment")
         for s in range(len(stacks)):
             for l in range(self.L - 1, -1, -1):
                 hg.hg_layer_bwd(g, self.params[l], self.H[s][l], self.saved[s][l], self.dH[s][l + 1], self.dH[s][l],
                                 self.grads[s][l], self.scratch, stream)
+        mark("backward")
 
 
 class Ring:
