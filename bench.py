@@ -201,7 +201,7 @@ def kernel_models(st: dict, sp) -> dict:
     m["proj_fwd_tc"] = (L * tf, L * tfl)
     m["ln_act_bwd"] = (L * lb, 0)
     m["proj_bwd_tc"] = (L * pb, L * pfl)
-    m["wgrad_tc"] = (L * 2 * row * RR, L * 2 * d * d * RR)  # G_r = M_r^T dU: read both operands once
+    m["wgrad_tc"] = (L * row * (RR + N), L * 2 * d * d * RR)  # G_r = M_r^T dU: M_r rows once, dU once per type
     m["radix_scatter"] = (2 * 3 * 2 * 12 * st["E"], 0)  # 2 layouts x 3 passes x read+write of key, edge id, endpoint
     no = st["n_ov"]
     m["align_colstats"] = (3 * 2 * no * (row + 4), 0)        # 3 passes over both gathered views
