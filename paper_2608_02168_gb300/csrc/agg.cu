@@ -2,9 +2,11 @@
 // transpose for the backward pass.
 //
 // Forward:  M_r[j] = (1/deg_r(j)) * sum_{(i -> j) in r} H[i]          (CSR row j of relation r)
-// Backward: dH[i]  = dY[i] + sum_r sum_{(i -> j) in r} dMs_r[j]         (CSC row i of relation r)
+// Backward: dH[i]  = dY[i] + sum_r sum_{(i -> j) in r} dMs_r[j]
 //           where dMs_r[j] = dM_r[j] / deg_r(j) is produced, already scaled, by the projection
-//           backward kernel, and dY[i] is the residual-path gradient of Eq. 11.
+//           backward kernel, and dY[i] is the residual-path gradient of Eq. 11.  The sum runs over
+//           node i's row of the node-major out-edge list (its CSC rows of every relation leaving
+//           its type, concatenated in relation order, each edge holding the dMs row it reads).
 //
 // Mapping: one group of G lanes per row, each lane owning 16-byte slices of the feature row
 // (G = d * sizeof(T) / 16, at most 32), gathers with 128-bit loads and eight neighbour rows in
@@ -185,12 +187,11 @@ __device__ __forceinline__ void store_row(T* __restrict__ dst, int lane, const f
 }
 
 // One CTA per chunk (grid-stride over the chunk list): fp32 partial sum of the chunk's rows.
-// rel_of_row: for CSC chunks the relation decides the index shift applied to csc_col.
 template <typename T, int D>
 __global__ void __launch_bounds__(256) agg_chunks(const int32_t* __restrict__ ptr, const int32_t* __restrict__ col,
                                                   const T* __restrict__ src, const int32_t* __restrict__ chunk_row,
                                                   const int32_t* __restrict__ chunk_ofs, int64_t rows,
-                                                  GraphMeta m, int transposed, float* __restrict__ partials) {
+                                                  float* __restrict__ partials) {
   using S = AggShape<T, D>;
   __shared__ float red[S::kGroups][D];
   const int grp = threadIdx.x / S::G, lane = threadIdx.x % S::G;
@@ -199,18 +200,10 @@ __global__ void __launch_bounds__(256) agg_chunks(const int32_t* __restrict__ pt
     const int row = chunk_row[c];
     const int64_t beg = (int64_t)ptr[row] + (int64_t)(c - chunk_ofs[row]) * kChunkEdges;
     const int64_t end = min((int64_t)ptr[row + 1], beg + kChunkEdges);
-    int64_t delta = 0;
-    if (transposed) {
-      int r = 0;
-#pragma unroll
-      for (int k = 1; k < kMaxRels; ++k)
-        if (k < m.num_rels && row >= m.csc_base[k]) r = k;
-      delta = m.row_base[r] - m.type_off[m.rel_dst[r]];
-    }
     float acc[S::F];
 #pragma unroll
     for (int q = 0; q < S::F; ++q) acc[q] = 0.f;
-    gather_sum<T, D, false>(col, beg + grp, end, S::kGroups, delta, src, lane, acc);
+    gather_sum<T, D, false>(col, beg + grp, end, S::kGroups, 0, src, lane, acc);
 #pragma unroll
     for (int v = 0; v < S::V; ++v)
 #pragma unroll
@@ -265,30 +258,30 @@ __global__ void __launch_bounds__(256) agg_fwd_rows(const int32_t* __restrict__ 
   }
 }
 
-// Backward nodes: dH[i] = dY[i] + sum over relations with source type tau(i) of the CSC row sums.
-// Persistent: each group strides over nodes.
+// Backward nodes: dH[i] = dY[i] + sum of the node's row in the node-major out-edge list (every
+// relation leaving its type, relation by relation, each edge holding the dMs row it reads).
+// Persistent: each group strides over nodes and fetches the next node's bounds while it gathers.
 template <typename T, int D>
-__global__ void __launch_bounds__(256) agg_bwd_nodes(GraphMeta m, const int32_t* __restrict__ cptr,
-                                                     const int32_t* __restrict__ ccol, const T* __restrict__ dMs,
+__global__ void __launch_bounds__(256) agg_bwd_nodes(int64_t N, const int32_t* __restrict__ nptr,
+                                                     const int32_t* __restrict__ ncol, const T* __restrict__ dMs,
                                                      const T* __restrict__ dY, T* __restrict__ dH,
                                                      const int32_t* __restrict__ chunk_ofs,
                                                      const float* __restrict__ partials) {
   using S = AggShape<T, D>;
   const int grp = threadIdx.x / S::G, lane = threadIdx.x % S::G;
-  const int64_t N = m.type_off[m.num_types];
   const int64_t step = (int64_t)gridDim.x * S::kGroups;
-  for (int64_t node = (int64_t)blockIdx.x * S::kGroups + grp; node < N; node += step) {
-    const int t = node_type_of(m, node);
-    // the node's CSC bounds in every relation leaving its type, all loaded before any gather
-    int beg[kMaxRels], end[kMaxRels];
-#pragma unroll
-    for (int r = 0; r < kMaxRels; ++r) {
-      beg[r] = end[r] = 0;
-      if (r < m.num_rels && m.rel_src[r] == t) {
-        const int64_t crow = m.csc_base[r] + (node - m.type_off[t]);
-        beg[r] = __ldg(cptr + crow);
-        end[r] = __ldg(cptr + crow + 1);
-      }
+  int64_t node = (int64_t)blockIdx.x * S::kGroups + grp;
+  int beg = 0, end = 0;
+  if (node < N) {
+    beg = __ldg(nptr + node);
+    end = __ldg(nptr + node + 1);
+  }
+  while (node < N) {
+    const int64_t next = node + step;
+    int nbeg = 0, nend = 0;
+    if (next < N) {
+      nbeg = __ldg(nptr + next);
+      nend = __ldg(nptr + next + 1);
     }
     float acc[S::F];
 #pragma unroll
@@ -298,17 +291,14 @@ __global__ void __launch_bounds__(256) agg_bwd_nodes(GraphMeta m, const int32_t*
 #pragma unroll
       for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] = f[q];
     }
-#pragma unroll
-    for (int r = 0; r < kMaxRels; ++r) {
-      if (end[r] == beg[r]) continue;
-      if (end[r] - beg[r] > kHubDegree) {
-        const int64_t crow = m.csc_base[r] + (node - m.type_off[t]);
-        add_partials<T, D>(partials, chunk_ofs[crow], chunk_ofs[crow + 1], lane, acc);
-      } else {
-        gather_sum<T, D>(ccol, beg[r], end[r], 1, m.row_base[r] - m.type_off[m.rel_dst[r]], dMs, lane, acc);
-      }
-    }
+    if (end - beg > kHubDegree)
+      add_partials<T, D>(partials, chunk_ofs[node], chunk_ofs[node + 1], lane, acc);
+    else
+      gather_sum<T, D>(ncol, beg, end, 1, 0, dMs, lane, acc);
     store_row<T, D>(dH + node * D, lane, acc, 1.0f);
+    node = next;
+    beg = nbeg;
+    end = nend;
   }
 }
 
@@ -333,8 +323,7 @@ static hg_status agg_fwd_t(const hg_graph* g, const void* H, void* M, float* par
   using S = AggShape<T, D>;
   HG_TRY(launch("agg_fwd_chunks", agg_chunks<T, D>, dim3(chunk_grid(g->chunk_cap_csr)), dim3(256), 0, s,
                 (const int32_t*)g->csr_ptr, (const int32_t*)g->csr_col, (const T*)H,
-                (const int32_t*)g->csr_chunk_row, (const int32_t*)g->csr_chunk_ofs, g->csr_rows, g->meta, 0,
-                partials));
+                (const int32_t*)g->csr_chunk_row, (const int32_t*)g->csr_chunk_ofs, g->csr_rows, partials));
   HG_TRY(launch("combine_chunk_partials", combine_chunk_partials<D>, dim3(chunk_grid(g->chunk_cap_csr)), dim3(D), 0, s,
                 (const int32_t*)g->csr_chunk_row, (const int32_t*)g->csr_chunk_ofs, g->csr_rows, partials));
   static int64_t pb = 0;
@@ -350,20 +339,18 @@ template <typename T, int D>
 static hg_status agg_bwd_t(const hg_graph* g, const void* dMs, const void* dY, void* dH, float* partials,
                            cudaStream_t s) {
   using S = AggShape<T, D>;
-  HG_TRY(launch("agg_bwd_chunks", agg_chunks<T, D>, dim3(chunk_grid(g->chunk_cap_csc)), dim3(256), 0, s,
-                (const int32_t*)g->csc_ptr, (const int32_t*)g->csc_col, (const T*)dMs,
-                (const int32_t*)g->csc_chunk_row, (const int32_t*)g->csc_chunk_ofs, g->csc_rows, g->meta, 1,
-                partials));
-  HG_TRY(launch("combine_chunk_partials", combine_chunk_partials<D>, dim3(chunk_grid(g->chunk_cap_csc)), dim3(D), 0, s,
-                (const int32_t*)g->csc_chunk_row, (const int32_t*)g->csc_chunk_ofs, g->csc_rows, partials));
   const int64_t N = g->meta.type_off[g->meta.num_types];
+  HG_TRY(launch("agg_bwd_chunks", agg_chunks<T, D>, dim3(chunk_grid(g->chunk_cap_node)), dim3(256), 0, s,
+                (const int32_t*)g->node_ptr, (const int32_t*)g->node_col, (const T*)dMs,
+                (const int32_t*)g->node_chunk_row, (const int32_t*)g->node_chunk_ofs, N, partials));
+  HG_TRY(launch("combine_chunk_partials", combine_chunk_partials<D>, dim3(chunk_grid(g->chunk_cap_node)), dim3(D), 0,
+                s, (const int32_t*)g->node_chunk_row, (const int32_t*)g->node_chunk_ofs, N, partials));
   static int64_t pb = 0;
   if (pb == 0) HG_TRY(persist_blocks(agg_bwd_nodes<T, D>, &pb));
   return launch("agg_bwd_nodes", agg_bwd_nodes<T, D>,
-                dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(N, S::kGroups), pb))),
-                dim3(256), 0, s,
-                g->meta, (const int32_t*)g->csc_ptr, (const int32_t*)g->csc_col, (const T*)dMs, (const T*)dY,
-                (T*)dH, (const int32_t*)g->csc_chunk_ofs, (const float*)partials);
+                dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(N, S::kGroups), pb))), dim3(256), 0, s,
+                N, (const int32_t*)g->node_ptr, (const int32_t*)g->node_col, (const T*)dMs, (const T*)dY, (T*)dH,
+                (const int32_t*)g->node_chunk_ofs, (const float*)partials);
 }
 
 #define HG_DISPATCH_TD(dtype, d, FN, ...)                                                   \

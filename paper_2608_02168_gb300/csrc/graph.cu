@@ -357,10 +357,35 @@ __global__ void csr_finish(const uint32_t* __restrict__ eid_sorted, const uint32
 
 // CSC arrays from the sorted (row key, edge id, destination id) triples; the relation is read off
 // the key, 1/deg_r(destination) from the CSR row pointers.
+// Out-degree of every node over all relations leaving its type (the length of its node-major row).
+__global__ void node_out_counts(const int32_t* __restrict__ cptr, GraphMeta m, int32_t* __restrict__ cnt) {
+  __shared__ int64_t cbase[kMaxRels];  // CSC row of the type's node 0 in relation r, minus the type offset
+  __shared__ int32_t rsrc[kMaxRels];
+  if (threadIdx.x < kMaxRels) {
+    const int r = threadIdx.x;
+    rsrc[r] = r < m.num_rels ? m.rel_src[r] : -1;
+    if (r < m.num_rels) cbase[r] = m.csc_base[r] - m.type_off[m.rel_src[r]];
+  }
+  __syncthreads();
+  const int64_t N = m.type_off[m.num_types];
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < N; i += (int64_t)gridDim.x * blockDim.x) {
+    const int t = node_type_of(m, i);
+    int c = 0;
+#pragma unroll
+    for (int r = 0; r < kMaxRels; ++r)
+      if (rsrc[r] == t) c += cptr[cbase[r] + i + 1] - cptr[cbase[r] + i];
+    cnt[i] = c;
+  }
+}
+
+// CSC arrays per relation, and the node-major list of out-edges used by the backward aggregation:
+// node i's row holds, relation by relation (ascending) and in CSC order within a relation, the
+// dMs row of each edge's destination (row_base[r] + local destination id).
 __global__ void csc_finish(const uint32_t* __restrict__ key_sorted, const uint32_t* __restrict__ eid_sorted,
                            const uint32_t* __restrict__ dst_sorted, const int32_t* __restrict__ cptr, int64_t crows,
-                           GraphMeta m, const int32_t* __restrict__ csr_ptr, int32_t* __restrict__ ccol,
-                           int32_t* __restrict__ ceid, float* __restrict__ coef) {
+                           GraphMeta m, const int32_t* __restrict__ csr_ptr, const int32_t* __restrict__ nptr,
+                           int32_t* __restrict__ ccol, int32_t* __restrict__ ceid, float* __restrict__ coef,
+                           int32_t* __restrict__ ncol) {
   const int64_t nv = cptr[crows];
   for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < nv;
        p += (int64_t)gridDim.x * blockDim.x) {
@@ -375,6 +400,14 @@ __global__ void csc_finish(const uint32_t* __restrict__ key_sorted, const uint32
     ceid[p] = (int32_t)eid_sorted[p];
     ccol[p] = j;
     coef[p] = __fdiv_rn(1.0f, (float)deg);
+    // node-major position: the node's row start, the edges of its earlier relations, the rank in this one
+    const int t = m.rel_src[r];
+    const int64_t il = key - m.csc_base[r];  // type-local source id
+    int64_t pos = nptr[m.type_off[t] + il] + (p - cptr[key]);
+#pragma unroll
+    for (int k = 0; k < kMaxRels; ++k)
+      if (k < r && m.rel_src[k] == t) pos += cptr[m.csc_base[k] + il + 1] - cptr[m.csc_base[k] + il];
+    ncol[pos] = (int32_t)row;
   }
 }
 
@@ -400,11 +433,12 @@ static int64_t chunk_cap(int64_t E) { return E / kChunkEdges + E / (kHubDegree +
 struct GraphLayout {
   int32_t *csr_ptr, *csr_col, *csr_eid, *csc_ptr, *csc_col, *csc_eid;
   float* csc_coef;
-  int32_t *csr_chunk_ofs, *csr_chunk_row, *csc_chunk_ofs, *csc_chunk_row, *invalid, *cnt;
+  int32_t *node_ptr, *node_col;  // node-major out-edges (dMs rows) for the backward aggregation
+  int32_t *csr_chunk_ofs, *csr_chunk_row, *node_chunk_ofs, *node_chunk_row, *invalid, *cnt;
   SortBuffers sort;
 };
 
-static size_t carve_graph(void* ws, int64_t E, int64_t rows, int64_t crows, GraphLayout* L) {
+static size_t carve_graph(void* ws, int64_t E, int64_t rows, int64_t crows, int64_t N, GraphLayout* L) {
   Carve c(ws);
   const int64_t Ea = std::max<int64_t>(E, 1);
   L->csr_ptr = c.take<int32_t>(rows + 1);
@@ -414,12 +448,14 @@ static size_t carve_graph(void* ws, int64_t E, int64_t rows, int64_t crows, Grap
   L->csc_col = c.take<int32_t>(Ea);
   L->csc_eid = c.take<int32_t>(Ea);
   L->csc_coef = c.take<float>(Ea);
+  L->node_ptr = c.take<int32_t>(N + 1);
+  L->node_col = c.take<int32_t>(Ea);
   L->csr_chunk_ofs = c.take<int32_t>(rows + 1);
   L->csr_chunk_row = c.take<int32_t>(chunk_cap(E));
-  L->csc_chunk_ofs = c.take<int32_t>(crows + 1);
-  L->csc_chunk_row = c.take<int32_t>(chunk_cap(E));
+  L->node_chunk_ofs = c.take<int32_t>(N + 1);
+  L->node_chunk_row = c.take<int32_t>(chunk_cap(E));
   L->invalid = c.take<int32_t>(1);
-  L->cnt = c.take<int32_t>(std::max(rows, crows) + 1);
+  L->cnt = c.take<int32_t>(std::max(std::max(rows, crows), N) + 1);
   L->sort.ckeys = c.take<uint32_t>(Ea);
   for (int i = 0; i < 2; ++i) {
     L->sort.keys[i] = c.take<uint32_t>(Ea);
@@ -428,7 +464,7 @@ static size_t carve_graph(void* ws, int64_t E, int64_t rows, int64_t crows, Grap
   }
   const int64_t hist_n = sort_tiles(E) * kRadix;
   L->sort.hist = c.take<int32_t>(hist_n + 1);
-  L->sort.scan_scratch = c.take<char>(scan_scratch_bytes(std::max(std::max(hist_n, rows), crows)));
+  L->sort.scan_scratch = c.take<char>(scan_scratch_bytes(std::max(std::max(hist_n, rows), std::max(crows, N))));
   return c.used;
 }
 
@@ -499,7 +535,7 @@ extern "C" hg_status hg_graph_workspace_size(int64_t num_edges, const int64_t* t
   GraphMeta m;
   HG_TRY(make_meta(type_offsets, num_types, rels, num_rels, &m));
   GraphLayout L;
-  *bytes = carve_graph(nullptr, num_edges, m.row_base[num_rels], m.csc_base[num_rels], &L);
+  *bytes = carve_graph(nullptr, num_edges, m.row_base[num_rels], m.csc_base[num_rels], m.type_off[m.num_types], &L);
   return HG_OK;
 }
 
@@ -522,12 +558,13 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
   HG_TRY(make_meta(type_offsets, num_types, rels, num_rels, &m));
   const int64_t E = num_edges, rows = m.row_base[num_rels], crows = m.csc_base[num_rels];
   GraphLayout L;
-  const size_t need = carve_graph(nullptr, E, rows, crows, &L);
+  const int64_t N = m.type_off[num_types];
+  const size_t need = carve_graph(nullptr, E, rows, crows, N, &L);
   if (workspace_bytes < need) {
     set_error("workspace has %zu bytes, %zu needed", workspace_bytes, need);
     return HG_ERR_WORKSPACE;
   }
-  carve_graph(workspace, E, rows, crows, &L);
+  carve_graph(workspace, E, rows, crows, N, &L);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
 
   const unsigned g = grid_for(E + 1);
@@ -535,6 +572,7 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
   if (E == 0) {
     HG_CUDA(cudaMemsetAsync(L.csr_ptr, 0, (rows + 1) * sizeof(int32_t), s));
     HG_CUDA(cudaMemsetAsync(L.csc_ptr, 0, (crows + 1) * sizeof(int32_t), s));
+    HG_CUDA(cudaMemsetAsync(L.node_ptr, 0, (N + 1) * sizeof(int32_t), s));
     HG_CUDA(cudaMemsetAsync(L.invalid, 0, sizeof(int32_t), s));
   } else {
     // keys of both layouts in one pass (the CSR keys in keys[0], which the first sort pass reads
@@ -555,9 +593,14 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
     HG_TRY(launch("row_ptr_from_keys", row_ptr_from_keys, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[res],
                   E, crows, L.csc_ptr));
     const uint32_t* dst_sorted = L.sort.vals2[res];
+    // node-major rows: out-degree per node over its relations, their scan, then the edges
+    HG_TRY(launch("node_out_counts", node_out_counts, dim3(grid_for(N)), dim3(256), 0, s, (const int32_t*)L.csc_ptr,
+                  m, L.cnt));
+    HG_TRY(exclusive_scan(L.cnt, L.node_ptr, N, L.sort.scan_scratch, s));
     HG_TRY(launch("csc_finish", csc_finish, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[res],
                   (const uint32_t*)L.sort.vals[res], dst_sorted, (const int32_t*)L.csc_ptr, crows, m,
-                  (const int32_t*)L.csr_ptr, L.csc_col, L.csc_eid, L.csc_coef));
+                  (const int32_t*)L.csr_ptr, (const int32_t*)L.node_ptr, L.csc_col, L.csc_eid, L.csc_coef,
+                  L.node_col));
   }
   // chunk tables for rows above the hub degree
   HG_TRY(launch("chunk_counts", chunk_counts, dim3(grid_for(rows)), dim3(256), 0, s,
@@ -565,11 +608,11 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
   HG_TRY(exclusive_scan(L.cnt, L.csr_chunk_ofs, rows, L.sort.scan_scratch, s));
   HG_TRY(launch("chunk_fill", chunk_fill, dim3(grid_for(rows)), dim3(256), 0, s,
                 (const int32_t*)L.csr_chunk_ofs, rows, L.csr_chunk_row));
-  HG_TRY(launch("chunk_counts", chunk_counts, dim3(grid_for(crows)), dim3(256), 0, s,
-                (const int32_t*)L.csc_ptr, crows, L.cnt));
-  HG_TRY(exclusive_scan(L.cnt, L.csc_chunk_ofs, crows, L.sort.scan_scratch, s));
-  HG_TRY(launch("chunk_fill", chunk_fill, dim3(grid_for(crows)), dim3(256), 0, s,
-                (const int32_t*)L.csc_chunk_ofs, crows, L.csc_chunk_row));
+  HG_TRY(launch("chunk_counts", chunk_counts, dim3(grid_for(N)), dim3(256), 0, s,
+                (const int32_t*)L.node_ptr, N, L.cnt));
+  HG_TRY(exclusive_scan(L.cnt, L.node_chunk_ofs, N, L.sort.scan_scratch, s));
+  HG_TRY(launch("chunk_fill", chunk_fill, dim3(grid_for(N)), dim3(256), 0, s,
+                (const int32_t*)L.node_chunk_ofs, N, L.node_chunk_row));
 
   hg_graph* gh = new hg_graph{};
   gh->meta = m;
@@ -577,7 +620,7 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
   gh->csr_rows = rows;
   gh->csc_rows = crows;
   gh->chunk_cap_csr = chunk_cap(E);
-  gh->chunk_cap_csc = chunk_cap(E);
+  gh->chunk_cap_node = chunk_cap(E);
   gh->stream = s;
   gh->csr_ptr = L.csr_ptr;
   gh->csr_col = L.csr_col;
@@ -588,8 +631,10 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
   gh->csc_coef = L.csc_coef;
   gh->csr_chunk_ofs = L.csr_chunk_ofs;
   gh->csr_chunk_row = L.csr_chunk_row;
-  gh->csc_chunk_ofs = L.csc_chunk_ofs;
-  gh->csc_chunk_row = L.csc_chunk_row;
+  gh->node_ptr = L.node_ptr;
+  gh->node_col = L.node_col;
+  gh->node_chunk_ofs = L.node_chunk_ofs;
+  gh->node_chunk_row = L.node_chunk_row;
   gh->invalid_count = L.invalid;
   *out = gh;
   return HG_OK;

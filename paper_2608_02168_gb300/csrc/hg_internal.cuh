@@ -109,7 +109,7 @@ struct hg_graph {
   int64_t csr_rows;       // meta.row_base[num_rels]
   int64_t csc_rows;       // meta.csc_base[num_rels]
   int64_t chunk_cap_csr;  // capacity of the chunk tables
-  int64_t chunk_cap_csc;
+  int64_t chunk_cap_node;
   cudaStream_t stream;    // build stream (hg_graph_check synchronises it)
   int32_t* csr_ptr;       // [csr_rows + 1]
   int32_t* csr_col;       // [num_edges] (valid prefix)
@@ -120,8 +120,10 @@ struct hg_graph {
   float* csc_coef;
   int32_t* csr_chunk_ofs;  // [csr_rows + 1] exclusive scan of chunks per row (0 for rows <= hub degree)
   int32_t* csr_chunk_row;  // [chunk_cap_csr] CSR row of each chunk
-  int32_t* csc_chunk_ofs;
-  int32_t* csc_chunk_row;
+  int32_t* node_ptr;        // [N + 1] node-major out-edges over all relations (backward aggregation)
+  int32_t* node_col;        // [num_edges] dMs row of each out-edge's destination
+  int32_t* node_chunk_ofs;  // [N + 1] chunks per node-major row above the hub degree
+  int32_t* node_chunk_row;
   int32_t* invalid_count;  // device scalar
 };
 

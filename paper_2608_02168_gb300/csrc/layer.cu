@@ -108,7 +108,7 @@ static void carve_layer(const hg_graph* g, int d, hg_dtype dt, void* saved, void
     L->V = s.take<char>(m.num_rels * dd * b);
     L->Vt = s.take<char>(m.num_rels * dd * b);
   }
-  L->agg_part = k.take<float>((size_t)std::max(g->chunk_cap_csr, g->chunk_cap_csc) * d);
+  L->agg_part = k.take<float>((size_t)std::max(g->chunk_cap_csr, g->chunk_cap_node) * d);
   L->dY = k.take<char>((size_t)N * d * b);
   L->dU = k.take<char>((size_t)N * d * b);
   if (!tc) L->dZ = k.take<char>((size_t)N * d * b);
