@@ -408,11 +408,9 @@ extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* 
       HG_TRY(proj_backward(p->dtype, d, a, s));
       blocks = (int)ceil_div(n, 64);
     }
-    HG_TRY(reduce_partials(L.cpart, 3LL * d, blocks, d, db, L.rtmp, s));
-    if (p->layernorm) {
-      HG_TRY(reduce_partials(L.cpart + d, 3LL * d, blocks, d, grads->dln_gamma + (size_t)t * d, L.rtmp, s));
-      HG_TRY(reduce_partials(L.cpart + 2 * d, 3LL * d, blocks, d, grads->dln_beta + (size_t)t * d, L.rtmp, s));
-    }
+    HG_TRY(reduce_partials3(L.cpart, 3LL * d, blocks, d, db,
+                            p->layernorm ? grads->dln_gamma + (size_t)t * d : nullptr,
+                            p->layernorm ? grads->dln_beta + (size_t)t * d : nullptr, s));
     const int64_t off = m.type_off[t];
     if (!tc)
       HG_TRY(weight_grad(p->dtype, d, L.Z, off, L.dU, off, n, L.wpart, grads->dW_agg + (size_t)t * d * d, L.rtmp, s));

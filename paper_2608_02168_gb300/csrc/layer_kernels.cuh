@@ -119,6 +119,10 @@ hg_status transpose_weights(hg_dtype dt, int d, const void* W, void* Wt, int cou
 hg_status reduce_partials(const float* part, int64_t stride, int splits, int64_t count, float* out, float* tmp,
                           cudaStream_t s);
 size_t reduce_tmp_floats(int splits, int64_t count);
+// The same over the first 1 to 3 segments of `seg` entries of each partial (entry k * seg + i of a
+// partial adds into out_k[i]); out1 / out2 NULL = fewer segments.
+hg_status reduce_partials3(const float* part, int64_t stride, int splits, int64_t seg, float* out0, float* out1,
+                           float* out2, cudaStream_t s);
 int wgrad_splits(int64_t n);
 
 }  // namespace hg

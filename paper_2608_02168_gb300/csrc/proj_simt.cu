@@ -312,8 +312,12 @@ __global__ void __launch_bounds__(256) wgrad_partial(const T* __restrict__ X, in
 // outputs (one per lane); warp w sums the splits k = w, w + kRedLanes, ... in ascending order, and the
 // kRedLanes warp sums are added in warp order.
 constexpr int kRedLanes = 32;
+// Outputs i in [k * seg, (k + 1) * seg) go to outs.p[k][i - k * seg] (up to three segments).
+struct RedOuts {
+  float* p[3];
+};
 __global__ void __launch_bounds__(32 * kRedLanes) reduce_lanes(const float* __restrict__ part, int64_t stride,
-                                                             int splits, int64_t count, float* __restrict__ out) {
+                                                             int splits, int64_t count, int64_t seg, RedOuts outs) {
   __shared__ float red[kRedLanes][33];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int64_t i = (int64_t)blockIdx.x * 32 + lane;
@@ -335,7 +339,8 @@ __global__ void __launch_bounds__(32 * kRedLanes) reduce_lanes(const float* __re
     float t = 0.f;
 #pragma unroll
     for (int k = 0; k < kRedLanes; ++k) t += red[k][lane];
-    out[i] = t;
+    const int64_t q = i / seg;
+    outs.p[q][i - q * seg] = t;
   }
 }
 
@@ -440,8 +445,19 @@ hg_status reduce_partials(const float* part, int64_t stride, int splits, int64_t
                           cudaStream_t s) {
   (void)tmp;
   if (count <= 0) return HG_OK;
+  RedOuts o{{out, nullptr, nullptr}};
   return launch("reduce_lanes", reduce_lanes, dim3((unsigned)ceil_div(count, 32)), dim3(32 * kRedLanes), 0, s, part,
-                stride, splits, count, out);
+                stride, splits, count, count, o);
+}
+
+hg_status reduce_partials3(const float* part, int64_t stride, int splits, int64_t seg, float* out0, float* out1,
+                           float* out2, cudaStream_t s) {
+  const int nseg = out1 ? (out2 ? 3 : 2) : 1;
+  const int64_t count = seg * nseg;
+  if (count <= 0) return HG_OK;
+  RedOuts o{{out0, out1, out2}};
+  return launch("reduce_lanes", reduce_lanes, dim3((unsigned)ceil_div(count, 32)), dim3(32 * kRedLanes), 0, s, part,
+                stride, splits, count, seg, o);
 }
 
 }  // namespace hg
