@@ -175,10 +175,20 @@ def kernel_models(st: dict, sp) -> dict:
     f, bw = st["fwd"], st["bwd"]
     row = d * b
     m = {}
-    m["agg_fwd_rows"] = (L * (4 * (RR + 1) + 4 * f["E_nh"] + row * f["U_nh"] + row * RR + 4 * d * f["chunks"]), 0)
-    m["agg_fwd_chunks"] = (L * (4 * f["E_h"] + row * f["U_h"] + 4 * d * f["chunks"]), 0)
-    m["agg_bwd_nodes"] = (L * (4 * (CC + 1) + 4 * bw["E_nh"] + row * bw["U_nh"] + 2 * row * N + 4 * d * bw["chunks"]), 0)
-    m["agg_bwd_chunks"] = (L * (4 * bw["E_h"] + row * bw["U_h"] + 4 * d * bw["chunks"]), 0)
+    # aggregation, per unit of work = one gathered edge: its 4-byte index and one feature row, with no
+    # cache reuse assumed (the per-edge model; 1/deg is folded into dMs, so the transposed pass reads
+    # no per-edge coefficient).  The compulsory bytes (each distinct row once) are in `compulsory`.
+    ge = 4 + row
+    m["agg_fwd_rows"] = (L * f["E_nh"] * ge, 0)
+    m["agg_fwd_chunks"] = (L * f["E_h"] * ge, 0)
+    m["agg_bwd_nodes"] = (L * bw["E_nh"] * ge, 0)
+    m["agg_bwd_chunks"] = (L * bw["E_h"] * ge, 0)
+    m["compulsory"] = {
+        "agg_fwd_rows": L * (4 * (RR + 1) + 4 * f["E_nh"] + row * f["U_nh"] + row * RR + 4 * d * f["chunks"]),
+        "agg_fwd_chunks": L * (4 * f["E_h"] + row * f["U_h"] + 4 * d * f["chunks"]),
+        "agg_bwd_nodes": L * (4 * (N + 1) + 4 * bw["E_nh"] + row * bw["U_nh"] + 2 * row * N + 4 * d * bw["chunks"]),
+        "agg_bwd_chunks": L * (4 * bw["E_h"] + row * bw["U_h"] + 4 * d * bw["chunks"]),
+    }
     fb = ff = bb = bf = 0
     for t in st["types"]:
         n, R = t["n"], t["R"]
@@ -238,10 +248,10 @@ def measured_traffic(kernel: str):
     return int(entry["bytes_per_launch"]) if h.hexdigest() == entry["sha256"] else None
 
 
-def roofline(report: dict, models: dict, steps: int, peaks: dict, src: str) -> tuple:
+def roofline(report: dict, models: dict, steps: int, peaks: dict, src: str, dom=None) -> tuple:
     total = sum(ms for _, ms in report.values()) or 1.0
     shares = {k: round(ms / total, 4) for k, (_, ms) in sorted(report.items(), key=lambda kv: -kv[1][1])}
-    dom = max(report, key=lambda k: report[k][1])
+    dom = dom or max(report, key=lambda k: report[k][1])
     n, ms = report[dom]
     by, fl = models.get(dom, (0, 0))
     secs = ms / 1e3
@@ -258,6 +268,10 @@ def roofline(report: dict, models: dict, steps: int, peaks: dict, src: str) -> t
     rf["traffic"] = measured_traffic(dom)
     rf.update(kernel=dom, launches=n, avg_launch_ms=round(ms / max(n, 1), 4),
               algorithmic_bytes_per_launch=int(by * steps / max(n, 1)), flops_per_launch=int(fl * steps / max(n, 1)))
+    comp = models.get("compulsory", {}).get(dom)
+    if comp is not None:
+        rf["compulsory_bytes_per_launch"] = int(comp * steps / max(n, 1))
+        rf["compulsory_frac"] = round(comp * steps / secs / 1e9 / peaks["hbm_gbs"], 4) if secs > 0 else None
     return rf, shares
 
 
@@ -431,6 +445,9 @@ def run_ours(args, sp, rank, world):
         return
     peaks, psrc = load_peaks()
     rf, shares = roofline(report, models, args.steps, peaks, psrc)
+    # the same figures for every modelled kernel among the largest shares
+    top = [k for k in shares if k in models and k != "compulsory"][:8]
+    kernel_rooflines = [roofline(report, models, args.steps, peaks, psrc, dom=k)[0] for k in top]
     cpu = None
     if not args.no_cpu_baseline:
         o = time_oracle(sp.name, ORACLE_SCALE)
@@ -443,7 +460,7 @@ def run_ours(args, sp, rank, world):
         "dtype": sp.dtype, "data": "synthetic",
         "config": {"workload": workload_desc(sp), "l2": "inputs larger than L2 (not flushed)",
                    "parallelism": f"{world} independent subgraph(s), one per GPU"},
-        "roofline": rf, "kernel_time_share": shares,
+        "roofline": rf, "kernel_rooflines": kernel_rooflines, "kernel_time_share": shares,
         "phases_ms": {k: round(v, 4) for k, v in phase_ms.items()},
         "layers_fwd_bwd_edges_per_s": edges_per_step / ((phase_ms.get("forward", 0) + phase_ms.get("backward", 0)) / 1e3)
         if phase_ms else None,
