@@ -116,10 +116,10 @@ hg_status exclusive_scan(const int32_t* in, int32_t* out, int64_t n, void* scrat
 // ---------------------------------------------------------------------------------------------
 // stable LSD radix sort of (uint32 key, uint32 value) pairs, 8-bit digits
 // ---------------------------------------------------------------------------------------------
-constexpr int kSortThreads = 256;
+constexpr int kSortThreads = 512;
 constexpr int kSortWarps = kSortThreads / 32;
 constexpr int kSortItems = 8;                           // per thread
-constexpr int kSortTile = kSortThreads * kSortItems;    // 2048 per block
+constexpr int kSortTile = kSortThreads * kSortItems;    // 4096 per block
 constexpr int kWarpSlice = kSortTile / kSortWarps;      // 256 consecutive items per warp
 constexpr int kRadix = 256;
 
@@ -148,13 +148,15 @@ __global__ void __launch_bounds__(kSortThreads) radix_hist(const uint32_t* __res
   for (int i = 0; i < kSortItems; ++i)
     if (first + i < n) atomicAdd(&h[warp][(k[i] >> shift) & (kRadix - 1)], 1);
   __syncthreads();
-  int t = 0;
+  if (threadIdx.x < kRadix) {
+    int t = 0;
 #pragma unroll
-  for (int w = 0; w < kSortWarps; ++w) t += h[w][threadIdx.x];
-  hist[(int64_t)threadIdx.x * tiles + blockIdx.x] = t;
+    for (int w = 0; w < kSortWarps; ++w) t += h[w][threadIdx.x];
+    hist[(int64_t)threadIdx.x * tiles + blockIdx.x] = t;
+  }
 }
 
-// Stable scatter of one 2048-item tile.  (1) Warp w reads its 256 consecutive items, 32 at a time
+// Stable scatter of one 4096-item tile.  (1) Warp w reads its 256 consecutive items, 32 at a time
 // (coalesced), into registers.  (2) It ranks them round by round with __match_any_sync, keeping
 // per-digit running counts, so the item order inside the tile is (warp, round, lane).  (3) Per-digit
 // prefixes over warps and over digits give every item its position in the tile sorted by digit
@@ -167,16 +169,18 @@ __global__ void __launch_bounds__(kSortThreads) radix_scatter(
     const uint32_t* __restrict__ vals2_in, uint32_t* __restrict__ keys_out, uint32_t* __restrict__ vals_out,
     uint32_t* __restrict__ vals2_out, int64_t n, int shift, const int32_t* __restrict__ offs, int64_t tiles) {
   constexpr int R = kWarpSlice / 32;  // rounds (items per thread)
-  __shared__ uint32_t skey[kSortTile], sval[kSortTile];  // sorted tile
-  __shared__ uint32_t sval2[kTwo ? kSortTile : 1];
-  __shared__ int whist[kSortWarps][kRadix];
+  extern __shared__ uint32_t sort_smem[];
+  uint32_t* skey = sort_smem;           // sorted tile
+  uint32_t* sval = skey + kSortTile;
+  uint32_t* sval2 = sval + kSortTile;   // (kTwo)
+  int (*whist)[kRadix] = reinterpret_cast<int (*)[kRadix]>(sval2 + (kTwo ? kSortTile : 0));
   __shared__ int dstart[kRadix];  // tile position where each digit's run starts
   __shared__ int gbase[kRadix];   // global position of the digit's run of this tile
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t t0 = (int64_t)blockIdx.x * kSortTile;
   const int cnt = (int)min((int64_t)kSortTile, n - t0);
   for (int i = threadIdx.x; i < kSortWarps * kRadix; i += kSortThreads) (&whist[0][0])[i] = 0;
-  gbase[threadIdx.x] = offs[(int64_t)threadIdx.x * tiles + blockIdx.x];
+  if (threadIdx.x < kRadix) gbase[threadIdx.x] = offs[(int64_t)threadIdx.x * tiles + blockIdx.x];
   uint32_t k[R], v[R], v2[R];
   int rank[R];
 #pragma unroll
@@ -202,7 +206,7 @@ __global__ void __launch_bounds__(kSortThreads) radix_scatter(
     rank[r] = c + __popc(peers & lt_mask);
   }
   __syncthreads();
-  {  // per digit: exclusive prefix over warps; tile total
+  if (threadIdx.x < kRadix) {  // per digit: exclusive prefix over warps; tile total
     int run = 0;
 #pragma unroll
     for (int w = 0; w < kSortWarps; ++w) {
@@ -266,12 +270,19 @@ struct SortBuffers {
 };
 
 static int64_t sort_tiles(int64_t n) { return std::max<int64_t>(1, ceil_div(n, kSortTile)); }
+// dynamic shared memory of radix_scatter<true>: the sorted tile (key, value, payload), warp histograms
+constexpr size_t kScatterSmem = 3 * kSortTile * sizeof(uint32_t) + kSortWarps * kRadix * sizeof(int);
 
 // Sorts (key, input position, second payload) by the low `bits` key bits (at least one pass), the
 // keys first read from keys_src and the payload from vals2_src; returns the buffer index holding
 // the result.
 static hg_status radix_sort(SortBuffers& b, int64_t n, int bits, const uint32_t* keys_src, const uint32_t* vals2_src,
                             cudaStream_t s, int* result) {
+  static bool attr = false;
+  if (!attr) {
+    HG_CUDA(cudaFuncSetAttribute(radix_scatter<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kScatterSmem));
+    attr = true;
+  }
   int cur = 0;
   const int64_t tiles = sort_tiles(n);
   const uint32_t* k = keys_src;
@@ -281,7 +292,7 @@ static hg_status radix_sort(SortBuffers& b, int64_t n, int bits, const uint32_t*
     HG_TRY(launch("radix_hist", radix_hist, dim3((unsigned)tiles), dim3(kSortThreads), 0, s, k, n, shift, b.hist,
                   tiles));
     HG_TRY(exclusive_scan(b.hist, b.hist, tiles * kRadix, b.scan_scratch, s));
-    HG_TRY(launch("radix_scatter", radix_scatter<true>, dim3((unsigned)tiles), dim3(kSortThreads), 0, s, k, v, v2,
+    HG_TRY(launch("radix_scatter", radix_scatter<true>, dim3((unsigned)tiles), dim3(kSortThreads), kScatterSmem, s, k, v, v2,
                   b.keys[cur ^ 1], b.vals[cur ^ 1], b.vals2[cur ^ 1], n, shift, (const int32_t*)b.hist, tiles));
     k = b.keys[cur ^ 1];
     v = b.vals[cur ^ 1];
