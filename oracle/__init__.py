@@ -4,3 +4,4 @@ from .hg_oracle import (  # noqa: F401
     align_backward, align_forward, build_csr, layer_backward, layer_backward_rows, layer_forward,
     layer_forward_rows, mean_aggregate, overlap_intersect, standardise, step, valid_edges,
 )
+from . import overlap_build  # noqa: F401  (overlapping-subgraph construction, Eq. 4-5)
