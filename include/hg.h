@@ -243,6 +243,41 @@ hg_status hg_overlap_align_loss_static(const void* H_a, int64_t rows_a, const in
                                        void* saved, hg_stream stream);
 
 /* ------------------------------------------------------------------------------------------- */
+/* Overlapping subgraph construction (Section 3.1, Eq. 4-5; Algorithm 1, construction loop)      */
+/* ------------------------------------------------------------------------------------------- */
+
+/* Subgraph k of K built from a global graph with global node ids [0, num_nodes), contiguous per
+ * node type:
+ *   base V_k     = { v : splitmix64(part_seed ^ v) mod K == k }   (random hash partition), where
+ *                  splitmix64(x) is the SplitMix64 output for state x (x + 0x9E3779B97F4A7C15,
+ *                  then the generator's two xor-shift-multiply steps and final xor-shift);
+ *   degree(v)    = incident edges over all relations, both directions (a self-loop twice);
+ *   h-index(v)   = the largest h with at least h incident edges leading to nodes of degree >= h;
+ *   C_k          = nodes outside V_k with an edge v -> u, u in V_k                        (Eq. 4);
+ *   C'_k         = the v in C_k with h-index(v) <= theta;
+ *   C_{k,M}      = the M members of C'_k with the smallest key (high 32 bits of
+ *                  splitmix64(sample_seed ^ (k << 40) ^ v)), ties by id; all of C'_k when fewer;
+ *   V~_k         = V_k united with C_{k,M}                                                (Eq. 5);
+ *   the induced subgraph: the edges with both endpoints in V~_k, in input order.
+ * Local ids follow ascending global id (so node types stay contiguous).  Edges with an endpoint
+ * outside [0, num_nodes) are ignored (neither incident nor induced).
+ * Inputs (device): src, dst, rel [num_edges].  type_offsets (HOST, num_types + 1) are the global
+ * type boundaries.  Outputs (device, capacities num_nodes / num_edges, entries past the counts
+ * untouched): gid_out (int64, ascending global ids of V~_k), src_out / dst_out (local ids),
+ * rel_out, eid_out (input edge ids), type_offsets_out (int64 [num_types + 1], local type
+ * boundaries), h_out (int32 [num_nodes] h-index of every global node; may be NULL), counts_out
+ * (int64 [6]: nodes, base nodes, expansion nodes, edges, |C_k|, |C'_k|).  K >= 1, 0 <= k < K,
+ * theta >= 0, M >= 0, num_nodes < 2^31, num_edges < 2^31; otherwise HG_ERR_INVALID_ARG or
+ * HG_ERR_UNSUPPORTED.  Integer work: the results are exact and reproducible. */
+hg_status hg_overlap_build_workspace_size(int64_t num_nodes, int64_t num_edges, size_t* bytes);
+hg_status hg_overlap_build(const int32_t* src, const int32_t* dst, const int32_t* rel, int64_t num_edges,
+                           int64_t num_nodes, const int64_t* type_offsets, int32_t num_types, int32_t K,
+                           int32_t k, int32_t theta, int64_t M, uint64_t part_seed, uint64_t sample_seed,
+                           int64_t* gid_out, int32_t* src_out, int32_t* dst_out, int32_t* rel_out,
+                           int32_t* eid_out, int64_t* type_offsets_out, int32_t* h_out, int64_t* counts_out,
+                           void* workspace, size_t workspace_bytes, hg_stream stream);
+
+/* ------------------------------------------------------------------------------------------- */
 /* Kernel timing (measurement support; off by default)                                          */
 /* ------------------------------------------------------------------------------------------- */
 

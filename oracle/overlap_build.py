@@ -22,7 +22,8 @@ Readings where the paper is silent or ambiguous (listed again in the design note
   (a counter-based generator, so both sides implement it from its definition);
   A_vu != 0 in Eq. 4 is an edge v -> u (messages from v reach the partition);
   a node's incident edges count both directions and every relation, multi-edges and self-loops
-  included (a self-loop is incident twice);
+  included (a self-loop is incident twice); edges with an endpoint outside the node range are
+  ignored;
   the paper writes "sample b nodes" and "TopM": the M candidates with the smallest sampling keys
   hash(sample_seed XOR (k << 40) XOR v) (high 32 bits), ties by global id -- a uniform sample
   without replacement in a reproducible order.
@@ -118,9 +119,10 @@ def build(src, dst, rel, type_offsets, K: int, k: int, theta: int, M: int, part_
     dst = np.asarray(dst, np.int64)
     rel = np.asarray(rel, np.int64)
     N = int(type_offsets[-1])
+    ok = (src >= 0) & (src < N) & (dst >= 0) & (dst < N)  # other edges are ignored
     part = partition(N, K, part_seed)
-    c_all = candidates(src, dst, part, k)
-    h = h_index(src, dst, N)
+    c_all = candidates(src[ok], dst[ok], part, k)
+    h = h_index(src[ok], dst[ok], N)
     cand = c_all[h[c_all] <= theta]  # C'_k
     keys = sample_keys(cand, k, sample_seed)
     order = np.lexsort((cand, keys))  # key ascending, ties by global id
@@ -130,9 +132,10 @@ def build(src, dst, rel, type_offsets, K: int, k: int, theta: int, M: int, part_
     gid = np.nonzero(member)[0].astype(np.int64)
     local = np.full(N, -1, dtype=np.int64)
     local[gid] = np.arange(len(gid))
-    keep = member[src] & member[dst]
+    keep = ok.copy()
+    keep[ok] = member[src[ok]] & member[dst[ok]]
     eid = np.nonzero(keep)[0].astype(np.int64)
     offs = np.searchsorted(gid, np.asarray(type_offsets, np.int64))
-    return {"gid": gid, "n_base": int((part == k).sum()), "expanded": chosen,
+    return {"gid": gid, "n_base": int((part == k).sum()), "expanded": chosen, "h": h,
             "type_offsets": offs.astype(np.int64), "src": local[src[keep]], "dst": local[dst[keep]],
             "rel": rel[keep], "eid": eid, "num_candidates": int(len(c_all)), "num_filtered": int(len(cand))}

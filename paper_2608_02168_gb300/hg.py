@@ -8,7 +8,7 @@ from __future__ import annotations
 
 import ctypes
 import os
-from ctypes import POINTER, Structure, byref, c_char_p, c_float, c_int32, c_int64, c_size_t, c_void_p
+from ctypes import POINTER, Structure, byref, c_char_p, c_float, c_int32, c_int64, c_size_t, c_uint64, c_void_p
 
 import torch
 
@@ -71,6 +71,10 @@ EXPORTS = {
     "hg_overlap_align_loss_static": (c_int32, [c_void_p, c_int64, c_void_p, c_void_p, c_int64, c_void_p, c_int64,
                                                c_void_p, c_int32, c_int32, c_float, c_float, c_void_p, c_void_p,
                                                c_void_p]),
+    "hg_overlap_build_workspace_size": (c_int32, [c_int64, c_int64, POINTER(c_size_t)]),
+    "hg_overlap_build": (c_int32, [c_void_p, c_void_p, c_void_p, c_int64, c_int64, POINTER(c_int64), c_int32, c_int32,
+                                   c_int32, c_int32, c_int64, c_uint64, c_uint64, c_void_p, c_void_p, c_void_p,
+                                   c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
     "hg_timing_enable": (c_int32, [c_int32]),
     "hg_timing_report": (c_int32, [c_char_p, c_size_t]),
 }
@@ -323,3 +327,45 @@ def hg_timing_report() -> dict:
         name, n, ms = line.split()
         out[name] = (int(n), float(ms))
     return out
+
+
+# -------------------------------------------------------------------------------------------------
+# overlapping subgraph construction
+# -------------------------------------------------------------------------------------------------
+def hg_overlap_build_workspace_size(num_nodes: int, num_edges: int) -> int:
+    n = c_size_t(0)
+    _check(lib().hg_overlap_build_workspace_size(int(num_nodes), int(num_edges), byref(n)),
+           "hg_overlap_build_workspace_size")
+    return n.value
+
+
+def hg_overlap_build(src, dst, rel, type_offsets, K: int, k: int, theta: int, M: int, part_seed: int,
+                     sample_seed: int, workspace=None, with_h: bool = False, stream=None) -> dict:
+    """Overlapping subgraph k of K of a global graph (device tensors src, dst, rel; host list
+    type_offsets).  Returns device tensors trimmed to the counts (one synchronisation to read them):
+    gid, src, dst, rel, eid, type_offsets, h (when with_h), and the counts as a dict."""
+    import torch
+    dev = src.device
+    N, E = int(type_offsets[-1]), int(src.numel())
+    T = len(type_offsets) - 1
+    if workspace is None:
+        workspace = torch.empty(hg_overlap_build_workspace_size(N, E), dtype=torch.uint8, device=dev)
+    gid = torch.empty(max(N, 1), dtype=torch.int64, device=dev)
+    out = {k2: torch.empty(max(E, 1), dtype=torch.int32, device=dev) for k2 in ("src", "dst", "rel", "eid")}
+    toff = torch.empty(T + 1, dtype=torch.int64, device=dev)
+    h = torch.empty(max(N, 1), dtype=torch.int32, device=dev) if with_h else None
+    counts = torch.empty(6, dtype=torch.int64, device=dev)
+    offs = (c_int64 * (T + 1))(*[int(x) for x in type_offsets])
+    _check(lib().hg_overlap_build(_ptr(src), _ptr(dst), _ptr(rel), E, N, offs, T, int(K), int(k), int(theta), int(M),
+                                  int(part_seed) & (2**64 - 1), int(sample_seed) & (2**64 - 1), _ptr(gid),
+                                  _ptr(out["src"]), _ptr(out["dst"]), _ptr(out["rel"]), _ptr(out["eid"]), _ptr(toff),
+                                  _ptr(h), _ptr(counts), _ptr(workspace), workspace.numel(), _stream(stream)),
+           "hg_overlap_build")
+    c = [int(x) for x in counts.cpu()]
+    names = ("nodes", "base", "expanded", "edges", "candidates", "filtered")
+    res = {"gid": gid[:c[0]], "type_offsets": toff, "counts": dict(zip(names, c))}
+    res.update({k2: v[:c[3]] for k2, v in out.items()})
+    if with_h:
+        res["h"] = h[:N]
+    return res
+

@@ -1,0 +1,90 @@
+"""Overlapping-subgraph construction on the GPU against the oracle, bit-exact (integer work)."""
+import numpy as np
+import pytest
+import torch
+
+import hgsynth
+from oracle import overlap_build as ob
+from tests.gpu_util import dev, lib, need_gpu
+
+pytestmark = pytest.mark.gpu
+
+
+def run(hg, src, dst, rel, offs, K, k, theta, M, ps=5, ss=9):
+    out = hg.hg_overlap_build(dev(src, torch.int32), dev(dst, torch.int32), dev(rel, torch.int32), list(offs), K, k,
+                              theta, M, ps, ss, with_h=True)
+    ref = ob.build(src, dst, rel, np.asarray(offs, np.int64), K, k, theta, M, ps, ss)
+    return out, ref
+
+
+def compare(out, ref, check_h=True):
+    c = out["counts"]
+    assert c["nodes"] == len(ref["gid"]) and c["base"] == ref["n_base"] and c["expanded"] == len(ref["expanded"])
+    assert c["edges"] == len(ref["eid"]) and c["candidates"] == ref["num_candidates"]
+    assert c["filtered"] == ref["num_filtered"]
+    np.testing.assert_array_equal(out["gid"].cpu().numpy(), ref["gid"])
+    np.testing.assert_array_equal(out["type_offsets"].cpu().numpy(), ref["type_offsets"])
+    for key in ("src", "dst", "rel", "eid"):
+        np.testing.assert_array_equal(out[key].cpu().numpy().astype(np.int64), ref[key], err_msg=key)
+    if check_h:
+        np.testing.assert_array_equal(out["h"].cpu().numpy().astype(np.int64), ref["h"])
+
+
+def random_graph(seed, n_user, n_risk, e, bad=0):
+    rng = np.random.default_rng(seed)
+    n = n_user + n_risk
+    src = rng.integers(0, n, e)
+    dst = rng.integers(0, n, e)
+    rel = rng.integers(0, 3, e)
+    if bad:
+        i = rng.choice(e, bad, replace=False)
+        src[i[: bad // 2]] = n + rng.integers(0, 5, bad // 2)
+        dst[i[bad // 2:]] = -1 - rng.integers(0, 5, bad - bad // 2)
+    return src.astype(np.int32), dst.astype(np.int32), rel.astype(np.int32), [0, n_user, n]
+
+
+@pytest.mark.parametrize("K,k,theta,M,bad", [(4, 0, 2, 50, 0), (4, 3, 1, 10_000, 40), (3, 1, 6, 0, 0),
+                                             (1, 0, 2, 100, 10), (8, 5, 0, 7, 0), (2, 1, 3, 123, 7)])
+def test_random_graphs(K, k, theta, M, bad):
+    need_gpu()
+    src, dst, rel, offs = random_graph(K * 7 + k, 900, 300, 6000, bad)
+    out, ref = run(lib(), src, dst, rel, offs, K, k, theta, M)
+    compare(out, ref)
+
+
+def test_power_law_graph_with_big_lists():
+    """tiny-10k as the global graph: power-law hubs with incidence lists above the CTA threshold
+    (4096 entries), long-tail candidates, the 15 % budget of the paper's setting."""
+    need_gpu()
+    g = hgsynth.make_graph(hgsynth.spec("tiny-10k"))
+    src, dst, rel = g["src"], g["dst"], g["rel"]
+    offs = [int(x) for x in g["type_offsets"]]
+    deg = np.bincount(src, minlength=offs[-1]) + np.bincount(dst, minlength=offs[-1])
+    assert deg.max() > 4096
+    M = int(0.15 * offs[-1] / 4)
+    for k in (0, 2):
+        out, ref = run(lib(), src, dst, rel, offs, 4, k, 2, M, ps=11, ss=13)
+        compare(out, ref)
+        c = out["counts"]
+        assert c["expanded"] == min(M, c["filtered"]) > 0
+
+
+def test_ties_and_budget_edges():
+    """Budgets below, at and above the number of eligible candidates select exactly the smallest
+    keys (ties by id), and an empty edge list gives the base partition alone."""
+    need_gpu()
+    hg = lib()
+    src, dst, rel, offs = random_graph(5, 400, 100, 3000)
+    ref_all = ob.build(src, dst, rel, np.asarray(offs), 3, 2, 10, 10**9, 1, 2)
+    f = ref_all["num_filtered"]
+    for M in (1, f - 1, f, f + 1):
+        out, ref = run(hg, src, dst, rel, offs, 3, 2, 10, M, 1, 2)
+        compare(out, ref, check_h=False)
+    e = np.zeros(0, np.int32)
+    out = hg.hg_overlap_build(torch.zeros(0, dtype=torch.int32, device="cuda"),
+                              torch.zeros(0, dtype=torch.int32, device="cuda"),
+                              torch.zeros(0, dtype=torch.int32, device="cuda"), offs, 3, 1, 2, 50, 1, 2)
+    ref = ob.build(e, e, e, np.asarray(offs), 3, 1, 2, 50, 1, 2)
+    assert out["counts"]["nodes"] == len(ref["gid"]) and out["counts"]["edges"] == 0
+    np.testing.assert_array_equal(out["gid"].cpu().numpy(), ref["gid"])
+    assert hg.hg_device_status() == 0

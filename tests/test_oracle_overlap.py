@@ -102,3 +102,15 @@ def test_overlap_between_subgraphs_exists():
     b = ob.build(src, dst, rel, offs, 4, 1, 50, 200, 1, 2)
     shared = np.intersect1d(a["gid"], b["gid"])
     assert len(shared) > 0  # Eq. 5: the expanded sets create overlaps between subgraphs
+
+
+def test_out_of_range_edges_are_ignored():
+    src, dst, rel = _random_graph(21, 50, 200)
+    offs = np.array([0, 40, 50], np.int64)
+    clean = ob.build(src, dst, rel, offs, 3, 1, 3, 20, 1, 2)
+    bad_src = np.concatenate([src, [-1, 7, 60]])
+    bad_dst = np.concatenate([dst, [3, 99, 2]])
+    bad_rel = np.concatenate([rel, [0, 1, 2]])
+    dirty = ob.build(bad_src, bad_dst, bad_rel, offs, 3, 1, 3, 20, 1, 2)
+    for key in ("gid", "expanded", "src", "dst", "rel", "eid", "h"):
+        np.testing.assert_array_equal(clean[key], dirty[key])
