@@ -31,6 +31,7 @@ import hgsynth  # noqa: E402
 METRIC = "GNN layer fwd+bwd edges/sec on 1 GB300; achieved HBM GB/s vs roofline"
 UNIT = "edges/s"
 ORACLE_SCALE = 40        # the CPU baseline runs the oracle on a 1/40-size instance of the workload
+BUILD_K, BUILD_THETA, BUILD_BUDGET = 8, 2, 0.15  # overlapping-subgraph construction: parts, h-index bound, M / N
 REFERENCE_SCALE = 100    # each reference-arm step runs the oracle on a 1/100-size instance
 FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "sm_max_mhz": 2070.0}
 
@@ -44,7 +45,9 @@ def parse():
     ap.add_argument("--workload", default="sub-1m", choices=sorted(hgsynth.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-build", action="store_true", help="skip the subgraph-construction measurement")
     ap.add_argument("--oracle-sample", type=int, default=0, help=argparse.SUPPRESS)  # internal: child process
+    ap.add_argument("--oracle-build-sample", type=int, default=0, help=argparse.SUPPRESS)  # internal: child process
     return ap.parse_args()
 
 
@@ -75,10 +78,22 @@ def oracle_sample_main(name: str, k: int):
                       "value": sp.layers * sp.num_edges / dt}))
 
 
-def time_oracle(name: str, k: int) -> dict:
+def oracle_build_sample_main(name: str, k: int):
+    """Child process: the construction oracle on a 1/k-size instance of the workload's graph."""
+    from oracle import overlap_build as ob
+    sp = scaled(hgsynth.spec(name), k)
+    g = hgsynth.make_graph(sp)
+    offs = np.asarray(g["type_offsets"], np.int64)
+    t0 = time.perf_counter()
+    ob.build(g["src"], g["dst"], g["rel"], offs, BUILD_K, 0, BUILD_THETA, int(BUILD_BUDGET * offs[-1] / BUILD_K), 21, 22)
+    dt = time.perf_counter() - t0
+    print(json.dumps({"seconds": dt, "edges": sp.num_edges, "value": sp.num_edges / dt}))
+
+
+def time_oracle(name: str, k: int, flag: str = "--oracle-sample") -> dict:
     env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
                CUDA_VISIBLE_DEVICES="")
-    r = subprocess.run([sys.executable, os.path.abspath(__file__), "--workload", name, "--oracle-sample", str(k)],
+    r = subprocess.run([sys.executable, os.path.abspath(__file__), "--workload", name, flag, str(k)],
                        capture_output=True, text=True, env=env)
     if r.returncode != 0:
         raise RuntimeError(f"oracle sample failed: {r.stderr[-2000:]}")
@@ -275,11 +290,71 @@ def roofline(report: dict, models: dict, steps: int, peaks: dict, src: str, dom=
     return rf, shares
 
 
+def measure_overlap_build(w, steps: int, warmup: int, dev, with_cpu: bool) -> dict:
+    """The overlapping-subgraph construction (Section 3.1; done once before training, so it is not
+    part of the step) on the workload's graph taken as the global graph: subgraph 0 of BUILD_K,
+    h-index bound BUILD_THETA, budget BUILD_BUDGET * N / BUILD_K.  Device time per call."""
+    import torch
+    from paper_2608_02168_gb300 import hg
+    g = w.graph
+    offs = [int(x) for x in g["type_offsets"]]
+    src, dst, rel = (torch.from_numpy(g[k]).to(dev) for k in ("src", "dst", "rel"))
+    ws = torch.empty(hg.hg_overlap_build_workspace_size(offs[-1], len(g["src"])), dtype=torch.uint8, device=dev)
+    M = int(BUILD_BUDGET * offs[-1] / BUILD_K)
+
+    def call():
+        return hg.hg_overlap_build(src, dst, rel, offs, BUILD_K, 0, BUILD_THETA, M, 21, 22, workspace=ws)
+
+    for _ in range(max(warmup, 1)):
+        out = call()
+    torch.cuda.synchronize()
+    # the binding reads the counts back (one synchronisation per call): time with events per call
+    times = []
+    for _ in range(steps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        out = call()
+        e1.record()
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1))
+    hg.hg_timing_enable(True)
+    hg.hg_timing_report()
+    call()
+    torch.cuda.synchronize()
+    hg.hg_timing_enable(False)
+    rep = hg.hg_timing_report()
+    tot = sum(ms for _, ms in rep.values()) or 1.0
+    ms = statistics.median(times)
+    # algorithmic bytes of one call: per edge, the endpoint reads of the degree, list-fill, candidate
+    # and keep passes (4 x 8 B), the neighbour degrees and list slots written by the fill (2 x 8 B),
+    # one read of both incidence entries by the h-index (8 B) and the keep flag (4 B); per node, the
+    # ten 4-byte node arrays written and read once (40 B)
+    peaks, psrc = load_peaks()
+    byt = 60 * len(g["src"]) + 40 * offs[-1]
+    ach = byt / (ms / 1e3) / 1e9
+    res = {"ms": round(ms, 4), "edges_per_s": len(g["src"]) / (ms / 1e3), "counts": out["counts"],
+           "roofline": {"bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                        "peak_source": f"{psrc} hbm_gbs", "frac": round(ach / peaks["hbm_gbs"], 4),
+                        "algorithmic_bytes_per_call": int(byt), "scope": "whole call"},
+           "config": {"K": BUILD_K, "k": 0, "theta": BUILD_THETA, "M": M},
+           "kernel_time_share": {k: round(v / tot, 4) for k, (_, v) in sorted(rep.items(), key=lambda kv: -kv[1][1])},
+           "cpu_baseline": None}
+    if with_cpu:
+        o = time_oracle(w.spec.name, ORACLE_SCALE, "--oracle-build-sample")
+        res["cpu_baseline"] = {"value": o["value"], "unit": "edges/s", "cores": 1, "kind": "oracle",
+                               "sample": f"1/{ORACLE_SCALE}-size instance ({o['edges']:,} edges), numpy oracle, one "
+                                         f"thread, {o['seconds']:.1f} s"}
+    return res
+
+
 # ------------------------------------------------------------------------------------------------
 def main():
     args = parse()
     if args.oracle_sample:
         oracle_sample_main(args.workload, args.oracle_sample)
+        return
+    if args.oracle_build_sample:
+        oracle_build_sample_main(args.workload, args.oracle_build_sample)
         return
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -443,6 +518,9 @@ def run_ours(args, sp, rank, world):
         if world > 1:
             torch.distributed.destroy_process_group()
         return
+    build = None
+    if not args.no_build:
+        build = measure_overlap_build(w, args.steps, args.warmup, dev, not args.no_cpu_baseline)
     peaks, psrc = load_peaks()
     rf, shares = roofline(report, models, args.steps, peaks, psrc)
     # the same figures for every modelled kernel among the largest shares
@@ -465,7 +543,7 @@ def run_ours(args, sp, rank, world):
         "layers_fwd_bwd_edges_per_s": edges_per_step / ((phase_ms.get("forward", 0) + phase_ms.get("backward", 0)) / 1e3)
         if phase_ms else None,
         "csr_build_edges_per_s": sp.num_edges / (phase_ms["graph"] / 1e3) if phase_ms.get("graph") else None,
-        "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+        "cpu_baseline": cpu, "e2e": e2e, "clocks": clk, "overlap_build": build,
         "gpu_launches": int(sum(n for n, _ in report.values())),
         "loss": [float(x) for x in path.loss.cpu()],
     }

@@ -43,13 +43,33 @@ __device__ __forceinline__ bool edge_ok(int32_t s, int32_t t, int64_t N) {
   return s >= 0 && s < N && t >= 0 && t < N;
 }
 
+// Warp-aggregated increment of ctr[key] by the lanes holding the same key (key < 0: none);
+// returns this lane's slot: the counter's old value plus its rank among those lanes.  Hub nodes
+// recur within a warp's edges, so one atomic serves all of a hub's occurrences.
+__device__ __forceinline__ int aggregated_claim(int32_t* ctr, int key) {
+  const int lane = threadIdx.x & 31;
+  const unsigned peers = __match_any_sync(0xffffffffu, key);
+  const int leader = __ffs(peers) - 1;
+  int base = 0;
+  if (key >= 0 && lane == leader) base = atomicAdd(&ctr[key], __popc(peers));
+  base = __shfl_sync(0xffffffffu, base, leader);
+  return base + __popc(peers & ((1u << lane) - 1u));
+}
+
+// (the loops run whole warps together: lanes past the end take key -1)
 __global__ void ob_degrees(const int32_t* __restrict__ src, const int32_t* __restrict__ dst, int64_t E, int64_t N,
                            int32_t* __restrict__ deg) {
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < E; e += (int64_t)gridDim.x * blockDim.x) {
-    const int32_t s = src[e], t = dst[e];
-    if (!edge_ok(s, t, N)) continue;
-    atomicAdd(&deg[s], 1);
-    atomicAdd(&deg[t], 1);
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); e0 < E; e0 += stride) {
+    const int64_t e = e0 + (threadIdx.x & 31);
+    int32_t s = -1, t = -1;
+    if (e < E) {
+      s = src[e];
+      t = dst[e];
+      if (!edge_ok(s, t, N)) s = t = -1;
+    }
+    aggregated_claim(deg, s);
+    aggregated_claim(deg, t);
   }
 }
 
@@ -57,11 +77,21 @@ __global__ void ob_degrees(const int32_t* __restrict__ src, const int32_t* __res
 __global__ void ob_fill_lists(const int32_t* __restrict__ src, const int32_t* __restrict__ dst, int64_t E, int64_t N,
                               const int32_t* __restrict__ deg, const int32_t* __restrict__ ofs,
                               int32_t* __restrict__ fill, int32_t* __restrict__ nbr) {
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < E; e += (int64_t)gridDim.x * blockDim.x) {
-    const int32_t s = src[e], t = dst[e];
-    if (!edge_ok(s, t, N)) continue;
-    nbr[ofs[s] + atomicAdd(&fill[s], 1)] = deg[t];
-    nbr[ofs[t] + atomicAdd(&fill[t], 1)] = deg[s];
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); e0 < E; e0 += stride) {
+    const int64_t e = e0 + (threadIdx.x & 31);
+    int32_t s = -1, t = -1;
+    if (e < E) {
+      s = src[e];
+      t = dst[e];
+      if (!edge_ok(s, t, N)) s = t = -1;
+    }
+    const int ps = aggregated_claim(fill, s);
+    const int pt = aggregated_claim(fill, t);
+    if (s >= 0) {
+      nbr[ofs[s] + ps] = deg[t];
+      nbr[ofs[t] + pt] = deg[s];
+    }
   }
 }
 
@@ -101,30 +131,101 @@ __global__ void ob_h_small(const int32_t* __restrict__ ofs, const int32_t* __res
   }
 }
 
-// one CTA per node with a list longer than kBigList (grid-stride over all nodes, skipping others)
-__global__ void __launch_bounds__(256) ob_h_big(const int32_t* __restrict__ ofs, const int32_t* __restrict__ nbr,
-                                                int64_t N, int32_t* __restrict__ h) {
-  __shared__ int part[8];
+// One CTA per node with a list longer than kBigList (grid-stride over all nodes, skipping others).
+// The h-index is the largest h with S(h) = #{degrees >= h} >= h.  Each pass bins the degrees over
+// [lo, hi] into at most kCap bins of width w (degrees above hi in the last bin, below lo dropped);
+// the suffix sums give S at every bin start, the largest bin start still satisfying S >= h brackets
+// the answer, and the next pass refines that bin.  Two passes cover lists of millions of entries
+// (multi-edges between hubs give hubs h-indices in the thousands).  The lowest bins, where most of
+// a hub's neighbours fall, are counted in registers before they reach shared memory.
+constexpr int kCap = 8192;
+constexpr int kRegBins = 8;
+constexpr int kBigThreads = 1024;
+__global__ void __launch_bounds__(kBigThreads) ob_h_big(const int32_t* __restrict__ ofs, const int32_t* __restrict__ nbr,
+                                                        int64_t N, int32_t* __restrict__ h) {
+  __shared__ int hist[kCap];
+  __shared__ int part[kBigThreads / 32];
+  __shared__ int best_s;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int64_t v = blockIdx.x; v < N; v += gridDim.x) {
     const int n = ofs[v + 1] - ofs[v];
     if (n <= kBigList) continue;
     const int32_t* nb = nbr + ofs[v];
-    int lo = 0, hi = n;
-    while (lo < hi) {  // uniform over the CTA
-      const int mid = (lo + hi + 1) >> 1;
-      int c = 0;
-      for (int i = threadIdx.x; i < n; i += blockDim.x) c += nb[i] >= mid;
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
-      if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = c;
+    int lo = 0, hi = n;  // S(lo) >= lo holds; the answer lies in [lo, hi]
+    while (true) {
+      const int span = hi - lo + 1;
+      int lw = 0;  // bin width 2^lw, the smallest giving at most kCap bins
+      while (((span + (1 << lw) - 1) >> lw) > kCap) ++lw;
+      const int w = 1 << lw;
+      const int nbins = (span + w - 1) >> lw;
+      for (int i = threadIdx.x; i < nbins; i += blockDim.x) hist[i] = 0;
+      if (threadIdx.x == 0) best_s = 0;
       __syncthreads();
-      int t = 0;
+      int reg[kRegBins] = {0, 0, 0, 0, 0, 0, 0, 0};
+      auto count = [&](int d) {
+        if (d < lo) return;
+        const int j = min((d - lo) >> lw, nbins - 1);
+        if (j < kRegBins) {
 #pragma unroll
-      for (int w = 0; w < 8; ++w) t += part[w];
+          for (int q = 0; q < kRegBins; ++q) reg[q] += j == q;
+        } else {
+          atomicAdd(&hist[j], 1);
+        }
+      };
+      int i = threadIdx.x;
+      for (; i + 3 * (int)blockDim.x < n; i += 4 * blockDim.x) {  // four loads in flight
+        const int d0 = nb[i], d1 = nb[i + blockDim.x], d2 = nb[i + 2 * blockDim.x], d3 = nb[i + 3 * blockDim.x];
+        count(d0);
+        count(d1);
+        count(d2);
+        count(d3);
+      }
+      for (; i < n; i += blockDim.x) count(nb[i]);
+#pragma unroll
+      for (int q = 0; q < kRegBins; ++q) {
+        int t = reg[q];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+        if (lane == 0 && t && q < nbins) atomicAdd(&hist[q], t);
+      }
       __syncthreads();
-      if (t >= mid) lo = mid; else hi = mid - 1;
+      // suffix sums: thread j owns bins [blo, bhi) counted from the top
+      const int per = (nbins + blockDim.x - 1) / blockDim.x;
+      const int bhi = nbins - threadIdx.x * per, blo = max(0, bhi - per);
+      int own = 0;
+      for (int b = blo; b < bhi; ++b) own += hist[b];
+      int incl = own;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      if (lane == 31) part[warp] = incl;
+      __syncthreads();
+      int run = incl - own;  // entries in higher bins of lower-numbered threads
+#pragma unroll
+      for (int ww = 0; ww < kBigThreads / 32; ++ww) run += ww < warp ? part[ww] : 0;
+      int found = -1;
+      for (int b = bhi - 1; b >= blo; --b) {  // S(lo + b w) from the top of the range down
+        run += hist[b];
+        if (run >= lo + b * w) {
+          found = b;
+          break;
+        }
+      }
+      if (found >= 0) atomicMax(&best_s, found);
+      __syncthreads();
+      const int j = best_s;  // bin 0 always qualifies (S(lo) >= lo)
+      __syncthreads();
+      if (w == 1) {
+        if (threadIdx.x == 0) h[v] = lo + j;
+        break;
+      }
+      const int nlo = lo + j * w;
+      hi = min(hi, nlo + w - 1);
+      lo = nlo;
     }
-    if (threadIdx.x == 0) h[v] = lo;
+    __syncthreads();
   }
 }
 
@@ -372,7 +473,7 @@ extern "C" hg_status hg_overlap_build(const int32_t* src, const int32_t* dst, co
   if (N > 0) {
     HG_TRY(launch("ob_h_small", ob_h_small, dim3(grid_of(32 * N)), dim3(256), 0, s, (const int32_t*)L.ofs,
                   (const int32_t*)L.nbr, N, h));
-    HG_TRY(launch("ob_h_big", ob_h_big, dim3((unsigned)std::min<int64_t>(N, 152 * 4)), dim3(256), 0, s,
+    HG_TRY(launch("ob_h_big", ob_h_big, dim3((unsigned)std::min<int64_t>(N, 152 * 2)), dim3(kBigThreads), 0, s,
                   (const int32_t*)L.ofs, (const int32_t*)L.nbr, N, h));
   }
   // candidates (Eq. 4), the h-index filter, the selection of the M smallest keys

@@ -137,3 +137,16 @@ def test_full_overlap_and_alignment(full):
     assert relerr(host(loss), np.array(ref)) <= 1e-4
     rA, _ = oracle.align_backward(w.X, ia, w.H_b, ib, 2e-4, 1e-8, 0.1)
     assert relerr(host(dA)[ia], rA[ia]) <= TOL[sp.dtype]
+
+
+def test_full_size_overlap_construction():
+    """The 1M-node / 20M-edge graph as the global graph of the subgraph construction, K = 8,
+    theta = 2 and a 15 % budget (the paper's setting): every output bit-exact against the oracle."""
+    need_gpu()
+    from tests.test_gpu_overlap_build import compare, run
+    g = hgsynth.make_graph(hgsynth.spec("sub-1m"))
+    offs = [int(x) for x in g["type_offsets"]]
+    M = int(0.15 * offs[-1] / 8)
+    out, ref = run(lib(), g["src"], g["dst"], g["rel"], offs, 8, 3, 2, M, ps=21, ss=22)
+    compare(out, ref)
+    assert out["counts"]["expanded"] == min(M, out["counts"]["filtered"]) > 0

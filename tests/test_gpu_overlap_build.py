@@ -88,3 +88,4 @@ def test_ties_and_budget_edges():
     assert out["counts"]["nodes"] == len(ref["gid"]) and out["counts"]["edges"] == 0
     np.testing.assert_array_equal(out["gid"].cpu().numpy(), ref["gid"])
     assert hg.hg_device_status() == 0
+
