@@ -16,6 +16,8 @@ from .graphs import (  # noqa: F401
     Workload,
     bf16_round,
     make_graph,
+    make_head_params,
+    make_labels,
     make_layer_params,
     make_ring_part,
     make_workload,

@@ -21,8 +21,12 @@ Recipe (stated once here, repeated in the design notes):
   the paper's threshold, because an h-index never exceeds the degree); "uniform" draws among all
   nodes.  Global ids are sorted random draws from an 8x larger id space, users below risk events,
   so local order equals global-id order.
+* Labels: 11.7 % of the users of a subgraph are labelled (the paper leaves 88.3 % unlabelled),
+  5 % of those positive (the paper gives no rate).  Head weights: Xavier uniform W1 (d x d) and
+  w2 (d), zero biases.
 * Seeds: graph = seed, features = seed+1, overlap = seed+2, second view / bank = seed+3,
-  upstream gradient = seed+4, layer l weights = seed+100+l; subgraph k mixes k into each seed.
+  upstream gradient = seed+4, labels = seed+5, layer l weights = seed+100+l, head weights =
+  seed+200; subgraph k mixes k into each seed.
 """
 from __future__ import annotations
 
@@ -349,3 +353,39 @@ def make_ring_part(sp: GraphSpec, k: int) -> RingPart:
     X = _global_features(sp, gid)
     dH_top = _store(_rng(sp.seed + 4, k).standard_normal((sp.num_nodes, sp.d), dtype=np.float32), sp.dtype)
     return RingPart(k, g, X, gid, dH_top)
+
+
+# ------------------------------------------------------------------------------------------------
+# labels and prediction-head weights
+# ------------------------------------------------------------------------------------------------
+LABELLED_FRACTION = 0.117  # the paper's data leaves 88.3 % of users unlabelled (Section 4.1)
+POSITIVE_RATE = 0.05  # not given by the paper; a rare positive class, as in fraud data
+
+
+def make_labels(sp: GraphSpec, sub: int = 0, fraction: float = LABELLED_FRACTION,
+                positive_rate: float = POSITIVE_RATE) -> tuple:
+    """Labelled user rows of one subgraph, ascending (int32), and their 0/1 labels (fp32): each user
+    is labelled with probability `fraction`, each label is 1 with probability `positive_rate`
+    (seed+5)."""
+    rng = _rng(sp.seed + 5, sub)
+    rows = np.flatnonzero(rng.random(sp.n_user) < fraction).astype(np.int32)
+    y = (rng.random(rows.shape[0]) < positive_rate).astype(np.float32)
+    return rows, y
+
+
+def make_head_params(sp: GraphSpec, random_bias: bool = False) -> dict:
+    """Two-layer head: W1 (d x d, input x hidden), b1 (d), w2 (d), b2 (1).  Xavier uniform weights,
+    zero biases, or small N(0, 0.1) biases for tests (seed+200)."""
+    rng = _rng(sp.seed + 200)
+    d = sp.d
+    a1 = math.sqrt(6.0 / (2 * d))
+    a2 = math.sqrt(6.0 / (d + 1))
+    W1 = rng.uniform(-a1, a1, size=(d, d)).astype(np.float32)
+    w2 = rng.uniform(-a2, a2, size=(d,)).astype(np.float32)
+    if random_bias:
+        b1 = 0.1 * rng.standard_normal(d, dtype=np.float32)
+        b2 = 0.1 * rng.standard_normal(1, dtype=np.float32)
+    else:
+        b1 = np.zeros(d, np.float32)
+        b2 = np.zeros(1, np.float32)
+    return {k: _store(v, sp.dtype) for k, v in dict(W1=W1, b1=b1, w2=w2, b2=b2).items()}

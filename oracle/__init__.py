@@ -5,3 +5,4 @@ from .hg_oracle import (  # noqa: F401
     layer_forward_rows, mean_aggregate, overlap_intersect, standardise, step, valid_edges,
 )
 from . import overlap_build  # noqa: F401  (overlapping-subgraph construction, Eq. 4-5)
+from . import head  # noqa: F401  (MeanAgg, MLP head, masked BCE and joint objective, Eq. 18-20)
