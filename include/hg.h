@@ -278,6 +278,67 @@ hg_status hg_overlap_build(const int32_t* src, const int32_t* dst, const int32_t
                            void* workspace, size_t workspace_bytes, hg_stream stream);
 
 /* ------------------------------------------------------------------------------------------- */
+/* Prediction head and joint objective (Section 3.4, Eq. 18-20; MeanAgg / MLP / loss steps of     */
+/* Algorithm 1)                                                                                   */
+/* ------------------------------------------------------------------------------------------- */
+
+/* Two-layer head on final embeddings of width d (hidden width d, one output logit), device
+ * pointers of the storage type: W1 d x d row-major (input x hidden, applied as h W1), b1 [d],
+ * w2 [d], b2 [1].  W1, b1 and w2 must be 16-byte aligned. */
+typedef struct {
+  int32_t d;
+  hg_dtype dtype;
+  const void* W1;
+  const void* b1;
+  const void* w2;
+  const void* b2;
+} hg_head_params;
+
+/* Head gradients, device fp32, OVERWRITTEN: dW1 [d x d], db1 [d], dw2 [d], db2 [1]. */
+typedef struct {
+  float* dW1;
+  float* db1;
+  float* dw2;
+  float* db2;
+} hg_head_grads;
+
+/* Buffer sizes for n_lab labelled rows of an H with `rows` rows. */
+hg_status hg_head_workspace_size(int64_t rows, int64_t n_lab, int32_t d, hg_dtype dtype, size_t* saved_bytes,
+                                 size_t* scratch_bytes);
+
+/* Masked BCE of the head over the labelled rows and the joint objective:
+ *   MeanAgg  h_r = H[lab_idx[r]], or, when that row is idx_a[k] of an overlap pair k < n_rep,
+ *            (H[idx_a[k]] + H_rep[idx_b[k]]) / 2 rounded to the storage type (the mean of the
+ *            node's two replicas);
+ *   Eq. 18   z_r = relu(h_r W1 + b1) . w2 + b2 (a logit; the probability is sigmoid(z_r));
+ *   Eq. 19   loss_out[1] = L_BCE = (1/n_lab) sum_r -[y_r log p_r + (1 - y_r) log(1 - p_r)];
+ *   Eq. 20   loss_out[0] = L_BCE + lambda_cca * cca_loss[0]  (cca_loss: device fp32, e.g. the
+ *            loss_out of hg_overlap_align_loss; NULL means L_BCE alone).
+ * H: rows x d, H_rep: rows_rep x d (row-major, storage type, 16-byte aligned).  idx_a / idx_b:
+ * device int32 [n_rep_max] overlap pairs (hg_overlap_intersect), each list of distinct rows;
+ * n_rep_dev: optional device int64 with the actual count (NULL = n_rep_max; a negative count
+ * means none); pairs with an index out of range are ignored.  lab_idx: device int32 [n_lab]
+ * DISTINCT rows of H; lab_y: device fp32 [n_lab] labels in [0, 1].  A lab_idx entry outside
+ * [0, rows) is never dereferenced: it makes the loss NaN and gets no gradient.  logits: device
+ * fp32 [n_lab] (z_r) or NULL.  loss_out: device fp32 [2].  saved: kept for hg_head_bwd.
+ * n_lab = 0 gives L_BCE = 0. */
+hg_status hg_head_loss(const hg_head_params* params, const void* H, int64_t rows, const void* H_rep,
+                       int64_t rows_rep, const int32_t* idx_a, const int32_t* idx_b, int64_t n_rep_max,
+                       const int64_t* n_rep_dev, const int32_t* lab_idx, const float* lab_y, int64_t n_lab,
+                       const float* cca_loss, float lambda_cca, float* loss_out, float* logits, void* saved,
+                       void* scratch, hg_stream stream);
+
+/* Gradient of dloss * L_BCE (dloss = 1 in training; the alignment term's gradient comes from
+ * hg_overlap_align_bwd with dloss = lambda_CCA).  grads are OVERWRITTEN.  The gradient at each
+ * labelled row's final embedding is ACCUMULATED into dH[lab_idx[r]] (storage type), or, for a
+ * row with a replica, half into dH[idx_a[k]] and half into dH_rep[idx_b[k]].  dH_rep may be NULL
+ * (a detached second view); dH may be NULL.  `saved` must come from hg_head_loss with the same
+ * params, lab_idx and n_lab. */
+hg_status hg_head_bwd(const hg_head_params* params, const int32_t* lab_idx, int64_t n_lab, float dloss,
+                      const void* saved, void* dH, void* dH_rep, const hg_head_grads* grads, void* scratch,
+                      hg_stream stream);
+
+/* ------------------------------------------------------------------------------------------- */
 /* Kernel timing (measurement support; off by default)                                          */
 /* ------------------------------------------------------------------------------------------- */
 

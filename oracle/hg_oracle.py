@@ -432,12 +432,15 @@ def overlap_intersect(gid_a, gid_b) -> tuple:
 # one whole step of the hot path (used for the CPU baseline and small end-to-end checks)
 # ----------------------------------------------------------------------------------------------
 def step(graph: dict, X, params: list, dH_top, view_b: dict, act="relu", layernorm=True,
-         ln_eps=1e-5, lambda_n=2e-4, var_eps=1e-8, dloss=0.1, store="f64") -> dict:
+         ln_eps=1e-5, lambda_n=2e-4, var_eps=1e-8, dloss=0.1, store="f64", head: dict | None = None) -> dict:
     """CSR build -> L layers forward -> overlap rows -> alignment loss and gradient -> L layers
     backward (view_b None: no alignment term, as for the first subgraph of a sequence).  With store="bf16" the tensors handed from layer to layer (outputs, their gradients)
     are rounded to bf16 as well, like every bf16 tensor the layer interface exchanges.  `view_b` is either {"H_b": bank rows, "gid_a", "gid_b"} (a detached neighbour view)
     or {"idx": overlap rows, "X_b": second input} (a second live stack on the same graph).
-    The last layer's upstream gradient is dH_top plus the alignment gradient."""
+    The last layer's upstream gradient is dH_top plus the alignment gradient.  With `head`
+    ({"params", "lab_idx", "lab_y"}) the head's gradient (MeanAgg, MLP, masked BCE; Eq. 18-19)
+    replaces dH_top, the joint objective L_BCE + dloss * L_CCA (Eq. 20, dloss = lambda_CCA) is
+    returned as res["head_loss"], and res["head_grads"] holds the head's parameter gradients."""
     offs, rels = graph["type_offsets"], graph["rels"]
     csr = build_csr(graph["src"], graph["dst"], graph["rel"], offs, rels)
 
@@ -459,10 +462,25 @@ def step(graph: dict, X, params: list, dH_top, view_b: dict, act="relu", layerno
         return dh, grads
 
     hs = run_stack(X)
+    from . import head as head_mod  # the head module builds on this one
+
+    def head_terms(Htop, ia, Hb, ib, l_cca):
+        hl = head_mod.head_loss(Htop, ia, Hb, ib, head["lab_idx"], head["lab_y"], head["params"], cca_loss=l_cca,
+                                lambda_cca=dloss, store=store)
+        hb = head_mod.head_backward(Htop, ia, Hb, ib, head["lab_idx"], head["lab_y"], head["params"], dloss=1.0,
+                                    store=store)
+        return (hl["total"], hl["bce"]), hb
+
     if view_b is None:  # first subgraph of a sequence: no alignment term
-        dX, grads = back_stack(hs, np.asarray(dH_top, F64))
-        return dict(H=hs, loss=(0.0, 0.0, 0.0), idx_a=np.zeros(0, np.int64), idx_b=np.zeros(0, np.int64), dX=dX,
-                    grads=grads)
+        res = dict(H=hs, loss=(0.0, 0.0, 0.0), idx_a=np.zeros(0, np.int64), idx_b=np.zeros(0, np.int64))
+        dtop = np.asarray(dH_top, F64) if head is None else None
+        if head is not None:
+            none = np.zeros(0, np.int64)
+            res["head_loss"], hb = head_terms(hs[-1], none, None, none, 0.0)
+            res["head_grads"] = {k: hb[k] for k in ("dW1", "db1", "dw2", "db2")}
+            dtop = hb["dH"]
+        res["dX"], res["grads"] = back_stack(hs, dtop)
+        return res
     if "H_b" in view_b:
         ia, ib = overlap_intersect(view_b["gid_a"], view_b["gid_b"])
         Hb = view_b["H_b"]
@@ -473,8 +491,16 @@ def step(graph: dict, X, params: list, dH_top, view_b: dict, act="relu", layerno
         Hb = hs_b[-1]
     loss = align_forward(hs[-1], ia, Hb, ib, lambda_n, var_eps)
     dA, dB = align_backward(hs[-1], ia, Hb, ib, lambda_n, var_eps, dloss)
-    dX, grads = back_stack(hs, np.asarray(dH_top, F64) + dA)
-    res = dict(H=hs, loss=loss, idx_a=ia, idx_b=ib, dX=dX, grads=grads)
+    res = dict(H=hs, loss=loss, idx_a=ia, idx_b=ib)
+    if head is None:
+        dtop = np.asarray(dH_top, F64) + dA
+    else:
+        res["head_loss"], hb = head_terms(hs[-1], ia, Hb, ib, loss[0])
+        res["head_grads"] = {k: hb[k] for k in ("dW1", "db1", "dw2", "db2")}
+        dtop = hb["dH"] + dA
+        dB = dB + hb["dH_rep"]
+    dX, grads = back_stack(hs, dtop)
+    res["dX"], res["grads"] = dX, grads
     if hs_b is not None:
         res["dX_b"], res["grads_b"] = back_stack(hs_b, dB)
         res["H_b"] = hs_b

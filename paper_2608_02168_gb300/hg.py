@@ -42,6 +42,15 @@ class hg_layer_grads(Structure):
                 ("dln_beta", c_void_p)]
 
 
+class hg_head_params(Structure):
+    _fields_ = [("d", c_int32), ("dtype", c_int32), ("W1", c_void_p), ("b1", c_void_p), ("w2", c_void_p),
+                ("b2", c_void_p)]
+
+
+class hg_head_grads(Structure):
+    _fields_ = [("dW1", c_void_p), ("db1", c_void_p), ("dw2", c_void_p), ("db2", c_void_p)]
+
+
 EXPORTS = {
     # name: (restype, argtypes)
     "hg_status_string": (c_char_p, [c_int32]),
@@ -75,6 +84,12 @@ EXPORTS = {
     "hg_overlap_build": (c_int32, [c_void_p, c_void_p, c_void_p, c_int64, c_int64, POINTER(c_int64), c_int32, c_int32,
                                    c_int32, c_int32, c_int64, c_uint64, c_uint64, c_void_p, c_void_p, c_void_p,
                                    c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
+    "hg_head_workspace_size": (c_int32, [c_int64, c_int64, c_int32, c_int32, POINTER(c_size_t), POINTER(c_size_t)]),
+    "hg_head_loss": (c_int32, [POINTER(hg_head_params), c_void_p, c_int64, c_void_p, c_int64, c_void_p, c_void_p,
+                               c_int64, c_void_p, c_void_p, c_void_p, c_int64, c_void_p, c_float, c_void_p, c_void_p,
+                               c_void_p, c_void_p, c_void_p]),
+    "hg_head_bwd": (c_int32, [POINTER(hg_head_params), c_void_p, c_int64, c_float, c_void_p, c_void_p, c_void_p,
+                              POINTER(hg_head_grads), c_void_p, c_void_p]),
     "hg_timing_enable": (c_int32, [c_int32]),
     "hg_timing_report": (c_int32, [c_char_p, c_size_t]),
 }
@@ -369,3 +384,42 @@ def hg_overlap_build(src, dst, rel, type_offsets, K: int, k: int, theta: int, M:
         res["h"] = h[:N]
     return res
 
+
+
+# ------------------------------------------------------------------------------------------------
+# prediction head and joint objective
+# ------------------------------------------------------------------------------------------------
+class HeadParams:
+    """Packed device parameters of the two-layer head (see hg_head_params)."""
+
+    def __init__(self, W1, b1, w2, b2):
+        self.W1, self.b1, self.w2, self.b2 = W1.contiguous(), b1.contiguous(), w2.contiguous(), b2.contiguous()
+        self.d = int(W1.shape[-1])
+        self.dtype = HG_F32 if W1.dtype == torch.float32 else HG_BF16
+
+    def c(self) -> hg_head_params:
+        return hg_head_params(self.d, self.dtype, _ptr(self.W1), _ptr(self.b1), _ptr(self.w2), _ptr(self.b2))
+
+
+def hg_head_workspace_size(rows: int, n_lab: int, d: int, dtype) -> tuple:
+    s, k = c_size_t(0), c_size_t(0)
+    dt = dtype if isinstance(dtype, int) else (HG_F32 if dtype == torch.float32 else HG_BF16)
+    _check(lib().hg_head_workspace_size(int(rows), int(n_lab), int(d), dt, byref(s), byref(k)),
+           "hg_head_workspace_size")
+    return s.value, k.value
+
+
+def hg_head_loss(params: HeadParams, H, H_rep, idx_a, idx_b, n_rep_max: int, n_rep_dev, lab_idx, lab_y, cca_loss,
+                 lambda_cca: float, loss_out, logits, saved, scratch, stream=None):
+    p = params.c()
+    _check(lib().hg_head_loss(byref(p), _ptr(H), H.shape[0], _ptr(H_rep), H_rep.shape[0] if H_rep is not None else 0,
+                              _ptr(idx_a), _ptr(idx_b), int(n_rep_max), _ptr(n_rep_dev), _ptr(lab_idx), _ptr(lab_y),
+                              lab_idx.numel(), _ptr(cca_loss), float(lambda_cca), _ptr(loss_out), _ptr(logits),
+                              _ptr(saved), _ptr(scratch), _stream(stream)), "hg_head_loss")
+
+
+def hg_head_bwd(params: HeadParams, lab_idx, dloss: float, saved, dH, dH_rep, grads: dict, scratch, stream=None):
+    p = params.c()
+    gr = hg_head_grads(_ptr(grads["W1"]), _ptr(grads["b1"]), _ptr(grads["w2"]), _ptr(grads["b2"]))
+    _check(lib().hg_head_bwd(byref(p), _ptr(lab_idx), lab_idx.numel(), float(dloss), _ptr(saved), _ptr(dH),
+                             _ptr(dH_rep), byref(gr), _ptr(scratch), _stream(stream)), "hg_head_bwd")

@@ -5,8 +5,12 @@ A step (Algorithm 1, the per-worker part of one iteration, on one GPU):
   hg_layer_fwd x L       heterogeneous mean-aggregation layers (Eq. 7, 10, 11)
   hg_overlap_intersect   overlap rows with the neighbouring subgraph (Section 3.3)
   hg_overlap_align_loss  CCA alignment loss (Eq. 14-17)
-  hg_overlap_align_bwd   its gradient, scaled by lambda_CCA (Eq. 20), added to the upstream
-                         gradient of the last layer's output
+  hg_head_loss           (with a head and labels) MeanAgg of the replicas, the two-layer MLP and
+                         the masked BCE over the labelled rows, and L_total = L_BCE + lambda_CCA
+                         L_CCA (Eq. 18-20)
+  hg_head_bwd            its gradient, which is then the last layer's upstream gradient (without
+                         a head the caller supplies that gradient, dH_top)
+  hg_overlap_align_bwd   the alignment gradient, scaled by lambda_CCA (Eq. 20), added to it
   hg_layer_bwd x L       gradients of every layer, including dL/dX of the first.
 This module only allocates buffers (torch) and marshals arguments; every computation runs in
 libhg's kernels.
@@ -38,7 +42,7 @@ class HotPath:
 
     def __init__(self, type_offsets, rels, num_edges: int, d: int, dtype: str, layer_params: list,
                  view: str, n_overlap_max: int, n_gid_a: int = 0, n_gid_b: int = 0, act: str = "relu",
-                 layernorm: bool = True, device="cuda"):
+                 layernorm: bool = True, device="cuda", head_params: dict | None = None, n_lab_max: int = 0):
         self.type_offsets = [int(x) for x in type_offsets]
         self.rels = [tuple(r) for r in rels]
         self.N = self.type_offsets[-1]
@@ -77,6 +81,16 @@ class HotPath:
             self.idx_b = torch.empty(cap, dtype=torch.int32, device=dev)
             self.isect_scratch = torch.empty(hg.hg_overlap_intersect_workspace_size(n_gid_a, n_gid_b),
                                              dtype=torch.uint8, device=dev)
+        self.head = None
+        if head_params is not None:
+            self.head = hg.HeadParams(*(torch.as_tensor(head_params[k], device=dev).to(td) for k in ("W1", "b1", "w2", "b2")))
+            h_s, h_k = hg.hg_head_workspace_size(self.N, max(1, int(n_lab_max)), d, td)
+            self.head_saved = torch.empty(h_s, dtype=torch.uint8, device=dev)
+            self.head_scratch = torch.empty(h_k, dtype=torch.uint8, device=dev)
+            self.head_loss = torch.zeros(2, dtype=torch.float32, device=dev)
+            f = torch.float32
+            self.head_grads = {"W1": torch.empty(d, d, dtype=f, device=dev), "b1": torch.empty(d, dtype=f, device=dev),
+                               "w2": torch.empty(d, dtype=f, device=dev), "b2": torch.empty(1, dtype=f, device=dev)}
         self.graph = None
 
     def _layer_sizes(self, num_edges: int):
@@ -105,11 +119,13 @@ class HotPath:
 
     # --------------------------------------------------------------------------------------------
     def step(self, src, dst, rel, X, dH_top, X_b=None, overlap_idx=None, gid_a=None, gid_b=None, H_bank=None,
-             stream=None, marks=None):
+             stream=None, marks=None, lab_idx=None, lab_y=None):
         """Run one step; all inputs are device tensors.  Returns nothing (results stay in the buffers:
-        self.H, self.loss, self.grads, self.dH[s][0] = dL/dX).  `marks`, if a list, receives
+        self.H, self.loss, self.grads, self.dH[s][0] = dL/dX; with a head, self.head_loss =
+        [L_total, L_BCE] and self.head_grads).  With a head and labels (lab_idx, lab_y) the last
+        layer's upstream gradient is the head's and dH_top is ignored.  `marks`, if a list, receives
         (phase, CUDA event) pairs recorded on the stream after the graph build, the forward layers,
-        the alignment and the backward layers."""
+        the alignment and head, and the backward layers."""
         def mark(name):
             if marks is not None:
                 ev = torch.cuda.Event(enable_timing=True)
@@ -127,10 +143,16 @@ class HotPath:
                 hg.hg_layer_fwd(g, self.params[l], self.H[s][l], self.H[s][l + 1], self.saved[s][l], self.scratch, stream)
         mark("forward")
         top = self.H[0][self.L]
-        self.dH[0][self.L].copy_(dH_top)
+        use_head = self.head is not None and lab_idx is not None
+        if use_head:
+            self.dH[0][self.L].zero_()
+        else:
+            self.dH[0][self.L].copy_(dH_top)
         if self.view == "bank" and H_bank is None:
             # first subgraph of a sequence: no neighbour view yet, no alignment term
             self.loss.zero_()
+            if use_head:
+                self._head(top, None, None, None, 0, None, None, lab_idx, lab_y, stream)
             mark("alignment")
             for l in range(self.L - 1, -1, -1):
                 hg.hg_layer_bwd(g, self.params[l], self.H[0][l], self.saved[0][l], self.dH[0][l + 1], self.dH[0][l],
@@ -149,6 +171,8 @@ class HotPath:
             dHb, n_dev = self.dH[1][self.L], None
         hg.hg_overlap_align_loss(top, ia, Hb, ib, n_max, n_dev, LAMBDA_N, VAR_EPS, self.loss, self.align_saved,
                                  self.align_scratch, stream)
+        if use_head:
+            self._head(top, Hb, ia, ib, n_max, n_dev, dHb, lab_idx, lab_y, stream)
         hg.hg_overlap_align_bwd(top, ia, Hb, ib, n_max, n_dev, LAMBDA_N, VAR_EPS, LAMBDA_CCA, self.align_saved,
                                 self.dH[0][self.L], dHb, self.align_scratch, stream)
         mark("alignment")
@@ -157,6 +181,14 @@ class HotPath:
                 hg.hg_layer_bwd(g, self.params[l], self.H[s][l], self.saved[s][l], self.dH[s][l + 1], self.dH[s][l],
                                 self.grads[s][l], self.scratch, stream)
         mark("backward")
+
+    def _head(self, top, H_rep, ia, ib, n_max, n_dev, dH_rep, lab_idx, lab_y, stream):
+        """Head loss (L_total with the alignment loss just computed) and its gradient into the last
+        layer's upstream gradient (and the second view's, when that view is live)."""
+        hg.hg_head_loss(self.head, top, H_rep, ia, ib, n_max, n_dev, lab_idx, lab_y, self.loss, LAMBDA_CCA,
+                        self.head_loss, None, self.head_saved, self.head_scratch, stream)
+        hg.hg_head_bwd(self.head, lab_idx, 1.0, self.head_saved, self.dH[0][self.L], dH_rep, self.head_grads,
+                       self.head_scratch, stream)
 
 
 class Ring:
