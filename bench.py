@@ -46,7 +46,10 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-build", action="store_true", help="skip the subgraph-construction measurement")
+    ap.add_argument("--no-head", action="store_true",
+                    help="drive the layers with a synthetic upstream gradient instead of the head and joint loss")
     ap.add_argument("--oracle-sample", type=int, default=0, help=argparse.SUPPRESS)  # internal: child process
+    ap.add_argument("--oracle-no-head", action="store_true", help=argparse.SUPPRESS)  # internal: child process
     ap.add_argument("--oracle-build-sample", type=int, default=0, help=argparse.SUPPRESS)  # internal: child process
     return ap.parse_args()
 
@@ -65,14 +68,18 @@ def workload_desc(sp) -> str:
 # ------------------------------------------------------------------------------------------------
 # oracle timing (CPU baseline / reference arm); runs in a child process with one thread
 # ------------------------------------------------------------------------------------------------
-def oracle_sample_main(name: str, k: int):
+def oracle_sample_main(name: str, k: int, with_head: bool = True):
     import oracle
     sp = scaled(hgsynth.spec(name), k)
     w = hgsynth.make_workload(sp)
     vb = {"idx": w.overlap_local, "X_b": w.X_b} if sp.view_b == "perturbed" else \
         {"H_b": w.H_b, "gid_a": w.gid_a, "gid_b": w.gid_b}
+    head = None
+    if with_head:
+        lab, y = hgsynth.make_labels(sp)
+        head = {"params": hgsynth.make_head_params(sp), "lab_idx": lab, "lab_y": y}
     t0 = time.perf_counter()
-    oracle.step(w.graph, w.X, w.params, w.dH_top, vb)
+    oracle.step(w.graph, w.X, w.params, w.dH_top, vb, head=head)
     dt = time.perf_counter() - t0
     print(json.dumps({"seconds": dt, "edges": sp.num_edges, "layers": sp.layers,
                       "value": sp.layers * sp.num_edges / dt}))
@@ -90,10 +97,11 @@ def oracle_build_sample_main(name: str, k: int):
     print(json.dumps({"seconds": dt, "edges": sp.num_edges, "value": sp.num_edges / dt}))
 
 
-def time_oracle(name: str, k: int, flag: str = "--oracle-sample") -> dict:
+def time_oracle(name: str, k: int, flag: str = "--oracle-sample", with_head: bool = True) -> dict:
     env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
                CUDA_VISIBLE_DEVICES="")
-    r = subprocess.run([sys.executable, os.path.abspath(__file__), "--workload", name, flag, str(k)],
+    extra = [] if with_head else ["--oracle-no-head"]
+    r = subprocess.run([sys.executable, os.path.abspath(__file__), "--workload", name, flag, str(k), *extra],
                        capture_output=True, text=True, env=env)
     if r.returncode != 0:
         raise RuntimeError(f"oracle sample failed: {r.stderr[-2000:]}")
@@ -228,6 +236,14 @@ def kernel_models(st: dict, sp) -> dict:
     m["proj_bwd_tc"] = (L * pb, L * pfl)
     m["wgrad_tc"] = (L * row * (RR + N), L * 2 * d * d * RR)  # G_r = M_r^T dU: M_r rows once, dU once per type
     m["radix_scatter"] = (2 * 3 * 2 * 12 * st["E"], 0)  # 2 layouts x 3 passes x read+write of key, edge id, endpoint
+    nl = st.get("n_lab", 0)
+    if nl:
+        # per labelled row: its H row (and a replica row for overlap rows, not counted), the saved Hm
+        # and dA rows written, the label; backward: dA read, dH row read and written
+        m["head_fwd_simt"] = (nl * (3 * row + 8), 2 * nl * d * d)
+        m["head_bwd_dx_simt"] = (nl * (3 * row + 8), 2 * nl * d * d)
+        wb, wf = m["wgrad_tc"]
+        m["wgrad_tc"] = (wb + 2 * nl * row, wf + 2 * nl * d * d)  # dW1 = Hm^T dA shares the kernel
     no = st["n_ov"]
     m["align_colstats"] = (3 * 2 * no * (row + 4), 0)        # 3 passes over both gathered views
     m["align_gram_tc"] = (2 * no * (row + 4), 2 * 2 * no * d * d)
@@ -351,7 +367,7 @@ def measure_overlap_build(w, steps: int, warmup: int, dev, with_cpu: bool) -> di
 def main():
     args = parse()
     if args.oracle_sample:
-        oracle_sample_main(args.workload, args.oracle_sample)
+        oracle_sample_main(args.workload, args.oracle_sample, not args.oracle_no_head)
         return
     if args.oracle_build_sample:
         oracle_build_sample_main(args.workload, args.oracle_build_sample)
@@ -369,13 +385,14 @@ def main():
 
 def run_reference(args, sp):
     for _ in range(args.warmup):
-        time_oracle(sp.name, REFERENCE_SCALE)
-    vals = [time_oracle(sp.name, REFERENCE_SCALE) for _ in range(args.steps)]
+        time_oracle(sp.name, REFERENCE_SCALE, with_head=not args.no_head)
+    vals = [time_oracle(sp.name, REFERENCE_SCALE, with_head=not args.no_head) for _ in range(args.steps)]
     secs = sum(v["seconds"] for v in vals)
     edges = sum(v["edges"] * v["layers"] for v in vals)
     value = edges / secs
     sample = (f"1/{REFERENCE_SCALE}-size instance of the workload per step "
-              f"({vals[0]['edges']:,} edges, same recipe), fp64 numpy oracle, one thread")
+              f"({vals[0]['edges']:,} edges, same recipe), fp64 numpy oracle"
+              f"{'' if args.no_head else ' with the head and joint loss'}, one thread")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps,
@@ -402,11 +419,18 @@ def run_ours(args, sp, rank, world):
     w = hgsynth.make_workload(sp, sub=rank)
     g = w.graph
     td = torch.float32 if sp.dtype == "f32" else torch.bfloat16
+    use_head = not args.no_head
+    lab, lab_y = hgsynth.make_labels(sp, sub=rank)
     path = HotPath(g["type_offsets"], g["rels"], len(g["src"]), sp.d, sp.dtype, w.params, view=sp.view_b,
                    n_overlap_max=len(w.overlap_local), n_gid_a=0 if w.gid_a is None else len(w.gid_a),
-                   n_gid_b=0 if w.gid_b is None else len(w.gid_b), device=dev)
+                   n_gid_b=0 if w.gid_b is None else len(w.gid_b), device=dev,
+                   head_params=hgsynth.make_head_params(sp) if use_head else None, n_lab_max=len(lab))
     host = {"src": torch.from_numpy(g["src"]), "dst": torch.from_numpy(g["dst"]), "rel": torch.from_numpy(g["rel"]),
-            "X": torch.from_numpy(w.X).to(td), "dH_top": torch.from_numpy(w.dH_top).to(td)}
+            "X": torch.from_numpy(w.X).to(td)}
+    if use_head:  # the head's gradient drives the backward; its inputs are the labels
+        host.update(lab_idx=torch.from_numpy(lab), lab_y=torch.from_numpy(lab_y))
+    else:
+        host["dH_top"] = torch.from_numpy(w.dH_top).to(td)
     if sp.view_b == "perturbed":
         host.update(X_b=torch.from_numpy(w.X_b).to(td), overlap_idx=torch.from_numpy(w.overlap_local))
     else:
@@ -426,13 +450,14 @@ def run_ours(args, sp, rank, world):
         return float(t.item())
 
     def step(inp, marks=None):
-        kw = {k: inp[k] for k in ("X_b", "overlap_idx", "gid_a", "gid_b", "H_bank") if k in inp}
-        path.step(inp["src"], inp["dst"], inp["rel"], inp["X"], inp["dH_top"], marks=marks, **kw)
+        kw = {k: inp[k] for k in ("X_b", "overlap_idx", "gid_a", "gid_b", "H_bank", "lab_idx", "lab_y") if k in inp}
+        path.step(inp["src"], inp["dst"], inp["rel"], inp["X"], inp.get("dH_top"), marks=marks, **kw)
 
     for _ in range(max(args.warmup, 0)):
         step(devin)
     torch.cuda.synchronize()
     stats = graph_stats(w)
+    stats["n_lab"] = len(lab) if use_head else 0
     models = kernel_models(stats, sp)
     clocks = Clocks(dev.index if dev.index is not None else 0)
     clocks.start()
@@ -481,7 +506,8 @@ def run_ours(args, sp, rank, world):
         # copy of step i+1's inputs (second device buffer set, copy stream) overlaps step i
         pinned = {k: v.pin_memory() for k, v in host.items()}
         h2d = sum(v.numel() * v.element_size() for v in pinned.values())
-        loss_host = torch.empty(3, dtype=torch.float32).pin_memory()
+        result = path.head_loss if use_head else path.loss  # L_total (Eq. 20), or the alignment loss
+        loss_host = torch.empty(result.numel(), dtype=torch.float32).pin_memory()
         bufs = [devin, {k: torch.empty_like(v) for k, v in devin.items()}]
         copy_stream = torch.cuda.Stream(device=dev)
         copied = [torch.cuda.Event(), torch.cuda.Event()]
@@ -507,7 +533,7 @@ def run_ours(args, sp, rank, world):
             stream.wait_event(copied[i % 2])
             step(bufs[i % 2])
             consumed[i % 2].record(stream)
-            loss_host.copy_(path.loss, non_blocking=True)
+            loss_host.copy_(result, non_blocking=True)
             stream.synchronize()  # the loss of step i is on the host
         torch.cuda.synchronize()
         te = max_over_ranks(time.perf_counter() - t0)
@@ -528,16 +554,19 @@ def run_ours(args, sp, rank, world):
     kernel_rooflines = [roofline(report, models, args.steps, peaks, psrc, dom=k)[0] for k in top]
     cpu = None
     if not args.no_cpu_baseline:
-        o = time_oracle(sp.name, ORACLE_SCALE)
+        o = time_oracle(sp.name, ORACLE_SCALE, with_head=use_head)
         cpu = {"value": o["value"], "unit": UNIT, "cores": 1, "kind": "oracle",
                "sample": f"1/{ORACLE_SCALE}-size instance of the workload ({o['edges']:,} edges, same recipe), one "
-                         f"full step of the fp64 numpy oracle, one thread, {o['seconds']:.1f} s"}
+                         f"full step of the fp64 numpy oracle{' with the head and joint loss' if use_head else ''}, "
+                         f"one thread, {o['seconds']:.1f} s"}
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1e3 * t / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": sp.dtype, "data": "synthetic",
         "config": {"workload": workload_desc(sp), "l2": "inputs larger than L2 (not flushed)",
-                   "parallelism": f"{world} independent subgraph(s), one per GPU"},
+                   "parallelism": f"{world} independent subgraph(s), one per GPU",
+                   "objective": (f"L_BCE over {len(lab):,} labelled users + 0.1 L_CCA (head: MeanAgg, 2-layer MLP)"
+                                 if use_head else "synthetic upstream gradient + 0.1 L_CCA")},
         "roofline": rf, "kernel_rooflines": kernel_rooflines, "kernel_time_share": shares,
         "phases_ms": {k: round(v, 4) for k, v in phase_ms.items()},
         "layers_fwd_bwd_edges_per_s": edges_per_step / ((phase_ms.get("forward", 0) + phase_ms.get("backward", 0)) / 1e3)
@@ -546,6 +575,7 @@ def run_ours(args, sp, rank, world):
         "cpu_baseline": cpu, "e2e": e2e, "clocks": clk, "overlap_build": build,
         "gpu_launches": int(sum(n for n, _ in report.values())),
         "loss": [float(x) for x in path.loss.cpu()],
+        "head_loss": [float(x) for x in path.head_loss.cpu()] if use_head else None,
     }
     print(json.dumps(out))
     if world > 1:

@@ -12,50 +12,21 @@
 // backward (hg_head_bwd) scales them by dloss, forms dh_r = dloss dA_r W1^T (split in halves over
 // the two replicas of an overlap row) and dW1 = dloss sum_r h_r^T dA_r.
 //
-// Row tiles of 64 rows on CUDA cores (fp32 FMA); dW1 on the tensor cores for bf16 storage.
-// Every sum over rows is a fixed-order reduction of per-block partials (deterministic).
+// fp32 storage: row tiles of 64 rows on CUDA cores (fp32 FMA).  bf16 storage: 128-row tiles on the
+// tensor cores (head_tc.cu), dW1 by the tensor-core weight-gradient kernel.  Every sum over rows is
+// a fixed-order reduction of per-block partials (deterministic).
 #include <cuda_bf16.h>
 
 #include <algorithm>
 
 #include "hg_internal.cuh"
+#include "head_kernels.cuh"
 #include "layer_kernels.cuh"
 #include "simt_tile.cuh"
 
 namespace hg {
 
 namespace {
-
-struct HeadFwdArgs {
-  const void* H;
-  int64_t rows;
-  const void* H_rep;
-  const int32_t* map;  // [rows] replica row in H_rep or -1
-  const int32_t* lab;
-  const float* y;
-  int64_t n;
-  float inv_n;
-  const void* W1;
-  const void* b1;
-  const void* w2;
-  const void* b2;
-  void* Hm;             // saved [n][D]: MeanAgg rows
-  void* dA;             // saved [n][D]: unit gradient of the hidden pre-activation
-  int32_t* rep_row;     // saved [n]: replica row of each labelled row, -1 none, -2 invalid row
-  float* logits;        // [n] or null
-  float* part;          // [blocks][2 + 2D]: loss, dz, dA column sums, dz * relu(a) column sums
-};
-
-struct HeadBwdArgs {
-  const void* dA;
-  const int32_t* lab;
-  const int32_t* rep_row;
-  int64_t n, rows;
-  const void* W1t;  // W1^T, D x D
-  float dloss;
-  void* dH;
-  void* dH_rep;
-};
 
 __device__ __forceinline__ float softplus_f(float x) { return fmaxf(x, 0.f) + log1pf(expf(-fabsf(x))); }
 
@@ -409,8 +380,15 @@ hg_status head_loss_t(const HeadIn& in, const float* cca, float lam, float* loss
   a.rep_row = L.rep_row;
   a.logits = logits;
   a.part = L.part;
-  const int blocks = head_blocks(in.n);
-  HG_TRY(launch("head_fwd_simt", head_fwd_simt<T, D>, dim3(blocks), dim3(256), HeadSmem<T, D>::kBytes, s, a));
+  a.status = device_status_ptr();
+  int blocks;
+  if constexpr (sizeof(T) == 2) {  // bf16: tensor cores
+    blocks = (int)ceil_div(in.n, kHeadTcRows);
+    HG_TRY(head_fwd_tc(D, a, s));
+  } else {
+    blocks = head_blocks(in.n);
+    HG_TRY(launch("head_fwd_simt", head_fwd_simt<T, D>, dim3(blocks), dim3(256), HeadSmem<T, D>::kBytes, s, a));
+  }
   HG_TRY(reduce_partials(L.part, 2 + 2 * D, blocks, 2 + 2 * D, L.sums, L.tmp, s));
   return launch("head_loss_finish", head_loss_finish, dim3(1), dim3(32), 0, s, (const float*)L.sums, in.n, cca, lam,
                 loss_out);
@@ -420,10 +398,12 @@ template <typename T, int D>
 hg_status head_bwd_t(const hg_head_params* p, const int32_t* lab, int64_t n, int64_t rows, float dloss,
                      const HeadLayout& L, void* dH, void* dH_rep, const hg_head_grads* g, cudaStream_t s) {
   constexpr hg_dtype kDt = sizeof(T) == 2 ? HG_BF16 : HG_F32;
-  if (n > 0) {
-    HG_TRY(transpose_weights(kDt, D, p->W1, L.W1t, 1, s));
-    if (dH || dH_rep) {
-      HeadBwdArgs a{L.dA, lab, L.rep_row, n, rows, L.W1t, dloss, dH, dH_rep};
+  if (n > 0 && (dH || dH_rep)) {
+    HeadBwdArgs a{L.dA, lab, L.rep_row, n, rows, p->W1, L.W1t, dloss, dH, dH_rep, device_status_ptr()};
+    if constexpr (sizeof(T) == 2) {  // bf16: tensor cores, W1 read as it is
+      HG_TRY(head_dx_tc(D, a, s));
+    } else {
+      HG_TRY(transpose_weights(kDt, D, p->W1, L.W1t, 1, s));
       const size_t smem = sizeof(float) * ((size_t)kBM * kAPad + (size_t)kKC * D);
       HG_TRY(launch("head_bwd_dx_simt", head_bwd_dx_simt<T, D>, dim3(head_blocks(n)), dim3(256), smem, s, a));
     }

@@ -125,7 +125,7 @@ class HotPath:
         [L_total, L_BCE] and self.head_grads).  With a head and labels (lab_idx, lab_y) the last
         layer's upstream gradient is the head's and dH_top is ignored.  `marks`, if a list, receives
         (phase, CUDA event) pairs recorded on the stream after the graph build, the forward layers,
-        the alignment and head, and the backward layers."""
+        the alignment, the head (when it runs) and the backward layers."""
         def mark(name):
             if marks is not None:
                 ev = torch.cuda.Event(enable_timing=True)
@@ -151,9 +151,10 @@ class HotPath:
         if self.view == "bank" and H_bank is None:
             # first subgraph of a sequence: no neighbour view yet, no alignment term
             self.loss.zero_()
+            mark("alignment")
             if use_head:
                 self._head(top, None, None, None, 0, None, None, lab_idx, lab_y, stream)
-            mark("alignment")
+                mark("head")
             for l in range(self.L - 1, -1, -1):
                 hg.hg_layer_bwd(g, self.params[l], self.H[0][l], self.saved[0][l], self.dH[0][l + 1], self.dH[0][l],
                                 self.grads[0][l], self.scratch, stream)
@@ -171,11 +172,12 @@ class HotPath:
             dHb, n_dev = self.dH[1][self.L], None
         hg.hg_overlap_align_loss(top, ia, Hb, ib, n_max, n_dev, LAMBDA_N, VAR_EPS, self.loss, self.align_saved,
                                  self.align_scratch, stream)
-        if use_head:
-            self._head(top, Hb, ia, ib, n_max, n_dev, dHb, lab_idx, lab_y, stream)
         hg.hg_overlap_align_bwd(top, ia, Hb, ib, n_max, n_dev, LAMBDA_N, VAR_EPS, LAMBDA_CCA, self.align_saved,
                                 self.dH[0][self.L], dHb, self.align_scratch, stream)
         mark("alignment")
+        if use_head:
+            self._head(top, Hb, ia, ib, n_max, n_dev, dHb, lab_idx, lab_y, stream)
+            mark("head")
         for s in range(len(stacks)):
             for l in range(self.L - 1, -1, -1):
                 hg.hg_layer_bwd(g, self.params[l], self.H[s][l], self.saved[s][l], self.dH[s][l + 1], self.dH[s][l],
