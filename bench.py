@@ -383,6 +383,33 @@ def main():
     run_ours(args, sp, rank, world)
 
 
+# ------------------------------------------------------------------------------------------------
+# multi-GPU harness: one independent subgraph per rank (no collective on the data path); the
+# timed region is bracketed by barriers and its duration is the maximum over the ranks
+# ------------------------------------------------------------------------------------------------
+def rank_barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_time_over_ranks(x: float, world: int, device) -> float:
+    """The largest of the ranks' durations (every rank gets it)."""
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def weak_scaling_value(world: int, edges_per_step: int, steps: int, seconds: float) -> float:
+    """Whole-job throughput: every rank processes its own subgraph of the same size, so the units
+    of all ranks over the slowest rank's time."""
+    return world * edges_per_step * steps / seconds
+
+
 def run_reference(args, sp):
     for _ in range(args.warmup):
         time_oracle(sp.name, REFERENCE_SCALE, with_head=not args.no_head)
@@ -439,15 +466,10 @@ def run_ours(args, sp, rank, world):
     stream = torch.cuda.current_stream()
 
     def barrier():
-        if world > 1:
-            torch.distributed.barrier()
+        rank_barrier(world)
 
     def max_over_ranks(x: float) -> float:
-        if world == 1:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        return float(t.item())
+        return max_time_over_ranks(x, world, dev)
 
     def step(inp, marks=None):
         kw = {k: inp[k] for k in ("X_b", "overlap_idx", "gid_a", "gid_b", "H_bank", "lab_idx", "lab_y") if k in inp}
@@ -497,7 +519,7 @@ def run_ours(args, sp, rank, world):
     hg.hg_timing_enable(False)
     report = hg.hg_timing_report()
     edges_per_step = sp.layers * sp.num_edges
-    value = world * edges_per_step * args.steps / t
+    value = weak_scaling_value(world, edges_per_step, args.steps, t)
 
     # end to end: pinned host inputs copied in, the step, the loss read back, every step
     e2e = None
@@ -537,7 +559,8 @@ def run_ours(args, sp, rank, world):
             stream.synchronize()  # the loss of step i is on the host
         torch.cuda.synchronize()
         te = max_over_ranks(time.perf_counter() - t0)
-        e2e = {"value": world * edges_per_step * args.steps / te, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+        e2e = {"value": weak_scaling_value(world, edges_per_step, args.steps, te), "unit": UNIT,
+               "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(loss_host.numel() * 4)}
 
     if rank != 0:
