@@ -339,6 +339,56 @@ hg_status hg_head_bwd(const hg_head_params* params, const int32_t* lab_idx, int6
                       hg_stream stream);
 
 /* ------------------------------------------------------------------------------------------- */
+/* Temporal module (Section 3.2, Eq. 12-13): attention over each node's last w states and a GRU  */
+/* ------------------------------------------------------------------------------------------- */
+
+/* Parameters, device pointers of the storage type: Wa = Q^T (d x d, input x output), r [d],
+ * W_i = [W_ir | W_iz | W_in] and W_h = [W_hr | W_hz | W_hn] (d x 3d each, input x output), b_i and
+ * b_h [3d].  1 <= w <= 8. */
+typedef struct {
+  int32_t d;
+  int32_t w;
+  hg_dtype dtype;
+  const void* Wa;
+  const void* r;
+  const void* W_i;
+  const void* W_h;
+  const void* b_i;
+  const void* b_h;
+} hg_temporal_params;
+
+/* Gradients, device fp32, OVERWRITTEN: dWa [d x d], dr [d], dW_i and dW_h [d x 3d], db_i, db_h [3d]. */
+typedef struct {
+  float* dWa;
+  float* dr;
+  float* dW_i;
+  float* dW_h;
+  float* db_i;
+  float* db_h;
+} hg_temporal_grads;
+
+hg_status hg_temporal_workspace_size(int64_t n, int32_t d, int32_t w, hg_dtype dtype, size_t* saved_bytes,
+                                     size_t* scratch_bytes);
+
+/* H_out = H^t for n nodes:
+ *   Eq. 12  u_k = tanh(c_k Wa), e_k = r . u_k, a = softmax over k < w of e, H~ = sum_k a_k c_k
+ *           (rounded to the storage type);
+ *   Eq. 13  r_g = sigmoid(x W_ir + b_ir + H~ W_hr + b_hr), z = sigmoid(x W_iz + b_iz + H~ W_hz + b_hz),
+ *           n_g = tanh(x W_in + b_in + r_g * (H~ W_hn + b_hn)), H^t = (1 - z) n_g + z H~.
+ * X: n x d, the spatial embeddings h^t (the last layer's output).  C: w x n x d, block k holding
+ * every node's state k + 1 snapshots back (c_{k+1}); zero rows where a state does not exist.
+ * H_out: n x d.  All row-major, storage type.  saved: H~ and a, kept for hg_temporal_bwd. */
+hg_status hg_temporal_fwd(const hg_temporal_params* params, const void* X, const void* C, int64_t n, void* H_out,
+                          void* saved, void* scratch, hg_stream stream);
+
+/* Backward of hg_temporal_fwd for the upstream gradient dH_out (n x d): dX (n x d, OVERWRITTEN) =
+ * dL/dX and every parameter gradient.  The context C receives no gradient (it holds earlier
+ * snapshots' outputs).  X, C, params and `saved` must be those of the forward. */
+hg_status hg_temporal_bwd(const hg_temporal_params* params, const void* X, const void* C, int64_t n,
+                          const void* saved, const void* dH_out, void* dX, const hg_temporal_grads* grads,
+                          void* scratch, hg_stream stream);
+
+/* ------------------------------------------------------------------------------------------- */
 /* Kernel timing (measurement support; off by default)                                          */
 /* ------------------------------------------------------------------------------------------- */
 

@@ -51,6 +51,16 @@ class hg_head_grads(Structure):
     _fields_ = [("dW1", c_void_p), ("db1", c_void_p), ("dw2", c_void_p), ("db2", c_void_p)]
 
 
+class hg_temporal_params(Structure):
+    _fields_ = [("d", c_int32), ("w", c_int32), ("dtype", c_int32), ("Wa", c_void_p), ("r", c_void_p),
+                ("W_i", c_void_p), ("W_h", c_void_p), ("b_i", c_void_p), ("b_h", c_void_p)]
+
+
+class hg_temporal_grads(Structure):
+    _fields_ = [("dWa", c_void_p), ("dr", c_void_p), ("dW_i", c_void_p), ("dW_h", c_void_p), ("db_i", c_void_p),
+                ("db_h", c_void_p)]
+
+
 EXPORTS = {
     # name: (restype, argtypes)
     "hg_status_string": (c_char_p, [c_int32]),
@@ -90,6 +100,12 @@ EXPORTS = {
                                c_void_p, c_void_p, c_void_p]),
     "hg_head_bwd": (c_int32, [POINTER(hg_head_params), c_void_p, c_int64, c_float, c_void_p, c_void_p, c_void_p,
                               POINTER(hg_head_grads), c_void_p, c_void_p]),
+    "hg_temporal_workspace_size": (c_int32, [c_int64, c_int32, c_int32, c_int32, POINTER(c_size_t),
+                                             POINTER(c_size_t)]),
+    "hg_temporal_fwd": (c_int32, [POINTER(hg_temporal_params), c_void_p, c_void_p, c_int64, c_void_p, c_void_p,
+                                  c_void_p, c_void_p]),
+    "hg_temporal_bwd": (c_int32, [POINTER(hg_temporal_params), c_void_p, c_void_p, c_int64, c_void_p, c_void_p,
+                                  c_void_p, POINTER(hg_temporal_grads), c_void_p, c_void_p]),
     "hg_timing_enable": (c_int32, [c_int32]),
     "hg_timing_report": (c_int32, [c_char_p, c_size_t]),
 }
@@ -423,3 +439,40 @@ def hg_head_bwd(params: HeadParams, lab_idx, dloss: float, saved, dH, dH_rep, gr
     gr = hg_head_grads(_ptr(grads["W1"]), _ptr(grads["b1"]), _ptr(grads["w2"]), _ptr(grads["b2"]))
     _check(lib().hg_head_bwd(byref(p), _ptr(lab_idx), lab_idx.numel(), float(dloss), _ptr(saved), _ptr(dH),
                              _ptr(dH_rep), byref(gr), _ptr(scratch), _stream(stream)), "hg_head_bwd")
+
+
+# ------------------------------------------------------------------------------------------------
+# temporal module
+# ------------------------------------------------------------------------------------------------
+class TemporalParams:
+    """Packed device parameters of the temporal module (see hg_temporal_params); w = context size."""
+
+    def __init__(self, Wa, r, W_i, W_h, b_i, b_h, w: int):
+        self.t = [x.contiguous() for x in (Wa, r, W_i, W_h, b_i, b_h)]
+        self.d = int(Wa.shape[-1])
+        self.w = int(w)
+        self.dtype = HG_F32 if Wa.dtype == torch.float32 else HG_BF16
+
+    def c(self) -> hg_temporal_params:
+        return hg_temporal_params(self.d, self.w, self.dtype, *(_ptr(x) for x in self.t))
+
+
+def hg_temporal_workspace_size(n: int, d: int, w: int, dtype) -> tuple:
+    s, k = c_size_t(0), c_size_t(0)
+    dt = dtype if isinstance(dtype, int) else (HG_F32 if dtype == torch.float32 else HG_BF16)
+    _check(lib().hg_temporal_workspace_size(int(n), int(d), int(w), dt, byref(s), byref(k)),
+           "hg_temporal_workspace_size")
+    return s.value, k.value
+
+
+def hg_temporal_fwd(params: TemporalParams, X, C, H_out, saved, scratch, stream=None):
+    p = params.c()
+    _check(lib().hg_temporal_fwd(byref(p), _ptr(X), _ptr(C), X.shape[0], _ptr(H_out), _ptr(saved), _ptr(scratch),
+                                 _stream(stream)), "hg_temporal_fwd")
+
+
+def hg_temporal_bwd(params: TemporalParams, X, C, saved, dH_out, dX, grads: dict, scratch, stream=None):
+    p = params.c()
+    gr = hg_temporal_grads(*(_ptr(grads[k]) for k in ("Wa", "r", "W_i", "W_h", "b_i", "b_h")))
+    _check(lib().hg_temporal_bwd(byref(p), _ptr(X), _ptr(C), X.shape[0], _ptr(saved), _ptr(dH_out), _ptr(dX),
+                                 byref(gr), _ptr(scratch), _stream(stream)), "hg_temporal_bwd")
