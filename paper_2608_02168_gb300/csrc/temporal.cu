@@ -10,9 +10,9 @@
 // products read).  The forward saves H~ and the attention weights a; the backward recomputes
 // the rest.
 //
-// This file holds the CUDA-core path (fp32 storage, and bf16 at d = 256): row-tile GEMMs on CUDA
-// cores into fp32 scratch and fused elementwise kernels.  bf16 at d <= 128 runs the tensor-core
-// kernels of temporal_tc.cu.
+// This file holds the CUDA-core path (fp32 storage; bf16 at d = 256 or with (w + 1) d > 512): row-tile
+// GEMMs on CUDA cores into fp32 scratch and fused elementwise kernels.  bf16 at d <= 128 runs the
+// tensor-core kernels of temporal_tc.cu.
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -281,8 +281,13 @@ struct TemporalLayout {
   void* WhT;     // 3d x d
   void* dpre;    // w n x d
   float* part;   // partial sums
-  float* G;      // d x d
+  float* G;      // d x d (3 d x d on the tensor-core path)
   float* tmp;
+  // tensor-core path
+  void* dG;      // 4 x n x d bf16
+  void* dhb;     // n x d bf16
+  void* dHtb;    // n x d bf16
+  float* sums;   // 4 d
 };
 
 int64_t temporal_part_floats(int64_t n, int d, int w) {
@@ -300,6 +305,18 @@ void carve_temporal(void* saved, void* scratch, int64_t n, int d, int w, hg_dtyp
   L->Ht = s.take<char>(nd * esz);
   L->a = s.take<float>((size_t)std::max<int64_t>(n, 1) * w);
   Carve k(scratch);
+  if (temporal_tc_supported(dt, d, w)) {
+    L->dG = k.take<char>(nd * 4 * esz);
+    L->dhb = k.take<char>(nd * esz);
+    L->dHtb = k.take<char>(nd * esz);
+    L->part = k.take<float>(temporal_tc_part_floats(n, d));
+    L->sums = k.take<float>((size_t)4 * d);
+    L->G = k.take<float>((size_t)3 * d * d);
+    L->tmp = k.take<float>(reduce_tmp_floats(1, (int64_t)d * d) + 4 * (size_t)d);
+    if (saved_bytes) *saved_bytes = s.used;
+    if (scratch_bytes) *scratch_bytes = k.used;
+    return;
+  }
   L->U = k.take<float>(nd * w);
   L->Gi = k.take<float>(nd * 3);
   L->Gh = k.take<float>(nd * 3);
@@ -463,6 +480,10 @@ extern "C" hg_status hg_temporal_fwd(const hg_temporal_params* params, const voi
   TemporalLayout L;
   carve_temporal(saved, scratch, n, params->d, params->w, params->dtype, &L, nullptr, nullptr);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (temporal_tc_supported(params->dtype, params->d, params->w)) {
+    const TemporalTcIn in{params, X, C, n, L.Ht, L.a};
+    return temporal_fwd_tc(in, H_out, s);
+  }
   HG_TEMPORAL_DISPATCH(params->dtype, params->d, fwd_simt, params, X, C, n, H_out, L, s);
 }
 
@@ -489,5 +510,10 @@ extern "C" hg_status hg_temporal_bwd(const hg_temporal_params* params, const voi
   }
   TemporalLayout L;
   carve_temporal(const_cast<void*>(saved), scratch, n, d, params->w, params->dtype, &L, nullptr, nullptr);
+  if (temporal_tc_supported(params->dtype, d, params->w)) {
+    const TemporalTcIn in{params, X, C, n, L.Ht, L.a};
+    const TemporalTcScratch sc{L.dG, L.dhb, L.dHtb, L.part, L.sums, L.G, L.tmp};
+    return temporal_bwd_tc(in, dH_out, dX, grads, sc, s);
+  }
   HG_TEMPORAL_DISPATCH(params->dtype, d, bwd_simt, params, X, C, n, dH_out, dX, grads, L, s);
 }

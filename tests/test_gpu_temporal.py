@@ -1,4 +1,7 @@
-"""Temporal module (context attention, Eq. 12; GRU cell, Eq. 13) through the C ABI against the oracle."""
+"""Temporal module (context attention, Eq. 12; GRU cell, Eq. 13) through the C ABI against the oracle.
+
+bf16 with d <= 128 and (w + 1) d <= 512 runs the tensor-core kernels (ragged last tiles, w from 1 to
+the largest the tensor memory holds); fp32, d = 256 and larger windows run the CUDA-core path."""
 import math
 
 import numpy as np
@@ -62,7 +65,7 @@ def check(X, C, p, dOut, dt, got_out, got_dX, got_g):
 
 @pytest.mark.parametrize("dt,d,n,w", [("f32", 64, 1000, 3), ("f32", 128, 777, 2), ("bf16", 128, 5000, 3),
                                       ("bf16", 64, 3001, 4), ("bf16", 256, 1500, 3), ("f32", 256, 300, 1),
-                                      ("bf16", 128, 129, 1)])
+                                      ("bf16", 128, 129, 1), ("bf16", 64, 200, 7), ("bf16", 128, 700, 4)])
 def test_temporal_matches_oracle(dt, d, n, w):
     need_gpu()
     hg = lib()
