@@ -51,6 +51,8 @@ def parse():
     ap.add_argument("--oracle-sample", type=int, default=0, help=argparse.SUPPRESS)  # internal: child process
     ap.add_argument("--oracle-no-head", action="store_true", help=argparse.SUPPRESS)  # internal: child process
     ap.add_argument("--oracle-build-sample", type=int, default=0, help=argparse.SUPPRESS)  # internal: child process
+    ap.add_argument("--oracle-temporal-sample", type=int, default=0, help=argparse.SUPPRESS)  # internal: child process
+    ap.add_argument("--no-temporal", action="store_true", help="skip the temporal-module measurement")
     return ap.parse_args()
 
 
@@ -95,6 +97,22 @@ def oracle_build_sample_main(name: str, k: int):
     ob.build(g["src"], g["dst"], g["rel"], offs, BUILD_K, 0, BUILD_THETA, int(BUILD_BUDGET * offs[-1] / BUILD_K), 21, 22)
     dt = time.perf_counter() - t0
     print(json.dumps({"seconds": dt, "edges": sp.num_edges, "value": sp.num_edges / dt}))
+
+
+def oracle_temporal_sample_main(name: str, k: int):
+    """Child process: the temporal module's oracle (forward and backward) on N / k nodes."""
+    from oracle import temporal as OT
+    sp = hgsynth.spec(name)
+    n = max(1, sp.num_nodes // k)
+    rng = np.random.default_rng(7)
+    X = hgsynth.bf16_round(rng.standard_normal((n, sp.d), dtype=np.float32))
+    C = hgsynth.make_context(sp, rows=n)
+    p = hgsynth.make_temporal_params(sp)
+    dOut = hgsynth.bf16_round(rng.standard_normal((n, sp.d), dtype=np.float32))
+    t0 = time.perf_counter()
+    OT.temporal_backward(X, C, p, dOut, store="bf16" if sp.dtype == "bf16" else "f64")
+    dt = time.perf_counter() - t0
+    print(json.dumps({"seconds": dt, "edges": n, "value": n / dt}))
 
 
 def time_oracle(name: str, k: int, flag: str = "--oracle-sample", with_head: bool = True) -> dict:
@@ -363,6 +381,76 @@ def measure_overlap_build(w, steps: int, warmup: int, dev, with_cpu: bool) -> di
     return res
 
 
+def measure_temporal(sp, steps: int, warmup: int, dev, with_cpu: bool) -> dict:
+    """The temporal module (Section 3.2, Eq. 12-13: attention over each node's last w = 3 states and
+    the GRU cell), forward and backward over every node of the workload, with synthetic spatial
+    embeddings, context states and upstream gradient.  Device time per forward + backward."""
+    import torch
+    from paper_2608_02168_gb300 import hg
+    n, d, w = sp.num_nodes, sp.d, hgsynth.TEMPORAL_WINDOW
+    td = torch.float32 if sp.dtype == "f32" else torch.bfloat16
+    rng = np.random.default_rng(7)
+    X = torch.from_numpy(hgsynth.bf16_round(rng.standard_normal((n, d), dtype=np.float32))).to(dev, td)
+    C = torch.from_numpy(hgsynth.make_context(sp)).to(dev, td)
+    dOut = torch.from_numpy(hgsynth.bf16_round(rng.standard_normal((n, d), dtype=np.float32))).to(dev, td)
+    p = hgsynth.make_temporal_params(sp)
+    prm = hg.TemporalParams(*(torch.from_numpy(p[k]).to(dev, td) for k in ("Wa", "r", "W_i", "W_h", "b_i", "b_h")),
+                            w=w)
+    s_b, k_b = hg.hg_temporal_workspace_size(n, d, w, td)
+    saved = torch.empty(s_b, dtype=torch.uint8, device=dev)
+    scratch = torch.empty(k_b, dtype=torch.uint8, device=dev)
+    out = torch.empty(n, d, dtype=td, device=dev)
+    dX = torch.empty_like(out)
+    f = dict(dtype=torch.float32, device=dev)
+    grads = {"Wa": torch.empty(d, d, **f), "r": torch.empty(d, **f), "W_i": torch.empty(d, 3 * d, **f),
+             "W_h": torch.empty(d, 3 * d, **f), "b_i": torch.empty(3 * d, **f), "b_h": torch.empty(3 * d, **f)}
+
+    def call():
+        hg.hg_temporal_fwd(prm, X, C, out, saved, scratch)
+        hg.hg_temporal_bwd(prm, X, C, saved, dOut, dX, grads, scratch)
+
+    for _ in range(max(warmup, 1)):
+        call()
+    torch.cuda.synchronize()
+    times = []
+    for _ in range(steps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        call()
+        e1.record()
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1))
+    hg.hg_timing_enable(True)
+    hg.hg_timing_report()
+    call()
+    torch.cuda.synchronize()
+    hg.hg_timing_enable(False)
+    rep = hg.hg_timing_report()
+    tot = sum(ms for _, ms in rep.values()) or 1.0
+    ms = statistics.median(times)
+    # algorithmic bytes per node: forward reads x and the w context rows and writes H^t, H~ and a;
+    # backward reads x, the context, dH^t, H~ and a and writes dX
+    b = 4 if sp.dtype == "f32" else 2
+    per_node = (2 * (1 + w) + 2 + 1 + 1 + 1) * d * b + 2 * 4 * w
+    flops = (2 * w + 12 + 36 + 4 * w) * d * d * n  # forward products, backward recomputation and gradients
+    peaks, psrc = load_peaks()
+    ach = per_node * n / (ms / 1e3) / 1e9
+    res = {"ms": round(ms, 4), "nodes_per_s": n / (ms / 1e3), "nodes": n, "w": w, "d": d, "dtype": sp.dtype,
+           "roofline": {"bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                        "peak_source": f"{psrc} hbm_gbs", "frac": round(ach / peaks["hbm_gbs"], 4),
+                        "algorithmic_bytes_per_call": int(per_node * n), "scope": "forward + backward"},
+           "tensor": {"achieved_tflops": round(flops / (ms / 1e3) / 1e12, 1), "peak": peaks.get("bf16_tflops"),
+                      "flops_per_call": int(flops)},
+           "kernel_time_share": {k: round(v / tot, 4) for k, (_, v) in sorted(rep.items(), key=lambda kv: -kv[1][1])},
+           "cpu_baseline": None}
+    if with_cpu:
+        o = time_oracle(sp.name, ORACLE_SCALE, "--oracle-temporal-sample")
+        res["cpu_baseline"] = {"value": o["value"], "unit": "nodes/s", "cores": 1, "kind": "oracle",
+                               "sample": f"{o['edges']:,} nodes (1/{ORACLE_SCALE} of the workload), forward and "
+                                         f"backward of the fp64 numpy oracle, one thread, {o['seconds']:.1f} s"}
+    return res
+
+
 # ------------------------------------------------------------------------------------------------
 def main():
     args = parse()
@@ -371,6 +459,9 @@ def main():
         return
     if args.oracle_build_sample:
         oracle_build_sample_main(args.workload, args.oracle_build_sample)
+        return
+    if args.oracle_temporal_sample:
+        oracle_temporal_sample_main(args.workload, args.oracle_temporal_sample)
         return
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -570,6 +661,9 @@ def run_ours(args, sp, rank, world):
     build = None
     if not args.no_build:
         build = measure_overlap_build(w, args.steps, args.warmup, dev, not args.no_cpu_baseline)
+    temporal = None
+    if not args.no_temporal:
+        temporal = measure_temporal(sp, args.steps, args.warmup, dev, not args.no_cpu_baseline)
     peaks, psrc = load_peaks()
     rf, shares = roofline(report, models, args.steps, peaks, psrc)
     # the same figures for every modelled kernel among the largest shares
@@ -595,7 +689,7 @@ def run_ours(args, sp, rank, world):
         "layers_fwd_bwd_edges_per_s": edges_per_step / ((phase_ms.get("forward", 0) + phase_ms.get("backward", 0)) / 1e3)
         if phase_ms else None,
         "csr_build_edges_per_s": sp.num_edges / (phase_ms["graph"] / 1e3) if phase_ms.get("graph") else None,
-        "cpu_baseline": cpu, "e2e": e2e, "clocks": clk, "overlap_build": build,
+        "cpu_baseline": cpu, "e2e": e2e, "clocks": clk, "overlap_build": build, "temporal": temporal,
         "gpu_launches": int(sum(n for n, _ in report.values())),
         "loss": [float(x) for x in path.loss.cpu()],
         "head_loss": [float(x) for x in path.head_loss.cpu()] if use_head else None,

@@ -15,11 +15,13 @@ from .graphs import (  # noqa: F401
     GraphSpec,
     Workload,
     bf16_round,
+    make_context,
     make_graph,
     make_head_params,
     make_labels,
     make_layer_params,
     make_ring_part,
+    make_temporal_params,
     make_workload,
     ring_ids,
     spec,

@@ -25,8 +25,10 @@ Recipe (stated once here, repeated in the design notes):
   5 % of those positive (the paper gives no rate).  Head weights: Xavier uniform W1 (d x d) and
   w2 (d), zero biases.
 * Seeds: graph = seed, features = seed+1, overlap = seed+2, second view / bank = seed+3,
-  upstream gradient = seed+4, labels = seed+5, layer l weights = seed+100+l, head weights =
-  seed+200; subgraph k mixes k into each seed.
+  upstream gradient = seed+4, labels = seed+5, temporal context = seed+6, layer l weights =
+  seed+100+l, head weights = seed+200, temporal weights = seed+300; subgraph k mixes k into each
+  seed.
+* Temporal context: the w = 3 earlier states of every node, N(0,1) rounded to the storage type.
 """
 from __future__ import annotations
 
@@ -389,3 +391,30 @@ def make_head_params(sp: GraphSpec, random_bias: bool = False) -> dict:
         b1 = np.zeros(d, np.float32)
         b2 = np.zeros(1, np.float32)
     return {k: _store(v, sp.dtype) for k, v in dict(W1=W1, b1=b1, w2=w2, b2=b2).items()}
+
+
+# ------------------------------------------------------------------------------------------------
+# temporal module: context states and weights
+# ------------------------------------------------------------------------------------------------
+TEMPORAL_WINDOW = 3  # w of Section 4.1
+
+
+def make_context(sp: GraphSpec, w: int = TEMPORAL_WINDOW, sub: int = 0, rows: int | None = None) -> np.ndarray:
+    """The w earlier states of every node (w x N x d), N(0,1) rounded to the storage type (seed+6);
+    block k holds the states k + 1 snapshots back."""
+    n = sp.num_nodes if rows is None else rows
+    rng = _rng(sp.seed + 6, sub)
+    return _store(rng.standard_normal((w, n, sp.d), dtype=np.float32), sp.dtype)
+
+
+def make_temporal_params(sp: GraphSpec) -> dict:
+    """Attention Wa (d x d) and r (d), GRU W_i, W_h (d x 3d) and b_i, b_h (3d) (seed+300): Xavier
+    uniform Wa, r ~ N(0, 4/d), and the GRU's usual U(+-1/sqrt(d)) for its weights and biases."""
+    rng = _rng(sp.seed + 300)
+    d = sp.d
+    a = math.sqrt(6.0 / (2 * d))
+    k = 1.0 / math.sqrt(d)
+    p = {"Wa": rng.uniform(-a, a, (d, d)), "r": 2.0 * rng.standard_normal(d) / math.sqrt(d),
+         "W_i": rng.uniform(-k, k, (d, 3 * d)), "W_h": rng.uniform(-k, k, (d, 3 * d)),
+         "b_i": rng.uniform(-k, k, 3 * d), "b_h": rng.uniform(-k, k, 3 * d)}
+    return {key: _store(v.astype(np.float32), sp.dtype) for key, v in p.items()}

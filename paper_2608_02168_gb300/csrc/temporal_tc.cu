@@ -30,9 +30,12 @@ using namespace tc;
 
 namespace {
 
-constexpr int kThreads = 128;
 constexpr int kRows = 128;
 constexpr int kABlk = kRows * 128;  // one 64-column block of a 128-row tile
+// Four warps per 32-lane quarter of tensor memory: warp w reads lanes 32 (w % 4) .. + 31 (rows of the
+// tile) and the column group w / 4, so sixteen warps share each epilogue.
+constexpr int kGroups = 4;
+constexpr int kThreads = 128 * kGroups;
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
@@ -85,6 +88,27 @@ __device__ __forceinline__ float tsum16(float (&v)[16]) {
   return v[0];
 }
 
+// Sum over the warp of v[L & 7], returned to lanes L, L + 8, L + 16 and L + 24.
+__device__ __forceinline__ float tsum8(float (&v)[8]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    v[i] += __shfl_xor_sync(0xffffffffu, v[i], 16);
+    v[i] += __shfl_xor_sync(0xffffffffu, v[i], 8);
+  }
+#pragma unroll
+  for (int s = 4; s >= 1; s >>= 1) {
+    const bool hi = (lane & s) != 0;
+#pragma unroll
+    for (int i = 0; i < s; ++i) {
+      const float send = hi ? v[i] : v[i + s];
+      const float keep = hi ? v[i + s] : v[i];
+      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, s);
+    }
+  }
+  return v[0];
+}
+
 // 8 bf16 of row `row` starting at column c (a multiple of 8) of a swizzled K-major tile.
 __device__ __forceinline__ void tile_row8(const uint8_t* tile, int row, int c, float* f) {
   unpack(ld16(tile + (c >> 6) * kABlk + sw128_offset(row, (c & 63) * 2)), f, __nv_bfloat16());
@@ -116,6 +140,7 @@ template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     temporal_attn_tc(const __grid_constant__ CUtensorMap tm_C, const __grid_constant__ CUtensorMap tm_Wa, TAttnArgs p) {
   using C = TCfg<D>;
+  constexpr int CW = D / kGroups;  // columns of a warp's group
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   uint8_t* Wimg = smem;
@@ -123,7 +148,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* bars = reinterpret_cast<uint64_t*>(Cimg + p.w * C::kA);
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2);
   float* rf = reinterpret_cast<float*>(bars + 4);
-  const int tid = threadIdx.x, warp = tid >> 5;
+  float* epart = rf + D;  // [kGroups][w][128]
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int q = warp & 3, cg = warp >> 2;
+  const int row = q * 32 + lane;
   const int64_t r0 = (int64_t)blockIdx.x * kRows;
   uint32_t tcols = 32;
   while (tcols < (uint32_t)(p.w * D)) tcols <<= 1;
@@ -162,21 +190,29 @@ __global__ void __launch_bounds__(kThreads, 1)
     ok = false;
   }
   fence_after_sync();
-  const int64_t r = r0 + tid;
-  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+  const int64_t r = r0 + row;
+  const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + cg * CW;
+  // partial scores over this warp's columns, combined over the groups in order
+  for (int k = 0; k < p.w; ++k) {
+    float s = 0.f;
+#pragma unroll
+    for (int c = 0; c < CW; c += 8) {
+      float u[8];
+      tmem_ld8(trow + k * D + c, u);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) s = fmaf(rf[cg * CW + c + e], tanhf(u[e]), s);
+    }
+    epart[(cg * p.w + k) * kRows + row] = s;
+  }
+  __syncthreads();
   float e[kTemporalMaxW];
   float m = -INFINITY;
 #pragma unroll
   for (int k = 0; k < kTemporalMaxW; ++k) {
     if (k >= p.w) break;
     float s = 0.f;
-#pragma unroll 1
-    for (int c = 0; c < D; c += 32) {
-      float u[32];
-      tmem_ld32(trow + k * D + c, u);
 #pragma unroll
-      for (int q = 0; q < 32; ++q) s = fmaf(rf[c + q], tanhf(u[q]), s);
-    }
+    for (int g = 0; g < kGroups; ++g) s += epart[(g * p.w + k) * kRows + row];
     e[k] = s;
     m = fmaxf(m, s);
   }
@@ -191,21 +227,22 @@ __global__ void __launch_bounds__(kThreads, 1)
   for (int k = 0; k < kTemporalMaxW; ++k) {
     if (k >= p.w) break;
     e[k] /= sum;
-    if (r < p.n) p.a[r * p.w + k] = e[k];
+    if (cg == 0 && r < p.n) p.a[r * p.w + k] = e[k];
   }
   if (r < p.n && ok) {
-#pragma unroll 1
-    for (int c = 0; c < D; c += 8) {
+#pragma unroll
+    for (int c = 0; c < CW; c += 8) {
+      const int col = cg * CW + c;
       float h[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int k = 0; k < kTemporalMaxW; ++k) {
         if (k >= p.w) break;
         float x[8];
-        tile_row8(Cimg + k * C::kA, tid, c, x);
+        tile_row8(Cimg + k * C::kA, row, col, x);
 #pragma unroll
-        for (int q = 0; q < 8; ++q) h[q] = fmaf(e[k], x[q], h[q]);
+        for (int t = 0; t < 8; ++t) h[t] = fmaf(e[k], x[t], h[t]);
       }
-      st16(p.Ht + r * D + c, pack(h, __nv_bfloat16()));
+      st16(p.Ht + r * D + col, pack(h, __nv_bfloat16()));
     }
   }
   fence_before_sync();
@@ -293,82 +330,76 @@ __global__ void __launch_bounds__(kThreads, 1)
     ok = false;
   }
   fence_after_sync();
-  const int64_t r = r0 + tid;
+  constexpr int CW = D / kGroups;
+  const int q = warp & 3, cg = warp >> 2;
+  const int row = q * 32 + lane;
+  const int64_t r = r0 + row;
   const bool live = ok && r < p.n;
-  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
-#pragma unroll 1
-  for (int c = 0; c < D; c += 16) {
-    float ar[16], az[16], anx[16], anh[16];
-    tmem_ld16(trow + 0 * D + c, ar);
-    tmem_ld16(trow + 1 * D + c, az);
-    tmem_ld16(trow + 2 * D + c, anx);
-    tmem_ld16(trow + 3 * D + c, anh);
-    float h[16], g[16];
-    tile_row8(Himg, tid, c, h);
-    tile_row8(Himg, tid, c + 8, h + 8);
+  const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16);
+#pragma unroll
+  for (int c0 = 0; c0 < CW; c0 += 8) {
+    const int c = cg * CW + c0;
+    float ar[8], az[8], anx[8], anh[8], h[8], g[8];
+    tmem_ld8(trow + 0 * D + c, ar);
+    tmem_ld8(trow + 1 * D + c, az);
+    tmem_ld8(trow + 2 * D + c, anx);
+    tmem_ld8(trow + 3 * D + c, anh);
+    tile_row8(Himg, row, c, h);
     if (kBwd) {
       if (live) {
         unpack(ld16(p.dOut + r * D + c), g, __nv_bfloat16());
-        unpack(ld16(p.dOut + r * D + c + 8), g + 8, __nv_bfloat16());
       } else {
 #pragma unroll
-        for (int q = 0; q < 16; ++q) g[q] = 0.f;
+        for (int t = 0; t < 8; ++t) g[t] = 0.f;
       }
     }
 #pragma unroll
-    for (int q = 0; q < 16; ++q) {
-      const int col = c + q;
-      const float rg = sigm(ar[q] + bias[col] + bias[3 * D + col]);
-      const float z = sigm(az[q] + bias[D + col] + bias[4 * D + col]);
-      const float hn = anh[q] + bias[5 * D + col];
-      const float nn = tanhf(anx[q] + bias[2 * D + col] + rg * hn);
+    for (int t = 0; t < 8; ++t) {
+      const int col = c + t;
+      const float rg = sigm(ar[t] + bias[col] + bias[3 * D + col]);
+      const float z = sigm(az[t] + bias[D + col] + bias[4 * D + col]);
+      const float hn = anh[t] + bias[5 * D + col];
+      const float nn = tanhf(anx[t] + bias[2 * D + col] + rg * hn);
       if (!kBwd) {
-        ar[q] = (1.f - z) * nn + z * h[q];
+        ar[t] = (1.f - z) * nn + z * h[t];
       } else {
-        const float dn = g[q] * (1.f - z);
-        const float dz = g[q] * (h[q] - nn);
+        const float dn = g[t] * (1.f - z);
+        const float dz = g[t] * (h[t] - nn);
         const float dpn = dn * (1.f - nn * nn);
-        ar[q] = dpn * hn * rg * (1.f - rg);  // dpre_r
-        az[q] = dz * z * (1.f - z);          // dpre_z
-        anx[q] = dpn;                        // dpre_n
-        anh[q] = dpn * rg;                   // dhn
-        h[q] = g[q] * z;                     // direct gradient of H~
+        ar[t] = dpn * hn * rg * (1.f - rg);  // dpre_r
+        az[t] = dz * z * (1.f - z);          // dpre_z
+        anx[t] = dpn;                        // dpre_n
+        anh[t] = dpn * rg;                   // dhn
+        h[t] = g[t] * z;                     // direct gradient of H~
       }
     }
     if (!kBwd) {
-      if (live) {
-        st16(p.out + r * D + c, pack(ar, __nv_bfloat16()));
-        st16(p.out + r * D + c + 8, pack(ar + 8, __nv_bfloat16()));
-      }
+      if (live) st16(p.out + r * D + c, pack(ar, __nv_bfloat16()));
     } else {
       if (live) {
         __nv_bfloat16* dst = p.dG + r * D + c;
         const int64_t blk = p.n * D;
         st16(dst, pack(ar, __nv_bfloat16()));
-        st16(dst + 8, pack(ar + 8, __nv_bfloat16()));
         st16(dst + blk, pack(az, __nv_bfloat16()));
-        st16(dst + blk + 8, pack(az + 8, __nv_bfloat16()));
         st16(dst + 2 * blk, pack(anx, __nv_bfloat16()));
-        st16(dst + 2 * blk + 8, pack(anx + 8, __nv_bfloat16()));
         st16(dst + 3 * blk, pack(anh, __nv_bfloat16()));
-        st16(dst + 3 * blk + 8, pack(anh + 8, __nv_bfloat16()));
         st16(p.dh + r * D + c, pack(h, __nv_bfloat16()));
-        st16(p.dh + r * D + c + 8, pack(h + 8, __nv_bfloat16()));
       }
-      const float s0 = tsum16(ar), s1 = tsum16(az), s2 = tsum16(anx), s3 = tsum16(anh);
-      if (lane < 16) {
-        colred[warp * 4 * D + 0 * D + c + lane] = s0;
-        colred[warp * 4 * D + 1 * D + c + lane] = s1;
-        colred[warp * 4 * D + 2 * D + c + lane] = s2;
-        colred[warp * 4 * D + 3 * D + c + lane] = s3;
+      const float s0 = tsum8(ar), s1 = tsum8(az), s2 = tsum8(anx), s3 = tsum8(anh);
+      if (lane < 8) {
+        float* cr = colred + q * 4 * D + c + lane;
+        cr[0 * D] = s0;
+        cr[1 * D] = s1;
+        cr[2 * D] = s2;
+        cr[3 * D] = s3;
       }
     }
   }
   if (kBwd) {
     __syncthreads();
-    for (int q = tid; q < 4 * D; q += kThreads)
-      p.part[(int64_t)blockIdx.x * 4 * D + q] =
-          ((colred[q] + colred[4 * D + q]) + colred[8 * D + q]) + colred[12 * D + q];
+    for (int t = tid; t < 4 * D; t += kThreads)
+      p.part[(int64_t)blockIdx.x * 4 * D + t] =
+          ((colred[t] + colred[4 * D + t]) + colred[8 * D + t]) + colred[12 * D + t];
   }
   fence_before_sync();
   __syncthreads();
@@ -454,27 +485,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     ok = false;
   }
   fence_after_sync();
-  const int64_t r = r0 + tid;
+  constexpr int CW = D / kGroups;
+  const int q = warp & 3, cg = warp >> 2, lane = tid & 31;
+  const int64_t r = r0 + q * 32 + lane;
   const bool live = ok && r < p.n;
-  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
-#pragma unroll 1
-  for (int c = 0; c < D; c += 16) {
-    float x[16], h[16];
-    tmem_ld16(trow + c, x);
-    tmem_ld16(trow + D + c, h);
-    if (live) {
-      float d0[8], d1[8];
-      unpack(ld16(p.dh + r * D + c), d0, __nv_bfloat16());
-      unpack(ld16(p.dh + r * D + c + 8), d1, __nv_bfloat16());
+  const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16);
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        h[q] += d0[q];
-        h[8 + q] += d1[q];
-      }
+  for (int c0 = 0; c0 < CW; c0 += 8) {
+    const int c = cg * CW + c0;
+    float x[8], h[8];
+    tmem_ld8(trow + c, x);
+    tmem_ld8(trow + D + c, h);
+    if (live) {
+      float d0[8];
+      unpack(ld16(p.dh + r * D + c), d0, __nv_bfloat16());
+#pragma unroll
+      for (int t = 0; t < 8; ++t) h[t] += d0[t];
       st16(p.dX + r * D + c, pack(x, __nv_bfloat16()));
-      st16(p.dX + r * D + c + 8, pack(x + 8, __nv_bfloat16()));
       st16(p.dHt + r * D + c, pack(h, __nv_bfloat16()));
-      st16(p.dHt + r * D + c + 8, pack(h + 8, __nv_bfloat16()));
     }
   }
   fence_before_sync();
@@ -501,6 +529,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     temporal_attn_bwd_tc(const __grid_constant__ CUtensorMap tm_C, const __grid_constant__ CUtensorMap tm_Wa,
                          TAttnBwdArgs p) {
   using C = TCfg<D>;
+  constexpr int CW = D / kGroups;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   uint8_t* Wimg = smem;
@@ -509,8 +538,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* bars = reinterpret_cast<uint64_t*>(Pimg + C::kA + kABlk);
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 4);
   float* rf = reinterpret_cast<float*>(bars + 6);
-  float* drred = rf + D;  // [4][D]
+  float* drred = rf + D;                    // [4 quarters][D]
+  float* dapart = drred + 4 * D;            // [kGroups][w][128]
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int q = warp & 3, cg = warp >> 2;
+  const int row = q * 32 + lane;
   uint32_t tcols = 32;
   while (tcols < (uint32_t)((p.w + 1) * D)) tcols <<= 1;
   if (tid == 0) {
@@ -524,10 +556,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   fence_after_sync();
   const uint32_t tmem = *tslot;
   const uint32_t acc_w = tmem + p.w * D;
-  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
-  float drl[D / 32];
+  const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + cg * CW;
+  float drl[CW / 8];
 #pragma unroll
-  for (int i = 0; i < D / 32; ++i) drl[i] = 0.f;
+  for (int i = 0; i < CW / 8; ++i) drl[i] = 0.f;
   bool ok = true;
   uint32_t it = 0, mm = 0;  // tiles done, dW_a commits done
   for (int t = blockIdx.x; t < p.tiles && ok; t += gridDim.x, ++it) {
@@ -551,41 +583,53 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     ok = __syncthreads_and(ok);
     if (!ok) break;
-    if (!mbar_wait(&bars[1], it & 1)) {
-      ok = false;
-    }
+    if (!mbar_wait(&bars[1], it & 1)) ok = false;
     ok = __syncthreads_and(ok);
     if (!ok) break;
     fence_after_sync();
-    const int64_t r = r0 + tid;
+    const int64_t r = r0 + row;
     const bool live = r < p.n;
-    // da_k = <dH~, c_k>, de = a (da - sum_k a_k da_k)
-    float de[kTemporalMaxW];
+    // partial da_k = <dH~, c_k> over this warp's columns, combined over the groups in order
     {
       float da[kTemporalMaxW];
 #pragma unroll
       for (int k = 0; k < kTemporalMaxW; ++k) da[k] = 0.f;
       if (live) {
-#pragma unroll 1
-        for (int c = 0; c < D; c += 8) {
+#pragma unroll
+        for (int c0 = 0; c0 < CW; c0 += 8) {
+          const int col = cg * CW + c0;
           float g[8];
-          unpack(ld16(p.dHt + r * D + c), g, __nv_bfloat16());
+          unpack(ld16(p.dHt + r * D + col), g, __nv_bfloat16());
 #pragma unroll
           for (int k = 0; k < kTemporalMaxW; ++k) {
             if (k >= p.w) break;
             float x[8];
-            tile_row8(Cimg + k * C::kA, tid, c, x);
+            tile_row8(Cimg + k * C::kA, row, col, x);
 #pragma unroll
-            for (int q = 0; q < 8; ++q) da[k] = fmaf(g[q], x[q], da[k]);
+            for (int e = 0; e < 8; ++e) da[k] = fmaf(g[e], x[e], da[k]);
           }
         }
       }
+#pragma unroll
+      for (int k = 0; k < kTemporalMaxW; ++k) {
+        if (k >= p.w) break;
+        dapart[(cg * p.w + k) * kRows + row] = da[k];
+      }
+    }
+    __syncthreads();
+    float de[kTemporalMaxW];
+    {
+      float da[kTemporalMaxW];
       float s = 0.f;
 #pragma unroll
       for (int k = 0; k < kTemporalMaxW; ++k) {
         if (k >= p.w) break;
+        float v = 0.f;
+#pragma unroll
+        for (int g = 0; g < kGroups; ++g) v += dapart[(g * p.w + k) * kRows + row];
+        da[k] = v;
         de[k] = live ? p.a[r * p.w + k] : 0.f;
-        s = fmaf(de[k], da[k], s);
+        s = fmaf(de[k], v, s);
       }
 #pragma unroll
       for (int k = 0; k < kTemporalMaxW; ++k) {
@@ -593,26 +637,27 @@ __global__ void __launch_bounds__(kThreads, 1)
         de[k] = de[k] * (da[k] - s);
       }
     }
+    for (int k = 0; k < p.w; ++k) {
+      float dek = 0.f;
 #pragma unroll
-    for (int k = 0; k < kTemporalMaxW; ++k) {
-      if (k >= p.w) break;
-#pragma unroll 1
-      for (int c = 0; c < D; c += 32) {
-        float u[32];
-        tmem_ld32(trow + k * D + c, u);
-        float pk[32];
+      for (int kk = 0; kk < kTemporalMaxW; ++kk)
+        if (kk == k) dek = de[kk];
 #pragma unroll
-        for (int q = 0; q < 32; ++q) {
-          const float th = tanhf(u[q]);
-          pk[q] = de[k] * rf[c + q] * (1.f - th * th);
-          u[q] = de[k] * th;
+      for (int c0 = 0; c0 < CW; c0 += 8) {
+        const int col = cg * CW + c0;
+        float u[8], pk[8];
+        tmem_ld8(trow + k * D + c0, u);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float th = tanhf(u[e]);
+          pk[e] = dek * rf[col + e] * (1.f - th * th);
+          u[e] = dek * th;
         }
+        tile_put8(Pimg, row, col, pk);
+        const float cs = tsum8(u);
 #pragma unroll
-        for (int q = 0; q < 32; q += 8) tile_put8(Pimg, tid, c + q, pk + q);
-        const float cs = tsum32(u);
-#pragma unroll
-        for (int i = 0; i < D / 32; ++i)
-          if (i == c / 32) drl[i] += cs;
+        for (int i = 0; i < CW / 8; ++i)
+          if (i == c0 / 8) drl[i] += cs;
       }
       fence_async_smem();
       __syncthreads();
@@ -636,21 +681,25 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   if (!ok) record_device_error(p.status, kErrTimeout);
-  // dW_a partial: thread t holds row t of the accumulator (rows < D are the gradient's)
+  // dW_a partial: TMEM lane t holds row t of the accumulator (rows < D are the gradient's); the four
+  // column groups write their columns
   float* outw = p.dWa_part + (int64_t)blockIdx.x * D * D;
-#pragma unroll 1
-  for (int c = 0; c < D; c += 32) {
-    float v[32];
-    tmem_ld32(trow + p.w * D + c, v);
-    if (tid < D) {
 #pragma unroll
-      for (int q = 0; q < 32; q += 4)
-        *reinterpret_cast<float4*>(outw + (int64_t)tid * D + c + q) =
-            ok && it > 0 ? make_float4(v[q], v[q + 1], v[q + 2], v[q + 3]) : make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int c0 = 0; c0 < CW; c0 += 8) {
+    float v[8];
+    tmem_ld8(tmem + ((uint32_t)(q * 32) << 16) + p.w * D + cg * CW + c0, v);
+    if (row < D) {
+      const bool good = ok && it > 0;
+      float* o = outw + (int64_t)row * D + cg * CW + c0;
+      *reinterpret_cast<float4*>(o) = good ? make_float4(v[0], v[1], v[2], v[3]) : make_float4(0.f, 0.f, 0.f, 0.f);
+      *reinterpret_cast<float4*>(o + 4) = good ? make_float4(v[4], v[5], v[6], v[7]) : make_float4(0.f, 0.f, 0.f, 0.f);
     }
   }
+  // dr partial: lane L of a warp holds column (L & 7) of each of its 8-column chunks
+  if (lane < 8) {
 #pragma unroll
-  for (int i = 0; i < D / 32; ++i) drred[warp * D + i * 32 + lane] = drl[i];
+    for (int i = 0; i < CW / 8; ++i) drred[q * D + cg * CW + i * 8 + lane] = drl[i];
+  }
   fence_before_sync();
   __syncthreads();
   for (int c = tid; c < D; c += kThreads)
@@ -703,7 +752,8 @@ inline size_t smem_for(size_t need, uint32_t tcols) {
 
 template <int D>
 size_t attn_smem(int w) {
-  return smem_for((size_t)TCfg<D>::kW + (size_t)w * TCfg<D>::kA + 32 + 4 * D + 1024, tmem_cols(w * D));
+  return smem_for((size_t)TCfg<D>::kW + (size_t)w * TCfg<D>::kA + 32 + 4 * D + 4 * kGroups * w * kRows + 1024,
+                  tmem_cols(w * D));
 }
 template <int D>
 size_t gru_smem() { return smem_for(2 * TCfg<D>::kA + 3 * TCfg<D>::kW + 48 + 88 * D + 1024, 4 * D); }
@@ -712,7 +762,8 @@ size_t dx_smem() { return smem_for(3 * TCfg<D>::kA + 3 * TCfg<D>::kW + 48 + 1024
 template <int D>
 size_t attn_bwd_smem(int w) {
   // persistent: one CTA per SM
-  return smem_for((size_t)TCfg<D>::kW + (size_t)(w + 1) * TCfg<D>::kA + kABlk + 48 + 20 * D + 1024, 512);
+  return smem_for((size_t)TCfg<D>::kW + (size_t)(w + 1) * TCfg<D>::kA + kABlk + 48 + 20 * D +
+                      4 * kGroups * w * kRows + 1024, 512);
 }
 
 template <int D>
