@@ -11,6 +11,7 @@ so the two sides see identical numbers.
 """
 from .graphs import (  # noqa: F401
     RELATIONS,
+    TEMPORAL_WINDOW,
     WORKLOADS,
     GraphSpec,
     Workload,
