@@ -7,3 +7,4 @@ from .hg_oracle import (  # noqa: F401
 from . import overlap_build  # noqa: F401  (overlapping-subgraph construction, Eq. 4-5)
 from . import head  # noqa: F401  (MeanAgg, MLP head, masked BCE and joint objective, Eq. 18-20)
 from . import temporal  # noqa: F401  (context attention over the last w states and the GRU cell, Eq. 12-13)
+from . import hgt  # noqa: F401  (attention variant of the layer, Eq. 6-11)
