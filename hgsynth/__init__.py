@@ -19,6 +19,7 @@ from .graphs import (  # noqa: F401
     make_context,
     make_graph,
     make_head_params,
+    make_hgt_params,
     make_labels,
     make_layer_params,
     make_ring_part,

@@ -418,3 +418,26 @@ def make_temporal_params(sp: GraphSpec) -> dict:
          "W_i": rng.uniform(-k, k, (d, 3 * d)), "W_h": rng.uniform(-k, k, (d, 3 * d)),
          "b_i": rng.uniform(-k, k, 3 * d), "b_h": rng.uniform(-k, k, 3 * d)}
     return {key: _store(v.astype(np.float32), sp.dtype) for key, v in p.items()}
+
+
+def make_hgt_params(sp: GraphSpec, heads: int, layer: int = 0, bias_margin: float | None = None) -> dict:
+    """Attention layer weights (seed+400+layer): Xavier uniform W_K, W_Q, W_V, W_agg (T x d x d); W_att,
+    W_msg (R x S x d_h x d_h) ~ N(0, 1/d_h); mu = 1 (fp32); small N(0, 0.1) biases and LayerNorm
+    shifts, gains 1 + N(0, 0.1); bias_margin: b_agg of +-margin per column (seeded signs)."""
+    rng = _rng(sp.seed + 400 + layer)
+    d, R, T = sp.d, sp.num_rels, 2
+    dh = d // heads
+    a = math.sqrt(6.0 / (2 * d))
+    p = {"W_K": rng.uniform(-a, a, (T, d, d)), "W_Q": rng.uniform(-a, a, (T, d, d)),
+         "W_V": rng.uniform(-a, a, (T, d, d)),
+         "b_K": 0.1 * rng.standard_normal((T, d)), "b_Q": 0.1 * rng.standard_normal((T, d)),
+         "b_V": 0.1 * rng.standard_normal((T, d)),
+         "W_att": rng.standard_normal((R, heads, dh, dh)) / math.sqrt(dh),
+         "W_msg": rng.standard_normal((R, heads, dh, dh)) / math.sqrt(dh),
+         "W_agg": rng.uniform(-a, a, (T, d, d)), "b_agg": 0.1 * rng.standard_normal((T, d)),
+         "ln_gamma": 1.0 + 0.1 * rng.standard_normal((T, d)), "ln_beta": 0.1 * rng.standard_normal((T, d))}
+    if bias_margin is not None:
+        p["b_agg"] = bias_margin * rng.choice([-1.0, 1.0], size=(T, d))
+    out = {k: _store(np.asarray(v, np.float32), sp.dtype) for k, v in p.items()}
+    out["mu"] = np.ones(R, np.float32)
+    return out

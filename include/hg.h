@@ -278,6 +278,74 @@ hg_status hg_overlap_build(const int32_t* src, const int32_t* dst, const int32_t
                            void* workspace, size_t workspace_bytes, hg_stream stream);
 
 /* ------------------------------------------------------------------------------------------- */
+/* Attention layer (Heterogeneous Graph Transformer, Section 3.2, Eq. 6-11)                       */
+/* ------------------------------------------------------------------------------------------- */
+
+/* Parameters of one attention layer, device pointers of the storage type unless noted; T node
+ * types, R relations, S heads of width d_h = d / S (S a power of two, 1 <= S <= 32):
+ *   W_K, W_Q, W_V  [T][d][d] (input x output), b_K, b_Q, b_V [T][d]   key / query / value maps
+ *   W_att, W_msg   [R][S][d_h][d_h]                                   per relation and head
+ *   mu             [R] fp32 (device)                                  prior of each relation
+ *   W_agg [T][d][d], b_agg [T][d], ln_gamma / ln_beta [T][d]           as in hg_layer_params */
+typedef struct {
+  int32_t d;
+  int32_t heads;
+  hg_dtype dtype;
+  hg_act act;
+  int32_t layernorm;
+  float ln_eps;
+  const void* W_K;
+  const void* W_Q;
+  const void* W_V;
+  const void* b_K;
+  const void* b_Q;
+  const void* b_V;
+  const void* W_att;
+  const void* W_msg;
+  const float* mu;
+  const void* W_agg;
+  const void* b_agg;
+  const void* ln_gamma;
+  const void* ln_beta;
+} hg_hgt_params;
+
+/* Gradients, device fp32, shapes as the parameters, OVERWRITTEN (dln_* may be NULL without
+ * LayerNorm). */
+typedef struct {
+  float* dW_K;
+  float* dW_Q;
+  float* dW_V;
+  float* db_K;
+  float* db_Q;
+  float* db_V;
+  float* dW_att;
+  float* dW_msg;
+  float* dmu;
+  float* dW_agg;
+  float* db_agg;
+  float* dln_gamma;
+  float* dln_beta;
+} hg_hgt_grads;
+
+hg_status hg_hgt_workspace_size(const hg_graph* graph, const hg_hgt_params* params, size_t* saved_bytes,
+                                size_t* scratch_bytes);
+
+/* One attention layer on the graph (node features H_in, N x d, storage type):
+ *   K, Q, V = H W_K + b_K, ... per node type;
+ *   Eq. 6    score^s(e) = (K^s(i) W_att[r, s] . Q^s(j)) mu[r] / sqrt(d_h) for an edge e = i -> j of r;
+ *   Eq. 8    alpha^s(e) = softmax over every in-edge of j (all relations);
+ *   Eq. 7, 9, 10  h~_j = concat_s sum_e alpha^s(e) V^s(i) W_msg[r, s];
+ *   Eq. 11   H_out = act(h~ W_agg + b_agg) + H_in, then LayerNorm per type when enabled.
+ * H_out must not alias H_in.  `saved` feeds hg_hgt_bwd. */
+hg_status hg_hgt_fwd(const hg_graph* graph, const hg_hgt_params* params, const void* H_in, void* H_out, void* saved,
+                     void* scratch, hg_stream stream);
+
+/* Backward: dH_in (N x d, OVERWRITTEN; NULL = skip) = dL/dH_in for the upstream gradient dH_out,
+ * and every parameter gradient. */
+hg_status hg_hgt_bwd(const hg_graph* graph, const hg_hgt_params* params, const void* H_in, const void* saved,
+                     const void* dH_out, void* dH_in, const hg_hgt_grads* grads, void* scratch, hg_stream stream);
+
+/* ------------------------------------------------------------------------------------------- */
 /* Prediction head and joint objective (Section 3.4, Eq. 18-20; MeanAgg / MLP / loss steps of     */
 /* Algorithm 1)                                                                                   */
 /* ------------------------------------------------------------------------------------------- */

@@ -66,33 +66,10 @@ void timing_end(int slot, cudaStream_t s) {
   cudaEventRecord(g_recs[slot].b, s);
 }
 
-// ---------------------------------------------------------------------------------------------
-// layer workspace layout
-// ---------------------------------------------------------------------------------------------
-struct LayerLayout {
-  void* M;        // saved: csr_rows x d relation means
-  void* Z;        // saved (fp32 storage only): N x d
-  void* U;        // saved: N x d pre-activation
-  float2* stats;  // saved: N row statistics
-  void* V;        // saved (bf16 only): R x d x d fused weights W_r W_agg
-  void* Vt;       // saved (bf16 only): their transposes
-  float* agg_part;  // scratch: chunk partials
-  void* dY;       // scratch: N x d
-  void* dU;
-  void* dZ;       // scratch (fp32 storage only)
-  void* dMs;      // scratch: csr_rows x d
-  float* cpart;   // scratch: column partials (blocks x 3 x d)
-  float* wpart;   // scratch: splits x d x d
-  float* rtmp;    // scratch: levels of the fixed-order reductions
-  float* G;       // scratch (bf16 only): R x d x d products M_r^T dU
-  void* WrelT;    // scratch (fp32 storage only): R x d x d
-  void* WaggT;    // scratch (fp32 storage only): T x d x d
-};
-
 static size_t elem_size(hg_dtype dt) { return dt == HG_F32 ? 4 : 2; }
 
-static void carve_layer(const hg_graph* g, int d, hg_dtype dt, void* saved, void* scratch, LayerLayout* L,
-                        size_t* saved_bytes, size_t* scratch_bytes) {
+void carve_layer(const hg_graph* g, int d, hg_dtype dt, void* saved, void* scratch, LayerLayout* L,
+                 size_t* saved_bytes, size_t* scratch_bytes) {
   const GraphMeta& m = g->meta;
   const int64_t N = m.type_off[m.num_types];
   const size_t b = elem_size(dt);
@@ -130,7 +107,7 @@ static void carve_layer(const hg_graph* g, int d, hg_dtype dt, void* saved, void
   if (scratch_bytes) *scratch_bytes = k.used;
 }
 
-static RelDst rel_dst_of(const GraphMeta& m) {
+RelDst rel_dst_of(const GraphMeta& m) {
   RelDst rd{};
   for (int r = 0; r < m.num_rels; ++r) rd.v[r] = m.rel_dst[r];
   return rd;
@@ -255,12 +232,22 @@ extern "C" hg_status hg_layer_fwd(const hg_graph* graph, const hg_layer_params* 
   HG_TRY(check_buf(scratch, "scratch"));
   HG_REQUIRE(H_in != H_out, "H_in and H_out must not alias");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  const GraphMeta& m = graph->meta;
   const int d = p->d;
-  const size_t b = elem_size(p->dtype);
   LayerLayout L;
   carve_layer(graph, d, p->dtype, saved, scratch, &L, nullptr, nullptr);
   HG_TRY(aggregate_forward(graph, p->dtype, d, H_in, L.M, L.agg_part, s));
+  return project_forward(graph, p, H_in, H_out, L, s);
+}
+
+namespace hg {
+
+// Eq. 7 and Eq. 11 from the relation rows in L.M: U = sum_r M_r W_r W_agg + b, activation,
+// residual, optional LayerNorm.
+hg_status project_forward(const hg_graph* graph, const hg_layer_params* p, const void* H_in, void* H_out,
+                          const LayerLayout& L, cudaStream_t s) {
+  const GraphMeta& m = graph->meta;
+  const int d = p->d;
+  const size_t b = elem_size(p->dtype);
   if (p->dtype == HG_BF16) {
     // tensor-core path: U = sum_r M_r V_r with the fused weights V_r = W_r W_agg[t_r]
     HG_TRY(tc_fuse_weights(d, p->W_rel, p->W_agg, rel_dst_of(m), m.num_rels, L.V, L.Vt, s));
@@ -318,6 +305,8 @@ extern "C" hg_status hg_layer_fwd(const hg_graph* graph, const hg_layer_params* 
   return HG_OK;
 }
 
+}  // namespace hg
+
 extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* p, const void* H_in, const void* saved,
                                   const void* dH_out, void* dH_in, const hg_layer_grads* grads, void* scratch,
                                   hg_stream stream) {
@@ -332,11 +321,22 @@ extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* 
   HG_REQUIRE(!p->layernorm || (grads->dln_gamma && grads->dln_beta), "layernorm needs dln_gamma and dln_beta");
   HG_REQUIRE(dH_in != dH_out, "dH_in and dH_out must not alias");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  LayerLayout L;
+  carve_layer(graph, p->d, p->dtype, const_cast<void*>(saved), scratch, &L, nullptr, nullptr);
+  HG_TRY(project_backward(graph, p, H_in, dH_out, grads, L, true, s));
+  if (dH_in) HG_TRY(aggregate_backward(graph, p->dtype, p->d, L.dMs, L.dY, dH_in, L.agg_part, s));
+  return HG_OK;
+}
+
+namespace hg {
+
+// Backward of project_forward: L.dY = the residual path's dL/dH_in, L.dMs = dL/dM_r (divided by
+// deg_r when deg_scale is set, for the mean's transposed gather), and every weight gradient.
+hg_status project_backward(const hg_graph* graph, const hg_layer_params* p, const void* H_in, const void* dH_out,
+                           const hg_layer_grads* grads, const LayerLayout& L, bool deg_scale, cudaStream_t s) {
   const GraphMeta& m = graph->meta;
   const int d = p->d;
   const size_t b = elem_size(p->dtype);
-  LayerLayout L;
-  carve_layer(graph, d, p->dtype, const_cast<void*>(saved), scratch, &L, nullptr, nullptr);
   const bool tc = p->dtype == HG_BF16;
   if (!tc) {
     HG_TRY(transpose_weights(p->dtype, d, p->W_rel, L.WrelT, m.num_rels, s));
@@ -369,7 +369,7 @@ extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* 
       a.U = (const __nv_bfloat16*)L.U;
       a.stats = L.stats;
       a.gamma = p->layernorm ? (const __nv_bfloat16*)p->ln_gamma + (size_t)t * d : nullptr;
-      a.csr_ptr = graph->csr_ptr;
+      a.csr_ptr = deg_scale ? graph->csr_ptr : nullptr;
       a.dY = (__nv_bfloat16*)L.dY;
       a.dU = (__nv_bfloat16*)L.dU;
       a.dMs = (__nv_bfloat16*)L.dMs;
@@ -395,7 +395,7 @@ extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* 
         a.W_relT[a.nrel] = (const char*)L.WrelT + (size_t)r * d * d * b;
         ++a.nrel;
       }
-      a.csr_ptr = graph->csr_ptr;
+      a.csr_ptr = deg_scale ? graph->csr_ptr : nullptr;
       a.dY = L.dY;
       a.dU = L.dU;
       a.dZ = L.dZ;
@@ -444,6 +444,7 @@ extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* 
   if (tc)  // dW_r = G_r W_agg^T, dW_agg[t] = sum_{r -> t} W_r^T G_r
     HG_TRY(tc_wgrad_finish(d, L.G, p->W_rel, p->W_agg, rel_dst_of(m), m.num_rels, m.num_types, grads->dW_rel,
                            grads->dW_agg, s));
-  if (dH_in) HG_TRY(aggregate_backward(graph, p->dtype, d, L.dMs, L.dY, dH_in, L.agg_part, s));
   return HG_OK;
 }
+
+}  // namespace hg

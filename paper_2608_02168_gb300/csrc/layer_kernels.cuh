@@ -37,7 +37,7 @@ struct BwdArgs {
   int nrel;
   int64_t mrow0[kMaxRels];
   const void* W_relT[kMaxRels];  // W_r^T
-  const int32_t* csr_ptr;        // degrees of the relation rows
+  const int32_t* csr_ptr;        // degrees of the relation rows (null: no 1/deg scaling)
   void* dY;                      // node rows
   void* dU;                      // node rows
   void* dZ;                      // node rows
@@ -124,5 +124,36 @@ size_t reduce_tmp_floats(int splits, int64_t count);
 hg_status reduce_partials3(const float* part, int64_t stride, int splits, int64_t seg, float* out0, float* out1,
                            float* out2, cudaStream_t s);
 int wgrad_splits(int64_t n);
+
+// Buffers of one layer (saved for the backward, and scratch).
+struct LayerLayout {
+  void* M;        // saved: csr_rows x d relation rows (means, or attention-weighted sums)
+  void* Z;        // saved (fp32 storage only): N x d
+  void* U;        // saved: N x d pre-activation
+  float2* stats;  // saved: N row statistics
+  void* V;        // saved (bf16 only): R x d x d fused weights W_r W_agg
+  void* Vt;       // saved (bf16 only): their transposes
+  float* agg_part;  // scratch: chunk partials
+  void* dY;       // scratch: N x d
+  void* dU;
+  void* dZ;       // scratch (fp32 storage only)
+  void* dMs;      // scratch: csr_rows x d
+  float* cpart;   // scratch: column partials (blocks x 3 x d)
+  float* wpart;   // scratch: splits x d x d
+  float* rtmp;    // scratch: levels of the fixed-order reductions
+  float* G;       // scratch (bf16 only): R x d x d products M_r^T dU
+  void* WrelT;    // scratch (fp32 storage only): R x d x d
+  void* WaggT;    // scratch (fp32 storage only): T x d x d
+};
+void carve_layer(const hg_graph* g, int d, hg_dtype dt, void* saved, void* scratch, LayerLayout* L,
+                 size_t* saved_bytes, size_t* scratch_bytes);
+RelDst rel_dst_of(const GraphMeta& m);
+// Eq. 7 and Eq. 11 from the relation rows in L.M (bias, activation, residual, optional LayerNorm).
+hg_status project_forward(const hg_graph* graph, const hg_layer_params* p, const void* H_in, void* H_out,
+                          const LayerLayout& L, cudaStream_t s);
+// Its backward: L.dY (residual path), L.dMs (dL/dM_r, divided by deg_r when deg_scale), the weight
+// gradients into grads.
+hg_status project_backward(const hg_graph* graph, const hg_layer_params* p, const void* H_in, const void* dH_out,
+                           const hg_layer_grads* grads, const LayerLayout& L, bool deg_scale, cudaStream_t s);
 
 }  // namespace hg

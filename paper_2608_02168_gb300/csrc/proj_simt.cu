@@ -227,8 +227,8 @@ __global__ void __launch_bounds__(256) proj_bwd_simt(BwdArgs a) {
       const int m = ty * RM + i;
       if (m >= nv) continue;
       const int64_t row = a.mrow0[r] + m0 + m;
-      const int deg = a.csr_ptr[row + 1] - a.csr_ptr[row];
-      const float sc = deg > 0 ? __fdiv_rn(1.0f, (float)deg) : 0.f;
+      const int deg = a.csr_ptr ? a.csr_ptr[row + 1] - a.csr_ptr[row] : 0;
+      const float sc = !a.csr_ptr ? 1.f : (deg > 0 ? __fdiv_rn(1.0f, (float)deg) : 0.f);
       float v[CN];
 #pragma unroll
       for (int j = 0; j < CN; ++j) v[j] = acc[i][j] * sc;

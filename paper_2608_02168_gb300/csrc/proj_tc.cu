@@ -690,8 +690,8 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
         if (jb % C::kEpiGroups != grp) continue;
         const uint32_t k = jb % NB;
         const int64_t crow = a.mrow0[r] + (live ? m : 0);
-        const int deg = live ? a.csr_ptr[crow + 1] - a.csr_ptr[crow] : 0;
-        const float sc = deg > 0 ? __fdiv_rn(1.0f, (float)deg) : 0.f;
+        const int deg = live && a.csr_ptr ? a.csr_ptr[crow + 1] - a.csr_ptr[crow] : 0;
+        const float sc = !a.csr_ptr ? 1.f : (deg > 0 ? __fdiv_rn(1.0f, (float)deg) : 0.f);
         ok = mbar_wait(&acc_full[k], (jb / NB) & 1);
         if (!ok) break;
         fence_after_sync();

@@ -42,6 +42,20 @@ class hg_layer_grads(Structure):
                 ("dln_beta", c_void_p)]
 
 
+class hg_hgt_params(Structure):
+    _fields_ = [("d", c_int32), ("heads", c_int32), ("dtype", c_int32), ("act", c_int32), ("layernorm", c_int32),
+                ("ln_eps", c_float), ("W_K", c_void_p), ("W_Q", c_void_p), ("W_V", c_void_p), ("b_K", c_void_p),
+                ("b_Q", c_void_p), ("b_V", c_void_p), ("W_att", c_void_p), ("W_msg", c_void_p), ("mu", c_void_p),
+                ("W_agg", c_void_p), ("b_agg", c_void_p), ("ln_gamma", c_void_p), ("ln_beta", c_void_p)]
+
+
+HGT_KEYS = ("W_K", "W_Q", "W_V", "b_K", "b_Q", "b_V", "W_att", "W_msg", "mu", "W_agg", "b_agg", "ln_gamma", "ln_beta")
+
+
+class hg_hgt_grads(Structure):
+    _fields_ = [("d" + k, c_void_p) for k in HGT_KEYS]
+
+
 class hg_head_params(Structure):
     _fields_ = [("d", c_int32), ("dtype", c_int32), ("W1", c_void_p), ("b1", c_void_p), ("w2", c_void_p),
                 ("b2", c_void_p)]
@@ -106,6 +120,10 @@ EXPORTS = {
                                   c_void_p, c_void_p]),
     "hg_temporal_bwd": (c_int32, [POINTER(hg_temporal_params), c_void_p, c_void_p, c_int64, c_void_p, c_void_p,
                                   c_void_p, POINTER(hg_temporal_grads), c_void_p, c_void_p]),
+    "hg_hgt_workspace_size": (c_int32, [c_void_p, POINTER(hg_hgt_params), POINTER(c_size_t), POINTER(c_size_t)]),
+    "hg_hgt_fwd": (c_int32, [c_void_p, POINTER(hg_hgt_params), c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),
+    "hg_hgt_bwd": (c_int32, [c_void_p, POINTER(hg_hgt_params), c_void_p, c_void_p, c_void_p, c_void_p,
+                             POINTER(hg_hgt_grads), c_void_p, c_void_p]),
     "hg_timing_enable": (c_int32, [c_int32]),
     "hg_timing_report": (c_int32, [c_char_p, c_size_t]),
 }
@@ -476,3 +494,40 @@ def hg_temporal_bwd(params: TemporalParams, X, C, saved, dH_out, dX, grads: dict
     gr = hg_temporal_grads(*(_ptr(grads[k]) for k in ("Wa", "r", "W_i", "W_h", "b_i", "b_h")))
     _check(lib().hg_temporal_bwd(byref(p), _ptr(X), _ptr(C), X.shape[0], _ptr(saved), _ptr(dH_out), _ptr(dX),
                                  byref(gr), _ptr(scratch), _stream(stream)), "hg_temporal_bwd")
+
+
+# ------------------------------------------------------------------------------------------------
+# attention layer (Heterogeneous Graph Transformer)
+# ------------------------------------------------------------------------------------------------
+class HgtParams:
+    """Packed device parameters of one attention layer (see hg_hgt_params); mu is fp32."""
+
+    def __init__(self, tensors: dict, heads: int, act: str = "relu", layernorm: bool = True, ln_eps: float = 1e-5):
+        self.t = {k: (tensors[k].contiguous() if tensors.get(k) is not None else None) for k in HGT_KEYS}
+        self.heads, self.act, self.layernorm, self.ln_eps = int(heads), act, layernorm, ln_eps
+        self.d = int(self.t["W_K"].shape[-1])
+        self.dtype = HG_F32 if self.t["W_K"].dtype == torch.float32 else HG_BF16
+
+    def c(self) -> hg_hgt_params:
+        return hg_hgt_params(self.d, self.heads, self.dtype, ACTS[self.act], 1 if self.layernorm else 0, self.ln_eps,
+                             *(_ptr(self.t[k]) for k in HGT_KEYS))
+
+
+def hg_hgt_workspace_size(g: Graph, params: HgtParams) -> tuple:
+    s, k = c_size_t(0), c_size_t(0)
+    p = params.c()
+    _check(lib().hg_hgt_workspace_size(g.handle, byref(p), byref(s), byref(k)), "hg_hgt_workspace_size")
+    return s.value, k.value
+
+
+def hg_hgt_fwd(g: Graph, params: HgtParams, H_in, H_out, saved, scratch, stream=None):
+    p = params.c()
+    _check(lib().hg_hgt_fwd(g.handle, byref(p), _ptr(H_in), _ptr(H_out), _ptr(saved), _ptr(scratch), _stream(stream)),
+           "hg_hgt_fwd")
+
+
+def hg_hgt_bwd(g: Graph, params: HgtParams, H_in, saved, dH_out, dH_in, grads: dict, scratch, stream=None):
+    p = params.c()
+    gr = hg_hgt_grads(*(_ptr(grads.get(k)) for k in HGT_KEYS))
+    _check(lib().hg_hgt_bwd(g.handle, byref(p), _ptr(H_in), _ptr(saved), _ptr(dH_out), _ptr(dH_in), byref(gr),
+                            _ptr(scratch), _stream(stream)), "hg_hgt_bwd")

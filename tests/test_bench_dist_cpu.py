@@ -76,3 +76,13 @@ def test_reference_arm_only_on_rank_zero():
     line = json.loads(r.stdout.strip().splitlines()[-1])
     assert line["impl"] == "reference" and line["value"] > 0 and line["e2e"]["h2d_bytes_per_step"] == 0
     assert line["cpu_baseline"]["kind"] == "oracle"
+
+
+def test_bench_generator_references_exist():
+    """Every hgsynth name bench.py uses exists (the bench runs only on a GPU machine)."""
+    import ast
+    import hgsynth
+    src = open(os.path.join(ROOT, "bench.py")).read()
+    names = {n.attr for n in ast.walk(ast.parse(src))
+             if isinstance(n, ast.Attribute) and isinstance(n.value, ast.Name) and n.value.id == "hgsynth"}
+    assert names and all(hasattr(hgsynth, n) for n in names), sorted(n for n in names if not hasattr(hgsynth, n))
