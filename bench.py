@@ -53,6 +53,8 @@ def parse():
     ap.add_argument("--oracle-build-sample", type=int, default=0, help=argparse.SUPPRESS)  # internal: child process
     ap.add_argument("--oracle-temporal-sample", type=int, default=0, help=argparse.SUPPRESS)  # internal: child process
     ap.add_argument("--no-temporal", action="store_true", help="skip the temporal-module measurement")
+    ap.add_argument("--no-hgt", action="store_true", help="skip the attention-layer measurement")
+    ap.add_argument("--oracle-hgt-sample", type=int, default=0, help=argparse.SUPPRESS)  # internal: child process
     return ap.parse_args()
 
 
@@ -113,6 +115,31 @@ def oracle_temporal_sample_main(name: str, k: int):
     OT.temporal_backward(X, C, p, dOut, store="bf16" if sp.dtype == "bf16" else "f64")
     dt = time.perf_counter() - t0
     print(json.dumps({"seconds": dt, "edges": n, "value": n / dt}))
+
+
+HGT_HEADS = 4  # attention heads (Section 4.1)
+
+
+def oracle_hgt_sample_main(name: str, k: int):
+    """Child process: the attention layer's oracle, L layers forward and backward, on a 1/k-size
+    instance of the workload."""
+    from oracle import hgt as OH
+    sp = scaled(hgsynth.spec(name), k)
+    w = hgsynth.make_workload(sp, with_ids=False)
+    g = w.graph
+    store = "bf16" if sp.dtype == "bf16" else "f64"
+    ps = [hgsynth.make_hgt_params(sp, HGT_HEADS, layer=l) for l in range(sp.layers)]
+    args = (g["src"], g["dst"], g["rel"], g["type_offsets"], g["rels"])
+    t0 = time.perf_counter()
+    hs = [np.asarray(w.X, np.float64)]
+    for p in ps:
+        hs.append(OH.hgt_forward(*args, p, hs[-1], HGT_HEADS, store=store)[0])
+    dh = np.asarray(w.dH_top, np.float64)
+    for l in range(sp.layers - 1, -1, -1):
+        dh, _ = OH.hgt_backward(*args, ps[l], hs[l], dh, HGT_HEADS, store=store)
+    dt = time.perf_counter() - t0
+    print(json.dumps({"seconds": dt, "edges": sp.num_edges, "layers": sp.layers,
+                      "value": sp.layers * sp.num_edges / dt}))
 
 
 def time_oracle(name: str, k: int, flag: str = "--oracle-sample", with_head: bool = True) -> dict:
@@ -451,6 +478,70 @@ def measure_temporal(sp, steps: int, warmup: int, dev, with_cpu: bool) -> dict:
     return res
 
 
+def measure_hgt(w, steps: int, warmup: int, dev, with_cpu: bool) -> dict:
+    """The attention variant of the layer (Eq. 6-11, HGT_HEADS heads): the workload's L layers
+    forward and backward on its graph (CSR built once), synthetic upstream gradient.  Device time
+    per forward + backward of the stack."""
+    import torch
+    from paper_2608_02168_gb300 import hg
+    sp, g = w.spec, w.graph
+    td = torch.float32 if sp.dtype == "f32" else torch.bfloat16
+    G = hg.hg_build_csr(*(torch.from_numpy(g[k]).to(dev) for k in ("src", "dst", "rel")), g["type_offsets"],
+                        g["rels"])
+    params = []
+    for l in range(sp.layers):
+        p = hgsynth.make_hgt_params(sp, HGT_HEADS, layer=l)
+        params.append(hg.HgtParams({k: torch.from_numpy(v).to(dev, torch.float32 if k == "mu" else td)
+                                    for k, v in p.items()}, HGT_HEADS))
+    sb, kb = hg.hg_hgt_workspace_size(G, params[0])
+    saved = [torch.empty(sb, dtype=torch.uint8, device=dev) for _ in params]
+    scratch = torch.empty(kb, dtype=torch.uint8, device=dev)
+    N, d = sp.num_nodes, sp.d
+    Hs = [torch.from_numpy(w.X).to(dev, td)] + [torch.empty(N, d, dtype=td, device=dev) for _ in params]
+    dHs = [torch.empty(N, d, dtype=td, device=dev) for _ in range(len(params))] + \
+          [torch.from_numpy(w.dH_top).to(dev, td)]
+    f = dict(dtype=torch.float32, device=dev)
+    grads = [{k: torch.empty(np.shape(v), **f) for k, v in hgsynth.make_hgt_params(sp, HGT_HEADS).items()}
+             for _ in params]
+
+    def call():
+        for l, P in enumerate(params):
+            hg.hg_hgt_fwd(G, P, Hs[l], Hs[l + 1], saved[l], scratch)
+        for l in range(len(params) - 1, -1, -1):
+            hg.hg_hgt_bwd(G, params[l], Hs[l], saved[l], dHs[l + 1], dHs[l], grads[l], scratch)
+
+    for _ in range(max(warmup, 1)):
+        call()
+    torch.cuda.synchronize()
+    times = []
+    for _ in range(steps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        call()
+        e1.record()
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1))
+    hg.hg_timing_enable(True)
+    hg.hg_timing_report()
+    call()
+    torch.cuda.synchronize()
+    hg.hg_timing_enable(False)
+    rep = hg.hg_timing_report()
+    tot = sum(ms for _, ms in rep.values()) or 1.0
+    ms = statistics.median(times)
+    res = {"ms": round(ms, 4), "layers": sp.layers, "heads": HGT_HEADS,
+           "layers_fwd_bwd_edges_per_s": sp.layers * sp.num_edges / (ms / 1e3),
+           "kernel_time_share": {k: round(v / tot, 4) for k, (_, v) in sorted(rep.items(), key=lambda kv: -kv[1][1])},
+           "cpu_baseline": None}
+    if with_cpu:
+        o = time_oracle(sp.name, REFERENCE_SCALE, "--oracle-hgt-sample")
+        res["cpu_baseline"] = {"value": o["value"], "unit": UNIT, "cores": 1, "kind": "oracle",
+                               "sample": f"1/{REFERENCE_SCALE}-size instance ({o['edges']:,} edges), {sp.layers} layers "
+                                         f"forward and backward of the fp64 numpy oracle, one thread, "
+                                         f"{o['seconds']:.1f} s"}
+    return res
+
+
 # ------------------------------------------------------------------------------------------------
 def main():
     args = parse()
@@ -462,6 +553,9 @@ def main():
         return
     if args.oracle_temporal_sample:
         oracle_temporal_sample_main(args.workload, args.oracle_temporal_sample)
+        return
+    if args.oracle_hgt_sample:
+        oracle_hgt_sample_main(args.workload, args.oracle_hgt_sample)
         return
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -664,6 +758,9 @@ def run_ours(args, sp, rank, world):
     temporal = None
     if not args.no_temporal:
         temporal = measure_temporal(sp, args.steps, args.warmup, dev, not args.no_cpu_baseline)
+    hgt = None
+    if not args.no_hgt:
+        hgt = measure_hgt(w, args.steps, args.warmup, dev, not args.no_cpu_baseline)
     peaks, psrc = load_peaks()
     rf, shares = roofline(report, models, args.steps, peaks, psrc)
     # the same figures for every modelled kernel among the largest shares
@@ -689,7 +786,7 @@ def run_ours(args, sp, rank, world):
         "layers_fwd_bwd_edges_per_s": edges_per_step / ((phase_ms.get("forward", 0) + phase_ms.get("backward", 0)) / 1e3)
         if phase_ms else None,
         "csr_build_edges_per_s": sp.num_edges / (phase_ms["graph"] / 1e3) if phase_ms.get("graph") else None,
-        "cpu_baseline": cpu, "e2e": e2e, "clocks": clk, "overlap_build": build, "temporal": temporal,
+        "cpu_baseline": cpu, "e2e": e2e, "clocks": clk, "overlap_build": build, "temporal": temporal, "hgt": hgt,
         "gpu_launches": int(sum(n for n, _ in report.values())),
         "loss": [float(x) for x in path.loss.cpu()],
         "head_loss": [float(x) for x in path.head_loss.cpu()] if use_head else None,

@@ -15,7 +15,8 @@
 //   and the dense products back to H and to the weights.
 // Edge work is warp per row (a lane holds d / 32 consecutive features, the 32 / S lanes of a head
 // reduce by shuffles); rows above the hub degree are split into chunks whose partial results are
-// merged in chunk order, so every reduction has a fixed order (deterministic, atomic-free).
+// merged in chunk order, so every reduction has a fixed order (deterministic, atomic-free).  The
+// dense row products run on the tensor cores for bf16 (rows_gemm_tc.cu) and on CUDA cores for fp32.
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -669,7 +670,7 @@ struct HgtLayout {
   float* Gq;      // R x d x d
 };
 
-constexpr int64_t kColRows = 2048;
+constexpr int64_t kColRows = 128;  // rows per block of the bias sums (many blocks in flight)
 
 int64_t max_type_rows(const GraphMeta& m) {
   int64_t r = 1;
@@ -763,6 +764,9 @@ template <typename T, int D>
 hg_status gemm(const void* A, int64_t lda, const void* B, const void* bias, int K, int64_t n, void* out, int64_t ldo,
                int ocol0, int accumulate, cudaStream_t s) {
   if (n <= 0) return HG_OK;
+  if constexpr (sizeof(T) == 2) {  // bf16: tensor cores (every product here has K = lda = D)
+    if (lda == D && K == D) return rows_gemm_tc(D, A, n, B, bias, out, ldo, ocol0, accumulate, s);
+  }
   return launch("hgt_gemm_simt", hgt_gemm_simt<T, D>, dim3((unsigned)ceil_div(n, kBM)), dim3(256),
                 sizeof(float) * kKC * D, s, (const T*)A, lda, (const T*)B, (const T*)bias, K, n, (T*)out, ldo, ocol0,
                 accumulate);

@@ -124,6 +124,10 @@ size_t reduce_tmp_floats(int splits, int64_t count);
 hg_status reduce_partials3(const float* part, int64_t stride, int splits, int64_t seg, float* out0, float* out1,
                            float* out2, cudaStream_t s);
 int wgrad_splits(int64_t n);
+// Tensor-core row product (bf16): out[r][ocol0 + c] (=, or += when accumulate) A[r] B + bias,
+// A: n x d rows (row stride d), B: d x d row-major, bias: d or null; out row stride ldo.
+hg_status rows_gemm_tc(int d, const void* A, int64_t n, const void* B, const void* bias, void* out, int64_t ldo,
+                       int ocol0, int accumulate, cudaStream_t s);
 
 // Buffers of one layer (saved for the backward, and scratch).
 struct LayerLayout {
