@@ -78,14 +78,6 @@ __device__ __forceinline__ float head_sum(float x, int lph) {
   return x;
 }
 
-__device__ __forceinline__ int rel_of_row(const GraphMeta& m, int64_t row) {
-  int r = 0;
-#pragma unroll
-  for (int k = 1; k < kMaxRels; ++k)
-    if (k < m.num_rels && row >= m.row_base[k]) r = k;
-  return r;
-}
-
 // ---------------------------------------------------------------------------------------------
 // derived weights (fp64 arithmetic, one rounding)
 // ---------------------------------------------------------------------------------------------
@@ -217,6 +209,7 @@ __global__ void hgt_colsum(const T* __restrict__ X, int64_t ldx, int d, int64_t 
 // ---------------------------------------------------------------------------------------------
 struct HgtArgs {
   GraphMeta meta;
+  int8_t rslot[kMaxTypes][kMaxRels];  // relations into each type in relation order, -1 past the last
   int64_t N, csr_rows;
   int S;
   const int32_t* csr_ptr;
@@ -232,7 +225,7 @@ struct HgtArgs {
   void* Srows;       // csr_rows x d: attention-weighted value sums (forward output, backward input)
   const void* dS;    // csr_rows x d
   float2* stats;     // N x S: running maximum and sum of each target's softmax
-  float* Dj;         // N x S: sum_r <dS_r(j), S_r(j)> per head
+  float4* rstat;     // csr_rows x S: the target's (max, 1 / sum, D_j) on each of its rows, per head
   void* dQp;         // csr_rows x d
   void* dK;          // N x d
   void* dV;          // N x d
@@ -326,8 +319,9 @@ __global__ void __launch_bounds__(256) hgt_fwd_chunks(HgtArgs a) {
 
 // One warp per node j: the softmax over all of j's in-edges (its rows of every relation into its
 // type, hub rows through their chunk partials in order), S_r(j) = sum alpha V for each relation.
-template <typename T, int D>
-__global__ void __launch_bounds__(256) hgt_fwd_nodes(HgtArgs a) {
+// The row bounds and query slices of all of j's rows are loaded before any edge.
+template <typename T, int D, int KS>
+__global__ void __launch_bounds__(256, (D <= 128 && KS <= 4) ? 3 : 1) hgt_fwd_nodes(HgtArgs a) {
   constexpr int E = D / 32;
   const int lane = threadIdx.x & 31, lph = 32 / a.S;
   const int64_t j = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -335,18 +329,32 @@ __global__ void __launch_bounds__(256) hgt_fwd_nodes(HgtArgs a) {
   const int t = node_type_of(a.meta, j);
   const int64_t jl = j - a.meta.type_off[t];
   const int stride = 2 * a.S + D;
-  float m = -INFINITY, l = 0.f, acc[kMaxRels][E];
+  int64_t row[KS];
+  int c0[KS], c1[KS];
+  int64_t e0[KS], e1[KS];
+  float q[KS][E];
 #pragma unroll
-  for (int k = 0; k < kMaxRels; ++k)
+  for (int k = 0; k < KS; ++k) {
+    const int r = a.rslot[t][k];
+    row[k] = r >= 0 ? a.meta.row_base[r] + jl : -1;
+    if (row[k] >= 0) {
+      c0[k] = a.csr_chunk_ofs[row[k]];
+      c1[k] = a.csr_chunk_ofs[row[k] + 1];
+      e0[k] = a.csr_ptr[row[k]];
+      e1[k] = a.csr_ptr[row[k] + 1];
+      load_slice<T, E>((const T*)a.Qp + row[k] * D + lane * E, q[k]);
+    }
+  }
+  float m = -INFINITY, l = 0.f, acc[KS][E];
+#pragma unroll
+  for (int k = 0; k < KS; ++k)
 #pragma unroll
     for (int e = 0; e < E; ++e) acc[k][e] = 0.f;
 #pragma unroll
-  for (int r = 0; r < kMaxRels; ++r) {
-    if (r >= a.meta.num_rels || a.meta.rel_dst[r] != t) continue;
-    const int64_t row = a.meta.row_base[r] + jl;
-    const int c0 = a.csr_chunk_ofs[row], c1 = a.csr_chunk_ofs[row + 1];
-    if (c1 > c0) {
-      for (int c = c0; c < c1; ++c) {
+  for (int k = 0; k < KS; ++k) {
+    if (row[k] < 0) continue;
+    if (c1[k] > c0[k]) {
+      for (int c = c0[k]; c < c1[k]; ++c) {
         const float* p = a.part + (int64_t)c * stride;
         const float pm = p[2 * (lane / lph)], pl = p[2 * (lane / lph) + 1];
         const float mn = fmaxf(m, pm);
@@ -354,35 +362,34 @@ __global__ void __launch_bounds__(256) hgt_fwd_nodes(HgtArgs a) {
           const float so = expf(m - mn);
           l *= so;
 #pragma unroll
-          for (int k = 0; k < kMaxRels; ++k)
+          for (int kk = 0; kk < KS; ++kk)
 #pragma unroll
-            for (int e = 0; e < E; ++e) acc[k][e] *= so;
+            for (int e = 0; e < E; ++e) acc[kk][e] *= so;
           m = mn;
         }
         const float sp = expf(pm - m);
         l = fmaf(pl, sp, l);
 #pragma unroll
-        for (int e = 0; e < E; ++e) acc[r][e] = fmaf(sp, p[2 * a.S + lane * E + e], acc[r][e]);
+        for (int e = 0; e < E; ++e) acc[k][e] = fmaf(sp, p[2 * a.S + lane * E + e], acc[k][e]);
       }
     } else {
-      float q[E];
-      load_slice<T, E>((const T*)a.Qp + row * D + lane * E, q);
-      fwd_edges<T, D, kMaxRels>(a, a.csr_ptr[row], a.csr_ptr[row + 1], q, lph, m, l, acc, r);
+      fwd_edges<T, D, KS>(a, e0[k], e1[k], q[k], lph, m, l, acc, k);
     }
   }
   const float inv = l > 0.f ? 1.f / l : 0.f;
 #pragma unroll
-  for (int r = 0; r < kMaxRels; ++r) {
-    if (r >= a.meta.num_rels || a.meta.rel_dst[r] != t) continue;
+  for (int k = 0; k < KS; ++k) {
+    if (row[k] < 0) continue;
     float o[E];
 #pragma unroll
-    for (int e = 0; e < E; ++e) o[e] = acc[r][e] * inv;
-    store_slice<T, E>((T*)a.Srows + (a.meta.row_base[r] + jl) * D + lane * E, o);
+    for (int e = 0; e < E; ++e) o[e] = acc[k][e] * inv;
+    store_slice<T, E>((T*)a.Srows + row[k] * D + lane * E, o);
   }
   if (lane % lph == 0) a.stats[j * a.S + lane / lph] = make_float2(l > 0.f ? m : 0.f, l);
 }
 
-// D^s_j = sum over j's relation rows of <dS_r(j), S_r(j)> on head s.  One warp per node.
+// D^s_j = sum over j's relation rows of <dS_r(j), S_r(j)> on head s, stored with the softmax statistics
+// on every row of j (the source pass reads them by row).  One warp per node.
 template <typename T, int D>
 __global__ void __launch_bounds__(256) hgt_bwd_dstats(HgtArgs a) {
   constexpr int E = D / 32;
@@ -403,7 +410,15 @@ __global__ void __launch_bounds__(256) hgt_bwd_dstats(HgtArgs a) {
     for (int e = 0; e < E; ++e) s = fmaf(x[e], y[e], s);
   }
   s = head_sum(s, lph);
-  if (lane % lph == 0) a.Dj[j * a.S + lane / lph] = s;
+  if (lane % lph == 0) {
+    const float2 st = a.stats[j * a.S + lane / lph];
+    const float4 v = make_float4(st.x, st.y > 0.f ? 1.f / st.y : 0.f, s, 0.f);
+#pragma unroll
+    for (int r = 0; r < kMaxRels; ++r) {
+      if (r >= a.meta.num_rels || a.meta.rel_dst[r] != t) continue;
+      a.rstat[(a.meta.row_base[r] + jl) * a.S + lane / lph] = v;
+    }
+  }
 }
 
 // sum over the edges [beg, end) of one row (relation r, target j) of de K(i), with
@@ -446,12 +461,6 @@ __device__ __forceinline__ void dst_edges(const HgtArgs& a, int64_t beg, int64_t
   }
 }
 
-// The target of CSR row `row` and the softmax statistics of this lane's head.
-__device__ __forceinline__ int64_t target_of(const GraphMeta& m, int64_t row) {
-  const int r = rel_of_row(m, row);
-  return row - m.row_base[r] + m.type_off[m.rel_dst[r]];
-}
-
 template <typename T, int D>
 __global__ void __launch_bounds__(256) hgt_bwd_dst_chunks(HgtArgs a) {
   constexpr int E = D / 32;
@@ -462,50 +471,60 @@ __global__ void __launch_bounds__(256) hgt_bwd_dst_chunks(HgtArgs a) {
     const int row = a.csr_chunk_row[c];
     const int64_t beg = (int64_t)a.csr_ptr[row] + (int64_t)(c - a.csr_chunk_ofs[row]) * kChunkEdges;
     const int64_t end = min((int64_t)a.csr_ptr[row + 1], beg + kChunkEdges);
-    const int64_t j = target_of(a.meta, row);
-    const float2 st = a.stats[j * a.S + h];
+    const float4 st = a.rstat[(int64_t)row * a.S + h];
     float q[E], g[E], acc[E];
     load_slice<T, E>((const T*)a.Qp + (int64_t)row * D + lane * E, q);
     load_slice<T, E>((const T*)a.dS + (int64_t)row * D + lane * E, g);
 #pragma unroll
     for (int e = 0; e < E; ++e) acc[e] = 0.f;
-    dst_edges<T, D>(a, beg, end, q, g, st.x, st.y > 0.f ? 1.f / st.y : 0.f, a.Dj[j * a.S + h], lph, acc);
+    dst_edges<T, D>(a, beg, end, q, g, st.x, st.y, st.z, lph, acc);
 #pragma unroll
     for (int e = 0; e < E; ++e) a.part[c * D + lane * E + e] = acc[e];
   }
 }
 
-// dQ'_r(j) for every relation row of node j (hub rows: their chunk partials in order).
-template <typename T, int D>
-__global__ void __launch_bounds__(256) hgt_bwd_dst_nodes(HgtArgs a) {
+// dQ'_r(j) for every relation row of node j (hub rows: their chunk partials in order); the row
+// bounds, query and gradient slices of all of j's rows are loaded before any edge.
+template <typename T, int D, int KS>
+__global__ void __launch_bounds__(256, (D <= 128 && KS <= 4) ? 3 : 1) hgt_bwd_dst_nodes(HgtArgs a) {
   constexpr int E = D / 32;
   const int lane = threadIdx.x & 31, lph = 32 / a.S, h = lane / lph;
   const int64_t j = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   if (j >= a.N) return;
   const int t = node_type_of(a.meta, j);
   const int64_t jl = j - a.meta.type_off[t];
-  const float2 st = a.stats[j * a.S + h];
-  const float inv_l = st.y > 0.f ? 1.f / st.y : 0.f;
-  const float Dh = a.Dj[j * a.S + h];
+  int64_t row[KS];
+  int c0[KS], c1[KS];
+  int64_t e0[KS], e1[KS];
+  float q[KS][E], g[KS][E];
 #pragma unroll
-  for (int r = 0; r < kMaxRels; ++r) {
-    if (r >= a.meta.num_rels || a.meta.rel_dst[r] != t) continue;
-    const int64_t row = a.meta.row_base[r] + jl;
+  for (int k = 0; k < KS; ++k) {
+    const int r = a.rslot[t][k];
+    row[k] = r >= 0 ? a.meta.row_base[r] + jl : -1;
+    if (row[k] >= 0) {
+      c0[k] = a.csr_chunk_ofs[row[k]];
+      c1[k] = a.csr_chunk_ofs[row[k] + 1];
+      e0[k] = a.csr_ptr[row[k]];
+      e1[k] = a.csr_ptr[row[k] + 1];
+      load_slice<T, E>((const T*)a.Qp + row[k] * D + lane * E, q[k]);
+      load_slice<T, E>((const T*)a.dS + row[k] * D + lane * E, g[k]);
+    }
+  }
+  const float4 st = row[0] >= 0 ? a.rstat[row[0] * a.S + h] : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+  for (int k = 0; k < KS; ++k) {
+    if (row[k] < 0) continue;
     float acc[E];
 #pragma unroll
     for (int e = 0; e < E; ++e) acc[e] = 0.f;
-    const int c0 = a.csr_chunk_ofs[row], c1 = a.csr_chunk_ofs[row + 1];
-    if (c1 > c0) {
-      for (int c = c0; c < c1; ++c)
+    if (c1[k] > c0[k]) {
+      for (int c = c0[k]; c < c1[k]; ++c)
 #pragma unroll
         for (int e = 0; e < E; ++e) acc[e] += a.part[(int64_t)c * D + lane * E + e];
     } else {
-      float q[E], g[E];
-      load_slice<T, E>((const T*)a.Qp + row * D + lane * E, q);
-      load_slice<T, E>((const T*)a.dS + row * D + lane * E, g);
-      dst_edges<T, D>(a, a.csr_ptr[row], a.csr_ptr[row + 1], q, g, st.x, inv_l, Dh, lph, acc);
+      dst_edges<T, D>(a, e0[k], e1[k], q[k], g[k], st.x, st.y, st.z, lph, acc);
     }
-    store_slice<T, E>((T*)a.dQp + row * D + lane * E, acc);
+    store_slice<T, E>((T*)a.dQp + row[k] * D + lane * E, acc);
   }
 }
 
@@ -522,16 +541,13 @@ __device__ __forceinline__ void src_edges(const HgtArgs& a, int64_t beg, int64_t
 #pragma unroll
     for (int u = 0; u < kBatch; ++u) row[u] = e0 + u < end ? __ldg(a.node_col + e0 + u) : -1;
     float q[kBatch][E], g[kBatch][E];
-    float2 st[kBatch];
-    float Dh[kBatch];
+    float4 st[kBatch];
 #pragma unroll
     for (int u = 0; u < kBatch; ++u) {
       if (row[u] >= 0) {
-        const int64_t j = target_of(a.meta, row[u]);
         load_slice<T, E>((const T*)a.Qp + (int64_t)row[u] * D + lane * E, q[u]);
         load_slice<T, E>((const T*)a.dS + (int64_t)row[u] * D + lane * E, g[u]);
-        st[u] = a.stats[j * a.S + h];
-        Dh[u] = a.Dj[j * a.S + h];
+        st[u] = a.rstat[(int64_t)row[u] * a.S + h];
       }
     }
 #pragma unroll
@@ -545,8 +561,8 @@ __device__ __forceinline__ void src_edges(const HgtArgs& a, int64_t beg, int64_t
       }
       s = head_sum(s, lph);
       da = head_sum(da, lph);
-      const float alpha = st[u].y > 0.f ? expf(s - st[u].x) / st[u].y : 0.f;
-      const float de = alpha * (da - Dh[u]);
+      const float alpha = expf(s - st[u].x) * st[u].y;
+      const float de = alpha * (da - st[u].z);
 #pragma unroll
       for (int e = 0; e < E; ++e) {
         ak[e] = fmaf(de, q[u][e], ak[e]);
@@ -658,7 +674,7 @@ struct HgtLayout {
   void* BDc;      // R x d x d
   void* WKt;      // T x d x d
   void* WVt;      // T x d x d
-  float* Dj;      // N x S
+  float4* rstat;  // csr_rows x S
   void* dQp;      // csr_rows x d
   void* dK;       // N x d
   void* dV;       // N x d
@@ -700,7 +716,7 @@ void carve_hgt(const hg_graph* g, const hg_hgt_params* p, void* saved, void* scr
   H->BDc = k.take<char>(m.num_rels * dd * b);
   H->WKt = k.take<char>(m.num_types * dd * b);
   H->WVt = k.take<char>(m.num_types * dd * b);
-  H->Dj = k.take<float>((size_t)std::max<int64_t>(N, 1) * S);
+  H->rstat = k.take<float4>((size_t)std::max<int64_t>(g->csr_rows, 1) * S);
   H->dQp = k.take<char>((size_t)std::max<int64_t>(g->csr_rows, 1) * d * b);
   H->dK = k.take<char>((size_t)std::max<int64_t>(N, 1) * d * b);
   H->dV = k.take<char>((size_t)std::max<int64_t>(N, 1) * d * b);
@@ -733,6 +749,12 @@ hg_layer_params projection_params(const hg_hgt_params* p, const HgtLayout& H) {
 HgtArgs edge_args(const hg_graph* g, const hg_hgt_params* p, const HgtLayout& H) {
   HgtArgs a{};
   a.meta = g->meta;
+  for (int t = 0; t < kMaxTypes; ++t) {
+    int k = 0;
+    for (int r = 0; r < kMaxRels; ++r) a.rslot[t][r] = -1;
+    for (int r = 0; r < g->meta.num_rels; ++r)
+      if (t < g->meta.num_types && g->meta.rel_dst[r] == t) a.rslot[t][k++] = (int8_t)r;
+  }
   a.N = g->meta.type_off[g->meta.num_types];
   a.csr_rows = g->csr_rows;
   a.S = p->heads;
@@ -749,12 +771,23 @@ HgtArgs edge_args(const hg_graph* g, const hg_hgt_params* p, const HgtLayout& H)
   a.Srows = H.L.M;
   a.dS = H.L.dMs;
   a.stats = H.stats;
-  a.Dj = H.Dj;
+  a.rstat = H.rstat;
   a.dQp = H.dQp;
   a.dK = H.dK;
   a.dV = H.dV;
   a.part = H.part;
   return a;
+}
+
+// Relations into the busiest type (the node kernels keep one slot per relation of a type).
+int max_rels_per_type(const GraphMeta& m) {
+  int best = 0;
+  for (int t = 0; t < m.num_types; ++t) {
+    int k = 0;
+    for (int r = 0; r < m.num_rels; ++r) k += m.rel_dst[r] == t;
+    best = std::max(best, k);
+  }
+  return best;
 }
 
 unsigned grid_of(int64_t threads) { return (unsigned)std::max<int64_t>(1, ceil_div(threads, 256)); }
@@ -830,7 +863,10 @@ hg_status hgt_fwd_t(const hg_graph* g, const hg_hgt_params* p, const void* H_in,
   // Eq. 6-10: softmax over the in-edges, weighted value sums per relation row
   const HgtArgs a = edge_args(g, p, H);
   HG_TRY(launch("hgt_fwd_chunks", hgt_fwd_chunks<T, D>, dim3(chunk_blocks(g->chunk_cap_csr)), dim3(256), 0, s, a));
-  HG_TRY(launch("hgt_fwd_nodes", hgt_fwd_nodes<T, D>, dim3(grid_of(N * 32)), dim3(256), 0, s, a));
+  if (max_rels_per_type(m) <= 4)
+    HG_TRY(launch("hgt_fwd_nodes", hgt_fwd_nodes<T, D, 4>, dim3(grid_of(N * 32)), dim3(256), 0, s, a));
+  else
+    HG_TRY(launch("hgt_fwd_nodes", hgt_fwd_nodes<T, D, kMaxRels>, dim3(grid_of(N * 32)), dim3(256), 0, s, a));
   // Eq. 11 on S_r with W_rel = blockdiag(W_msg[r])
   const hg_layer_params lp = projection_params(p, H);
   return project_forward(g, &lp, H_in, H_out, H.L, s);
@@ -860,7 +896,11 @@ hg_status hgt_bwd_t(const hg_graph* g, const hg_hgt_params* p, const void* H_in,
   HG_TRY(launch("hgt_bwd_dstats", hgt_bwd_dstats<T, D>, dim3(grid_of(N * 32)), dim3(256), 0, s, a));
   HG_TRY(launch("hgt_bwd_dst_chunks", hgt_bwd_dst_chunks<T, D>, dim3(chunk_blocks(g->chunk_cap_csr)), dim3(256), 0, s,
                 a));
-  HG_TRY(launch("hgt_bwd_dst_nodes", hgt_bwd_dst_nodes<T, D>, dim3(grid_of(N * 32)), dim3(256), 0, s, a));
+  if (max_rels_per_type(m) <= 4)
+    HG_TRY(launch("hgt_bwd_dst_nodes", hgt_bwd_dst_nodes<T, D, 4>, dim3(grid_of(N * 32)), dim3(256), 0, s, a));
+  else
+    HG_TRY(launch("hgt_bwd_dst_nodes", hgt_bwd_dst_nodes<T, D, kMaxRels>, dim3(grid_of(N * 32)), dim3(256), 0, s,
+                  a));
   HG_TRY(launch("hgt_bwd_src_chunks", hgt_bwd_src_chunks<T, D>, dim3(chunk_blocks(g->chunk_cap_node)), dim3(256), 0,
                 s, a));
   HG_TRY(launch("hgt_bwd_src_nodes", hgt_bwd_src_nodes<T, D>, dim3(grid_of(N * 32)), dim3(256), 0, s, a));
