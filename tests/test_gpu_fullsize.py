@@ -168,3 +168,76 @@ def test_full_size_head():
     ib = np.sort(rng.choice(N, sp.n_overlap, replace=False)).astype(np.int32)
     got = head_gpu(lib(), H, Hr, ia, ib, lab, y, p, "bf16", cca=3.0, lam=0.1)
     check(got, H, Hr, ia, ib, lab, y, p, "bf16", cca=3.0, lam=0.1)
+
+
+def test_full_size_temporal():
+    """The temporal module over the 1M nodes of the benchmark workload (w = 3, bf16 d = 128, the
+    tensor-core path): every output row the oracle computes on 3,000 sampled nodes (the module is
+    row by row), and the weight gradients exactly for an upstream gradient supported on those
+    nodes (the other rows then contribute nothing)."""
+    need_gpu()
+    from oracle import temporal as OT
+    hg = lib()
+    sp = hgsynth.spec("sub-1m")
+    n, d, w = sp.num_nodes, sp.d, hgsynth.TEMPORAL_WINDOW
+    rng = np.random.default_rng(31)
+    X = hgsynth.bf16_round(rng.standard_normal((n, d), dtype=np.float32))
+    C = hgsynth.make_context(sp)
+    p = hgsynth.make_temporal_params(sp)
+    rows = np.unique(np.concatenate([rng.choice(n, 3000, replace=False), [0, n - 1]]))
+    dOut = np.zeros((n, d), np.float32)
+    dOut[rows] = hgsynth.bf16_round(rng.standard_normal((len(rows), d), dtype=np.float32))
+    td = torch.bfloat16
+    keys = ("Wa", "r", "W_i", "W_h", "b_i", "b_h")
+    prm = hg.TemporalParams(*(dev(p[k], td) for k in keys), w=w)
+    sb, kb = hg.hg_temporal_workspace_size(n, d, w, td)
+    saved = torch.empty(sb, dtype=torch.uint8, device="cuda")
+    scratch = torch.empty(kb, dtype=torch.uint8, device="cuda")
+    Xd, Cd = dev(X, td), dev(C, td)
+    out = torch.empty(n, d, dtype=td, device="cuda")
+    hg.hg_temporal_fwd(prm, Xd, Cd, out, saved, scratch)
+    f = dict(dtype=torch.float32, device="cuda")
+    grads = {"Wa": torch.empty(d, d, **f), "r": torch.empty(d, **f), "W_i": torch.empty(d, 3 * d, **f),
+             "W_h": torch.empty(d, 3 * d, **f), "b_i": torch.empty(3 * d, **f), "b_h": torch.empty(3 * d, **f)}
+    dX = torch.empty_like(out)
+    hg.hg_temporal_bwd(prm, Xd, Cd, saved, dev(dOut, td), dX, grads, scratch)
+    torch.cuda.synchronize()
+    ref = OT.temporal_backward(X[rows], C[:, rows], p, dOut[rows], store="bf16")
+    tol = TOL["bf16"]
+    assert relerr(host(out)[rows], ref["out"]) <= tol
+    assert relerr(host(dX)[rows], ref["dX"]) <= tol
+    for k in keys:
+        assert relerr(host(grads[k]), ref["d" + k]) <= tol, k
+    assert hg.hg_device_status() == 0
+
+
+def test_full_size_attention_layer_sampled_targets():
+    """The attention layer (4 heads) on the benchmark graph (1M nodes, 20M edges, hubs of ~1M
+    in-edges): the output rows of sampled targets -- random rows, the largest in-degree hubs and
+    rows without in-edges -- against the oracle run on the subgraph of their in-edges (a row's
+    output depends only on its own features and those of its in-neighbours)."""
+    need_gpu()
+    from oracle import hgt as OH
+    hg = lib()
+    sp = hgsynth.spec("sub-1m")
+    w = hgsynth.make_workload(sp, with_ids=False)
+    g = w.graph
+    p = hgsynth.make_hgt_params(sp, 4, bias_margin=3.0)
+    td = torch.bfloat16
+    G = hg.hg_build_csr(dev(g["src"]), dev(g["dst"]), dev(g["rel"]), g["type_offsets"], g["rels"])
+    P = hg.HgtParams({k: dev(v, torch.float32 if k == "mu" else td) for k, v in p.items()}, 4)
+    sb, kb = hg.hg_hgt_workspace_size(G, P)
+    saved = torch.empty(sb, dtype=torch.uint8, device="cuda")
+    scratch = torch.empty(kb, dtype=torch.uint8, device="cuda")
+    X = dev(w.X, td)
+    out = torch.empty_like(X)
+    hg.hg_hgt_fwd(G, P, X, out, saved, scratch)
+    torch.cuda.synchronize()
+    rows = sample_rows(w, 400, 33)
+    keep = np.isin(g["dst"], rows)
+    nodes = np.unique(np.concatenate([rows, g["src"][keep]]))
+    # the subgraph keeps global ids (rows outside it have no in-edges and are not compared)
+    ref, _ = OH.hgt_forward(g["src"][keep], g["dst"][keep], g["rel"][keep], g["type_offsets"], g["rels"], p,
+                            np.where(np.isin(np.arange(sp.num_nodes), nodes)[:, None], w.X, 0.0), 4, store="bf16")
+    assert relerr(host(out)[rows], ref[rows]) <= TOL["bf16"]
+    assert hg.hg_device_status() == 0
