@@ -54,6 +54,7 @@ def parse():
     ap.add_argument("--oracle-temporal-sample", type=int, default=0, help=argparse.SUPPRESS)  # internal: child process
     ap.add_argument("--no-temporal", action="store_true", help="skip the temporal-module measurement")
     ap.add_argument("--no-hgt", action="store_true", help="skip the attention-layer measurement")
+    ap.add_argument("--scale", type=int, default=1, help=argparse.SUPPRESS)  # profiling: a 1/k-size instance
     ap.add_argument("--oracle-hgt-sample", type=int, default=0, help=argparse.SUPPRESS)  # internal: child process
     return ap.parse_args()
 
@@ -529,8 +530,21 @@ def measure_hgt(w, steps: int, warmup: int, dev, with_cpu: bool) -> dict:
     rep = hg.hg_timing_report()
     tot = sum(ms for _, ms in rep.values()) or 1.0
     ms = statistics.median(times)
+    # no-reuse model per layer: the forward and the two backward edge passes each gather a 4-byte
+    # index and two rows per edge (K and V; K and V; Q' and dS), plus the dense rows (K, V, Q', S
+    # written and read, the projection's and the backward products' rows)
+    b = 4 if sp.dtype == "f32" else 2
+    offs = [int(x) for x in g["type_offsets"]]
+    RR = sum(offs[t + 1] - offs[t] for _, t in g["rels"])
+    per_layer = 3 * len(g["src"]) * (4 + 2 * sp.d * b) + (2 * RR + 10 * sp.num_nodes) * sp.d * b
+    peaks, psrc = load_peaks()
+    ach = sp.layers * per_layer / (ms / 1e3) / 1e9
     res = {"ms": round(ms, 4), "layers": sp.layers, "heads": HGT_HEADS,
            "layers_fwd_bwd_edges_per_s": sp.layers * sp.num_edges / (ms / 1e3),
+           "roofline": {"bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                        "peak_source": f"{psrc} hbm_gbs", "frac": round(ach / peaks["hbm_gbs"], 4),
+                        "model": "no-reuse: 3 edge passes x (4 + 2 d b) per edge + (2 csr_rows + 10 N) d b per layer",
+                        "algorithmic_bytes_per_call": int(sp.layers * per_layer)},
            "kernel_time_share": {k: round(v / tot, 4) for k, (_, v) in sorted(rep.items(), key=lambda kv: -kv[1][1])},
            "cpu_baseline": None}
     if with_cpu:
@@ -560,6 +574,8 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     sp = hgsynth.spec(args.workload)
+    if args.scale > 1:  # a smaller instance of the same recipe, for profiler captures only
+        sp = scaled(sp, args.scale)
     if args.impl == "reference":
         if rank != 0:
             return

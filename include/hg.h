@@ -398,13 +398,15 @@ hg_status hg_head_loss(const hg_head_params* params, const void* H, int64_t rows
 
 /* Gradient of dloss * L_BCE (dloss = 1 in training; the alignment term's gradient comes from
  * hg_overlap_align_bwd with dloss = lambda_CCA).  grads are OVERWRITTEN.  The gradient at each
- * labelled row's final embedding is ACCUMULATED into dH[lab_idx[r]] (storage type), or, for a
- * row with a replica, half into dH[idx_a[k]] and half into dH_rep[idx_b[k]].  dH_rep may be NULL
- * (a detached second view); dH may be NULL.  `saved` must come from hg_head_loss with the same
- * params, lab_idx and n_lab. */
+ * labelled row's final embedding is added to dH[lab_idx[r]] (storage type), or, for a row with a
+ * replica, half to dH[idx_a[k]] and half to dH_rep[idx_b[k]].  dH (rows x d) and dH_rep
+ * (rows_rep x d) are ACCUMULATED into, or, when overwrite is nonzero, first set to zero (so they
+ * end up holding the head's gradient alone, e.g. the last layer's upstream gradient before the
+ * alignment term is added).  dH_rep may be NULL (a detached second view); dH may be NULL.  `saved`
+ * must come from hg_head_loss with the same params, lab_idx and n_lab. */
 hg_status hg_head_bwd(const hg_head_params* params, const int32_t* lab_idx, int64_t n_lab, float dloss,
-                      const void* saved, void* dH, void* dH_rep, const hg_head_grads* grads, void* scratch,
-                      hg_stream stream);
+                      const void* saved, void* dH, int64_t rows, void* dH_rep, int64_t rows_rep, int32_t overwrite,
+                      const hg_head_grads* grads, void* scratch, hg_stream stream);
 
 /* ------------------------------------------------------------------------------------------- */
 /* Temporal module (Section 3.2, Eq. 12-13): attention over each node's last w states and a GRU  */

@@ -500,8 +500,8 @@ extern "C" hg_status hg_head_loss(const hg_head_params* params, const void* H, i
 }
 
 extern "C" hg_status hg_head_bwd(const hg_head_params* params, const int32_t* lab_idx, int64_t n_lab, float dloss,
-                                const void* saved, void* dH, void* dH_rep, const hg_head_grads* grads, void* scratch,
-                                hg_stream stream) {
+                                const void* saved, void* dH, int64_t rows, void* dH_rep, int64_t rows_rep,
+                                int32_t overwrite, const hg_head_grads* grads, void* scratch, hg_stream stream) {
   clear_error();
   HG_TRY(check_head_params(params));
   HG_REQUIRE(saved && scratch && grads, "saved, scratch and grads must be non-null");
@@ -510,8 +510,15 @@ extern "C" hg_status hg_head_bwd(const hg_head_params* params, const int32_t* la
   HG_REQUIRE(n_lab >= 0 && n_lab < (int64_t(1) << 31), "n_lab must be in [0, 2^31)");
   HG_REQUIRE(n_lab == 0 || lab_idx, "lab_idx is needed when n_lab > 0");
   HG_REQUIRE(((uintptr_t)dH & 15) == 0 && ((uintptr_t)dH_rep & 15) == 0, "dH and dH_rep must be 16-byte aligned");
+  HG_REQUIRE(rows >= 0 && rows_rep >= 0, "rows and rows_rep must be >= 0");
   HeadLayout L;
   carve_head(const_cast<void*>(saved), scratch, 0, n_lab, params->d, params->dtype, &L, nullptr, nullptr);
+  if (overwrite) {
+    const size_t row_bytes = (size_t)params->d * (params->dtype == HG_BF16 ? 2 : 4);
+    cudaStream_t s0 = reinterpret_cast<cudaStream_t>(stream);
+    if (dH && rows > 0) HG_CUDA(cudaMemsetAsync(dH, 0, (size_t)rows * row_bytes, s0));
+    if (dH_rep && rows_rep > 0) HG_CUDA(cudaMemsetAsync(dH_rep, 0, (size_t)rows_rep * row_bytes, s0));
+  }
   return head_bwd_dispatch(params, lab_idx, n_lab, 0, dloss, L, dH, dH_rep, grads,
                            reinterpret_cast<cudaStream_t>(stream));
 }

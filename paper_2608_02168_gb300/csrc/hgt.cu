@@ -232,7 +232,8 @@ struct HgtArgs {
   float* part;       // chunk partials
 };
 
-constexpr int kBatch = 4;  // edges of a row in flight per warp
+constexpr int kBatch = 4;       // edges of a row in flight per warp (node kernels)
+constexpr int kBatchChunk = 4;  // the same for the chunk kernels (eight was slower: registers)
 
 // Online softmax step for one edge (per lane: its head's running maximum m and sum l; the value
 // accumulators are rescaled when the maximum grows).
@@ -259,26 +260,26 @@ __device__ __forceinline__ void online_step(float s, const float (&v)[E], float&
 }
 
 // The edges [beg, end) of one CSR row against the query slice q, folded into (m, l, acc[slot]).
-template <typename T, int D, int NACC>
+template <typename T, int D, int NACC, int NB = kBatch>
 __device__ __forceinline__ void fwd_edges(const HgtArgs& a, int64_t beg, int64_t end, const float (&q)[D / 32], int lph,
                                           float& m, float& l, float (&acc)[NACC][D / 32], int slot) {
   constexpr int E = D / 32;
   const int lane = threadIdx.x & 31;
   const T* KV = (const T*)a.KV;
-  for (int64_t e0 = beg; e0 < end; e0 += kBatch) {
-    int src[kBatch];
+  for (int64_t e0 = beg; e0 < end; e0 += NB) {
+    int src[NB];
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u) src[u] = e0 + u < end ? __ldg(a.csr_col + e0 + u) : -1;
-    float k[kBatch][E], v[kBatch][E];
+    for (int u = 0; u < NB; ++u) src[u] = e0 + u < end ? __ldg(a.csr_col + e0 + u) : -1;
+    float k[NB][E], v[NB][E];
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u) {
+    for (int u = 0; u < NB; ++u) {
       if (src[u] >= 0) {
         load_slice<T, E>(KV + (int64_t)src[u] * 2 * D + lane * E, k[u]);
         load_slice<T, E>(KV + (int64_t)src[u] * 2 * D + D + lane * E, v[u]);
       }
     }
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u) {
+    for (int u = 0; u < NB; ++u) {
       if (src[u] < 0) break;
       float s = 0.f;
 #pragma unroll
@@ -306,7 +307,7 @@ __global__ void __launch_bounds__(256) hgt_fwd_chunks(HgtArgs a) {
     float m = -INFINITY, l = 0.f, acc[1][E];
 #pragma unroll
     for (int e = 0; e < E; ++e) acc[0][e] = 0.f;
-    fwd_edges<T, D, 1>(a, beg, end, q, lph, m, l, acc, 0);
+    fwd_edges<T, D, 1, kBatchChunk>(a, beg, end, q, lph, m, l, acc, 0);
     float* p = a.part + c * stride;
     if (lane % lph == 0) {
       p[2 * (lane / lph)] = m;
@@ -423,27 +424,27 @@ __global__ void __launch_bounds__(256) hgt_bwd_dstats(HgtArgs a) {
 
 // sum over the edges [beg, end) of one row (relation r, target j) of de K(i), with
 // de = alpha (<dS_r(j), V(i)> - D_j) and alpha from the saved softmax statistics.
-template <typename T, int D>
+template <typename T, int D, int NB = kBatch>
 __device__ __forceinline__ void dst_edges(const HgtArgs& a, int64_t beg, int64_t end, const float (&q)[D / 32],
                                           const float (&g)[D / 32], float m, float inv_l, float Dh, int lph,
                                           float (&acc)[D / 32]) {
   constexpr int E = D / 32;
   const int lane = threadIdx.x & 31;
   const T* KV = (const T*)a.KV;
-  for (int64_t e0 = beg; e0 < end; e0 += kBatch) {
-    int src[kBatch];
+  for (int64_t e0 = beg; e0 < end; e0 += NB) {
+    int src[NB];
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u) src[u] = e0 + u < end ? __ldg(a.csr_col + e0 + u) : -1;
-    float k[kBatch][E], v[kBatch][E];
+    for (int u = 0; u < NB; ++u) src[u] = e0 + u < end ? __ldg(a.csr_col + e0 + u) : -1;
+    float k[NB][E], v[NB][E];
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u) {
+    for (int u = 0; u < NB; ++u) {
       if (src[u] >= 0) {
         load_slice<T, E>(KV + (int64_t)src[u] * 2 * D + lane * E, k[u]);
         load_slice<T, E>(KV + (int64_t)src[u] * 2 * D + D + lane * E, v[u]);
       }
     }
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u) {
+    for (int u = 0; u < NB; ++u) {
       if (src[u] < 0) break;
       float s = 0.f, da = 0.f;
 #pragma unroll
@@ -477,7 +478,7 @@ __global__ void __launch_bounds__(256) hgt_bwd_dst_chunks(HgtArgs a) {
     load_slice<T, E>((const T*)a.dS + (int64_t)row * D + lane * E, g);
 #pragma unroll
     for (int e = 0; e < E; ++e) acc[e] = 0.f;
-    dst_edges<T, D>(a, beg, end, q, g, st.x, st.y, st.z, lph, acc);
+    dst_edges<T, D, kBatchChunk>(a, beg, end, q, g, st.x, st.y, st.z, lph, acc);
 #pragma unroll
     for (int e = 0; e < E; ++e) a.part[c * D + lane * E + e] = acc[e];
   }
@@ -530,20 +531,20 @@ __global__ void __launch_bounds__(256, (D <= 128 && KS <= 4) ? 3 : 1) hgt_bwd_ds
 
 // Out-edges [beg, end) of source i (node-major list; each entry is the CSR row of the edge's
 // target): dK(i) += de Q'_r(j), dV(i) += alpha dS_r(j).
-template <typename T, int D>
+template <typename T, int D, int NB = kBatch>
 __device__ __forceinline__ void src_edges(const HgtArgs& a, int64_t beg, int64_t end, const float (&k)[D / 32],
                                           const float (&v)[D / 32], int lph, float (&ak)[D / 32],
                                           float (&av)[D / 32]) {
   constexpr int E = D / 32;
   const int lane = threadIdx.x & 31, h = lane / lph;
-  for (int64_t e0 = beg; e0 < end; e0 += kBatch) {
-    int row[kBatch];
+  for (int64_t e0 = beg; e0 < end; e0 += NB) {
+    int row[NB];
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u) row[u] = e0 + u < end ? __ldg(a.node_col + e0 + u) : -1;
-    float q[kBatch][E], g[kBatch][E];
-    float4 st[kBatch];
+    for (int u = 0; u < NB; ++u) row[u] = e0 + u < end ? __ldg(a.node_col + e0 + u) : -1;
+    float q[NB][E], g[NB][E];
+    float4 st[NB];
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u) {
+    for (int u = 0; u < NB; ++u) {
       if (row[u] >= 0) {
         load_slice<T, E>((const T*)a.Qp + (int64_t)row[u] * D + lane * E, q[u]);
         load_slice<T, E>((const T*)a.dS + (int64_t)row[u] * D + lane * E, g[u]);
@@ -551,7 +552,7 @@ __device__ __forceinline__ void src_edges(const HgtArgs& a, int64_t beg, int64_t
       }
     }
 #pragma unroll
-    for (int u = 0; u < kBatch; ++u) {
+    for (int u = 0; u < NB; ++u) {
       if (row[u] < 0) break;
       float s = 0.f, da = 0.f;
 #pragma unroll
@@ -588,7 +589,7 @@ __global__ void __launch_bounds__(256) hgt_bwd_src_chunks(HgtArgs a) {
     load_slice<T, E>(KV + (int64_t)i * 2 * D + D + lane * E, v);
 #pragma unroll
     for (int e = 0; e < E; ++e) ak[e] = av[e] = 0.f;
-    src_edges<T, D>(a, beg, end, k, v, lph, ak, av);
+    src_edges<T, D, kBatchChunk>(a, beg, end, k, v, lph, ak, av);
 #pragma unroll
     for (int e = 0; e < E; ++e) {
       a.part[c * 2 * D + lane * E + e] = ak[e];

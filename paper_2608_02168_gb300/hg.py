@@ -112,7 +112,8 @@ EXPORTS = {
     "hg_head_loss": (c_int32, [POINTER(hg_head_params), c_void_p, c_int64, c_void_p, c_int64, c_void_p, c_void_p,
                                c_int64, c_void_p, c_void_p, c_void_p, c_int64, c_void_p, c_float, c_void_p, c_void_p,
                                c_void_p, c_void_p, c_void_p]),
-    "hg_head_bwd": (c_int32, [POINTER(hg_head_params), c_void_p, c_int64, c_float, c_void_p, c_void_p, c_void_p,
+    "hg_head_bwd": (c_int32, [POINTER(hg_head_params), c_void_p, c_int64, c_float, c_void_p, c_void_p, c_int64,
+                              c_void_p, c_int64, c_int32,
                               POINTER(hg_head_grads), c_void_p, c_void_p]),
     "hg_temporal_workspace_size": (c_int32, [c_int64, c_int32, c_int32, c_int32, POINTER(c_size_t),
                                              POINTER(c_size_t)]),
@@ -452,11 +453,14 @@ def hg_head_loss(params: HeadParams, H, H_rep, idx_a, idx_b, n_rep_max: int, n_r
                               _ptr(saved), _ptr(scratch), _stream(stream)), "hg_head_loss")
 
 
-def hg_head_bwd(params: HeadParams, lab_idx, dloss: float, saved, dH, dH_rep, grads: dict, scratch, stream=None):
+def hg_head_bwd(params: HeadParams, lab_idx, dloss: float, saved, dH, dH_rep, grads: dict, scratch, stream=None,
+                overwrite: bool = False):
     p = params.c()
     gr = hg_head_grads(_ptr(grads["W1"]), _ptr(grads["b1"]), _ptr(grads["w2"]), _ptr(grads["b2"]))
     _check(lib().hg_head_bwd(byref(p), _ptr(lab_idx), lab_idx.numel(), float(dloss), _ptr(saved), _ptr(dH),
-                             _ptr(dH_rep), byref(gr), _ptr(scratch), _stream(stream)), "hg_head_bwd")
+                             dH.shape[0] if dH is not None else 0, _ptr(dH_rep),
+                             dH_rep.shape[0] if dH_rep is not None else 0, 1 if overwrite else 0, byref(gr),
+                             _ptr(scratch), _stream(stream)), "hg_head_bwd")
 
 
 # ------------------------------------------------------------------------------------------------

@@ -8,8 +8,8 @@ A step (Algorithm 1, the per-worker part of one iteration, on one GPU):
   hg_head_loss           (with a head and labels) MeanAgg of the replicas, the two-layer MLP and
                          the masked BCE over the labelled rows, and L_total = L_BCE + lambda_CCA
                          L_CCA (Eq. 18-20)
-  hg_head_bwd            its gradient, which is then the last layer's upstream gradient (without
-                         a head the caller supplies that gradient, dH_top)
+  hg_head_bwd            its gradient, written as the last layer's upstream gradient (without a
+                         head the caller supplies that gradient, dH_top)
   hg_overlap_align_bwd   the alignment gradient, scaled by lambda_CCA (Eq. 20), added to it
   hg_layer_bwd x L       gradients of every layer, including dL/dX of the first.
 This module only allocates buffers (torch) and marshals arguments; every computation runs in
@@ -125,7 +125,7 @@ class HotPath:
         [L_total, L_BCE] and self.head_grads).  With a head and labels (lab_idx, lab_y) the last
         layer's upstream gradient is the head's and dH_top is ignored.  `marks`, if a list, receives
         (phase, CUDA event) pairs recorded on the stream after the graph build, the forward layers,
-        the alignment, the head (when it runs) and the backward layers."""
+        the alignment loss, the head (when it runs), the alignment gradient and the backward layers."""
         def mark(name):
             if marks is not None:
                 ev = torch.cuda.Event(enable_timing=True)
@@ -144,9 +144,7 @@ class HotPath:
         mark("forward")
         top = self.H[0][self.L]
         use_head = self.head is not None and lab_idx is not None
-        if use_head:
-            self.dH[0][self.L].zero_()
-        else:
+        if not use_head:  # with a head, hg_head_bwd writes the whole upstream gradient
             self.dH[0][self.L].copy_(dH_top)
         if self.view == "bank" and H_bank is None:
             # first subgraph of a sequence: no neighbour view yet, no alignment term
@@ -168,16 +166,18 @@ class HotPath:
             n_max = int(overlap_idx.numel())
             ia = ib = overlap_idx
             Hb = self.H[1][self.L]
-            self.dH[1][self.L].zero_()
             dHb, n_dev = self.dH[1][self.L], None
+            if not use_head:
+                dHb.zero_()
         hg.hg_overlap_align_loss(top, ia, Hb, ib, n_max, n_dev, LAMBDA_N, VAR_EPS, self.loss, self.align_saved,
                                  self.align_scratch, stream)
-        hg.hg_overlap_align_bwd(top, ia, Hb, ib, n_max, n_dev, LAMBDA_N, VAR_EPS, LAMBDA_CCA, self.align_saved,
-                                self.dH[0][self.L], dHb, self.align_scratch, stream)
         mark("alignment")
-        if use_head:
+        if use_head:  # L_total needs L_CCA; the head's gradient overwrites the upstream gradient buffers
             self._head(top, Hb, ia, ib, n_max, n_dev, dHb, lab_idx, lab_y, stream)
             mark("head")
+        hg.hg_overlap_align_bwd(top, ia, Hb, ib, n_max, n_dev, LAMBDA_N, VAR_EPS, LAMBDA_CCA, self.align_saved,
+                                self.dH[0][self.L], dHb, self.align_scratch, stream)
+        mark("alignment_bwd")
         for s in range(len(stacks)):
             for l in range(self.L - 1, -1, -1):
                 hg.hg_layer_bwd(g, self.params[l], self.H[s][l], self.saved[s][l], self.dH[s][l + 1], self.dH[s][l],
@@ -190,7 +190,7 @@ class HotPath:
         hg.hg_head_loss(self.head, top, H_rep, ia, ib, n_max, n_dev, lab_idx, lab_y, self.loss, LAMBDA_CCA,
                         self.head_loss, None, self.head_saved, self.head_scratch, stream)
         hg.hg_head_bwd(self.head, lab_idx, 1.0, self.head_saved, self.dH[0][self.L], dH_rep, self.head_grads,
-                       self.head_scratch, stream)
+                       self.head_scratch, stream, overwrite=True)
 
 
 class Ring:

@@ -170,3 +170,28 @@ def test_head_deterministic():
     b = head_gpu(hg, H, Hr, ia, ib, lab, y, p, "bf16")
     for k in ("loss", "logits", "dW1", "db1", "dw2", "db2", "dH", "dH_rep"):
         assert np.array_equal(a[k], b[k]), k
+
+
+def test_head_overwrite_mode():
+    """overwrite=True: dH and dH_rep are cleared first, so they hold the head's gradient alone."""
+    need_gpu()
+    hg = lib()
+    H, Hr, ia, ib, lab, y, p = problem(23, 2000, 64, 600, 300, "f32")
+    td = torch.float32
+    prm = hg.HeadParams(dev(p["W1"], td), dev(p["b1"], td), dev(p["w2"], td), dev(p["b2"], td))
+    s, k = hg.hg_head_workspace_size(H.shape[0], len(lab), 64, td)
+    saved = torch.empty(s, dtype=torch.uint8, device="cuda")
+    scratch = torch.empty(k, dtype=torch.uint8, device="cuda")
+    A, B = dev(H, td), dev(Hr, td)
+    loss = torch.empty(2, dtype=torch.float32, device="cuda")
+    hg.hg_head_loss(prm, A, B, dev(ia), dev(ib), len(ia), None, dev(lab), dev(y), None, 0.1, loss, None, saved, scratch)
+    f = dict(dtype=torch.float32, device="cuda")
+    grads = {"W1": torch.empty(64, 64, **f), "b1": torch.empty(64, **f), "w2": torch.empty(64, **f),
+             "b2": torch.empty(1, **f)}
+    dH = torch.randn_like(A)  # stale contents that must not survive
+    dR = torch.randn_like(B)
+    hg.hg_head_bwd(prm, dev(lab), 1.0, saved, dH, dR, grads, scratch, overwrite=True)
+    torch.cuda.synchronize()
+    g = OH.head_backward(H, ia, Hr, ib, lab, y, p)
+    assert relerr(host(dH), g["dH"]) <= 1e-5 and relerr(host(dR), g["dH_rep"]) <= 1e-5
+    assert np.all(host(dH)[g["dH"] == 0] == 0)
