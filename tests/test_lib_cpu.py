@@ -88,3 +88,54 @@ def test_product_path_has_no_fallback():
             src = open(os.path.join(pkg, f)).read()
             assert "oracle" not in src.replace("oracle.", ""), f
             assert "import numpy" not in src, f
+
+
+def test_host_argument_checks_of_the_widened_rows(hg):
+    """Head, temporal module, attention layer and subgraph construction reject bad arguments on
+    the host (fake aligned addresses stand in for device buffers: nothing is dereferenced)."""
+    so = hg.lib()
+    A = 1 << 20  # a 256-byte-aligned stand-in address
+    # head: unsupported width, misaligned weights, null loss output, negative sizes
+    p = hg.hg_head_params(96, 1, A, A, A, A)
+    assert so.hg_head_loss(ctypes.byref(p), A, 10, None, 0, None, None, 0, None, A, A, 4, None, 0.1, A, None, A, A,
+                           None) == 2
+    p = hg.hg_head_params(64, 1, A + 2, A, A, A)
+    assert so.hg_head_loss(ctypes.byref(p), A, 10, None, 0, None, None, 0, None, A, A, 4, None, 0.1, A, None, A, A,
+                           None) == 1
+    p = hg.hg_head_params(64, 1, A, A, A, A)
+    assert so.hg_head_loss(ctypes.byref(p), A, 10, None, 0, None, None, 0, None, A, A, 4, None, 0.1, None, None, A, A,
+                           None) == 1
+    assert so.hg_head_loss(ctypes.byref(p), A, 10, None, 0, None, None, 0, None, A, A, -1, None, 0.1, A, None, A, A,
+                           None) == 1
+    gr = hg.hg_head_grads(A, A, None, A)
+    assert so.hg_head_bwd(ctypes.byref(p), A, 4, 1.0, A, A, 10, None, 0, 0, ctypes.byref(gr), A, None) == 1
+    # temporal: window out of range, unsupported width, null pointers with rows
+    t = hg.hg_temporal_params(64, 9, 1, A, A, A, A, A, A)
+    assert so.hg_temporal_fwd(ctypes.byref(t), A, A, 10, A, A, A, None) == 1
+    t = hg.hg_temporal_params(80, 3, 1, A, A, A, A, A, A)
+    assert so.hg_temporal_fwd(ctypes.byref(t), A, A, 10, A, A, A, None) == 2
+    t = hg.hg_temporal_params(64, 3, 1, A, A, A, A, A, A)
+    assert so.hg_temporal_fwd(ctypes.byref(t), None, A, 10, A, A, A, None) == 1
+    assert so.hg_temporal_workspace_size(10, 64, 0, 1, ctypes.byref(ctypes.c_size_t()),
+                                         ctypes.byref(ctypes.c_size_t())) == 1
+    # attention layer: heads not a power of two, null graph
+    h = hg.hg_hgt_params(128, 3, 1, 0, 1, 1e-5, *([A] * 13))
+    assert so.hg_hgt_workspace_size(A, ctypes.byref(h), ctypes.byref(ctypes.c_size_t()),
+                                    ctypes.byref(ctypes.c_size_t())) == 1
+    h = hg.hg_hgt_params(128, 4, 1, 0, 1, 1e-5, *([A] * 13))
+    assert so.hg_hgt_fwd(None, ctypes.byref(h), A, A, A, A, None) == 1
+    # construction: partition index out of range
+    offs = (ctypes.c_int64 * 3)(0, 8, 10)
+    assert so.hg_overlap_build(A, A, A, 5, 10, offs, 2, 4, 4, 2, 3, 1, 2, A, A, A, A, A, A, None, A, A, 1 << 30,
+                               None) == 1
+
+
+def test_widened_workspace_queries_are_host_only(hg):
+    import torch
+    s, k = hg.hg_head_workspace_size(1000, 100, 128, torch.bfloat16)
+    assert s >= 2 * 100 * 128 * 2 and k >= 1000 * 4
+    s, k = hg.hg_temporal_workspace_size(1000, 128, 3, torch.bfloat16)
+    assert s >= 1000 * 128 * 2 + 1000 * 3 * 4 and k >= 4 * 1000 * 128 * 2
+    s2, k2 = hg.hg_temporal_workspace_size(1000, 256, 3, torch.bfloat16)  # CUDA-core path: fp32 scratch
+    assert k2 > k
+    assert hg.hg_overlap_build_workspace_size(1000, 5000) > 5000 * 4
