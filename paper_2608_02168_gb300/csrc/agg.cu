@@ -11,9 +11,10 @@
 // Mapping: one group of G lanes per row, each lane owning 16-byte slices of the feature row
 // (G = d * sizeof(T) / 16, at most 32), gathers with 128-bit loads and eight neighbour rows in
 // flight, fp32 accumulation; the row kernels are persistent (one wave of blocks striding over
-// rows).  Rows above kHubDegree edges are split into kChunkEdges-edge chunks: a whole CTA reduces
-// one chunk (its groups interleave over the chunk's edges, then combine in group order) into an
-// fp32 partial, runs of 64 partials are summed in order, and the row adds the run sums in order.
+// rows), and the backward one loads the next node's first indices while the current one gathers.
+// Rows above kHubDegree edges are split into kChunkEdges-edge chunks: a whole CTA reduces one
+// chunk (its groups interleave over the chunk's edges, then combine in group order) into an fp32
+// partial, runs of 64 partials are summed in order, and the row adds the run sums in order.
 // Every sum has a fixed order, so results are bitwise reproducible run to run.
 #include <algorithm>
 
@@ -219,6 +220,46 @@ __global__ void __launch_bounds__(256) agg_chunks(const int32_t* __restrict__ pt
   }
 }
 
+// The backward node kernel runs a two-deep pipeline per group: while node i gathers, the first
+// kFirst indices of node i + step and the bounds of node i + 2 step are in flight, so a short
+// row's gathers are issued without waiting on an index load.  Indices past the row's end, and
+// those of a row that takes the chunk path, are -1.  (The forward row kernel keeps a plain scalar
+// loop over short rows: with the extra registers of the pipeline it ran slower.)
+constexpr int kFirst = 8;
+
+__device__ __forceinline__ void load_first(const int32_t* __restrict__ col, int beg, int end, int* c) {
+  const bool small = end - beg <= kHubDegree;
+#pragma unroll
+  for (int u = 0; u < kFirst; ++u) c[u] = small && beg + u < end ? __ldg(col + beg + u) : -1;
+}
+
+// acc += the rows of the preloaded first indices c (in order), then the row's edges from
+// beg + kFirst on, so every row is still summed in edge order.
+template <typename T, int D, bool kBatchTail>
+__device__ __forceinline__ void gather_row(const int32_t* __restrict__ col, int beg, int end, const int* c,
+                                           const T* __restrict__ src, int lane, float* acc) {
+  using S = AggShape<T, D>;
+  const T* base = src + lane * S::kVec;
+  uint4 x[kFirst][S::V];
+#pragma unroll
+  for (int u = 0; u < kFirst; ++u)
+#pragma unroll
+    for (int v = 0; v < S::V; ++v)
+      x[u][v] = c[u] >= 0 ? ldg16(base + (int64_t)c[u] * D + v * S::G * S::kVec) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+  for (int u = 0; u < kFirst; ++u) {
+    if (c[u] < 0) break;
+#pragma unroll
+    for (int v = 0; v < S::V; ++v) {
+      float f[S::kVec];
+      unpack(x[u][v], f, T());
+#pragma unroll
+      for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] += f[q];
+    }
+  }
+  if (end - beg > kFirst) gather_sum<T, D, kBatchTail>(col, beg + kFirst, end, 1, 0, src, lane, acc);
+}
+
 // Forward rows: M[row] = mean over the row's neighbours (concatenated CSR rows of all relations).
 // Persistent: each group strides over rows and fetches the next row's bounds while it gathers.
 template <typename T, int D>
@@ -260,9 +301,9 @@ __global__ void __launch_bounds__(256) agg_fwd_rows(const int32_t* __restrict__ 
 
 // Backward nodes: dH[i] = dY[i] + sum of the node's row in the node-major out-edge list (every
 // relation leaving its type, relation by relation, each edge holding the dMs row it reads).
-// Persistent: each group strides over nodes and fetches the next node's bounds while it gathers.
+// Persistent: each group strides over nodes (pipelined as above).
 template <typename T, int D>
-__global__ void __launch_bounds__(256) agg_bwd_nodes(int64_t N, const int32_t* __restrict__ nptr,
+__global__ void __launch_bounds__(256, 4) agg_bwd_nodes(int64_t N, const int32_t* __restrict__ nptr,
                                                      const int32_t* __restrict__ ncol, const T* __restrict__ dMs,
                                                      const T* __restrict__ dY, T* __restrict__ dH,
                                                      const int32_t* __restrict__ chunk_ofs,
@@ -271,17 +312,25 @@ __global__ void __launch_bounds__(256) agg_bwd_nodes(int64_t N, const int32_t* _
   const int grp = threadIdx.x / S::G, lane = threadIdx.x % S::G;
   const int64_t step = (int64_t)gridDim.x * S::kGroups;
   int64_t node = (int64_t)blockIdx.x * S::kGroups + grp;
-  int beg = 0, end = 0;
+  int beg = 0, end = 0, nbeg = 0, nend = 0;
   if (node < N) {
     beg = __ldg(nptr + node);
     end = __ldg(nptr + node + 1);
   }
+  if (node + step < N) {
+    nbeg = __ldg(nptr + node + step);
+    nend = __ldg(nptr + node + step + 1);
+  }
+  int c[kFirst];
+  load_first(ncol, beg, end, c);
   while (node < N) {
-    const int64_t next = node + step;
-    int nbeg = 0, nend = 0;
-    if (next < N) {
-      nbeg = __ldg(nptr + next);
-      nend = __ldg(nptr + next + 1);
+    int cn[kFirst];
+    load_first(ncol, nbeg, nend, cn);
+    const int64_t node2 = node + 2 * step;
+    int b2 = 0, e2 = 0;
+    if (node2 < N) {
+      b2 = __ldg(nptr + node2);
+      e2 = __ldg(nptr + node2 + 1);
     }
     float acc[S::F];
 #pragma unroll
@@ -294,11 +343,15 @@ __global__ void __launch_bounds__(256) agg_bwd_nodes(int64_t N, const int32_t* _
     if (end - beg > kHubDegree)
       add_partials<T, D>(partials, chunk_ofs[node], chunk_ofs[node + 1], lane, acc);
     else
-      gather_sum<T, D>(ncol, beg, end, 1, 0, dMs, lane, acc);
+      gather_row<T, D, true>(ncol, beg, end, c, dMs, lane, acc);
     store_row<T, D>(dH + node * D, lane, acc, 1.0f);
-    node = next;
+    node += step;
     beg = nbeg;
     end = nend;
+    nbeg = b2;
+    nend = e2;
+#pragma unroll
+    for (int u = 0; u < kFirst; ++u) c[u] = cn[u];
   }
 }
 
