@@ -27,6 +27,10 @@
  *     [type_offsets[t], type_offsets[t+1]).  Features are row-major N x d.
  *   - Supported feature widths: d in {64, 128, 256}; dtypes HG_F32 and HG_BF16 (storage type of
  *     features, weights and activations; arithmetic accumulates in fp32).  Edge counts < 2^31.
+ *   - One process drives one GPU through this library (one process per GPU, as in data-parallel
+ *     training): kernel attributes (large shared-memory carve-outs) and the address of the device
+ *     status word are set up once, for the device current at the first call that needs them.
+ *     Only hg_overlap_align_loss_static keeps its set-up per device.
  */
 #ifndef HG_H_
 #define HG_H_
