@@ -34,6 +34,7 @@ ORACLE_SCALE = 40        # the CPU baseline runs the oracle on a 1/40-size insta
 BUILD_K, BUILD_THETA, BUILD_BUDGET = 8, 2, 0.15  # overlapping-subgraph construction: parts, h-index bound, M / N
 REFERENCE_SCALE = 100    # each reference-arm step runs the oracle on a 1/100-size instance
 FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "sm_max_mhz": 2070.0}
+NOMINAL_HBM_GBS = 7900.0  # GB300 HBM3e data-sheet bandwidth, reported beside the measured copy peak
 
 
 def parse():
@@ -224,16 +225,29 @@ def graph_stats(w) -> dict:
         st["RR"] += n_t
         st["CC"] += n_s
         st["rels"].append(dict(n_t=n_t, n_s=n_s, E=int(m.sum())))
-        for key, rows, other, nrow in (("fwd", d_r, s_r, N), ("bwd", s_r, d_r, N)):
-            deg = np.bincount(rows, minlength=N)
-            hub_edge = deg[rows] > HUB
-            a = st[key]
-            a["E_h"] += int(hub_edge.sum())
-            a["E_nh"] += int((~hub_edge).sum())
-            a["U_h"] += int(np.count_nonzero(np.bincount(other[hub_edge], minlength=nrow)))
-            a["U_nh"] += int(np.count_nonzero(np.bincount(other[~hub_edge], minlength=nrow)))
-            hd = deg[deg > HUB]
-            a["chunks"] += int(((hd + CHUNK - 1) // CHUNK).sum())
+        # forward: one CSR row per (relation, destination), reading source rows of H
+        deg = np.bincount(d_r, minlength=N)
+        hub_edge = deg[d_r] > HUB
+        a = st["fwd"]
+        a["E_h"] += int(hub_edge.sum())
+        a["E_nh"] += int((~hub_edge).sum())
+        a["U_h"] += int(np.count_nonzero(np.bincount(s_r[hub_edge], minlength=N)))
+        a["U_nh"] += int(np.count_nonzero(np.bincount(s_r[~hub_edge], minlength=N)))
+        hd = deg[deg > HUB]
+        a["chunks"] += int(((hd + CHUNK - 1) // CHUNK).sum())
+    # backward: one node-major row per node (its out-edges of every relation), each edge reading the
+    # dMs row of its (relation, destination); the hub split follows the node's total out-degree
+    deg = np.bincount(src, minlength=N)
+    hub_edge = deg[src] > HUB
+    read = rel.astype(np.int64) * N + dst
+    nread = len(g["rels"]) * N
+    a = st["bwd"]
+    a["E_h"] = int(hub_edge.sum())
+    a["E_nh"] = int((~hub_edge).sum())
+    a["U_h"] = int(np.count_nonzero(np.bincount(read[hub_edge], minlength=nread)))
+    a["U_nh"] = int(np.count_nonzero(np.bincount(read[~hub_edge], minlength=nread)))
+    hd = deg[deg > HUB]
+    a["chunks"] = int(((hd + CHUNK - 1) // CHUNK).sum())
     return st
 
 
@@ -281,7 +295,10 @@ def kernel_models(st: dict, sp) -> dict:
     m["ln_act_bwd"] = (L * lb, 0)
     m["proj_bwd_tc"] = (L * pb, L * pfl)
     m["wgrad_tc"] = (L * row * (RR + N), L * 2 * d * d * RR)  # G_r = M_r^T dU: M_r rows once, dU once per type
-    m["radix_scatter"] = (2 * 3 * 2 * 12 * st["E"], 0)  # 2 layouts x 3 passes x read+write of key, edge id, endpoint
+    # per 8-bit pass over the keys (the row ids, invalid edges keyed one past the last row): read and
+    # write of key, edge id and endpoint; one sort per layout
+    passes = lambda rows: max(1, -(-int(rows).bit_length() // 8))  # noqa: E731
+    m["radix_scatter"] = (2 * 12 * st["E"] * (passes(RR) + passes(CC)), 0)
     nl = st.get("n_lab", 0)
     if nl:
         # per labelled row: its H row (and a replica row for overlap rows, not counted), the saved Hm
@@ -342,6 +359,8 @@ def roofline(report: dict, models: dict, steps: int, peaks: dict, src: str, dom=
         rf = dict(bound="hbm", achieved=round(ach, 1), peak=peaks["hbm_gbs"], unit="GB/s",
                   peak_source=f"{src} hbm_gbs")
     rf["frac"] = round(rf["achieved"] / rf["peak"], 4) if rf["peak"] else None
+    if rf["bound"] == "hbm":
+        rf["frac_of_nominal"] = round(rf["achieved"] / NOMINAL_HBM_GBS, 4)
     rf["traffic"] = measured_traffic(dom)
     rf.update(kernel=dom, launches=n, avg_launch_ms=round(ms / max(n, 1), 4),
               algorithmic_bytes_per_launch=int(by * steps / max(n, 1)), flops_per_launch=int(fl * steps / max(n, 1)))
@@ -397,6 +416,7 @@ def measure_overlap_build(w, steps: int, warmup: int, dev, with_cpu: bool) -> di
     res = {"ms": round(ms, 4), "edges_per_s": len(g["src"]) / (ms / 1e3), "counts": out["counts"],
            "roofline": {"bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
                         "peak_source": f"{psrc} hbm_gbs", "frac": round(ach / peaks["hbm_gbs"], 4),
+                        "frac_of_nominal": round(ach / NOMINAL_HBM_GBS, 4),
                         "algorithmic_bytes_per_call": int(byt), "scope": "whole call"},
            "config": {"K": BUILD_K, "k": 0, "theta": BUILD_THETA, "M": M},
            "kernel_time_share": {k: round(v / tot, 4) for k, (_, v) in sorted(rep.items(), key=lambda kv: -kv[1][1])},
@@ -466,6 +486,7 @@ def measure_temporal(sp, steps: int, warmup: int, dev, with_cpu: bool) -> dict:
     res = {"ms": round(ms, 4), "nodes_per_s": n / (ms / 1e3), "nodes": n, "w": w, "d": d, "dtype": sp.dtype,
            "roofline": {"bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
                         "peak_source": f"{psrc} hbm_gbs", "frac": round(ach / peaks["hbm_gbs"], 4),
+                        "frac_of_nominal": round(ach / NOMINAL_HBM_GBS, 4),
                         "algorithmic_bytes_per_call": int(per_node * n), "scope": "forward + backward"},
            "tensor": {"achieved_tflops": round(flops / (ms / 1e3) / 1e12, 1), "peak": peaks.get("bf16_tflops"),
                       "flops_per_call": int(flops)},
@@ -543,6 +564,7 @@ def measure_hgt(w, steps: int, warmup: int, dev, with_cpu: bool) -> dict:
            "layers_fwd_bwd_edges_per_s": sp.layers * sp.num_edges / (ms / 1e3),
            "roofline": {"bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
                         "peak_source": f"{psrc} hbm_gbs", "frac": round(ach / peaks["hbm_gbs"], 4),
+                        "frac_of_nominal": round(ach / NOMINAL_HBM_GBS, 4),
                         "model": "no-reuse: 3 edge passes x (4 + 2 d b) per edge + (2 csr_rows + 10 N) d b per layer",
                         "algorithmic_bytes_per_call": int(sp.layers * per_layer)},
            "kernel_time_share": {k: round(v / tot, 4) for k, (_, v) in sorted(rep.items(), key=lambda kv: -kv[1][1])},
