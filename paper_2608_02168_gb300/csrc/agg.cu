@@ -230,7 +230,7 @@ constexpr int kFirst = 8;
 __device__ __forceinline__ void load_first(const int32_t* __restrict__ col, int beg, int end, int* c) {
   const bool small = end - beg <= kHubDegree;
 #pragma unroll
-  for (int u = 0; u < kFirst; ++u) c[u] = small && beg + u < end ? __ldg(col + beg + u) : -1;
+  for (int u = 0; u < kFirst; ++u) c[u] = small && u < end - beg ? __ldg(col + beg + u) : -1;
 }
 
 // acc += the rows of the preloaded first indices c (in order), then the row's edges from
