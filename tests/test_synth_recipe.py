@@ -109,3 +109,28 @@ def test_features_and_weights_recipe():
     assert p["W_rel"].shape == (sp.num_rels, sp.d, sp.d) and p["W_agg"].shape == (2, sp.d, sp.d)
     assert np.abs(p["W_rel"]).max() <= a * (1 + 2 ** -8) and np.abs(p["W_agg"]).max() <= a * (1 + 2 ** -8)
     assert not p["b_agg"].any() and np.all(p["ln_gamma"] == 1) and not p["ln_beta"].any()
+
+
+def test_ring_of_subgraphs_shares_exactly_the_overlap_with_the_next():
+    # 16 subgraphs of 2M nodes; each shares 400k nodes (20 %) with the next and none with the one after
+    sp = WORKLOADS["ring16-2m"]
+    ids = [hgsynth.graphs.ring_ids(sp, k) for k in range(3)]
+    for a in ids:
+        assert a.shape[0] == sp.num_nodes and np.all(np.diff(a) > 0)
+    assert np.intersect1d(ids[0], ids[1], assume_unique=True).shape[0] == sp.n_overlap
+    assert np.intersect1d(ids[1], ids[2], assume_unique=True).shape[0] == sp.n_overlap
+    assert np.intersect1d(ids[0], ids[2], assume_unique=True).shape[0] == 0
+    # users below risk events, so local order is global-id order within each type
+    last = hgsynth.graphs.ring_ids(sp, sp.num_subgraphs - 1)
+    assert last[sp.n_user - 1] < ids[0][sp.n_user]
+
+
+def test_ring_parts_carry_identical_rows_for_shared_nodes():
+    sp = hgsynth.spec("ring16-2m", n_user=9_000, n_risk=1_000, num_edges=50_000, n_overlap=2_000, d=64)
+    p0, p1 = hgsynth.graphs.make_ring_part(sp, 0), hgsynth.graphs.make_ring_part(sp, 1)
+    shared, i0, i1 = np.intersect1d(p0.gid, p1.gid, return_indices=True)
+    assert shared.shape[0] == sp.n_overlap
+    assert np.array_equal(p0.X[i0], p1.X[i1])
+    # independent edges per subgraph, and different rows for different nodes
+    assert not np.array_equal(p0.graph["src"], p1.graph["src"])
+    assert not np.array_equal(p0.X[: sp.n_overlap], p1.X[: sp.n_overlap])
