@@ -161,8 +161,16 @@ def _check(status: int, where: str):
 
 
 def _ptr(t) -> int | None:
+    """Device address of a tensor argument (None passes NULL).  The library reads rows by address from
+    device memory, so anything but a contiguous CUDA tensor is rejected here instead of being read
+    wrongly (or faulting the GPU)."""
     if t is None:
         return None
+    if not t.is_cuda:
+        raise ValueError(f"libhg takes device memory; got a tensor on {t.device}")
+    if not t.is_contiguous():
+        raise ValueError(f"libhg reads rows by address; the tensor of shape {tuple(t.shape)} and strides "
+                         f"{t.stride()} must be contiguous (call .contiguous())")
     return t.data_ptr()
 
 

@@ -139,3 +139,14 @@ def test_widened_workspace_queries_are_host_only(hg):
     s2, k2 = hg.hg_temporal_workspace_size(1000, 256, 3, torch.bfloat16)  # CUDA-core path: fp32 scratch
     assert k2 > k
     assert hg.hg_overlap_build_workspace_size(1000, 5000) > 5000 * 4
+
+
+def test_binding_rejects_host_tensors_before_any_call(hg):
+    """The binding passes device addresses only: a host tensor is refused on the host, before the
+    library sees it (a host address handed to a kernel would fault or read the wrong memory)."""
+    import torch
+    a = torch.arange(8, dtype=torch.int64)
+    out = torch.empty(8, dtype=torch.int32)
+    with pytest.raises(ValueError, match="device memory"):
+        hg.hg_overlap_intersect(a, a, out, out, torch.empty(1, dtype=torch.int64), torch.empty(64, dtype=torch.uint8))
+    assert hg._ptr(None) is None
