@@ -1,8 +1,8 @@
 """CPU oracle of the attention variant of the layer (Heterogeneous Graph Transformer).  TEST
 INFRASTRUCTURE ONLY.
 
-Only tests/, __graft_entry__.smoke() and bench.py's CPU-baseline leg import this module; the product path never calls it
-and shares no code with it.  Plain numpy in fp64, written edge by edge.
+Only tests/, __graft_entry__.smoke() and bench.py's CPU-baseline leg import this module; the
+product path never calls it and shares no code with it.  Plain numpy in fp64, written edge by edge.
 
 What is computed (Section 3.2, Eq. 6-11), for one layer over the typed graph, with S heads of
 width d_h = d / S:

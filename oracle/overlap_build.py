@@ -1,7 +1,7 @@
 """CPU oracle of the overlapping-subgraph construction.  TEST INFRASTRUCTURE ONLY.
 
-Only tests/, __graft_entry__.smoke() and bench.py's CPU-baseline leg import this module; the product path never calls it
-and shares no code with it.  Plain numpy (integer work, no floating point).
+Only tests/, __graft_entry__.smoke() and bench.py's CPU-baseline leg import this module; the
+product path never calls it and shares no code with it.  Plain numpy (integer work, no floating point).
 
 What is computed (Section 3.1, Eq. 4-5 and the construction part of Algorithm 1):
 
