@@ -30,7 +30,8 @@
  *   - One process drives one GPU through this library (one process per GPU, as in data-parallel
  *     training): kernel attributes (large shared-memory carve-outs) and the address of the device
  *     status word are set up once, for the device current at the first call that needs them.
- *     Only hg_overlap_align_loss_static keeps its set-up per device.
+ *     (hg_overlap_align_loss_static looks up its scratch address per device, but the kernels it
+ *     launches share the one-time set-up above.)
  */
 #ifndef HG_H_
 #define HG_H_
