@@ -366,6 +366,8 @@ def roofline(report: dict, models: dict, steps: int, peaks: dict, src: str, dom=
               algorithmic_bytes_per_launch=int(by * steps / max(n, 1)), flops_per_launch=int(fl * steps / max(n, 1)))
     comp = models.get("compulsory", {}).get(dom)
     if comp is not None:
+        rf["model"] = ("per gathered edge: its index and one feature row, with no cache reuse (rows served by L1/L2 "
+                       "count as traffic, so frac can exceed 1); compulsory_*: each distinct row once")
         rf["compulsory_bytes_per_launch"] = int(comp * steps / max(n, 1))
         rf["compulsory_frac"] = round(comp * steps / secs / 1e9 / peaks["hbm_gbs"], 4) if secs > 0 else None
     return rf, shares

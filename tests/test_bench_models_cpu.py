@@ -92,6 +92,7 @@ def test_roofline_arithmetic():
     assert abs(rf["frac_of_nominal"] - achieved / bench.NOMINAL_HBM_GBS) < 1e-4
     assert rf["algorithmic_bytes_per_launch"] == int(1.2e9 * 5 / 10)
     assert abs(rf["compulsory_frac"] - 0.6e9 * 5 / 2e-3 / 1e9 / 6000.0) < 1e-4
+    assert "no cache reuse" in rf["model"]
     assert abs(sum(shares.values()) - 1.0) < 1e-3 and shares["k_hbm"] > shares["k_simt"]
     rs, _ = bench.roofline(report, models, 5, peaks, "test", dom="k_simt")
     assert rs["bound"] == "alu" and rs["unit"] == "TFLOP/s"
