@@ -375,9 +375,10 @@ def make_labels(sp: GraphSpec, sub: int = 0, fraction: float = LABELLED_FRACTION
     return rows, y
 
 
-def make_head_params(sp: GraphSpec, random_bias: bool = False) -> dict:
+def make_head_params(sp: GraphSpec, random_bias: bool = False, bias_margin: float | None = None) -> dict:
     """Two-layer head: W1 (d x d, input x hidden), b1 (d), w2 (d), b2 (1).  Xavier uniform weights,
-    zero biases, or small N(0, 0.1) biases for tests (seed+200)."""
+    zero biases, or small N(0, 0.1) biases for tests (seed+200).  bias_margin: b1 of +-margin per
+    hidden unit (seeded signs), keeping the hidden pre-activations away from the ReLU's kink."""
     rng = _rng(sp.seed + 200)
     d = sp.d
     a1 = math.sqrt(6.0 / (2 * d))
@@ -390,6 +391,8 @@ def make_head_params(sp: GraphSpec, random_bias: bool = False) -> dict:
     else:
         b1 = np.zeros(d, np.float32)
         b2 = np.zeros(1, np.float32)
+    if bias_margin is not None:
+        b1 = (bias_margin * rng.choice([-1.0, 1.0], size=d)).astype(np.float32)
     return {k: _store(v, sp.dtype) for k, v in dict(W1=W1, b1=b1, w2=w2, b2=b2).items()}
 
 

@@ -29,9 +29,9 @@
  *     features, weights and activations; arithmetic accumulates in fp32).  Edge counts < 2^31.
  *   - One process drives one GPU through this library (one process per GPU, as in data-parallel
  *     training): kernel attributes (large shared-memory carve-outs) and the address of the device
- *     status word are set up once, for the device current at the first call that needs them.
- *     (hg_overlap_align_loss_static looks up its scratch address per device, but the kernels it
- *     launches share the one-time set-up above.)
+ *     status word are set up once, and the library binds itself to the device current at its
+ *     first kernel-launching call (or to the one named by hg_bind_device).  A later call made
+ *     with another device current returns HG_ERR_UNSUPPORTED before launching anything.
  */
 #ifndef HG_H_
 #define HG_H_
@@ -73,6 +73,11 @@ const char* hg_status_string(hg_status status);
 const char* hg_last_error(void);
 /* Version of this ABI (bumped on any incompatible change). */
 int32_t hg_abi_version(void);
+/* Binds the library to device ordinal `device` (the CUDA runtime's numbering) before its first
+ * kernel-launching call; without it the first such call binds the device current then.  HG_OK if
+ * the library is unbound or already bound to `device`; HG_ERR_UNSUPPORTED if it is bound to
+ * another device; HG_ERR_INVALID_ARG for a negative ordinal.  Makes no CUDA call. */
+hg_status hg_bind_device(int32_t device);
 /* SYNCHRONISES the device, then reports and clears the library's device status word.  Every wait
  * inside a kernel of this library is bounded; a wait that gave up sets a flag here (its kernel's
  * results are then invalid) and this call returns HG_ERR_TIMEOUT.  flags may be NULL. */
@@ -381,8 +386,9 @@ hg_status hg_head_workspace_size(int64_t rows, int64_t n_lab, int32_t d, hg_dtyp
 
 /* Masked BCE of the head over the labelled rows and the joint objective:
  *   MeanAgg  h_r = H[lab_idx[r]], or, when that row is idx_a[k] of an overlap pair k < n_rep,
- *            (H[idx_a[k]] + H_rep[idx_b[k]]) / 2 rounded to the storage type (the mean of the
- *            node's two replicas);
+ *            (H[idx_a[k]] + H_rep[idx_b[k]]) / 2 (the mean of the node's two replicas; the
+ *            pre-activation below is formed from the two stored rows in fp32, the rows kept for
+ *            the weight gradient are the mean rounded to the storage type);
  *   Eq. 18   z_r = relu(h_r W1 + b1) . w2 + b2 (a logit; the probability is sigmoid(z_r));
  *   Eq. 19   loss_out[1] = L_BCE = (1/n_lab) sum_r -[y_r log p_r + (1 - y_r) log(1 - p_r)];
  *   Eq. 20   loss_out[0] = L_BCE + lambda_cca * cca_loss[0]  (cca_loss: device fp32, e.g. the

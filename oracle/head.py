@@ -26,9 +26,10 @@ Readings where the paper is silent or ambiguous (listed again in the design note
   MeanAgg averages the replicas present in the step (this subgraph's row and, for an overlap
   node, the second view's row); a detached second view receives no gradient;
   N_m is the number of labelled rows handed to the head; labels may be fractional (y in [0, 1]);
-  store="bf16": the averaged rows are rounded to bf16 (round to nearest even) like every bf16
-  embedding the interface exchanges, so the ReLU decisions that follow see the same inputs on
-  both sides; all other arithmetic stays fp64.
+  store="bf16": the averaged rows are rounded to bf16 (round to nearest even), as the bf16 kernel
+  stores them for the weight gradient; all other arithmetic stays fp64.  (The kernel's
+  pre-activation uses the unrounded mean of the two stored rows; the GPU tests compare with the
+  plain definition, store="f64".)
 """
 from __future__ import annotations
 

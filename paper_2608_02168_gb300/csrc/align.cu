@@ -629,6 +629,7 @@ extern "C" hg_status hg_overlap_intersect(const int64_t* gid_a, int64_t n_a, con
                                           int32_t* idx_a, int32_t* idx_b, int64_t* n_out, void* scratch,
                                           size_t scratch_bytes, hg_stream stream) {
   clear_error();
+  HG_TRY(device_guard());
   size_t need = 0;
   HG_TRY(hg_overlap_intersect_workspace_size(n_a, n_b, &need));
   HG_REQUIRE(n_out && scratch, "n_out and scratch must be non-null");
@@ -669,6 +670,7 @@ extern "C" hg_status hg_overlap_align_loss(const void* H_a, int64_t rows_a, cons
                                            int32_t d, hg_dtype dtype, float lambda_n, float var_eps, float* loss_out,
                                            void* saved, void* scratch, hg_stream stream) {
   clear_error();
+  HG_TRY(device_guard());
   const AlignIn in{H_a, rows_a, idx_a, H_b, rows_b, idx_b, n_max, n_dev};
   HG_TRY(check_align_args(in, d, dtype, saved, scratch));
   HG_REQUIRE(loss_out != nullptr, "loss_out must be non-null");
@@ -683,6 +685,7 @@ extern "C" hg_status hg_overlap_align_bwd(const void* H_a, int64_t rows_a, const
                                           int32_t d, hg_dtype dtype, float lambda_n, float var_eps, float dloss,
                                           const void* saved, void* dH_a, void* dH_b, void* scratch, hg_stream stream) {
   clear_error();
+  HG_TRY(device_guard());
   (void)var_eps;  // s = sqrt(var + eps) is part of `saved`
   const AlignIn in{H_a, rows_a, idx_a, H_b, rows_b, idx_b, n_max, n_dev};
   HG_TRY(check_align_args(in, d, dtype, saved, scratch));
@@ -764,6 +767,7 @@ extern "C" hg_status hg_overlap_align_loss_static(const void* H_a, int64_t rows_
                                                   float lambda_n, float var_eps, float* loss_out, void* saved,
                                                   hg_stream stream) {
   clear_error();
+  HG_TRY(device_guard());
   const AlignIn in{H_a, rows_a, idx_a, H_b, rows_b, idx_b, n_max, n_dev};
   void* scratch = nullptr;
   HG_TRY(static_align_scratch(&scratch));

@@ -555,6 +555,7 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
                                   const hg_rel_desc* rels, int32_t num_rels, void* workspace,
                                   size_t workspace_bytes, hg_stream stream, hg_graph** out) {
   clear_error();
+  HG_TRY(device_guard());
   HG_REQUIRE(out != nullptr, "out must be non-null");
   *out = nullptr;
   HG_REQUIRE(num_edges >= 0, "num_edges must be >= 0");
@@ -658,6 +659,7 @@ extern "C" hg_status hg_graph_destroy(hg_graph* graph) {
 
 extern "C" hg_status hg_graph_check(const hg_graph* graph, int64_t* num_invalid_edges) {
   clear_error();
+  HG_TRY(device_guard());
   HG_REQUIRE(graph != nullptr, "graph must be non-null");
   int32_t bad = 0;
   HG_CUDA(cudaMemcpyAsync(&bad, graph->invalid_count, sizeof(int32_t), cudaMemcpyDeviceToHost,

@@ -2,8 +2,10 @@
 // Algorithm 1).
 //
 // Forward (hg_head_loss), for the labelled rows r < n of one subgraph:
-//   MeanAgg   h_r = H[lab[r]], or (H[lab[r]] + H_rep[j]) / 2 rounded to the storage type when row
-//             lab[r] has a replica j in the second view (the overlap pairs idx_a -> idx_b)
+//   MeanAgg   h_r = H[lab[r]], or (H[lab[r]] + H_rep[j]) / 2 when row lab[r] has a replica j in
+//             the second view (the overlap pairs idx_a -> idx_b); the pre-activation uses that
+//             mean unrounded (fp32 here, two tensor-core chains for bf16), the rows saved for dW1
+//             are rounded to the storage type
 //   Eq. 18    a_r = h_r W1 + b1, z_r = relu(a_r) . w2 + b2                 (hidden width d)
 //   Eq. 19    L_BCE = (1/n) sum_r [y_r softplus(-z_r) + (1 - y_r) softplus(z_r)]
 //   Eq. 20    L_total = L_BCE + lambda_CCA L_CCA
@@ -108,7 +110,7 @@ __global__ void __launch_bounds__(256) head_fwd_simt(HeadFwdArgs a) {
           float g[VEC];
           unpack(ldg16(Hr + (int64_t)j * D + cv * VEC), g, T());
 #pragma unroll
-          for (int q = 0; q < VEC; ++q) f[q] = round_to<T>(0.5f * (f[q] + g[q]));
+          for (int q = 0; q < VEC; ++q) f[q] = 0.5f * (f[q] + g[q]);
         }
       }
       st16((T*)a.Hm + r * D + cv * VEC, pack(f, T()));
@@ -482,6 +484,7 @@ extern "C" hg_status hg_head_loss(const hg_head_params* params, const void* H, i
                                  const float* cca_loss, float lambda_cca, float* loss_out, float* logits, void* saved,
                                  void* scratch, hg_stream stream) {
   clear_error();
+  HG_TRY(device_guard());
   HG_TRY(check_head_params(params));
   HG_REQUIRE(loss_out && saved && scratch, "loss_out, saved and scratch must be non-null");
   HG_REQUIRE(((uintptr_t)saved & 255) == 0 && ((uintptr_t)scratch & 255) == 0, "buffers must be 256-byte aligned");
@@ -503,6 +506,7 @@ extern "C" hg_status hg_head_bwd(const hg_head_params* params, const int32_t* la
                                 const void* saved, void* dH, int64_t rows, void* dH_rep, int64_t rows_rep,
                                 int32_t overwrite, const hg_head_grads* grads, void* scratch, hg_stream stream) {
   clear_error();
+  HG_TRY(device_guard());
   HG_TRY(check_head_params(params));
   HG_REQUIRE(saved && scratch && grads, "saved, scratch and grads must be non-null");
   HG_REQUIRE(grads->dW1 && grads->db1 && grads->dw2 && grads->db2, "every gradient pointer must be non-null");

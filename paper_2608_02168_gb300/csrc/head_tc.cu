@@ -1,10 +1,14 @@
 // Tensor-core kernels of the bf16 prediction head (Section 3.4, Eq. 18-19).
 //
-// Forward, one CTA of 128 threads per 128 labelled rows: the threads gather the rows' MeanAgg
-// embeddings (one row of H, or the bf16-rounded mean of the row and its replica in H_rep) into a
-// 128-byte-swizzled K-major tile in shared memory and into the saved Hm; W1 arrives by TMA as an
-// MN-major operand (its rows are the K dimension, 64-column blocks along the hidden units); one
-// chain of tcgen05.mma puts A = Hm W1 (fp32, 128 x d) in tensor memory.  Thread t then owns row t:
+// Forward, one CTA of 128 threads per 128 labelled rows: the threads gather the labelled rows of H
+// into a 128-byte-swizzled K-major tile in shared memory (and the rows' MeanAgg embedding, the
+// mean with the replica in H_rep rounded to bf16, into the saved Hm for the weight gradient); W1
+// arrives by TMA as an MN-major operand (its rows are the K dimension, 64-column blocks along the
+// hidden units); one chain of tcgen05.mma puts H W1 (fp32, 128 x d) in tensor memory.  When rows
+// of the tile have a replica, the tile is refilled with the replica rows (zero elsewhere) once the
+// first chain has read it, and a second chain adds H_rep W1; the epilogue halves those rows.  So
+// the pre-activation a = ((h + h_rep) / 2) W1 is formed from the stored bf16 rows without rounding
+// their mean.  Thread t then owns row t:
 // it adds b1, forms the logit z = relu(a) . w2 + b2, the loss term and the unit gradient
 // dA = (sigmoid(z) - y)/n * w2 * [a > 0], stores dA (bf16), and the CTA writes its partial sums
 // (loss, dz, column sums of dA and of dz relu(a)) in a fixed order.
@@ -158,29 +162,58 @@ __global__ void __launch_bounds__(kThreads, 1)
         h = pack(x, __nv_bfloat16());
       }
       if (r < a.n) st16((__nv_bfloat16*)a.Hm + r * D + g * 8, h);
-      st16(Aimg + (g >> 3) * kABlk + sw128_offset(rl, (g & 7) * 16), h);
+      st16(Aimg + (g >> 3) * kABlk + sw128_offset(rl, (g & 7) * 16), v[q]);
     }
   }
   fence_async_smem();
-  __syncthreads();
+  const bool two = __syncthreads_or(rowi[tid] >= 0 && repi[tid] >= 0) != 0;  // any replica in the tile
+  auto issue_chain = [&](bool accumulate) {
+    fence_after_sync();
+    const uint32_t A = smem_u32(Aimg), W = smem_u32(Wimg);
+    const uint32_t idesc = idesc_bf16(128, D, false, true);
+#pragma unroll
+    for (int j = 0; j < D / 16; ++j)
+      mma_bf16(tmem, desc_sw128(A + (j >> 2) * kABlk + (j & 3) * 32, 16, 1024),
+               desc_sw128(W + j * 2048, C::kWBlk, 1024), idesc, (accumulate || j > 0) ? 1u : 0u);
+    mma_commit(&bars[1]);
+  };
   bool ok = true;
   if (tid == 0) {
     ok = mbar_wait(&bars[0], 0);
-    if (ok) {
-      fence_after_sync();
-      const uint32_t A = smem_u32(Aimg), W = smem_u32(Wimg);
-      const uint32_t idesc = idesc_bf16(128, D, false, true);
-#pragma unroll
-      for (int j = 0; j < D / 16; ++j)
-        mma_bf16(tmem, desc_sw128(A + (j >> 2) * kABlk + (j & 3) * 32, 16, 1024),
-                 desc_sw128(W + j * 2048, C::kWBlk, 1024), idesc, j > 0 ? 1u : 0u);
-      mma_commit(&bars[1]);
-    } else {
+    if (ok)
+      issue_chain(false);
+    else
       record_device_error(a.status, kErrTimeout);
-    }
   }
   ok = __syncthreads_and(ok);
-  if (ok && !mbar_wait(&bars[1], 0)) {
+  if (ok && two) {
+    // the first chain has read the tile: refill it with the replica rows (zero for rows without)
+    if (!mbar_wait(&bars[1], 0)) {
+      record_device_error(a.status, kErrTimeout);
+      ok = false;
+    }
+    ok = __syncthreads_and(ok);
+    if (ok) {
+      fence_after_sync();
+#pragma unroll 1
+      for (int p0 = 0; p0 < PASSES; p0 += BATCH) {
+        uint4 u[BATCH];
+#pragma unroll
+        for (int q = 0; q < BATCH; ++q) {
+          const int rl = sub + (p0 + q) * RPP;
+          const int32_t i = rowi[rl], j = repi[rl];
+          u[q] = (i >= 0 && j >= 0) ? ldg16(Hr + (int64_t)j * D + g * 8) : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int q = 0; q < BATCH; ++q)
+          st16(Aimg + (g >> 3) * kABlk + sw128_offset(sub + (p0 + q) * RPP, (g & 7) * 16), u[q]);
+      }
+      fence_async_smem();
+      __syncthreads();
+      if (tid == 0) issue_chain(true);
+    }
+  }
+  if (ok && !mbar_wait(&bars[1], two ? 1 : 0)) {
     record_device_error(a.status, kErrTimeout);
     ok = false;
   }
@@ -192,13 +225,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   const bool valid = live && rowi[rl] >= 0;
   const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
   const float b2 = __bfloat162float(((const __nv_bfloat16*)a.b2)[0]);
+  const float half = (rowi[rl] >= 0 && repi[rl] >= 0) ? 0.5f : 1.f;  // (h + h_rep) W1 / 2
   float zpart = 0.f;
 #pragma unroll 1
   for (int c = 0; c < D; c += 32) {
     float acc[32];
     tmem_ld32(trow + c, acc);
 #pragma unroll
-    for (int e = 0; e < 32; ++e) zpart = fmaf(fmaxf(acc[e] + b1f[c + e], 0.f), w2f[c + e], zpart);
+    for (int e = 0; e < 32; ++e) zpart = fmaf(fmaxf(fmaf(half, acc[e], b1f[c + e]), 0.f), w2f[c + e], zpart);
   }
   const float z = zpart + b2;
   float term = 0.f, dz = 0.f;
@@ -219,7 +253,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_ld32(trow + c, acc);
 #pragma unroll
     for (int e = 0; e < 32; ++e) {
-      const float h = acc[e] + b1f[c + e];
+      const float h = fmaf(half, acc[e], b1f[c + e]);
       da[e] = h > 0.f ? dz * w2f[c + e] : 0.f;
       dw[e] = dz * fmaxf(h, 0.f);
     }

@@ -27,6 +27,9 @@ constexpr int kChunkEdges = 512;
 // ---------------------------------------------------------------------------------------------
 void set_error(const char* fmt, ...);
 void clear_error();
+// HG_OK when the current device is the one this process's library state is bound to (binding it
+// at the first call); HG_ERR_UNSUPPORTED, before any launch, when another device is current.
+hg_status device_guard();
 
 #define HG_REQUIRE(cond, ...)              \
   do {                                     \

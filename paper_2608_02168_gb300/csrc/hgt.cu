@@ -2,17 +2,22 @@
 //
 // With S heads of width d_h and c_r = mu[r] / sqrt(d_h), the layer is computed as
 //   K, V = H W_K + b_K, H W_V + b_V (per source type; one N x 2d array, a node's K then V)
-//   Q'_r(j) = (H_j W_Q + b_Q) blockdiag(W_att[r])^T c_r   (one row per (relation, target): the CSR
-//             row layout of the mean layer)                  so that score^s(e) = K^s(i) . Q'^s_r(j)
+//   Q       = H W_Q + b_Q (per target type)
+//   Q'_r(j) = c_r Q_j blockdiag(W_att[r])^T   (one row per (relation, target): the CSR row layout
+//             of the mean layer; c_r applied in fp32)    so that score^s(e) = K^s(i) . Q'^s_r(j)
 //   alpha   = softmax over every in-edge of j, per head (online: running maximum and sum)
 //   S_r(j)  = sum over the r-edges into j of alpha V(i)    (per head; CSR row layout)
 //   U       = sum_r S_r blockdiag(W_msg[r]) W_agg + b_agg, then activation, residual, LayerNorm:
 //             the mean layer's projection with W_rel = blockdiag(W_msg[r]).
+// Every product has a stored bf16 weight as one factor (W_K, W_Q, W_V, blockdiag(W_att[r]),
+// blockdiag(W_msg[r]) paired with W_agg as the projection's hi / lo fused weights), so no product
+// of two weights is ever rounded to bf16; the scalar c_r multiplies in the fp32 epilogue.
 // The backward reuses that projection's backward (without the 1/deg scaling) for dS_r, then
 //   target pass  D^s_j = sum_r <dS_r(j), S_r(j)>^s, de = alpha (<dS_r(j), V(i)>^s - D^s_j),
 //                dQ'_r(j) = sum de K(i)
 //   source pass  dK(i) = sum over out-edges de Q'_r(j), dV(i) = sum alpha dS_r(j)
-//   and the dense products back to H and to the weights.
+//   and the dense products back to H (dQ = sum_r c_r dQ'_r blockdiag(W_att[r]), then dQ W_Q^T) and
+//   to the weights.
 // Edge work is warp per row (a lane holds d / 32 consecutive features, the 32 / S lanes of a head
 // reduce by shuffles); rows above the hub degree are split into chunks whose partial results are
 // merged in chunk order, so every reduction has a fixed order (deterministic, atomic-free).  The
@@ -79,58 +84,23 @@ __device__ __forceinline__ float head_sum(float x, int lph) {
 }
 
 // ---------------------------------------------------------------------------------------------
-// derived weights (fp64 arithmetic, one rounding)
+// block-diagonal expansion of per-head weights (exact copies, no arithmetic)
 // ---------------------------------------------------------------------------------------------
-// kind 0: WQp[r] = W_Q[t_r] blockdiag(W_att[r])^T c_r     (d x d; also bQp[r] = b_Q[t_r] (...))
-// kind 1: BDmsg[r] = blockdiag(W_msg[r])                  (d x d)
-// kind 2: FQ[r] = c_r blockdiag(W_att[r]) W_Q[t_r]^T      (d x d: dQ'_r -> dH)
-// kind 3: BDc[r] = c_r blockdiag(W_att[r])                (d x d: dQ'_r -> dQ)
+// out[r] = blockdiag(W[r]) (d x d, S blocks of d_h x d_h), or its transpose when transpose != 0.
 template <typename T>
-__global__ void hgt_prep(int kind, const T* __restrict__ W_Q, const T* __restrict__ b_Q, const T* __restrict__ W_att,
-                         const T* __restrict__ W_msg, const float* __restrict__ mu, RelDst rd, int R, int d, int S,
-                         T* __restrict__ out, T* __restrict__ bout) {
+__global__ void hgt_blockdiag(const T* __restrict__ W, int R, int d, int S, int transpose, T* __restrict__ out) {
   const int dh = d / S;
-  const double rs = 1.0 / sqrt((double)dh);
   const int64_t total = (int64_t)R * d * d;
-  for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < total + (kind == 0 ? R * d : 0);
-       q += (int64_t)gridDim.x * blockDim.x) {
-    if (q >= total) {  // bias of kind 0
-      const int r = (int)((q - total) / d), b = (int)((q - total) % d);
-      const int s = b / dh, bb = b % dh;
-      const T* Wa = W_att + ((int64_t)r * S + s) * dh * dh;
-      const T* bq = b_Q + (int64_t)rd.v[r] * d;
-      double acc = 0.0;
-      for (int k = 0; k < dh; ++k) acc += (double)to_f32(bq[s * dh + k]) * (double)to_f32(Wa[bb * dh + k]);
-      bout[(int64_t)r * d + b] = from_f32<T>((float)(acc * mu[r] * rs));
-      continue;
-    }
+  for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < total; q += (int64_t)gridDim.x * blockDim.x) {
     const int r = (int)(q / ((int64_t)d * d));
-    const int a = (int)((q / d) % d), b = (int)(q % d);
-    const int t = rd.v[r];
-    const double c = mu[r] * rs;
-    double v = 0.0;
-    if (kind == 1) {
-      const int s = a / dh;
-      if (b / dh == s) v = to_f32(W_msg[((int64_t)r * S + s) * dh * dh + (a % dh) * dh + (b % dh)]);
-    } else if (kind == 3) {
-      const int s = a / dh;
-      if (b / dh == s) v = c * to_f32(W_att[((int64_t)r * S + s) * dh * dh + (a % dh) * dh + (b % dh)]);
-    } else if (kind == 0) {
-      // (W_Q BD^T)[a][b] = sum_k W_Q[a][k] BD[b][k], k in the head of b
-      const int s = b / dh, bb = b % dh;
-      const T* Wa = W_att + ((int64_t)r * S + s) * dh * dh;
-      const T* wq = W_Q + (int64_t)t * d * d + (int64_t)a * d;
-      for (int k = 0; k < dh; ++k) v += (double)to_f32(wq[s * dh + k]) * (double)to_f32(Wa[bb * dh + k]);
-      v *= c;
-    } else {
-      // (BD W_Q^T)[a][b] = sum_k BD[a][k] W_Q[b][k], k in the head of a
-      const int s = a / dh, aa = a % dh;
-      const T* Wa = W_att + ((int64_t)r * S + s) * dh * dh;
-      const T* wq = W_Q + (int64_t)t * d * d + (int64_t)b * d;
-      for (int k = 0; k < dh; ++k) v += (double)to_f32(Wa[aa * dh + k]) * (double)to_f32(wq[s * dh + k]);
-      v *= c;
+    int a = (int)((q / d) % d), b = (int)(q % d);
+    if (transpose) {
+      const int t = a;
+      a = b;
+      b = t;
     }
-    out[q] = from_f32<T>((float)v);
+    const int s = a / dh;
+    out[q] = b / dh == s ? W[((int64_t)r * S + s) * dh * dh + (a % dh) * dh + (b % dh)] : from_f32<T>(0.f);
   }
 }
 
@@ -146,13 +116,15 @@ __global__ void hgt_transpose(const T* __restrict__ W, int count, int d, T* __re
 }
 
 // ---------------------------------------------------------------------------------------------
-// dense row products on CUDA cores: out[r][ocol0 + c] (=, or +=) sum_k A[r][k] B[k][c] (+ bias[c]),
-// c < D, rows [0, n), K a multiple of 32; A row stride lda, out row stride ldo, B is K x D.
+// dense row products on CUDA cores: out[r][ocol0 + c] (=, or +=) scale sum_k A[r][k] B[k][c]
+// (+ bias[c]), c < D, rows [0, n), K a multiple of 32; A row stride lda, out row stride ldo, B is
+// K x D; scale = scale_mul * (*scale_ptr) (null scale_ptr: 1).
 // ---------------------------------------------------------------------------------------------
 template <typename T, int D>
 __global__ void __launch_bounds__(256) hgt_gemm_simt(const T* __restrict__ A, int64_t lda, const T* __restrict__ B,
                                                      const T* __restrict__ bias, int K, int64_t n, T* __restrict__ out,
-                                                     int64_t ldo, int ocol0, int accumulate) {
+                                                     int64_t ldo, int ocol0, int accumulate,
+                                                     const float* __restrict__ scale_ptr, float scale_mul) {
   using Tl = Tile<float, D>;
   constexpr int CN = Tl::CN, RM = Tl::RM;
   __shared__ __align__(16) float As[kBM][kAPad];
@@ -177,6 +149,7 @@ __global__ void __launch_bounds__(256) hgt_gemm_simt(const T* __restrict__ A, in
     __syncthreads();
   }
   const int ty = threadIdx.x / 16, tx = threadIdx.x % 16;
+  const float sc = scale_mul * (scale_ptr ? *scale_ptr : 1.f);
 #pragma unroll
   for (int i = 0; i < RM; ++i) {
     const int64_t r = r0 + ty * RM + i;
@@ -184,7 +157,7 @@ __global__ void __launch_bounds__(256) hgt_gemm_simt(const T* __restrict__ A, in
     T* o = out + r * ldo + ocol0 + tx * CN;
 #pragma unroll
     for (int j = 0; j < CN; ++j) {
-      float v = acc[i][j];
+      float v = sc * acc[i][j];
       if (bias) v += to_f32(bias[tx * CN + j]);
       if (accumulate) v += to_f32(o[j]);
       o[j] = from_f32<T>(v);
@@ -667,19 +640,18 @@ struct HgtLayout {
   void* KV;       // N x 2d
   void* Qp;       // csr_rows x d
   float2* stats;  // N x S
-  void* BDmsg;    // R x d x d
+  void* BDmsg;    // R x d x d  blockdiag(W_msg[r])
   // scratch
-  void* WQp;      // R x d x d
-  void* bQp;      // R x d
-  void* FQ;       // R x d x d
-  void* BDc;      // R x d x d
+  void* BDattT;   // R x d x d  blockdiag(W_att[r])^T
+  void* BDatt;    // R x d x d  blockdiag(W_att[r])
   void* WKt;      // T x d x d
   void* WVt;      // T x d x d
+  void* WQt;      // T x d x d
   float4* rstat;  // csr_rows x S
   void* dQp;      // csr_rows x d
   void* dK;       // N x d
   void* dV;       // N x d
-  void* Qbuf;     // N x d (recomputed Q)
+  void* Qbuf;     // N x d: Q (forward), recomputed in the backward
   void* dQ;       // N x d
   float* part;    // chunk partials
   float* cs;      // column-sum partials
@@ -711,12 +683,11 @@ void carve_hgt(const hg_graph* g, const hg_hgt_params* p, void* saved, void* scr
   H->Qp = s.take<char>((size_t)std::max<int64_t>(g->csr_rows, 1) * d * b);
   H->stats = s.take<float2>((size_t)std::max<int64_t>(N, 1) * S);
   H->BDmsg = s.take<char>(m.num_rels * dd * b);
-  H->WQp = k.take<char>(m.num_rels * dd * b);
-  H->bQp = k.take<char>((size_t)m.num_rels * d * b);
-  H->FQ = k.take<char>(m.num_rels * dd * b);
-  H->BDc = k.take<char>(m.num_rels * dd * b);
+  H->BDattT = k.take<char>(m.num_rels * dd * b);
+  H->BDatt = k.take<char>(m.num_rels * dd * b);
   H->WKt = k.take<char>(m.num_types * dd * b);
   H->WVt = k.take<char>(m.num_types * dd * b);
+  H->WQt = k.take<char>(m.num_types * dd * b);
   H->rstat = k.take<float4>((size_t)std::max<int64_t>(g->csr_rows, 1) * S);
   H->dQp = k.take<char>((size_t)std::max<int64_t>(g->csr_rows, 1) * d * b);
   H->dK = k.take<char>((size_t)std::max<int64_t>(N, 1) * d * b);
@@ -796,14 +767,15 @@ unsigned chunk_blocks(int64_t cap) { return (unsigned)std::max<int64_t>(1, std::
 
 template <typename T, int D>
 hg_status gemm(const void* A, int64_t lda, const void* B, const void* bias, int K, int64_t n, void* out, int64_t ldo,
-               int ocol0, int accumulate, cudaStream_t s) {
+               int ocol0, int accumulate, cudaStream_t s, const float* scale_ptr = nullptr, float scale_mul = 1.f) {
   if (n <= 0) return HG_OK;
   if constexpr (sizeof(T) == 2) {  // bf16: tensor cores (every product here has K = lda = D)
-    if (lda == D && K == D) return rows_gemm_tc(D, A, n, B, bias, out, ldo, ocol0, accumulate, s);
+    if (lda == D && K == D)
+      return rows_gemm_tc(D, A, n, B, bias, out, ldo, ocol0, accumulate, scale_ptr, scale_mul, s);
   }
   return launch("hgt_gemm_simt", hgt_gemm_simt<T, D>, dim3((unsigned)ceil_div(n, kBM)), dim3(256),
                 sizeof(float) * kKC * D, s, (const T*)A, lda, (const T*)B, (const T*)bias, K, n, (T*)out, ldo, ocol0,
-                accumulate);
+                accumulate, scale_ptr, scale_mul);
 }
 
 template <typename T>
@@ -839,27 +811,27 @@ hg_status hgt_fwd_t(const hg_graph* g, const hg_hgt_params* p, const void* H_in,
   const int64_t N = m.type_off[m.num_types];
   const size_t dd = (size_t)D * D;
   const T* Hin = (const T*)H_in;
-  const RelDst rd = rel_dst_of(m);
-  // derived weights: relation-scaled query maps and the block-diagonal message matrices
-  HG_TRY(launch("hgt_prep", hgt_prep<T>, dim3(grid_of((int64_t)m.num_rels * dd + m.num_rels * D)), dim3(256), 0, s, 0,
-                (const T*)p->W_Q, (const T*)p->b_Q, (const T*)p->W_att, (const T*)p->W_msg, p->mu, rd, m.num_rels, D,
-                S, (T*)H.WQp, (T*)H.bQp));
-  HG_TRY(launch("hgt_prep", hgt_prep<T>, dim3(grid_of((int64_t)m.num_rels * dd)), dim3(256), 0, s, 1,
-                (const T*)p->W_Q, (const T*)p->b_Q, (const T*)p->W_att, (const T*)p->W_msg, p->mu, rd, m.num_rels, D,
-                S, (T*)H.BDmsg, (T*)nullptr));
-  // K and V of every node, Q' of every (relation, target) row
+  const float rs = (float)(1.0 / std::sqrt((double)(D / S)));
+  // block-diagonal attention (transposed) and message matrices
+  HG_TRY(launch("hgt_blockdiag", hgt_blockdiag<T>, dim3(grid_of((int64_t)m.num_rels * dd)), dim3(256), 0, s,
+                (const T*)p->W_att, m.num_rels, D, S, 1, (T*)H.BDattT));
+  HG_TRY(launch("hgt_blockdiag", hgt_blockdiag<T>, dim3(grid_of((int64_t)m.num_rels * dd)), dim3(256), 0, s,
+                (const T*)p->W_msg, m.num_rels, D, S, 0, (T*)H.BDmsg));
+  // K, V and Q of every node, Q' of every (relation, target) row
   for (int t = 0; t < m.num_types; ++t) {
     const int64_t off = m.type_off[t], n = m.type_off[t + 1] - off;
     HG_TRY((gemm<T, D>(Hin + off * D, D, (const T*)p->W_K + t * dd, (const T*)p->b_K + (size_t)t * D, D, n,
                        (T*)H.KV + off * 2 * D, 2 * D, 0, 0, s)));
     HG_TRY((gemm<T, D>(Hin + off * D, D, (const T*)p->W_V + t * dd, (const T*)p->b_V + (size_t)t * D, D, n,
                        (T*)H.KV + off * 2 * D, 2 * D, D, 0, s)));
+    HG_TRY((gemm<T, D>(Hin + off * D, D, (const T*)p->W_Q + t * dd, (const T*)p->b_Q + (size_t)t * D, D, n,
+                       (T*)H.Qbuf + off * D, D, 0, 0, s)));
   }
-  for (int r = 0; r < m.num_rels; ++r) {
+  for (int r = 0; r < m.num_rels; ++r) {  // Q'_r = c_r Q blockdiag(W_att[r])^T, c_r = mu[r] / sqrt(d_h)
     const int t = m.rel_dst[r];
     const int64_t off = m.type_off[t], n = m.type_off[t + 1] - off;
-    HG_TRY((gemm<T, D>(Hin + off * D, D, (const T*)H.WQp + r * dd, (const T*)H.bQp + (size_t)r * D, D, n,
-                       (T*)H.Qp + m.row_base[r] * D, D, 0, 0, s)));
+    HG_TRY((gemm<T, D>((const T*)H.Qbuf + off * D, D, (const T*)H.BDattT + r * dd, nullptr, D, n,
+                       (T*)H.Qp + m.row_base[r] * D, D, 0, 0, s, p->mu + r, rs)));
   }
   // Eq. 6-10: softmax over the in-edges, weighted value sums per relation row
   const HgtArgs a = edge_args(g, p, H);
@@ -882,7 +854,7 @@ hg_status hgt_bwd_t(const hg_graph* g, const hg_hgt_params* p, const void* H_in,
   const int64_t N = m.type_off[m.num_types];
   const size_t dd = (size_t)D * D;
   const T* Hin = (const T*)H_in;
-  const RelDst rd = rel_dst_of(m);
+  const float rs = (float)(1.0 / std::sqrt((double)(D / S)));
   // Eq. 11 backward: dY (residual), dS_r (no degree scaling), dW of blockdiag(W_msg), dW_agg, db, LN
   const hg_layer_params lp = projection_params(p, H);
   hg_layer_grads lg{};
@@ -905,18 +877,28 @@ hg_status hgt_bwd_t(const hg_graph* g, const hg_hgt_params* p, const void* H_in,
   HG_TRY(launch("hgt_bwd_src_chunks", hgt_bwd_src_chunks<T, D>, dim3(chunk_blocks(g->chunk_cap_node)), dim3(256), 0,
                 s, a));
   HG_TRY(launch("hgt_bwd_src_nodes", hgt_bwd_src_nodes<T, D>, dim3(grid_of(N * 32)), dim3(256), 0, s, a));
-  // derived weights of the backward products
-  HG_TRY(launch("hgt_prep", hgt_prep<T>, dim3(grid_of((int64_t)m.num_rels * dd)), dim3(256), 0, s, 2,
-                (const T*)p->W_Q, (const T*)p->b_Q, (const T*)p->W_att, (const T*)p->W_msg, p->mu, rd, m.num_rels, D,
-                S, (T*)H.FQ, (T*)nullptr));
-  HG_TRY(launch("hgt_prep", hgt_prep<T>, dim3(grid_of((int64_t)m.num_rels * dd)), dim3(256), 0, s, 3,
-                (const T*)p->W_Q, (const T*)p->b_Q, (const T*)p->W_att, (const T*)p->W_msg, p->mu, rd, m.num_rels, D,
-                S, (T*)H.BDc, (T*)nullptr));
+  // weights of the backward products (exact copies and transposes)
+  HG_TRY(launch("hgt_blockdiag", hgt_blockdiag<T>, dim3(grid_of((int64_t)m.num_rels * dd)), dim3(256), 0, s,
+                (const T*)p->W_att, m.num_rels, D, S, 0, (T*)H.BDatt));
   HG_TRY(launch("hgt_transpose", hgt_transpose<T>, dim3(grid_of((int64_t)m.num_types * dd)), dim3(256), 0, s,
                 (const T*)p->W_K, m.num_types, D, (T*)H.WKt));
   HG_TRY(launch("hgt_transpose", hgt_transpose<T>, dim3(grid_of((int64_t)m.num_types * dd)), dim3(256), 0, s,
                 (const T*)p->W_V, m.num_types, D, (T*)H.WVt));
-  // dH_in = dY + dK W_K^T + dV W_V^T + sum_r dQ'_r (c_r blockdiag(W_att[r]) W_Q^T)
+  HG_TRY(launch("hgt_transpose", hgt_transpose<T>, dim3(grid_of((int64_t)m.num_types * dd)), dim3(256), 0, s,
+                (const T*)p->W_Q, m.num_types, D, (T*)H.WQt));
+  // dQ = sum_r c_r dQ'_r blockdiag(W_att[r]) per target type
+  for (int t = 0; t < m.num_types; ++t) {
+    const int64_t off = m.type_off[t], n = m.type_off[t + 1] - off;
+    int k = 0;
+    for (int r = 0; r < m.num_rels; ++r) {
+      if (m.rel_dst[r] != t) continue;
+      HG_TRY((gemm<T, D>((const T*)H.dQp + m.row_base[r] * D, D, (const T*)H.BDatt + r * dd, nullptr, D, n,
+                         (T*)H.dQ + off * D, D, 0, k > 0, s, p->mu + r, rs)));
+      ++k;
+    }
+    if (k == 0 && n > 0) HG_CUDA(cudaMemsetAsync((T*)H.dQ + off * D, 0, (size_t)n * D * sizeof(T), s));
+  }
+  // dH_in = dY + dK W_K^T + dV W_V^T + dQ W_Q^T
   if (dH_in) {
     HG_CUDA(cudaMemcpyAsync(dH_in, H.L.dY, (size_t)N * D * sizeof(T), cudaMemcpyDeviceToDevice, s));
     T* dH = (T*)dH_in;
@@ -926,29 +908,18 @@ hg_status hgt_bwd_t(const hg_graph* g, const hg_hgt_params* p, const void* H_in,
                          s)));
       HG_TRY((gemm<T, D>((const T*)H.dV + off * D, D, (const T*)H.WVt + t * dd, nullptr, D, n, dH + off * D, D, 0, 1,
                          s)));
-      for (int r = 0; r < m.num_rels; ++r) {
-        if (m.rel_dst[r] != t) continue;
-        HG_TRY((gemm<T, D>((const T*)H.dQp + m.row_base[r] * D, D, (const T*)H.FQ + r * dd, nullptr, D, n,
-                           dH + off * D, D, 0, 1, s)));
-      }
+      HG_TRY((gemm<T, D>((const T*)H.dQ + off * D, D, (const T*)H.WQt + t * dd, nullptr, D, n, dH + off * D, D, 0, 1,
+                         s)));
     }
   }
-  // weight gradients of the three typed maps: dW = H^T dZ, db = column sums of dZ
+  // weight gradients of the three typed maps: dW = H^T dZ, db = column sums of dZ; Q recomputed for
+  // the attention matrices' gradients
   for (int t = 0; t < m.num_types; ++t) {
     const int64_t off = m.type_off[t], n = m.type_off[t + 1] - off;
     HG_TRY(wgrad(kDt, D, H_in, off, H.dK, off, n, gr->dW_K + t * dd, H.L, s));
     HG_TRY(wgrad(kDt, D, H_in, off, H.dV, off, n, gr->dW_V + t * dd, H.L, s));
     HG_TRY(colsum<T>((const T*)H.dK + off * D, D, D, n, H.cs, gr->db_K + (size_t)t * D, H.L.rtmp, s));
     HG_TRY(colsum<T>((const T*)H.dV + off * D, D, D, n, H.cs, gr->db_V + (size_t)t * D, H.L.rtmp, s));
-    // dQ = sum_r dQ'_r c_r blockdiag(W_att[r]); Q recomputed for the attention matrices' gradients
-    int k = 0;
-    for (int r = 0; r < m.num_rels; ++r) {
-      if (m.rel_dst[r] != t) continue;
-      HG_TRY((gemm<T, D>((const T*)H.dQp + m.row_base[r] * D, D, (const T*)H.BDc + r * dd, nullptr, D, n,
-                         (T*)H.dQ + off * D, D, 0, k > 0, s)));
-      ++k;
-    }
-    if (k == 0 && n > 0) HG_CUDA(cudaMemsetAsync((T*)H.dQ + off * D, 0, (size_t)n * D * sizeof(T), s));
     HG_TRY(wgrad(kDt, D, H_in, off, H.dQ, off, n, gr->dW_Q + t * dd, H.L, s));
     HG_TRY(colsum<T>((const T*)H.dQ + off * D, D, D, n, H.cs, gr->db_Q + (size_t)t * D, H.L.rtmp, s));
     HG_TRY((gemm<T, D>(Hin + off * D, D, (const T*)p->W_Q + t * dd, (const T*)p->b_Q + (size_t)t * D, D, n,
@@ -1018,6 +989,7 @@ extern "C" hg_status hg_hgt_workspace_size(const hg_graph* graph, const hg_hgt_p
 extern "C" hg_status hg_hgt_fwd(const hg_graph* graph, const hg_hgt_params* params, const void* H_in, void* H_out,
                                void* saved, void* scratch, hg_stream stream) {
   clear_error();
+  HG_TRY(device_guard());
   HG_TRY(check_hgt(graph, params));
   HG_TRY(check_buf256(H_in, "H_in"));
   HG_TRY(check_buf256(H_out, "H_out"));
@@ -1034,6 +1006,7 @@ extern "C" hg_status hg_hgt_bwd(const hg_graph* graph, const hg_hgt_params* para
                                const void* saved, const void* dH_out, void* dH_in, const hg_hgt_grads* grads,
                                void* scratch, hg_stream stream) {
   clear_error();
+  HG_TRY(device_guard());
   HG_TRY(check_hgt(graph, params));
   HG_TRY(check_buf256(H_in, "H_in"));
   HG_TRY(check_buf256(saved, "saved"));

@@ -82,8 +82,8 @@ void carve_layer(const hg_graph* g, int d, hg_dtype dt, void* saved, void* scrat
   L->U = s.take<char>((size_t)N * d * b);
   L->stats = s.take<float2>(std::max<int64_t>(N, 1));
   if (tc) {
-    L->V = s.take<char>(m.num_rels * dd * b);
-    L->Vt = s.take<char>(m.num_rels * dd * b);
+    L->V = s.take<char>(2 * m.num_rels * dd * b);  // hi and lo halves of each fused weight
+    L->Vt = s.take<char>(2 * m.num_rels * dd * b);
   }
   L->agg_part = k.take<float>((size_t)std::max(g->chunk_cap_csr, g->chunk_cap_node) * d);
   L->dY = k.take<char>((size_t)N * d * b);
@@ -159,6 +159,7 @@ extern "C" int32_t hg_abi_version(void) { return 1; }
 
 extern "C" hg_status hg_device_status(int32_t* flags) {
   clear_error();
+  HG_TRY(device_guard());
   int* p = device_status_ptr();
   HG_REQUIRE(p != nullptr, "device status word unavailable");
   int v = 0;
@@ -225,6 +226,7 @@ extern "C" hg_status hg_layer_workspace_size(const hg_graph* graph, const hg_lay
 extern "C" hg_status hg_layer_fwd(const hg_graph* graph, const hg_layer_params* p, const void* H_in, void* H_out,
                                   void* saved, void* scratch, hg_stream stream) {
   clear_error();
+  HG_TRY(device_guard());
   HG_TRY(check_params(graph, p));
   HG_TRY(check_buf(H_in, "H_in"));
   HG_TRY(check_buf(H_out, "H_out"));
@@ -311,6 +313,7 @@ extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* 
                                   const void* dH_out, void* dH_in, const hg_layer_grads* grads, void* scratch,
                                   hg_stream stream) {
   clear_error();
+  HG_TRY(device_guard());
   HG_TRY(check_params(graph, p));
   HG_TRY(check_buf(H_in, "H_in"));
   HG_TRY(check_buf(saved, "saved"));

@@ -124,10 +124,11 @@ size_t reduce_tmp_floats(int splits, int64_t count);
 hg_status reduce_partials3(const float* part, int64_t stride, int splits, int64_t seg, float* out0, float* out1,
                            float* out2, cudaStream_t s);
 int wgrad_splits(int64_t n);
-// Tensor-core row product (bf16): out[r][ocol0 + c] (=, or += when accumulate) A[r] B + bias,
-// A: n x d rows (row stride d), B: d x d row-major, bias: d or null; out row stride ldo.
+// Tensor-core row product (bf16): out[r][ocol0 + c] (=, or += when accumulate) scale A[r] B + bias,
+// A: n x d rows (row stride d), B: d x d row-major, bias: d or null; out row stride ldo; scale =
+// scale_mul * (*scale_ptr), scale_ptr a device fp32 scalar or null (1).
 hg_status rows_gemm_tc(int d, const void* A, int64_t n, const void* B, const void* bias, void* out, int64_t ldo,
-                       int ocol0, int accumulate, cudaStream_t s);
+                       int ocol0, int accumulate, const float* scale_ptr, float scale_mul, cudaStream_t s);
 
 // Buffers of one layer (saved for the backward, and scratch).
 struct LayerLayout {
@@ -135,8 +136,8 @@ struct LayerLayout {
   void* Z;        // saved (fp32 storage only): N x d
   void* U;        // saved: N x d pre-activation
   float2* stats;  // saved: N row statistics
-  void* V;        // saved (bf16 only): R x d x d fused weights W_r W_agg
-  void* Vt;       // saved (bf16 only): their transposes
+  void* V;        // saved (bf16 only): R x 2 x d x d fused weights W_r W_agg (hi, lo halves)
+  void* Vt;       // saved (bf16 only): their transposes (same order)
   float* agg_part;  // scratch: chunk partials
   void* dY;       // scratch: N x d
   void* dU;

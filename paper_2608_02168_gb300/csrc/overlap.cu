@@ -434,6 +434,7 @@ extern "C" hg_status hg_overlap_build(const int32_t* src, const int32_t* dst, co
                                       int64_t* counts_out, void* workspace, size_t workspace_bytes,
                                       hg_stream stream) {
   clear_error();
+  HG_TRY(device_guard());
   size_t need = 0;
   HG_TRY(hg_overlap_build_workspace_size(num_nodes, num_edges, &need));
   HG_REQUIRE(K >= 1 && k >= 0 && k < K, "need K >= 1 and 0 <= k < K");

@@ -2,16 +2,23 @@
 // fp32 accumulation in tensor memory).  Used for bf16 storage; fp32 storage stays on CUDA cores.
 //
 // The two products of Eq. 7 and Eq. 11 are associated as U = sum_r M_r V_r + b with the fused
-// weights V_r = W_r W_agg[t_r] (computed once per layer in fp64, stored in bf16): the same value
-// as (sum_r M_r W_r) W_agg up to rounding, with one GEMM instead of two and no intermediate Z.
+// weights V_r = W_r W_agg[t_r] (computed once per layer in fp64): the same value as
+// (sum_r M_r W_r) W_agg, with one GEMM instead of two and no intermediate Z.  A product of two
+// weight matrices is not a bf16 number, and one rounding of V_r would shift every row's
+// pre-activation the same way (an error that the weight gradients, sums over all rows, do not
+// average out), so V_r is kept as an unevaluated pair V_r = V_hi + V_lo of bf16 matrices (V_hi =
+// bf16(V_r), V_lo = bf16(V_r - V_hi); about 16 significant bits) and every product with it is two
+// MMAs into the same fp32 accumulator.
 //
 // Forward, one CTA per 128 destination rows of type t:
 //   U = sum_{r -> t} M_r V_r      A = relation means (TMA, 128 x 64 tiles), B = V_r^T chunks
+//                                 (the hi and lo halves of a chunk in one pipeline stage)
 //   epilogue: U += b, stored; Y = act(U) + H_in; H_out = LayerNorm(Y); row statistics saved.
 // Backward:
 //   ln_act_bwd   (warp per row)  dY = LayerNorm backward, dU = dY act'(U); column partials of the
 //                                bias / gain / shift gradients
-//   proj_bwd_tc  (CTA per 128 rows)  dMs_r = (dU V_r^T) / deg_r   (A = dU by TMA, B = V_r chunks)
+//   proj_bwd_tc  (CTA per 128 rows)  dMs_r = (dU V_r^T) / deg_r   (A = dU by TMA, B = V_r chunks,
+//                                hi and lo halves)
 //   weight gradients: G_r = M_r^T dU (split-K GEMM, MN-major TMA operands), then
 //                     dW_r = G_r W_agg^T and dW_agg[t] = sum_{r -> t} W_r^T G_r (wgrad_finish).
 //
@@ -39,15 +46,16 @@ constexpr int kATile = kTileRows * 128;  // 128 rows x 64 bf16
 // overlap the loads and MMAs of the next.
 template <int D>
 struct FwdCfg {
-  static constexpr int kStages = D == 256 ? 3 : 4;
-  static constexpr int kB = D * 128;  // D rows x 64 bf16
-  static constexpr int kStage = kATile + kB;
+  static constexpr int kStages = D == 256 ? 2 : (D == 128 ? 3 : 4);
+  static constexpr int kB = D * 128;  // D rows x 64 bf16 (one half of the weight pair)
+  static constexpr int kStage = kATile + 2 * kB;  // A | B_hi | B_lo
   // The H_in tile (residual) is fetched by TMA, double-buffered, where shared memory allows it; at
   // D = 256 the epilogue reads H_in from global memory.
   static constexpr bool kHTile = D <= 128;
   static constexpr int kH = kHTile ? kTileRows * D * 2 : 0;
   static constexpr int kParams = 3 * D * 4;  // bias, gamma, beta in fp32
   static constexpr int kSmem = kStages * kStage + 2 * kH + kParams + 512 + 1024;
+  static_assert(kSmem <= 227 * 1024, "shared memory of proj_fwd_tc");
   static constexpr int kAccCols = D < 32 ? 32 : D;
   static constexpr int kTmemCols = 2 * kAccCols;
   static constexpr int kThreads = 192;
@@ -143,9 +151,10 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
           if (!ok) break;
           uint8_t* A = stage + s * C::kStage;
           const int r = j / KC, kc = j % KC;
-          mbar_expect_tx(&full[s], kATile + C::kB);
+          mbar_expect_tx(&full[s], C::kStage);
           tma_load_2d(A, &tm_M, kc * 64, (int)(a.mrow0[r] + m0), &full[s]);
-          tma_load_2d(A + kATile, &tm_Vt, kc * 64, a.rel[r] * D, &full[s]);
+          tma_load_2d(A + kATile, &tm_Vt, kc * 64, 2 * a.rel[r] * D, &full[s]);           // hi
+          tma_load_2d(A + kATile + C::kB, &tm_Vt, kc * 64, (2 * a.rel[r] + 1) * D, &full[s]);  // lo
         }
       }
       if (!ok) atomicOr(a.status, kErrTimeout);
@@ -171,9 +180,11 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
           fence_after_sync();
           const uint32_t A = smem_u32(stage + s * C::kStage);
 #pragma unroll
-          for (int ks = 0; ks < 4; ++ks)
-            mma_bf16(acc, desc_sw128(A + ks * 32, 16, 1024), desc_sw128(A + kATile + ks * 32, 16, 1024), idesc,
-                     (j > 0 || ks > 0) ? 1u : 0u);
+          for (int ks = 0; ks < 4; ++ks) {
+            const uint64_t ad = desc_sw128(A + ks * 32, 16, 1024);
+            mma_bf16(acc, ad, desc_sw128(A + kATile + ks * 32, 16, 1024), idesc, (j > 0 || ks > 0) ? 1u : 0u);
+            mma_bf16(acc, ad, desc_sw128(A + kATile + C::kB + ks * 32, 16, 1024), idesc, 1u);
+          }
           mma_commit(&empty[s]);
         }
         mma_commit(&acc_full[b]);
@@ -327,7 +338,8 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
 }
 
 // Fused weights V_r = W_r W_agg[t_r] accumulated in fp64 (exact for bf16 factors of these sizes),
-// rounded once to bf16; both V_r and its transpose are written.  Grid (D/32, D/32, relations): a
+// written as the pair V_hi = bf16(V_r), V_lo = bf16(V_r - V_hi): V holds [relation][hi, lo][D][D]
+// and Vt the transposes in the same order.  Grid (D/32, D/32, relations): a
 // block computes a 32 x 32 tile from 32-wide K slices staged in shared memory; thread (ty, tx)
 // owns rows ty, ty + 8, ty + 16, ty + 24 of column tx.
 template <int D>
@@ -361,9 +373,13 @@ __global__ void __launch_bounds__(256) fuse_weights(const __nv_bfloat16* __restr
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     const int i = i0 + ty + 8 * q, j = j0 + tx;
-    const __nv_bfloat16 v = __float2bfloat16_rn(__double2float_rn(acc[q]));
-    V[(int64_t)r * D * D + (int64_t)i * D + j] = v;
-    Vt[(int64_t)r * D * D + (int64_t)j * D + i] = v;
+    const __nv_bfloat16 hi = __float2bfloat16_rn(__double2float_rn(acc[q]));
+    const __nv_bfloat16 lo = __float2bfloat16_rn(__double2float_rn(acc[q] - (double)__bfloat162float(hi)));
+    const int64_t base = (int64_t)2 * r * D * D;
+    V[base + (int64_t)i * D + j] = hi;
+    V[base + (int64_t)D * D + (int64_t)i * D + j] = lo;
+    Vt[base + (int64_t)j * D + i] = hi;
+    Vt[base + (int64_t)D * D + (int64_t)j * D + i] = lo;
   }
 }
 
@@ -543,9 +559,11 @@ __global__ void __launch_bounds__(256) ln_act_bwd(TcBwdArgs a) {
 // ---------------------------------------------------------------------------------------------
 template <int D>
 struct BwdCfg {
-  static constexpr int kStages = D == 256 ? 2 : 4;     // ring of V_r chunks (D rows x 64 columns)
-  static constexpr int kB = D * 128;
-  static constexpr int kT = kTileRows * D * 2;          // dU operand tile (KC x 16 KB), double-buffered
+  static constexpr int kStages = D == 64 ? 4 : (D == 128 ? 3 : 2);  // ring of V_r chunks (hi and lo)
+  static constexpr int kB = D * 128;                    // D rows x 64 columns, one half of the pair
+  static constexpr int kBStage = 2 * kB;
+  static constexpr int kT = kTileRows * D * 2;          // dU operand tile (KC x 16 KB)
+  static constexpr int kABuf = D == 256 ? 1 : 2;        // dU tiles in flight (shared memory allowing)
   static constexpr int kAcc = D < 32 ? 32 : D;
   static constexpr int kNumAcc = 512 / kAcc < 4 ? 512 / kAcc : 4;  // ring of TMEM accumulators
   static constexpr int kTmemCols = kNumAcc * kAcc;
@@ -554,8 +572,9 @@ struct BwdCfg {
   // TMA, where shared memory allows it; at D = 256 each thread stores its own row.
   static constexpr bool kTmaOut = D <= 128;
   static constexpr int kOut = kTmaOut ? kTileRows * D * 2 : 0;
-  static constexpr int kSmem = kStages * kB + 2 * kT + kEpiGroups * kOut + 512 + 1024;
+  static constexpr int kSmem = kStages * kBStage + kABuf * kT + kEpiGroups * kOut + 512 + 1024;
   static constexpr int kThreads = 64 + kEpiGroups * 128;
+  static_assert(kSmem <= 227 * 1024, "shared memory of proj_bwd_tc");
 };
 
 // one tensor map per relation over its dMs rows [mrow0[r], mrow0[r] + n): a partial last tile is
@@ -578,13 +597,14 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
   constexpr int KC = D / 64;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  uint8_t* bstage = smem;                 // S x B chunk
-  uint8_t* tiles = smem + S * C::kB;      // 2 x (KC x 16 KB)
-  uint8_t* outs = tiles + 2 * C::kT;      // kEpiGroups x (KC x 16 KB) output staging
+  constexpr int NA = C::kABuf;
+  uint8_t* bstage = smem;                 // S x (B_hi | B_lo) chunk
+  uint8_t* tiles = smem + S * C::kBStage;  // NA x (KC x 16 KB)
+  uint8_t* outs = tiles + NA * C::kT;     // kEpiGroups x (KC x 16 KB) output staging
   uint64_t* b_full = reinterpret_cast<uint64_t*>(outs + C::kEpiGroups * C::kOut);
   uint64_t* b_empty = b_full + S;
-  uint64_t* a_full = b_empty + S;       // [2] dU tile loaded
-  uint64_t* a_empty = a_full + 2;       // [2] every product of the tile done
+  uint64_t* a_full = b_empty + S;       // [NA] dU tile loaded
+  uint64_t* a_empty = a_full + 2;       // [NA] every product of the tile done
   uint64_t* acc_full = a_empty + 2;     // [NB]
   uint64_t* acc_empty = acc_full + NB;  // [NB]
   uint32_t* tslot = reinterpret_cast<uint32_t*>(acc_empty + NB);
@@ -596,7 +616,7 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
       mbar_init(&b_full[s], 1);
       mbar_init(&b_empty[s], 1);
     }
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < NA; ++b) {
       mbar_init(&a_full[b], 1);
       mbar_init(&a_empty[b], 1);
     }
@@ -620,8 +640,8 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
       uint32_t g = 0;
       int it = 0;
       for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
-        const int ab = it & 1;
-        if (it >= 2) ok = mbar_wait(&a_empty[ab], ((it >> 1) - 1) & 1);
+        const int ab = it % NA;
+        if (it >= NA) ok = mbar_wait(&a_empty[ab], ((it / NA) - 1) & 1);
         if (!ok) break;
         mbar_expect_tx(&a_full[ab], C::kT);
         for (int kc = 0; kc < KC; ++kc)
@@ -630,8 +650,10 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
           const uint32_t s = g % S;
           if (g >= (uint32_t)S) ok = mbar_wait(&b_empty[s], ((g / S) - 1) & 1);
           if (!ok) break;
-          mbar_expect_tx(&b_full[s], C::kB);
-          tma_load_2d(bstage + s * C::kB, &tm_V, (j % KC) * 64, a.rel[j / KC] * D, &b_full[s]);
+          mbar_expect_tx(&b_full[s], C::kBStage);
+          tma_load_2d(bstage + s * C::kBStage, &tm_V, (j % KC) * 64, 2 * a.rel[j / KC] * D, &b_full[s]);
+          tma_load_2d(bstage + s * C::kBStage + C::kB, &tm_V, (j % KC) * 64, (2 * a.rel[j / KC] + 1) * D,
+                      &b_full[s]);
         }
       }
       if (!ok) atomicOr(a.status, kErrTimeout);
@@ -644,8 +666,8 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
       uint32_t g = 0, jb = 0;
       int it = 0;
       for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
-        const int ab = it & 1;
-        ok = mbar_wait(&a_full[ab], (it >> 1) & 1);
+        const int ab = it % NA;
+        ok = mbar_wait(&a_full[ab], (it / NA) & 1);
         if (!ok) break;
         const uint32_t A0 = smem_u32(tiles + ab * C::kT);
         for (int r = 0; r < a.nrel && ok; ++r, ++jb) {
@@ -660,11 +682,13 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
             if (!ok) break;
             fence_after_sync();
             const uint32_t A = A0 + kc * kATile;
-            const uint32_t B = smem_u32(bstage + s * C::kB);
+            const uint32_t B = smem_u32(bstage + s * C::kBStage);
 #pragma unroll
-            for (int ks = 0; ks < 4; ++ks)
-              mma_bf16(acc, desc_sw128(A + ks * 32, 16, 1024), desc_sw128(B + ks * 32, 16, 1024), idesc,
-                       (kc > 0 || ks > 0) ? 1u : 0u);
+            for (int ks = 0; ks < 4; ++ks) {
+              const uint64_t ad = desc_sw128(A + ks * 32, 16, 1024);
+              mma_bf16(acc, ad, desc_sw128(B + ks * 32, 16, 1024), idesc, (kc > 0 || ks > 0) ? 1u : 0u);
+              mma_bf16(acc, ad, desc_sw128(B + C::kB + ks * 32, 16, 1024), idesc, 1u);
+            }
             mma_commit(&b_empty[s]);
           }
           mma_commit(&acc_full[k]);
@@ -896,7 +920,7 @@ static hg_status tc_fwd_t(const TcFwdArgs& a, const void* M, int64_t m_rows, con
   HG_TRY(smem_attr_once<D>());
   CUtensorMap tm_M, tm_V, tm_H;
   HG_TRY(make_tmap_bf16(&tm_M, M, (uint64_t)std::max<int64_t>(m_rows, 1), D, kTileRows));
-  HG_TRY(make_tmap_bf16(&tm_V, Vt, (uint64_t)num_rels * D, D, D));
+  HG_TRY(make_tmap_bf16(&tm_V, Vt, (uint64_t)2 * num_rels * D, D, D));
   if (FwdCfg<D>::kHTile) {
     HG_TRY(make_tmap_bf16(&tm_H, a.H_in + a.off * D, (uint64_t)a.n, D, kTileRows));
   } else {
@@ -932,7 +956,7 @@ static hg_status tc_bwd_t(const TcBwdArgs& a, const void* V, int num_rels, cudaS
   if (a.nrel == 0) return HG_OK;
   CUtensorMap tm_dU, tm_V;
   HG_TRY(make_tmap_bf16(&tm_dU, a.dU + a.off * D, (uint64_t)a.n, D, kTileRows));
-  HG_TRY(make_tmap_bf16(&tm_V, V, (uint64_t)num_rels * D, D, D));
+  HG_TRY(make_tmap_bf16(&tm_V, V, (uint64_t)2 * num_rels * D, D, D));
   int sms = 0, dev = 0;
   HG_CUDA(cudaGetDevice(&dev));
   HG_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));

@@ -1,5 +1,8 @@
 // Dense row products on the tensor cores (bf16 storage, fp32 accumulation):
-//   out[r][ocol0 + c] (=, or +=) sum_k A[r][k] B[k][c] (+ bias[c]),   rows r < n, c < D, k < D.
+//   out[r][ocol0 + c] (=, or +=) scale * sum_k A[r][k] B[k][c] (+ bias[c]),   rows r < n, c < D,
+//   k < D, with scale = scale_mul * (*scale_ptr) (scale_ptr a device fp32 scalar, or null for 1):
+//   a scalar factor of a weight is applied here in fp32 instead of being folded into B, where the
+//   product would have to be rounded to bf16.
 // One CTA per 128 rows: the A tile arrives by TMA as a K-major operand, B (D x D, row-major, as
 // stored) by TMA as an MN-major operand, one tcgen05 chain puts the 128 x D product in tensor
 // memory, and sixteen warps (four per 32-lane quarter, each a column group) add the bias or the
@@ -37,6 +40,8 @@ struct GCfg {
 
 struct GArgs {
   int64_t n;
+  const float* scale_ptr;
+  float scale_mul;
   const __nv_bfloat16* bias;
   __nv_bfloat16* out;
   int64_t ldo;
@@ -101,6 +106,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int64_t r = r0 + q * 32 + lane;
   const bool live = ok && r < p.n;
   const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + cg * CW;
+  const float sc = p.scale_mul * (p.scale_ptr ? *p.scale_ptr : 1.f);
 #pragma unroll
   for (int c0 = 0; c0 < CW; c0 += 8) {
     const int c = cg * CW + c0;
@@ -116,7 +122,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int e = 0; e < 8; ++e) x[e] = 0.f;
       }
 #pragma unroll
-      for (int e = 0; e < 8; ++e) x[e] += v[e] + bf[c + e];
+      for (int e = 0; e < 8; ++e) x[e] += fmaf(sc, v[e], bf[c + e]);
       st16(o, pack(x, __nv_bfloat16()));
     }
   }
@@ -133,7 +139,7 @@ inline size_t gemm_smem(size_t need, int tcols) {
 
 template <int D>
 hg_status rows_gemm_t(const void* A, int64_t n, const void* B, const void* bias, void* out, int64_t ldo, int ocol0,
-                      int accumulate, cudaStream_t s) {
+                      int accumulate, const float* scale_ptr, float scale_mul, cudaStream_t s) {
   static bool done = false;
   if (!done) {
     HG_CUDA(cudaFuncSetAttribute(rows_gemm_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448));
@@ -142,7 +148,8 @@ hg_status rows_gemm_t(const void* A, int64_t n, const void* B, const void* bias,
   CUtensorMap tm_A, tm_B;
   HG_TRY(make_tmap_bf16(&tm_A, A, (uint64_t)n, D, kRows));
   HG_TRY(make_tmap_bf16(&tm_B, B, D, D, D));
-  GArgs g{n, (const __nv_bfloat16*)bias, (__nv_bfloat16*)out, ldo, ocol0, accumulate, device_status_ptr()};
+  GArgs g{n, scale_ptr, scale_mul, (const __nv_bfloat16*)bias, (__nv_bfloat16*)out, ldo, ocol0, accumulate,
+          device_status_ptr()};
   return launch("rows_gemm_tc", rows_gemm_tc_kernel<D>, dim3((unsigned)ceil_div(n, kRows)), dim3(kThreads),
                 gemm_smem(GCfg<D>::kNeed, D), s, tm_A, tm_B, g);
 }
@@ -150,15 +157,15 @@ hg_status rows_gemm_t(const void* A, int64_t n, const void* B, const void* bias,
 }  // namespace
 
 hg_status rows_gemm_tc(int d, const void* A, int64_t n, const void* B, const void* bias, void* out, int64_t ldo,
-                       int ocol0, int accumulate, cudaStream_t s) {
+                       int ocol0, int accumulate, const float* scale_ptr, float scale_mul, cudaStream_t s) {
   if (n <= 0) return HG_OK;
   if (((uintptr_t)A & 15) || ((uintptr_t)B & 15) || ((uintptr_t)out & 15) || (ldo % 8) || (ocol0 % 8)) {
     set_error("rows_gemm_tc: operands must be 16-byte aligned");
     return HG_ERR_INVALID_ARG;
   }
-  if (d == 64) return rows_gemm_t<64>(A, n, B, bias, out, ldo, ocol0, accumulate, s);
-  if (d == 128) return rows_gemm_t<128>(A, n, B, bias, out, ldo, ocol0, accumulate, s);
-  if (d == 256) return rows_gemm_t<256>(A, n, B, bias, out, ldo, ocol0, accumulate, s);
+  if (d == 64) return rows_gemm_t<64>(A, n, B, bias, out, ldo, ocol0, accumulate, scale_ptr, scale_mul, s);
+  if (d == 128) return rows_gemm_t<128>(A, n, B, bias, out, ldo, ocol0, accumulate, scale_ptr, scale_mul, s);
+  if (d == 256) return rows_gemm_t<256>(A, n, B, bias, out, ldo, ocol0, accumulate, scale_ptr, scale_mul, s);
   set_error("rows_gemm_tc: unsupported d=%d", d);
   return HG_ERR_UNSUPPORTED;
 }

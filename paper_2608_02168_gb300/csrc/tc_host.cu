@@ -2,9 +2,26 @@
 // link against libcuda), and the library's device status word.
 #include <cudaTypedefs.h>
 
+#include <atomic>
+
 #include "tc_util.cuh"
 
 namespace hg {
+
+// The device this process's library state belongs to (-1 until the first call binds it).
+static std::atomic<int> g_bound_device{-1};
+
+hg_status device_guard() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return HG_OK;  // no usable device: the call's own CUDA calls report it
+  }
+  int bound = -1;
+  if (g_bound_device.compare_exchange_strong(bound, dev) || bound == dev) return HG_OK;
+  set_error("this library is bound to device %d (its one-time set-up ran there); device %d is current", bound, dev);
+  return HG_ERR_UNSUPPORTED;
+}
 
 __device__ int g_device_status = 0;
 
@@ -56,3 +73,12 @@ int* device_status_ptr() {
 }
 
 }  // namespace hg
+
+extern "C" hg_status hg_bind_device(int32_t device) {
+  hg::clear_error();
+  HG_REQUIRE(device >= 0, "device must be >= 0");
+  int bound = -1;
+  if (hg::g_bound_device.compare_exchange_strong(bound, device) || bound == device) return HG_OK;
+  hg::set_error("this library is already bound to device %d", bound);
+  return HG_ERR_UNSUPPORTED;
+}

@@ -472,6 +472,7 @@ extern "C" hg_status hg_temporal_workspace_size(int64_t n, int32_t d, int32_t w,
 extern "C" hg_status hg_temporal_fwd(const hg_temporal_params* params, const void* X, const void* C, int64_t n,
                                     void* H_out, void* saved, void* scratch, hg_stream stream) {
   clear_error();
+  HG_TRY(device_guard());
   HG_TRY(check_temporal(params, n));
   HG_REQUIRE(saved && scratch, "saved and scratch must be non-null");
   HG_REQUIRE(((uintptr_t)saved & 255) == 0 && ((uintptr_t)scratch & 255) == 0, "buffers must be 256-byte aligned");
@@ -491,6 +492,7 @@ extern "C" hg_status hg_temporal_bwd(const hg_temporal_params* params, const voi
                                     const void* saved, const void* dH_out, void* dX, const hg_temporal_grads* grads,
                                     void* scratch, hg_stream stream) {
   clear_error();
+  HG_TRY(device_guard());
   HG_TRY(check_temporal(params, n));
   HG_REQUIRE(saved && scratch && grads, "saved, scratch and grads must be non-null");
   HG_REQUIRE(grads->dWa && grads->dr && grads->dW_i && grads->dW_h && grads->db_i && grads->db_h,

@@ -81,6 +81,7 @@ EXPORTS = {
     "hg_last_error": (c_char_p, []),
     "hg_abi_version": (c_int32, []),
     "hg_device_status": (c_int32, [POINTER(c_int32)]),
+    "hg_bind_device": (c_int32, [c_int32]),
     "hg_graph_workspace_size": (c_int32, [c_int64, POINTER(c_int64), c_int32, POINTER(hg_rel_desc), c_int32,
                                           POINTER(c_size_t)]),
     "hg_build_csr": (c_int32, [c_void_p, c_void_p, c_void_p, c_int64, POINTER(c_int64), c_int32,

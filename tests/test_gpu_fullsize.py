@@ -9,7 +9,7 @@ import torch
 
 import hgsynth
 import oracle
-from tests.gpu_util import TOL, dev, grad_bufs, host, layer_params, lib, need_gpu, relerr, tdtype
+from tests.gpu_util import BF16_RELU_MARGIN, TOL, dev, grad_bufs, host, layer_params, lib, need_gpu, relerr, tdtype
 
 pytestmark = pytest.mark.gpu
 
@@ -19,8 +19,9 @@ def full(request):
     need_gpu()
     hg = lib()
     sp = hgsynth.spec(request.param)
-    # biases of +-3 keep the ReLU decisions unambiguous (see test_gpu_layer)
-    w = hgsynth.make_workload(sp, random_affine=True, with_ids=True, bias_margin=3.0)
+    # wide bias margins keep the ReLU decisions unambiguous (see test_gpu_layer); every value check
+    # below is against the plain fp64 definition
+    w = hgsynth.make_workload(sp, random_affine=True, with_ids=True, bias_margin=BF16_RELU_MARGIN)
     g = w.graph
     G = hg.hg_build_csr(dev(g["src"]), dev(g["dst"]), dev(g["rel"]), g["type_offsets"], g["rels"])
     assert hg.hg_graph_check(G) == 0
@@ -84,8 +85,7 @@ def test_full_layer_sampled_rows(full):
     out = torch.empty_like(X)
     hg.hg_layer_fwd(G, P, X, out, saved, scratch)
     rows = sample_rows(w, 3000, 1)
-    ref, _ = oracle.layer_forward_rows(g["src"], g["dst"], g["rel"], g["type_offsets"], g["rels"], p, w.X, rows,
-                                       store="bf16")
+    ref, _ = oracle.layer_forward_rows(g["src"], g["dst"], g["rel"], g["type_offsets"], g["rels"], p, w.X, rows)
     assert relerr(host(out[torch.from_numpy(rows).cuda()]), ref) <= TOL[sp.dtype]
     # backward with an upstream gradient supported on a row sample S
     S = sample_rows(w, 2000, 2)
@@ -100,7 +100,7 @@ def test_full_layer_sampled_rows(full):
     q = np.unique(np.concatenate([S[:500], rng.choice(into_S, min(1500, len(into_S)), replace=False),
                                   rng.choice(int(g["type_offsets"][-1]), 500, replace=False)]))
     dq, gref = oracle.layer_backward_rows(g["src"], g["dst"], g["rel"], g["type_offsets"], g["rels"], p, w.X, S,
-                                          w.dH_top[S], q, store="bf16")
+                                          w.dH_top[S], q)
     tol = TOL[sp.dtype]
     assert relerr(host(dH_in[torch.from_numpy(q).cuda()]), dq) <= tol
     for k, v in gref.items():
@@ -202,7 +202,7 @@ def test_full_size_temporal():
     dX = torch.empty_like(out)
     hg.hg_temporal_bwd(prm, Xd, Cd, saved, dev(dOut, td), dX, grads, scratch)
     torch.cuda.synchronize()
-    ref = OT.temporal_backward(X[rows], C[:, rows], p, dOut[rows], store="bf16")
+    ref = OT.temporal_backward(X[rows], C[:, rows], p, dOut[rows])
     tol = TOL["bf16"]
     assert relerr(host(out)[rows], ref["out"]) <= tol
     assert relerr(host(dX)[rows], ref["dX"]) <= tol
@@ -238,6 +238,6 @@ def test_full_size_attention_layer_sampled_targets():
     nodes = np.unique(np.concatenate([rows, g["src"][keep]]))
     # the subgraph keeps global ids (rows outside it have no in-edges and are not compared)
     ref, _ = OH.hgt_forward(g["src"][keep], g["dst"][keep], g["rel"][keep], g["type_offsets"], g["rels"], p,
-                            np.where(np.isin(np.arange(sp.num_nodes), nodes)[:, None], w.X, 0.0), 4, store="bf16")
+                            np.where(np.isin(np.arange(sp.num_nodes), nodes)[:, None], w.X, 0.0), 4)
     assert relerr(host(out)[rows], ref[rows]) <= TOL["bf16"]
     assert hg.hg_device_status() == 0

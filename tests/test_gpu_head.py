@@ -70,9 +70,9 @@ def head_gpu(hg, H, Hr, ia, ib, lab, y, p, dt, dloss=1.0, cca=None, lam=0.1, n_r
 
 
 def check(got, H, Hr, ia, ib, lab, y, p, dt, dloss=1.0, cca=None, lam=0.1, ltol=None):
-    store = "bf16" if dt == "bf16" else "f64"
-    ref = OH.head_loss(H, ia, Hr, ib, lab, y, p, cca_loss=cca, lambda_cca=lam, store=store)
-    g = OH.head_backward(H, ia, Hr, ib, lab, y, p, dloss=dloss, store=store)
+    # the plain fp64 definition of Eq. 18-20 for both storage types
+    ref = OH.head_loss(H, ia, Hr, ib, lab, y, p, cca_loss=cca, lambda_cca=lam)
+    g = OH.head_backward(H, ia, Hr, ib, lab, y, p, dloss=dloss)
     ltol = ltol or (1e-5 if dt == "f32" else 1e-4)
     assert abs(got["loss"][1] - ref["bce"]) <= ltol * max(abs(ref["bce"]), 1e-6), (got["loss"], ref["bce"])
     assert abs(got["loss"][0] - ref["total"]) <= ltol * max(abs(ref["total"]), 1e-6), (got["loss"], ref["total"])
@@ -104,8 +104,7 @@ def test_head_fractional_labels_dloss_and_accumulation():
     H, Hr, ia, ib, lab, y, p = problem(5, 4000, 128, 1500, 900, "bf16", frac_y=True)
     got = head_gpu(hg, H, Hr, ia, ib, lab, y, p, "bf16", dloss=0.37, base=1.0)
     # accumulated onto N(0,1) bf16 values: the increment carries the rounding of the sum
-    store = "bf16"
-    g = OH.head_backward(H, ia, Hr, ib, lab, y, p, dloss=0.37, store=store)
+    g = OH.head_backward(H, ia, Hr, ib, lab, y, p, dloss=0.37)
     for k in ("dW1", "db1", "dw2", "db2"):
         assert relerr(got[k].reshape(g[k].shape), g[k]) <= TOL["bf16"], k
     rows = np.unique(np.concatenate([lab]))

@@ -54,12 +54,11 @@ def test_hgt_matches_oracle(case, ln):
     p = hgsynth.make_hgt_params(sp, heads, bias_margin=3.0 if sp.dtype == "bf16" else None)
     g = w.graph
     out, dH, gr = run_gpu(hg, w, p, heads, ln, w.dH_top)
-    store = "bf16" if sp.dtype == "bf16" else "f64"
     args = (g["src"], g["dst"], g["rel"], g["type_offsets"], g["rels"], p, w.X)
-    ref, _ = OH.hgt_forward(*args, heads, layernorm=ln, store=store)
+    ref, _ = OH.hgt_forward(*args, heads, layernorm=ln)  # the plain fp64 definition (Eq. 6-11)
     tol = TOL[sp.dtype]
     assert relerr(out, ref) <= tol, ("H_out", relerr(out, ref))
-    dref, gref = OH.hgt_backward(*args, w.dH_top, heads, layernorm=ln, store=store)
+    dref, gref = OH.hgt_backward(*args, w.dH_top, heads, layernorm=ln)
     assert relerr(dH, dref) <= tol, ("dH_in", relerr(dH, dref))
     for k in KEYS:
         if not ln and k in ("ln_gamma", "ln_beta"):

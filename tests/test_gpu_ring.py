@@ -7,7 +7,7 @@ import torch
 
 import hgsynth
 import oracle
-from tests.gpu_util import TOL, dev, host, lib, need_gpu, relerr, tdtype
+from tests.gpu_util import BF16_RELU_MARGIN, TOL, dev, host, lib, need_gpu, relerr, tdtype
 
 pytestmark = pytest.mark.gpu
 
@@ -17,7 +17,8 @@ def test_ring_sequence_matches_oracle():
     lib()
     from paper_2608_02168_gb300.step import Ring
     sp = hgsynth.spec("ring16-2m", n_user=9_000, n_risk=1_000, num_edges=150_000, n_overlap=2_000, num_subgraphs=4)
-    params = [hgsynth.make_layer_params(sp, l, random_affine=True, bias_margin=3.0) for l in range(sp.layers)]
+    params = [hgsynth.make_layer_params(sp, l, random_affine=True, bias_margin=BF16_RELU_MARGIN)
+              for l in range(sp.layers)]
     td = tdtype(sp.dtype)
     ring = None
     prev_H, prev_gid = None, None
@@ -30,7 +31,7 @@ def test_ring_sequence_matches_oracle():
                          dev(part.gid))
         torch.cuda.synchronize()
         vb = None if prev_H is None else {"H_b": prev_H, "gid_a": part.gid, "gid_b": prev_gid}
-        ref = oracle.step(g, part.X, params, part.dH_top, vb, store="bf16")
+        ref = oracle.step(g, part.X, params, part.dH_top, vb)  # the plain fp64 definition
         p = ring.path
         assert relerr(host(bank), ref["H"][-1]) <= TOL[sp.dtype], k
         if k > 0:

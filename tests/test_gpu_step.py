@@ -6,7 +6,7 @@ import torch
 
 import hgsynth
 import oracle
-from tests.gpu_util import TOL, dev, host, lib, need_gpu, relerr, tdtype
+from tests.gpu_util import BF16_RELU_MARGIN, TOL, dev, host, lib, need_gpu, relerr, tdtype
 
 pytestmark = pytest.mark.gpu
 
@@ -43,17 +43,20 @@ def test_step_matches_oracle(variant, with_head):
         sp = hgsynth.spec("tiny-10k")
     else:
         sp = hgsynth.spec("sub-1m", n_user=18_000, n_risk=2_000, num_edges=300_000, n_overlap=2_609)
-    # bf16: biases of +-3 keep the ReLU decisions unambiguous (see test_gpu_layer)
-    w = hgsynth.make_workload(sp, random_affine=True, bias_margin=3.0 if sp.dtype == "bf16" else None)
+    # bf16: wide bias margins keep the ReLU decisions of the layers and the head unambiguous (see
+    # test_gpu_layer); the comparison is with the plain fp64 definition
+    bf = sp.dtype == "bf16"
+    w = hgsynth.make_workload(sp, random_affine=True, bias_margin=BF16_RELU_MARGIN if bf else None)
     head = None
     if with_head:
         lab, y = hgsynth.make_labels(sp, positive_rate=0.3)
-        head = {"params": hgsynth.make_head_params(sp, random_bias=True), "lab_idx": lab, "lab_y": y}
+        head = {"params": hgsynth.make_head_params(sp, random_bias=True, bias_margin=BF16_RELU_MARGIN if bf else None),
+                "lab_idx": lab, "lab_y": y}
     path = make_path(w, head)
     run(path, w, head)
     vb = {"idx": w.overlap_local, "X_b": w.X_b} if sp.view_b == "perturbed" else \
         {"H_b": w.H_b, "gid_a": w.gid_a, "gid_b": w.gid_b}
-    ref = oracle.step(w.graph, w.X, w.params, w.dH_top, vb, store="bf16" if sp.dtype == "bf16" else "f64", head=head)
+    ref = oracle.step(w.graph, w.X, w.params, w.dH_top, vb, head=head)
     tol = TOL[sp.dtype]
     assert relerr(host(path.loss), np.array(ref["loss"])) <= (1e-4 if sp.dtype == "f32" else 2e-2)
     if with_head:

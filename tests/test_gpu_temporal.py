@@ -54,8 +54,7 @@ def temporal_gpu(hg, X, C, p, dOut, dt, w):
 
 
 def check(X, C, p, dOut, dt, got_out, got_dX, got_g):
-    store = "bf16" if dt == "bf16" else "f64"
-    ref = OT.temporal_backward(X, C, p, dOut, store=store)
+    ref = OT.temporal_backward(X, C, p, dOut)  # the plain fp64 definition (Eq. 12-13)
     tol = TOL[dt]
     assert relerr(got_out, ref["out"]) <= tol, ("out", relerr(got_out, ref["out"]))
     assert relerr(got_dX, ref["dX"]) <= tol, ("dX", relerr(got_dX, ref["dX"]))

@@ -150,3 +150,15 @@ def test_binding_rejects_host_tensors_before_any_call(hg):
     with pytest.raises(ValueError, match="device memory"):
         hg.hg_overlap_intersect(a, a, out, out, torch.empty(1, dtype=torch.int64), torch.empty(64, dtype=torch.uint8))
     assert hg._ptr(None) is None
+
+
+def test_device_binding_is_first_come_and_exclusive(hg):
+    """hg_bind_device makes no CUDA call: it is checked here without a GPU, in a fresh process whose
+    library state is unbound."""
+    import subprocess
+    import sys
+    child = (f"import ctypes; so = ctypes.CDLL({hg.lib()._name!r}); "
+             "assert so.hg_bind_device(3) == 0; assert so.hg_bind_device(3) == 0; "
+             "assert so.hg_bind_device(1) == 2; assert so.hg_bind_device(-1) == 1; print('ok')")
+    r = subprocess.run([sys.executable, "-c", child], capture_output=True, text=True, timeout=120)
+    assert r.returncode == 0 and r.stdout.strip() == "ok", r.stdout + r.stderr

@@ -195,6 +195,6 @@ def test_bf16_storage_points():
     g, H, p = graph(11, heads=2)
     out_b, cb = OH.hgt_forward(*g, p, H, 2, store="bf16")
     out_f, cf = OH.hgt_forward(*g, p, H, 2)
-    for k in ("K", "V", "Qp", "Ssum", "U"):
+    for k in ("K", "V", "Q", "Qp", "Ssum", "U"):
         assert np.array_equal(cb[k], bf16_round(cb[k]).astype(np.float64)), k
     assert np.abs(out_b - out_f).max() <= 2e-2 * np.abs(out_f).max()
