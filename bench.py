@@ -1,13 +1,18 @@
 #!/usr/bin/env python
 """Benchmark of the hot path: GNN layer forward+backward edges/s on one GB300.
 
-One step = one pass of the whole hot path over one overlapping subgraph (relation-typed CSR/CSC
-build, L layers forward, overlap intersection, alignment loss and gradient, L layers backward,
-dL/dX included).  value = L * E * steps * ranks / (max over ranks of the device time of the timed
-steps).  Inputs are seeded synthetic graphs of the named workload (default: 1M nodes, 20M edges,
-bf16 d=128, 2 layers), resident in HBM before timing; they are larger than L2, which is not
-flushed.  Multi-GPU (torchrun): every rank runs its own subgraph (weak scaling), no collective on
-the data path.  `--impl reference` times the CPU oracle on a bounded sample of the same workload.
+One step = one pass of the whole hot path over one overlapping subgraph: the relation-typed CSR /
+CSC build, L layers forward, the overlap intersection, the alignment loss, the head's loss and
+gradient (joint objective of Eq. 20), the alignment gradient and L layers backward, dL/dX included.
+value = L * E * steps * ranks / (max over ranks of the device time of the timed steps).  The
+default workload is the largest single-GPU one: 10M nodes, 200M edges (Zipf s = 1.2, top-100 hubs
+of >= 500k out-edges), bf16 d = 128, 3 layers.  Inputs are seeded synthetic instances of the
+workload recipe drawn on the GPU (hgsynth.device), resident in HBM before timing and larger than
+L2, which is not flushed.  Beside the headline the line reports the L-layer stack alone (forward +
+backward, the metric's own definition), the CSR build, the other workloads (tiny-10k, sub-1m,
+tail-5m) and one full pass over the sixteen-subgraph ring.  Multi-GPU (torchrun): every rank runs
+its own subgraph (weak scaling), no collective on the data path.  `--impl reference` times the CPU
+oracle on a bounded sample of the same workload.
 
 Prints one JSON line (rank 0).
 """
@@ -30,11 +35,13 @@ import hgsynth  # noqa: E402
 
 METRIC = "GNN layer fwd+bwd edges/sec on 1 GB300; achieved HBM GB/s vs roofline"
 UNIT = "edges/s"
-ORACLE_SCALE = 40        # the CPU baseline runs the oracle on a 1/40-size instance of the workload
+SAMPLE_EDGES = 150_000   # the CPU oracle runs on instances of about this many edges (same recipe)
 BUILD_K, BUILD_THETA, BUILD_BUDGET = 8, 2, 0.15  # overlapping-subgraph construction: parts, h-index bound, M / N
-REFERENCE_SCALE = 100    # each reference-arm step runs the oracle on a 1/100-size instance
 FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "sm_max_mhz": 2070.0}
 NOMINAL_HBM_GBS = 7900.0  # GB300 HBM3e data-sheet bandwidth, reported beside the measured copy peak
+EXTRA_WORKLOADS = ("tiny-10k", "sub-1m", "tail-5m")
+SIDE_WORKLOAD = "sub-1m"  # the construction, temporal module and attention layer are measured here
+HGT_HEADS = 4  # attention heads (Section 4.1)
 
 
 def parse():
@@ -43,26 +50,37 @@ def parse():
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="sub-1m", choices=sorted(hgsynth.WORKLOADS))
+    ap.add_argument("--workload", default="big-10m", choices=sorted(hgsynth.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-extra", action="store_true", help="skip the other workloads and the ring pass")
     ap.add_argument("--no-build", action="store_true", help="skip the subgraph-construction measurement")
     ap.add_argument("--no-head", action="store_true",
                     help="drive the layers with a synthetic upstream gradient instead of the head and joint loss")
-    ap.add_argument("--oracle-sample", type=int, default=0, help=argparse.SUPPRESS)  # internal: child process
-    ap.add_argument("--oracle-no-head", action="store_true", help=argparse.SUPPRESS)  # internal: child process
-    ap.add_argument("--oracle-build-sample", type=int, default=0, help=argparse.SUPPRESS)  # internal: child process
-    ap.add_argument("--oracle-temporal-sample", type=int, default=0, help=argparse.SUPPRESS)  # internal: child process
     ap.add_argument("--no-temporal", action="store_true", help="skip the temporal-module measurement")
     ap.add_argument("--no-hgt", action="store_true", help="skip the attention-layer measurement")
     ap.add_argument("--scale", type=int, default=1, help=argparse.SUPPRESS)  # profiling: a 1/k-size instance
-    ap.add_argument("--oracle-hgt-sample", type=int, default=0, help=argparse.SUPPRESS)  # internal: child process
+    ap.add_argument("--oracle-child", default="", help=argparse.SUPPRESS)  # internal: child process kind
+    ap.add_argument("--oracle-k", type=int, default=1, help=argparse.SUPPRESS)
+    ap.add_argument("--oracle-steps", type=int, default=1, help=argparse.SUPPRESS)
+    ap.add_argument("--oracle-warmup", type=int, default=0, help=argparse.SUPPRESS)
     return ap.parse_args()
 
 
 def scaled(spec, k: int):
+    """A 1/k-size instance of the same recipe (nodes, edges, overlap set, hub floor and out-degree
+    cap all divided by k)."""
+    if k <= 1:
+        return spec
+    floor = None if spec.hub_floor is None else (spec.hub_floor[0], max(1, spec.hub_floor[1] // k))
+    cap = None if spec.out_cap is None else max(1, spec.out_cap // k)
     return hgsynth.spec(spec.name, n_user=max(1, spec.n_user // k), n_risk=max(1, spec.n_risk // k),
-                        num_edges=spec.num_edges // k, n_overlap=max(2, spec.n_overlap // k))
+                        num_edges=spec.num_edges // k, n_overlap=max(2, spec.n_overlap // k), hub_floor=floor,
+                        out_cap=cap)
+
+
+def sample_scale(sp) -> int:
+    return max(1, sp.num_edges // SAMPLE_EDGES)
 
 
 def workload_desc(sp) -> str:
@@ -72,87 +90,100 @@ def workload_desc(sp) -> str:
 
 
 # ------------------------------------------------------------------------------------------------
-# oracle timing (CPU baseline / reference arm); runs in a child process with one thread
+# oracle timing (CPU baseline / reference arm): a child process with the numpy oracle on a 1/k
+# instance drawn by hgsynth.graphs, its BLAS allowed every host core
 # ------------------------------------------------------------------------------------------------
-def oracle_sample_main(name: str, k: int, with_head: bool = True):
+def oracle_child_main(kind: str, name: str, k: int, steps: int, warmup: int, with_head: bool):
     import oracle
     sp = scaled(hgsynth.spec(name), k)
-    w = hgsynth.make_workload(sp)
-    vb = {"idx": w.overlap_local, "X_b": w.X_b} if sp.view_b == "perturbed" else \
-        {"H_b": w.H_b, "gid_a": w.gid_a, "gid_b": w.gid_b}
-    head = None
-    if with_head:
-        lab, y = hgsynth.make_labels(sp)
-        head = {"params": hgsynth.make_head_params(sp), "lab_idx": lab, "lab_y": y}
-    t0 = time.perf_counter()
-    oracle.step(w.graph, w.X, w.params, w.dH_top, vb, head=head)
-    dt = time.perf_counter() - t0
-    print(json.dumps({"seconds": dt, "edges": sp.num_edges, "layers": sp.layers,
-                      "value": sp.layers * sp.num_edges / dt}))
+    times = []
+    if kind == "step":
+        w = hgsynth.make_workload(sp)
+        vb = {"idx": w.overlap_local, "X_b": w.X_b} if sp.view_b == "perturbed" else \
+            {"H_b": w.H_b, "gid_a": w.gid_a, "gid_b": w.gid_b}
+        head = None
+        if with_head:
+            lab, y = hgsynth.make_labels(sp)
+            head = {"params": hgsynth.make_head_params(sp), "lab_idx": lab, "lab_y": y}
+        units = sp.layers * sp.num_edges
+        for i in range(warmup + steps):
+            t0 = time.perf_counter()
+            oracle.step(w.graph, w.X, w.params, w.dH_top, vb, head=head)
+            if i >= warmup:
+                times.append(time.perf_counter() - t0)
+    elif kind == "build":
+        from oracle import overlap_build as ob
+        g = hgsynth.make_graph(sp)
+        offs = np.asarray(g["type_offsets"], np.int64)
+        units = sp.num_edges
+        for i in range(warmup + steps):
+            t0 = time.perf_counter()
+            ob.build(g["src"], g["dst"], g["rel"], offs, BUILD_K, 0, BUILD_THETA, int(BUILD_BUDGET * offs[-1] / BUILD_K),
+                     21, 22)
+            if i >= warmup:
+                times.append(time.perf_counter() - t0)
+    elif kind == "temporal":
+        from oracle import temporal as OT
+        sp = hgsynth.spec(name)
+        n = max(1, sp.num_nodes // k)
+        rng = np.random.default_rng(7)
+        X = hgsynth.bf16_round(rng.standard_normal((n, sp.d), dtype=np.float32))
+        C = hgsynth.make_context(sp, rows=n)
+        p = hgsynth.make_temporal_params(sp)
+        dOut = hgsynth.bf16_round(rng.standard_normal((n, sp.d), dtype=np.float32))
+        units = n
+        for i in range(warmup + steps):
+            t0 = time.perf_counter()
+            OT.temporal_backward(X, C, p, dOut)
+            if i >= warmup:
+                times.append(time.perf_counter() - t0)
+    elif kind == "hgt":
+        from oracle import hgt as OH
+        w = hgsynth.make_workload(sp, with_ids=False)
+        g = w.graph
+        ps = [hgsynth.make_hgt_params(sp, HGT_HEADS, layer=l) for l in range(sp.layers)]
+        args = (g["src"], g["dst"], g["rel"], g["type_offsets"], g["rels"])
+        units = sp.layers * sp.num_edges
+        for i in range(warmup + steps):
+            t0 = time.perf_counter()
+            hs = [np.asarray(w.X, np.float64)]
+            for p in ps:
+                hs.append(OH.hgt_forward(*args, p, hs[-1], HGT_HEADS)[0])
+            dh = np.asarray(w.dH_top, np.float64)
+            for l in range(sp.layers - 1, -1, -1):
+                dh, _ = OH.hgt_backward(*args, ps[l], hs[l], dh, HGT_HEADS)
+            if i >= warmup:
+                times.append(time.perf_counter() - t0)
+    else:
+        raise ValueError(kind)
+    print(json.dumps({"seconds": times, "units": units, "edges": sp.num_edges, "value": units * len(times) / sum(times)}))
 
 
-def oracle_build_sample_main(name: str, k: int):
-    """Child process: the construction oracle on a 1/k-size instance of the workload's graph."""
-    from oracle import overlap_build as ob
-    sp = scaled(hgsynth.spec(name), k)
-    g = hgsynth.make_graph(sp)
-    offs = np.asarray(g["type_offsets"], np.int64)
-    t0 = time.perf_counter()
-    ob.build(g["src"], g["dst"], g["rel"], offs, BUILD_K, 0, BUILD_THETA, int(BUILD_BUDGET * offs[-1] / BUILD_K), 21, 22)
-    dt = time.perf_counter() - t0
-    print(json.dumps({"seconds": dt, "edges": sp.num_edges, "value": sp.num_edges / dt}))
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
 
 
-def oracle_temporal_sample_main(name: str, k: int):
-    """Child process: the temporal module's oracle (forward and backward) on N / k nodes."""
-    from oracle import temporal as OT
-    sp = hgsynth.spec(name)
-    n = max(1, sp.num_nodes // k)
-    rng = np.random.default_rng(7)
-    X = hgsynth.bf16_round(rng.standard_normal((n, sp.d), dtype=np.float32))
-    C = hgsynth.make_context(sp, rows=n)
-    p = hgsynth.make_temporal_params(sp)
-    dOut = hgsynth.bf16_round(rng.standard_normal((n, sp.d), dtype=np.float32))
-    t0 = time.perf_counter()
-    OT.temporal_backward(X, C, p, dOut, store="bf16" if sp.dtype == "bf16" else "f64")
-    dt = time.perf_counter() - t0
-    print(json.dumps({"seconds": dt, "edges": n, "value": n / dt}))
-
-
-HGT_HEADS = 4  # attention heads (Section 4.1)
-
-
-def oracle_hgt_sample_main(name: str, k: int):
-    """Child process: the attention layer's oracle, L layers forward and backward, on a 1/k-size
-    instance of the workload."""
-    from oracle import hgt as OH
-    sp = scaled(hgsynth.spec(name), k)
-    w = hgsynth.make_workload(sp, with_ids=False)
-    g = w.graph
-    store = "bf16" if sp.dtype == "bf16" else "f64"
-    ps = [hgsynth.make_hgt_params(sp, HGT_HEADS, layer=l) for l in range(sp.layers)]
-    args = (g["src"], g["dst"], g["rel"], g["type_offsets"], g["rels"])
-    t0 = time.perf_counter()
-    hs = [np.asarray(w.X, np.float64)]
-    for p in ps:
-        hs.append(OH.hgt_forward(*args, p, hs[-1], HGT_HEADS, store=store)[0])
-    dh = np.asarray(w.dH_top, np.float64)
-    for l in range(sp.layers - 1, -1, -1):
-        dh, _ = OH.hgt_backward(*args, ps[l], hs[l], dh, HGT_HEADS, store=store)
-    dt = time.perf_counter() - t0
-    print(json.dumps({"seconds": dt, "edges": sp.num_edges, "layers": sp.layers,
-                      "value": sp.layers * sp.num_edges / dt}))
-
-
-def time_oracle(name: str, k: int, flag: str = "--oracle-sample", with_head: bool = True) -> dict:
-    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+def time_oracle(name: str, k: int, kind: str = "step", with_head: bool = True, steps: int = 1, warmup: int = 0) -> dict:
+    cores = host_cores()
+    env = dict(os.environ, OMP_NUM_THREADS=str(cores), OPENBLAS_NUM_THREADS=str(cores), MKL_NUM_THREADS=str(cores),
                CUDA_VISIBLE_DEVICES="")
-    extra = [] if with_head else ["--oracle-no-head"]
-    r = subprocess.run([sys.executable, os.path.abspath(__file__), "--workload", name, flag, str(k), *extra],
-                       capture_output=True, text=True, env=env)
+    cmd = [sys.executable, os.path.abspath(__file__), "--workload", name, "--oracle-child", kind, "--oracle-k", str(k),
+           "--oracle-steps", str(steps), "--oracle-warmup", str(warmup)] + ([] if with_head else ["--no-head"])
+    r = subprocess.run(cmd, capture_output=True, text=True, env=env)
     if r.returncode != 0:
         raise RuntimeError(f"oracle sample failed: {r.stderr[-2000:]}")
-    return json.loads(r.stdout.strip().splitlines()[-1])
+    out = json.loads(r.stdout.strip().splitlines()[-1])
+    out["cores"] = cores
+    return out
+
+
+def oracle_sample_text(o: dict, what: str) -> str:
+    return (f"{what}: {o['edges']:,}-edge instance of the same recipe, the fp64 numpy oracle as it stands, "
+            f"{len(o['seconds'])} run(s) of {statistics.median(o['seconds']):.2f} s, BLAS allowed {o['cores']} "
+            f"host threads (the segment sums run on one)")
 
 
 # ------------------------------------------------------------------------------------------------
@@ -207,47 +238,69 @@ class Clocks:
 HUB, CHUNK = 512, 512
 
 
+def _graph_of(w):
+    """(graph dict, overlap rows) of a hgsynth Workload (numpy) or a hgsynth.device workload (torch)."""
+    if isinstance(w, dict):
+        return w["graph"], int(len(w["overlap_local"]))
+    return w.graph, int(len(w.overlap_local))
+
+
 def graph_stats(w) -> dict:
-    g = w.graph
-    sp = w.spec
-    offs = g["type_offsets"]
-    N = int(offs[-1])
-    src, dst, rel = g["src"].astype(np.int64), g["dst"].astype(np.int64), g["rel"]
-    st = dict(N=N, E=len(src), RR=0, CC=0, n_ov=int(len(w.overlap_local)),
-              fwd=dict(E_nh=0, E_h=0, U_nh=0, U_h=0, chunks=0),
-              bwd=dict(E_nh=0, E_h=0, U_nh=0, U_h=0, chunks=0), types=[], rels=[])
+    """Row, run and edge counts as the mean layer's aggregation kernels see them (torch, on the
+    arrays' device).  A run is one entry of an aggregation list: the parallel edges of a node pair
+    (same relation) with their multiplicity.  Forward rows are the CSR rows of each (relation,
+    destination); backward rows are node-major (a node's out-edges of every relation); a row above
+    HUB runs goes through chunks of CHUNK runs."""
+    import torch
+    g, n_ov = _graph_of(w)
+    tt_ = lambda a: a if torch.is_tensor(a) else torch.from_numpy(np.ascontiguousarray(a))  # noqa: E731
+    src, dst, rel = tt_(g["src"]).long(), tt_(g["dst"]).long(), tt_(g["rel"]).long()
+    offs = [int(x) for x in g["type_offsets"]]
+    N, R = offs[-1], len(g["rels"])
+    nz = lambda x: int(torch.count_nonzero(x))  # noqa: E731
+    blank = lambda: dict(E_nh=0, E_h=0, R_nh=0, R_h=0, U_nh=0, U_h=0, chunks=0)  # noqa: E731
+    st = dict(N=N, E=int(src.shape[0]), RR=0, CC=0, n_ov=n_ov, fwd=blank(), bwd=blank(), types=[], rels=[])
     for t in range(len(offs) - 1):
-        st["types"].append(dict(n=int(offs[t + 1] - offs[t]), R=sum(1 for r in g["rels"] if r[1] == t)))
+        st["types"].append(dict(n=offs[t + 1] - offs[t], R=sum(1 for r in g["rels"] if r[1] == t)))
     for r, (ts, tt) in enumerate(g["rels"]):
         m = rel == r
         s_r, d_r = src[m], dst[m]
-        n_t, n_s = int(offs[tt + 1] - offs[tt]), int(offs[ts + 1] - offs[ts])
-        st["RR"] += n_t
-        st["CC"] += n_s
-        st["rels"].append(dict(n_t=n_t, n_s=n_s, E=int(m.sum())))
-        # forward: one CSR row per (relation, destination), reading source rows of H
-        deg = np.bincount(d_r, minlength=N)
-        hub_edge = deg[d_r] > HUB
+        st["RR"] += offs[tt + 1] - offs[tt]
+        st["CC"] += offs[ts + 1] - offs[ts]
+        st["rels"].append(dict(n_t=offs[tt + 1] - offs[tt], n_s=offs[ts + 1] - offs[ts], E=int(s_r.shape[0])))
+        # forward: one CSR row per (relation, destination); its runs are the distinct sources
+        u = torch.unique(d_r * N + s_r)
+        u_dst, u_src = u // N, u % N
+        runs = torch.bincount(u_dst, minlength=N)
+        hub_run = runs[u_dst] > HUB
+        edges = torch.bincount(d_r, minlength=N)
         a = st["fwd"]
-        a["E_h"] += int(hub_edge.sum())
-        a["E_nh"] += int((~hub_edge).sum())
-        a["U_h"] += int(np.count_nonzero(np.bincount(s_r[hub_edge], minlength=N)))
-        a["U_nh"] += int(np.count_nonzero(np.bincount(s_r[~hub_edge], minlength=N)))
-        hd = deg[deg > HUB]
-        a["chunks"] += int(((hd + CHUNK - 1) // CHUNK).sum())
-    # backward: one node-major row per node (its out-edges of every relation), each edge reading the
-    # dMs row of its (relation, destination); the hub split follows the node's total out-degree
-    deg = np.bincount(src, minlength=N)
-    hub_edge = deg[src] > HUB
-    read = rel.astype(np.int64) * N + dst
-    nread = len(g["rels"]) * N
+        a["R_h"] += nz(hub_run)
+        a["R_nh"] += int(u.shape[0]) - nz(hub_run)
+        a["E_h"] += int(edges[runs > HUB].sum())
+        a["E_nh"] += int(edges[runs <= HUB].sum())
+        a["U_h"] += nz(torch.bincount(u_src[hub_run], minlength=N))
+        a["U_nh"] += nz(torch.bincount(u_src[~hub_run], minlength=N))
+        hr = runs[runs > HUB]
+        a["chunks"] += int(((hr + CHUNK - 1) // CHUNK).sum())
+        del u, u_dst, u_src, runs, hub_run, edges
+    # backward: one node-major row per node; its runs are the distinct (relation, destination) dMs
+    # rows it reads
+    read = rel * N + dst
+    u = torch.unique(src * (R * N) + read)
+    u_src, u_read = u // (R * N), u % (R * N)
+    runs = torch.bincount(u_src, minlength=N)
+    hub_run = runs[u_src] > HUB
+    edges = torch.bincount(src, minlength=N)
     a = st["bwd"]
-    a["E_h"] = int(hub_edge.sum())
-    a["E_nh"] = int((~hub_edge).sum())
-    a["U_h"] = int(np.count_nonzero(np.bincount(read[hub_edge], minlength=nread)))
-    a["U_nh"] = int(np.count_nonzero(np.bincount(read[~hub_edge], minlength=nread)))
-    hd = deg[deg > HUB]
-    a["chunks"] = int(((hd + CHUNK - 1) // CHUNK).sum())
+    a["R_h"] = nz(hub_run)
+    a["R_nh"] = int(u.shape[0]) - a["R_h"]
+    a["E_h"] = int(edges[runs > HUB].sum())
+    a["E_nh"] = int(edges[runs <= HUB].sum())
+    a["U_h"] = nz(torch.bincount(u_read[hub_run], minlength=R * N))
+    a["U_nh"] = nz(torch.bincount(u_read[~hub_run], minlength=R * N))
+    hr = runs[runs > HUB]
+    a["chunks"] = int(((hr + CHUNK - 1) // CHUNK).sum())
     return st
 
 
@@ -258,20 +311,16 @@ def kernel_models(st: dict, sp) -> dict:
     f, bw = st["fwd"], st["bwd"]
     row = d * b
     m = {}
-    # aggregation, per unit of work = one gathered edge: its 4-byte index and one feature row, with no
-    # cache reuse assumed (the per-edge model; 1/deg is folded into dMs, so the transposed pass reads
-    # no per-edge coefficient).  The compulsory bytes (each distinct row once) are in `compulsory`.
-    ge = 4 + row
-    m["agg_fwd_rows"] = (L * f["E_nh"] * ge, 0)
-    m["agg_fwd_chunks"] = (L * f["E_h"] * ge, 0)
-    m["agg_bwd_nodes"] = (L * bw["E_nh"] * ge, 0)
-    m["agg_bwd_chunks"] = (L * bw["E_h"] * ge, 0)
-    m["compulsory"] = {
-        "agg_fwd_rows": L * (4 * (RR + 1) + 4 * f["E_nh"] + row * f["U_nh"] + row * RR + 4 * d * f["chunks"]),
-        "agg_fwd_chunks": L * (4 * f["E_h"] + row * f["U_h"] + 4 * d * f["chunks"]),
-        "agg_bwd_nodes": L * (4 * (N + 1) + 4 * bw["E_nh"] + row * bw["U_nh"] + 2 * row * N + 4 * d * bw["chunks"]),
-        "agg_bwd_chunks": L * (4 * bw["E_h"] + row * bw["U_h"] + 4 * d * bw["chunks"]),
-    }
+    # aggregation (mean layer), compulsory bytes per step: each distinct row it reads once, the
+    # run lists (column and count, 8 bytes per run) and row pointers once, every output row written
+    # once, the fp32 chunk partials written and read.  The rows gathered per run (one per run, served
+    # by L1 / L2 where a row recurs) are reported beside them as `gathered` (not HBM traffic).
+    m["agg_fwd_rows"] = (L * (8 * (RR + 1) + 8 * f["R_nh"] + row * f["U_nh"] + row * RR + 4 * d * f["chunks"]), 0)
+    m["agg_fwd_chunks"] = (L * (8 * f["R_h"] + row * f["U_h"] + 4 * d * f["chunks"]), 0)
+    m["agg_bwd_nodes"] = (L * (4 * (N + 1) + 8 * bw["R_nh"] + row * bw["U_nh"] + 2 * row * N + 4 * d * bw["chunks"]), 0)
+    m["agg_bwd_chunks"] = (L * (8 * bw["R_h"] + row * bw["U_h"] + 4 * d * bw["chunks"]), 0)
+    m["gathered"] = {"agg_fwd_rows": L * f["R_nh"] * (8 + row), "agg_fwd_chunks": L * f["R_h"] * (8 + row),
+                     "agg_bwd_nodes": L * bw["R_nh"] * (8 + row), "agg_bwd_chunks": L * bw["R_h"] * (8 + row)}
     fb = ff = bb = bf = 0
     for t in st["types"]:
         n, R = t["n"], t["R"]
@@ -295,10 +344,10 @@ def kernel_models(st: dict, sp) -> dict:
     m["ln_act_bwd"] = (L * lb, 0)
     m["proj_bwd_tc"] = (L * pb, L * pfl)
     m["wgrad_tc"] = (L * row * (RR + N), L * 2 * d * d * RR)  # G_r = M_r^T dU: M_r rows once, dU once per type
-    # per 8-bit pass over the keys (the row ids, invalid edges keyed one past the last row): read and
-    # write of key, edge id and endpoint; one sort per layout
+    # per 8-bit pass over the keys: read and write of key, edge id and endpoint; three stable sorts
+    # (by source id, then CSR row: (row, source, edge id); that order by CSC row)
     passes = lambda rows: max(1, -(-int(rows).bit_length() // 8))  # noqa: E731
-    m["radix_scatter"] = (2 * 12 * st["E"] * (passes(RR) + passes(CC)), 0)
+    m["radix_scatter"] = (2 * 12 * st["E"] * (passes(N) + passes(RR) + passes(CC)), 0)
     nl = st.get("n_lab", 0)
     if nl:
         # per labelled row: its H row (and a replica row for overlap rows, not counted), the saved Hm
@@ -364,25 +413,26 @@ def roofline(report: dict, models: dict, steps: int, peaks: dict, src: str, dom=
     rf["traffic"] = measured_traffic(dom)
     rf.update(kernel=dom, launches=n, avg_launch_ms=round(ms / max(n, 1), 4),
               algorithmic_bytes_per_launch=int(by * steps / max(n, 1)), flops_per_launch=int(fl * steps / max(n, 1)))
-    comp = models.get("compulsory", {}).get(dom)
-    if comp is not None:
-        rf["model"] = ("per gathered edge: its index and one feature row, with no cache reuse (rows served by L1/L2 "
-                       "count as traffic, so frac can exceed 1); compulsory_*: each distinct row once")
-        rf["compulsory_bytes_per_launch"] = int(comp * steps / max(n, 1))
-        rf["compulsory_frac"] = round(comp * steps / secs / 1e9 / peaks["hbm_gbs"], 4) if secs > 0 else None
+    gat = models.get("gathered", {}).get(dom)
+    if gat is not None:
+        rf["model"] = ("compulsory: each distinct row read once, run lists and pointers once, outputs written once; "
+                       "gathered_*: one feature row and its 8-byte run entry per run, repeated rows served by L1/L2")
+        rf["gathered_bytes_per_launch"] = int(gat * steps / max(n, 1))
+        rf["gathered_gbs"] = round(gat * steps / secs / 1e9, 1) if secs > 0 else None
     return rf, shares
 
 
-def measure_overlap_build(w, steps: int, warmup: int, dev, with_cpu: bool) -> dict:
+def measure_overlap_build(w: dict, steps: int, warmup: int, dev, with_cpu: bool) -> dict:
     """The overlapping-subgraph construction (Section 3.1; done once before training, so it is not
     part of the step) on the workload's graph taken as the global graph: subgraph 0 of BUILD_K,
     h-index bound BUILD_THETA, budget BUILD_BUDGET * N / BUILD_K.  Device time per call."""
     import torch
     from paper_2608_02168_gb300 import hg
-    g = w.graph
+    g = w["graph"]
     offs = [int(x) for x in g["type_offsets"]]
-    src, dst, rel = (torch.from_numpy(g[k]).to(dev) for k in ("src", "dst", "rel"))
-    ws = torch.empty(hg.hg_overlap_build_workspace_size(offs[-1], len(g["src"])), dtype=torch.uint8, device=dev)
+    src, dst, rel = g["src"], g["dst"], g["rel"]
+    E = int(src.shape[0])
+    ws = torch.empty(hg.hg_overlap_build_workspace_size(offs[-1], E), dtype=torch.uint8, device=dev)
     M = int(BUILD_BUDGET * offs[-1] / BUILD_K)
 
     def call():
@@ -413,9 +463,10 @@ def measure_overlap_build(w, steps: int, warmup: int, dev, with_cpu: bool) -> di
     # one read of both incidence entries by the h-index (8 B) and the keep flag (4 B); per node, the
     # ten 4-byte node arrays written and read once (40 B)
     peaks, psrc = load_peaks()
-    byt = 60 * len(g["src"]) + 40 * offs[-1]
+    byt = 60 * E + 40 * offs[-1]
     ach = byt / (ms / 1e3) / 1e9
-    res = {"ms": round(ms, 4), "edges_per_s": len(g["src"]) / (ms / 1e3), "counts": out["counts"],
+    res = {"workload": workload_desc(w["spec"]), "ms": round(ms, 4), "edges_per_s": E / (ms / 1e3),
+           "counts": out["counts"],
            "roofline": {"bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
                         "peak_source": f"{psrc} hbm_gbs", "frac": round(ach / peaks["hbm_gbs"], 4),
                         "frac_of_nominal": round(ach / NOMINAL_HBM_GBS, 4),
@@ -424,10 +475,9 @@ def measure_overlap_build(w, steps: int, warmup: int, dev, with_cpu: bool) -> di
            "kernel_time_share": {k: round(v / tot, 4) for k, (_, v) in sorted(rep.items(), key=lambda kv: -kv[1][1])},
            "cpu_baseline": None}
     if with_cpu:
-        o = time_oracle(w.spec.name, ORACLE_SCALE, "--oracle-build-sample")
-        res["cpu_baseline"] = {"value": o["value"], "unit": "edges/s", "cores": 1, "kind": "oracle",
-                               "sample": f"1/{ORACLE_SCALE}-size instance ({o['edges']:,} edges), numpy oracle, one "
-                                         f"thread, {o['seconds']:.1f} s"}
+        o = time_oracle(w["spec"].name, sample_scale(w["spec"]), "build")
+        res["cpu_baseline"] = {"value": o["value"], "unit": "edges/s", "cores": o["cores"], "kind": "oracle",
+                               "sample": oracle_sample_text(o, "the construction")}
     return res
 
 
@@ -495,23 +545,21 @@ def measure_temporal(sp, steps: int, warmup: int, dev, with_cpu: bool) -> dict:
            "kernel_time_share": {k: round(v / tot, 4) for k, (_, v) in sorted(rep.items(), key=lambda kv: -kv[1][1])},
            "cpu_baseline": None}
     if with_cpu:
-        o = time_oracle(sp.name, ORACLE_SCALE, "--oracle-temporal-sample")
-        res["cpu_baseline"] = {"value": o["value"], "unit": "nodes/s", "cores": 1, "kind": "oracle",
-                               "sample": f"{o['edges']:,} nodes (1/{ORACLE_SCALE} of the workload), forward and "
-                                         f"backward of the fp64 numpy oracle, one thread, {o['seconds']:.1f} s"}
+        o = time_oracle(sp.name, max(1, n // 25_000), "temporal")
+        res["cpu_baseline"] = {"value": o["value"], "unit": "nodes/s", "cores": o["cores"], "kind": "oracle",
+                               "sample": oracle_sample_text(o, f"forward and backward over {o['units']:,} nodes")}
     return res
 
 
-def measure_hgt(w, steps: int, warmup: int, dev, with_cpu: bool) -> dict:
+def measure_hgt(w: dict, steps: int, warmup: int, dev, with_cpu: bool) -> dict:
     """The attention variant of the layer (Eq. 6-11, HGT_HEADS heads): the workload's L layers
     forward and backward on its graph (CSR built once), synthetic upstream gradient.  Device time
     per forward + backward of the stack."""
     import torch
     from paper_2608_02168_gb300 import hg
-    sp, g = w.spec, w.graph
+    sp, g = w["spec"], w["graph"]
     td = torch.float32 if sp.dtype == "f32" else torch.bfloat16
-    G = hg.hg_build_csr(*(torch.from_numpy(g[k]).to(dev) for k in ("src", "dst", "rel")), g["type_offsets"],
-                        g["rels"])
+    G = hg.hg_build_csr(g["src"], g["dst"], g["rel"], g["type_offsets"], g["rels"])
     params = []
     for l in range(sp.layers):
         p = hgsynth.make_hgt_params(sp, HGT_HEADS, layer=l)
@@ -521,9 +569,8 @@ def measure_hgt(w, steps: int, warmup: int, dev, with_cpu: bool) -> dict:
     saved = [torch.empty(sb, dtype=torch.uint8, device=dev) for _ in params]
     scratch = torch.empty(kb, dtype=torch.uint8, device=dev)
     N, d = sp.num_nodes, sp.d
-    Hs = [torch.from_numpy(w.X).to(dev, td)] + [torch.empty(N, d, dtype=td, device=dev) for _ in params]
-    dHs = [torch.empty(N, d, dtype=td, device=dev) for _ in range(len(params))] + \
-          [torch.from_numpy(w.dH_top).to(dev, td)]
+    Hs = [w["X"]] + [torch.empty(N, d, dtype=td, device=dev) for _ in params]
+    dHs = [torch.empty(N, d, dtype=td, device=dev) for _ in range(len(params))] + [w["dH_top"]]
     f = dict(dtype=torch.float32, device=dev)
     grads = [{k: torch.empty(np.shape(v), **f) for k, v in hgsynth.make_hgt_params(sp, HGT_HEADS).items()}
              for _ in params]
@@ -559,10 +606,10 @@ def measure_hgt(w, steps: int, warmup: int, dev, with_cpu: bool) -> dict:
     b = 4 if sp.dtype == "f32" else 2
     offs = [int(x) for x in g["type_offsets"]]
     RR = sum(offs[t + 1] - offs[t] for _, t in g["rels"])
-    per_layer = 3 * len(g["src"]) * (4 + 2 * sp.d * b) + (2 * RR + 10 * sp.num_nodes) * sp.d * b
+    per_layer = 3 * sp.num_edges * (4 + 2 * sp.d * b) + (2 * RR + 10 * sp.num_nodes) * sp.d * b
     peaks, psrc = load_peaks()
     ach = sp.layers * per_layer / (ms / 1e3) / 1e9
-    res = {"ms": round(ms, 4), "layers": sp.layers, "heads": HGT_HEADS,
+    res = {"workload": workload_desc(sp), "ms": round(ms, 4), "layers": sp.layers, "heads": HGT_HEADS,
            "layers_fwd_bwd_edges_per_s": sp.layers * sp.num_edges / (ms / 1e3),
            "roofline": {"bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
                         "peak_source": f"{psrc} hbm_gbs", "frac": round(ach / peaks["hbm_gbs"], 4),
@@ -572,28 +619,231 @@ def measure_hgt(w, steps: int, warmup: int, dev, with_cpu: bool) -> dict:
            "kernel_time_share": {k: round(v / tot, 4) for k, (_, v) in sorted(rep.items(), key=lambda kv: -kv[1][1])},
            "cpu_baseline": None}
     if with_cpu:
-        o = time_oracle(sp.name, REFERENCE_SCALE, "--oracle-hgt-sample")
-        res["cpu_baseline"] = {"value": o["value"], "unit": UNIT, "cores": 1, "kind": "oracle",
-                               "sample": f"1/{REFERENCE_SCALE}-size instance ({o['edges']:,} edges), {sp.layers} layers "
-                                         f"forward and backward of the fp64 numpy oracle, one thread, "
-                                         f"{o['seconds']:.1f} s"}
+        o = time_oracle(sp.name, 4 * sample_scale(sp), "hgt")
+        res["cpu_baseline"] = {"value": o["value"], "unit": UNIT, "cores": o["cores"], "kind": "oracle",
+                               "sample": oracle_sample_text(o, f"{sp.layers} attention layers forward and backward")}
     return res
+
+
+LAYER_KERNELS = ("agg_fwd_rows", "agg_fwd_chunks", "agg_bwd_nodes", "agg_bwd_chunks", "combine_chunk_partials",
+                 "fuse_weights", "proj_fwd_tc", "ln_act_bwd", "proj_bwd_tc", "wgrad_tc", "wgrad_finish", "reduce_lanes",
+                 "proj_fwd_simt", "proj_bwd_simt", "wgrad_partial")
+
+
+def layer_stack_bytes(models: dict) -> int:
+    """Algorithmic bytes of the L-layer forward + backward in one step: the aggregations' compulsory
+    bytes (each distinct row once) and the projections' streamed bytes."""
+    total = 0
+    for k in ("agg_fwd_rows", "agg_fwd_chunks", "agg_bwd_nodes", "agg_bwd_chunks", "proj_fwd_tc", "ln_act_bwd",
+              "proj_bwd_tc", "wgrad_tc"):
+        total += models.get(k, (0, 0))[0]
+    return int(total)
+
+
+# ------------------------------------------------------------------------------------------------
+# the hot-path step on one workload
+# ------------------------------------------------------------------------------------------------
+def step_inputs(w: dict, use_head: bool) -> dict:
+    g = w["graph"]
+    inp = {"src": g["src"], "dst": g["dst"], "rel": g["rel"], "X": w["X"]}
+    if use_head:
+        inp.update(lab_idx=w["lab_idx"], lab_y=w["lab_y"])
+    else:
+        inp["dH_top"] = w["dH_top"]
+    if w["spec"].view_b == "perturbed":
+        inp.update(X_b=w["X_b"], overlap_idx=w["overlap_local"])
+    else:
+        inp.update(gid_a=w["gid_a"], gid_b=w["gid_b"], H_bank=w["H_b"])
+    return inp
+
+
+def make_path(w: dict, dev, use_head: bool):
+    from paper_2608_02168_gb300.step import HotPath
+    sp, g = w["spec"], w["graph"]
+    return HotPath(g["type_offsets"], g["rels"], int(g["src"].shape[0]), sp.d, sp.dtype, w["params"], view=sp.view_b,
+                   n_overlap_max=int(len(w["overlap_local"])),
+                   n_gid_a=0 if "gid_a" not in w else int(len(w["gid_a"])),
+                   n_gid_b=0 if "gid_b" not in w else int(len(w["gid_b"])), device=dev,
+                   head_params=hgsynth.make_head_params(sp) if use_head else None,
+                   n_lab_max=int(len(w["lab_idx"])) if use_head else 0)
+
+
+def run_hot_path(w: dict, dev, steps: int, warmup: int, world: int, use_head: bool, clocks=None, e2e: bool = False) -> dict:
+    """Times `steps` steps (after `warmup`), then the phases of the step and the per-kernel report;
+    optionally the same steps end to end from pinned host inputs."""
+    import torch
+    from paper_2608_02168_gb300 import hg
+    sp = w["spec"]
+    path = make_path(w, dev, use_head)
+    devin = step_inputs(w, use_head)
+    stream = torch.cuda.current_stream()
+
+    def step(inp, marks=None):
+        kw = {k: inp[k] for k in ("X_b", "overlap_idx", "gid_a", "gid_b", "H_bank", "lab_idx", "lab_y") if k in inp}
+        path.step(inp["src"], inp["dst"], inp["rel"], inp["X"], inp.get("dH_top"), marks=marks, **kw)
+
+    for _ in range(max(warmup, 0)):
+        step(devin)
+    torch.cuda.synchronize()
+    if clocks is not None:
+        clocks.start()
+    rank_barrier(world)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        torch.cuda.nvtx.range_push("step")  # profilers select the timed steps by this range
+        step(devin)
+        torch.cuda.nvtx.range_pop()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    rank_barrier(world)
+    clk = clocks.stop() if clocks is not None else None
+    t = max_time_over_ranks(e0.elapsed_time(e1) / 1e3, world, dev)
+    # phases of the step (uninstrumented)
+    phase_ms = {}
+    for _ in range(steps):
+        marks = []
+        m0 = torch.cuda.Event(enable_timing=True)
+        m0.record(stream)
+        step(devin, marks)
+        torch.cuda.synchronize()
+        prev = m0
+        for name, ev in marks:
+            phase_ms[name] = phase_ms.get(name, 0.0) + prev.elapsed_time(ev) / steps
+            prev = ev
+    # per-kernel durations from a second, instrumented run of the same steps (the library records
+    # CUDA events around each of its launches, which the headline timing leaves out)
+    hg.hg_timing_enable(True)
+    hg.hg_timing_report()
+    for _ in range(steps):
+        step(devin)
+    torch.cuda.synchronize()
+    hg.hg_timing_enable(False)
+    report = hg.hg_timing_report()
+    units = sp.layers * int(w["graph"]["src"].shape[0])
+    res = {"t": t, "value": weak_scaling_value(world, units, steps, t), "ms_per_step": 1e3 * t / steps,
+           "phases_ms": {k: round(v, 4) for k, v in phase_ms.items()}, "report": report, "clocks": clk,
+           "launches_per_step": sum(n for n, _ in report.values()) / max(steps, 1)}
+    lay = phase_ms.get("forward", 0) + phase_ms.get("backward", 0)
+    res["layers_fwd_bwd_edges_per_s"] = units / (lay / 1e3) if lay else None
+    res["csr_build_edges_per_s"] = units / sp.layers / (phase_ms["graph"] / 1e3) if phase_ms.get("graph") else None
+    if e2e:
+        res["e2e"] = run_e2e(path, step, devin, dev, steps, world, units, use_head)
+    res["loss"] = [float(x) for x in path.loss.cpu()]
+    res["head_loss"] = [float(x) for x in path.head_loss.cpu()] if use_head else None
+    del path
+    return res
+
+
+def run_e2e(path, step, devin, dev, steps, world, units, use_head) -> dict:
+    """Same steps through the public API with every step's inputs copied in from pinned host memory
+    (the copy of step i+1's inputs overlaps step i) and its loss read back."""
+    import torch
+    stream = torch.cuda.current_stream()
+    pinned = {k: v.cpu().pin_memory() for k, v in devin.items()}
+    h2d = sum(v.numel() * v.element_size() for v in pinned.values())
+    result = path.head_loss if use_head else path.loss  # L_total (Eq. 20), or the alignment loss
+    loss_host = torch.empty(result.numel(), dtype=torch.float32).pin_memory()
+    bufs = [devin, {k: torch.empty_like(v) for k, v in devin.items()}]
+    copy_stream = torch.cuda.Stream(device=dev)
+    copied = [torch.cuda.Event(), torch.cuda.Event()]
+    consumed = [torch.cuda.Event(), torch.cuda.Event()]
+
+    def copy_in(i):
+        b = i % 2
+        with torch.cuda.stream(copy_stream):
+            copy_stream.wait_event(consumed[b])  # the step that last read this buffer set is done
+            for k, v in pinned.items():
+                bufs[b][k].copy_(v, non_blocking=True)
+            copied[b].record(copy_stream)
+
+    rank_barrier(world)
+    torch.cuda.synchronize()
+    for ev in consumed:
+        ev.record(stream)
+    t0 = time.perf_counter()
+    copy_in(0)
+    for i in range(steps):
+        if i + 1 < steps:
+            copy_in(i + 1)
+        stream.wait_event(copied[i % 2])
+        step(bufs[i % 2])
+        consumed[i % 2].record(stream)
+        loss_host.copy_(result, non_blocking=True)
+        stream.synchronize()  # the loss of step i is on the host
+    torch.cuda.synchronize()
+    te = max_time_over_ranks(time.perf_counter() - t0, world, dev)
+    out = {"value": weak_scaling_value(world, units, steps, te), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+           "d2h_bytes_per_step": int(loss_host.numel() * 4)}
+    del bufs, pinned
+    return out
+
+
+def workload_summary(w: dict, res: dict, models: dict, steps: int, peaks: dict, psrc: str) -> dict:
+    """The per-workload figures: whole step, layer stack (with its roofline over the summed
+    algorithmic bytes of the layer kernels), CSR build, phases, dominant kernel."""
+    sp = w["spec"]
+    lay_ms = res["phases_ms"].get("forward", 0) + res["phases_ms"].get("backward", 0)
+    lb = layer_stack_bytes(models)
+    ach = lb / (lay_ms / 1e3) / 1e9 if lay_ms else 0.0
+    rf, shares = roofline(res["report"], models, steps, peaks, psrc)
+    return {"workload": workload_desc(sp), "value": res["value"], "unit": UNIT, "ms_per_step": round(res["ms_per_step"], 4),
+            "layers_fwd_bwd_edges_per_s": res["layers_fwd_bwd_edges_per_s"],
+            "csr_build_edges_per_s": res["csr_build_edges_per_s"], "phases_ms": res["phases_ms"],
+            "layer_stack_roofline": {"bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                                     "frac": round(ach / peaks["hbm_gbs"], 4), "algorithmic_bytes_per_step": lb,
+                                     "model": "aggregations: each distinct row once; projections: rows streamed"},
+            "roofline": rf, "kernel_time_share": dict(list(shares.items())[:12]),
+            "gpu_launches_per_step": res["launches_per_step"]}
+
+
+def measure_ring(sp, dev, warmup: int) -> dict:
+    """One full pass over the ring of sparse overlapping subgraphs (Algorithm 1 run in sequence on one
+    GPU): subgraph k aligns with the detached final embeddings of subgraph k-1 (the first has no
+    alignment term), synthetic upstream gradient.  Device time of the 16 steps after `warmup`
+    steps on the first subgraphs."""
+    import torch
+    from hgsynth import device as hd
+    from paper_2608_02168_gb300.step import Ring
+    table = hd.ring_features(sp, dev)
+    parts = [hd.make_ring_part(sp, k, table, dev) for k in range(sp.num_subgraphs)]
+    del table
+    dH = hd.make_features(sp, 0, dev, 4)
+    params = [hgsynth.make_layer_params(sp, l) for l in range(sp.layers)]
+    g0 = parts[0]["graph"]
+    E = int(g0["src"].shape[0])
+    ring = Ring(g0["type_offsets"], g0["rels"], E, sp.d, sp.dtype, params, device=dev)
+
+    def run(p):
+        g = p["graph"]
+        ring.step(g["src"], g["dst"], g["rel"], p["X"], dH, p["gid"])
+
+    for k in range(max(warmup, 1)):
+        run(parts[k % len(parts)])
+    ring.have_bank = False  # the timed pass starts a fresh sequence
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for p in parts:
+        run(p)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    units = sp.num_subgraphs * sp.layers * E
+    n_ov = int(ring.path.n_dev.item())
+    del ring, parts
+    return {"workload": workload_desc(sp), "subgraphs": sp.num_subgraphs, "ms_per_pass": round(ms, 3),
+            "edges_per_s": units / (ms / 1e3), "overlap_rows_last_step": n_ov,
+            "objective": "synthetic upstream gradient + 0.1 L_CCA against the previous subgraph"}
 
 
 # ------------------------------------------------------------------------------------------------
 def main():
     args = parse()
-    if args.oracle_sample:
-        oracle_sample_main(args.workload, args.oracle_sample, not args.oracle_no_head)
-        return
-    if args.oracle_build_sample:
-        oracle_build_sample_main(args.workload, args.oracle_build_sample)
-        return
-    if args.oracle_temporal_sample:
-        oracle_temporal_sample_main(args.workload, args.oracle_temporal_sample)
-        return
-    if args.oracle_hgt_sample:
-        oracle_hgt_sample_main(args.workload, args.oracle_hgt_sample)
+    if args.oracle_child:
+        oracle_child_main(args.oracle_child, args.workload, args.oracle_k, args.oracle_steps, args.oracle_warmup,
+                          not args.no_head)
         return
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -636,23 +886,29 @@ def weak_scaling_value(world: int, edges_per_step: int, steps: int, seconds: flo
 
 
 def run_reference(args, sp):
-    for _ in range(args.warmup):
-        time_oracle(sp.name, REFERENCE_SCALE, with_head=not args.no_head)
-    vals = [time_oracle(sp.name, REFERENCE_SCALE, with_head=not args.no_head) for _ in range(args.steps)]
-    secs = sum(v["seconds"] for v in vals)
-    edges = sum(v["edges"] * v["layers"] for v in vals)
-    value = edges / secs
-    sample = (f"1/{REFERENCE_SCALE}-size instance of the workload per step "
-              f"({vals[0]['edges']:,} edges, same recipe), fp64 numpy oracle"
-              f"{'' if args.no_head else ' with the head and joint loss'}, one thread")
+    """The oracle, as it stands, on a bounded sample of the workload (one child process, its BLAS on
+    every host core): warm-up and timed steps each one full step of the oracle."""
+    k = sample_scale(sp)
+    o = time_oracle(sp.name, k, "step", with_head=not args.no_head, steps=args.steps, warmup=args.warmup)
+    secs = sum(o["seconds"])
+    value = o["units"] * len(o["seconds"]) / secs
+    sample = oracle_sample_text(o, "one step per timed step" + ("" if args.no_head else ", with the head and joint loss"))
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * secs / max(len(o["seconds"]), 1),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": workload_desc(sp)},
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "config": {"workload": workload_desc(sp), "sample": f"1/{k}-size instance of the same recipe"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": o["cores"], "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }))
+
+
+def free_device_memory():
+    import gc
+    import torch
+    gc.collect()
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
 
 
 def run_ours(args, sp, rank, world):
@@ -664,172 +920,76 @@ def run_ours(args, sp, rank, world):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     from paper_2608_02168_gb300 import build as hbuild
     hbuild.build()
-    from paper_2608_02168_gb300 import hg
-    from paper_2608_02168_gb300.step import HotPath
+    from hgsynth import device as hd
 
     dev = torch.device("cuda", torch.cuda.current_device())
-    w = hgsynth.make_workload(sp, sub=rank)
-    g = w.graph
-    td = torch.float32 if sp.dtype == "f32" else torch.bfloat16
     use_head = not args.no_head
-    lab, lab_y = hgsynth.make_labels(sp, sub=rank)
-    path = HotPath(g["type_offsets"], g["rels"], len(g["src"]), sp.d, sp.dtype, w.params, view=sp.view_b,
-                   n_overlap_max=len(w.overlap_local), n_gid_a=0 if w.gid_a is None else len(w.gid_a),
-                   n_gid_b=0 if w.gid_b is None else len(w.gid_b), device=dev,
-                   head_params=hgsynth.make_head_params(sp) if use_head else None, n_lab_max=len(lab))
-    host = {"src": torch.from_numpy(g["src"]), "dst": torch.from_numpy(g["dst"]), "rel": torch.from_numpy(g["rel"]),
-            "X": torch.from_numpy(w.X).to(td)}
-    if use_head:  # the head's gradient drives the backward; its inputs are the labels
-        host.update(lab_idx=torch.from_numpy(lab), lab_y=torch.from_numpy(lab_y))
-    else:
-        host["dH_top"] = torch.from_numpy(w.dH_top).to(td)
-    if sp.view_b == "perturbed":
-        host.update(X_b=torch.from_numpy(w.X_b).to(td), overlap_idx=torch.from_numpy(w.overlap_local))
-    else:
-        host.update(gid_a=torch.from_numpy(w.gid_a), gid_b=torch.from_numpy(w.gid_b), H_bank=torch.from_numpy(w.H_b).to(td))
-    devin = {k: v.to(dev) for k, v in host.items()}
-    stream = torch.cuda.current_stream()
-
-    def barrier():
-        rank_barrier(world)
-
-    def max_over_ranks(x: float) -> float:
-        return max_time_over_ranks(x, world, dev)
-
-    def step(inp, marks=None):
-        kw = {k: inp[k] for k in ("X_b", "overlap_idx", "gid_a", "gid_b", "H_bank", "lab_idx", "lab_y") if k in inp}
-        path.step(inp["src"], inp["dst"], inp["rel"], inp["X"], inp.get("dH_top"), marks=marks, **kw)
-
-    for _ in range(max(args.warmup, 0)):
-        step(devin)
+    peaks, psrc = load_peaks()
+    # the headline workload: this rank's subgraph, drawn on the device
+    w = hd.make_workload(sp, sub=rank, device=dev, with_dH_top=not use_head)
     torch.cuda.synchronize()
-    stats = graph_stats(w)
-    stats["n_lab"] = len(lab) if use_head else 0
-    models = kernel_models(stats, sp)
     clocks = Clocks(dev.index if dev.index is not None else 0)
-    clocks.start()
-    barrier()
-    torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.steps):
-        torch.cuda.nvtx.range_push("step")  # profilers select the timed steps by this range
-        step(devin)
-        torch.cuda.nvtx.range_pop()
-    e1.record(stream)
-    torch.cuda.synchronize()
-    barrier()
-    clk = clocks.stop()
-    t = max_over_ranks(e0.elapsed_time(e1) / 1e3)
-    # phases of the step (uninstrumented): graph build, forward layers, alignment (intersection,
-    # loss, gradient), backward layers
-    phase_ms = {}
-    for _ in range(args.steps):
-        marks = []
-        m0 = torch.cuda.Event(enable_timing=True)
-        m0.record(stream)
-        step(devin, marks)
-        torch.cuda.synchronize()
-        prev = m0
-        for name, ev in marks:
-            phase_ms[name] = phase_ms.get(name, 0.0) + prev.elapsed_time(ev) / args.steps
-            prev = ev
-    # per-kernel durations (shares, roofline) from a second, instrumented run of the same steps: the
-    # library records CUDA events around each of its launches, which the headline timing leaves out
-    hg.hg_timing_enable(True)
-    hg.hg_timing_report()  # clear
-    for _ in range(args.steps):
-        step(devin)
-    torch.cuda.synchronize()
-    hg.hg_timing_enable(False)
-    report = hg.hg_timing_report()
-    edges_per_step = sp.layers * sp.num_edges
-    value = weak_scaling_value(world, edges_per_step, args.steps, t)
-
-    # end to end: pinned host inputs copied in, the step, the loss read back, every step
-    e2e = None
-    if not args.no_e2e:
-        # every step copies its own inputs in from pinned host memory and reads its loss back; the
-        # copy of step i+1's inputs (second device buffer set, copy stream) overlaps step i
-        pinned = {k: v.pin_memory() for k, v in host.items()}
-        h2d = sum(v.numel() * v.element_size() for v in pinned.values())
-        result = path.head_loss if use_head else path.loss  # L_total (Eq. 20), or the alignment loss
-        loss_host = torch.empty(result.numel(), dtype=torch.float32).pin_memory()
-        bufs = [devin, {k: torch.empty_like(v) for k, v in devin.items()}]
-        copy_stream = torch.cuda.Stream(device=dev)
-        copied = [torch.cuda.Event(), torch.cuda.Event()]
-        consumed = [torch.cuda.Event(), torch.cuda.Event()]
-
-        def copy_in(i):
-            b = i % 2
-            with torch.cuda.stream(copy_stream):
-                copy_stream.wait_event(consumed[b])  # the step that last read this buffer set is done
-                for k, v in pinned.items():
-                    bufs[b][k].copy_(v, non_blocking=True)
-                copied[b].record(copy_stream)
-
-        barrier()
-        torch.cuda.synchronize()
-        for ev in consumed:
-            ev.record(stream)
-        t0 = time.perf_counter()
-        copy_in(0)
-        for i in range(args.steps):
-            if i + 1 < args.steps:
-                copy_in(i + 1)
-            stream.wait_event(copied[i % 2])
-            step(bufs[i % 2])
-            consumed[i % 2].record(stream)
-            loss_host.copy_(result, non_blocking=True)
-            stream.synchronize()  # the loss of step i is on the host
-        torch.cuda.synchronize()
-        te = max_over_ranks(time.perf_counter() - t0)
-        e2e = {"value": weak_scaling_value(world, edges_per_step, args.steps, te), "unit": UNIT,
-               "h2d_bytes_per_step": int(h2d),
-               "d2h_bytes_per_step": int(loss_host.numel() * 4)}
-
+    res = run_hot_path(w, dev, args.steps, args.warmup, world, use_head, clocks=clocks, e2e=not args.no_e2e)
+    stats = graph_stats(w)
+    stats["n_lab"] = int(len(w["lab_idx"])) if use_head else 0
+    models = kernel_models(stats, sp)
+    head = workload_summary(w, res, models, args.steps, peaks, psrc)
+    rf, shares = roofline(res["report"], models, args.steps, peaks, psrc)
+    top = [k for k in shares if k in models and k != "gathered"][:8]
+    kernel_rooflines = [roofline(res["report"], models, args.steps, peaks, psrc, dom=k)[0] for k in top]
+    del w
+    free_device_memory()
     if rank != 0:
         if world > 1:
             torch.distributed.destroy_process_group()
         return
-    build = None
-    if not args.no_build:
-        build = measure_overlap_build(w, args.steps, args.warmup, dev, not args.no_cpu_baseline)
-    temporal = None
-    if not args.no_temporal:
-        temporal = measure_temporal(sp, args.steps, args.warmup, dev, not args.no_cpu_baseline)
-    hgt = None
-    if not args.no_hgt:
-        hgt = measure_hgt(w, args.steps, args.warmup, dev, not args.no_cpu_baseline)
-    peaks, psrc = load_peaks()
-    rf, shares = roofline(report, models, args.steps, peaks, psrc)
-    # the same figures for every modelled kernel among the largest shares
-    top = [k for k in shares if k in models and k != "compulsory"][:8]
-    kernel_rooflines = [roofline(report, models, args.steps, peaks, psrc, dom=k)[0] for k in top]
+    # the other workloads (fewer steps) and one pass over the ring
+    extra = {}
+    if not args.no_extra and args.scale == 1:
+        for name in EXTRA_WORKLOADS:
+            if name == sp.name:
+                continue
+            spx = hgsynth.spec(name)
+            wx = hd.make_workload(spx, device=dev, with_dH_top=not use_head)
+            rx = run_hot_path(wx, dev, min(args.steps, 5), min(max(args.warmup, 1), 2), 1, use_head)
+            stx = graph_stats(wx)
+            stx["n_lab"] = int(len(wx["lab_idx"])) if use_head else 0
+            extra[name] = workload_summary(wx, rx, kernel_models(stx, spx), min(args.steps, 5), peaks, psrc)
+            del wx
+            free_device_memory()
+        extra["ring16-2m"] = measure_ring(hgsynth.spec("ring16-2m"), dev, warmup=2)
+        free_device_memory()
+    side_needed = not (args.no_build and args.no_temporal and args.no_hgt)
+    ws = hd.make_workload(hgsynth.spec(SIDE_WORKLOAD), device=dev, with_dH_top=True) if side_needed else None
+    with_cpu = not args.no_cpu_baseline
+    build = None if args.no_build else measure_overlap_build(ws, args.steps, args.warmup, dev, with_cpu)
+    temporal = None if args.no_temporal else measure_temporal(hgsynth.spec(SIDE_WORKLOAD), args.steps, args.warmup,
+                                                                dev, with_cpu)
+    hgt = None if args.no_hgt else measure_hgt(ws, args.steps, args.warmup, dev, with_cpu)
+    del ws
     cpu = None
-    if not args.no_cpu_baseline:
-        o = time_oracle(sp.name, ORACLE_SCALE, with_head=use_head)
-        cpu = {"value": o["value"], "unit": UNIT, "cores": 1, "kind": "oracle",
-               "sample": f"1/{ORACLE_SCALE}-size instance of the workload ({o['edges']:,} edges, same recipe), one "
-                         f"full step of the fp64 numpy oracle{' with the head and joint loss' if use_head else ''}, "
-                         f"one thread, {o['seconds']:.1f} s"}
+    if with_cpu:
+        o = time_oracle(sp.name, sample_scale(sp), "step", with_head=use_head)
+        cpu = {"value": o["value"], "unit": UNIT, "cores": o["cores"], "kind": "oracle",
+               "sample": oracle_sample_text(o, "one full step" + (" with the head and joint loss" if use_head else ""))}
     out = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": 1e3 * t / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": sp.dtype, "data": "synthetic",
+        "metric": METRIC, "value": res["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": res["ms_per_step"], "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": sp.dtype, "data": "synthetic",
         "config": {"workload": workload_desc(sp), "l2": "inputs larger than L2 (not flushed)",
                    "parallelism": f"{world} independent subgraph(s), one per GPU",
-                   "objective": (f"L_BCE over {len(lab):,} labelled users + 0.1 L_CCA (head: MeanAgg, 2-layer MLP)"
+                   "generator": "hgsynth.device: the workload recipe drawn on the GPU (seeded)",
+                   "objective": ("L_BCE over the labelled users + 0.1 L_CCA (head: MeanAgg, 2-layer MLP)"
                                  if use_head else "synthetic upstream gradient + 0.1 L_CCA")},
         "roofline": rf, "kernel_rooflines": kernel_rooflines, "kernel_time_share": shares,
-        "phases_ms": {k: round(v, 4) for k, v in phase_ms.items()},
-        "layers_fwd_bwd_edges_per_s": edges_per_step / ((phase_ms.get("forward", 0) + phase_ms.get("backward", 0)) / 1e3)
-        if phase_ms else None,
-        "csr_build_edges_per_s": sp.num_edges / (phase_ms["graph"] / 1e3) if phase_ms.get("graph") else None,
-        "cpu_baseline": cpu, "e2e": e2e, "clocks": clk, "overlap_build": build, "temporal": temporal, "hgt": hgt,
-        "gpu_launches": int(sum(n for n, _ in report.values())),
-        "loss": [float(x) for x in path.loss.cpu()],
-        "head_loss": [float(x) for x in path.head_loss.cpu()] if use_head else None,
+        "phases_ms": res["phases_ms"],
+        "layers_fwd_bwd_edges_per_s": res["layers_fwd_bwd_edges_per_s"],
+        "layer_stack_roofline": head["layer_stack_roofline"],
+        "csr_build_edges_per_s": res["csr_build_edges_per_s"],
+        "cpu_baseline": cpu, "e2e": res.get("e2e"), "clocks": res["clocks"], "workloads": extra,
+        "overlap_build": build, "temporal": temporal, "hgt": hgt,
+        "gpu_launches": int(sum(n for n, _ in res["report"].values())),
+        "loss": res["loss"], "head_loss": res["head_loss"],
     }
     print(json.dumps(out))
     if world > 1:

@@ -92,10 +92,12 @@ hg_status hg_graph_workspace_size(int64_t num_edges, const int64_t* type_offsets
                                   const hg_rel_desc* rels, int32_t num_rels, size_t* bytes);
 
 /* Builds, on the device, per relation r: CSR by destination (rows = destination nodes of type
- * rels[r].dst_type in local order; each row lists its in-edges in ascending input edge id) and CSC
- * by source (rows = source nodes of type rels[r].src_type; out-edges in ascending edge id), plus
- * the per-CSC-edge coefficient 1/deg_r(destination) as an IEEE fp32 quotient, and the split tables
- * the aggregation kernels use for high-degree rows.
+ * rels[r].dst_type in local order; each row lists its in-edges by ascending (source id, input edge
+ * id)) and CSC by source (rows = source nodes of type rels[r].src_type; out-edges by ascending
+ * (destination id, edge id)), plus the per-CSC-edge coefficient 1/deg_r(destination) as an IEEE
+ * fp32 quotient, the split tables the aggregation kernels use for high-degree rows, and the
+ * aggregation lists of the mean layer, in which the parallel edges of a node pair (adjacent in
+ * that order) are one entry with their multiplicity.
  *   src, dst, rel : device int32 arrays of num_edges entries (COO, any order).
  *   type_offsets  : host int64 [num_types + 1], type_offsets[0] = 0, non-decreasing.
  *   rels          : host [num_rels].

@@ -33,8 +33,9 @@ Readings where the paper is silent or ambiguous (listed again in the design note
   variance; both loss terms are plain sums (squared Frobenius norms); lambda_n = 2e-4.
 
 Storage precision of intermediates (store="bf16").  For bf16 workloads the kernels store the
-relation means M_r in bf16 and the pre-activation U in bf16 (the activation and its derivative
-are taken at the stored U); weights, and products of weights, are never rounded.  The ReLU mask
+relation means M_r in bf16 and the pre-activation without its bias, Z W_agg, in bf16 (the
+activation and its derivative are taken at that stored value plus the bias); weights, and
+products of weights, are never rounded.  The ReLU mask
 is an integer decision made by floating point, and the paper fixes no precision; where a
 pre-activation lies within a rounding of zero either mask is a valid outcome.  store="bf16"
 rounds M_r and U to bf16 (round to nearest, ties to even; its own rounding routine) and keeps
@@ -95,7 +96,9 @@ def valid_edges(src, dst, rel, type_offsets, rels) -> np.ndarray:
 def build_csr(src, dst, rel, type_offsets, rels) -> list:
     """Per relation r: CSR by destination (row_ptr over the n_t destination rows, col = source node
     id, eid) and CSC by source (csc_ptr over the n_s source rows, csc_col = destination node id,
-    csc_eid, csc_coef = fp32 1/deg_r(destination)).  Row order: local id within the type."""
+    csc_eid, csc_coef = fp32 1/deg_r(destination)).  Row order: local id within the type.  Within a
+    CSR row the in-edges ascend by (source id, edge id), within a CSC row the out-edges by
+    (destination id, edge id), so the parallel edges of a node pair are adjacent."""
     src = np.asarray(src, np.int64)
     dst = np.asarray(dst, np.int64)
     rel = np.asarray(rel, np.int64)
@@ -107,11 +110,11 @@ def build_csr(src, dst, rel, type_offsets, rels) -> list:
         n_t = int(offs[tt + 1] - offs[tt])
         eids = np.flatnonzero(ok & (rel == r))  # ascending edge id
         dl = dst[eids] - offs[tt]
-        by_dst = eids[np.argsort(dl, kind="stable")]
+        sl = src[eids] - offs[ts]
+        by_dst = eids[np.argsort(dl * n_s + sl, kind="stable")]  # (destination, source, edge id)
         deg = np.bincount(dl, minlength=n_t)
         row_ptr = np.concatenate([[0], np.cumsum(deg)]).astype(np.int64)
-        sl = src[eids] - offs[ts]
-        by_src = eids[np.argsort(sl, kind="stable")]
+        by_src = eids[np.argsort(sl * n_t + dl, kind="stable")]  # (source, destination, edge id)
         odeg = np.bincount(sl, minlength=n_s)
         csc_ptr = np.concatenate([[0], np.cumsum(odeg)]).astype(np.int64)
         coef = np.float32(1.0) / deg[dst[by_src] - offs[tt]].astype(np.float32)
@@ -178,7 +181,7 @@ def layer_forward(csr: list, type_offsets, rels, params: dict, H, act: str = "re
             M = _stored(mean_aggregate(csr[r], H), store)
             cache["M"][r] = M
             Z += M @ p["W_rel"][r]
-        U = _stored(Z @ p["W_agg"][t] + p["b_agg"][t], store)
+        U = _stored(Z @ p["W_agg"][t], store) + p["b_agg"][t]  # U is stored without its bias
         Y = act_fwd(U, act) + H[lo:hi]
         c = {"Z": Z, "U": U, "Y": Y}
         if layernorm:
@@ -279,7 +282,7 @@ def layer_forward_rows(src, dst, rel, type_offsets, rels, params, H, rows, act="
     for r in range(R):
         m = ty == rt[r]
         Z[m] += M[m, r] @ p["W_rel"][r]
-    U = _stored(np.einsum("nk,nkj->nj", Z, p["W_agg"][ty]) + p["b_agg"][ty], store)
+    U = _stored(np.einsum("nk,nkj->nj", Z, p["W_agg"][ty]), store) + p["b_agg"][ty]
     Y = act_fwd(U, act) + np.asarray(H, F64)[rows]
     cache = dict(M=M, Z=Z, U=U, Y=Y, deg=deg, ty=ty)
     if layernorm:
@@ -419,10 +422,14 @@ def overlap_intersect(gid_a, gid_b) -> tuple:
 # one whole step of the hot path (used for the CPU baseline and small end-to-end checks)
 # ----------------------------------------------------------------------------------------------
 def step(graph: dict, X, params: list, dH_top, view_b: dict, act="relu", layernorm=True,
-         ln_eps=1e-5, lambda_n=2e-4, var_eps=1e-8, dloss=0.1, store="f64", head: dict | None = None) -> dict:
+         ln_eps=1e-5, lambda_n=2e-4, var_eps=1e-8, dloss=0.1, store="f64", head: dict | None = None,
+         interface: str = "f64") -> dict:
     """CSR build -> L layers forward -> overlap rows -> alignment loss and gradient -> L layers
-    backward (view_b None: no alignment term, as for the first subgraph of a sequence).  With store="bf16" the tensors handed from layer to layer (outputs, their gradients)
-    are rounded to bf16 as well, like every bf16 tensor the layer interface exchanges.  `view_b` is either {"H_b": bank rows, "gid_a", "gid_b"} (a detached neighbour view)
+    backward (view_b None: no alignment term, as for the first subgraph of a sequence).
+    interface="bf16": the tensors handed from layer to layer (each layer's output, and the gradient
+    with respect to it) are rounded to bf16, the storage type of every tensor the layer interface
+    exchanges for a bf16 workload; the layers' own arithmetic stays as `store` says (fp64 by
+    default).  store="bf16" implies interface="bf16".  `view_b` is either {"H_b": bank rows, "gid_a", "gid_b"} (a detached neighbour view)
     or {"idx": overlap rows, "X_b": second input} (a second live stack on the same graph).
     The last layer's upstream gradient is dH_top plus the alignment gradient.  With `head`
     ({"params", "lab_idx", "lab_y"}) the head's gradient (MeanAgg, MLP, masked BCE; Eq. 18-19)
@@ -432,7 +439,7 @@ def step(graph: dict, X, params: list, dH_top, view_b: dict, act="relu", layerno
     csr = build_csr(graph["src"], graph["dst"], graph["rel"], offs, rels)
 
     # layer outputs and gradients passed between layers are tensors of the storage type
-    io = (lambda x: x) if store == "f64" else round_bf16
+    io = round_bf16 if (store == "bf16" or interface == "bf16") else (lambda x: x)
 
     def run_stack(H0):
         hs = [np.asarray(H0, F64)]

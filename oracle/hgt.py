@@ -29,7 +29,7 @@ Readings where the paper is silent or ambiguous (listed again in the design note
   residual needs d_in = d_out; LayerNorm after the residual (population variance, eps 1e-5).
   store="bf16": the tensors the bf16 kernels store -- K, V, Q, the relation-scaled queries
   Q'_r(j) = Q(j) blockdiag(W_att[r])^T mu[r] / sqrt(d_h), the per-relation weighted sums
-  S_r(j) = sum over the r-edges into j of alpha V(i), and U -- are rounded to bf16; weights and
+  S_r(j) = sum over the r-edges into j of alpha V(i), and U without its bias -- are rounded to bf16; weights and
   products of weights are not; all other arithmetic stays fp64.  The GPU tests compare with the
   plain definition (store="f64"); this mode serves to study the effect of those roundings.
 """
@@ -114,7 +114,7 @@ def hgt_forward(src, dst, rel, type_offsets, rels, params: dict, H, heads: int, 
             if tt == t:
                 Vr = blockdiag(P["W_msg"][r]) @ P["W_agg"][t]
                 u += Ssum[r, lo:hi] @ Vr
-        U[lo:hi] = rnd(u + P["b_agg"][t])
+        U[lo:hi] = rnd(u) + P["b_agg"][t]  # stored without its bias, as the kernels do
     Y = act_fwd(U, act) + H
     out = Y
     mean = rstd = None

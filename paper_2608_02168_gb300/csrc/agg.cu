@@ -7,6 +7,10 @@
 //           backward kernel, and dY[i] is the residual-path gradient of Eq. 11.  The sum runs over
 //           node i's row of the node-major out-edge list (its CSC rows of every relation leaving
 //           its type, concatenated in relation order, each edge holding the dMs row it reads).
+// Parallel edges (the same source, destination and relation) are summed once with their
+// multiplicity: the rows read here are the build's runs (column, count), so each distinct
+// neighbour row is gathered once per row and multiplied by its count (deg_r(j) is still the
+// number of edges, the CSR row length).
 //
 // Mapping: one group of G lanes per row, each lane owning 16-byte slices of the feature row
 // (G = d * sizeof(T) / 16, at most 32), gathers with 128-bit loads and eight neighbour rows in
@@ -33,20 +37,24 @@ struct AggShape {
   static constexpr int kGroups = kThreads / G;
 };
 
-// acc += sum of rows src[col[e] + delta] for e = beg, beg + stride, ... < end, added in edge
+// acc += sum of cnt[e] * src[col[e] + delta] for e = beg, beg + stride, ... < end, added in run
 // order; eight neighbour rows are loaded before they are added.
 template <typename T, int D, bool kBatchTail = true>
-__device__ __forceinline__ void gather_sum(const int32_t* __restrict__ col, int64_t beg, int64_t end,
-                                           int stride, int64_t delta, const T* __restrict__ src,
-                                           int lane, float* acc) {
+__device__ __forceinline__ void gather_sum(const int32_t* __restrict__ col, const int32_t* __restrict__ cnt,
+                                           int64_t beg, int64_t end, int stride, int64_t delta,
+                                           const T* __restrict__ src, int lane, float* acc) {
   using S = AggShape<T, D>;
   constexpr int U = 8;
   const T* base = src + delta * D + lane * S::kVec;
   int64_t e = beg;
   for (; e + (U - 1) * (int64_t)stride < end; e += U * (int64_t)stride) {
     int c[U];
+    float w[U];
 #pragma unroll
-    for (int u = 0; u < U; ++u) c[u] = __ldg(col + e + u * stride);
+    for (int u = 0; u < U; ++u) {
+      c[u] = __ldg(col + e + u * stride);
+      w[u] = (float)__ldg(cnt + e + u * stride);
+    }
     uint4 x[U][S::V];
 #pragma unroll
     for (int u = 0; u < U; ++u)
@@ -59,24 +67,30 @@ __device__ __forceinline__ void gather_sum(const int32_t* __restrict__ col, int6
         float f[S::kVec];
         unpack(x[u][v], f, T());
 #pragma unroll
-        for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] += f[q];
+        for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] = fmaf(w[u], f[q], acc[v * S::kVec + q]);
       }
   }
   if (!kBatchTail) {
     for (; e < end; e += stride) {
       const int c = __ldg(col + e);
+      const float w = (float)__ldg(cnt + e);
 #pragma unroll
       for (int v = 0; v < S::V; ++v) {
         float f[S::kVec];
         unpack(ldg16(base + (int64_t)c * D + v * S::G * S::kVec), f, T());
 #pragma unroll
-        for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] += f[q];
+        for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] = fmaf(w, f[q], acc[v * S::kVec + q]);
       }
     }
   } else if (e < end) {  // the last (fewer than U) rows as one predicated batch
     int c[U];
+    float w[U];
 #pragma unroll
-    for (int u = 0; u < U; ++u) c[u] = e + u * (int64_t)stride < end ? __ldg(col + e + u * stride) : -1;
+    for (int u = 0; u < U; ++u) {
+      const bool in = e + u * (int64_t)stride < end;
+      c[u] = in ? __ldg(col + e + u * stride) : -1;
+      w[u] = in ? (float)__ldg(cnt + e + u * stride) : 0.f;
+    }
     uint4 x[U][S::V];
 #pragma unroll
     for (int u = 0; u < U; ++u)
@@ -91,7 +105,7 @@ __device__ __forceinline__ void gather_sum(const int32_t* __restrict__ col, int6
         float f[S::kVec];
         unpack(x[u][v], f, T());
 #pragma unroll
-        for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] += f[q];
+        for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] = fmaf(w[u], f[q], acc[v * S::kVec + q]);
       }
     }
   }
@@ -187,9 +201,11 @@ __device__ __forceinline__ void store_row(T* __restrict__ dst, int lane, const f
   }
 }
 
-// One CTA per chunk (grid-stride over the chunk list): fp32 partial sum of the chunk's rows.
+// One CTA per chunk of kChunkEdges runs (grid-stride over the chunk list): fp32 partial sum of the
+// chunk's rows, each times its multiplicity.
 template <typename T, int D>
 __global__ void __launch_bounds__(256) agg_chunks(const int32_t* __restrict__ ptr, const int32_t* __restrict__ col,
+                                                  const int32_t* __restrict__ cnt,
                                                   const T* __restrict__ src, const int32_t* __restrict__ chunk_row,
                                                   const int32_t* __restrict__ chunk_ofs, int64_t rows,
                                                   float* __restrict__ partials) {
@@ -204,7 +220,7 @@ __global__ void __launch_bounds__(256) agg_chunks(const int32_t* __restrict__ pt
     float acc[S::F];
 #pragma unroll
     for (int q = 0; q < S::F; ++q) acc[q] = 0.f;
-    gather_sum<T, D, false>(col, beg + grp, end, S::kGroups, 0, src, lane, acc);
+    gather_sum<T, D, false>(col, cnt, beg + grp, end, S::kGroups, 0, src, lane, acc);
 #pragma unroll
     for (int v = 0; v < S::V; ++v)
 #pragma unroll
@@ -221,11 +237,11 @@ __global__ void __launch_bounds__(256) agg_chunks(const int32_t* __restrict__ pt
 }
 
 // The backward node kernel runs a two-deep pipeline per group: while node i gathers, the first
-// kFirst indices of node i + step and the bounds of node i + 2 step are in flight, so a short
+// kFirst runs of node i + step and the bounds of node i + 2 step are in flight, so a short
 // row's gathers are issued without waiting on an index load.  Indices past the row's end, and
 // those of a row that takes the chunk path, are -1.  (The forward row kernel keeps a plain scalar
 // loop over short rows: with the extra registers of the pipeline it ran slower.)
-constexpr int kFirst = 8;
+constexpr int kFirst = 4;  // a node row averages 3-4 runs once parallel edges are coalesced
 
 __device__ __forceinline__ void load_first(const int32_t* __restrict__ col, int beg, int end, int* c) {
   const bool small = end - beg <= kHubDegree;
@@ -236,10 +252,13 @@ __device__ __forceinline__ void load_first(const int32_t* __restrict__ col, int 
 // acc += the rows of the preloaded first indices c (in order), then the row's edges from
 // beg + kFirst on, so every row is still summed in edge order.
 template <typename T, int D, bool kBatchTail>
-__device__ __forceinline__ void gather_row(const int32_t* __restrict__ col, int beg, int end, const int* c,
-                                           const T* __restrict__ src, int lane, float* acc) {
+__device__ __forceinline__ void gather_row(const int32_t* __restrict__ col, const int32_t* __restrict__ cnt, int beg,
+                                           int end, const int* c, const T* __restrict__ src, int lane, float* acc) {
   using S = AggShape<T, D>;
   const T* base = src + lane * S::kVec;
+  float w[kFirst];  // multiplicities: loaded beside the rows (they depend only on beg)
+#pragma unroll
+  for (int u = 0; u < kFirst; ++u) w[u] = c[u] >= 0 ? (float)__ldg(cnt + beg + u) : 0.f;
   uint4 x[kFirst][S::V];
 #pragma unroll
   for (int u = 0; u < kFirst; ++u)
@@ -254,48 +273,53 @@ __device__ __forceinline__ void gather_row(const int32_t* __restrict__ col, int 
       float f[S::kVec];
       unpack(x[u][v], f, T());
 #pragma unroll
-      for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] += f[q];
+      for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] = fmaf(w[u], f[q], acc[v * S::kVec + q]);
     }
   }
-  if (end - beg > kFirst) gather_sum<T, D, kBatchTail>(col, beg + kFirst, end, 1, 0, src, lane, acc);
+  if (end - beg > kFirst) gather_sum<T, D, kBatchTail>(col, cnt, beg + kFirst, end, 1, 0, src, lane, acc);
 }
 
-// Forward rows: M[row] = mean over the row's neighbours (concatenated CSR rows of all relations).
-// Persistent: each group strides over rows and fetches the next row's bounds while it gathers.
+// Forward rows: M[row] = mean over the row's neighbours: the row's runs (column, multiplicity),
+// divided by the row's edge count deg (the CSR row length).  Persistent: each group strides over
+// rows and fetches the next row's bounds while it gathers.
 template <typename T, int D>
 __global__ void __launch_bounds__(256) agg_fwd_rows(const int32_t* __restrict__ ptr, const int32_t* __restrict__ col,
-                                                    const T* __restrict__ H, T* __restrict__ M, int64_t rows,
+                                                    const int32_t* __restrict__ cnt,
+                                                    const int32_t* __restrict__ eptr, const T* __restrict__ H,
+                                                    T* __restrict__ M, int64_t rows,
                                                     const int32_t* __restrict__ chunk_ofs,
                                                     const float* __restrict__ partials) {
   using S = AggShape<T, D>;
   const int grp = threadIdx.x / S::G, lane = threadIdx.x % S::G;
   const int64_t step = (int64_t)gridDim.x * S::kGroups;
   int64_t row = (int64_t)blockIdx.x * S::kGroups + grp;
-  int beg = 0, end = 0;
+  int beg = 0, end = 0, deg = 0;
   if (row < rows) {
     beg = __ldg(ptr + row);
     end = __ldg(ptr + row + 1);
+    deg = __ldg(eptr + row + 1) - __ldg(eptr + row);
   }
   while (row < rows) {
     const int64_t nrow = row + step;
-    int nbeg = 0, nend = 0;
+    int nbeg = 0, nend = 0, ndeg = 0;
     if (nrow < rows) {
       nbeg = __ldg(ptr + nrow);
       nend = __ldg(ptr + nrow + 1);
+      ndeg = __ldg(eptr + nrow + 1) - __ldg(eptr + nrow);
     }
-    const int deg = end - beg;
     float acc[S::F];
 #pragma unroll
     for (int q = 0; q < S::F; ++q) acc[q] = 0.f;
-    if (deg > kHubDegree)
+    if (end - beg > kHubDegree)
       add_partials<T, D>(partials, chunk_ofs[row], chunk_ofs[row + 1], lane, acc);
     else
-      gather_sum<T, D, false>(col, beg, end, 1, 0, H, lane, acc);
+      gather_sum<T, D, false>(col, cnt, beg, end, 1, 0, H, lane, acc);
     const float scale = deg > 0 ? __fdiv_rn(1.0f, (float)deg) : 0.f;
     store_row<T, D>(M + row * D, lane, acc, scale);
     row = nrow;
     beg = nbeg;
     end = nend;
+    deg = ndeg;
   }
 }
 
@@ -304,7 +328,8 @@ __global__ void __launch_bounds__(256) agg_fwd_rows(const int32_t* __restrict__ 
 // Persistent: each group strides over nodes (pipelined as above).
 template <typename T, int D>
 __global__ void __launch_bounds__(256, 4) agg_bwd_nodes(int64_t N, const int32_t* __restrict__ nptr,
-                                                     const int32_t* __restrict__ ncol, const T* __restrict__ dMs,
+                                                     const int32_t* __restrict__ ncol,
+                                                     const int32_t* __restrict__ ncnt, const T* __restrict__ dMs,
                                                      const T* __restrict__ dY, T* __restrict__ dH,
                                                      const int32_t* __restrict__ chunk_ofs,
                                                      const float* __restrict__ partials) {
@@ -343,7 +368,7 @@ __global__ void __launch_bounds__(256, 4) agg_bwd_nodes(int64_t N, const int32_t
     if (end - beg > kHubDegree)
       add_partials<T, D>(partials, chunk_ofs[node], chunk_ofs[node + 1], lane, acc);
     else
-      gather_row<T, D, true>(ncol, beg, end, c, dMs, lane, acc);
+      gather_row<T, D, true>(ncol, ncnt, beg, end, c, dMs, lane, acc);
     store_row<T, D>(dH + node * D, lane, acc, 1.0f);
     node += step;
     beg = nbeg;
@@ -375,17 +400,18 @@ template <typename T, int D>
 static hg_status agg_fwd_t(const hg_graph* g, const void* H, void* M, float* partials, cudaStream_t s) {
   using S = AggShape<T, D>;
   HG_TRY(launch("agg_fwd_chunks", agg_chunks<T, D>, dim3(chunk_grid(g->chunk_cap_csr)), dim3(256), 0, s,
-                (const int32_t*)g->csr_ptr, (const int32_t*)g->csr_col, (const T*)H,
-                (const int32_t*)g->csr_chunk_row, (const int32_t*)g->csr_chunk_ofs, g->csr_rows, partials));
+                (const int32_t*)g->agg_ptr, (const int32_t*)g->agg_col, (const int32_t*)g->agg_cnt, (const T*)H,
+                (const int32_t*)g->agg_chunk_row, (const int32_t*)g->agg_chunk_ofs, g->csr_rows, partials));
   HG_TRY(launch("combine_chunk_partials", combine_chunk_partials<D>, dim3(chunk_grid(g->chunk_cap_csr)), dim3(D), 0, s,
-                (const int32_t*)g->csr_chunk_row, (const int32_t*)g->csr_chunk_ofs, g->csr_rows, partials));
+                (const int32_t*)g->agg_chunk_row, (const int32_t*)g->agg_chunk_ofs, g->csr_rows, partials));
   static int64_t pb = 0;
   if (pb == 0) HG_TRY(persist_blocks(agg_fwd_rows<T, D>, &pb));
   return launch("agg_fwd_rows", agg_fwd_rows<T, D>,
                 dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(g->csr_rows, S::kGroups), pb))),
                 dim3(256),
-                0, s, (const int32_t*)g->csr_ptr, (const int32_t*)g->csr_col, (const T*)H, (T*)M, g->csr_rows,
-                (const int32_t*)g->csr_chunk_ofs, (const float*)partials);
+                0, s, (const int32_t*)g->agg_ptr, (const int32_t*)g->agg_col, (const int32_t*)g->agg_cnt,
+                (const int32_t*)g->csr_ptr, (const T*)H, (T*)M, g->csr_rows, (const int32_t*)g->agg_chunk_ofs,
+                (const float*)partials);
 }
 
 template <typename T, int D>
@@ -394,16 +420,16 @@ static hg_status agg_bwd_t(const hg_graph* g, const void* dMs, const void* dY, v
   using S = AggShape<T, D>;
   const int64_t N = g->meta.type_off[g->meta.num_types];
   HG_TRY(launch("agg_bwd_chunks", agg_chunks<T, D>, dim3(chunk_grid(g->chunk_cap_node)), dim3(256), 0, s,
-                (const int32_t*)g->node_ptr, (const int32_t*)g->node_col, (const T*)dMs,
-                (const int32_t*)g->node_chunk_row, (const int32_t*)g->node_chunk_ofs, N, partials));
+                (const int32_t*)g->bagg_ptr, (const int32_t*)g->bagg_col, (const int32_t*)g->bagg_cnt, (const T*)dMs,
+                (const int32_t*)g->bagg_chunk_row, (const int32_t*)g->bagg_chunk_ofs, N, partials));
   HG_TRY(launch("combine_chunk_partials", combine_chunk_partials<D>, dim3(chunk_grid(g->chunk_cap_node)), dim3(D), 0,
-                s, (const int32_t*)g->node_chunk_row, (const int32_t*)g->node_chunk_ofs, N, partials));
+                s, (const int32_t*)g->bagg_chunk_row, (const int32_t*)g->bagg_chunk_ofs, N, partials));
   static int64_t pb = 0;
   if (pb == 0) HG_TRY(persist_blocks(agg_bwd_nodes<T, D>, &pb));
   return launch("agg_bwd_nodes", agg_bwd_nodes<T, D>,
                 dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(N, S::kGroups), pb))), dim3(256), 0, s,
-                N, (const int32_t*)g->node_ptr, (const int32_t*)g->node_col, (const T*)dMs, (const T*)dY, (T*)dH,
-                (const int32_t*)g->node_chunk_ofs, (const float*)partials);
+                N, (const int32_t*)g->bagg_ptr, (const int32_t*)g->bagg_col, (const int32_t*)g->bagg_cnt,
+                (const T*)dMs, (const T*)dY, (T*)dH, (const int32_t*)g->bagg_chunk_ofs, (const float*)partials);
 }
 
 #define HG_DISPATCH_TD(dtype, d, FN, ...)                                                   \

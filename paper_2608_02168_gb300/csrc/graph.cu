@@ -261,7 +261,7 @@ __global__ void __launch_bounds__(kSortThreads) radix_scatter(
 }
 
 struct SortBuffers {
-  uint32_t* ckeys;  // CSC keys, written together with the CSR keys
+  uint32_t* ckeys;  // CSR row keys (payload of the first sort), then the CSC keys
   uint32_t* keys[2];
   uint32_t* vals[2];
   uint32_t* vals2[2];  // second payload (carried so the finish passes read sequentially)
@@ -273,20 +273,20 @@ static int64_t sort_tiles(int64_t n) { return std::max<int64_t>(1, ceil_div(n, k
 // dynamic shared memory of radix_scatter<true>: the sorted tile (key, value, payload), warp histograms
 constexpr size_t kScatterSmem = 3 * kSortTile * sizeof(uint32_t) + kSortWarps * kRadix * sizeof(int);
 
-// Sorts (key, input position, second payload) by the low `bits` key bits (at least one pass), the
-// keys first read from keys_src and the payload from vals2_src; returns the buffer index holding
-// the result.
-static hg_status radix_sort(SortBuffers& b, int64_t n, int bits, const uint32_t* keys_src, const uint32_t* vals2_src,
-                            cudaStream_t s, int* result) {
+// Sorts (key, value, second payload) triples by the low `bits` key bits (at least one pass), stable.
+// The first pass reads keys_src, vals_src (null: the input positions) and vals2_src, which may lie
+// in buffer `start` (it writes buffer start ^ 1 first); returns the buffer index holding the result.
+static hg_status radix_sort(SortBuffers& b, int64_t n, int bits, const uint32_t* keys_src, const uint32_t* vals_src,
+                            const uint32_t* vals2_src, int start, cudaStream_t s, int* result) {
   static bool attr = false;
   if (!attr) {
     HG_CUDA(cudaFuncSetAttribute(radix_scatter<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kScatterSmem));
     attr = true;
   }
-  int cur = 0;
+  int cur = start;
   const int64_t tiles = sort_tiles(n);
   const uint32_t* k = keys_src;
-  const uint32_t* v = nullptr;  // first pass: values are the input positions
+  const uint32_t* v = vals_src;
   const uint32_t* v2 = vals2_src;
   for (int shift = 0; shift < std::max(bits, 1); shift += 8) {
     HG_TRY(launch("radix_hist", radix_hist, dim3((unsigned)tiles), dim3(kSortThreads), 0, s, k, n, shift, b.hist,
@@ -306,14 +306,15 @@ static hg_status radix_sort(SortBuffers& b, int64_t n, int bits, const uint32_t*
 // ---------------------------------------------------------------------------------------------
 // CSR / CSC kernels
 // ---------------------------------------------------------------------------------------------
-// Row keys of every edge in both layouts: CSR key = destination row, CSC key = source row;
-// invalid edges (relation or endpoint out of range, endpoint of the wrong type) get the sentinel
-// key past the last row.  The relation tables are read from shared memory.
+// Keys of the first sort: the source node id of every valid edge (0 for invalid ones), and, as its
+// payload, the CSR row key (destination row; the sentinel past the last row for an invalid edge:
+// relation or endpoint out of range, endpoint of the wrong type).  The relation tables are read
+// from shared memory.
 __global__ void __launch_bounds__(256) edge_keys(const int32_t* __restrict__ src, const int32_t* __restrict__ dst,
                                                  const int32_t* __restrict__ rel, int64_t E, GraphMeta m,
-                                                 int64_t rows, int64_t crows, uint32_t* __restrict__ keys,
-                                                 uint32_t* __restrict__ ckeys) {
-  __shared__ int64_t row0[kMaxRels], crow0[kMaxRels];  // first row of relation r minus its type offset
+                                                 int64_t rows, uint32_t* __restrict__ skeys,
+                                                 uint32_t* __restrict__ rkeys) {
+  __shared__ int64_t row0[kMaxRels];  // first row of relation r minus its destination type's offset
   __shared__ int32_t rsrc[kMaxRels], rdst[kMaxRels];
   if (threadIdx.x < kMaxRels) {
     const int r = threadIdx.x;
@@ -321,7 +322,6 @@ __global__ void __launch_bounds__(256) edge_keys(const int32_t* __restrict__ src
       rsrc[r] = m.rel_src[r];
       rdst[r] = m.rel_dst[r];
       row0[r] = m.row_base[r] - m.type_off[m.rel_dst[r]];
-      crow0[r] = m.csc_base[r] - m.type_off[m.rel_src[r]];
     }
   }
   __syncthreads();
@@ -330,14 +330,83 @@ __global__ void __launch_bounds__(256) edge_keys(const int32_t* __restrict__ src
     const int r = rel[e];
     const int64_t sn = src[e], tn = dst[e];
     bool ok = r >= 0 && r < m.num_rels && sn >= 0 && sn < N && tn >= 0 && tn < N;
-    int64_t key = rows, ckey = crows;  // invalid edges sort after every row
-    if (ok && node_type_of(m, sn) == rsrc[r] && node_type_of(m, tn) == rdst[r]) {
-      key = row0[r] + tn;
-      ckey = crow0[r] + sn;
-    }
-    keys[e] = (uint32_t)key;
-    ckeys[e] = (uint32_t)ckey;
+    int64_t key = rows;  // invalid edges sort after every row
+    if (ok && node_type_of(m, sn) == rsrc[r] && node_type_of(m, tn) == rdst[r]) key = row0[r] + tn;
+    else ok = false;
+    skeys[e] = ok ? (uint32_t)sn : 0u;
+    rkeys[e] = (uint32_t)key;
   }
+}
+
+// Keys of the CSC sort, read off the CSR order (row key, source id) position by position: the CSC
+// row (relation, source) of each valid edge and its destination node id; invalid edges (positions
+// from ptr[rows] on) get the sentinel past the last CSC row.  A stable sort of the CSR order by
+// these keys lists each CSC row by (destination, edge id).  dst_out may alias rkey (each position
+// is read before it is written, by the same thread).
+__global__ void csc_keys_from_csr(const uint32_t* rkey, const uint32_t* __restrict__ srcs, int64_t E,
+                                  const int32_t* __restrict__ ptr, int64_t rows, int64_t crows, GraphMeta m,
+                                  uint32_t* __restrict__ ckey, uint32_t* dst_out) {
+  const int64_t nv = ptr[rows];
+  for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < E; p += (int64_t)gridDim.x * blockDim.x) {
+    if (p >= nv) {
+      ckey[p] = (uint32_t)crows;
+      dst_out[p] = 0u;
+      continue;
+    }
+    const int64_t key = rkey[p];
+    int r = 0;
+#pragma unroll
+    for (int k = 1; k < kMaxRels; ++k)
+      if (k < m.num_rels && key >= m.row_base[k]) r = k;
+    const int64_t d = m.type_off[m.rel_dst[r]] + (key - m.row_base[r]);
+    ckey[p] = (uint32_t)(m.csc_base[r] + ((int64_t)srcs[p] - m.type_off[m.rel_src[r]]));
+    dst_out[p] = (uint32_t)d;
+  }
+}
+
+// ---------------------------------------------------------------------------------------------
+// run-length coalescing of parallel edges: a row (ptr, col) whose equal entries are adjacent
+// becomes (uptr, ucol, ucnt): one entry per distinct column with its multiplicity, in the same order
+// ---------------------------------------------------------------------------------------------
+// flag[p] = 1 where a run starts: p = 0 or col[p] != col[p - 1] (row starts are added next), for
+// p < ptr[rows]; 0 up to cap (the capacity the scan runs over).
+__global__ void run_flags(const int32_t* __restrict__ col, const int32_t* __restrict__ ptr, int64_t rows, int64_t cap,
+                          int32_t* __restrict__ flag) {
+  const int64_t n = ptr[rows];
+  for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < cap; p += (int64_t)gridDim.x * blockDim.x)
+    flag[p] = (p < n && (p == 0 || col[p] != col[p - 1])) ? 1 : 0;
+}
+
+// every non-empty row starts a run
+__global__ void run_row_starts(const int32_t* __restrict__ ptr, int64_t rows, int32_t* __restrict__ flag) {
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < rows; r += (int64_t)gridDim.x * blockDim.x)
+    if (ptr[r + 1] > ptr[r]) flag[ptr[r]] = 1;
+}
+
+// With u = the exclusive scan of the flags (u[n] = number of runs): run k = u[p] of a flagged
+// position p gets ucol[k] = col[p] and its start upos[k] = p; upos[U] = n.
+__global__ void run_write(const int32_t* __restrict__ flag, const int32_t* __restrict__ u,
+                          const int32_t* __restrict__ col, const int32_t* __restrict__ ptr, int64_t rows,
+                          int32_t* __restrict__ ucol, int32_t* __restrict__ upos) {
+  const int64_t n = ptr[rows];
+  for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p <= n; p += (int64_t)gridDim.x * blockDim.x) {
+    if (p == n) {
+      upos[u[n]] = (int32_t)n;
+    } else if (flag[p]) {
+      ucol[u[p]] = col[p];
+      upos[u[p]] = (int32_t)p;
+    }
+  }
+}
+
+// ucnt[k] = upos[k + 1] - upos[k] (the run's length) for k < U; uptr[r] = u[ptr[r]] for r <= rows.
+__global__ void run_finish(const int32_t* __restrict__ u, const int32_t* __restrict__ upos,
+                           const int32_t* __restrict__ ptr, int64_t rows, int32_t* __restrict__ ucnt,
+                           int32_t* __restrict__ uptr) {
+  const int64_t U = u[ptr[rows]];
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < U; k += stride) ucnt[k] = upos[k + 1] - upos[k];
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r <= rows; r += stride) uptr[r] = u[ptr[r]];
 }
 
 // Row pointers from the sorted keys: ptr[k] = first position whose key is >= k, k in [0, rows].
@@ -446,6 +515,9 @@ struct GraphLayout {
   float* csc_coef;
   int32_t *node_ptr, *node_col;  // node-major out-edges (dMs rows) for the backward aggregation
   int32_t *csr_chunk_ofs, *csr_chunk_row, *node_chunk_ofs, *node_chunk_row, *invalid, *cnt;
+  // parallel edges coalesced: CSR rows and node-major rows as (column, multiplicity) runs
+  int32_t *agg_ptr, *agg_col, *agg_cnt, *agg_chunk_ofs, *agg_chunk_row;
+  int32_t *bagg_ptr, *bagg_col, *bagg_cnt, *bagg_chunk_ofs, *bagg_chunk_row;
   SortBuffers sort;
 };
 
@@ -465,17 +537,28 @@ static size_t carve_graph(void* ws, int64_t E, int64_t rows, int64_t crows, int6
   L->csr_chunk_row = c.take<int32_t>(chunk_cap(E));
   L->node_chunk_ofs = c.take<int32_t>(N + 1);
   L->node_chunk_row = c.take<int32_t>(chunk_cap(E));
+  L->agg_ptr = c.take<int32_t>(rows + 1);
+  L->agg_col = c.take<int32_t>(Ea);
+  L->agg_cnt = c.take<int32_t>(Ea);
+  L->agg_chunk_ofs = c.take<int32_t>(rows + 1);
+  L->agg_chunk_row = c.take<int32_t>(chunk_cap(E));
+  L->bagg_ptr = c.take<int32_t>(N + 1);
+  L->bagg_col = c.take<int32_t>(Ea);
+  L->bagg_cnt = c.take<int32_t>(Ea);
+  L->bagg_chunk_ofs = c.take<int32_t>(N + 1);
+  L->bagg_chunk_row = c.take<int32_t>(chunk_cap(E));
   L->invalid = c.take<int32_t>(1);
   L->cnt = c.take<int32_t>(std::max(std::max(rows, crows), N) + 1);
-  L->sort.ckeys = c.take<uint32_t>(Ea);
-  for (int i = 0; i < 2; ++i) {
-    L->sort.keys[i] = c.take<uint32_t>(Ea);
-    L->sort.vals[i] = c.take<uint32_t>(Ea);
-    L->sort.vals2[i] = c.take<uint32_t>(Ea);
+  L->sort.ckeys = c.take<uint32_t>(Ea + 1);
+  for (int i = 0; i < 2; ++i) {  // one entry more than the edges: the coalescing scans reuse them
+    L->sort.keys[i] = c.take<uint32_t>(Ea + 1);
+    L->sort.vals[i] = c.take<uint32_t>(Ea + 1);
+    L->sort.vals2[i] = c.take<uint32_t>(Ea + 1);
   }
   const int64_t hist_n = sort_tiles(E) * kRadix;
   L->sort.hist = c.take<int32_t>(hist_n + 1);
-  L->sort.scan_scratch = c.take<char>(scan_scratch_bytes(std::max(std::max(hist_n, rows), std::max(crows, N))));
+  L->sort.scan_scratch =
+      c.take<char>(scan_scratch_bytes(std::max(std::max(std::max(hist_n, rows), std::max(crows, N)), Ea)));
   return c.used;
 }
 
@@ -527,6 +610,30 @@ static int bit_width(uint64_t x) {
 
 static unsigned grid_for(int64_t n, int threads = 256) {
   return (unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(n, threads), 152 * 16));
+}
+
+// Runs of equal adjacent entries of (ptr, col): the flags, their scan (the run index of each
+// position) and the runs' columns, multiplicities and row pointers.  Uses the sort buffers.
+static hg_status coalesce_runs(const int32_t* col, const int32_t* ptr, int64_t rows, int64_t E, GraphLayout& L,
+                               int32_t* ucol, int32_t* ucnt, int32_t* uptr, cudaStream_t s) {
+  int32_t* flag = reinterpret_cast<int32_t*>(L.sort.keys[0]);
+  int32_t* u = reinterpret_cast<int32_t*>(L.sort.keys[1]);
+  int32_t* upos = reinterpret_cast<int32_t*>(L.sort.vals[0]);
+  HG_TRY(launch("run_flags", run_flags, dim3(grid_for(E)), dim3(256), 0, s, col, ptr, rows, E, flag));
+  HG_TRY(launch("run_row_starts", run_row_starts, dim3(grid_for(rows)), dim3(256), 0, s, ptr, rows, flag));
+  HG_TRY(exclusive_scan(flag, u, E, L.sort.scan_scratch, s));
+  HG_TRY(launch("run_write", run_write, dim3(grid_for(E + 1)), dim3(256), 0, s, (const int32_t*)flag,
+                (const int32_t*)u, col, ptr, rows, ucol, upos));
+  return launch("run_finish", run_finish, dim3(grid_for(std::max(E, rows + 1))), dim3(256), 0, s, (const int32_t*)u,
+                (const int32_t*)upos, ptr, rows, ucnt, uptr);
+}
+
+// ofs = exclusive scan of the chunk counts of the rows above the hub degree, row = the row of each chunk.
+static hg_status chunk_table(const int32_t* ptr, int64_t rows, int32_t* ofs, int32_t* row, GraphLayout& L,
+                             cudaStream_t s) {
+  HG_TRY(launch("chunk_counts", chunk_counts, dim3(grid_for(rows)), dim3(256), 0, s, ptr, rows, L.cnt));
+  HG_TRY(exclusive_scan(L.cnt, ofs, rows, L.sort.scan_scratch, s));
+  return launch("chunk_fill", chunk_fill, dim3(grid_for(rows)), dim3(256), 0, s, (const int32_t*)ofs, rows, row);
 }
 
 }  // namespace hg
@@ -585,46 +692,49 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
     HG_CUDA(cudaMemsetAsync(L.csr_ptr, 0, (rows + 1) * sizeof(int32_t), s));
     HG_CUDA(cudaMemsetAsync(L.csc_ptr, 0, (crows + 1) * sizeof(int32_t), s));
     HG_CUDA(cudaMemsetAsync(L.node_ptr, 0, (N + 1) * sizeof(int32_t), s));
+    HG_CUDA(cudaMemsetAsync(L.agg_ptr, 0, (rows + 1) * sizeof(int32_t), s));
+    HG_CUDA(cudaMemsetAsync(L.bagg_ptr, 0, (N + 1) * sizeof(int32_t), s));
     HG_CUDA(cudaMemsetAsync(L.invalid, 0, sizeof(int32_t), s));
   } else {
-    // keys of both layouts in one pass (the CSR keys in keys[0], which the first sort pass reads
-    // while it writes keys[1]; the CSC keys wait in their own buffer)
-    HG_TRY(launch("edge_keys", edge_keys, dim3(g), dim3(256), 0, s, src, dst, rel, E, m, rows, crows,
-                  L.sort.keys[0], L.sort.ckeys));
-    // CSR by destination
-    HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)rows), (const uint32_t*)L.sort.keys[0], (const uint32_t*)src, s,
-                      &res));
+    // CSR by (destination row, source, edge id): a stable sort by source, then by row
+    HG_TRY(launch("edge_keys", edge_keys, dim3(g), dim3(256), 0, s, src, dst, rel, E, m, rows, L.sort.keys[0],
+                  L.sort.ckeys));
+    int r1 = 0;
+    HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)N), (const uint32_t*)L.sort.keys[0], (const uint32_t*)nullptr,
+                      (const uint32_t*)L.sort.ckeys, 0, s, &r1));
+    HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)rows), (const uint32_t*)L.sort.vals2[r1],
+                      (const uint32_t*)L.sort.vals[r1], (const uint32_t*)L.sort.keys[r1], r1, s, &res));
     HG_TRY(launch("row_ptr_from_keys", row_ptr_from_keys, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[res],
                   E, rows, L.csr_ptr));
-    const uint32_t* src_sorted = L.sort.vals2[res];
-    HG_TRY(launch("csr_finish", csr_finish, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.vals[res], src_sorted,
-                  (const int32_t*)L.csr_ptr, rows, E, L.csr_col, L.csr_eid, L.invalid));
-    // CSC by source
-    HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)crows), (const uint32_t*)L.sort.ckeys, (const uint32_t*)dst, s,
-                      &res));
+    HG_TRY(launch("csr_finish", csr_finish, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.vals[res],
+                  (const uint32_t*)L.sort.vals2[res], (const int32_t*)L.csr_ptr, rows, E, L.csr_col, L.csr_eid,
+                  L.invalid));
+    // CSC by (source row, destination, edge id): the CSR order sorted stably by source row
+    const int r2 = res;
+    HG_TRY(launch("csc_keys_from_csr", csc_keys_from_csr, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[r2],
+                  (const uint32_t*)L.sort.vals2[r2], E, (const int32_t*)L.csr_ptr, rows, crows, m, L.sort.ckeys,
+                  L.sort.keys[r2]));
+    HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)crows), (const uint32_t*)L.sort.ckeys,
+                      (const uint32_t*)L.sort.vals[r2], (const uint32_t*)L.sort.keys[r2], r2, s, &res));
     HG_TRY(launch("row_ptr_from_keys", row_ptr_from_keys, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[res],
                   E, crows, L.csc_ptr));
-    const uint32_t* dst_sorted = L.sort.vals2[res];
     // node-major rows: out-degree per node over its relations, their scan, then the edges
     HG_TRY(launch("node_out_counts", node_out_counts, dim3(grid_for(N)), dim3(256), 0, s, (const int32_t*)L.csc_ptr,
                   m, L.cnt));
     HG_TRY(exclusive_scan(L.cnt, L.node_ptr, N, L.sort.scan_scratch, s));
     HG_TRY(launch("csc_finish", csc_finish, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[res],
-                  (const uint32_t*)L.sort.vals[res], dst_sorted, (const int32_t*)L.csc_ptr, crows, m,
-                  (const int32_t*)L.csr_ptr, (const int32_t*)L.node_ptr, L.csc_col, L.csc_eid, L.csc_coef,
+                  (const uint32_t*)L.sort.vals[res], (const uint32_t*)L.sort.vals2[res], (const int32_t*)L.csc_ptr,
+                  crows, m, (const int32_t*)L.csr_ptr, (const int32_t*)L.node_ptr, L.csc_col, L.csc_eid, L.csc_coef,
                   L.node_col));
+    // parallel edges coalesced into (column, multiplicity) runs, in both aggregation orders
+    HG_TRY(coalesce_runs(L.csr_col, L.csr_ptr, rows, E, L, L.agg_col, L.agg_cnt, L.agg_ptr, s));
+    HG_TRY(coalesce_runs(L.node_col, L.node_ptr, N, E, L, L.bagg_col, L.bagg_cnt, L.bagg_ptr, s));
   }
-  // chunk tables for rows above the hub degree
-  HG_TRY(launch("chunk_counts", chunk_counts, dim3(grid_for(rows)), dim3(256), 0, s,
-                (const int32_t*)L.csr_ptr, rows, L.cnt));
-  HG_TRY(exclusive_scan(L.cnt, L.csr_chunk_ofs, rows, L.sort.scan_scratch, s));
-  HG_TRY(launch("chunk_fill", chunk_fill, dim3(grid_for(rows)), dim3(256), 0, s,
-                (const int32_t*)L.csr_chunk_ofs, rows, L.csr_chunk_row));
-  HG_TRY(launch("chunk_counts", chunk_counts, dim3(grid_for(N)), dim3(256), 0, s,
-                (const int32_t*)L.node_ptr, N, L.cnt));
-  HG_TRY(exclusive_scan(L.cnt, L.node_chunk_ofs, N, L.sort.scan_scratch, s));
-  HG_TRY(launch("chunk_fill", chunk_fill, dim3(grid_for(N)), dim3(256), 0, s,
-                (const int32_t*)L.node_chunk_ofs, N, L.node_chunk_row));
+  // chunk tables for rows above the hub degree: per edge (attention layer), per run (mean layer)
+  HG_TRY(chunk_table(L.csr_ptr, rows, L.csr_chunk_ofs, L.csr_chunk_row, L, s));
+  HG_TRY(chunk_table(L.node_ptr, N, L.node_chunk_ofs, L.node_chunk_row, L, s));
+  HG_TRY(chunk_table(L.agg_ptr, rows, L.agg_chunk_ofs, L.agg_chunk_row, L, s));
+  HG_TRY(chunk_table(L.bagg_ptr, N, L.bagg_chunk_ofs, L.bagg_chunk_row, L, s));
 
   hg_graph* gh = new hg_graph{};
   gh->meta = m;
@@ -647,6 +757,16 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
   gh->node_col = L.node_col;
   gh->node_chunk_ofs = L.node_chunk_ofs;
   gh->node_chunk_row = L.node_chunk_row;
+  gh->agg_ptr = L.agg_ptr;
+  gh->agg_col = L.agg_col;
+  gh->agg_cnt = L.agg_cnt;
+  gh->agg_chunk_ofs = L.agg_chunk_ofs;
+  gh->agg_chunk_row = L.agg_chunk_row;
+  gh->bagg_ptr = L.bagg_ptr;
+  gh->bagg_col = L.bagg_col;
+  gh->bagg_cnt = L.bagg_cnt;
+  gh->bagg_chunk_ofs = L.bagg_chunk_ofs;
+  gh->bagg_chunk_row = L.bagg_chunk_row;
   gh->invalid_count = L.invalid;
   *out = gh;
   return HG_OK;

@@ -127,6 +127,19 @@ struct hg_graph {
   int32_t* node_col;        // [num_edges] dMs row of each out-edge's destination
   int32_t* node_chunk_ofs;  // [N + 1] chunks per node-major row above the hub degree
   int32_t* node_chunk_row;
+  // Parallel edges coalesced (the mean layer's aggregation lists): the CSR rows as runs of equal
+  // source ids (agg_col = source, agg_cnt = multiplicity; deg = sum of the counts = CSR row length)
+  // and the node-major rows as runs of equal dMs rows; chunk tables over runs, as above.
+  int32_t* agg_ptr;         // [csr_rows + 1]
+  int32_t* agg_col;         // [runs]
+  int32_t* agg_cnt;
+  int32_t* agg_chunk_ofs;   // [csr_rows + 1]
+  int32_t* agg_chunk_row;   // [chunk_cap_csr]
+  int32_t* bagg_ptr;        // [N + 1]
+  int32_t* bagg_col;
+  int32_t* bagg_cnt;
+  int32_t* bagg_chunk_ofs;  // [N + 1]
+  int32_t* bagg_chunk_row;  // [chunk_cap_node]
   int32_t* invalid_count;  // device scalar
 };
 

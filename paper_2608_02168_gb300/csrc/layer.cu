@@ -372,6 +372,7 @@ hg_status project_backward(const hg_graph* graph, const hg_layer_params* p, cons
       a.U = (const __nv_bfloat16*)L.U;
       a.stats = L.stats;
       a.gamma = p->layernorm ? (const __nv_bfloat16*)p->ln_gamma + (size_t)t * d : nullptr;
+      a.b = (const __nv_bfloat16*)p->b_agg + (size_t)t * d;
       a.csr_ptr = deg_scale ? graph->csr_ptr : nullptr;
       a.dY = (__nv_bfloat16*)L.dY;
       a.dU = (__nv_bfloat16*)L.dU;

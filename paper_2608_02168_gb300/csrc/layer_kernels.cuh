@@ -73,9 +73,10 @@ struct TcBwdArgs {
   int type;
   const __nv_bfloat16* dH_out;
   const __nv_bfloat16* H_in;
-  const __nv_bfloat16* U;
+  const __nv_bfloat16* U;     // the stored pre-activation without its bias (bf16(Z W_agg))
   const float2* stats;
   const __nv_bfloat16* gamma;
+  const __nv_bfloat16* b;     // the type's bias b_agg, added back to U in fp32
   const int32_t* csr_ptr;
   __nv_bfloat16* dY;
   __nv_bfloat16* dU;

@@ -13,7 +13,10 @@
 // Forward, one CTA per 128 destination rows of type t:
 //   U = sum_{r -> t} M_r V_r      A = relation means (TMA, 128 x 64 tiles), B = V_r^T chunks
 //                                 (the hi and lo halves of a chunk in one pipeline stage)
-//   epilogue: U += b, stored; Y = act(U) + H_in; H_out = LayerNorm(Y); row statistics saved.
+//   epilogue: U_s = bf16(U) stored, then U = U_s + b in fp32; Y = act(U) + H_in;
+//             H_out = LayerNorm(Y); row statistics saved.  U is stored without its bias: the
+//             rounding then scales with the data (Z W_agg), not with a large bias, and the
+//             backward adds the same bias back, so both passes see the same U.
 // Backward:
 //   ln_act_bwd   (warp per row)  dY = LayerNorm backward, dU = dY act'(U); column partials of the
 //                                bias / gain / shift gradients
@@ -218,8 +221,8 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
       fence_after_sync();
       const uint32_t trow = tmem + b * C::kAccCols + ((uint32_t)(q * 32) << 16);
       const uint8_t* ht = htile + b * C::kH;
-      // U = bf16(acc + b) for columns c .. c+15 (acc already in u when preloaded), stored;
-      // returned unpacked in u
+      // U_s = bf16(acc) for columns c .. c+15 (acc already in u when preloaded), stored;
+      // returned as U_s + b in u
       auto u16 = [&](int c, float* u, bool store, bool preloaded = false) {
         if (!preloaded) {
           if (CT > 0) {
@@ -231,15 +234,15 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
         }
         uint32_t up[8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) up[i] = pack_bf16x2(u[2 * i] + pb[c + 2 * i], u[2 * i + 1] + pb[c + 2 * i + 1]);
+        for (int i = 0; i < 8; ++i) up[i] = pack_bf16x2(u[2 * i], u[2 * i + 1]);
         if (store && live) {
           st16(a.U + node * D + c, make_uint4(up[0], up[1], up[2], up[3]));
           st16(a.U + node * D + c + 8, make_uint4(up[4], up[5], up[6], up[7]));
         }
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
-          u[2 * i] = __uint_as_float(up[i] << 16);
-          u[2 * i + 1] = __uint_as_float(up[i] & 0xFFFF0000u);
+          u[2 * i] = __uint_as_float(up[i] << 16) + pb[c + 2 * i];
+          u[2 * i + 1] = __uint_as_float(up[i] & 0xFFFF0000u) + pb[c + 2 * i + 1];
         }
       };
       auto h16 = [&](int c, float* h) {  // residual row, columns c .. c+15
@@ -444,7 +447,8 @@ __global__ void __launch_bounds__(256) wgrad_finish(const float* __restrict__ G,
 }
 
 // LayerNorm / activation backward, one warp per row (coalesced rows, D / 32 columns per lane):
-// dY = rstd (dXh - mean(dXh) - Xh mean(dXh Xh)), dXh = dH_out gamma, dU = dY act'(U); per-block
+// U = stored U_s + b (as in the forward), dY = rstd (dXh - mean(dXh) - Xh mean(dXh Xh)),
+// dXh = dH_out gamma, dU = dY act'(U); per-block
 // column partials part[block] = {sum dU, sum dH_out Xh, sum dH_out} over the block's rows.
 template <int D>
 __global__ void __launch_bounds__(256) ln_act_bwd(TcBwdArgs a) {
@@ -452,9 +456,12 @@ __global__ void __launch_bounds__(256) ln_act_bwd(TcBwdArgs a) {
   __shared__ float red[8][3][D];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int c0 = lane * E;
-  float g[E];
+  float g[E], bias[E];
 #pragma unroll
-  for (int i = 0; i < E; ++i) g[i] = a.ln ? __bfloat162float(a.gamma[c0 + i]) : 1.f;
+  for (int i = 0; i < E; ++i) {
+    g[i] = a.ln ? __bfloat162float(a.gamma[c0 + i]) : 1.f;
+    bias[i] = __bfloat162float(a.b[c0 + i]);
+  }
   float pdb[E], pdg[E], pdbe[E];
 #pragma unroll
   for (int i = 0; i < E; ++i) pdb[i] = pdg[i] = pdbe[i] = 0.f;
@@ -495,6 +502,8 @@ __global__ void __launch_bounds__(256) ln_act_bwd(TcBwdArgs a) {
       const int64_t node = a.off + (has[k] ? row : row0);
       load(a.dH_out + node * D + c0, dv[k]);
       load(a.U + node * D + c0, uv[k]);
+#pragma unroll
+      for (int i = 0; i < E; ++i) uv[k][i] += bias[i];
       load(a.H_in + node * D + c0, hv[k]);
       st[k] = a.ln ? a.stats[node] : make_float2(0.f, 1.f);
     }

@@ -45,7 +45,8 @@ def test_full_csr_invariants(full):
         assert np.all(deg >= 0) and b - a == int((rel == r).sum())
         assert np.all(rel[eid] == r) and np.all(dst[eid] - offs[tt] == rows) and np.array_equal(src[eid], col)
         same = rows[1:] == rows[:-1]
-        assert np.all(np.diff(eid)[same] > 0)  # ascending edge id within a row
+        ds, de = np.diff(col.astype(np.int64))[same], np.diff(eid)[same]
+        assert np.all((ds > 0) | ((ds == 0) & (de > 0)))  # ascending (source, edge id) within a row
         assert not seen[eid].any()
         seen[eid] = True
         cp = v["csc_ptr"].cpu().numpy().astype(np.int64)
@@ -53,7 +54,10 @@ def test_full_csr_invariants(full):
         ceid = v["csc_eid"][ca:cb].cpu().numpy().astype(np.int64)
         crow = np.repeat(np.arange(len(cp) - 1), np.diff(cp))
         assert np.all(src[ceid] - offs[ts] == crow) and np.all(rel[ceid] == r)
-        assert np.all(np.diff(ceid)[crow[1:] == crow[:-1]] > 0)
+        ccol = v["csc_col"][ca:cb].cpu().numpy().astype(np.int64)
+        same = crow[1:] == crow[:-1]
+        ds, de = np.diff(ccol)[same], np.diff(ceid)[same]
+        assert np.all((ds > 0) | ((ds == 0) & (de > 0)))  # ascending (destination, edge id)
         coef = v["csc_coef"][ca:cb].cpu().numpy()
         want = np.float32(1) / deg[dst[ceid] - offs[tt]].astype(np.float32)
         assert np.array_equal(coef.view(np.uint32), want.view(np.uint32))
@@ -159,7 +163,7 @@ def test_full_size_head():
     from tests.test_gpu_head import check, head_gpu
     sp = hgsynth.spec("sub-1m")
     lab, y = hgsynth.make_labels(sp)
-    p = hgsynth.make_head_params(sp, random_bias=True)
+    p = hgsynth.make_head_params(sp, random_bias=True, bias_margin=BF16_RELU_MARGIN)  # see test_gpu_head
     rng = np.random.default_rng(5)
     N, d = sp.num_nodes, sp.d
     H = hgsynth.bf16_round(rng.standard_normal((N, d), dtype=np.float32))

@@ -6,7 +6,7 @@ import pytest
 import torch
 
 from oracle import head as OH
-from tests.gpu_util import TOL, dev, host, lib, need_gpu, relerr, tdtype
+from tests.gpu_util import BF16_RELU_MARGIN, TOL, dev, host, lib, need_gpu, relerr, tdtype
 from hgsynth import bf16_round
 
 pytestmark = pytest.mark.gpu
@@ -29,6 +29,10 @@ def problem(seed, N, d, n_lab, n_rep, dt, rows_rep=None, frac_y=False):
     p = {"W1": rng.uniform(-a1, a1, (d, d)).astype(np.float32), "b1": (0.1 * rng.standard_normal(d)).astype(np.float32),
          "w2": rng.uniform(-a2, a2, d).astype(np.float32), "b2": np.array([0.3], np.float32)}
     if dt == "bf16":
+        # hidden biases of +-8 keep every pre-activation clear of the ReLU's kink: the tensor cores'
+        # fp32 accumulation may put a pre-activation within 1e-5 of zero on the other side, and each
+        # such decision moves its row's input gradient by percents (rows are not sums over rows)
+        p["b1"] = (BF16_RELU_MARGIN * rng.choice([-1.0, 1.0], d)).astype(np.float32)
         H, Hr = bf16_round(H), bf16_round(Hr)
         p = {key: bf16_round(v) for key, v in p.items()}
     return H, Hr, ia, ib, lab, y, p

@@ -31,7 +31,8 @@ def test_ring_sequence_matches_oracle():
                          dev(part.gid))
         torch.cuda.synchronize()
         vb = None if prev_H is None else {"H_b": prev_H, "gid_a": part.gid, "gid_b": prev_gid}
-        ref = oracle.step(g, part.X, params, part.dH_top, vb)  # the plain fp64 definition
+        # the plain fp64 definition, with the interface's bf16 layer outputs and gradients
+        ref = oracle.step(g, part.X, params, part.dH_top, vb, interface="bf16")
         p = ring.path
         assert relerr(host(bank), ref["H"][-1]) <= TOL[sp.dtype], k
         if k > 0:

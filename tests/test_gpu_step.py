@@ -56,7 +56,9 @@ def test_step_matches_oracle(variant, with_head):
     run(path, w, head)
     vb = {"idx": w.overlap_local, "X_b": w.X_b} if sp.view_b == "perturbed" else \
         {"H_b": w.H_b, "gid_a": w.gid_a, "gid_b": w.gid_b}
-    ref = oracle.step(w.graph, w.X, w.params, w.dH_top, vb, head=head)
+    # the plain fp64 definition; the layer outputs and their gradients are bf16 tensors of the
+    # interface for a bf16 workload, so the oracle rounds them there (and nowhere else)
+    ref = oracle.step(w.graph, w.X, w.params, w.dH_top, vb, head=head, interface=sp.dtype)
     tol = TOL[sp.dtype]
     assert relerr(host(path.loss), np.array(ref["loss"])) <= (1e-4 if sp.dtype == "f32" else 2e-2)
     if with_head:

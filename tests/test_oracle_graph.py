@@ -52,7 +52,7 @@ def brute_force_rows(src, dst, rel, offs, rels, by_dst=True):
             key = t if by_dst else s
             other = s if by_dst else t
             rows[key - offs[key_t]].append((e, other))
-        out[rr] = [sorted(x) for x in rows]  # ascending edge id
+        out[rr] = [sorted(x, key=lambda eo: (eo[1], eo[0])) for x in rows]  # ascending (other end, edge id)
     return out
 
 
@@ -87,12 +87,13 @@ def test_csr_invariants():
     for r, c in enumerate(csr):
         assert np.all(np.diff(c["row_ptr"]) >= 0) and c["row_ptr"][0] == 0
         assert c["row_ptr"][-1] == c["csc_ptr"][-1] == np.sum(ok & (rel == r))
-        # every edge sits in the row of its destination, in ascending edge order
+        # every edge sits in the row of its destination, in ascending (source, edge id) order
         rows = np.repeat(np.arange(len(c["deg"])), c["deg"])
         assert np.all(dst[c["eid"]] - offs[rels[r][1]] == rows)
         assert np.all(src[c["eid"]] == c["col"])
         same_row = rows[1:] == rows[:-1]
-        assert np.all(np.diff(c["eid"])[same_row] > 0)
+        ds, de = np.diff(c["col"].astype(np.int64))[same_row], np.diff(c["eid"])[same_row]
+        assert np.all((ds > 0) | ((ds == 0) & (de > 0)))
         seen.append(c["eid"])
     seen = np.sort(np.concatenate(seen))
     assert np.array_equal(seen, np.flatnonzero(ok))  # a permutation of the valid edges

@@ -195,6 +195,8 @@ def test_bf16_storage_points():
     g, H, p = graph(11, heads=2)
     out_b, cb = OH.hgt_forward(*g, p, H, 2, store="bf16")
     out_f, cf = OH.hgt_forward(*g, p, H, 2)
-    for k in ("K", "V", "Q", "Qp", "Ssum", "U"):
+    for k in ("K", "V", "Q", "Qp", "Ssum"):
         assert np.array_equal(cb[k], bf16_round(cb[k]).astype(np.float64)), k
+    ub = cb["U"] - p["b_agg"][cb["types"]]  # U is stored without its bias
+    assert np.allclose(ub, bf16_round(ub).astype(np.float64), rtol=0, atol=1e-12)
     assert np.abs(out_b - out_f).max() <= 2e-2 * np.abs(out_f).max()

@@ -274,7 +274,8 @@ def test_round_bf16_matches_torch():
 
 
 def test_bf16_store_mode_matches_torch_with_bf16_casts():
-    """store='bf16' = the dense torch formulation with M_r and U cast through torch.bfloat16."""
+    """store='bf16' = the dense torch formulation with M_r and Z W_agg (U without its bias) cast
+    through torch.bfloat16."""
     src, dst, rel, offs, rels, H, params = small_graph(13, d=8)
     csr = oracle.build_csr(src, dst, rel, offs, rels)
     out, _ = oracle.layer_forward(csr, offs, rels, params, H, store="bf16")
@@ -289,7 +290,7 @@ def test_bf16_store_mode_matches_torch_with_bf16_casts():
             if tt == t:
                 A = torch.tensor(dense_mean_matrix(src, dst, rel, offs, rels, r))
                 Z = Z + bf(A @ Ht) @ P["W_rel"][r]
-        U = bf(Z @ P["W_agg"][t] + P["b_agg"][t])
+        U = bf(Z @ P["W_agg"][t]) + P["b_agg"][t]
         Y = torch.relu(U) + Ht[lo:hi]
         outs.append(torch.nn.functional.layer_norm(Y, (H.shape[1],), P["ln_gamma"][t], P["ln_beta"][t], 1e-5))
     assert np.allclose(out, torch.cat(outs).numpy(), rtol=0, atol=1e-12)
