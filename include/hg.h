@@ -78,6 +78,12 @@ int32_t hg_abi_version(void);
  * the library is unbound or already bound to `device`; HG_ERR_UNSUPPORTED if it is bound to
  * another device; HG_ERR_INVALID_ARG for a negative ordinal.  Makes no CUDA call. */
 hg_status hg_bind_device(int32_t device);
+/* Diagnostic of the bounded waits: launches one CTA whose thread waits `polls` times (1 <= polls
+ * <= 2^20) on an mbarrier that nothing arrives at -- with no copy, store or MMA in flight -- and
+ * records the give-up in the device status word exactly as a tensor-core kernel whose wait runs
+ * out does, so a caller can check that hg_device_status reports it and that the context stays
+ * usable.  The paper has no counterpart. */
+hg_status hg_selftest_bounded_wait(uint32_t polls, hg_stream stream);
 /* SYNCHRONISES the device, then reports and clears the library's device status word.  Every wait
  * inside a kernel of this library is bounded; a wait that gave up sets a flag here (its kernel's
  * results are then invalid) and this call returns HG_ERR_TIMEOUT.  flags may be NULL. */

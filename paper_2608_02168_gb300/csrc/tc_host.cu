@@ -62,6 +62,19 @@ hg_status make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint
   return HG_OK;
 }
 
+// Self-test of the bounded waits: thread 0 of one CTA waits `polls` times on an mbarrier that
+// nothing arrives at (no copy, store or MMA is in flight) and records the give-up in the status
+// word, as every tensor-core kernel does when one of its waits runs out.
+__global__ void selftest_bounded_wait(uint32_t polls, int* status) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    tc::mbar_init(&bar, 1);
+    tc::fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && !tc::mbar_wait_n(&bar, 0, polls)) record_device_error(status, tc::kErrTimeout);
+}
+
 // Resolved once per process on the current device (the library drives one GPU per process).
 int* device_status_ptr() {
   static int* addr = nullptr;
@@ -73,6 +86,16 @@ int* device_status_ptr() {
 }
 
 }  // namespace hg
+
+extern "C" hg_status hg_selftest_bounded_wait(uint32_t polls, hg_stream stream) {
+  hg::clear_error();
+  HG_TRY(hg::device_guard());
+  HG_REQUIRE(polls >= 1 && polls <= (1u << 20), "polls must be in [1, 2^20]");
+  int* status = hg::device_status_ptr();
+  HG_REQUIRE(status != nullptr, "device status word unavailable");
+  return hg::launch("selftest_bounded_wait", hg::selftest_bounded_wait, dim3(1), dim3(32), 0,
+                    reinterpret_cast<cudaStream_t>(stream), polls, status);
+}
 
 extern "C" hg_status hg_bind_device(int32_t device) {
   hg::clear_error();

@@ -82,6 +82,7 @@ EXPORTS = {
     "hg_abi_version": (c_int32, []),
     "hg_device_status": (c_int32, [POINTER(c_int32)]),
     "hg_bind_device": (c_int32, [c_int32]),
+    "hg_selftest_bounded_wait": (c_int32, [ctypes.c_uint32, c_void_p]),
     "hg_graph_workspace_size": (c_int32, [c_int64, POINTER(c_int64), c_int32, POINTER(hg_rel_desc), c_int32,
                                           POINTER(c_size_t)]),
     "hg_build_csr": (c_int32, [c_void_p, c_void_p, c_void_p, c_int64, POINTER(c_int64), c_int32,
@@ -358,6 +359,11 @@ def hg_device_status() -> int:
     if st not in (0, 6):
         _check(st, "hg_device_status")
     return f.value
+
+
+def hg_selftest_bounded_wait(polls: int, stream=None):
+    """One wait on an mbarrier nothing arrives at, giving up after `polls` polls (see hg.h)."""
+    _check(lib().hg_selftest_bounded_wait(int(polls), _stream(stream)), "hg_selftest_bounded_wait")
 
 
 def hg_overlap_align_loss_static(H_a, idx_a, H_b, idx_b, n_max: int, n_dev, lambda_n: float, var_eps: float,

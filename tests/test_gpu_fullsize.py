@@ -226,7 +226,7 @@ def test_full_size_attention_layer_sampled_targets():
     sp = hgsynth.spec("sub-1m")
     w = hgsynth.make_workload(sp, with_ids=False)
     g = w.graph
-    p = hgsynth.make_hgt_params(sp, 4, bias_margin=3.0)
+    p = hgsynth.make_hgt_params(sp, 4, bias_margin=BF16_RELU_MARGIN)
     td = torch.bfloat16
     G = hg.hg_build_csr(dev(g["src"]), dev(g["dst"]), dev(g["rel"]), g["type_offsets"], g["rels"])
     P = hg.HgtParams({k: dev(v, torch.float32 if k == "mu" else td) for k, v in p.items()}, 4)

@@ -7,7 +7,7 @@ import torch
 
 import hgsynth
 from oracle import hgt as OH
-from tests.gpu_util import TOL, dev, host, lib, need_gpu, relerr, tdtype
+from tests.gpu_util import BF16_RELU_MARGIN, TOL, dev, host, lib, need_gpu, relerr, tdtype
 
 pytestmark = pytest.mark.gpu
 
@@ -49,9 +49,9 @@ def test_hgt_matches_oracle(case, ln):
     hg = lib()
     name, ov, heads = CASES[case]
     sp = hgsynth.spec(name, **ov)
-    # bf16 ReLU: biases of +-3 keep the pre-activations clear of the kink (as for the mean layer)
+    # bf16 ReLU: biases of +-8 keep the pre-activations clear of the kink (as for the mean layer)
     w = hgsynth.make_workload(sp, random_affine=True, with_ids=False)
-    p = hgsynth.make_hgt_params(sp, heads, bias_margin=3.0 if sp.dtype == "bf16" else None)
+    p = hgsynth.make_hgt_params(sp, heads, bias_margin=BF16_RELU_MARGIN if sp.dtype == "bf16" else None)
     g = w.graph
     out, dH, gr = run_gpu(hg, w, p, heads, ln, w.dH_top)
     args = (g["src"], g["dst"], g["rel"], g["type_offsets"], g["rels"], p, w.X)

@@ -58,6 +58,8 @@ def test_host_argument_checks(hg):
     assert so.hg_graph_workspace_size(5, offs, 2, rels, 9, ctypes.byref(ctypes.c_size_t())) == 2
     # edge count beyond int32
     assert so.hg_graph_workspace_size(1 << 31, offs, 2, rels, 1, ctypes.byref(ctypes.c_size_t())) == 2
+    # bounded-wait self-test: poll count out of range
+    assert so.hg_selftest_bounded_wait(0, None) == 1 and so.hg_selftest_bounded_wait((1 << 20) + 1, None) == 1
     # a relation pointing at a type that does not exist
     bad = (hg.hg_rel_desc * 1)(hg.hg_rel_desc(0, 2))
     assert so.hg_graph_workspace_size(5, offs, 2, bad, 1, ctypes.byref(ctypes.c_size_t())) == 1
