@@ -261,13 +261,14 @@ def graph_stats(w) -> dict:
     blank = lambda: dict(E_nh=0, E_h=0, R_nh=0, R_h=0, U_nh=0, U_h=0, chunks=0)  # noqa: E731
     st = dict(N=N, E=int(src.shape[0]), RR=0, CC=0, n_ov=n_ov, fwd=blank(), bwd=blank(), types=[], rels=[])
     for t in range(len(offs) - 1):
-        st["types"].append(dict(n=offs[t + 1] - offs[t], R=sum(1 for r in g["rels"] if r[1] == t)))
+        st["types"].append(dict(n=offs[t + 1] - offs[t], R=sum(1 for r in g["rels"] if r[1] == t), nnz=0))
     for r, (ts, tt) in enumerate(g["rels"]):
         m = rel == r
         s_r, d_r = src[m], dst[m]
         st["RR"] += offs[tt + 1] - offs[tt]
         st["CC"] += offs[ts + 1] - offs[ts]
-        st["rels"].append(dict(n_t=offs[tt + 1] - offs[tt], n_s=offs[ts + 1] - offs[ts], E=int(s_r.shape[0])))
+        st["rels"].append(dict(n_t=offs[tt + 1] - offs[tt], n_s=offs[ts + 1] - offs[ts], E=int(s_r.shape[0]),
+                               nnz=nz(torch.bincount(d_r - offs[tt], minlength=offs[tt + 1] - offs[tt]))))
         # forward: one CSR row per (relation, destination); its runs are the distinct sources
         u = torch.unique(d_r * N + s_r)
         u_dst, u_src = u // N, u % N
@@ -284,6 +285,9 @@ def graph_stats(w) -> dict:
         hr = runs[runs > HUB]
         a["chunks"] += int(((hr + CHUNK - 1) // CHUNK).sum())
         del u, u_dst, u_src, runs, hub_run, edges
+    for r, (_, tt) in enumerate(g["rels"]):
+        st["types"][tt]["nnz"] += st["rels"][r]["nnz"]  # stored relation rows (non-empty CSR rows)
+    st["NNZ"] = sum(r["nnz"] for r in st["rels"])
     # backward: one node-major row per node; its runs are the distinct (relation, destination) dMs
     # rows it reads
     read = rel * N + dst
@@ -315,7 +319,8 @@ def kernel_models(st: dict, sp) -> dict:
     # run lists (column and count, 8 bytes per run) and row pointers once, every output row written
     # once, the fp32 chunk partials written and read.  The rows gathered per run (one per run, served
     # by L1 / L2 where a row recurs) are reported beside them as `gathered` (not HBM traffic).
-    m["agg_fwd_rows"] = (L * (8 * (RR + 1) + 8 * f["R_nh"] + row * f["U_nh"] + row * RR + 4 * d * f["chunks"]), 0)
+    NNZ = st.get("NNZ", RR)  # stored (non-empty) relation rows
+    m["agg_fwd_rows"] = (L * (12 * NNZ + 8 * f["R_nh"] + row * f["U_nh"] + row * NNZ + 4 * d * f["chunks"]), 0)
     m["agg_fwd_chunks"] = (L * (8 * f["R_h"] + row * f["U_h"] + 4 * d * f["chunks"]), 0)
     m["agg_bwd_nodes"] = (L * (4 * (N + 1) + 8 * bw["R_nh"] + row * bw["U_nh"] + 2 * row * N + 4 * d * bw["chunks"]), 0)
     m["agg_bwd_chunks"] = (L * (8 * bw["R_h"] + row * bw["U_h"] + 4 * d * bw["chunks"]), 0)
@@ -331,19 +336,21 @@ def kernel_models(st: dict, sp) -> dict:
     m["proj_fwd_simt"] = (L * fb, L * ff)
     m["proj_bwd_simt"] = (L * bb, L * bf)
     m["wgrad_partial"] = (L * 2 * row * (N + RR), L * 2 * d * d * (N + RR))
-    # tensor-core path (fused weights V_r = W_r W_agg): per node of type t with R relations into t
+    # tensor-core path (fused weights V_r = W_r W_agg as hi / lo bf16 pairs), M_r and dM_r stored
+    # for the non-empty relation rows only: per node of type t with R relations into t, nnz of them
+    # stored
     tf = tfl = lb = pb = pfl = 0
     for t in st["types"]:
-        n, R = t["n"], t["R"]
-        tf += n * row * (R + 3) + 8 * n      # read M_r (R rows), H_in; write U, H_out; row statistics
-        tfl += 2 * n * d * d * R
+        n, R, nnz = t["n"], t["R"], t.get("nnz", t["n"] * t["R"])
+        tf += n * (3 * row + 8) + row * nnz   # read H_in, the stored M_r rows; write U, H_out, statistics
+        tfl += 2 * 2 * n * d * d * R         # two products per relation (hi, lo)
         lb += n * (5 * row + 8)              # read dH_out, U, H_in, statistics; write dY, dU
-        pb += n * row * (R + 1) + 4 * n * R  # read dU, degrees; write dM_r (R rows)
-        pfl += 2 * n * d * d * R
+        pb += nnz * (2 * row + 12)           # gather dU, write dM_r, read the row list and degrees
+        pfl += 2 * 2 * nnz * d * d
     m["proj_fwd_tc"] = (L * tf, L * tfl)
     m["ln_act_bwd"] = (L * lb, 0)
     m["proj_bwd_tc"] = (L * pb, L * pfl)
-    m["wgrad_tc"] = (L * row * (RR + N), L * 2 * d * d * RR)  # G_r = M_r^T dU: M_r rows once, dU once per type
+    m["wgrad_tc"] = (L * (2 * row + 4) * NNZ, L * 2 * d * d * NNZ)  # G_r = M_r^T dU over the stored rows
     # per 8-bit pass over the keys: read and write of key, edge id and endpoint; three stable sorts
     # (by source id, then CSR row: (row, source, edge id); that order by CSC row)
     passes = lambda rows: max(1, -(-int(rows).bit_length() // 8))  # noqa: E731

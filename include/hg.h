@@ -186,7 +186,8 @@ hg_status hg_layer_workspace_size(const hg_graph* graph, const hg_layer_params* 
                                   size_t* saved_bytes, size_t* scratch_bytes);
 
 /* Forward pass.  H_in, H_out: N x d in params->dtype (N = type_offsets[num_types]); they must not
- * overlap.  saved: keeps what the backward pass needs (per-relation means, Z, U, row statistics). */
+ * overlap.  saved: keeps what the backward pass needs (the per-relation means of the destination
+ * rows that have in-edges, Z, U, row statistics). */
 hg_status hg_layer_fwd(const hg_graph* graph, const hg_layer_params* params, const void* H_in,
                        void* H_out, void* saved, void* scratch, hg_stream stream);
 

@@ -7,6 +7,9 @@
 //           backward kernel, and dY[i] is the residual-path gradient of Eq. 11.  The sum runs over
 //           node i's row of the node-major out-edge list (its CSC rows of every relation leaving
 //           its type, concatenated in relation order, each edge holding the dMs row it reads).
+// M_r and dMs_r are stored for the non-empty CSR rows only, in the graph's compact order (a row
+// without in-edges has M_r = 0 and is never stored, read or gathered; the projections read it as
+// zeros), and the backward runs name those compact rows.
 // Parallel edges (the same source, destination and relation) are summed once with their
 // multiplicity: the rows read here are the build's runs (column, count), so each distinct
 // neighbour row is gathered once per row and multiplied by its count (deg_r(j) is still the
@@ -279,33 +282,39 @@ __device__ __forceinline__ void gather_row(const int32_t* __restrict__ col, cons
   if (end - beg > kFirst) gather_sum<T, D, kBatchTail>(col, cnt, beg + kFirst, end, 1, 0, src, lane, acc);
 }
 
-// Forward rows: M[row] = mean over the row's neighbours: the row's runs (column, multiplicity),
-// divided by the row's edge count deg (the CSR row length).  Persistent: each group strides over
-// rows and fetches the next row's bounds while it gathers.
+// Forward rows: M[k] = mean over the neighbours of the k-th non-empty CSR row (row = mlist[k]):
+// the row's runs (column, multiplicity), divided by the row's edge count (the CSR row length).
+// Rows without in-edges are not stored (their M is 0; the projection reads them as zeros).
+// Persistent: each group strides over the compact rows and fetches the next row's bounds while it
+// gathers.
 template <typename T, int D>
 __global__ void __launch_bounds__(256) agg_fwd_rows(const int32_t* __restrict__ ptr, const int32_t* __restrict__ col,
                                                     const int32_t* __restrict__ cnt,
-                                                    const int32_t* __restrict__ eptr, const T* __restrict__ H,
-                                                    T* __restrict__ M, int64_t rows,
-                                                    const int32_t* __restrict__ chunk_ofs,
+                                                    const int32_t* __restrict__ eptr, const int32_t* __restrict__ mlist,
+                                                    const int32_t* __restrict__ nnz_p, const T* __restrict__ H,
+                                                    T* __restrict__ M, const int32_t* __restrict__ chunk_ofs,
                                                     const float* __restrict__ partials) {
   using S = AggShape<T, D>;
   const int grp = threadIdx.x / S::G, lane = threadIdx.x % S::G;
   const int64_t step = (int64_t)gridDim.x * S::kGroups;
-  int64_t row = (int64_t)blockIdx.x * S::kGroups + grp;
-  int beg = 0, end = 0, deg = 0;
-  if (row < rows) {
+  const int64_t nnz = *nnz_p;
+  int64_t k = (int64_t)blockIdx.x * S::kGroups + grp;
+  int row = 0, beg = 0, end = 0, deg = 0;
+  if (k < nnz) {
+    row = __ldg(mlist + k);
     beg = __ldg(ptr + row);
     end = __ldg(ptr + row + 1);
     deg = __ldg(eptr + row + 1) - __ldg(eptr + row);
   }
-  while (row < rows) {
-    const int64_t nrow = row + step;
-    int nbeg = 0, nend = 0, ndeg = 0;
-    if (nrow < rows) {
+  int nrow = k + step < nnz ? __ldg(mlist + k + step) : 0;
+  while (k < nnz) {
+    const int64_t nk = k + step;
+    int nbeg = 0, nend = 0, ndeg = 0, nnrow = 0;
+    if (nk < nnz) {
       nbeg = __ldg(ptr + nrow);
       nend = __ldg(ptr + nrow + 1);
       ndeg = __ldg(eptr + nrow + 1) - __ldg(eptr + nrow);
+      if (nk + step < nnz) nnrow = __ldg(mlist + nk + step);
     }
     float acc[S::F];
 #pragma unroll
@@ -314,12 +323,13 @@ __global__ void __launch_bounds__(256) agg_fwd_rows(const int32_t* __restrict__ 
       add_partials<T, D>(partials, chunk_ofs[row], chunk_ofs[row + 1], lane, acc);
     else
       gather_sum<T, D, false>(col, cnt, beg, end, 1, 0, H, lane, acc);
-    const float scale = deg > 0 ? __fdiv_rn(1.0f, (float)deg) : 0.f;
-    store_row<T, D>(M + row * D, lane, acc, scale);
+    store_row<T, D>(M + k * D, lane, acc, __fdiv_rn(1.0f, (float)deg));
+    k = nk;
     row = nrow;
     beg = nbeg;
     end = nend;
     deg = ndeg;
+    nrow = nnrow;
   }
 }
 
@@ -410,8 +420,8 @@ static hg_status agg_fwd_t(const hg_graph* g, const void* H, void* M, float* par
                 dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(g->csr_rows, S::kGroups), pb))),
                 dim3(256),
                 0, s, (const int32_t*)g->agg_ptr, (const int32_t*)g->agg_col, (const int32_t*)g->agg_cnt,
-                (const int32_t*)g->csr_ptr, (const T*)H, (T*)M, g->csr_rows, (const int32_t*)g->agg_chunk_ofs,
-                (const float*)partials);
+                (const int32_t*)g->csr_ptr, (const int32_t*)g->mlist, (const int32_t*)(g->mbase + g->meta.num_rels),
+                (const T*)H, (T*)M, (const int32_t*)g->agg_chunk_ofs, (const float*)partials);
 }
 
 template <typename T, int D>

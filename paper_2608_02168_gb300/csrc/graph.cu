@@ -11,6 +11,12 @@
 // STABLE least-significant-digit radix sort of (key, edge id) places every edge in its row with
 // ascending edge ids, and the row pointers are read off the sorted keys (no atomics, so hub rows
 // cost nothing extra).  The layout is therefore unique and bit-reproducible.
+//
+// Three stable sorts build both layouts: by source id, then by CSR row (so a CSR row lists its
+// in-edges by (source, edge id)), then that order by CSC row (a CSC row lists its out-edges by
+// (destination, edge id)).  Parallel edges are thus adjacent in both, and runs of equal neighbours
+// become the mean layer's aggregation lists (column, multiplicity); the non-empty CSR rows get a
+// compact numbering, the rows in which the mean layer stores M_r and dMs_r.
 #include <algorithm>
 
 #include "hg_internal.cuh"
@@ -365,6 +371,36 @@ __global__ void csc_keys_from_csr(const uint32_t* rkey, const uint32_t* __restri
 }
 
 // ---------------------------------------------------------------------------------------------
+// non-empty CSR rows: the relation rows the mean layer stores (a row without in-edges has M = 0
+// and is never stored, read or gathered)
+// ---------------------------------------------------------------------------------------------
+__global__ void nonempty_flags(const int32_t* __restrict__ ptr, int64_t rows, int32_t* __restrict__ flag) {
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < rows; r += (int64_t)gridDim.x * blockDim.x)
+    flag[r] = ptr[r + 1] > ptr[r] ? 1 : 0;
+}
+
+// mbase[r] = compact index of relation r's first non-empty row (pos = the scan of the flags, whose
+// entry `rows` is the number of non-empty rows).
+__global__ void compact_bases(const int32_t* __restrict__ pos, GraphMeta m, int32_t* __restrict__ mbase) {
+  const int r = threadIdx.x;
+  if (r <= m.num_rels) mbase[r] = pos[m.row_base[r]];
+}
+
+// In place: mrow[row] = its compact index when non-empty, `rows` (out of range) otherwise; mlist[k]
+// = the CSR row of compact row k.
+__global__ void compact_rows(const int32_t* __restrict__ flag, int64_t rows, int32_t* __restrict__ mrow,
+                             int32_t* __restrict__ mlist) {
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < rows; r += (int64_t)gridDim.x * blockDim.x) {
+    const int32_t k = mrow[r];
+    if (flag[r]) {
+      mlist[k] = (int32_t)r;
+    } else {
+      mrow[r] = (int32_t)rows;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------------------------
 // run-length coalescing of parallel edges: a row (ptr, col) whose equal entries are adjacent
 // becomes (uptr, ucol, ucnt): one entry per distinct column with its multiplicity, in the same order
 // ---------------------------------------------------------------------------------------------
@@ -384,16 +420,17 @@ __global__ void run_row_starts(const int32_t* __restrict__ ptr, int64_t rows, in
 }
 
 // With u = the exclusive scan of the flags (u[n] = number of runs): run k = u[p] of a flagged
-// position p gets ucol[k] = col[p] and its start upos[k] = p; upos[U] = n.
+// position p gets ucol[k] = col[p] (or map[col[p]] when a map is given) and its start upos[k] = p;
+// upos[U] = n.
 __global__ void run_write(const int32_t* __restrict__ flag, const int32_t* __restrict__ u,
                           const int32_t* __restrict__ col, const int32_t* __restrict__ ptr, int64_t rows,
-                          int32_t* __restrict__ ucol, int32_t* __restrict__ upos) {
+                          const int32_t* __restrict__ map, int32_t* __restrict__ ucol, int32_t* __restrict__ upos) {
   const int64_t n = ptr[rows];
   for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p <= n; p += (int64_t)gridDim.x * blockDim.x) {
     if (p == n) {
       upos[u[n]] = (int32_t)n;
     } else if (flag[p]) {
-      ucol[u[p]] = col[p];
+      ucol[u[p]] = map ? map[col[p]] : col[p];
       upos[u[p]] = (int32_t)p;
     }
   }
@@ -518,6 +555,7 @@ struct GraphLayout {
   // parallel edges coalesced: CSR rows and node-major rows as (column, multiplicity) runs
   int32_t *agg_ptr, *agg_col, *agg_cnt, *agg_chunk_ofs, *agg_chunk_row;
   int32_t *bagg_ptr, *bagg_col, *bagg_cnt, *bagg_chunk_ofs, *bagg_chunk_row;
+  int32_t *mrow, *mlist, *mbase;  // non-empty CSR rows: compact index per row, row per index, per relation
   SortBuffers sort;
 };
 
@@ -547,6 +585,9 @@ static size_t carve_graph(void* ws, int64_t E, int64_t rows, int64_t crows, int6
   L->bagg_cnt = c.take<int32_t>(Ea);
   L->bagg_chunk_ofs = c.take<int32_t>(N + 1);
   L->bagg_chunk_row = c.take<int32_t>(chunk_cap(E));
+  L->mrow = c.take<int32_t>(rows + 1);
+  L->mlist = c.take<int32_t>(rows + 1);
+  L->mbase = c.take<int32_t>(kMaxRels + 1);
   L->invalid = c.take<int32_t>(1);
   L->cnt = c.take<int32_t>(std::max(std::max(rows, crows), N) + 1);
   L->sort.ckeys = c.take<uint32_t>(Ea + 1);
@@ -614,8 +655,8 @@ static unsigned grid_for(int64_t n, int threads = 256) {
 
 // Runs of equal adjacent entries of (ptr, col): the flags, their scan (the run index of each
 // position) and the runs' columns, multiplicities and row pointers.  Uses the sort buffers.
-static hg_status coalesce_runs(const int32_t* col, const int32_t* ptr, int64_t rows, int64_t E, GraphLayout& L,
-                               int32_t* ucol, int32_t* ucnt, int32_t* uptr, cudaStream_t s) {
+static hg_status coalesce_runs(const int32_t* col, const int32_t* ptr, int64_t rows, int64_t E, const int32_t* map,
+                               GraphLayout& L, int32_t* ucol, int32_t* ucnt, int32_t* uptr, cudaStream_t s) {
   int32_t* flag = reinterpret_cast<int32_t*>(L.sort.keys[0]);
   int32_t* u = reinterpret_cast<int32_t*>(L.sort.keys[1]);
   int32_t* upos = reinterpret_cast<int32_t*>(L.sort.vals[0]);
@@ -623,7 +664,7 @@ static hg_status coalesce_runs(const int32_t* col, const int32_t* ptr, int64_t r
   HG_TRY(launch("run_row_starts", run_row_starts, dim3(grid_for(rows)), dim3(256), 0, s, ptr, rows, flag));
   HG_TRY(exclusive_scan(flag, u, E, L.sort.scan_scratch, s));
   HG_TRY(launch("run_write", run_write, dim3(grid_for(E + 1)), dim3(256), 0, s, (const int32_t*)flag,
-                (const int32_t*)u, col, ptr, rows, ucol, upos));
+                (const int32_t*)u, col, ptr, rows, map, ucol, upos));
   return launch("run_finish", run_finish, dim3(grid_for(std::max(E, rows + 1))), dim3(256), 0, s, (const int32_t*)u,
                 (const int32_t*)upos, ptr, rows, ucnt, uptr);
 }
@@ -726,9 +767,19 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
                   (const uint32_t*)L.sort.vals[res], (const uint32_t*)L.sort.vals2[res], (const int32_t*)L.csc_ptr,
                   crows, m, (const int32_t*)L.csr_ptr, (const int32_t*)L.node_ptr, L.csc_col, L.csc_eid, L.csc_coef,
                   L.node_col));
-    // parallel edges coalesced into (column, multiplicity) runs, in both aggregation orders
-    HG_TRY(coalesce_runs(L.csr_col, L.csr_ptr, rows, E, L, L.agg_col, L.agg_cnt, L.agg_ptr, s));
-    HG_TRY(coalesce_runs(L.node_col, L.node_ptr, N, E, L, L.bagg_col, L.bagg_cnt, L.bagg_ptr, s));
+  }
+  // non-empty CSR rows (the rows the mean layer stores) and their compact numbering
+  HG_TRY(launch("nonempty_flags", nonempty_flags, dim3(grid_for(rows)), dim3(256), 0, s, (const int32_t*)L.csr_ptr,
+                rows, L.cnt));
+  HG_TRY(exclusive_scan(L.cnt, L.mrow, rows, L.sort.scan_scratch, s));
+  HG_TRY(launch("compact_bases", compact_bases, dim3(1), dim3(32), 0, s, (const int32_t*)L.mrow, m, L.mbase));
+  HG_TRY(launch("compact_rows", compact_rows, dim3(grid_for(rows)), dim3(256), 0, s, (const int32_t*)L.cnt, rows,
+                L.mrow, L.mlist));
+  if (E > 0) {
+    // parallel edges coalesced into (column, multiplicity) runs, in both aggregation orders; the
+    // backward runs name the compact row of the dMs row they read
+    HG_TRY(coalesce_runs(L.csr_col, L.csr_ptr, rows, E, nullptr, L, L.agg_col, L.agg_cnt, L.agg_ptr, s));
+    HG_TRY(coalesce_runs(L.node_col, L.node_ptr, N, E, L.mrow, L, L.bagg_col, L.bagg_cnt, L.bagg_ptr, s));
   }
   // chunk tables for rows above the hub degree: per edge (attention layer), per run (mean layer)
   HG_TRY(chunk_table(L.csr_ptr, rows, L.csr_chunk_ofs, L.csr_chunk_row, L, s));
@@ -767,6 +818,9 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
   gh->bagg_cnt = L.bagg_cnt;
   gh->bagg_chunk_ofs = L.bagg_chunk_ofs;
   gh->bagg_chunk_row = L.bagg_chunk_row;
+  gh->mrow = L.mrow;
+  gh->mlist = L.mlist;
+  gh->mbase = L.mbase;
   gh->invalid_count = L.invalid;
   *out = gh;
   return HG_OK;

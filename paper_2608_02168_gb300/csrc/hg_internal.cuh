@@ -140,6 +140,13 @@ struct hg_graph {
   int32_t* bagg_cnt;
   int32_t* bagg_chunk_ofs;  // [N + 1]
   int32_t* bagg_chunk_row;  // [chunk_cap_node]
+  // Non-empty CSR rows (the mean layer stores M_r and dMs_r only for them, in compact order):
+  // mrow[row] = compact index, or csr_rows for an empty row (an out-of-range row, read as zeros by
+  // the tensor-core loads); mlist[k] = CSR row of compact row k; mbase[r] = first compact row of
+  // relation r (mbase[num_rels] = their number).  The backward runs (bagg_col) hold compact rows.
+  int32_t* mrow;            // [csr_rows + 1]
+  int32_t* mlist;           // [csr_rows + 1]
+  int32_t* mbase;           // [kMaxRels + 1], device
   int32_t* invalid_count;  // device scalar
 };
 

@@ -842,7 +842,7 @@ hg_status hgt_fwd_t(const hg_graph* g, const hg_hgt_params* p, const void* H_in,
     HG_TRY(launch("hgt_fwd_nodes", hgt_fwd_nodes<T, D, kMaxRels>, dim3(grid_of(N * 32)), dim3(256), 0, s, a));
   // Eq. 11 on S_r with W_rel = blockdiag(W_msg[r])
   const hg_layer_params lp = projection_params(p, H);
-  return project_forward(g, &lp, H_in, H_out, H.L, s);
+  return project_forward(g, &lp, H_in, H_out, H.L, false, s);
 }
 
 template <typename T, int D>
@@ -863,7 +863,7 @@ hg_status hgt_bwd_t(const hg_graph* g, const hg_hgt_params* p, const void* H_in,
   lg.db_agg = gr->db_agg;
   lg.dln_gamma = gr->dln_gamma;
   lg.dln_beta = gr->dln_beta;
-  HG_TRY(project_backward(g, &lp, H_in, dH_out, &lg, H.L, false, s));
+  HG_TRY(project_backward(g, &lp, H_in, dH_out, &lg, H.L, false, false, s));
   // attention backward: target pass (dQ'), source pass (dK, dV)
   const HgtArgs a = edge_args(g, p, H);
   HG_TRY(launch("hgt_bwd_dstats", hgt_bwd_dstats<T, D>, dim3(grid_of(N * 32)), dim3(256), 0, s, a));

@@ -238,7 +238,7 @@ extern "C" hg_status hg_layer_fwd(const hg_graph* graph, const hg_layer_params* 
   LayerLayout L;
   carve_layer(graph, d, p->dtype, saved, scratch, &L, nullptr, nullptr);
   HG_TRY(aggregate_forward(graph, p->dtype, d, H_in, L.M, L.agg_part, s));
-  return project_forward(graph, p, H_in, H_out, L, s);
+  return project_forward(graph, p, H_in, H_out, L, true, s);
 }
 
 namespace hg {
@@ -246,7 +246,7 @@ namespace hg {
 // Eq. 7 and Eq. 11 from the relation rows in L.M: U = sum_r M_r W_r W_agg + b, activation,
 // residual, optional LayerNorm.
 hg_status project_forward(const hg_graph* graph, const hg_layer_params* p, const void* H_in, void* H_out,
-                          const LayerLayout& L, cudaStream_t s) {
+                          const LayerLayout& L, bool compact, cudaStream_t s) {
   const GraphMeta& m = graph->meta;
   const int d = p->d;
   const size_t b = elem_size(p->dtype);
@@ -262,6 +262,8 @@ hg_status project_forward(const hg_graph* graph, const hg_layer_params* p, const
         ++a.nrel;
       }
       a.type = t;
+      a.mrow = compact ? graph->mrow : nullptr;
+      a.msent = graph->csr_rows;
       a.b = (const __nv_bfloat16*)p->b_agg + (size_t)t * d;
       a.gamma = p->layernorm ? (const __nv_bfloat16*)p->ln_gamma + (size_t)t * d : nullptr;
       a.beta = p->layernorm ? (const __nv_bfloat16*)p->ln_beta + (size_t)t * d : nullptr;
@@ -282,6 +284,8 @@ hg_status project_forward(const hg_graph* graph, const hg_layer_params* p, const
   for (int t = 0; t < m.num_types; ++t) {
     FwdArgs a{};
     a.M = L.M;
+    a.mrow = compact ? graph->mrow : nullptr;
+    a.msent = graph->csr_rows;
     for (int r = 0; r < m.num_rels; ++r) {
       if (m.rel_dst[r] != t) continue;
       a.mrow0[a.nrel] = m.row_base[r];
@@ -326,7 +330,7 @@ extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   LayerLayout L;
   carve_layer(graph, p->d, p->dtype, const_cast<void*>(saved), scratch, &L, nullptr, nullptr);
-  HG_TRY(project_backward(graph, p, H_in, dH_out, grads, L, true, s));
+  HG_TRY(project_backward(graph, p, H_in, dH_out, grads, L, true, true, s));
   if (dH_in) HG_TRY(aggregate_backward(graph, p->dtype, p->d, L.dMs, L.dY, dH_in, L.agg_part, s));
   return HG_OK;
 }
@@ -336,7 +340,8 @@ namespace hg {
 // Backward of project_forward: L.dY = the residual path's dL/dH_in, L.dMs = dL/dM_r (divided by
 // deg_r when deg_scale is set, for the mean's transposed gather), and every weight gradient.
 hg_status project_backward(const hg_graph* graph, const hg_layer_params* p, const void* H_in, const void* dH_out,
-                           const hg_layer_grads* grads, const LayerLayout& L, bool deg_scale, cudaStream_t s) {
+                           const hg_layer_grads* grads, const LayerLayout& L, bool deg_scale, bool compact,
+                           cudaStream_t s) {
   const GraphMeta& m = graph->meta;
   const int d = p->d;
   const size_t b = elem_size(p->dtype);
@@ -374,6 +379,8 @@ hg_status project_backward(const hg_graph* graph, const hg_layer_params* p, cons
       a.gamma = p->layernorm ? (const __nv_bfloat16*)p->ln_gamma + (size_t)t * d : nullptr;
       a.b = (const __nv_bfloat16*)p->b_agg + (size_t)t * d;
       a.csr_ptr = deg_scale ? graph->csr_ptr : nullptr;
+      a.mlist = compact ? graph->mlist : nullptr;
+      a.mbase = compact ? graph->mbase : nullptr;
       a.dY = (__nv_bfloat16*)L.dY;
       a.dU = (__nv_bfloat16*)L.dU;
       a.dMs = (__nv_bfloat16*)L.dMs;
@@ -400,6 +407,8 @@ hg_status project_backward(const hg_graph* graph, const hg_layer_params* p, cons
         ++a.nrel;
       }
       a.csr_ptr = deg_scale ? graph->csr_ptr : nullptr;
+      a.mrow = compact ? graph->mrow : nullptr;
+      a.msent = graph->csr_rows;
       a.dY = L.dY;
       a.dU = L.dU;
       a.dZ = L.dZ;
@@ -419,7 +428,14 @@ hg_status project_backward(const hg_graph* graph, const hg_layer_params* p, cons
     if (!tc)
       HG_TRY(weight_grad(p->dtype, d, L.Z, off, L.dU, off, n, L.wpart, grads->dW_agg + (size_t)t * d * d, L.rtmp, s));
   }
-  if (tc) {  // G_r = M_r^T dU, the relations into one type sharing the loads of dU
+  if (tc && compact) {  // G_r = M_r^T dU over each relation's stored rows (dU rows gathered)
+    for (int r = 0; r < m.num_rels; ++r) {
+      const int t = m.rel_dst[r];
+      HG_TRY(tc_weight_grad_rows(d, L.M, graph->csr_rows, graph->mlist, graph->mbase, r, m.row_base[r], L.dU,
+                                 m.type_off[t], m.type_off[t + 1] - m.type_off[t], L.wpart, L.G + (size_t)r * d * d,
+                                 L.rtmp, s));
+    }
+  } else if (tc) {  // G_r = M_r^T dU, the relations into one type sharing the loads of dU
     for (int t = 0; t < m.num_types; ++t) {
       const int64_t n = m.type_off[t + 1] - m.type_off[t];
       int64_t x0[kMaxRels];
@@ -442,7 +458,8 @@ hg_status project_backward(const hg_graph* graph, const hg_layer_params* p, cons
       const int t = m.rel_dst[r];
       const int64_t n = m.type_off[t + 1] - m.type_off[t];
       HG_TRY(weight_grad(p->dtype, d, L.M, m.row_base[r], L.dZ, m.type_off[t], n, L.wpart,
-                         grads->dW_rel + (size_t)r * d * d, L.rtmp, s));
+                         grads->dW_rel + (size_t)r * d * d, L.rtmp, s, compact ? graph->mrow : nullptr,
+                         graph->csr_rows));
     }
   }
   if (tc)  // dW_r = G_r W_agg^T, dW_agg[t] = sum_{r -> t} W_r^T G_r

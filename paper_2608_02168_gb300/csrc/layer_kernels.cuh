@@ -9,7 +9,9 @@
 namespace hg {
 
 struct FwdArgs {
-  const void* M;                 // saved relation means, concatenated CSR rows
+  const void* M;                 // saved relation means, concatenated CSR rows (or compact rows)
+  const int32_t* mrow;           // compact index of each CSR row (>= msent: empty); null: M by CSR row
+  int64_t msent;
   int nrel;
   int64_t mrow0[kMaxRels];       // first CSR row of each relation into this type
   const void* W_rel[kMaxRels];   // its D x D message matrix (d_in x d_out)
@@ -41,7 +43,9 @@ struct BwdArgs {
   void* dY;                      // node rows
   void* dU;                      // node rows
   void* dZ;                      // node rows
-  void* dMs;                     // concatenated CSR rows (scaled by 1/deg)
+  void* dMs;                     // concatenated CSR rows (scaled by 1/deg), or compact rows
+  const int32_t* mrow;           // compact index of each CSR row (>= msent: empty, not stored); null: CSR rows
+  int64_t msent;
   float* part;                   // [blocks][3][D]: db, dgamma, dbeta partials
   int64_t off, n;
   int act, ln;
@@ -52,6 +56,8 @@ struct TcFwdArgs {
   int nrel;
   int rel[kMaxRels];          // relation ids into this type (row block of W_rel^T)
   int64_t mrow0[kMaxRels];    // first CSR row of each
+  const int32_t* mrow;        // row of M holding each CSR row (>= msent: an empty row, read as zeros);
+  int64_t msent;              // null: M is indexed by CSR row.  msent = the row extent of M
   int type;
   const __nv_bfloat16* b;
   const __nv_bfloat16* gamma;
@@ -70,6 +76,8 @@ struct TcBwdArgs {
   int nrel;
   int rel[kMaxRels];
   int64_t mrow0[kMaxRels];
+  const int32_t* mlist;       // CSR row of each compact row; mbase[r] .. mbase[r + 1] = relation r's
+  const int32_t* mbase;       // compact rows (device).  null: every CSR row, dMs indexed by CSR row
   int type;
   const __nv_bfloat16* dH_out;
   const __nv_bfloat16* H_in;
@@ -99,6 +107,11 @@ hg_status tc_ln_act_backward(int d, const TcBwdArgs& a, int* blocks, cudaStream_
 hg_status tc_proj_backward(int d, const TcBwdArgs& a, const void* V, int num_rels, cudaStream_t s);
 // outs[r] = X[x0[r] .. x0[r]+n)^T Y[y0 .. y0+n) for r < R (R <= wgrad_tc_max_rels(d)); the R
 // products share the loads of Y.  part: R x wgrad_tc_splits(n, d) x d x d floats.
+// out = G_r = M^T dU over relation `rel`'s stored rows: compact rows mbase[rel] .. mbase[rel + 1]
+// of M (m_rows rows in all) paired with dU rows mlist[k] - row0 (of the type's n rows at y0).
+hg_status tc_weight_grad_rows(int d, const void* M, int64_t m_rows, const int32_t* mlist, const int32_t* mbase, int rel,
+                              int64_t row0, const void* dU, int64_t y0, int64_t n, float* part, float* out, float* tmp,
+                              cudaStream_t s);
 hg_status tc_weight_grad(int d, const void* X, const int64_t* x0, int R, const void* Y, int64_t y0, int64_t n,
                          float* part, float* const* outs, float* tmp, cudaStream_t s);
 int wgrad_tc_max_rels(int d);
@@ -113,8 +126,10 @@ hg_status aggregate_backward(const hg_graph* g, hg_dtype dt, int d, const void* 
                              float* partials, cudaStream_t s);
 hg_status proj_forward(hg_dtype dt, int d, const FwdArgs& a, cudaStream_t s);
 hg_status proj_backward(hg_dtype dt, int d, const BwdArgs& a, cudaStream_t s);
+// out = X^T Y over rows [x0, x0 + n) of X and [y0, y0 + n) of Y; with xmap, X row x0 + k is
+// X[xmap[x0 + k]] and a mapped row >= xsent is zero (X stored for non-empty rows only).
 hg_status weight_grad(hg_dtype dt, int d, const void* X, int64_t x0, const void* Y, int64_t y0, int64_t n, float* part,
-                      float* out, float* tmp, cudaStream_t s);
+                      float* out, float* tmp, cudaStream_t s, const int32_t* xmap = nullptr, int64_t xsent = 0);
 hg_status transpose_weights(hg_dtype dt, int d, const void* W, void* Wt, int count, cudaStream_t s);
 // fixed-order sum of `splits` partial arrays (tmp: reduce_tmp_floats(splits, count) floats)
 hg_status reduce_partials(const float* part, int64_t stride, int splits, int64_t count, float* out, float* tmp,
@@ -155,11 +170,14 @@ void carve_layer(const hg_graph* g, int d, hg_dtype dt, void* saved, void* scrat
                  size_t* saved_bytes, size_t* scratch_bytes);
 RelDst rel_dst_of(const GraphMeta& m);
 // Eq. 7 and Eq. 11 from the relation rows in L.M (bias, activation, residual, optional LayerNorm).
+// compact: L.M holds the non-empty CSR rows only, in the graph's compact order (the mean layer);
+// otherwise one row per CSR row (the attention layer's weighted sums).
 hg_status project_forward(const hg_graph* graph, const hg_layer_params* p, const void* H_in, void* H_out,
-                          const LayerLayout& L, cudaStream_t s);
-// Its backward: L.dY (residual path), L.dMs (dL/dM_r, divided by deg_r when deg_scale), the weight
-// gradients into grads.
+                          const LayerLayout& L, bool compact, cudaStream_t s);
+// Its backward: L.dY (residual path), L.dMs (dL/dM_r, divided by deg_r when deg_scale; compact rows
+// when compact), the weight gradients into grads.
 hg_status project_backward(const hg_graph* graph, const hg_layer_params* p, const void* H_in, const void* dH_out,
-                           const hg_layer_grads* grads, const LayerLayout& L, bool deg_scale, cudaStream_t s);
+                           const hg_layer_grads* grads, const LayerLayout& L, bool deg_scale, bool compact,
+                           cudaStream_t s);
 
 }  // namespace hg

@@ -42,7 +42,7 @@ __global__ void __launch_bounds__(256) proj_fwd_simt(FwdArgs a) {
     for (int j = 0; j < CN; ++j) acc[i][j] = 0.f;
   for (int r = 0; r < a.nrel; ++r) {
     for (int k0 = 0; k0 < D; k0 += kKC) {
-      stage_a<T, D>(As, (const T*)a.M, a.mrow0[r] + m0, nv, k0);
+      stage_a<T, D>(As, (const T*)a.M, a.mrow0[r] + m0, nv, k0, a.mrow, a.msent);
       stage_b<T, D>(Bs, (const T*)a.W_rel[r], k0);
       __syncthreads();
       mma_chunk<D, RM, CN>(&As[0][0], kAPad, 0, Bs, acc);
@@ -227,12 +227,14 @@ __global__ void __launch_bounds__(256) proj_bwd_simt(BwdArgs a) {
       const int m = ty * RM + i;
       if (m >= nv) continue;
       const int64_t row = a.mrow0[r] + m0 + m;
+      const int64_t out = a.mrow ? (int64_t)a.mrow[row] : row;  // compact rows: empty rows are not stored
+      if (a.mrow && out >= a.msent) continue;
       const int deg = a.csr_ptr ? a.csr_ptr[row + 1] - a.csr_ptr[row] : 0;
       const float sc = !a.csr_ptr ? 1.f : (deg > 0 ? __fdiv_rn(1.0f, (float)deg) : 0.f);
       float v[CN];
 #pragma unroll
       for (int j = 0; j < CN; ++j) v[j] = acc[i][j] * sc;
-      store_cols<T, CN>((T*)a.dMs + row * D + tx * CN, v);
+      store_cols<T, CN>((T*)a.dMs + out * D + tx * CN, v);
     }
   }
 }
@@ -246,7 +248,8 @@ constexpr int kWR = 32;   // rows per step
 template <typename T, int D>
 __global__ void __launch_bounds__(256) wgrad_partial(const T* __restrict__ X, int64_t x0, const T* __restrict__ Y,
                                                      int64_t y0, int64_t n, int64_t rows_per_split,
-                                                     float* __restrict__ part) {
+                                                     float* __restrict__ part, const int32_t* __restrict__ xmap,
+                                                     int64_t xsent) {
   constexpr int TW = D < kWT ? D : kWT;
   constexpr int TPT = TW / 16;  // outputs per thread per dim
   constexpr int VEC = VecTraits<T>::kElems;
@@ -266,8 +269,9 @@ __global__ void __launch_bounds__(256) wgrad_partial(const T* __restrict__ X, in
     for (int idx = threadIdx.x; idx < kWR * TW / VEC; idx += blockDim.x) {
       const int k = idx / (TW / VEC), cv = idx % (TW / VEC);
       float fx[VEC], fy[VEC];
-      if (rb + k < r1) {
-        unpack(ldg16(X + (x0 + rb + k) * D + ti * TW + cv * VEC), fx, T());
+      const int64_t xr = rb + k < r1 ? (xmap ? (int64_t)xmap[x0 + rb + k] : x0 + rb + k) : 0;
+      if (rb + k < r1 && (!xmap || xr < xsent)) {
+        unpack(ldg16(X + xr * D + ti * TW + cv * VEC), fx, T());
         unpack(ldg16(Y + (y0 + rb + k) * D + tj * TW + cv * VEC), fy, T());
       } else {
 #pragma unroll
@@ -395,13 +399,13 @@ hg_status reduce_partials(const float* part, int64_t stride, int splits, int64_t
 
 template <typename T, int D>
 static hg_status wgrad_t(const void* X, int64_t x0, const void* Y, int64_t y0, int64_t n, float* part, float* out,
-                         float* tmp, cudaStream_t s) {
+                         float* tmp, const int32_t* xmap, int64_t xsent, cudaStream_t s) {
   const int splits = wgrad_splits(n);
   const int64_t rps = ceil_div(std::max<int64_t>(n, 1), splits);
   constexpr int TW = D < kWT ? D : kWT;
   const int tiles = (D / TW) * (D / TW);
   HG_TRY(launch("wgrad_partial", wgrad_partial<T, D>, dim3(tiles, splits), dim3(256), 0, s, (const T*)X, x0,
-                (const T*)Y, y0, n, rps, part));
+                (const T*)Y, y0, n, rps, part, xmap, xsent));
   return reduce_partials(part, (int64_t)D * D, splits, (int64_t)D * D, out, tmp, s);
 }
 
@@ -429,8 +433,8 @@ static hg_status transpose_t(const void* W, void* Wt, int count, cudaStream_t s)
 hg_status proj_forward(hg_dtype dt, int d, const FwdArgs& a, cudaStream_t s) { HG_DISPATCH_TD2(dt, d, proj_fwd_t, a, s); }
 hg_status proj_backward(hg_dtype dt, int d, const BwdArgs& a, cudaStream_t s) { HG_DISPATCH_TD2(dt, d, proj_bwd_t, a, s); }
 hg_status weight_grad(hg_dtype dt, int d, const void* X, int64_t x0, const void* Y, int64_t y0, int64_t n, float* part,
-                      float* out, float* tmp, cudaStream_t s) {
-  HG_DISPATCH_TD2(dt, d, wgrad_t, X, x0, Y, y0, n, part, out, tmp, s);
+                      float* out, float* tmp, cudaStream_t s, const int32_t* xmap, int64_t xsent) {
+  HG_DISPATCH_TD2(dt, d, wgrad_t, X, x0, Y, y0, n, part, out, tmp, xmap, xsent, s);
 }
 hg_status transpose_weights(hg_dtype dt, int d, const void* W, void* Wt, int count, cudaStream_t s) {
   HG_DISPATCH_TD2(dt, d, transpose_t, W, Wt, count, s);

@@ -57,7 +57,8 @@ struct FwdCfg {
   static constexpr bool kHTile = D <= 128;
   static constexpr int kH = kHTile ? kTileRows * D * 2 : 0;
   static constexpr int kParams = 3 * D * 4;  // bias, gamma, beta in fp32
-  static constexpr int kSmem = kStages * kStage + 2 * kH + kParams + 512 + 1024;
+  static constexpr int kIdx = kTileRows * 4;  // the tile's A-row coordinates
+  static constexpr int kSmem = kStages * kStage + 2 * kH + kParams + kIdx + 512 + 1024;
   static_assert(kSmem <= 227 * 1024, "shared memory of proj_fwd_tc");
   static constexpr int kAccCols = D < 32 ? 32 : D;
   static constexpr int kTmemCols = 2 * kAccCols;
@@ -100,7 +101,8 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
   uint8_t* stage = smem;                  // S x (A | B)
   uint8_t* htile = smem + S * C::kStage;  // 2 x KC x 16 KB, 128B-swizzled rows
   float* params = reinterpret_cast<float*>(htile + 2 * C::kH);  // [3][D]: b, gamma, beta
-  uint64_t* full = reinterpret_cast<uint64_t*>(params + 3 * D);
+  int32_t* sidx = reinterpret_cast<int32_t*>(params + 3 * D);    // [128] rows of M gathered into A
+  uint64_t* full = reinterpret_cast<uint64_t*>(sidx + kTileRows);
   uint64_t* empty = full + S;
   uint64_t* acc_full = empty + S;   // [2] MMA -> epilogue
   uint64_t* acc_empty = acc_full + 2;  // [2] epilogue -> MMA
@@ -134,34 +136,52 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
   const uint32_t tmem = *tslot;
 
   if (warp == 0) {
-    // ---- TMA producer
-    if (lane == 0) {
-      bool ok = true;
-      uint32_t g = 0;
-      int it = 0;
-      for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
-        const int64_t m0 = tile * kTileRows;
-        const int b = it & 1;
-        if (C::kHTile) {
-          if (it >= 2) ok = mbar_wait(&h_empty[b], ((it >> 1) - 1) & 1);
-          if (!ok) break;
+    // ---- TMA producer (the warp writes each relation tile's row coordinates, lane 0 issues):
+    // A rows by gather (four rows per copy), a row past the type or an empty relation row at or past
+    // the map's extent reads zeros; V_r^T hi / lo chunks and the residual tile by tile loads
+    bool ok = true;
+    uint32_t g = 0;
+    int it = 0;
+    for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
+      const int64_t m0 = tile * kTileRows;
+      const int b = it & 1;
+      if (C::kHTile && lane == 0) {
+        if (it >= 2) ok = mbar_wait(&h_empty[b], ((it >> 1) - 1) & 1);
+        if (ok) {
           mbar_expect_tx(&h_full[b], C::kH);
-          for (int kc = 0; kc < KC; ++kc) tma_load_2d(htile + b * C::kH + kc * kATile, &tm_H, kc * 64, (int)m0, &h_full[b]);
-        }
-        for (int j = 0; j < CT && ok; ++j, ++g) {
-          const uint32_t s = g % S;
-          if (g >= (uint32_t)S) ok = mbar_wait(&empty[s], ((g / S) - 1) & 1);
-          if (!ok) break;
-          uint8_t* A = stage + s * C::kStage;
-          const int r = j / KC, kc = j % KC;
-          mbar_expect_tx(&full[s], C::kStage);
-          tma_load_2d(A, &tm_M, kc * 64, (int)(a.mrow0[r] + m0), &full[s]);
-          tma_load_2d(A + kATile, &tm_Vt, kc * 64, 2 * a.rel[r] * D, &full[s]);           // hi
-          tma_load_2d(A + kATile + C::kB, &tm_Vt, kc * 64, (2 * a.rel[r] + 1) * D, &full[s]);  // lo
+          for (int kc = 0; kc < KC; ++kc)
+            tma_load_2d(htile + b * C::kH + kc * kATile, &tm_H, kc * 64, (int)m0, &h_full[b]);
         }
       }
-      if (!ok) atomicOr(a.status, kErrTimeout);
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      for (int r = 0; r < a.nrel && ok; ++r) {
+        for (int i = lane; i < kTileRows; i += 32) {
+          const int64_t m = m0 + i;
+          int64_t c = a.msent;
+          if (m < a.n) c = a.mrow ? (int64_t)a.mrow[a.mrow0[r] + m] : a.mrow0[r] + m;
+          sidx[i] = (int32_t)c;
+        }
+        __syncwarp();
+        if (lane == 0) {
+          for (int kc = 0; kc < KC && ok; ++kc, ++g) {
+            const uint32_t s = g % S;
+            if (g >= (uint32_t)S) ok = mbar_wait(&empty[s], ((g / S) - 1) & 1);
+            if (!ok) break;
+            uint8_t* A = stage + s * C::kStage;
+            mbar_expect_tx(&full[s], C::kStage);
+#pragma unroll 4
+            for (int q = 0; q < kTileRows / 4; ++q)
+              tma_gather4(A + q * 512, &tm_M, kc * 64, sidx[4 * q], sidx[4 * q + 1], sidx[4 * q + 2], sidx[4 * q + 3],
+                          &full[s]);
+            tma_load_2d(A + kATile, &tm_Vt, kc * 64, 2 * a.rel[r] * D, &full[s]);           // hi
+            tma_load_2d(A + kATile + C::kB, &tm_Vt, kc * 64, (2 * a.rel[r] + 1) * D, &full[s]);  // lo
+          }
+        }
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        __syncwarp();  // the coordinates are rewritten for the next relation
+      }
     }
+    if (lane == 0 && !ok) atomicOr(a.status, kErrTimeout);
     __syncwarp();
   } else if (warp == 1) {
     // ---- MMA issuer: U_tile = sum_r M_r V_r into accumulator (it & 1)
@@ -571,56 +591,76 @@ struct BwdCfg {
   static constexpr int kStages = D == 64 ? 4 : (D == 128 ? 3 : 2);  // ring of V_r chunks (hi and lo)
   static constexpr int kB = D * 128;                    // D rows x 64 columns, one half of the pair
   static constexpr int kBStage = 2 * kB;
-  static constexpr int kT = kTileRows * D * 2;          // dU operand tile (KC x 16 KB)
+  static constexpr int kT = kTileRows * D * 2;          // gathered dU operand tile (KC x 16 KB)
   static constexpr int kABuf = D == 256 ? 1 : 2;        // dU tiles in flight (shared memory allowing)
   static constexpr int kAcc = D < 32 ? 32 : D;
   static constexpr int kNumAcc = 512 / kAcc < 4 ? 512 / kAcc : 4;  // ring of TMEM accumulators
   static constexpr int kTmemCols = kNumAcc * kAcc;
   static constexpr int kEpiGroups = 2;  // epilogue warp groups, taking alternate accumulators
-  // Output tiles staged in shared memory (128B-swizzled, one per epilogue group) and written by
-  // TMA, where shared memory allows it; at D = 256 each thread stores its own row.
-  static constexpr bool kTmaOut = D <= 128;
-  static constexpr int kOut = kTmaOut ? kTileRows * D * 2 : 0;
-  static constexpr int kSmem = kStages * kBStage + kABuf * kT + kEpiGroups * kOut + 512 + 1024;
+  static constexpr int kIdx = kTileRows * 4;
+  static constexpr int kSmem = kStages * kBStage + kABuf * kT + kIdx + 512 + 1024;
   static constexpr int kThreads = 64 + kEpiGroups * 128;
   static_assert(kSmem <= 227 * 1024, "shared memory of proj_bwd_tc");
 };
 
-// one tensor map per relation over its dMs rows [mrow0[r], mrow0[r] + n): a partial last tile is
-// clipped at the relation's end instead of running into the next relation's rows
+// one tensor map per relation (used by the weight-gradient kernel's operands)
 struct RelMaps {
   CUtensorMap m[kMaxRels];
 };
 
-// dMs_r = (dU V_r^T) / deg_r for every relation r into this type.  Persistent, one CTA per SM:
-// warp 0 loads dU tiles and V_r chunks (TMA), warp 1 issues one MMA chain per (tile, relation)
-// into a ring of TMEM accumulators, and two groups of four warps (2-5, 6-9) scale and store
-// alternate accumulators, so the stores of one relation overlap the products of the next.
+// The jobs of proj_bwd_tc: 128 rows of one relation's stored rows each, relation by relation.
+struct BwdJobs {
+  int nrel;
+  int64_t base[kMaxRels];   // first stored row of relation j (compact index, or 0 by CSR row)
+  int64_t count[kMaxRels];  // its stored rows
+  int64_t first[kMaxRels + 1];  // first job of relation j; first[nrel] = the number of jobs
+  __device__ __forceinline__ void init(const TcBwdArgs& a) {  // one thread
+    nrel = a.nrel;
+    first[0] = 0;
+    for (int j = 0; j < a.nrel; ++j) {
+      base[j] = a.mlist ? (int64_t)a.mbase[a.rel[j]] : 0;
+      count[j] = a.mlist ? (int64_t)a.mbase[a.rel[j] + 1] - base[j] : a.n;
+      first[j + 1] = first[j] + (count[j] + kTileRows - 1) / kTileRows;
+    }
+  }
+  __device__ __forceinline__ int rel_of(int64_t job) const {
+    int j = 0;
+    while (j + 1 < nrel && job >= first[j + 1]) ++j;
+    return j;
+  }
+};
+
+// dMs_r = (dU V_r^T) / deg_r for the stored rows of every relation r into this type (the non-empty
+// CSR rows, in compact order; or every CSR row without a compact list).  Persistent, one CTA per
+// SM, one job = 128 stored rows of one relation: warp 0 gathers the rows' dU (TMA gathers by the
+// rows' destination nodes) and streams V_r chunks (hi and lo halves), warp 1 issues the job's MMA
+// chain into a ring of TMEM accumulators, and two groups of four warps (2-5, 6-9) scale alternate
+// jobs by 1/deg and store them, so the stores of one job overlap the products of the next.
 template <int D>
 __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
-    proj_bwd_tc(const __grid_constant__ CUtensorMap tm_dU, const __grid_constant__ CUtensorMap tm_V,
-                const __grid_constant__ RelMaps tm_out, TcBwdArgs a) {
+    proj_bwd_tc(const __grid_constant__ CUtensorMap tm_dU, const __grid_constant__ CUtensorMap tm_V, TcBwdArgs a) {
   using C = BwdCfg<D>;
   constexpr int S = C::kStages;
   constexpr int NB = C::kNumAcc;
+  constexpr int NA = C::kABuf;
   constexpr int KC = D / 64;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  constexpr int NA = C::kABuf;
-  uint8_t* bstage = smem;                 // S x (B_hi | B_lo) chunk
+  uint8_t* bstage = smem;                  // S x (B_hi | B_lo) chunk
   uint8_t* tiles = smem + S * C::kBStage;  // NA x (KC x 16 KB)
-  uint8_t* outs = tiles + NA * C::kT;     // kEpiGroups x (KC x 16 KB) output staging
-  uint64_t* b_full = reinterpret_cast<uint64_t*>(outs + C::kEpiGroups * C::kOut);
+  int32_t* sidx = reinterpret_cast<int32_t*>(tiles + NA * C::kT);  // [128] gathered dU rows
+  uint64_t* b_full = reinterpret_cast<uint64_t*>(sidx + kTileRows);
   uint64_t* b_empty = b_full + S;
-  uint64_t* a_full = b_empty + S;       // [NA] dU tile loaded
-  uint64_t* a_empty = a_full + 2;       // [NA] every product of the tile done
+  uint64_t* a_full = b_empty + S;       // [NA] dU tile gathered
+  uint64_t* a_empty = a_full + 2;       // [NA] the job's products done
   uint64_t* acc_full = a_empty + 2;     // [NB]
   uint64_t* acc_empty = acc_full + NB;  // [NB]
   uint32_t* tslot = reinterpret_cast<uint32_t*>(acc_empty + NB);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t ntiles = (a.n + kTileRows - 1) / kTileRows;
+  __shared__ BwdJobs J;
   if (threadIdx.x == 0) {
+    J.init(a);
     for (int s = 0; s < S; ++s) {
       mbar_init(&b_full[s], 1);
       mbar_init(&b_empty[s], 1);
@@ -642,135 +682,119 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
   __syncthreads();
   fence_after_sync();
   const uint32_t tmem = *tslot;
+  const int64_t njobs = J.first[J.nrel];
 
-  if (warp == 0) {
-    if (lane == 0) {  // ---- TMA producer
-      bool ok = true;
-      uint32_t g = 0;
-      int it = 0;
-      for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
+  if (warp == 0) {  // ---- producer: the warp writes the job's dU rows, lane 0 issues the copies
+    bool ok = true;
+    uint32_t g = 0;
+    int it = 0;
+    for (int64_t job = blockIdx.x; job < njobs && ok; job += gridDim.x, ++it) {
+      const int j = J.rel_of(job);
+      const int64_t i0 = (job - J.first[j]) * kTileRows;  // first row of the job within the relation
+      for (int t = lane; t < kTileRows; t += 32) {
+        const int64_t k = i0 + t;
+        int64_t local = a.n;  // past the relation's rows: zeros
+        if (k < J.count[j]) local = a.mlist ? (int64_t)a.mlist[J.base[j] + k] - a.mrow0[j] : k;
+        sidx[t] = (int32_t)local;
+      }
+      __syncwarp();
+      if (lane == 0) {
         const int ab = it % NA;
         if (it >= NA) ok = mbar_wait(&a_empty[ab], ((it / NA) - 1) & 1);
-        if (!ok) break;
-        mbar_expect_tx(&a_full[ab], C::kT);
-        for (int kc = 0; kc < KC; ++kc)
-          tma_load_2d(tiles + ab * C::kT + kc * kATile, &tm_dU, kc * 64, (int)(tile * kTileRows), &a_full[ab]);
-        for (int j = 0; j < a.nrel * KC && ok; ++j, ++g) {
+        if (ok) {
+          mbar_expect_tx(&a_full[ab], C::kT);
+          uint8_t* A = tiles + ab * C::kT;
+          for (int kc = 0; kc < KC; ++kc)
+#pragma unroll 4
+            for (int q = 0; q < kTileRows / 4; ++q)
+              tma_gather4(A + kc * kATile + q * 512, &tm_dU, kc * 64, sidx[4 * q], sidx[4 * q + 1], sidx[4 * q + 2],
+                          sidx[4 * q + 3], &a_full[ab]);
+        }
+        for (int kc = 0; kc < KC && ok; ++kc, ++g) {
           const uint32_t s = g % S;
           if (g >= (uint32_t)S) ok = mbar_wait(&b_empty[s], ((g / S) - 1) & 1);
           if (!ok) break;
           mbar_expect_tx(&b_full[s], C::kBStage);
-          tma_load_2d(bstage + s * C::kBStage, &tm_V, (j % KC) * 64, 2 * a.rel[j / KC] * D, &b_full[s]);
-          tma_load_2d(bstage + s * C::kBStage + C::kB, &tm_V, (j % KC) * 64, (2 * a.rel[j / KC] + 1) * D,
-                      &b_full[s]);
+          tma_load_2d(bstage + s * C::kBStage, &tm_V, kc * 64, 2 * a.rel[j] * D, &b_full[s]);
+          tma_load_2d(bstage + s * C::kBStage + C::kB, &tm_V, kc * 64, (2 * a.rel[j] + 1) * D, &b_full[s]);
         }
       }
-      if (!ok) atomicOr(a.status, kErrTimeout);
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      __syncwarp();  // the row list is rewritten for the next job
     }
+    if (lane == 0 && !ok) atomicOr(a.status, kErrTimeout);
     __syncwarp();
   } else if (warp == 1) {
-    if (lane == 0) {  // ---- MMA issuer
+    if (lane == 0) {  // ---- MMA issuer: one chain per job into accumulator (job count mod NB)
       const uint32_t idesc = idesc_bf16(128, D, false, false);
       bool ok = true;
       uint32_t g = 0, jb = 0;
       int it = 0;
-      for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
+      for (int64_t job = blockIdx.x; job < njobs && ok; job += gridDim.x, ++it, ++jb) {
         const int ab = it % NA;
         ok = mbar_wait(&a_full[ab], (it / NA) & 1);
         if (!ok) break;
+        const uint32_t k = jb % NB;
+        if (jb >= (uint32_t)NB) ok = mbar_wait(&acc_empty[k], ((jb / NB) - 1) & 1);
+        if (!ok) break;
+        fence_after_sync();
+        const uint32_t acc = tmem + k * C::kAcc;
         const uint32_t A0 = smem_u32(tiles + ab * C::kT);
-        for (int r = 0; r < a.nrel && ok; ++r, ++jb) {
-          const uint32_t k = jb % NB;
-          if (jb >= (uint32_t)NB) ok = mbar_wait(&acc_empty[k], ((jb / NB) - 1) & 1);
+        for (int kc = 0; kc < KC && ok; ++kc, ++g) {
+          const uint32_t s = g % S;
+          ok = mbar_wait(&b_full[s], (g / S) & 1);
           if (!ok) break;
           fence_after_sync();
-          const uint32_t acc = tmem + k * C::kAcc;
-          for (int kc = 0; kc < KC && ok; ++kc, ++g) {
-            const uint32_t s = g % S;
-            ok = mbar_wait(&b_full[s], (g / S) & 1);
-            if (!ok) break;
-            fence_after_sync();
-            const uint32_t A = A0 + kc * kATile;
-            const uint32_t B = smem_u32(bstage + s * C::kBStage);
+          const uint32_t A = A0 + kc * kATile;
+          const uint32_t B = smem_u32(bstage + s * C::kBStage);
 #pragma unroll
-            for (int ks = 0; ks < 4; ++ks) {
-              const uint64_t ad = desc_sw128(A + ks * 32, 16, 1024);
-              mma_bf16(acc, ad, desc_sw128(B + ks * 32, 16, 1024), idesc, (kc > 0 || ks > 0) ? 1u : 0u);
-              mma_bf16(acc, ad, desc_sw128(B + C::kB + ks * 32, 16, 1024), idesc, 1u);
-            }
-            mma_commit(&b_empty[s]);
+          for (int ks = 0; ks < 4; ++ks) {
+            const uint64_t ad = desc_sw128(A + ks * 32, 16, 1024);
+            mma_bf16(acc, ad, desc_sw128(B + ks * 32, 16, 1024), idesc, (kc > 0 || ks > 0) ? 1u : 0u);
+            mma_bf16(acc, ad, desc_sw128(B + C::kB + ks * 32, 16, 1024), idesc, 1u);
           }
-          mma_commit(&acc_full[k]);
+          mma_commit(&b_empty[s]);
         }
+        mma_commit(&acc_full[k]);
         mma_commit(&a_empty[ab]);
       }
       if (!ok) atomicOr(a.status, kErrTimeout);
     }
     __syncwarp();
-  } else {  // ---- epilogue: scale by 1 / deg_r and store dMs_r rows
+  } else {  // ---- epilogue: scale by 1 / deg_r and store the job's dMs rows
     const int q = warp & 3;
     const int row = q * 32 + lane;
     const uint32_t grp = (uint32_t)(warp - 2) / 4;  // this group takes jobs jb = grp mod kEpiGroups
-    const bool leader = (threadIdx.x & 127) == 0;   // issues the group's TMA stores
-    uint8_t* out = outs + grp * C::kOut;
-    auto group_sync = [&]() { asm volatile("bar.sync %0, 128;" ::"r"(1 + (int)grp) : "memory"); };
     bool ok = true;
     uint32_t jb = 0;
-    for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
-      const int64_t m = tile * kTileRows + row;
-      const bool live = m < a.n;
-      for (int r = 0; r < a.nrel && ok; ++r, ++jb) {
-        if (jb % C::kEpiGroups != grp) continue;
-        const uint32_t k = jb % NB;
-        const int64_t crow = a.mrow0[r] + (live ? m : 0);
-        const int deg = live && a.csr_ptr ? a.csr_ptr[crow + 1] - a.csr_ptr[crow] : 0;
-        const float sc = !a.csr_ptr ? 1.f : (deg > 0 ? __fdiv_rn(1.0f, (float)deg) : 0.f);
-        ok = mbar_wait(&acc_full[k], (jb / NB) & 1);
-        if (!ok) break;
-        fence_after_sync();
-        const uint32_t trow = tmem + k * C::kAcc + ((uint32_t)(q * 32) << 16);
-        if constexpr (C::kTmaOut) {
-          if (leader) bulk_wait_read();  // the group's previous tile has left the staging buffer
-          group_sync();
+    for (int64_t job = blockIdx.x; job < njobs && ok; job += gridDim.x, ++jb) {
+      if (jb % C::kEpiGroups != grp) continue;
+      const int j = J.rel_of(job);
+      const int64_t kr = (job - J.first[j]) * kTileRows + row;  // row within the relation's stored rows
+      const bool live = kr < J.count[j];
+      const int64_t crow = !live ? 0 : (a.mlist ? (int64_t)a.mlist[J.base[j] + kr] : a.mrow0[j] + kr);
+      const int64_t out = a.mlist ? J.base[j] + kr : crow;  // compact row, or CSR row
+      const int deg = live && a.csr_ptr ? a.csr_ptr[crow + 1] - a.csr_ptr[crow] : 0;
+      const float sc = !a.csr_ptr ? 1.f : (deg > 0 ? __fdiv_rn(1.0f, (float)deg) : 0.f);
+      const uint32_t k = jb % NB;
+      ok = mbar_wait(&acc_full[k], (jb / NB) & 1);
+      if (!ok) break;
+      fence_after_sync();
+      const uint32_t trow = tmem + k * C::kAcc + ((uint32_t)(q * 32) << 16);
 #pragma unroll
-          for (int c = 0; c < D; c += 32) {
-            float v[32];
-            tmem_ld32(trow + c, v);
+      for (int c = 0; c < D; c += 32) {
+        float v[32];
+        tmem_ld32(trow + c, v);
 #pragma unroll
-            for (int h = 0; h < 32; h += 8) {
-              float w8[8];
-#pragma unroll
-              for (int i = 0; i < 8; ++i) w8[i] = v[h + i] * sc;
-              const int cc = c + h;
-              st16(out + (cc >> 6) * kATile + sw128_offset(row, (uint32_t)(cc & 63) * 2), pack(w8, __nv_bfloat16()));
-            }
-          }
-          fence_before_sync();
-          mbar_arrive(&acc_empty[k]);
-          fence_async_smem();
-          group_sync();
-          if (leader) {
-            for (int kc = 0; kc < KC; ++kc) tma_store_2d(&tm_out.m[r], out + kc * kATile, kc * 64, (int)(tile * kTileRows));
-            bulk_commit();
-          }
-        } else {
-#pragma unroll
-          for (int c = 0; c < D; c += 32) {
-            float v[32];
-            tmem_ld32(trow + c, v);
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] *= sc;
-            if (live) {
-              store16_bf16(a.dMs + crow * D + c, v);
-              store16_bf16(a.dMs + crow * D + c + 16, v + 16);
-            }
-          }
-          fence_before_sync();
-          mbar_arrive(&acc_empty[k]);
+        for (int i = 0; i < 32; ++i) v[i] *= sc;
+        if (live) {
+          store16_bf16(a.dMs + out * D + c, v);
+          store16_bf16(a.dMs + out * D + c + 16, v + 16);
         }
       }
+      fence_before_sync();
+      mbar_arrive(&acc_empty[k]);
     }
-    if (C::kTmaOut && leader) bulk_wait();
     if (!ok) atomicOr(a.status, kErrTimeout);
   }
   fence_before_sync();
@@ -898,6 +922,126 @@ __global__ void __launch_bounds__(WgCfg<D>::kThreads, 1)
   if (warp == 0) tmem_dealloc(tmem, ncols);
 }
 
+// G_r = M_r^T dU over the stored (non-empty) rows of one relation r: row k of the relation's compact
+// range of M pairs with the dU row of its destination node.  Both operands are gathered by TMA
+// (one-row boxes, four rows per copy) as MN-major tiles of 64 rows; rows past the relation's count
+// read zeros.  Warp 0 writes each chunk's row coordinates and its lane 0 issues the copies, warp 1's
+// lane 0 the MMAs; the chunks are shared among the grid's splits by the count read on the device.
+// Grid (M tiles of 128 output rows, splits); part[split][D][D].
+template <int D>
+__global__ void __launch_bounds__(WgCfg<D>::kThreads, 1)
+    wgrad_rows_tc(const __grid_constant__ CUtensorMap tm_X, const __grid_constant__ CUtensorMap tm_Y, int S,
+                  const int32_t* __restrict__ mlist, const int32_t* __restrict__ mbase, int rel, int64_t row0,
+                  int64_t xsent, int64_t ysent, float* __restrict__ part, int* __restrict__ status) {
+  using C = WgCfg<D>;
+  constexpr int NB = D / 64;  // 64-wide column blocks of Y
+  constexpr int kStage = C::kA + NB * 8192;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  int32_t* sx = reinterpret_cast<int32_t*>(smem + S * kStage);  // [64] rows of M
+  int32_t* sy = sx + 64;                                        // [64] rows of dU
+  uint64_t* full = reinterpret_cast<uint64_t*>(sy + 64);
+  uint64_t* empty = full + S;
+  uint64_t* accb = empty + S;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(accb + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int mt = blockIdx.x;  // 128-wide block of X's columns (output rows)
+  const int64_t base = mbase[rel], count = (int64_t)mbase[rel + 1] - base;
+  const int64_t nchunks = (count + 63) / 64;
+  const int64_t cps = (nchunks + gridDim.y - 1) / gridDim.y;
+  const int64_t c0 = (int64_t)blockIdx.y * cps;
+  const int CT = (int)max((int64_t)0, min(nchunks, c0 + cps) - c0);
+  if (threadIdx.x == 0) {
+    for (int st = 0; st < S; ++st) {
+      mbar_init(&full[st], 1);
+      mbar_init(&empty[st], 1);
+    }
+    mbar_init(accb, 1);
+    fence_mbar_init();
+    prefetch_tmap(&tm_X);
+    prefetch_tmap(&tm_Y);
+  }
+  if (warp == 0) tmem_alloc(tslot, D);
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  const uint32_t tmem = *tslot;
+  if (warp == 0) {  // ---- producer
+    bool ok = true;
+    for (int g = 0; g < CT && ok; ++g) {
+      for (int t = lane; t < 64; t += 32) {
+        const int64_t k = (c0 + g) * 64 + t;
+        const bool in = k < count;
+        sx[t] = (int32_t)(in ? base + k : xsent);
+        sy[t] = (int32_t)(in ? (int64_t)mlist[base + k] - row0 : ysent);
+      }
+      __syncwarp();
+      if (lane == 0) {
+        const int st = g % S;
+        if (g >= S) ok = mbar_wait(&empty[st], ((g / S) - 1) & 1);
+        if (ok) {
+          uint8_t* stage = smem + st * kStage;
+          mbar_expect_tx(&full[st], kStage);
+          for (int b = 0; b < 2; ++b)
+#pragma unroll 4
+            for (int q = 0; q < 16; ++q)
+              tma_gather4(stage + b * 8192 + q * 512, &tm_X, mt * 128 + b * 64, sx[4 * q], sx[4 * q + 1], sx[4 * q + 2],
+                          sx[4 * q + 3], &full[st]);
+          for (int b = 0; b < NB; ++b)
+#pragma unroll 4
+            for (int q = 0; q < 16; ++q)
+              tma_gather4(stage + C::kA + b * 8192 + q * 512, &tm_Y, b * 64, sy[4 * q], sy[4 * q + 1], sy[4 * q + 2],
+                          sy[4 * q + 3], &full[st]);
+        }
+      }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      __syncwarp();  // the coordinates are rewritten for the next chunk
+    }
+    if (lane == 0 && !ok) atomicOr(status, kErrTimeout);
+  } else if (warp == 1 && lane == 0) {  // ---- MMA issuer
+    const uint32_t idesc = idesc_bf16(128, D, true, true);
+    bool ok = true;
+    for (int g = 0; g < CT && ok; ++g) {
+      const int st = g % S;
+      ok = mbar_wait(&full[st], (g / S) & 1);
+      if (!ok) break;
+      fence_after_sync();
+      const uint32_t A0 = smem_u32(smem + st * kStage);
+      const uint32_t B = A0 + C::kA;
+#pragma unroll
+      for (int ks = 0; ks < 4; ++ks)
+        mma_bf16(tmem, desc_sw128(A0 + ks * 2048, 8192, 1024), desc_sw128(B + ks * 2048, 8192, 1024), idesc,
+                 (g > 0 || ks > 0) ? 1u : 0u);
+      mma_commit(&empty[st]);
+    }
+    if (!ok) atomicOr(status, kErrTimeout);
+    mma_commit(accb);
+  }
+  __syncwarp();
+  if (!mbar_wait(accb, 0)) atomicOr(status, kErrTimeout);
+  fence_after_sync();
+  const int orow = mt * 128 + warp * 32 + lane;  // output row i (column of X)
+  float* out = part + (int64_t)blockIdx.y * D * D;
+#pragma unroll 1
+  for (int c = 0; c < D; c += 16) {
+    float v[16];
+    if (CT > 0) {
+      tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + c, v);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 16; ++i) v[i] = 0.f;
+    }
+    if (orow < D) {
+#pragma unroll
+      for (int i = 0; i < 16; i += 4)
+        *reinterpret_cast<float4*>(out + (int64_t)orow * D + c + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+    }
+  }
+  fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, D);
+}
+
 // ---------------------------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------------------------
@@ -908,6 +1052,7 @@ static hg_status smem_attr_once() {
     HG_CUDA(cudaFuncSetAttribute(proj_fwd_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, FwdCfg<D>::kSmem));
     HG_CUDA(cudaFuncSetAttribute(proj_bwd_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, BwdCfg<D>::kSmem));
     HG_CUDA(cudaFuncSetAttribute(wgrad_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, WgCfg<D>::kSmem));
+    HG_CUDA(cudaFuncSetAttribute(wgrad_rows_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, WgCfg<D>::kSmem));
     done = true;
   }
   return HG_OK;
@@ -928,7 +1073,7 @@ static hg_status tc_fwd_t(const TcFwdArgs& a, const void* M, int64_t m_rows, con
                           cudaStream_t s) {
   HG_TRY(smem_attr_once<D>());
   CUtensorMap tm_M, tm_V, tm_H;
-  HG_TRY(make_tmap_bf16(&tm_M, M, (uint64_t)std::max<int64_t>(m_rows, 1), D, kTileRows));
+  HG_TRY(make_tmap_bf16(&tm_M, M, (uint64_t)std::max<int64_t>(m_rows, 1), D, 1));  // one-row box: gathers
   HG_TRY(make_tmap_bf16(&tm_V, Vt, (uint64_t)2 * num_rels * D, D, D));
   if (FwdCfg<D>::kHTile) {
     HG_TRY(make_tmap_bf16(&tm_H, a.H_in + a.off * D, (uint64_t)a.n, D, kTileRows));
@@ -964,19 +1109,16 @@ static hg_status tc_bwd_t(const TcBwdArgs& a, const void* V, int num_rels, cudaS
   HG_TRY(smem_attr_once<D>());
   if (a.nrel == 0) return HG_OK;
   CUtensorMap tm_dU, tm_V;
-  HG_TRY(make_tmap_bf16(&tm_dU, a.dU + a.off * D, (uint64_t)a.n, D, kTileRows));
+  HG_TRY(make_tmap_bf16(&tm_dU, a.dU + a.off * D, (uint64_t)a.n, D, 1));  // one-row box: gathers
   HG_TRY(make_tmap_bf16(&tm_V, V, (uint64_t)2 * num_rels * D, D, D));
   int sms = 0, dev = 0;
   HG_CUDA(cudaGetDevice(&dev));
   HG_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
-  const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(a.n, kTileRows), sms));
-  RelMaps outs;
-  std::memset(&outs, 0, sizeof(outs));
-  if (BwdCfg<D>::kTmaOut)
-    for (int r = 0; r < a.nrel; ++r)
-      HG_TRY(make_tmap_bf16(&outs.m[r], a.dMs + a.mrow0[r] * D, (uint64_t)a.n, D, kTileRows));
+  // the jobs (128 stored rows of one relation) are counted on the device; at most this many
+  const int64_t cap = (int64_t)a.nrel * ceil_div(a.n, kTileRows);
+  const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(cap, sms));
   return launch("proj_bwd_tc", proj_bwd_tc<D>, dim3(grid), dim3(BwdCfg<D>::kThreads), BwdCfg<D>::kSmem, s, tm_dU,
-                tm_V, outs, a);
+                tm_V, a);
 }
 
 int wgrad_tc_splits(int64_t n, int d) {
@@ -1019,6 +1161,28 @@ static hg_status tc_wgrad_t(const void* X, const int64_t* x0, int R, const void*
 }
 
 template <int D>
+static hg_status tc_wgrad_rows_t(const void* M, int64_t m_rows, const int32_t* mlist, const int32_t* mbase, int rel,
+                                 int64_t row0, const void* dU, int64_t y0, int64_t n, float* part, float* out,
+                                 float* tmp, cudaStream_t s) {
+  HG_TRY(smem_attr_once<D>());
+  if (n == 0) {
+    HG_CUDA(cudaMemsetAsync(out, 0, (size_t)D * D * sizeof(float), s));
+    return HG_OK;
+  }
+  const int mtiles = D > 128 ? D / 128 : 1;
+  const int splits = wgrad_tc_splits(n, D);  // the stored rows (at most n) are split on the device
+  const int stage_bytes = WgCfg<D>::kA + (D / 64) * 8192;
+  const int stages = std::min(4, (WgCfg<D>::kSmem - 1024 - 256 - 512) / stage_bytes);
+  CUtensorMap tm_X, tm_Y;
+  HG_TRY(make_tmap_bf16(&tm_X, M, (uint64_t)std::max<int64_t>(m_rows, 1), D, 1));
+  HG_TRY(make_tmap_bf16(&tm_Y, (const __nv_bfloat16*)dU + y0 * D, (uint64_t)n, D, 1));
+  HG_TRY(launch("wgrad_tc", wgrad_rows_tc<D>, dim3(mtiles, splits), dim3(WgCfg<D>::kThreads),
+                (size_t)stages * stage_bytes + 512 + 256 + 1024, s, tm_X, tm_Y, stages, mlist, mbase, rel, row0,
+                m_rows, n, part, device_status_ptr()));
+  return reduce_partials(part, (int64_t)D * D, splits, (int64_t)D * D, out, tmp, s);
+}
+
+template <int D>
 static hg_status tc_finish_t(const float* G, const void* W_rel, const void* W_agg, RelDst rd, int num_rels,
                              int num_types, float* dW_rel, float* dW_agg, cudaStream_t s) {
   return launch("wgrad_finish", wgrad_finish<D>, dim3(D / 32, D / 32, num_rels + num_types), dim3(256),
@@ -1052,6 +1216,11 @@ hg_status tc_proj_backward(int d, const TcBwdArgs& a, const void* V, int num_rel
 hg_status tc_weight_grad(int d, const void* X, const int64_t* x0, int R, const void* Y, int64_t y0, int64_t n,
                          float* part, float* const* outs, float* tmp, cudaStream_t s) {
   HG_TC_DISPATCH(d, tc_wgrad_t, X, x0, R, Y, y0, n, part, outs, tmp, s);
+}
+hg_status tc_weight_grad_rows(int d, const void* M, int64_t m_rows, const int32_t* mlist, const int32_t* mbase, int rel,
+                              int64_t row0, const void* dU, int64_t y0, int64_t n, float* part, float* out, float* tmp,
+                              cudaStream_t s) {
+  HG_TC_DISPATCH(d, tc_wgrad_rows_t, M, m_rows, mlist, mbase, rel, row0, dU, y0, n, part, out, tmp, s);
 }
 int wgrad_tc_max_rels(int d) { return d == 64 ? WgCfg<64>::kMaxR : (d == 128 ? WgCfg<128>::kMaxR : WgCfg<256>::kMaxR); }
 hg_status tc_wgrad_finish(int d, const float* G, const void* W_rel, const void* W_agg, RelDst rd, int num_rels,

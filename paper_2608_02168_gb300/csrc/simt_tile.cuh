@@ -38,17 +38,19 @@ struct Tile {
   static constexpr int kVec = VecTraits<T>::kElems;
 };
 
-// Stage A[m][k0 .. k0+KC) for rows a_row0 + m (m < kBM, zero past n_valid) into As (fp32).
+// Stage A[m][k0 .. k0+KC) for rows a_row0 + m (m < kBM, zero past n_valid) into As (fp32).  With
+// a row map, row a_row0 + m of A is A[map[a_row0 + m]], and a mapped index >= sentinel is a zero row.
 template <typename T, int D>
 __device__ __forceinline__ void stage_a(float (*As)[kAPad], const T* __restrict__ A, int64_t a_row0, int64_t n_valid,
-                                        int k0) {
+                                        int k0, const int32_t* __restrict__ map = nullptr, int64_t sentinel = 0) {
   constexpr int VEC = VecTraits<T>::kElems;
   constexpr int PER_ROW = kKC / VEC;
   for (int idx = threadIdx.x; idx < kBM * PER_ROW; idx += blockDim.x) {
     const int m = idx / PER_ROW, kv = idx % PER_ROW;
     float f[VEC];
-    if (m < n_valid) {
-      unpack(ldg16(A + (a_row0 + m) * D + k0 + kv * VEC), f, T());
+    const int64_t row = m < n_valid ? (map ? (int64_t)map[a_row0 + m] : a_row0 + m) : 0;
+    if (m < n_valid && (!map || row < sentinel)) {
+      unpack(ldg16(A + row * D + k0 + kv * VEC), f, T());
     } else {
 #pragma unroll
       for (int q = 0; q < VEC; ++q) f[q] = 0.f;

@@ -69,6 +69,19 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
       ::"r"(smem_u32(dst)), "l"(map), "r"(x), "r"(y), "r"(smem_u32(bar))
       : "memory");
 }
+// Four rows r0..r3 of 64 columns from column x (x a multiple of 64 elements here) of a 2-D tensor
+// map whose box is one row high, written one after another (512 B for bf16) at dst; a row index at
+// or past the map's row extent reads zeros.  The 128-byte swizzle follows the destination address,
+// as for a tile load, so rows gathered into consecutive 128-byte slots of a 1024-byte-aligned tile
+// form the same operand layout.  Completion counted in bytes on `bar`.
+__device__ __forceinline__ void tma_gather4(void* dst, const CUtensorMap* map, int x, int r0, int r1, int r2, int r3,
+                                            uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
+      "%4, %5, %6}], [%7];" ::"r"(smem_u32(dst)),
+      "l"(map), "r"(x), "r"(r0), "r"(r1), "r"(r2), "r"(r3), "r"(smem_u32(bar))
+      : "memory");
+}
 // 2-D tiled store of a shared-memory box to global memory (bulk async-group completion); rows
 // and columns outside the tensor map's extent are not written.
 __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int x, int y) {

@@ -77,7 +77,11 @@ def test_aggregation_models_are_compulsory_bytes():
     m = bench.kernel_models(st, sp)
     row, L, f = sp.d * 2, sp.layers, st["fwd"]
     assert m["agg_fwd_chunks"][0] == L * (8 * f["R_h"] + row * f["U_h"] + 4 * sp.d * f["chunks"])
-    assert m["agg_fwd_rows"][0] == L * (8 * (st["RR"] + 1) + 8 * f["R_nh"] + row * f["U_nh"] + row * st["RR"] +
+    # the forward rows write only the stored (non-empty) relation rows
+    assert 0 < st["NNZ"] < st["RR"]
+    assert st["NNZ"] == sum(int(np.count_nonzero(np.bincount(w.graph["dst"][w.graph["rel"] == r], minlength=sp.num_nodes)))
+                            for r in range(sp.num_rels))
+    assert m["agg_fwd_rows"][0] == L * (12 * st["NNZ"] + 8 * f["R_nh"] + row * f["U_nh"] + row * st["NNZ"] +
                                         4 * sp.d * f["chunks"])
     # one gathered row and run entry per run, over both kernels of a direction
     runs_f = st["fwd"]["R_h"] + st["fwd"]["R_nh"]
