@@ -60,6 +60,9 @@ def parse():
     ap.add_argument("--no-temporal", action="store_true", help="skip the temporal-module measurement")
     ap.add_argument("--no-hgt", action="store_true", help="skip the attention-layer measurement")
     ap.add_argument("--scale", type=int, default=1, help=argparse.SUPPRESS)  # profiling: a 1/k-size instance
+    ap.add_argument("--ncu-traffic", default="",
+                    help="fold an ncu CSV (--metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum "
+                         "--csv) into profiles/traffic.json, each kernel stamped with its source hash, and exit")
     ap.add_argument("--oracle-child", default="", help=argparse.SUPPRESS)  # internal: child process kind
     ap.add_argument("--oracle-k", type=int, default=1, help=argparse.SUPPRESS)
     ap.add_argument("--oracle-steps", type=int, default=1, help=argparse.SUPPRESS)
@@ -378,24 +381,85 @@ def load_peaks() -> tuple:
     return dict(FALLBACK), "fallback"
 
 
+# kernels the library times under another name than their function's
+KERNEL_ALIASES = {"agg_fwd_chunks": "agg_chunks", "agg_bwd_chunks": "agg_chunks"}
+
+
+def _source_hash(source: str) -> str:
+    import glob
+    import hashlib
+    csrc = os.path.join(ROOT, "paper_2608_02168_gb300", "csrc")
+    h = hashlib.sha256()
+    for f in [os.path.join(csrc, source)] + sorted(glob.glob(os.path.join(csrc, "*.cuh"))):
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def _kernel_source(fn: str) -> str | None:
+    """The .cu file of paper_2608_02168_gb300/csrc that defines kernel `fn`."""
+    import glob
+    import re
+    pat = re.compile(r"__global__[^;{]*?\b" + re.escape(fn) + r"\s*\(", re.S)
+    for f in sorted(glob.glob(os.path.join(ROOT, "paper_2608_02168_gb300", "csrc", "*.cu"))):
+        with open(f) as fh:
+            if pat.search(fh.read()):
+                return os.path.basename(f)
+    return None
+
+
+def fold_ncu_traffic(csv_path: str, out_path: str) -> dict:
+    """DRAM bytes per launch of every kernel in an ncu metrics CSV (one row per launch and metric),
+    keyed by kernel function name, with the launch count and the SHA-256 of the kernel's source file
+    and the shared headers (measured_traffic uses an entry only while that hash still matches)."""
+    import csv
+    import re
+    acc = {}
+    with open(csv_path, newline="") as fh:
+        lines = [ln for ln in fh if ln.startswith('"')]
+    for row in csv.DictReader(lines):
+        name = row.get("Kernel Name", "")
+        m = re.match(r"(?:void\s+)?(?:[\w:]*::)?(\w+)", name.replace("hg::", ""))
+        if not m:
+            continue
+        fn = m.group(1)
+        e = acc.setdefault(fn, {"ids": set(), "read": 0.0, "write": 0.0, "ns": 0.0})
+        e["ids"].add(row["ID"])
+        v = float(row["Metric Value"].replace(",", ""))
+        unit = row.get("Metric Unit", "")
+        scale = {"byte": 1, "Kbyte": 1e3, "Mbyte": 1e6, "Gbyte": 1e9, "nsecond": 1, "usecond": 1e3, "msecond": 1e6}
+        v *= scale.get(unit, 1)
+        metric = row["Metric Name"]
+        if metric == "dram__bytes_read.sum":
+            e["read"] += v
+        elif metric == "dram__bytes_write.sum":
+            e["write"] += v
+        elif metric == "gpu__time_duration.sum":
+            e["ns"] += v
+    out = {}
+    for fn, e in sorted(acc.items()):
+        src = _kernel_source(fn)
+        if src is None or not (e["read"] or e["write"]):
+            continue
+        n = len(e["ids"])
+        out[fn] = {"launches": n, "bytes_per_launch": int(round((e["read"] + e["write"]) / n)),
+                   "ns_per_launch": int(round(e["ns"] / n)), "source": src, "sha256": _source_hash(src)}
+    with open(out_path, "w") as fh:
+        json.dump(out, fh, indent=1, sort_keys=True)
+    return out
+
+
 def measured_traffic(kernel: str):
     """DRAM bytes per launch of `kernel` from the committed ncu capture (profiles/traffic.json), or
     None when there is none or the kernel's sources changed since it was taken."""
-    import glob
-    import hashlib
     p = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(p):
         return None
     with open(p) as fh:
-        entry = json.load(fh).get(kernel)
+        entry = json.load(fh).get(KERNEL_ALIASES.get(kernel, kernel))
     if not entry:
         return None
-    csrc = os.path.join(ROOT, "paper_2608_02168_gb300", "csrc")
-    h = hashlib.sha256()
-    for f in [os.path.join(csrc, entry["source"])] + sorted(glob.glob(os.path.join(csrc, "*.cuh"))):
-        with open(f, "rb") as fh:
-            h.update(fh.read())
-    return int(entry["bytes_per_launch"]) if h.hexdigest() == entry["sha256"] else None
+    return int(entry["bytes_per_launch"]) if _source_hash(entry["source"]) == entry["sha256"] else None
 
 
 def roofline(report: dict, models: dict, steps: int, peaks: dict, src: str, dom=None) -> tuple:
@@ -848,6 +912,10 @@ def measure_ring(sp, dev, warmup: int) -> dict:
 # ------------------------------------------------------------------------------------------------
 def main():
     args = parse()
+    if args.ncu_traffic:
+        out = fold_ncu_traffic(args.ncu_traffic, os.path.join(ROOT, "profiles", "traffic.json"))
+        print(json.dumps({k: v["bytes_per_launch"] for k, v in out.items()}))
+        return
     if args.oracle_child:
         oracle_child_main(args.oracle_child, args.workload, args.oracle_k, args.oracle_steps, args.oracle_warmup,
                           not args.no_head)

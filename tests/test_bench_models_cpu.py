@@ -116,3 +116,24 @@ def test_roofline_arithmetic():
     assert rs["bound"] == "alu" and rs["unit"] == "TFLOP/s"
     assert abs(rs["peak"] - 152 * 128 * 2 * 2000e6 / 1e12) < 0.1
     assert abs(rs["achieved"] - 4e10 * 5 / 1e-3 / 1e12) < 1e-3
+
+
+def test_ncu_traffic_folding(tmp_path):
+    """ncu's per-launch CSV folds into bytes per launch per kernel function, stamped with the source
+    hash that measured_traffic checks."""
+    head = ('"ID","Process ID","Process Name","Host Name","Kernel Name","Context","Stream","Block Size","Grid Size",'
+            '"Device","CC","Section Name","Metric Name","Metric Unit","Metric Value"\n')
+    rows = []
+    for i, (read, write) in enumerate([(100, 50), (300, 150)]):
+        k = f'"{i}","1","py","h","void hg::agg_chunks<__nv_bfloat16, 128>(const int *, int *)","1","7","(256, 1, 1)","(1, 1, 1)","0","10.3","m"'
+        rows += [k + f',"dram__bytes_read.sum","byte","{read}"\n', k + f',"dram__bytes_write.sum","Kbyte","{write / 1000}"\n',
+                 k + ',"gpu__time_duration.sum","usecond","2.5"\n']
+    k = '"2","1","py","h","edge_keys(const int *, const int *)","1","7","(256, 1, 1)","(1, 1, 1)","0","10.3","m"'
+    rows += [k + ',"dram__bytes_read.sum","Mbyte","1.5"\n', k + ',"dram__bytes_write.sum","byte","500"\n']
+    csv_path = tmp_path / "t.csv"
+    csv_path.write_text("==PROF== noise\n" + head + "".join(rows))
+    out = bench.fold_ncu_traffic(str(csv_path), str(tmp_path / "traffic.json"))
+    assert out["agg_chunks"]["launches"] == 2 and out["agg_chunks"]["bytes_per_launch"] == 300
+    assert out["agg_chunks"]["ns_per_launch"] == 2500 and out["agg_chunks"]["source"] == "agg.cu"
+    assert out["edge_keys"]["bytes_per_launch"] == 1_500_500 and out["edge_keys"]["source"] == "graph.cu"
+    assert out["agg_chunks"]["sha256"] == bench._source_hash("agg.cu")
