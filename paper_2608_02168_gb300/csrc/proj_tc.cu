@@ -101,8 +101,7 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
   uint8_t* stage = smem;                  // S x (A | B)
   uint8_t* htile = smem + S * C::kStage;  // 2 x KC x 16 KB, 128B-swizzled rows
   float* params = reinterpret_cast<float*>(htile + 2 * C::kH);  // [3][D]: b, gamma, beta
-  int32_t* sidx = reinterpret_cast<int32_t*>(params + 3 * D);    // [128] rows of M gathered into A
-  uint64_t* full = reinterpret_cast<uint64_t*>(sidx + kTileRows);
+  uint64_t* full = reinterpret_cast<uint64_t*>(params + 3 * D + kTileRows);  // (a 512-byte gap before the barriers)
   uint64_t* empty = full + S;
   uint64_t* acc_full = empty + S;   // [2] MMA -> epilogue
   uint64_t* acc_empty = acc_full + 2;  // [2] epilogue -> MMA
@@ -136,12 +135,22 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
   const uint32_t tmem = *tslot;
 
   if (warp == 0) {
-    // ---- TMA producer (the warp writes each relation tile's row coordinates, lane 0 issues):
-    // A rows by gather (four rows per copy), a row past the type or an empty relation row at or past
-    // the map's extent reads zeros; V_r^T hi / lo chunks and the residual tile by tile loads
+    // ---- TMA producer: lane q gathers A rows 4q .. 4q + 3 of every chunk (four rows per copy; a row
+    // past the type or an empty relation row, at or past the map's extent, reads zeros), its row
+    // indices loaded one relation ahead; lane 0 posts each stage's byte count first and loads the
+    // V_r^T hi / lo chunks and the residual tile
     bool ok = true;
     uint32_t g = 0;
     int it = 0;
+    auto rows_of = [&](int64_t m0, int r, int* c) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int64_t m = m0 + 4 * lane + i;
+        int64_t v = a.msent;
+        if (r < a.nrel && m < a.n) v = a.mrow ? (int64_t)__ldg(a.mrow + a.mrow0[r] + m) : a.mrow0[r] + m;
+        c[i] = (int)v;
+      }
+    };
     for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
       const int64_t m0 = tile * kTileRows;
       const int b = it & 1;
@@ -154,31 +163,26 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
         }
       }
       ok = __shfl_sync(0xffffffffu, ok, 0);
+      int c[4], cn[4];
+      rows_of(m0, 0, c);
       for (int r = 0; r < a.nrel && ok; ++r) {
-        for (int i = lane; i < kTileRows; i += 32) {
-          const int64_t m = m0 + i;
-          int64_t c = a.msent;
-          if (m < a.n) c = a.mrow ? (int64_t)a.mrow[a.mrow0[r] + m] : a.mrow0[r] + m;
-          sidx[i] = (int32_t)c;
-        }
-        __syncwarp();
-        if (lane == 0) {
-          for (int kc = 0; kc < KC && ok; ++kc, ++g) {
-            const uint32_t s = g % S;
+        rows_of(m0, r + 1, cn);  // the next relation's rows, in flight while these are issued
+        for (int kc = 0; kc < KC && ok; ++kc, ++g) {
+          const uint32_t s = g % S;
+          uint8_t* A = stage + s * C::kStage;
+          if (lane == 0) {
             if (g >= (uint32_t)S) ok = mbar_wait(&empty[s], ((g / S) - 1) & 1);
-            if (!ok) break;
-            uint8_t* A = stage + s * C::kStage;
-            mbar_expect_tx(&full[s], C::kStage);
-#pragma unroll 4
-            for (int q = 0; q < kTileRows / 4; ++q)
-              tma_gather4(A + q * 512, &tm_M, kc * 64, sidx[4 * q], sidx[4 * q + 1], sidx[4 * q + 2], sidx[4 * q + 3],
-                          &full[s]);
-            tma_load_2d(A + kATile, &tm_Vt, kc * 64, 2 * a.rel[r] * D, &full[s]);           // hi
-            tma_load_2d(A + kATile + C::kB, &tm_Vt, kc * 64, (2 * a.rel[r] + 1) * D, &full[s]);  // lo
+            if (ok) {
+              mbar_expect_tx(&full[s], C::kStage);
+              tma_load_2d(A + kATile, &tm_Vt, kc * 64, 2 * a.rel[r] * D, &full[s]);           // hi
+              tma_load_2d(A + kATile + C::kB, &tm_Vt, kc * 64, (2 * a.rel[r] + 1) * D, &full[s]);  // lo
+            }
           }
+          ok = __shfl_sync(0xffffffffu, ok, 0);
+          if (ok) tma_gather4(A + lane * 512, &tm_M, kc * 64, c[0], c[1], c[2], c[3], &full[s]);
         }
-        ok = __shfl_sync(0xffffffffu, ok, 0);
-        __syncwarp();  // the coordinates are rewritten for the next relation
+#pragma unroll
+        for (int i = 0; i < 4; ++i) c[i] = cn[i];
       }
     }
     if (lane == 0 && !ok) atomicOr(a.status, kErrTimeout);
@@ -648,8 +652,7 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
   uint8_t* smem = align1024(smem_raw);
   uint8_t* bstage = smem;                  // S x (B_hi | B_lo) chunk
   uint8_t* tiles = smem + S * C::kBStage;  // NA x (KC x 16 KB)
-  int32_t* sidx = reinterpret_cast<int32_t*>(tiles + NA * C::kT);  // [128] gathered dU rows
-  uint64_t* b_full = reinterpret_cast<uint64_t*>(sidx + kTileRows);
+  uint64_t* b_full = reinterpret_cast<uint64_t*>(tiles + NA * C::kT + C::kIdx);
   uint64_t* b_empty = b_full + S;
   uint64_t* a_full = b_empty + S;       // [NA] dU tile gathered
   uint64_t* a_empty = a_full + 2;       // [NA] the job's products done
@@ -684,32 +687,33 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
   const uint32_t tmem = *tslot;
   const int64_t njobs = J.first[J.nrel];
 
-  if (warp == 0) {  // ---- producer: the warp writes the job's dU rows, lane 0 issues the copies
+  if (warp == 0) {  // ---- producer: lane q gathers the job's dU rows 4q .. 4q + 3, lane 0 streams V_r
     bool ok = true;
     uint32_t g = 0;
     int it = 0;
     for (int64_t job = blockIdx.x; job < njobs && ok; job += gridDim.x, ++it) {
       const int j = J.rel_of(job);
       const int64_t i0 = (job - J.first[j]) * kTileRows;  // first row of the job within the relation
-      for (int t = lane; t < kTileRows; t += 32) {
-        const int64_t k = i0 + t;
+      int c[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int64_t k = i0 + 4 * lane + i;
         int64_t local = a.n;  // past the relation's rows: zeros
-        if (k < J.count[j]) local = a.mlist ? (int64_t)a.mlist[J.base[j] + k] - a.mrow0[j] : k;
-        sidx[t] = (int32_t)local;
+        if (k < J.count[j]) local = a.mlist ? (int64_t)__ldg(a.mlist + J.base[j] + k) - a.mrow0[j] : k;
+        c[i] = (int)local;
       }
-      __syncwarp();
+      const int ab = it % NA;
       if (lane == 0) {
-        const int ab = it % NA;
         if (it >= NA) ok = mbar_wait(&a_empty[ab], ((it / NA) - 1) & 1);
-        if (ok) {
-          mbar_expect_tx(&a_full[ab], C::kT);
-          uint8_t* A = tiles + ab * C::kT;
-          for (int kc = 0; kc < KC; ++kc)
-#pragma unroll 4
-            for (int q = 0; q < kTileRows / 4; ++q)
-              tma_gather4(A + kc * kATile + q * 512, &tm_dU, kc * 64, sidx[4 * q], sidx[4 * q + 1], sidx[4 * q + 2],
-                          sidx[4 * q + 3], &a_full[ab]);
-        }
+        if (ok) mbar_expect_tx(&a_full[ab], C::kT);
+      }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (ok) {
+        uint8_t* A = tiles + ab * C::kT;
+        for (int kc = 0; kc < KC; ++kc)
+          tma_gather4(A + kc * kATile + lane * 512, &tm_dU, kc * 64, c[0], c[1], c[2], c[3], &a_full[ab]);
+      }
+      if (lane == 0) {
         for (int kc = 0; kc < KC && ok; ++kc, ++g) {
           const uint32_t s = g % S;
           if (g >= (uint32_t)S) ok = mbar_wait(&b_empty[s], ((g / S) - 1) & 1);
@@ -720,7 +724,6 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
         }
       }
       ok = __shfl_sync(0xffffffffu, ok, 0);
-      __syncwarp();  // the row list is rewritten for the next job
     }
     if (lane == 0 && !ok) atomicOr(a.status, kErrTimeout);
     __syncwarp();
@@ -938,9 +941,7 @@ __global__ void __launch_bounds__(WgCfg<D>::kThreads, 1)
   constexpr int kStage = C::kA + NB * 8192;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  int32_t* sx = reinterpret_cast<int32_t*>(smem + S * kStage);  // [64] rows of M
-  int32_t* sy = sx + 64;                                        // [64] rows of dU
-  uint64_t* full = reinterpret_cast<uint64_t*>(sy + 64);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S * kStage);
   uint64_t* empty = full + S;
   uint64_t* accb = empty + S;
   uint32_t* tslot = reinterpret_cast<uint32_t*>(accb + 1);
@@ -966,36 +967,40 @@ __global__ void __launch_bounds__(WgCfg<D>::kThreads, 1)
   __syncthreads();
   fence_after_sync();
   const uint32_t tmem = *tslot;
-  if (warp == 0) {  // ---- producer
+  if (warp == 0) {  // ---- producer: lanes 0-15 gather X rows 4q .. 4q + 3, lanes 16-31 the same rows of Y
     bool ok = true;
-    for (int g = 0; g < CT && ok; ++g) {
-      for (int t = lane; t < 64; t += 32) {
-        const int64_t k = (c0 + g) * 64 + t;
-        const bool in = k < count;
-        sx[t] = (int32_t)(in ? base + k : xsent);
-        sy[t] = (int32_t)(in ? (int64_t)mlist[base + k] - row0 : ysent);
+    const int q = lane & 15;
+    const bool isx = lane < 16;
+    auto coords = [&](int g, int* c) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int64_t k = (c0 + g) * 64 + 4 * q + i;
+        const bool in = g < CT && k < count;
+        c[i] = (int)(isx ? (in ? base + k : xsent) : (in ? (int64_t)__ldg(mlist + base + k) - row0 : ysent));
       }
-      __syncwarp();
+    };
+    int c[4], cn[4];
+    coords(0, c);
+    for (int g = 0; g < CT && ok; ++g) {
+      coords(g + 1, cn);  // the next chunk's rows, in flight while these are issued
+      const int st = g % S;
+      uint8_t* stage = smem + st * kStage;
       if (lane == 0) {
-        const int st = g % S;
         if (g >= S) ok = mbar_wait(&empty[st], ((g / S) - 1) & 1);
-        if (ok) {
-          uint8_t* stage = smem + st * kStage;
-          mbar_expect_tx(&full[st], kStage);
-          for (int b = 0; b < 2; ++b)
-#pragma unroll 4
-            for (int q = 0; q < 16; ++q)
-              tma_gather4(stage + b * 8192 + q * 512, &tm_X, mt * 128 + b * 64, sx[4 * q], sx[4 * q + 1], sx[4 * q + 2],
-                          sx[4 * q + 3], &full[st]);
-          for (int b = 0; b < NB; ++b)
-#pragma unroll 4
-            for (int q = 0; q < 16; ++q)
-              tma_gather4(stage + C::kA + b * 8192 + q * 512, &tm_Y, b * 64, sy[4 * q], sy[4 * q + 1], sy[4 * q + 2],
-                          sy[4 * q + 3], &full[st]);
-        }
+        if (ok) mbar_expect_tx(&full[st], kStage);
       }
       ok = __shfl_sync(0xffffffffu, ok, 0);
-      __syncwarp();  // the coordinates are rewritten for the next chunk
+      if (ok) {
+        if (isx) {
+          for (int b = 0; b < 2; ++b)
+            tma_gather4(stage + b * 8192 + q * 512, &tm_X, mt * 128 + b * 64, c[0], c[1], c[2], c[3], &full[st]);
+        } else {
+          for (int b = 0; b < NB; ++b)
+            tma_gather4(stage + C::kA + b * 8192 + q * 512, &tm_Y, b * 64, c[0], c[1], c[2], c[3], &full[st]);
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) c[i] = cn[i];
     }
     if (lane == 0 && !ok) atomicOr(status, kErrTimeout);
   } else if (warp == 1 && lane == 0) {  // ---- MMA issuer
@@ -1172,12 +1177,12 @@ static hg_status tc_wgrad_rows_t(const void* M, int64_t m_rows, const int32_t* m
   const int mtiles = D > 128 ? D / 128 : 1;
   const int splits = wgrad_tc_splits(n, D);  // the stored rows (at most n) are split on the device
   const int stage_bytes = WgCfg<D>::kA + (D / 64) * 8192;
-  const int stages = std::min(4, (WgCfg<D>::kSmem - 1024 - 256 - 512) / stage_bytes);
+  const int stages = std::min(4, (WgCfg<D>::kSmem - 1024 - 256) / stage_bytes);
   CUtensorMap tm_X, tm_Y;
   HG_TRY(make_tmap_bf16(&tm_X, M, (uint64_t)std::max<int64_t>(m_rows, 1), D, 1));
   HG_TRY(make_tmap_bf16(&tm_Y, (const __nv_bfloat16*)dU + y0 * D, (uint64_t)n, D, 1));
   HG_TRY(launch("wgrad_tc", wgrad_rows_tc<D>, dim3(mtiles, splits), dim3(WgCfg<D>::kThreads),
-                (size_t)stages * stage_bytes + 512 + 256 + 1024, s, tm_X, tm_Y, stages, mlist, mbase, rel, row0,
+                (size_t)stages * stage_bytes + 256 + 1024, s, tm_X, tm_Y, stages, mlist, mbase, rel, row0,
                 m_rows, n, part, device_status_ptr()));
   return reduce_partials(part, (int64_t)D * D, splits, (int64_t)D * D, out, tmp, s);
 }
