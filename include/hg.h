@@ -141,6 +141,22 @@ typedef struct {
 } hg_graph_arrays;
 hg_status hg_graph_view(const hg_graph* graph, int32_t rel, hg_graph_arrays* out);
 
+/* The order in which the bf16 forward projection (hg_layer_fwd) visits the destination nodes of one
+ * type, built by hg_build_csr.  The relation mask of a node has bit k set when the k-th relation
+ * into the type (relations by ascending id) has an in-edge at the node (M_r of Eq. 10 non-zero).
+ * perm[i] (n entries) is the local id of the node at position i: the type's nodes sorted stably by
+ * their mask.  tile_mask[q] (tiles = ceil(n / tile_rows) entries) is the OR of the masks at positions
+ * tile_rows q .. tile_rows q + tile_rows - 1: the relations whose products a tile computes.  Device
+ * arrays inside the graph's workspace (read only; for tests).  HG_ERR_INVALID for a type out of
+ * range. */
+typedef struct {
+  int64_t n, tiles;
+  int32_t tile_rows;
+  const int32_t* perm;
+  const int32_t* tile_mask;
+} hg_node_order;
+hg_status hg_graph_node_order(const hg_graph* graph, int32_t type, hg_node_order* out);
+
 /* ------------------------------------------------------------------------------------------- */
 /* Layer (Eq. 7, Eq. 10 with mean aggregation, Eq. 11, optional LayerNorm)                      */
 /* ------------------------------------------------------------------------------------------- */

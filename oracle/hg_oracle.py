@@ -123,6 +123,28 @@ def build_csr(src, dst, rel, type_offsets, rels) -> list:
     return out
 
 
+def node_order(csr: list, type_offsets, rels, node_type: int, tile_rows: int = 128) -> tuple:
+    """The order in which the tensor-core forward projection visits the nodes of one type (a layout
+    of the kernels, not of the paper): the relation mask of local node j has bit k set when the k-th
+    relation into the type (ascending relation id) has an in-edge at j; perm lists the local ids by
+    ascending (mask, id); tile_mask[q] is the OR of the masks at positions tile_rows q onwards."""
+    offs = np.asarray(type_offsets, np.int64)
+    n = int(offs[node_type + 1] - offs[node_type])
+    mask = np.zeros(n, np.int64)
+    k = 0
+    for r, (_, tt) in enumerate(rels):
+        if tt != node_type:
+            continue
+        mask |= (csr[r]["deg"] > 0).astype(np.int64) << k
+        k += 1
+    perm = np.argsort(mask, kind="stable")
+    tiles = -(-n // tile_rows)
+    tile_mask = np.zeros(tiles, np.int64)
+    for q in range(tiles):
+        tile_mask[q] = np.bitwise_or.reduce(mask[perm[q * tile_rows:(q + 1) * tile_rows]])
+    return perm, tile_mask
+
+
 # ----------------------------------------------------------------------------------------------
 # layer
 # ----------------------------------------------------------------------------------------------

@@ -543,6 +543,98 @@ __global__ void chunk_fill(const int32_t* __restrict__ ofs, int64_t rows, int32_
   }
 }
 
+// ---- node order of the forward projection: a stable counting sort of each type's nodes by relation
+// mask (at most kMaxRels relations into a type: 2^8 mask values).  Blocks own kOrderTile nodes.
+constexpr int kOrderTile = 2048;
+constexpr int kMaskValues = 1 << kMaxRels;
+
+struct TypeRels {
+  int n;                     // relations into the type
+  int64_t row0[kMaxRels];    // CSR row of the type's local node 0 in each, by ascending relation id
+};
+
+__device__ __forceinline__ uint32_t node_mask(const int32_t* __restrict__ csr_ptr, const TypeRels& tr, int64_t j) {
+  uint32_t m = 0;
+  for (int k = 0; k < tr.n; ++k) {
+    const int64_t row = tr.row0[k] + j;
+    if (__ldg(csr_ptr + row + 1) > __ldg(csr_ptr + row)) m |= 1u << k;
+  }
+  return m;
+}
+
+// hist[v * nblk + block] = nodes of the block with mask v
+__global__ void __launch_bounds__(256) order_hist(const int32_t* __restrict__ csr_ptr, TypeRels tr, int64_t n,
+                                                  int nblk, int32_t* __restrict__ hist) {
+  __shared__ int32_t h[kMaskValues];
+  const int V = 1 << tr.n;
+  for (int v = threadIdx.x; v < V; v += blockDim.x) h[v] = 0;
+  __syncthreads();
+  const int64_t j0 = (int64_t)blockIdx.x * kOrderTile;
+  for (int k = threadIdx.x; k < kOrderTile; k += blockDim.x) {
+    const int64_t j = j0 + k;
+    if (j < n) atomicAdd(&h[node_mask(csr_ptr, tr, j)], 1);
+  }
+  __syncthreads();
+  for (int v = threadIdx.x; v < V; v += blockDim.x) hist[(int64_t)v * nblk + blockIdx.x] = h[v];
+}
+
+// perm[ofs[v * nblk + block] + rank] = j, rank = the node's place among the block's nodes with mask v
+// in ascending id (rounds of 256 nodes; within a round, warp-level ranks plus earlier warps' counts)
+__global__ void __launch_bounds__(256) order_scatter(const int32_t* __restrict__ csr_ptr, TypeRels tr, int64_t n,
+                                                     int nblk, const int32_t* __restrict__ ofs,
+                                                     int32_t* __restrict__ perm) {
+  __shared__ int32_t next[kMaskValues];
+  __shared__ int32_t wcnt[8][kMaskValues];
+  const int V = 1 << tr.n;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int v = threadIdx.x; v < V; v += 256) next[v] = ofs[(int64_t)v * nblk + blockIdx.x];
+  const int64_t j0 = (int64_t)blockIdx.x * kOrderTile;
+  for (int k = 0; k < kOrderTile; k += 256) {
+    for (int i = threadIdx.x; i < 8 * V; i += 256) wcnt[i / V][i % V] = 0;
+    __syncthreads();
+    const int64_t j = j0 + k + threadIdx.x;
+    const bool live = j < n;
+    const uint32_t mk = live ? node_mask(csr_ptr, tr, j) : 0xFFFFFFFFu;
+    const uint32_t peers = __match_any_sync(0xffffffffu, mk);
+    const int lrank = __popc(peers & ((1u << lane) - 1u));
+    if (live && lrank == 0) wcnt[warp][mk] = __popc(peers);
+    __syncthreads();
+    if (live) {
+      int pos = next[mk] + lrank;
+      for (int w = 0; w < warp; ++w) pos += wcnt[w][mk];
+      perm[pos] = (int32_t)j;
+    }
+    __syncthreads();
+    for (int v = threadIdx.x; v < V; v += 256) {
+      int c = 0;
+      for (int w = 0; w < 8; ++w) c += wcnt[w][v];
+      next[v] += c;
+    }
+    __syncthreads();
+  }
+}
+
+// tmask[q] = OR of the masks at positions kProjTileRows q .. + kProjTileRows - 1 (one warp per tile)
+__global__ void __launch_bounds__(256) order_tiles(const int32_t* __restrict__ csr_ptr, TypeRels tr, int64_t n,
+                                                   const int32_t* __restrict__ perm, int64_t tiles,
+                                                   int32_t* __restrict__ tmask) {
+  const int64_t q = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (q >= tiles) return;
+  uint32_t m = 0;
+  for (int i = lane; i < kProjTileRows; i += 32) {
+    const int64_t p = q * kProjTileRows + i;
+    if (p < n) m |= node_mask(csr_ptr, tr, perm[p]);
+  }
+  m = __reduce_or_sync(0xffffffffu, m);
+  if (lane == 0) tmask[q] = (int32_t)m;
+}
+
+static int64_t order_blocks(int64_t n) { return ceil_div(n, kOrderTile); }
+// histogram entries over all types: sum_t 2^n_t ceil(n_t / kOrderTile) <= 2^8 (N / kOrderTile + kMaxTypes)
+static int64_t order_hist_cap(int64_t N) { return (int64_t)kMaskValues * (N / kOrderTile + kMaxTypes); }
+static int64_t order_tiles_cap(int64_t N) { return N / kProjTileRows + kMaxTypes; }
+
 // Rows above kHubDegree hold sum ceil(deg / kChunkEdges) <= E / kChunkEdges + E / (kHubDegree + 1)
 // chunks (each such row adds at most one partial chunk); +2 covers the integer floors.
 static int64_t chunk_cap(int64_t E) { return E / kChunkEdges + E / (kHubDegree + 1) + 2; }
@@ -556,6 +648,7 @@ struct GraphLayout {
   int32_t *agg_ptr, *agg_col, *agg_cnt, *agg_chunk_ofs, *agg_chunk_row;
   int32_t *bagg_ptr, *bagg_col, *bagg_cnt, *bagg_chunk_ofs, *bagg_chunk_row;
   int32_t *mrow, *mlist, *mbase;  // non-empty CSR rows: compact index per row, row per index, per relation
+  int32_t *nperm, *tmask, *ohist, *oofs;  // node order by relation mask, tile masks, the sort's counts
   SortBuffers sort;
 };
 
@@ -588,6 +681,10 @@ static size_t carve_graph(void* ws, int64_t E, int64_t rows, int64_t crows, int6
   L->mrow = c.take<int32_t>(rows + 1);
   L->mlist = c.take<int32_t>(rows + 1);
   L->mbase = c.take<int32_t>(kMaxRels + 1);
+  L->nperm = c.take<int32_t>(std::max<int64_t>(N, 1));
+  L->tmask = c.take<int32_t>(order_tiles_cap(N));
+  L->ohist = c.take<int32_t>(order_hist_cap(N) + 1);
+  L->oofs = c.take<int32_t>(order_hist_cap(N) + 1);
   L->invalid = c.take<int32_t>(1);
   L->cnt = c.take<int32_t>(std::max(std::max(rows, crows), N) + 1);
   L->sort.ckeys = c.take<uint32_t>(Ea + 1);
@@ -599,7 +696,8 @@ static size_t carve_graph(void* ws, int64_t E, int64_t rows, int64_t crows, int6
   const int64_t hist_n = sort_tiles(E) * kRadix;
   L->sort.hist = c.take<int32_t>(hist_n + 1);
   L->sort.scan_scratch =
-      c.take<char>(scan_scratch_bytes(std::max(std::max(std::max(hist_n, rows), std::max(crows, N)), Ea)));
+      c.take<char>(scan_scratch_bytes(std::max(std::max(std::max(hist_n, rows), std::max(crows, N)),
+                                               std::max(Ea, order_hist_cap(N)))));
   return c.used;
 }
 
@@ -781,6 +879,27 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
     HG_TRY(coalesce_runs(L.csr_col, L.csr_ptr, rows, E, nullptr, L, L.agg_col, L.agg_cnt, L.agg_ptr, s));
     HG_TRY(coalesce_runs(L.node_col, L.node_ptr, N, E, L.mrow, L, L.bagg_col, L.bagg_cnt, L.bagg_ptr, s));
   }
+  // node order of the forward projection, per type: sorted by relation mask, and each tile's mask
+  int64_t tile_base[kMaxTypes + 1] = {0};
+  for (int t = 0; t < m.num_types; ++t) {
+    const int64_t n = m.type_off[t + 1] - m.type_off[t];
+    tile_base[t + 1] = tile_base[t] + ceil_div(n, kProjTileRows);
+    if (n == 0) continue;
+    TypeRels tr{};
+    for (int r = 0; r < num_rels; ++r)
+      if (m.rel_dst[r] == t) tr.row0[tr.n++] = m.row_base[r];
+    const int nblk = (int)order_blocks(n);
+    const int64_t nh = ((int64_t)1 << tr.n) * nblk;
+    HG_TRY(launch("order_hist", order_hist, dim3(nblk), dim3(256), 0, s, (const int32_t*)L.csr_ptr, tr, n, nblk,
+                  L.ohist));
+    HG_TRY(exclusive_scan(L.ohist, L.oofs, nh, L.sort.scan_scratch, s));
+    int32_t* perm = L.nperm + m.type_off[t];
+    HG_TRY(launch("order_scatter", order_scatter, dim3(nblk), dim3(256), 0, s, (const int32_t*)L.csr_ptr, tr, n,
+                  nblk, (const int32_t*)L.oofs, perm));
+    const int64_t tiles = tile_base[t + 1] - tile_base[t];
+    HG_TRY(launch("order_tiles", order_tiles, dim3((unsigned)ceil_div(tiles * 32, 256)), dim3(256), 0, s,
+                  (const int32_t*)L.csr_ptr, tr, n, (const int32_t*)perm, tiles, L.tmask + tile_base[t]));
+  }
   // chunk tables for rows above the hub degree: per edge (attention layer), per run (mean layer)
   HG_TRY(chunk_table(L.csr_ptr, rows, L.csr_chunk_ofs, L.csr_chunk_row, L, s));
   HG_TRY(chunk_table(L.node_ptr, N, L.node_chunk_ofs, L.node_chunk_row, L, s));
@@ -821,8 +940,24 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
   gh->mrow = L.mrow;
   gh->mlist = L.mlist;
   gh->mbase = L.mbase;
+  gh->nperm = L.nperm;
+  gh->tmask = L.tmask;
+  for (int t = 0; t <= kMaxTypes; ++t) gh->tile_base[t] = tile_base[std::min(t, m.num_types)];
   gh->invalid_count = L.invalid;
   *out = gh;
+  return HG_OK;
+}
+
+extern "C" hg_status hg_graph_node_order(const hg_graph* graph, int32_t type, hg_node_order* out) {
+  clear_error();
+  HG_REQUIRE(graph != nullptr && out != nullptr, "graph and out must be non-null");
+  const GraphMeta& m = graph->meta;
+  HG_REQUIRE(type >= 0 && type < m.num_types, "type %d out of range", type);
+  out->n = m.type_off[type + 1] - m.type_off[type];
+  out->tiles = graph->tile_base[type + 1] - graph->tile_base[type];
+  out->tile_rows = kProjTileRows;
+  out->perm = graph->nperm + m.type_off[type];
+  out->tile_mask = graph->tmask + graph->tile_base[type];
   return HG_OK;
 }
 

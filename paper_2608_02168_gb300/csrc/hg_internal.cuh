@@ -16,6 +16,7 @@ namespace hg {
 // ---------------------------------------------------------------------------------------------
 constexpr int kMaxTypes = 4;
 constexpr int kMaxRels = 8;
+constexpr int kProjTileRows = 128;  // output rows per tile of the tensor-core forward projection
 // A CSR/CSC row with more than kHubDegree edges is split into chunks of kChunkEdges edges; each
 // chunk's fp32 partial sum goes to scratch and the row is finished by adding the chunk partials
 // in chunk order, so the reduction order is fixed (deterministic, atomic-free).
@@ -147,6 +148,13 @@ struct hg_graph {
   int32_t* mrow;            // [csr_rows + 1]
   int32_t* mlist;           // [csr_rows + 1]
   int32_t* mbase;           // [kMaxRels + 1], device
+  // Node order of the bf16 forward projection, per type t: the type's nodes sorted stably by their
+  // relation mask (bit k = the k-th relation into t, by ascending id, has an in-edge at the node),
+  // so that a 128-row tile rarely mixes masks.  nperm[type_off[t] + i] = local id of position i;
+  // tmask[tile_base[t] + q] = OR of the masks of positions 128 q .. 128 q + 127.
+  int32_t* nperm;           // [N]
+  int32_t* tmask;           // [tile_base[num_types]]
+  int64_t tile_base[hg::kMaxTypes + 1];
   int32_t* invalid_count;  // device scalar
 };
 

@@ -264,6 +264,8 @@ hg_status project_forward(const hg_graph* graph, const hg_layer_params* p, const
       a.type = t;
       a.mrow = compact ? graph->mrow : nullptr;
       a.msent = graph->csr_rows;
+      a.perm = compact ? graph->nperm + m.type_off[t] : nullptr;
+      a.tmask = compact ? graph->tmask + graph->tile_base[t] : nullptr;
       a.b = (const __nv_bfloat16*)p->b_agg + (size_t)t * d;
       a.gamma = p->layernorm ? (const __nv_bfloat16*)p->ln_gamma + (size_t)t * d : nullptr;
       a.beta = p->layernorm ? (const __nv_bfloat16*)p->ln_beta + (size_t)t * d : nullptr;

@@ -58,6 +58,9 @@ struct TcFwdArgs {
   int64_t mrow0[kMaxRels];    // first CSR row of each
   const int32_t* mrow;        // row of M holding each CSR row (>= msent: an empty row, read as zeros);
   int64_t msent;              // null: M is indexed by CSR row.  msent = the row extent of M
+  const __nv_bfloat16* M;     // relation means, [msent][D]
+  const int32_t* perm;        // tile position -> local node (the type's nodes by relation mask); null: identity
+  const int32_t* tmask;       // per tile, the relations (bit k = rel[k]) with a stored row in it; null: all
   int type;
   const __nv_bfloat16* b;
   const __nv_bfloat16* gamma;

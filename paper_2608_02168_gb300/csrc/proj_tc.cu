@@ -10,9 +10,12 @@
 // bf16(V_r), V_lo = bf16(V_r - V_hi); about 16 significant bits) and every product with it is two
 // MMAs into the same fp32 accumulator.
 //
-// Forward, one CTA per 128 destination rows of type t:
-//   U = sum_{r -> t} M_r V_r      A = relation means (TMA, 128 x 64 tiles), B = V_r^T chunks
-//                                 (the hi and lo halves of a chunk in one pipeline stage)
+// Forward, one CTA per 128 destination rows of type t, rows in the graph's node order (the type's
+// nodes sorted by which relations have in-edges at them, so that a tile's rows share their stored
+// relation rows):
+//   U = sum_{r -> t} M_r V_r      over the relations with a stored row in the tile; A = the rows'
+//                                 relation means (cp.async gathers, 128 x 64 tiles, empty rows zero),
+//                                 B = V_r^T chunks (hi and lo halves of a chunk in one stage)
 //   epilogue: U_s = bf16(U) stored, then U = U_s + b in fp32; Y = act(U) + H_in;
 //             H_out = LayerNorm(Y); row statistics saved.  U is stored without its bias: the
 //             rounding then scales with the data (Z W_agg), not with a large bias, and the
@@ -25,9 +28,9 @@
 //   weight gradients: G_r = M_r^T dU (split-K GEMM, MN-major TMA operands), then
 //                     dW_r = G_r W_agg^T and dW_agg[t] = sum_{r -> t} W_r^T G_r (wgrad_finish).
 //
-// Thread layout of the tensor-core kernels: 128 threads; thread (warp w, lane l) owns accumulator
-// row 32 w + l (its TMEM lane).  Thread 0 issues every TMA load and MMA.  All waits are bounded
-// (tc::kSpinLimit) and report through the library status word.
+// Epilogue threads own one accumulator row each (warp w reads TMEM lanes 32 (w % 4) ..); one
+// thread issues the MMAs.  All waits are bounded (tc::kSpinLimit) and report through the library
+// status word.
 #include <algorithm>
 #include <cstring>
 
@@ -44,26 +47,34 @@ namespace {
 constexpr int kTileRows = 128;
 constexpr int kATile = kTileRows * 128;  // 128 rows x 64 bf16
 
-// Persistent forward: one CTA per SM, warp 0 loads (TMA), warp 1 issues the MMAs, warps 2-5 run
-// the epilogue; two TMEM accumulators and two residual tiles let the epilogue of one 128-row tile
-// overlap the loads and MMAs of the next.
+// Persistent forward: one CTA per SM.  Warps 0-1 load the operands (cp.async gathers of A rows,
+// thread 0 also the weight chunks by TMA), warp 2 issues the MMAs, warps 3-10 run the epilogue, two
+// threads per row (one per column half; eight warps, two per scheduler).  Two TMEM accumulators and
+// two residual tiles let the epilogue of one 128-row tile overlap the loads and MMAs of the next,
+// and every role loads the next tile's metadata (relations, node order, rows of M) ahead of time.
 template <int D>
 struct FwdCfg {
   static constexpr int kStages = D == 256 ? 2 : (D == 128 ? 3 : 4);
   static constexpr int kB = D * 128;  // D rows x 64 bf16 (one half of the weight pair)
   static constexpr int kStage = kATile + 2 * kB;  // A | B_hi | B_lo
-  // The H_in tile (residual) is fetched by TMA, double-buffered, where shared memory allows it; at
+  // The H_in rows (residual) are staged in shared memory, double-buffered, where it has room; at
   // D = 256 the epilogue reads H_in from global memory.
   static constexpr bool kHTile = D <= 128;
   static constexpr int kH = kHTile ? kTileRows * D * 2 : 0;
   static constexpr int kParams = 3 * D * 4;  // bias, gamma, beta in fp32
-  static constexpr int kIdx = kTileRows * 4;  // the tile's A-row coordinates
-  static constexpr int kSmem = kStages * kStage + 2 * kH + kParams + kIdx + 512 + 1024;
+  static constexpr int kRed = 2 * 2 * kTileRows * 4;  // row partial sums of the two column halves
+  static constexpr int kSmem = kStages * kStage + 2 * kH + kParams + kRed + 256 + 1024;
   static_assert(kSmem <= 227 * 1024, "shared memory of proj_fwd_tc");
   static constexpr int kAccCols = D < 32 ? 32 : D;
   static constexpr int kTmemCols = 2 * kAccCols;
-  static constexpr int kThreads = 192;
+  static constexpr int kProducers = 64;  // threads; 64 A rows each of a stage's 128 per warp
+  static constexpr int kMmaWarp = 2;
+  static constexpr int kEpiWarp0 = 3;
+  static constexpr int kEpiThreads = 2 * kTileRows;
+  static constexpr int kThreads = 96 + kEpiThreads;
+  static constexpr int kHalf = D / 2;  // columns per epilogue thread
 };
+static_assert(kTileRows == kProjTileRows, "tile of the node order");
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
@@ -91,175 +102,283 @@ __device__ __forceinline__ void store16_bf16(__nv_bfloat16* p, const float* v) {
 
 template <int D>
 __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
-    proj_fwd_tc(const __grid_constant__ CUtensorMap tm_M, const __grid_constant__ CUtensorMap tm_Vt,
-                const __grid_constant__ CUtensorMap tm_H, TcFwdArgs a) {
+    proj_fwd_tc(const __grid_constant__ CUtensorMap tm_Vt, TcFwdArgs a) {
   using C = FwdCfg<D>;
   constexpr int S = C::kStages;
-  constexpr int KC = D / 64;  // 64-wide K chunks per D
+  constexpr int KC = D / 64;        // 64-wide K chunks per D
+  constexpr uint32_t kLag = S - 1;  // stages a producer thread keeps in flight before releasing one
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   uint8_t* stage = smem;                  // S x (A | B)
   uint8_t* htile = smem + S * C::kStage;  // 2 x KC x 16 KB, 128B-swizzled rows
   float* params = reinterpret_cast<float*>(htile + 2 * C::kH);  // [3][D]: b, gamma, beta
-  uint64_t* full = reinterpret_cast<uint64_t*>(params + 3 * D + kTileRows);  // (a 512-byte gap before the barriers)
+  float* red = params + 3 * D;                                  // [2 sums][2 halves][128 rows]
+  uint64_t* full = reinterpret_cast<uint64_t*>(red + 4 * kTileRows);
   uint64_t* empty = full + S;
-  uint64_t* acc_full = empty + S;   // [2] MMA -> epilogue
+  uint64_t* acc_full = empty + S;      // [2] MMA -> epilogue
   uint64_t* acc_empty = acc_full + 2;  // [2] epilogue -> MMA
-  uint64_t* h_full = acc_empty + 2;    // [2] TMA -> epilogue
-  uint64_t* h_empty = h_full + 2;      // [2] epilogue -> TMA
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(h_empty + 2);
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(acc_empty + 2);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t ntiles = (a.n + kTileRows - 1) / kTileRows;
-  const int CT = a.nrel * KC;
+  const int64_t G = gridDim.x;
+  const uint32_t all = (1u << a.nrel) - 1u;
+  // the relations whose products tile q computes (a relation without a stored row in it is skipped)
+  auto rels_of = [&](int64_t q) -> uint32_t {
+    if (q >= ntiles) return 0u;
+    return a.tmask ? (uint32_t)__ldg(a.tmask + q) & all : all;
+  };
+  // local node at position m of the order; -1 past the type
+  auto node_at = [&](int64_t m) -> int64_t {
+    if (m >= a.n) return -1;
+    return a.perm ? (int64_t)__ldg(a.perm + m) : m;
+  };
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
-      mbar_init(&full[s], 1);
+      mbar_init(&full[s], C::kProducers + 1);  // the producer threads and the weight loads' byte count
       mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
-      mbar_init(&acc_empty[b], kTileRows);
-      mbar_init(&h_full[b], 1);
-      mbar_init(&h_empty[b], kTileRows);
+      mbar_init(&acc_empty[b], C::kEpiThreads);
     }
     fence_mbar_init();
-    prefetch_tmap(&tm_M);
     prefetch_tmap(&tm_Vt);
-    if (C::kHTile) prefetch_tmap(&tm_H);
   }
-  if (warp == 1) tmem_alloc(tslot, C::kTmemCols);
+  if (warp == C::kMmaWarp) tmem_alloc(tslot, C::kTmemCols);
   fence_before_sync();
   __syncthreads();
   fence_after_sync();
   const uint32_t tmem = *tslot;
 
-  if (warp == 0) {
-    // ---- TMA producer: lane q gathers A rows 4q .. 4q + 3 of every chunk (four rows per copy; a row
-    // past the type or an empty relation row, at or past the map's extent, reads zeros), its row
-    // indices loaded one relation ahead; lane 0 posts each stage's byte count first and loads the
-    // V_r^T hi / lo chunks and the residual tile
+  if (warp < C::kMmaWarp) {
+    // ---- producers.  Warp w fills rows 64 w .. 64 w + 63 of every A stage from M with cp.async:
+    // one instruction copies four whole 128-byte row chunks (lane l: chunk l % 8 of row 4 k + l / 8),
+    // into the 128B-swizzled layout the MMA reads; a row past the type or without a stored relation
+    // row is zero-filled without a read.  Thread 0 also loads the stage's V_r^T hi / lo chunks by
+    // TMA.  A thread releases a stage kLag stages after issuing it: once its own copies have landed
+    // (wait_group) and are fenced for the async proxy, it arrives on the stage's barrier.  The
+    // nodes of the tile after next and the rows of M of the next tile are loaded while a tile's
+    // stages are issued.
+    const int t = threadIdx.x;
+    const int rbase = warp * 64;
     bool ok = true;
-    uint32_t g = 0;
-    int it = 0;
-    auto rows_of = [&](int64_t m0, int r, int* c) {
+    uint32_t g = 0, done = 0;  // stages issued, stages released
+    // nodes of this lane's two rows (rbase + lane, rbase + 32 + lane) of tile q
+    auto nodes = [&](int64_t q, int64_t* j) {
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int64_t m = m0 + 4 * lane + i;
-        int64_t v = a.msent;
-        if (r < a.nrel && m < a.n) v = a.mrow ? (int64_t)__ldg(a.mrow + a.mrow0[r] + m) : a.mrow0[r] + m;
-        c[i] = (int)v;
-      }
+      for (int h = 0; h < 2; ++h) j[h] = q < ntiles ? node_at(q * kTileRows + rbase + 32 * h + lane) : -1;
     };
-    for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
-      const int64_t m0 = tile * kTileRows;
-      const int b = it & 1;
-      if (C::kHTile && lane == 0) {
-        if (it >= 2) ok = mbar_wait(&h_empty[b], ((it >> 1) - 1) & 1);
-        if (ok) {
-          mbar_expect_tx(&h_full[b], C::kH);
-          for (int kc = 0; kc < KC; ++kc)
-            tma_load_2d(htile + b * C::kH + kc * kATile, &tm_H, kc * 64, (int)m0, &h_full[b]);
+    // rows of M of those nodes for each relation of tm (-1: zeros)
+    auto mrows = [&](uint32_t tm, const int64_t* j, int32_t (*v)[2]) {
+#pragma unroll
+      for (int r = 0; r < kMaxRels; ++r)
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          int64_t x = -1;
+          if (((tm >> r) & 1u) && j[h] >= 0)
+            x = a.mrow ? (int64_t)__ldg(a.mrow + a.mrow0[r] + j[h]) : a.mrow0[r] + j[h];
+          v[r][h] = x >= 0 && x < a.msent ? (int32_t)x : -1;
+        }
+    };
+    int64_t tile = blockIdx.x;
+    uint32_t tm_c = rels_of(tile), tm_n = rels_of(tile + G);
+    int64_t j_c[2], j_n[2];
+    int32_t v_c[kMaxRels][2];
+    nodes(tile, j_c);
+    nodes(tile + G, j_n);
+    mrows(tm_c, j_c, v_c);
+    for (; tile < ntiles && ok; tile += G) {
+      int32_t v_n[kMaxRels][2];
+      mrows(tm_n, j_n, v_n);  // the next tile's rows of M (its nodes were loaded a tile ago)
+      const uint32_t tm_nn = rels_of(tile + 2 * G);
+      int64_t j_nn[2];
+      nodes(tile + 2 * G, j_nn);
+#pragma unroll
+      for (int r = 0; r < kMaxRels; ++r) {
+        if (!((tm_c >> r) & 1u) || !ok) continue;
+        int32_t vk[16];  // the row this lane copies in instruction k: 4 k + lane / 8
+#pragma unroll
+        for (int k = 0; k < 16; ++k) vk[k] = __shfl_sync(0xffffffffu, v_c[r][k >> 3], ((4 * k) & 31) + (lane >> 3));
+        for (int kc = 0; kc < KC; ++kc, ++g) {
+          const uint32_t s = g % S;
+          if (g >= (uint32_t)S) ok = mbar_wait(&empty[s], ((g / S) - 1) & 1);
+          if (!ok) break;
+          uint8_t* A = stage + s * C::kStage;
+          if (t == 0) {
+            mbar_expect_tx(&full[s], 2 * C::kB);
+            tma_load_2d(A + kATile, &tm_Vt, kc * 64, 2 * a.rel[r] * D, &full[s]);                // hi
+            tma_load_2d(A + kATile + C::kB, &tm_Vt, kc * 64, (2 * a.rel[r] + 1) * D, &full[s]);  // lo
+          }
+          const int ch = lane & 7;
+#pragma unroll
+          for (int k = 0; k < 16; ++k) {
+            const int rr = rbase + 4 * k + (lane >> 3);
+            cp_async16(A + sw128_offset(rr, ch * 16), a.M + (int64_t)max(vk[k], 0) * D + kc * 64 + ch * 8, vk[k] >= 0);
+          }
+          cp_async_commit();
+          if (g + 1 - done > kLag) {
+            cp_async_wait<kLag>();
+            fence_async_smem();
+            mbar_arrive(&full[done % S]);
+            ++done;
+          }
         }
       }
-      ok = __shfl_sync(0xffffffffu, ok, 0);
-      int c[4], cn[4];
-      rows_of(m0, 0, c);
-      for (int r = 0; r < a.nrel && ok; ++r) {
-        rows_of(m0, r + 1, cn);  // the next relation's rows, in flight while these are issued
-        for (int kc = 0; kc < KC && ok; ++kc, ++g) {
-          const uint32_t s = g % S;
-          uint8_t* A = stage + s * C::kStage;
-          if (lane == 0) {
-            if (g >= (uint32_t)S) ok = mbar_wait(&empty[s], ((g / S) - 1) & 1);
-            if (ok) {
-              mbar_expect_tx(&full[s], C::kStage);
-              tma_load_2d(A + kATile, &tm_Vt, kc * 64, 2 * a.rel[r] * D, &full[s]);           // hi
-              tma_load_2d(A + kATile + C::kB, &tm_Vt, kc * 64, (2 * a.rel[r] + 1) * D, &full[s]);  // lo
-            }
-          }
-          ok = __shfl_sync(0xffffffffu, ok, 0);
-          if (ok) tma_gather4(A + lane * 512, &tm_M, kc * 64, c[0], c[1], c[2], c[3], &full[s]);
-        }
+      tm_c = tm_n;
+      tm_n = tm_nn;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) c[i] = cn[i];
+      for (int h = 0; h < 2; ++h) {
+        j_n[h] = j_nn[h];
+#pragma unroll
+        for (int r = 0; r < kMaxRels; ++r) v_c[r][h] = v_n[r][h];
       }
     }
-    if (lane == 0 && !ok) atomicOr(a.status, kErrTimeout);
-    __syncwarp();
-  } else if (warp == 1) {
-    // ---- MMA issuer: U_tile = sum_r M_r V_r into accumulator (it & 1)
+    cp_async_wait<0>();  // also on the give-up path: no copy outlives the kernel
+    if (ok) {
+      fence_async_smem();
+      for (; done < g; ++done) mbar_arrive(&full[done % S]);
+    } else {
+      atomicOr(a.status, kErrTimeout);
+    }
+  } else if (warp == C::kMmaWarp) {
+    // ---- MMA issuer: U_tile = sum_r M_r V_r into accumulator (it & 1), over the tile's relations
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16(128, D, false, false);
       bool ok = true;
       uint32_t g = 0;
       int it = 0;
-      for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
+      uint32_t tm_n = rels_of(blockIdx.x);
+      for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += G, ++it) {
+        const uint32_t tm = tm_n;
+        tm_n = rels_of(tile + G);  // in flight during this tile
         const int b = it & 1;
         if (it >= 2) ok = mbar_wait(&acc_empty[b], ((it >> 1) - 1) & 1);
         if (!ok) break;
         fence_after_sync();
         const uint32_t acc = tmem + b * C::kAccCols;
-        for (int j = 0; j < CT && ok; ++j, ++g) {
-          const uint32_t s = g % S;
-          ok = mbar_wait(&full[s], (g / S) & 1);
-          if (!ok) break;
-          fence_after_sync();
-          const uint32_t A = smem_u32(stage + s * C::kStage);
+        bool first = true;
+        for (int r = 0; r < a.nrel && ok; ++r) {
+          if (!((tm >> r) & 1u)) continue;
+          for (int kc = 0; kc < KC; ++kc, ++g) {
+            const uint32_t s = g % S;
+            ok = mbar_wait(&full[s], (g / S) & 1);
+            if (!ok) break;
+            fence_after_sync();
+            const uint32_t A = smem_u32(stage + s * C::kStage);
 #pragma unroll
-          for (int ks = 0; ks < 4; ++ks) {
-            const uint64_t ad = desc_sw128(A + ks * 32, 16, 1024);
-            mma_bf16(acc, ad, desc_sw128(A + kATile + ks * 32, 16, 1024), idesc, (j > 0 || ks > 0) ? 1u : 0u);
-            mma_bf16(acc, ad, desc_sw128(A + kATile + C::kB + ks * 32, 16, 1024), idesc, 1u);
+            for (int ks = 0; ks < 4; ++ks) {
+              const uint64_t ad = desc_sw128(A + ks * 32, 16, 1024);
+              mma_bf16(acc, ad, desc_sw128(A + kATile + ks * 32, 16, 1024), idesc, (first && ks == 0) ? 0u : 1u);
+              mma_bf16(acc, ad, desc_sw128(A + kATile + C::kB + ks * 32, 16, 1024), idesc, 1u);
+            }
+            first = false;
+            mma_commit(&empty[s]);
           }
-          mma_commit(&empty[s]);
         }
-        mma_commit(&acc_full[b]);
+        if (!ok) break;
+        if (tm != 0) {
+          mma_commit(&acc_full[b]);
+        } else {
+          mbar_arrive(&acc_full[b]);  // no products: the epilogue reads no accumulator
+        }
       }
       if (!ok) atomicOr(a.status, kErrTimeout);
     }
     __syncwarp();
   } else {
-    // ---- epilogue: bias, activation, residual, LayerNorm; warp w owns TMEM lanes 32 (w % 4) ..
+    // ---- epilogue: bias, activation, residual, LayerNorm.  Warp w owns TMEM lanes 32 (w % 4) ..;
+    // thread (row, half) handles columns kHalf * half .. + kHalf of its row; the two halves of a
+    // row add their partial sums through shared memory (a barrier per pair of warps).
     const int q = warp & 3;
+    const int hf = (warp - C::kEpiWarp0) >> 2;
     const int row = q * 32 + lane;
+    const int c0 = hf * C::kHalf;
     const float* pb = params;
     const float* pgm = params + D;
     const float* pbe = params + 2 * D;
-    for (int c = threadIdx.x - 64; c < D; c += kTileRows) {
+    for (int c = threadIdx.x - C::kEpiWarp0 * 32; c < D; c += C::kEpiThreads) {
       params[c] = __bfloat162float(a.b[c]);
       params[D + c] = a.ln ? __bfloat162float(a.gamma[c]) : 1.f;
       params[2 * D + c] = a.ln ? __bfloat162float(a.beta[c]) : 0.f;
     }
-    asm volatile("bar.sync 1, 128;" ::: "memory");  // the four epilogue warps
+    asm volatile("bar.sync 1, %0;" ::"n"(C::kEpiThreads) : "memory");  // the epilogue warps
+    const uint32_t pair_bar = 2 + q;  // warps q and q + 4 of the epilogue: the two halves of its rows
+    // the row's total of v over both halves (the same sum, v0 + v1, in both threads)
+    auto pair_sum = [&](float v, int which) -> float {
+      red[(which * 2 + hf) * kTileRows + row] = v;
+      asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
+      return v + red[(which * 2 + (hf ^ 1)) * kTileRows + row];
+    };
+    // Row transfers between global memory and the warp's 32 rows (its column half) of a
+    // 128B-swizzled tile: lane l moves 16-byte chunk l % kCh of row kRpi k + l / kCh, the row's
+    // node taken from the lane that owns it.
+    constexpr int kCh = C::kHalf / 8, kRpi = 32 / kCh;
+    auto chunk_at = [&](uint8_t* t, int rr, int ch) {  // rr: row within the warp's 32
+      const int cg = hf * kCh + ch;                     // chunk within the full row
+      return t + (cg >> 3) * kATile + sw128_offset(q * 32 + rr, (cg & 7) * 16);
+    };
+    // the residual of the warp's rows (nodes jw, per lane) into buffer hb; one commit group per call
+    auto fetch_h = [&](int64_t jw, int hb) {
+      if constexpr (C::kHTile) {
+        uint8_t* t = htile + hb * C::kH;
+#pragma unroll
+        for (int k = 0; k < 32 / kRpi; ++k) {
+          const int rr = kRpi * k + lane / kCh, ch = lane % kCh;
+          const int64_t jj = __shfl_sync(0xffffffffu, jw, rr);
+          if (jj >= 0) cp_async16(chunk_at(t, rr, ch), a.H_in + (a.off + jj) * D + c0 + ch * 8, true);
+        }
+        cp_async_commit();
+      }
+    };
+    // the warp's rows of tile buffer t to out (the rows of nodes jw)
+    auto store_rows = [&](uint8_t* t, int64_t jw, __nv_bfloat16* out) {
+#pragma unroll
+      for (int k = 0; k < 32 / kRpi; ++k) {
+        const int rr = kRpi * k + lane / kCh, ch = lane % kCh;
+        const int64_t jj = __shfl_sync(0xffffffffu, jw, rr);
+        if (jj >= 0) st16(out + (a.off + jj) * D + c0 + ch * 8, *reinterpret_cast<const uint4*>(chunk_at(t, rr, ch)));
+      }
+    };
     bool ok = true;
     int it = 0;
-    for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
+    int64_t j_c = node_at((int64_t)blockIdx.x * kTileRows + row);  // this tile's node at the row
+    int64_t j_n = node_at(((int64_t)blockIdx.x + G) * kTileRows + row);  // the next tile's
+    bool has_n = rels_of(blockIdx.x) != 0;
+    fetch_h(j_c, 0);
+    for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += G, ++it) {
       const int b = it & 1;
-      const int64_t m = tile * kTileRows + row;
-      const bool live = m < a.n;
-      const int64_t node = a.off + (live ? m : 0);
+      const int64_t j = j_c;
+      const bool live = j >= 0;
+      const int64_t node = a.off + (live ? j : 0);
+      const bool has = has_n;  // else U = 0 without an accumulator
+      has_n = rels_of(tile + G) != 0;
+      fetch_h(j_n, b ^ 1);  // the next tile's residual rows, in flight during this tile
+      const int64_t j_nn = node_at((tile + 2 * G) * kTileRows + row);
       ok = mbar_wait(&acc_full[b], (it >> 1) & 1);
-      if (ok && C::kHTile) ok = mbar_wait(&h_full[b], (it >> 1) & 1);
+      ok = bar_and(pair_bar, 64, ok);  // both halves of a row give up together (no lone pair barrier)
       if (!ok) break;
       fence_after_sync();
+      if constexpr (C::kHTile) {
+        cp_async_wait<1>();  // this tile's residual rows have landed (this lane's copies) ...
+        __syncwarp();        // ... and the other lanes'
+      }
       const uint32_t trow = tmem + b * C::kAccCols + ((uint32_t)(q * 32) << 16);
-      const uint8_t* ht = htile + b * C::kH;
-      // U_s = bf16(acc) for columns c .. c+15 (acc already in u when preloaded), stored;
-      // returned as U_s + b in u
-      auto u16 = [&](int c, float* u, bool store, bool preloaded = false) {
+      uint8_t* ht = htile + b * C::kH;
+      // U_s = bf16(acc) for columns c .. c+15 (acc already in u when preloaded), stored to global
+      // memory when store_g; returned as U_s + b in u, and packed in up
+      auto u16 = [&](int c, float* u, uint32_t* up, bool store_g, bool preloaded = false) {
         if (!preloaded) {
-          if (CT > 0) {
+          if (has) {
             tmem_ld16(trow + c, u);
           } else {
 #pragma unroll
             for (int i = 0; i < 16; ++i) u[i] = 0.f;
           }
         }
-        uint32_t up[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) up[i] = pack_bf16x2(u[2 * i], u[2 * i + 1]);
-        if (store && live) {
+        if (store_g && live) {
           st16(a.U + node * D + c, make_uint4(up[0], up[1], up[2], up[3]));
           st16(a.U + node * D + c + 8, make_uint4(up[4], up[5], up[6], up[7]));
         }
@@ -279,21 +398,31 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
           load16_bf16(a.H_in + node * D + c, h);
         }
       };
-      auto out16 = [&](int c, const float* y, float mean, float rstd) {  // H_out columns c .. c+15
-        float o[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) o[i] = a.ln ? (y[i] - mean) * rstd * pgm[c + i] + pbe[c + i] : y[i];
-        if (live) store16_bf16(a.H_out + node * D + c, o);
+      auto put16 = [&](int c, const uint32_t* up) {  // 16 packed columns into this thread's tile row
+        uint8_t* t = ht + (c >> 6) * kATile;
+        const uint32_t cb = (uint32_t)(c & 63) * 2;
+        *reinterpret_cast<uint4*>(t + sw128_offset(row, cb)) = make_uint4(up[0], up[1], up[2], up[3]);
+        *reinterpret_cast<uint4*>(t + sw128_offset(row, cb + 16)) = make_uint4(up[4], up[5], up[6], up[7]);
       };
-      if constexpr (D <= 128) {
-        // the whole row in registers: one pass over TMEM
-        float y[D];
+      auto out16 = [&](int c, const float* y, float mean, float rstd, uint32_t* up) {  // H_out, c .. c+15
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int k0 = 2 * i, k1 = k0 + 1;
+          const float o0 = a.ln ? (y[k0] - mean) * rstd * pgm[c + k0] + pbe[c + k0] : y[k0];
+          const float o1 = a.ln ? (y[k1] - mean) * rstd * pgm[c + k1] + pbe[c + k1] : y[k1];
+          up[i] = pack_bf16x2(o0, o1);
+        }
+      };
+      if constexpr (C::kHTile) {
+        // the half row in registers: one pass over TMEM.  U_s replaces the residual in the tile row
+        // once read, then H_out; each leaves as whole row chunks per instruction.
+        float y[C::kHalf];
         float sum = 0.f;
 #pragma unroll
-        for (int c = 0; c < D; c += 32) {
+        for (int cc = 0; cc < C::kHalf; cc += 32) {
           float u[32];
-          if (CT > 0) {
-            tmem_ld32(trow + c, u);
+          if (has) {
+            tmem_ld32(trow + c0 + cc, u);
           } else {
 #pragma unroll
             for (int i = 0; i < 32; ++i) u[i] = 0.f;
@@ -301,67 +430,89 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
 #pragma unroll
           for (int hh = 0; hh < 32; hh += 16) {
             float h[16];
-            u16(c + hh, u + hh, true, true);
-            h16(c + hh, h);
+            uint32_t up[8];
+            h16(c0 + cc + hh, h);
+            u16(c0 + cc + hh, u + hh, up, false, true);
+            put16(c0 + cc + hh, up);
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
-              y[c + hh + i] = act_apply(u[hh + i], a.act) + h[i];
-              sum += y[c + hh + i];
+              y[cc + hh + i] = act_apply(u[hh + i], a.act) + h[i];
+              sum += y[cc + hh + i];
             }
           }
         }
-        const float mean = sum * (1.f / D);
+        fence_before_sync();
+        mbar_arrive(&acc_empty[b]);  // the accumulator is read: the MMAs of tile it + 2 may start
+        __syncwarp();
+        store_rows(ht, j, a.U);
+        const float mean = pair_sum(sum, 0) * (1.f / D);
         float qq = 0.f;
 #pragma unroll
-        for (int i = 0; i < D; ++i) qq += (y[i] - mean) * (y[i] - mean);
-        const float rstd = rsqrtf(qq * (1.f / D) + a.eps);
+        for (int i = 0; i < C::kHalf; ++i) qq += (y[i] - mean) * (y[i] - mean);
+        const float rstd = rsqrtf(pair_sum(qq, 1) * (1.f / D) + a.eps);
+        __syncwarp();  // every lane has read U_s from the tile
 #pragma unroll
-        for (int c = 0; c < D; c += 16) out16(c, y + c, mean, rstd);
-        if (a.ln && live) a.stats[node] = make_float2(mean, rstd);
+        for (int cc = 0; cc < C::kHalf; cc += 16) {
+          uint32_t up[8];
+          out16(c0 + cc, y + cc, mean, rstd, up);
+          put16(c0 + cc, up);
+        }
+        __syncwarp();
+        store_rows(ht, j, a.H_out);
+        if (a.ln && live && hf == 0) a.stats[node] = make_float2(mean, rstd);
+        __syncwarp();  // the tile buffer is refilled two tiles on
       } else {
         // three passes over TMEM and the residual (row sum, centred sum of squares, output)
         auto y16 = [&](int c, float* y, bool store) {
           float u[16], h[16];
-          u16(c, u, store);
+          uint32_t up[8];
+          u16(c, u, up, store);
           h16(c, h);
 #pragma unroll
           for (int i = 0; i < 16; ++i) y[i] = act_apply(u[i], a.act) + h[i];
         };
         float sum = 0.f;
 #pragma unroll 1
-        for (int c = 0; c < D; c += 16) {
+        for (int cc = 0; cc < C::kHalf; cc += 16) {
           float y[16];
-          y16(c, y, true);
+          y16(c0 + cc, y, true);
 #pragma unroll
           for (int i = 0; i < 16; ++i) sum += y[i];
         }
-        const float mean = sum * (1.f / D);
+        const float mean = pair_sum(sum, 0) * (1.f / D);
         float qq = 0.f;
 #pragma unroll 1
-        for (int c = 0; c < D; c += 16) {
+        for (int cc = 0; cc < C::kHalf; cc += 16) {
           float y[16];
-          y16(c, y, false);
+          y16(c0 + cc, y, false);
 #pragma unroll
           for (int i = 0; i < 16; ++i) qq += (y[i] - mean) * (y[i] - mean);
         }
-        const float rstd = rsqrtf(qq * (1.f / D) + a.eps);
+        const float rstd = rsqrtf(pair_sum(qq, 1) * (1.f / D) + a.eps);
 #pragma unroll 1
-        for (int c = 0; c < D; c += 16) {
+        for (int cc = 0; cc < C::kHalf; cc += 16) {
           float y[16];
-          y16(c, y, false);
-          out16(c, y, mean, rstd);
+          uint32_t up[8];
+          y16(c0 + cc, y, false);
+          out16(c0 + cc, y, mean, rstd, up);
+          if (live) {
+            st16(a.H_out + node * D + c0 + cc, make_uint4(up[0], up[1], up[2], up[3]));
+            st16(a.H_out + node * D + c0 + cc + 8, make_uint4(up[4], up[5], up[6], up[7]));
+          }
         }
-        if (a.ln && live) a.stats[node] = make_float2(mean, rstd);
+        if (a.ln && live && hf == 0) a.stats[node] = make_float2(mean, rstd);
+        fence_before_sync();
+        mbar_arrive(&acc_empty[b]);
       }
-      fence_before_sync();
-      mbar_arrive(&acc_empty[b]);
-      if (C::kHTile) mbar_arrive(&h_empty[b]);
+      j_c = j_n;
+      j_n = j_nn;
     }
+    if constexpr (C::kHTile) cp_async_wait<0>();  // no residual copy outlives the kernel
     if (!ok) atomicOr(a.status, kErrTimeout);
   }
   fence_before_sync();
   __syncthreads();
-  if (warp == 1) tmem_dealloc(tmem, C::kTmemCols);
+  if (warp == C::kMmaWarp) tmem_dealloc(tmem, C::kTmemCols);
 }
 
 // Fused weights V_r = W_r W_agg[t_r] accumulated in fp64 (exact for bf16 factors of these sizes),
@@ -1074,23 +1225,20 @@ static hg_status tc_fuse_t(const void* W_rel, const void* W_agg, RelDst rd, int 
 }
 
 template <int D>
-static hg_status tc_fwd_t(const TcFwdArgs& a, const void* M, int64_t m_rows, const void* Vt, int num_rels,
+static hg_status tc_fwd_t(const TcFwdArgs& a0, const void* M, int64_t m_rows, const void* Vt, int num_rels,
                           cudaStream_t s) {
   HG_TRY(smem_attr_once<D>());
-  CUtensorMap tm_M, tm_V, tm_H;
-  HG_TRY(make_tmap_bf16(&tm_M, M, (uint64_t)std::max<int64_t>(m_rows, 1), D, 1));  // one-row box: gathers
+  TcFwdArgs a = a0;
+  a.M = (const __nv_bfloat16*)M;
+  a.msent = m_rows;
+  CUtensorMap tm_V;
   HG_TRY(make_tmap_bf16(&tm_V, Vt, (uint64_t)2 * num_rels * D, D, D));
-  if (FwdCfg<D>::kHTile) {
-    HG_TRY(make_tmap_bf16(&tm_H, a.H_in + a.off * D, (uint64_t)a.n, D, kTileRows));
-  } else {
-    tm_H = tm_M;  // unused
-  }
   int sms = 0, dev = 0;
   HG_CUDA(cudaGetDevice(&dev));
   HG_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
   const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(a.n, kTileRows), sms));
-  return launch("proj_fwd_tc", proj_fwd_tc<D>, dim3(grid), dim3(FwdCfg<D>::kThreads), FwdCfg<D>::kSmem, s, tm_M,
-                tm_V, tm_H, a);
+  return launch("proj_fwd_tc", proj_fwd_tc<D>, dim3(grid), dim3(FwdCfg<D>::kThreads), FwdCfg<D>::kSmem, s, tm_V,
+                a);
 }
 
 template <int D>

@@ -31,6 +31,11 @@ class hg_graph_arrays(Structure):
                 ("csc_eid", c_void_p), ("csc_coef", c_void_p)]
 
 
+class hg_node_order(Structure):
+    _fields_ = [("n", c_int64), ("tiles", c_int64), ("tile_rows", c_int32), ("perm", c_void_p),
+                ("tile_mask", c_void_p)]
+
+
 class hg_layer_params(Structure):
     _fields_ = [("d", c_int32), ("dtype", c_int32), ("act", c_int32), ("layernorm", c_int32), ("ln_eps", c_float),
                 ("W_rel", c_void_p), ("W_agg", c_void_p), ("b_agg", c_void_p), ("ln_gamma", c_void_p),
@@ -90,6 +95,7 @@ EXPORTS = {
     "hg_graph_destroy": (c_int32, [c_void_p]),
     "hg_graph_check": (c_int32, [c_void_p, POINTER(c_int64)]),
     "hg_graph_view": (c_int32, [c_void_p, c_int32, POINTER(hg_graph_arrays)]),
+    "hg_graph_node_order": (c_int32, [c_void_p, c_int32, POINTER(hg_node_order)]),
     "hg_layer_workspace_size": (c_int32, [c_void_p, POINTER(hg_layer_params), POINTER(c_size_t), POINTER(c_size_t)]),
     "hg_layer_fwd": (c_int32, [c_void_p, POINTER(hg_layer_params), c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),
     "hg_layer_bwd": (c_int32, [c_void_p, POINTER(hg_layer_params), c_void_p, c_void_p, c_void_p, c_void_p,
@@ -264,6 +270,22 @@ def hg_graph_view(g: Graph, rel: int) -> dict:
                 col=view(a.col, E, torch.int32), eid=view(a.eid, E, torch.int32),
                 csc_ptr=view(a.csc_ptr, a.n_src + 1, torch.int32), csc_col=view(a.csc_col, E, torch.int32),
                 csc_eid=view(a.csc_eid, E, torch.int32), csc_coef=view(a.csc_coef, E, torch.float32))
+
+
+def hg_graph_node_order(g: Graph, node_type: int) -> dict:
+    """Device views of the forward projection's node order of one type: perm (position -> local id,
+    sorted stably by relation mask) and tile_mask (OR of the masks of each tile of tile_rows rows)."""
+    a = hg_node_order()
+    _check(lib().hg_graph_node_order(g.handle, int(node_type), byref(a)), "hg_graph_node_order")
+    ws = g.workspace
+    base = ws.data_ptr()
+
+    def view(ptr, n):
+        off = ptr - base
+        return ws[off:off + n * 4].view(torch.int32)
+
+    return dict(n=a.n, tiles=a.tiles, tile_rows=a.tile_rows, perm=view(a.perm, a.n),
+                tile_mask=view(a.tile_mask, a.tiles))
 
 
 # ------------------------------------------------------------------------------------------------

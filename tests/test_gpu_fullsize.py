@@ -62,6 +62,15 @@ def test_full_csr_invariants(full):
         want = np.float32(1) / deg[dst[ceid] - offs[tt]].astype(np.float32)
         assert np.array_equal(coef.view(np.uint32), want.view(np.uint32))
     assert seen.all()
+    # the forward projection's node order, bit-exact against its definition on in-degrees counted
+    # from the COO list
+    degs = [dict(deg=np.bincount(dst[rel == r] - offs[tt], minlength=int(offs[tt + 1] - offs[tt])))
+            for r, (_, tt) in enumerate(g["rels"])]
+    for t in range(len(offs) - 1):
+        o = hg.hg_graph_node_order(G, t)
+        perm, tmask = oracle.node_order(degs, offs, g["rels"], t, tile_rows=o["tile_rows"])
+        assert np.array_equal(o["perm"].cpu().numpy(), perm), f"perm t{t}"
+        assert np.array_equal(o["tile_mask"].cpu().numpy(), tmask), f"tile_mask t{t}"
 
 
 def sample_rows(w, k, seed):

@@ -18,6 +18,15 @@ def gpu_csr(hg, src, dst, rel, offs, rels):
     return G, bad
 
 
+def compare_node_order(hg, G, ref, offs, rels):
+    for t in range(len(offs) - 1):
+        o = hg.hg_graph_node_order(G, t)
+        perm, tmask = oracle.node_order(ref, offs, rels, t, tile_rows=o["tile_rows"])
+        assert o["n"] == len(perm) and o["tiles"] == len(tmask)
+        assert np.array_equal(o["perm"].cpu().numpy(), perm), f"perm t{t}"
+        assert np.array_equal(o["tile_mask"].cpu().numpy(), tmask), f"tile_mask t{t}"
+
+
 def compare_layout(hg, G, ref, rels):
     for r in range(len(rels)):
         v = hg.hg_graph_view(G, r)
@@ -43,7 +52,9 @@ def test_random_coo_with_invalid_edges(seed):
     src, dst, rel, offs, rels = random_coo(seed, n_user=300, n_risk=70, num_edges=20_000, bad=300)
     G, bad = gpu_csr(hg, src, dst, rel, offs, rels)
     assert bad == int((~oracle.valid_edges(src, dst, rel, offs, rels)).sum()) == 300
-    compare_layout(hg, G, oracle.build_csr(src, dst, rel, offs, rels), rels)
+    ref = oracle.build_csr(src, dst, rel, offs, rels)
+    compare_layout(hg, G, ref, rels)
+    compare_node_order(hg, G, ref, offs, rels)
 
 
 def test_tiny_workload_graph():
@@ -52,7 +63,9 @@ def test_tiny_workload_graph():
     g = hgsynth.make_graph(hgsynth.spec("tiny-10k"))
     G, bad = gpu_csr(hg, g["src"], g["dst"], g["rel"], g["type_offsets"], g["rels"])
     assert bad == 0
-    compare_layout(hg, G, oracle.build_csr(g["src"], g["dst"], g["rel"], g["type_offsets"], g["rels"]), g["rels"])
+    ref = oracle.build_csr(g["src"], g["dst"], g["rel"], g["type_offsets"], g["rels"])
+    compare_layout(hg, G, ref, g["rels"])
+    compare_node_order(hg, G, ref, g["type_offsets"], g["rels"])
 
 
 def test_hub_rows_and_degenerate_graphs():
@@ -69,12 +82,16 @@ def test_hub_rows_and_degenerate_graphs():
     src, dst, rel = src[perm], dst[perm], rel[perm]
     G, bad = gpu_csr(hg, src, dst, rel, offs, rels)
     assert bad == 0
-    compare_layout(hg, G, oracle.build_csr(src, dst, rel, offs, rels), rels)
+    ref = oracle.build_csr(src, dst, rel, offs, rels)
+    compare_layout(hg, G, ref, rels)
+    compare_node_order(hg, G, ref, offs, rels)
     # no edges at all
     e = np.zeros(0, np.int64)
     G, bad = gpu_csr(hg, e, e, e, offs, rels)
     assert bad == 0
-    compare_layout(hg, G, oracle.build_csr(e, e, e, offs, rels), rels)
+    ref = oracle.build_csr(e, e, e, offs, rels)
+    compare_layout(hg, G, ref, rels)
+    compare_node_order(hg, G, ref, offs, rels)
     # every edge invalid
     G, bad = gpu_csr(hg, np.full(10, 5000), np.zeros(10, np.int64), np.zeros(10, np.int64), offs, rels)
     assert bad == 10
@@ -85,7 +102,9 @@ def test_hub_rows_and_degenerate_graphs():
     r2 = np.zeros(400, np.int64)
     G, bad = gpu_csr(hg, s2, d2, r2, offs2, rels)
     assert bad == 0
-    compare_layout(hg, G, oracle.build_csr(s2, d2, r2, offs2, rels), rels)
+    ref = oracle.build_csr(s2, d2, r2, offs2, rels)
+    compare_layout(hg, G, ref, rels)
+    compare_node_order(hg, G, ref, offs2, rels)
 
 
 def test_build_is_repeatable():
@@ -97,3 +116,30 @@ def test_build_is_repeatable():
         G, bad = gpu_csr(hg, src, dst, rel, offs, rels)
         assert bad == 10
         compare_layout(hg, G, ref, rels)
+        compare_node_order(hg, G, ref, offs, rels)
+
+
+def test_node_order_with_eight_relations_into_one_type():
+    # 2^8 relation masks over 50,000 destinations (25 blocks of the counting sort, a ragged last tile):
+    # Zipf-like destinations per relation so that every mask value from sparse to dense occurs
+    need_gpu()
+    hg = lib()
+    rels = tuple([(0, 0)] * 4 + [(1, 0)] * 4)
+    offs = np.array([0, 50_001, 53_001], np.int64)
+    rng = np.random.default_rng(11)
+    src, dst, rel = [], [], []
+    for r, (ts, _) in enumerate(rels):
+        k = 20_000 + 6_000 * r
+        d = np.minimum((rng.pareto(0.8 + 0.1 * r, k) * 50).astype(np.int64), 50_000)
+        dst.append(d)
+        src.append(offs[ts] + rng.integers(0, offs[ts + 1] - offs[ts], k))
+        rel.append(np.full(k, r))
+    src, dst, rel = np.concatenate(src), np.concatenate(dst), np.concatenate(rel)
+    perm = rng.permutation(len(src))
+    src, dst, rel = src[perm], dst[perm], rel[perm]
+    G, bad = gpu_csr(hg, src, dst, rel, offs, rels)
+    assert bad == 0
+    ref = oracle.build_csr(src, dst, rel, offs, rels)
+    compare_node_order(hg, G, ref, offs, rels)
+    mask = sum((ref[r]["deg"] > 0).astype(np.int64) << r for r in range(8))
+    assert len(np.unique(mask)) > 200  # nearly every mask value occurs

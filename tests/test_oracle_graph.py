@@ -78,6 +78,35 @@ def test_csr_matches_brute_force(seed):
                 assert c["csc_coef"][a + k] == np.float32(1.0) / np.float32(len(bf[r][t - offs[tt]]))
 
 
+@pytest.mark.parametrize("seed", [0, 3])
+def test_node_order_matches_brute_force(seed):
+    # the forward projection's node order: a Python sorted() by (mask, id), the mask built edge by
+    # edge from the valid COO entries; tile masks by OR loops over tiles of 8 rows (ragged last tile)
+    src, dst, rel, offs, rels = random_coo(seed, n_user=61, n_risk=13, num_edges=300)
+    csr = oracle.build_csr(src, dst, rel, offs, rels)
+    ok = oracle.valid_edges(src, dst, rel, offs, rels)
+    for t in range(len(offs) - 1):
+        n = int(offs[t + 1] - offs[t])
+        into = [r for r, (_, tt) in enumerate(rels) if tt == t]
+        mask = [0] * n
+        for e in range(len(src)):
+            if ok[e] and rel[e] in into:
+                mask[int(dst[e] - offs[t])] |= 1 << into.index(int(rel[e]))
+        want = sorted(range(n), key=lambda j: (mask[j], j))
+        perm, tmask = oracle.node_order(csr, offs, rels, t, tile_rows=8)
+        assert list(perm) == want
+        for q in range(len(tmask)):
+            m = 0
+            for j in want[8 * q:8 * q + 8]:
+                m |= mask[j]
+            assert tmask[q] == m
+        assert len(tmask) == (n + 7) // 8
+    # a type without incoming relations (type 1 when the only relation is user -> user) keeps its
+    # local order, every mask 0
+    perm, tmask = oracle.node_order(csr[:1], offs, [(0, 0)], 1)
+    assert list(perm) == list(range(int(offs[2] - offs[1]))) and not tmask.any()
+
+
 def test_csr_invariants():
     src, dst, rel, offs, rels = random_coo(7, num_edges=2000, bad=50)
     csr = oracle.build_csr(src, dst, rel, offs, rels)
