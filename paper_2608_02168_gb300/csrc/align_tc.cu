@@ -336,6 +336,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                    desc_sw128(B + kc * (D * 128) + ks * 32, 16, 1024), idesc, (kc > 0 || ks > 0) ? 1u : 0u);
     } else {
       atomicOr(status, kErrTimeout);
+      mbar_wait(bbar, 0);  // give-up path: the weight load still lands before the CTA moves on
     }
     mma_commit(accb);
   }

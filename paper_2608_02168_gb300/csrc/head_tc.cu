@@ -167,7 +167,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   fence_async_smem();
   const bool two = __syncthreads_or(rowi[tid] >= 0 && repi[tid] >= 0) != 0;  // any replica in the tile
+  int chains = 0;  // MMA chains issued (thread 0)
   auto issue_chain = [&](bool accumulate) {
+    ++chains;
     fence_after_sync();
     const uint32_t A = smem_u32(Aimg), W = smem_u32(Wimg);
     const uint32_t idesc = idesc_bf16(128, D, false, true);
@@ -279,6 +281,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     out[0] = ((rowred[0] + rowred[2]) + rowred[4]) + rowred[6];
     out[1] = ((rowred[1] + rowred[3]) + rowred[5]) + rowred[7];
   }
+  if (!ok && tid == 0) {  // give-up path: the weight load and the MMAs issued complete first
+    mbar_wait(&bars[0], 0);
+    if (chains > 0) mbar_wait(&bars[1], (uint32_t)(chains - 1) & 1u);
+  }
+  __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, D);
 }
 
@@ -325,12 +332,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       mma_commit(&bars[1]);
     } else {
       record_device_error(a.status, kErrTimeout);
+      mbar_wait(&bars[0], 0);  // give-up path: the loads land before the CTA moves on
     }
   }
   ok = __syncthreads_and(ok);
   if (ok && !mbar_wait(&bars[1], 0)) {
     record_device_error(a.status, kErrTimeout);
     ok = false;
+    if (tid == 0) mbar_wait(&bars[1], 0);  // the MMAs issued complete before TMEM is released
   }
   fence_after_sync();
   const int64_t r = r0 + tid;

@@ -117,7 +117,8 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
   uint64_t* empty = full + S;
   uint64_t* acc_full = empty + S;      // [2] MMA -> epilogue
   uint64_t* acc_empty = acc_full + 2;  // [2] epilogue -> MMA
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(acc_empty + 2);
+  uint64_t* drainb = acc_empty + 2;    // the MMA issuer's give-up path
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(drainb + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t ntiles = (a.n + kTileRows - 1) / kTileRows;
@@ -142,6 +143,7 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
       mbar_init(&acc_full[b], 1);
       mbar_init(&acc_empty[b], C::kEpiThreads);
     }
+    mbar_init(drainb, 1);
     fence_mbar_init();
     prefetch_tmap(&tm_Vt);
   }
@@ -234,12 +236,14 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
         for (int r = 0; r < kMaxRels; ++r) v_c[r][h] = v_n[r][h];
       }
     }
-    cp_async_wait<0>();  // also on the give-up path: no copy outlives the kernel
-    if (ok) {
-      fence_async_smem();
-      for (; done < g; ++done) mbar_arrive(&full[done % S]);
-    } else {
+    // Every stage issued is released, also on the give-up path: its phase can then complete, and
+    // thread 0 waits (bounded) for the weight loads of each stage's last round before the CTA exits.
+    cp_async_wait<0>();
+    fence_async_smem();
+    for (; done < g; ++done) mbar_arrive(&full[done % S]);
+    if (!ok) {
       atomicOr(a.status, kErrTimeout);
+      if (t == 0) drain_rounds(full, S, g);
     }
   } else if (warp == C::kMmaWarp) {
     // ---- MMA issuer: U_tile = sum_r M_r V_r into accumulator (it & 1), over the tile's relations
@@ -283,7 +287,10 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
           mbar_arrive(&acc_full[b]);  // no products: the epilogue reads no accumulator
         }
       }
-      if (!ok) atomicOr(a.status, kErrTimeout);
+      if (!ok) {
+        atomicOr(a.status, kErrTimeout);
+        drain_mma(drainb, 0);  // the MMAs issued so far complete before TMEM is released
+      }
     }
     __syncwarp();
   } else {
@@ -621,13 +628,22 @@ __global__ void __launch_bounds__(256) wgrad_finish(const float* __restrict__ G,
   }
 }
 
+// ln_act_bwd: rows per warp whose loads are in flight together, and resident blocks per SM (the
+// register budget that keeps them without spills)
+template <int D>
+struct LnCfg {
+  static constexpr int kRows = D == 256 ? 2 : (D == 128 ? 3 : 4);
+  static constexpr int kBlocks = D == 256 ? 1 : (D == 128 ? 3 : 4);
+};
+
 // LayerNorm / activation backward, one warp per row (coalesced rows, D / 32 columns per lane):
 // U = stored U_s + b (as in the forward), dY = rstd (dXh - mean(dXh) - Xh mean(dXh Xh)),
 // dXh = dH_out gamma, dU = dY act'(U); per-block
 // column partials part[block] = {sum dU, sum dH_out Xh, sum dH_out} over the block's rows.
 template <int D>
-__global__ void __launch_bounds__(256) ln_act_bwd(TcBwdArgs a) {
+__global__ void __launch_bounds__(256, LnCfg<D>::kBlocks) ln_act_bwd(TcBwdArgs a) {
   constexpr int E = D / 32;
+  constexpr int kLnRows = LnCfg<D>::kRows;
   __shared__ float red[8][3][D];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int c0 = lane * E;
@@ -640,21 +656,6 @@ __global__ void __launch_bounds__(256) ln_act_bwd(TcBwdArgs a) {
   float pdb[E], pdg[E], pdbe[E];
 #pragma unroll
   for (int i = 0; i < E; ++i) pdb[i] = pdg[i] = pdbe[i] = 0.f;
-  auto load = [&](const __nv_bfloat16* p, float* v) {
-    if constexpr (E == 2) {
-      const uint32_t w = *reinterpret_cast<const uint32_t*>(p);
-      v[0] = __uint_as_float(w << 16);
-      v[1] = __uint_as_float(w & 0xFFFF0000u);
-    } else if constexpr (E == 4) {
-      const uint2 w = *reinterpret_cast<const uint2*>(p);
-      v[0] = __uint_as_float(w.x << 16);
-      v[1] = __uint_as_float(w.x & 0xFFFF0000u);
-      v[2] = __uint_as_float(w.y << 16);
-      v[3] = __uint_as_float(w.y & 0xFFFF0000u);
-    } else {
-      unpack(ld16(p), v, __nv_bfloat16());
-    }
-  };
   auto store = [&](__nv_bfloat16* p, const float* v) {
     if constexpr (E == 2) {
       *reinterpret_cast<uint32_t*>(p) = pack_bf16x2(v[0], v[1]);
@@ -664,35 +665,51 @@ __global__ void __launch_bounds__(256) ln_act_bwd(TcBwdArgs a) {
       st16(p, pack(v, __nv_bfloat16()));
     }
   };
-  // two rows per iteration: both rows' loads are in flight before either is computed
+  // kLnRows rows per iteration: all their loads are in flight before any is computed (held as the
+  // raw bf16 words, E / 2 registers per tensor and row)
+  using Raw = typename std::conditional<E == 2, uint32_t, typename std::conditional<E == 4, uint2, uint4>::type>::type;
+  auto unpack_raw = [&](const Raw& w, float* v) {
+    if constexpr (E == 2) {
+      v[0] = __uint_as_float(w << 16);
+      v[1] = __uint_as_float(w & 0xFFFF0000u);
+    } else if constexpr (E == 4) {
+      v[0] = __uint_as_float(w.x << 16);
+      v[1] = __uint_as_float(w.x & 0xFFFF0000u);
+      v[2] = __uint_as_float(w.y << 16);
+      v[3] = __uint_as_float(w.y & 0xFFFF0000u);
+    } else {
+      unpack(w, v, __nv_bfloat16());
+    }
+  };
   const int64_t step = (int64_t)gridDim.x * 8;
-  for (int64_t row0 = (int64_t)blockIdx.x * 8 + warp; row0 < a.n; row0 += 2 * step) {
-    float dv[2][E], uv[2][E], hv[2][E];
-    float2 st[2];
-    bool has[2];
+  for (int64_t row0 = (int64_t)blockIdx.x * 8 + warp; row0 < a.n; row0 += kLnRows * step) {
+    Raw rd[kLnRows], ru[kLnRows], rh[kLnRows];
+    float2 st[kLnRows];
 #pragma unroll
-    for (int k = 0; k < 2; ++k) {
+    for (int k = 0; k < kLnRows; ++k) {
       const int64_t row = row0 + k * step;
-      has[k] = row < a.n;
-      const int64_t node = a.off + (has[k] ? row : row0);
-      load(a.dH_out + node * D + c0, dv[k]);
-      load(a.U + node * D + c0, uv[k]);
-#pragma unroll
-      for (int i = 0; i < E; ++i) uv[k][i] += bias[i];
-      load(a.H_in + node * D + c0, hv[k]);
-      st[k] = a.ln ? a.stats[node] : make_float2(0.f, 1.f);
+      const int64_t o = (a.off + (row < a.n ? row : row0)) * D + c0;
+      rd[k] = *reinterpret_cast<const Raw*>(a.dH_out + o);
+      ru[k] = *reinterpret_cast<const Raw*>(a.U + o);
+      rh[k] = *reinterpret_cast<const Raw*>(a.H_in + o);
+      st[k] = a.ln ? a.stats[a.off + (row < a.n ? row : row0)] : make_float2(0.f, 1.f);
     }
 #pragma unroll
-    for (int k = 0; k < 2; ++k) {
-      if (!has[k]) continue;
-      const int64_t node = a.off + row0 + k * step;
-      float dy[E], du[E], xh[E];
+    for (int k = 0; k < kLnRows; ++k) {
+      const int64_t row = row0 + k * step;
+      if (row >= a.n) continue;
+      float dv[E], uv[E], hv[E], dy[E], du[E], xh[E];
+      unpack_raw(rd[k], dv);
+      unpack_raw(ru[k], uv);
+      unpack_raw(rh[k], hv);
+#pragma unroll
+      for (int i = 0; i < E; ++i) uv[i] += bias[i];
       if (a.ln) {
         float s1 = 0.f, s2 = 0.f;
 #pragma unroll
         for (int i = 0; i < E; ++i) {
-          xh[i] = (act_apply(uv[k][i], a.act) + hv[k][i] - st[k].x) * st[k].y;
-          const float dxh = dv[k][i] * g[i];
+          xh[i] = (act_apply(uv[i], a.act) + hv[i] - st[k].x) * st[k].y;
+          const float dxh = dv[i] * g[i];
           s1 += dxh;
           s2 += dxh * xh[i];
         }
@@ -703,23 +720,24 @@ __global__ void __launch_bounds__(256) ln_act_bwd(TcBwdArgs a) {
         }
         const float mean1 = s1 * (1.f / D), mean2 = s2 * (1.f / D);
 #pragma unroll
-        for (int i = 0; i < E; ++i) dy[i] = st[k].y * (dv[k][i] * g[i] - mean1 - xh[i] * mean2);
+        for (int i = 0; i < E; ++i) dy[i] = st[k].y * (dv[i] * g[i] - mean1 - xh[i] * mean2);
       } else {
 #pragma unroll
         for (int i = 0; i < E; ++i) {
-          dy[i] = dv[k][i];
+          dy[i] = dv[i];
           xh[i] = 0.f;
         }
       }
 #pragma unroll
       for (int i = 0; i < E; ++i) {
-        du[i] = __bfloat162float(__float2bfloat16_rn(dy[i] * act_grad(uv[k][i], a.act)));
+        du[i] = __bfloat162float(__float2bfloat16_rn(dy[i] * act_grad(uv[i], a.act)));
         pdb[i] += du[i];
-        pdg[i] += dv[k][i] * xh[i];
-        pdbe[i] += dv[k][i];
+        pdg[i] += dv[i] * xh[i];
+        pdbe[i] += dv[i];
       }
-      store(a.dY + node * D + c0, dy);
-      store(a.dU + node * D + c0, du);
+      const int64_t o = (a.off + row) * D + c0;
+      store(a.dY + o, dy);
+      store(a.dU + o, du);
     }
   }
 #pragma unroll
@@ -809,7 +827,8 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
   uint64_t* a_empty = a_full + 2;       // [NA] the job's products done
   uint64_t* acc_full = a_empty + 2;     // [NB]
   uint64_t* acc_empty = acc_full + NB;  // [NB]
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(acc_empty + NB);
+  uint64_t* drainb = acc_empty + NB;    // the MMA issuer's give-up path
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(drainb + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   __shared__ BwdJobs J;
@@ -827,6 +846,7 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
       mbar_init(&acc_full[k], 1);
       mbar_init(&acc_empty[k], kTileRows);
     }
+    mbar_init(drainb, 1);
     fence_mbar_init();
     prefetch_tmap(&tm_dU);
     prefetch_tmap(&tm_V);
@@ -840,7 +860,7 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
 
   if (warp == 0) {  // ---- producer: lane q gathers the job's dU rows 4q .. 4q + 3, lane 0 streams V_r
     bool ok = true;
-    uint32_t g = 0;
+    uint32_t g = 0, a_issued = 0;
     int it = 0;
     for (int64_t job = blockIdx.x; job < njobs && ok; job += gridDim.x, ++it) {
       const int j = J.rel_of(job);
@@ -863,6 +883,7 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
         uint8_t* A = tiles + ab * C::kT;
         for (int kc = 0; kc < KC; ++kc)
           tma_gather4(A + kc * kATile + lane * 512, &tm_dU, kc * 64, c[0], c[1], c[2], c[3], &a_full[ab]);
+        ++a_issued;
       }
       if (lane == 0) {
         for (int kc = 0; kc < KC && ok; ++kc, ++g) {
@@ -876,7 +897,11 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
       }
       ok = __shfl_sync(0xffffffffu, ok, 0);
     }
-    if (lane == 0 && !ok) atomicOr(a.status, kErrTimeout);
+    if (lane == 0 && !ok) {
+      atomicOr(a.status, kErrTimeout);
+      drain_rounds(a_full, NA, a_issued);  // no gather or weight load still writes shared memory
+      drain_rounds(b_full, S, g);
+    }
     __syncwarp();
   } else if (warp == 1) {
     if (lane == 0) {  // ---- MMA issuer: one chain per job into accumulator (job count mod NB)
@@ -912,7 +937,10 @@ __global__ void __launch_bounds__(BwdCfg<D>::kThreads, 1)
         mma_commit(&acc_full[k]);
         mma_commit(&a_empty[ab]);
       }
-      if (!ok) atomicOr(a.status, kErrTimeout);
+      if (!ok) {
+        atomicOr(a.status, kErrTimeout);
+        drain_mma(drainb, 0);
+      }
     }
     __syncwarp();
   } else {  // ---- epilogue: scale by 1 / deg_r and store the job's dMs rows
@@ -1011,11 +1039,13 @@ __global__ void __launch_bounds__(WgCfg<D>::kThreads, 1)
   const uint32_t tmem = *tslot;
   if (warp == 0) {
     if (lane == 0) {
+      uint32_t issued = 0;
       auto issue_load = [&](int g) {
         const int st = g % S;
         uint8_t* stage = smem + st * stage_bytes;
         uint8_t* B = stage + R * C::kA;
         const int y = (int)((c0 + g) * 64);
+        ++issued;
         mbar_expect_tx(&full[st], stage_bytes);
         for (int r = 0; r < R; ++r) {
           tma_load_2d(stage + r * C::kA, &tm_X.m[r], mt * 128, y, &full[st]);
@@ -1045,8 +1075,11 @@ __global__ void __launch_bounds__(WgCfg<D>::kThreads, 1)
           if (ok) issue_load(g + S);
         }
       }
-      if (!ok) atomicOr(status, kErrTimeout);
-      mma_commit(accb);
+      if (!ok) {
+        atomicOr(status, kErrTimeout);
+        drain_rounds(full, S, issued);  // no load still writes shared memory
+      }
+      mma_commit(accb);  // the MMAs issued complete before TMEM is read and released
     }
     __syncwarp();
   }
@@ -1077,22 +1110,36 @@ __global__ void __launch_bounds__(WgCfg<D>::kThreads, 1)
 }
 
 // G_r = M_r^T dU over the stored (non-empty) rows of one relation r: row k of the relation's compact
-// range of M pairs with the dU row of its destination node.  Both operands are gathered by TMA
-// (one-row boxes, four rows per copy) as MN-major tiles of 64 rows; rows past the relation's count
-// read zeros.  Warp 0 writes each chunk's row coordinates and its lane 0 issues the copies, warp 1's
-// lane 0 the MMAs; the chunks are shared among the grid's splits by the count read on the device.
-// Grid (M tiles of 128 output rows, splits); part[split][D][D].
+// range of M pairs with the dU row of its destination node.  Warps 0-3 copy each 64-row chunk of
+// both operands with cp.async into MN-major 128B-swizzled tiles (one instruction: four whole
+// 128-byte row blocks; rows past the relation's count, and X columns past D, are zero-filled without
+// a read), releasing a stage kLag chunks after issuing it (wait_group, proxy fence, arrive); warp
+// 4's lane 0 issues the MMAs; warps 0-3 then read the accumulator.  The chunks are shared among the
+// grid's splits by the count read on the device.  Grid (M tiles of 128 output rows, splits);
+// part[split][D][D].
 template <int D>
-__global__ void __launch_bounds__(WgCfg<D>::kThreads, 1)
-    wgrad_rows_tc(const __grid_constant__ CUtensorMap tm_X, const __grid_constant__ CUtensorMap tm_Y, int S,
+struct WgRowsCfg {
+  static constexpr int kStages = 4;
+  static constexpr int kA = 2 * 8192;        // 64 rows x 128 columns of X (two 64-wide blocks)
+  static constexpr int kB = D / 64 * 8192;   // 64 rows x D columns of Y
+  static constexpr int kStage = kA + kB;
+  static constexpr int kSmem = kStages * kStage + 256 + 1024;
+  static_assert(kSmem <= 227 * 1024, "shared memory of wgrad_rows_tc");
+  static constexpr int kThreads = 160;
+};
+
+template <int D>
+__global__ void __launch_bounds__(WgRowsCfg<D>::kThreads, 1)
+    wgrad_rows_tc(const __nv_bfloat16* __restrict__ X, const __nv_bfloat16* __restrict__ Y,
                   const int32_t* __restrict__ mlist, const int32_t* __restrict__ mbase, int rel, int64_t row0,
-                  int64_t xsent, int64_t ysent, float* __restrict__ part, int* __restrict__ status) {
-  using C = WgCfg<D>;
+                  int64_t ny, float* __restrict__ part, int* __restrict__ status) {
+  using C = WgRowsCfg<D>;
+  constexpr int S = C::kStages;
+  constexpr uint32_t kLag = S - 1;
   constexpr int NB = D / 64;  // 64-wide column blocks of Y
-  constexpr int kStage = C::kA + NB * 8192;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S * kStage);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S * C::kStage);
   uint64_t* empty = full + S;
   uint64_t* accb = empty + S;
   uint32_t* tslot = reinterpret_cast<uint32_t*>(accb + 1);
@@ -1105,56 +1152,77 @@ __global__ void __launch_bounds__(WgCfg<D>::kThreads, 1)
   const int CT = (int)max((int64_t)0, min(nchunks, c0 + cps) - c0);
   if (threadIdx.x == 0) {
     for (int st = 0; st < S; ++st) {
-      mbar_init(&full[st], 1);
+      mbar_init(&full[st], 128);  // the four producer warps
       mbar_init(&empty[st], 1);
     }
     mbar_init(accb, 1);
     fence_mbar_init();
-    prefetch_tmap(&tm_X);
-    prefetch_tmap(&tm_Y);
   }
-  if (warp == 0) tmem_alloc(tslot, D);
+  if (warp == 4) tmem_alloc(tslot, D);
   fence_before_sync();
   __syncthreads();
   fence_after_sync();
   const uint32_t tmem = *tslot;
-  if (warp == 0) {  // ---- producer: lanes 0-15 gather X rows 4q .. 4q + 3, lanes 16-31 the same rows of Y
+  if (warp < 4) {
+    // ---- producers: warp w copies chunk rows 16 w .. 16 w + 15, lane l chunk l % 8 of a 64-wide
+    // block of row 16 w + 4 i + l / 8
     bool ok = true;
-    const int q = lane & 15;
-    const bool isx = lane < 16;
-    auto coords = [&](int g, int* c) {
+    uint32_t done = 0, issued = 0;
+    const int ch = lane & 7;
+    // rows of X (compact index) and Y (local destination) of this lane's four rows of chunk g; -1: zeros
+    auto rows_of = [&](int g, int64_t* xr, int64_t* yr) {
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
-        const int64_t k = (c0 + g) * 64 + 4 * q + i;
+        const int64_t k = (c0 + g) * 64 + 16 * warp + 4 * i + (lane >> 3);
         const bool in = g < CT && k < count;
-        c[i] = (int)(isx ? (in ? base + k : xsent) : (in ? (int64_t)__ldg(mlist + base + k) - row0 : ysent));
+        xr[i] = in ? base + k : -1;
+        yr[i] = in ? (int64_t)__ldg(mlist + base + k) - row0 : -1;
+        if (yr[i] >= ny) yr[i] = -1;
       }
     };
-    int c[4], cn[4];
-    coords(0, c);
+    int64_t xr[4], yr[4], xn[4], yn[4];
+    rows_of(0, xr, yr);
     for (int g = 0; g < CT && ok; ++g) {
-      coords(g + 1, cn);  // the next chunk's rows, in flight while these are issued
+      rows_of(g + 1, xn, yn);  // the next chunk's rows, in flight while these are issued
       const int st = g % S;
-      uint8_t* stage = smem + st * kStage;
-      if (lane == 0) {
-        if (g >= S) ok = mbar_wait(&empty[st], ((g / S) - 1) & 1);
-        if (ok) mbar_expect_tx(&full[st], kStage);
-      }
-      ok = __shfl_sync(0xffffffffu, ok, 0);
-      if (ok) {
-        if (isx) {
-          for (int b = 0; b < 2; ++b)
-            tma_gather4(stage + b * 8192 + q * 512, &tm_X, mt * 128 + b * 64, c[0], c[1], c[2], c[3], &full[st]);
-        } else {
-          for (int b = 0; b < NB; ++b)
-            tma_gather4(stage + C::kA + b * 8192 + q * 512, &tm_Y, b * 64, c[0], c[1], c[2], c[3], &full[st]);
+      if (g >= S) ok = mbar_wait(&empty[st], ((g / S) - 1) & 1);
+      if (!ok) break;
+      uint8_t* stage = smem + st * C::kStage;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int kr = 16 * warp + 4 * i + (lane >> 3);  // row of the chunk (K index)
+#pragma unroll
+        for (int b = 0; b < 2; ++b) {  // X columns mt * 128 + 64 b ..
+          const int col = mt * 128 + b * 64 + ch * 8;
+          const bool v = xr[i] >= 0 && col < D;
+          cp_async16(stage + b * 8192 + sw128_offset(kr, ch * 16), X + (v ? xr[i] * D + col : 0), v);
+        }
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+          const bool v = yr[i] >= 0;
+          cp_async16(stage + C::kA + b * 8192 + sw128_offset(kr, ch * 16), Y + (v ? yr[i] * D + b * 64 + ch * 8 : 0), v);
         }
       }
+      cp_async_commit();
+      ++issued;
+      if (issued - done > kLag) {
+        cp_async_wait<kLag>();
+        fence_async_smem();
+        mbar_arrive(&full[done % S]);
+        ++done;
+      }
 #pragma unroll
-      for (int i = 0; i < 4; ++i) c[i] = cn[i];
+      for (int i = 0; i < 4; ++i) {
+        xr[i] = xn[i];
+        yr[i] = yn[i];
+      }
     }
-    if (lane == 0 && !ok) atomicOr(status, kErrTimeout);
-  } else if (warp == 1 && lane == 0) {  // ---- MMA issuer
+    // every chunk issued is released, also on the give-up path (nothing else is in flight)
+    cp_async_wait<0>();
+    fence_async_smem();
+    for (; done < issued; ++done) mbar_arrive(&full[done % S]);
+    if (!ok && lane == 0) atomicOr(status, kErrTimeout);
+  } else if (lane == 0) {  // ---- MMA issuer
     const uint32_t idesc = idesc_bf16(128, D, true, true);
     bool ok = true;
     for (int g = 0; g < CT && ok; ++g) {
@@ -1162,7 +1230,7 @@ __global__ void __launch_bounds__(WgCfg<D>::kThreads, 1)
       ok = mbar_wait(&full[st], (g / S) & 1);
       if (!ok) break;
       fence_after_sync();
-      const uint32_t A0 = smem_u32(smem + st * kStage);
+      const uint32_t A0 = smem_u32(smem + st * C::kStage);
       const uint32_t B = A0 + C::kA;
 #pragma unroll
       for (int ks = 0; ks < 4; ++ks)
@@ -1171,31 +1239,33 @@ __global__ void __launch_bounds__(WgCfg<D>::kThreads, 1)
       mma_commit(&empty[st]);
     }
     if (!ok) atomicOr(status, kErrTimeout);
-    mma_commit(accb);
+    mma_commit(accb);  // also on the give-up path: the MMAs issued complete before TMEM is released
   }
   __syncwarp();
   if (!mbar_wait(accb, 0)) atomicOr(status, kErrTimeout);
   fence_after_sync();
-  const int orow = mt * 128 + warp * 32 + lane;  // output row i (column of X)
-  float* out = part + (int64_t)blockIdx.y * D * D;
+  if (warp < 4) {
+    const int orow = mt * 128 + warp * 32 + lane;  // output row i (column of X)
+    float* out = part + (int64_t)blockIdx.y * D * D;
 #pragma unroll 1
-  for (int c = 0; c < D; c += 16) {
-    float v[16];
-    if (CT > 0) {
-      tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + c, v);
-    } else {
+    for (int c = 0; c < D; c += 16) {
+      float v[16];
+      if (CT > 0) {
+        tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + c, v);
+      } else {
 #pragma unroll
-      for (int i = 0; i < 16; ++i) v[i] = 0.f;
-    }
-    if (orow < D) {
+        for (int i = 0; i < 16; ++i) v[i] = 0.f;
+      }
+      if (orow < D) {
 #pragma unroll
-      for (int i = 0; i < 16; i += 4)
-        *reinterpret_cast<float4*>(out + (int64_t)orow * D + c + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+        for (int i = 0; i < 16; i += 4)
+          *reinterpret_cast<float4*>(out + (int64_t)orow * D + c + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+      }
     }
   }
   fence_before_sync();
   __syncthreads();
-  if (warp == 0) tmem_dealloc(tmem, D);
+  if (warp == 4) tmem_dealloc(tmem, D);
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -1208,7 +1278,7 @@ static hg_status smem_attr_once() {
     HG_CUDA(cudaFuncSetAttribute(proj_fwd_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, FwdCfg<D>::kSmem));
     HG_CUDA(cudaFuncSetAttribute(proj_bwd_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, BwdCfg<D>::kSmem));
     HG_CUDA(cudaFuncSetAttribute(wgrad_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, WgCfg<D>::kSmem));
-    HG_CUDA(cudaFuncSetAttribute(wgrad_rows_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, WgCfg<D>::kSmem));
+    HG_CUDA(cudaFuncSetAttribute(wgrad_rows_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, WgRowsCfg<D>::kSmem));
     done = true;
   }
   return HG_OK;
@@ -1324,14 +1394,10 @@ static hg_status tc_wgrad_rows_t(const void* M, int64_t m_rows, const int32_t* m
   }
   const int mtiles = D > 128 ? D / 128 : 1;
   const int splits = wgrad_tc_splits(n, D);  // the stored rows (at most n) are split on the device
-  const int stage_bytes = WgCfg<D>::kA + (D / 64) * 8192;
-  const int stages = std::min(4, (WgCfg<D>::kSmem - 1024 - 256) / stage_bytes);
-  CUtensorMap tm_X, tm_Y;
-  HG_TRY(make_tmap_bf16(&tm_X, M, (uint64_t)std::max<int64_t>(m_rows, 1), D, 1));
-  HG_TRY(make_tmap_bf16(&tm_Y, (const __nv_bfloat16*)dU + y0 * D, (uint64_t)n, D, 1));
-  HG_TRY(launch("wgrad_tc", wgrad_rows_tc<D>, dim3(mtiles, splits), dim3(WgCfg<D>::kThreads),
-                (size_t)stages * stage_bytes + 256 + 1024, s, tm_X, tm_Y, stages, mlist, mbase, rel, row0,
-                m_rows, n, part, device_status_ptr()));
+  (void)m_rows;
+  HG_TRY(launch("wgrad_tc", wgrad_rows_tc<D>, dim3(mtiles, splits), dim3(WgRowsCfg<D>::kThreads),
+                (size_t)WgRowsCfg<D>::kSmem, s, (const __nv_bfloat16*)M, (const __nv_bfloat16*)dU + y0 * D, mlist,
+                mbase, rel, row0, n, part, device_status_ptr()));
   return reduce_partials(part, (int64_t)D * D, splits, (int64_t)D * D, out, tmp, s);
 }
 

@@ -95,12 +95,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       mma_commit(&bars[1]);
     } else {
       record_device_error(p.status, kErrTimeout);
+      mbar_wait(&bars[0], 0);  // give-up path: the loads land before the CTA moves on
     }
   }
   ok = __syncthreads_and(ok);
   if (ok && !mbar_wait(&bars[1], 0)) {
     record_device_error(p.status, kErrTimeout);
     ok = false;
+    if (tid == 0) mbar_wait(&bars[1], 0);  // the MMAs issued complete before TMEM is released
   }
   fence_after_sync();
   const int64_t r = r0 + q * 32 + lane;

@@ -120,6 +120,19 @@ __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
 __device__ __forceinline__ void fence_before_sync() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void fence_after_sync() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 // generic-proxy shared-memory writes -> visible to the async proxy (tensor core operand reads)
+// The barriers one issuing thread uses, with the phases it has begun on each (an expect_tx or a
+// commit), for its give-up path: drain() waits, bounded, for the last phase begun on each, so no
+// copy or MMA it issued is still in flight when the CTA releases TMEM or exits.
+template <int N>
+struct IssueLog {
+  uint32_t begun[N] = {};
+  __device__ __forceinline__ void begin(int i) { ++begun[i]; }
+  __device__ __forceinline__ void drain(uint64_t* bars) const {
+#pragma unroll
+    for (int i = 0; i < N; ++i)
+      if (begun[i] > 0) mbar_wait(&bars[i], (begun[i] - 1u) & 1u);
+  }
+};
 // Named barrier over `count` threads (whole warps) that also ANDs a predicate across them.
 __device__ __forceinline__ bool bar_and(uint32_t id, uint32_t count, bool p) {
   uint32_t r;
@@ -188,6 +201,22 @@ __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
                : "memory");
+}
+// Give-up path of a producer (after a bounded wait failed): waits, bounded, until the last round
+// issued on each of the S stage barriers (round g on barrier g % S; `issued` rounds so far) has
+// completed, so that no bulk copy still writes the CTA's shared memory when it moves on.
+__device__ __forceinline__ void drain_rounds(uint64_t* bar, int S, uint32_t issued) {
+  for (uint32_t s = 0; s < (uint32_t)S && s < issued; ++s) {
+    const uint32_t last = s + (uint32_t)S * ((issued - 1u - s) / (uint32_t)S);
+    mbar_wait(&bar[s], (last / (uint32_t)S) & 1u);
+  }
+}
+// Give-up path of an MMA issuer: every MMA this thread issued has completed (tracked by a commit to
+// a barrier that nothing else uses, waited at `parity`, bounded) before TMEM or shared memory is
+// released.
+__device__ __forceinline__ void drain_mma(uint64_t* bar, uint32_t parity) {
+  mma_commit(bar);
+  mbar_wait(bar, parity);
 }
 
 // Shared-memory matrix descriptor, 128-byte swizzle, sm_100 format (version 1 at bits 46-47,

@@ -167,8 +167,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   fence_after_sync();
   const uint32_t tmem = *tslot;
   bool ok = true;
+  IssueLog<3> lg;  // thread 0's copies and MMAs, for the give-up path
   if (tid == 0) {
     mbar_expect_tx(&bars[0], (uint32_t)(C::kW + p.w * C::kA));
+    lg.begin(0);
     for (int b = 0; b < C::NB; ++b) tma_load_2d(Wimg + b * C::kWBlk, &tm_Wa, b * 64, 0, &bars[0]);
     for (int k = 0; k < p.w; ++k)
       for (int b = 0; b < C::NB; ++b)
@@ -180,6 +182,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int k = 0; k < p.w; ++k)
         mma_kmaj_mn<D>(tmem + k * D, smem_u32(Cimg + k * C::kA), smem_u32(Wimg), idesc, false);
       mma_commit(&bars[1]);
+      lg.begin(1);
     } else {
       record_device_error(p.status, kErrTimeout);
     }
@@ -247,6 +250,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   fence_before_sync();
   __syncthreads();
+  if (!ok && tid == 0) lg.drain(bars);  // give-up path: nothing issued is still in flight
+  __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, tcols);
 }
 
@@ -294,9 +299,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   fence_after_sync();
   const uint32_t tmem = *tslot;
   bool ok = true;
+  IssueLog<3> lg;  // thread 0's copies and MMAs, for the give-up path
   if (tid == 0) {
     const uint32_t idesc = idesc_bf16(128, D, false, true);
     mbar_expect_tx(&bars[0], (uint32_t)(2 * C::kA + 3 * C::kW));
+    lg.begin(0);
     for (int b = 0; b < C::NB; ++b) {
       tma_load_2d(Ximg + b * kABlk, &tm_X, b * 64, (int)r0, &bars[0]);
       tma_load_2d(Himg + b * kABlk, &tm_Ht, b * 64, (int)r0, &bars[0]);
@@ -308,10 +315,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int g = 0; g < 3; ++g)
         mma_kmaj_mn<D>(tmem + g * D, smem_u32(Ximg), smem_u32(Wimg + g * C::NB * C::kWBlk), idesc, false);
       mma_commit(&bars[1]);
+      lg.begin(1);
       ok = mbar_wait(&bars[1], 0);  // W_i no longer read: load W_h into its buffer
     }
     if (ok) {
       mbar_expect_tx(&bars[0], (uint32_t)(3 * C::kW));
+      lg.begin(0);
       for (int b = 0; b < 3 * C::NB; ++b) tma_load_2d(Wimg + b * C::kWBlk, &tm_Wh, b * 64, 0, &bars[0]);
       ok = mbar_wait(&bars[0], 1);
     }
@@ -321,6 +330,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mma_kmaj_mn<D>(tmem + 1 * D, smem_u32(Himg), smem_u32(Wimg + C::NB * C::kWBlk), idesc, true);
       mma_kmaj_mn<D>(tmem + 3 * D, smem_u32(Himg), smem_u32(Wimg + 2 * C::NB * C::kWBlk), idesc, false);
       mma_commit(&bars[2]);
+      lg.begin(2);
     }
     if (!ok) record_device_error(p.status, kErrTimeout);
   }
@@ -403,6 +413,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   fence_before_sync();
   __syncthreads();
+  if (!ok && tid == 0) lg.drain(bars);  // give-up path: nothing issued is still in flight
+  __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, kCols);
 }
 
@@ -450,10 +462,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   fence_after_sync();
   const uint32_t tmem = *tslot;
   bool ok = true;
+  IssueLog<3> lg;  // thread 0's copies and MMAs, for the give-up path
   if (tid == 0) {
     const uint32_t idesc = idesc_bf16(128, D, false, false);
     const uint32_t A[3] = {smem_u32(Aimg), smem_u32(Aimg + C::kA), smem_u32(Aimg + 2 * C::kA)};
     mbar_expect_tx(&bars[0], (uint32_t)(3 * C::kA + 3 * C::kW));
+    lg.begin(0);
     for (int g = 0; g < 3; ++g)
       for (int b = 0; b < C::NB; ++b)
         tma_load_2d(Aimg + g * C::kA + b * kABlk, &tm_dG, b * 64, (int)(g * p.n + r0), &bars[0]);
@@ -463,10 +477,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       fence_after_sync();
       mma_gates_kmaj<D>(tmem, A, smem_u32(Wimg), idesc);
       mma_commit(&bars[1]);
+      lg.begin(1);
       ok = mbar_wait(&bars[1], 0);  // third tile and W_i no longer read
     }
     if (ok) {
       mbar_expect_tx(&bars[0], (uint32_t)(C::kA + 3 * C::kW));
+      lg.begin(0);
       for (int b = 0; b < C::NB; ++b)
         tma_load_2d(Aimg + 2 * C::kA + b * kABlk, &tm_dG, b * 64, (int)(3 * p.n + r0), &bars[0]);
       for (int b = 0; b < 3 * C::NB; ++b) tma_load_2d(Wimg + b * C::kWBlk, &tm_Wh, b * 64, 0, &bars[0]);
@@ -476,6 +492,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       fence_after_sync();
       mma_gates_kmaj<D>(tmem + D, A, smem_u32(Wimg), idesc);
       mma_commit(&bars[2]);
+      lg.begin(2);
     }
     if (!ok) record_device_error(p.status, kErrTimeout);
   }
@@ -506,6 +523,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   fence_before_sync();
+  __syncthreads();
+  if (!ok && tid == 0) lg.drain(bars);  // give-up path: nothing issued is still in flight
   __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, kCols);
 }
@@ -561,12 +580,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
   for (int i = 0; i < CW / 8; ++i) drl[i] = 0.f;
   bool ok = true;
+  IssueLog<3> lg;  // thread 0's copies and MMAs, for the give-up path
   uint32_t it = 0, mm = 0;  // tiles done, dW_a commits done
   for (int t = blockIdx.x; t < p.tiles && ok; t += gridDim.x, ++it) {
     const int64_t r0 = (int64_t)t * kRows;
     if (tid == 0) {
       const uint32_t bytes = (uint32_t)(p.w * C::kA + (it == 0 ? C::kW : 0));
       mbar_expect_tx(&bars[0], bytes);
+      lg.begin(0);
       if (it == 0)
         for (int b = 0; b < C::NB; ++b) tma_load_2d(Wimg + b * C::kWBlk, &tm_Wa, b * 64, 0, &bars[0]);
       for (int k = 0; k < p.w; ++k)
@@ -579,6 +600,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int k = 0; k < p.w; ++k)
           mma_kmaj_mn<D>(tmem + k * D, smem_u32(Cimg + k * C::kA), smem_u32(Wimg), idesc, false);
         mma_commit(&bars[1]);
+        lg.begin(1);
       }
     }
     ok = __syncthreads_and(ok);
@@ -672,6 +694,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           mma_bf16(acc_w, desc_sw128(A + j * 2048, kABlk, 1024), desc_sw128(B + j * 2048, kABlk, 1024), idesc,
                    (it > 0 || k > 0 || j > 0) ? 1u : 0u);
         mma_commit(&bars[2]);
+        lg.begin(2);
       }
       if (!mbar_wait(&bars[2], mm & 1)) ok = false;
       ++mm;
@@ -704,6 +727,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   for (int c = tid; c < D; c += kThreads)
     p.dr_part[(int64_t)blockIdx.x * D + c] = ((drred[c] + drred[D + c]) + drred[2 * D + c]) + drred[3 * D + c];
+  if (!ok && tid == 0) lg.drain(bars);  // give-up path: nothing issued is still in flight
+  __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, tcols);
 }
 
