@@ -15,10 +15,11 @@
 // neighbour row is gathered once per row and multiplied by its count (deg_r(j) is still the
 // number of edges, the CSR row length).
 //
-// Mapping: one group of G lanes per row, each lane owning 16-byte slices of the feature row
+// Mapping: a group of G lanes per row, each lane owning 16-byte slices of the feature row
 // (G = d * sizeof(T) / 16, at most 32), gathers with 128-bit loads and eight neighbour rows in
-// flight, fp32 accumulation; the row kernels are persistent (one wave of blocks striding over
-// rows), and the backward one loads the next node's first indices while the current one gathers.
+// flight, fp32 accumulation.  The row kernels are persistent (one wave of blocks): the forward one
+// streams chunks of consecutive compact rows through their contiguous runs, the backward one loads
+// the next node's first indices while the current one gathers.
 // Rows above kHubDegree edges are split into kChunkEdges-edge chunks: a whole CTA reduces one
 // chunk (its groups interleave over the chunk's edges, then combine in group order) into an fp32
 // partial, runs of 64 partials are summed in order, and the row adds the run sums in order.
@@ -239,6 +240,134 @@ __global__ void __launch_bounds__(256) agg_chunks(const int32_t* __restrict__ pt
   }
 }
 
+// Forward rows, streamed: M[k] = mean over the neighbours of the k-th non-empty CSR row (row
+// mlist[k]; the count of such rows is read on the device).  A group of G lanes takes a chunk of CR
+// consecutive compact rows (lane l < CR holds row l's bounds and scale) and streams through the
+// chunk's runs, which are contiguous, in batches of eight gathered rows that cross row boundaries;
+// a row is written (divided by its edge count, the CSR row length) when its last run is added, so
+// the loads of a short row do not wait on those of the row before.  Each row's runs are added one
+// by one, in run order, into an fp32 accumulator that starts at 0.  The bounds of the next chunk
+// (and the rows of the one after) are loaded while a chunk streams.  Rows above kHubDegree runs take
+// their sum from the chunk partials.  Persistent: each group strides over chunks.
+template <typename T, int D>
+struct StreamShape {
+  static constexpr int G = AggShape<T, D>::G;
+  static constexpr int CR = G < 16 ? G : 16;  // rows per chunk
+};
+
+template <typename T, int D>
+__global__ void __launch_bounds__(256) agg_fwd_rows(const int32_t* __restrict__ ptr, const int32_t* __restrict__ col,
+                                                    const int32_t* __restrict__ cnt, const int32_t* __restrict__ eptr,
+                                                    const int32_t* __restrict__ mlist, const int32_t* __restrict__ nnz_p,
+                                                    const T* __restrict__ H, T* __restrict__ M,
+                                                    const int32_t* __restrict__ chunk_ofs,
+                                                    const float* __restrict__ partials) {
+  using S = AggShape<T, D>;
+  constexpr int G = S::G, CR = StreamShape<T, D>::CR;
+  constexpr int U = 8;
+  const int grp = threadIdx.x / G, lane = threadIdx.x % G;
+  const int gshift = (threadIdx.x & 31) / G * G;
+  const unsigned gmask = G == 32 ? 0xffffffffu : (((1u << G) - 1u) << gshift);
+  const int64_t nrows = *nnz_p;
+  const int64_t nchunks = (nrows + CR - 1) / CR;
+  const int64_t step = (int64_t)gridDim.x * S::kGroups;
+  const T* base = H + lane * S::kVec;
+  // CSR row of chunk ch's row `lane` (-1: none)
+  auto row_of = [&](int64_t ch) -> int {
+    const int64_t k = ch * CR + lane;
+    if (ch >= nchunks || lane >= CR || k >= nrows) return -1;
+    return __ldg(mlist + k);
+  };
+  auto bounds = [&](int row, int& rb, int& re, float& sc) {
+    rb = re = 0;
+    sc = 1.f;
+    if (row >= 0) {
+      rb = __ldg(ptr + row);
+      re = __ldg(ptr + row + 1);
+      sc = __fdiv_rn(1.0f, (float)(__ldg(eptr + row + 1) - __ldg(eptr + row)));
+    }
+  };
+  int64_t ch = (int64_t)blockIdx.x * S::kGroups + grp;
+  int row = row_of(ch), rb, re;
+  float sc;
+  bounds(row, rb, re, sc);
+  int nrow = row_of(ch + step);
+  for (; ch < nchunks; ch += step) {
+    const int64_t k0 = ch * CR;
+    const int nr = (int)min((int64_t)CR, nrows - k0);
+    // the next chunk's bounds (its rows were loaded a chunk ago) and the rows of the one after
+    int nrb, nre;
+    float nsc;
+    bounds(nrow, nrb, nre, nsc);
+    const int nnrow = row_of(ch + 2 * step);
+
+    const unsigned hubs = (__ballot_sync(gmask, lane < nr && re - rb > kHubDegree) >> gshift) & ((1u << CR) - 1u);
+    const int chunk_end = __shfl_sync(gmask, re, nr - 1, G);
+    int e = __shfl_sync(gmask, rb, 0, G);
+    int cur = 0;                              // row of the chunk being summed
+    int cend = __shfl_sync(gmask, re, 0, G);  // its last run + 1
+    float acc[S::F];
+#pragma unroll
+    for (int q = 0; q < S::F; ++q) acc[q] = 0.f;
+    // writes row cur and moves to the next row
+    auto flush = [&]() {
+      store_row<T, D>(M + (k0 + cur) * D, lane, acc, __shfl_sync(gmask, sc, cur, G));
+#pragma unroll
+      for (int q = 0; q < S::F; ++q) acc[q] = 0.f;
+      ++cur;
+      if (cur < nr) cend = __shfl_sync(gmask, re, cur, G);
+    };
+    while (cur < nr) {
+      if ((hubs >> cur) & 1u) {  // a hub row: the sum of its chunk partials
+        const int hrow = __shfl_sync(gmask, row, cur, G);
+        add_partials<T, D>(partials, chunk_ofs[hrow], chunk_ofs[hrow + 1], lane, acc);
+        e = cend;
+        flush();
+        continue;
+      }
+      if (e >= cend) {  // the row's runs are all added
+        flush();
+        continue;
+      }
+      // up to U runs from e on, stopping at the next hub row (whose runs are not gathered)
+      const unsigned later = hubs & ~((2u << cur) - 1u);
+      const int stop = later ? __shfl_sync(gmask, rb, __ffs(later) - 1, G) : chunk_end;
+      const int nb = min(U, stop - e);
+      int c[U];
+      float w[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        c[u] = u < nb ? __ldg(col + e + u) : -1;
+        w[u] = u < nb ? (float)__ldg(cnt + e + u) : 0.f;
+      }
+      uint4 x[U][S::V];
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+#pragma unroll
+        for (int v = 0; v < S::V; ++v)
+          x[u][v] = c[u] >= 0 ? ldg16(base + (int64_t)c[u] * D + v * S::G * S::kVec) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        if (u >= nb) break;
+        while (e + u >= cend) flush();  // run e + u belongs to a later row (not a hub: nb stops before)
+#pragma unroll
+        for (int v = 0; v < S::V; ++v) {
+          float f[S::kVec];
+          unpack(x[u][v], f, T());
+#pragma unroll
+          for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] = fmaf(w[u], f[q], acc[v * S::kVec + q]);
+        }
+      }
+      e += nb;
+    }
+    row = nrow;
+    rb = nrb;
+    re = nre;
+    sc = nsc;
+    nrow = nnrow;
+  }
+}
+
 // The backward node kernel runs a two-deep pipeline per group: while node i gathers, the first
 // kFirst runs of node i + step and the bounds of node i + 2 step are in flight, so a short
 // row's gathers are issued without waiting on an index load.  Indices past the row's end, and
@@ -280,57 +409,6 @@ __device__ __forceinline__ void gather_row(const int32_t* __restrict__ col, cons
     }
   }
   if (end - beg > kFirst) gather_sum<T, D, kBatchTail>(col, cnt, beg + kFirst, end, 1, 0, src, lane, acc);
-}
-
-// Forward rows: M[k] = mean over the neighbours of the k-th non-empty CSR row (row = mlist[k]):
-// the row's runs (column, multiplicity), divided by the row's edge count (the CSR row length).
-// Rows without in-edges are not stored (their M is 0; the projection reads them as zeros).
-// Persistent: each group strides over the compact rows and fetches the next row's bounds while it
-// gathers.
-template <typename T, int D>
-__global__ void __launch_bounds__(256) agg_fwd_rows(const int32_t* __restrict__ ptr, const int32_t* __restrict__ col,
-                                                    const int32_t* __restrict__ cnt,
-                                                    const int32_t* __restrict__ eptr, const int32_t* __restrict__ mlist,
-                                                    const int32_t* __restrict__ nnz_p, const T* __restrict__ H,
-                                                    T* __restrict__ M, const int32_t* __restrict__ chunk_ofs,
-                                                    const float* __restrict__ partials) {
-  using S = AggShape<T, D>;
-  const int grp = threadIdx.x / S::G, lane = threadIdx.x % S::G;
-  const int64_t step = (int64_t)gridDim.x * S::kGroups;
-  const int64_t nnz = *nnz_p;
-  int64_t k = (int64_t)blockIdx.x * S::kGroups + grp;
-  int row = 0, beg = 0, end = 0, deg = 0;
-  if (k < nnz) {
-    row = __ldg(mlist + k);
-    beg = __ldg(ptr + row);
-    end = __ldg(ptr + row + 1);
-    deg = __ldg(eptr + row + 1) - __ldg(eptr + row);
-  }
-  int nrow = k + step < nnz ? __ldg(mlist + k + step) : 0;
-  while (k < nnz) {
-    const int64_t nk = k + step;
-    int nbeg = 0, nend = 0, ndeg = 0, nnrow = 0;
-    if (nk < nnz) {
-      nbeg = __ldg(ptr + nrow);
-      nend = __ldg(ptr + nrow + 1);
-      ndeg = __ldg(eptr + nrow + 1) - __ldg(eptr + nrow);
-      if (nk + step < nnz) nnrow = __ldg(mlist + nk + step);
-    }
-    float acc[S::F];
-#pragma unroll
-    for (int q = 0; q < S::F; ++q) acc[q] = 0.f;
-    if (end - beg > kHubDegree)
-      add_partials<T, D>(partials, chunk_ofs[row], chunk_ofs[row + 1], lane, acc);
-    else
-      gather_sum<T, D, false>(col, cnt, beg, end, 1, 0, H, lane, acc);
-    store_row<T, D>(M + k * D, lane, acc, __fdiv_rn(1.0f, (float)deg));
-    k = nk;
-    row = nrow;
-    beg = nbeg;
-    end = nend;
-    deg = ndeg;
-    nrow = nnrow;
-  }
 }
 
 // Backward nodes: dH[i] = dY[i] + sum of the node's row in the node-major out-edge list (every
@@ -395,11 +473,11 @@ __global__ void __launch_bounds__(256, 4) agg_bwd_nodes(int64_t N, const int32_t
 // ---------------------------------------------------------------------------------------------
 // Persistent grids: as many 256-thread blocks as are resident at once (occupancy of the kernel).
 template <typename K>
-static hg_status persist_blocks(K kernel, int64_t* blocks) {
+static hg_status persist_blocks(K kernel, int64_t* blocks, size_t smem = 0) {
   int dev = 0, sms = 0, per_sm = 0;
   HG_CUDA(cudaGetDevice(&dev));
   HG_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
-  HG_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, 256, 0));
+  HG_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, 256, smem));
   *blocks = (int64_t)sms * std::max(1, per_sm);
   return HG_OK;
 }
@@ -416,10 +494,10 @@ static hg_status agg_fwd_t(const hg_graph* g, const void* H, void* M, float* par
                 (const int32_t*)g->agg_chunk_row, (const int32_t*)g->agg_chunk_ofs, g->csr_rows, partials));
   static int64_t pb = 0;
   if (pb == 0) HG_TRY(persist_blocks(agg_fwd_rows<T, D>, &pb));
+  const int64_t groups = ceil_div(g->csr_rows, StreamShape<T, D>::CR);  // chunks (the compact rows are fewer)
   return launch("agg_fwd_rows", agg_fwd_rows<T, D>,
-                dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(g->csr_rows, S::kGroups), pb))),
-                dim3(256),
-                0, s, (const int32_t*)g->agg_ptr, (const int32_t*)g->agg_col, (const int32_t*)g->agg_cnt,
+                dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(groups, S::kGroups), pb))), dim3(256), 0,
+                s, (const int32_t*)g->agg_ptr, (const int32_t*)g->agg_col, (const int32_t*)g->agg_cnt,
                 (const int32_t*)g->csr_ptr, (const int32_t*)g->mlist, (const int32_t*)(g->mbase + g->meta.num_rels),
                 (const T*)H, (T*)M, (const int32_t*)g->agg_chunk_ofs, (const float*)partials);
 }

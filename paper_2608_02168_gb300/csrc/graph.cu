@@ -27,8 +27,9 @@ namespace hg {
 // exclusive scan (int32), three phases: tile sums -> scan of tile sums (recursive) -> tile scan
 // ---------------------------------------------------------------------------------------------
 constexpr int kScanThreads = 256;
-constexpr int kScanItems = 8;
-constexpr int kScanTile = kScanThreads * kScanItems;
+constexpr int kScanSub = 4;                                            // 128-item sub-blocks per warp
+constexpr int kScanWarpItems = 128 * kScanSub;                         // a warp's contiguous segment
+constexpr int kScanTile = kScanThreads / 32 * kScanWarpItems;          // 4096 items per block
 
 __device__ __forceinline__ int warp_inclusive_scan(int v) {
   const int lane = threadIdx.x & 31;
@@ -40,56 +41,107 @@ __device__ __forceinline__ int warp_inclusive_scan(int v) {
   return v;
 }
 
-// Exclusive block scan of one value per thread; *total receives the block total.
-__device__ __forceinline__ int block_exclusive_scan(int v, int* total) {
-  __shared__ int warp_tot[33];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
-  int incl = warp_inclusive_scan(v);
-  if (lane == 31) warp_tot[warp] = incl;
-  __syncthreads();
-  if (warp == 0) {
-    int x = lane < nwarps ? warp_tot[lane] : 0;
-    int xi = warp_inclusive_scan(x);
-    if (lane < nwarps) warp_tot[lane] = xi - x;
-    if (lane == 31) warp_tot[32] = xi;
-  }
-  __syncthreads();
-  int r = warp_tot[warp] + incl - v;
-  *total = warp_tot[32];
-  __syncthreads();
+__device__ __forceinline__ int warp_sum_i(int v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Items i .. i + 3 (zero past n): one 16-byte load where the array is aligned and the four are in
+// range.  A warp's lanes cover 128 consecutive items per call, so every access is coalesced.
+__device__ __forceinline__ int4 scan_load4(const int32_t* in, int64_t i, int64_t n, bool vec) {
+  if (vec && i + 3 < n) return *reinterpret_cast<const int4*>(in + i);
+  int4 r;
+  r.x = i < n ? in[i] : 0;
+  r.y = i + 1 < n ? in[i + 1] : 0;
+  r.z = i + 2 < n ? in[i + 2] : 0;
+  r.w = i + 3 < n ? in[i + 3] : 0;
   return r;
 }
 
-__global__ void scan_tile_sums(const int32_t* __restrict__ in, int64_t n, int32_t* __restrict__ sums) {
-  const int64_t base = (int64_t)blockIdx.x * kScanTile + (int64_t)threadIdx.x * kScanItems;
-  int s = 0;
-#pragma unroll
-  for (int i = 0; i < kScanItems; ++i)
-    if (base + i < n) s += in[base + i];
-  int total;
-  block_exclusive_scan(s, &total);
-  if (threadIdx.x == 0) sums[blockIdx.x] = total;
+__device__ __forceinline__ void scan_store4(int32_t* out, int64_t i, int64_t n, int4 v, bool vec) {
+  if (vec && i + 3 < n) {
+    *reinterpret_cast<int4*>(out + i) = v;
+    return;
+  }
+  if (i < n) out[i] = v.x;
+  if (i + 1 < n) out[i + 1] = v.y;
+  if (i + 2 < n) out[i + 2] = v.z;
+  if (i + 3 < n) out[i + 3] = v.w;
 }
 
-// tile_off == nullptr: a single tile starting at 0.  Writes out[n] = grand total from the last tile.
-__global__ void scan_tiles(const int32_t* in, int32_t* out, int64_t n, const int32_t* __restrict__ tile_off) {
-  const int64_t base = (int64_t)blockIdx.x * kScanTile + (int64_t)threadIdx.x * kScanItems;
-  int v[kScanItems];
+// sums[tile] = sum of the tile's kScanTile items (warp w: items tile * kScanTile + w * 512 ..)
+__global__ void __launch_bounds__(kScanThreads) scan_tile_sums(const int32_t* __restrict__ in, int64_t n,
+                                                                int32_t* __restrict__ sums) {
+  __shared__ int wt[kScanThreads / 32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const bool vec = (reinterpret_cast<uintptr_t>(in) & 15) == 0;
+  const int64_t seg = (int64_t)blockIdx.x * kScanTile + (int64_t)warp * kScanWarpItems;
   int s = 0;
 #pragma unroll
-  for (int i = 0; i < kScanItems; ++i) {
-    v[i] = base + i < n ? in[base + i] : 0;
-    s += v[i];
+  for (int j = 0; j < kScanSub; ++j) {
+    const int4 v = scan_load4(in, seg + 128 * j + 4 * lane, n, vec);
+    s += v.x + v.y + v.z + v.w;
   }
-  int total;
-  int run = block_exclusive_scan(s, &total) + (tile_off ? tile_off[blockIdx.x] : 0);
+  s = warp_sum_i(s);
+  if (lane == 0) wt[warp] = s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int t = 0;
 #pragma unroll
-  for (int i = 0; i < kScanItems; ++i) {
-    if (base + i < n) out[base + i] = run;
-    run += v[i];
+    for (int w = 0; w < kScanThreads / 32; ++w) t += wt[w];
+    sums[blockIdx.x] = t;
   }
-  if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0)
-    out[n] = (tile_off ? tile_off[blockIdx.x] : 0) + total;
+}
+
+// Exclusive scan of one tile plus tile_off[tile] (nullptr: a single tile starting at 0); the last
+// tile also writes out[n] = the grand total.  out may equal in.
+__global__ void __launch_bounds__(kScanThreads) scan_tiles(const int32_t* in, int32_t* out, int64_t n,
+                                                            const int32_t* __restrict__ tile_off) {
+  __shared__ int wt[kScanThreads / 32 + 1];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const bool vec = ((reinterpret_cast<uintptr_t>(in) | reinterpret_cast<uintptr_t>(out)) & 15) == 0;
+  const int64_t seg = (int64_t)blockIdx.x * kScanTile + (int64_t)warp * kScanWarpItems;
+  int4 v[kScanSub];
+  int ls[kScanSub];
+  int s = 0;
+#pragma unroll
+  for (int j = 0; j < kScanSub; ++j) {
+    v[j] = scan_load4(in, seg + 128 * j + 4 * lane, n, vec);
+    ls[j] = v[j].x + v[j].y + v[j].z + v[j].w;
+    s += ls[j];
+  }
+  s = warp_sum_i(s);
+  if (lane == 0) wt[warp] = s;
+  __syncthreads();
+  if (threadIdx.x == 0) {  // exclusive prefix over the warps, block total last
+    int run = tile_off ? tile_off[blockIdx.x] : 0;
+#pragma unroll
+    for (int w = 0; w < kScanThreads / 32; ++w) {
+      const int t = wt[w];
+      wt[w] = run;
+      run += t;
+    }
+    wt[kScanThreads / 32] = run;
+  }
+  __syncthreads();
+  int carry = wt[warp];
+#pragma unroll
+  for (int j = 0; j < kScanSub; ++j) {
+    const int incl = warp_inclusive_scan(ls[j]);
+    int run = carry + incl - ls[j];
+    int4 o;
+    o.x = run;
+    run += v[j].x;
+    o.y = run;
+    run += v[j].y;
+    o.z = run;
+    run += v[j].z;
+    o.w = run;
+    scan_store4(out, seg + 128 * j + 4 * lane, n, o, vec);
+    carry += __shfl_sync(0xffffffffu, incl, 31);
+  }
+  if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0) out[n] = wt[kScanThreads / 32];
 }
 
 size_t scan_scratch_bytes(int64_t n) {
