@@ -27,6 +27,7 @@
 #include <algorithm>
 
 #include "layer_kernels.cuh"
+#include "tc_util.cuh"
 
 namespace hg {
 
@@ -205,8 +206,24 @@ __device__ __forceinline__ void store_row(T* __restrict__ dst, int lane, const f
   }
 }
 
-// One CTA per chunk of kChunkEdges runs (grid-stride over the chunk list): fp32 partial sum of the
-// chunk's rows, each times its multiplicity.
+// Hub chunks: one CTA per chunk of kChunkEdges runs (grid-stride over the chunk list), fp32 partial
+// sum of the chunk's rows, each times its multiplicity.  The chunk's run entries are copied to
+// shared memory (cp.async) while the CTA sums the chunk before.  Group g sums runs g, g + kGroups,
+// ... in order: each lane copies its 16-byte slices of eight gathered rows per stage into its own
+// slots of a two-stage ring in shared memory (cp.async, so rows in flight hold no registers and no
+// lane waits on another), and adds a stage while the next one lands.  The groups' sums are then
+// added in group order (16-byte shared stores, the row stages reused).
+template <typename T, int D>
+struct ChunkCfg {
+  using S = AggShape<T, D>;
+  static constexpr int kRows = 8;  // gathered rows per stage and group
+  static constexpr int kStageBytes = kRows * D * (int)sizeof(T);
+  static constexpr int kRingBytes = S::kGroups * 2 * kStageBytes;  // also holds the groups' fp32 sums
+  static_assert(S::kGroups * D * 4 <= kRingBytes, "reduction buffer");
+  static constexpr int kIdxBytes = 2 * 2 * kChunkEdges * 4;  // column and count, two chunks
+  static constexpr int kSmem = kRingBytes + kIdxBytes;
+};
+
 template <typename T, int D>
 __global__ void __launch_bounds__(256) agg_chunks(const int32_t* __restrict__ ptr, const int32_t* __restrict__ col,
                                                   const int32_t* __restrict__ cnt,
@@ -214,30 +231,103 @@ __global__ void __launch_bounds__(256) agg_chunks(const int32_t* __restrict__ pt
                                                   const int32_t* __restrict__ chunk_ofs, int64_t rows,
                                                   float* __restrict__ partials) {
   using S = AggShape<T, D>;
-  __shared__ float red[S::kGroups][D];
+  using C = ChunkCfg<T, D>;
+  extern __shared__ uint4 chunk_smem[];
+  uint8_t* ring = reinterpret_cast<uint8_t*>(chunk_smem);
+  int32_t* sidx = reinterpret_cast<int32_t*>(ring + C::kRingBytes);  // [2][col | cnt][kChunkEdges]
+  float* red = reinterpret_cast<float*>(ring);                        // [kGroups][D], after the sums
   const int grp = threadIdx.x / S::G, lane = threadIdx.x % S::G;
   const int nchunks = chunk_ofs[rows];
-  for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
+  // runs [beg, end) of chunk c
+  auto span = [&](int c, int64_t& beg, int64_t& end) {
     const int row = chunk_row[c];
-    const int64_t beg = (int64_t)ptr[row] + (int64_t)(c - chunk_ofs[row]) * kChunkEdges;
-    const int64_t end = min((int64_t)ptr[row + 1], beg + kChunkEdges);
+    beg = (int64_t)ptr[row] + (int64_t)(c - chunk_ofs[row]) * kChunkEdges;
+    end = min((int64_t)ptr[row + 1], beg + kChunkEdges);
+  };
+  auto load_idx = [&](int c, int buf) {  // every thread: a few entries of chunk c's runs
+    int64_t b, e;
+    span(c, b, e);
+    int32_t* d = sidx + buf * 2 * kChunkEdges;
+    for (int k = threadIdx.x; k < e - b; k += blockDim.x) {
+      tc::cp_async4(d + k, col + b + k);
+      tc::cp_async4(d + kChunkEdges + k, cnt + b + k);
+    }
+  };
+  uint8_t* myring = ring + grp * 2 * C::kStageBytes;
+  if (blockIdx.x < nchunks) load_idx(blockIdx.x, 0);
+  tc::cp_async_commit();
+  int it = 0;
+  for (int c = blockIdx.x; c < nchunks; c += gridDim.x, ++it) {
+    const int buf = it & 1;
+    int64_t beg, end;
+    span(c, beg, end);
+    const int n = (int)(end - beg);
+    if (c + (int)gridDim.x < nchunks) load_idx(c + gridDim.x, buf ^ 1);  // the next chunk's runs
+    tc::cp_async_commit();
+    tc::cp_async_wait<1>();  // this chunk's run entries (this thread's copies) ...
+    __syncthreads();         // ... and every thread's
+    const int32_t* scol = sidx + buf * 2 * kChunkEdges;
+    const int32_t* scnt = scol + kChunkEdges;
+    const int mine = grp < n ? (n - grp + S::kGroups - 1) / S::kGroups : 0;  // runs of this group
+    const int nb = (mine + C::kRows - 1) / C::kRows;
+    auto issue = [&](int b) {  // batch b into stage b & 1 (an empty commit past the last batch)
+      uint8_t* st = myring + (b & 1) * C::kStageBytes;
+#pragma unroll
+      for (int u = 0; u < C::kRows; ++u) {
+        const int j = b * C::kRows + u;
+        if (j < mine) {
+          const int cidx = scol[grp + j * S::kGroups];
+#pragma unroll
+          for (int v = 0; v < S::V; ++v) {
+            const int o = (lane + v * S::G) * S::kVec;
+            tc::cp_async16(st + u * D * (int)sizeof(T) + o * (int)sizeof(T), src + (int64_t)cidx * D + o, true);
+          }
+        }
+      }
+      tc::cp_async_commit();
+    };
     float acc[S::F];
 #pragma unroll
     for (int q = 0; q < S::F; ++q) acc[q] = 0.f;
-    gather_sum<T, D, false>(col, cnt, beg + grp, end, S::kGroups, 0, src, lane, acc);
+    issue(0);
+    for (int b = 0; b < nb; ++b) {
+      issue(b + 1);
+      tc::cp_async_wait<1>();  // batch b (this lane's slices) has landed
+      const uint8_t* st = myring + (b & 1) * C::kStageBytes;
+#pragma unroll
+      for (int u = 0; u < C::kRows; ++u) {
+        const int j = b * C::kRows + u;
+        if (j >= mine) break;
+        const float w = (float)scnt[grp + j * S::kGroups];
+#pragma unroll
+        for (int v = 0; v < S::V; ++v) {
+          const int o = (lane + v * S::G) * S::kVec;
+          float f[S::kVec];
+          unpack(*reinterpret_cast<const uint4*>(st + u * D * (int)sizeof(T) + o * (int)sizeof(T)), f, T());
+#pragma unroll
+          for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] = fmaf(w, f[q], acc[v * S::kVec + q]);
+        }
+      }
+    }
+    tc::cp_async_wait<0>();
+    __syncthreads();  // every group is done with its ring: it becomes the reduction buffer
 #pragma unroll
     for (int v = 0; v < S::V; ++v)
 #pragma unroll
-      for (int q = 0; q < S::kVec; ++q) red[grp][(lane + v * S::G) * S::kVec + q] = acc[v * S::kVec + q];
+      for (int q = 0; q < S::kVec; q += 4)
+        *reinterpret_cast<float4*>(red + grp * D + (lane + v * S::G) * S::kVec + q) =
+            make_float4(acc[v * S::kVec + q], acc[v * S::kVec + q + 1], acc[v * S::kVec + q + 2],
+                        acc[v * S::kVec + q + 3]);
     __syncthreads();
     for (int k = threadIdx.x; k < D; k += blockDim.x) {
       float s = 0.f;
 #pragma unroll
-      for (int g = 0; g < S::kGroups; ++g) s += red[g][k];
+      for (int g = 0; g < S::kGroups; ++g) s += red[g * D + k];
       partials[(int64_t)c * D + k] = s;
     }
     __syncthreads();
   }
+  tc::cp_async_wait<0>();
 }
 
 // Forward rows, streamed: M[k] = mean over the neighbours of the k-th non-empty CSR row (row
@@ -484,10 +574,25 @@ static hg_status persist_blocks(K kernel, int64_t* blocks, size_t smem = 0) {
 
 static unsigned chunk_grid(int64_t cap) { return (unsigned)std::max<int64_t>(1, std::min<int64_t>(cap, 152 * 8)); }
 
+// resident blocks of the hub-chunk kernel (its shared memory set up once)
+template <typename T, int D>
+static hg_status chunk_blocks(int64_t* blocks) {
+  static int64_t cb = 0;
+  if (cb == 0) {
+    HG_CUDA(cudaFuncSetAttribute(agg_chunks<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, ChunkCfg<T, D>::kSmem));
+    HG_TRY(persist_blocks(agg_chunks<T, D>, &cb, ChunkCfg<T, D>::kSmem));
+  }
+  *blocks = cb;
+  return HG_OK;
+}
+
 template <typename T, int D>
 static hg_status agg_fwd_t(const hg_graph* g, const void* H, void* M, float* partials, cudaStream_t s) {
   using S = AggShape<T, D>;
-  HG_TRY(launch("agg_fwd_chunks", agg_chunks<T, D>, dim3(chunk_grid(g->chunk_cap_csr)), dim3(256), 0, s,
+  int64_t cb = 0;
+  HG_TRY((chunk_blocks<T, D>(&cb)));
+  HG_TRY(launch("agg_fwd_chunks", agg_chunks<T, D>, dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(g->chunk_cap_csr, cb))), dim3(256),
+                ChunkCfg<T, D>::kSmem, s,
                 (const int32_t*)g->agg_ptr, (const int32_t*)g->agg_col, (const int32_t*)g->agg_cnt, (const T*)H,
                 (const int32_t*)g->agg_chunk_row, (const int32_t*)g->agg_chunk_ofs, g->csr_rows, partials));
   HG_TRY(launch("combine_chunk_partials", combine_chunk_partials<D>, dim3(chunk_grid(g->chunk_cap_csr)), dim3(D), 0, s,
@@ -506,8 +611,11 @@ template <typename T, int D>
 static hg_status agg_bwd_t(const hg_graph* g, const void* dMs, const void* dY, void* dH, float* partials,
                            cudaStream_t s) {
   using S = AggShape<T, D>;
+  int64_t cb = 0;
   const int64_t N = g->meta.type_off[g->meta.num_types];
-  HG_TRY(launch("agg_bwd_chunks", agg_chunks<T, D>, dim3(chunk_grid(g->chunk_cap_node)), dim3(256), 0, s,
+  HG_TRY((chunk_blocks<T, D>(&cb)));
+  HG_TRY(launch("agg_bwd_chunks", agg_chunks<T, D>, dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(g->chunk_cap_node, cb))), dim3(256),
+                ChunkCfg<T, D>::kSmem, s,
                 (const int32_t*)g->bagg_ptr, (const int32_t*)g->bagg_col, (const int32_t*)g->bagg_cnt, (const T*)dMs,
                 (const int32_t*)g->bagg_chunk_row, (const int32_t*)g->bagg_chunk_ofs, N, partials));
   HG_TRY(launch("combine_chunk_partials", combine_chunk_partials<D>, dim3(chunk_grid(g->chunk_cap_node)), dim3(D), 0,
