@@ -330,43 +330,130 @@ __global__ void __launch_bounds__(256) agg_chunks(const int32_t* __restrict__ pt
   tc::cp_async_wait<0>();
 }
 
-// Forward rows, streamed: M[k] = mean over the neighbours of the k-th non-empty CSR row (row
-// mlist[k]; the count of such rows is read on the device).  A group of G lanes takes a chunk of CR
-// consecutive compact rows (lane l < CR holds row l's bounds and scale) and streams through the
-// chunk's runs, which are contiguous, in batches of eight gathered rows that cross row boundaries;
-// a row is written (divided by its edge count, the CSR row length) when its last run is added, so
-// the loads of a short row do not wait on those of the row before.  Each row's runs are added one
-// by one, in run order, into an fp32 accumulator that starts at 0.  The bounds of the next chunk
-// (and the rows of the one after) are loaded while a chunk streams.  Rows above kHubDegree runs take
-// their sum from the chunk partials.  Persistent: each group strides over chunks.
+// A lane's share of a feature row held by a whole warp: E = D / 32 consecutive elements (4 to 32
+// bytes), loaded with one or two vector loads and widened to fp32.
 template <typename T, int D>
-struct StreamShape {
-  static constexpr int G = AggShape<T, D>::G;
-  static constexpr int CR = G < 16 ? G : 16;  // rows per chunk
+struct Slice {
+  static constexpr int E = D / 32;
+  static constexpr int kWords = E * (int)sizeof(T) / 4;  // 32-bit words
+  uint32_t w[kWords];
+  __device__ __forceinline__ void load(const T* p) {
+    if constexpr (kWords == 1) {
+      w[0] = __ldg(reinterpret_cast<const uint32_t*>(p));
+    } else if constexpr (kWords == 2) {
+      const uint2 v = __ldg(reinterpret_cast<const uint2*>(p));
+      w[0] = v.x;
+      w[1] = v.y;
+    } else {
+#pragma unroll
+      for (int i = 0; i < kWords / 4; ++i) {
+        const uint4 v = __ldg(reinterpret_cast<const uint4*>(p) + i);
+        w[4 * i] = v.x;
+        w[4 * i + 1] = v.y;
+        w[4 * i + 2] = v.z;
+        w[4 * i + 3] = v.w;
+      }
+    }
+  }
+  __device__ __forceinline__ void to_float(float* f) const {
+    if constexpr (sizeof(T) == 4) {
+#pragma unroll
+      for (int i = 0; i < E; ++i) f[i] = __uint_as_float(w[i]);
+    } else {
+#pragma unroll
+      for (int i = 0; i < kWords; ++i) {
+        f[2 * i] = __uint_as_float(w[i] << 16);
+        f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+      }
+    }
+  }
+  // v * scale rounded to T, stored at p
+  __device__ __forceinline__ static void store(T* p, const float* v, float scale) {
+    uint32_t o[kWords];
+    if constexpr (sizeof(T) == 4) {
+#pragma unroll
+      for (int i = 0; i < E; ++i) o[i] = __float_as_uint(v[i] * scale);
+    } else {
+#pragma unroll
+      for (int i = 0; i < kWords; ++i) {
+        __nv_bfloat162 h = __floats2bfloat162_rn(v[2 * i] * scale, v[2 * i + 1] * scale);
+        o[i] = *reinterpret_cast<uint32_t*>(&h);
+      }
+    }
+    if constexpr (kWords == 1) {
+      *reinterpret_cast<uint32_t*>(p) = o[0];
+    } else if constexpr (kWords == 2) {
+      *reinterpret_cast<uint2*>(p) = make_uint2(o[0], o[1]);
+    } else {
+#pragma unroll
+      for (int i = 0; i < kWords / 4; ++i)
+        reinterpret_cast<uint4*>(p)[i] = make_uint4(o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
+    }
+  }
 };
 
+// Row kernels, streamed (agg_fwd_rows, agg_bwd_nodes).  A warp takes a chunk of 16 consecutive rows
+// (lane l < 16 holds row l's bounds and scale; every lane owns D / 32 columns) and streams through
+// the chunk's runs, which are contiguous, in batches of eight gathered rows that cross row
+// boundaries; a row is written when its last run is added, so the loads of a short row do not wait
+// on those of the row before.  Each row's runs are added one by one, in run order, into an fp32
+// accumulator that starts at 0.  The bounds of the next chunk (and the rows of the one after) are
+// loaded while a chunk streams.  Rows above kHubDegree runs take their sum from the chunk partials.
+// Persistent, with dynamic work: chunk costs are heavy-tailed, so a warp claims blocks of kClaim
+// chunks from a counter (zeroed before the launch; the next block claimed a block ahead).
+//   forward  (kBwd = false): rows = the non-empty CSR rows in compact order (row mlist[k]; their
+//            count read on the device); M[k] = sum / deg (deg = the CSR row length, eptr).
+//   backward (kBwd = true):  rows = nodes 0 .. n - 1 of the node-major lists; dH[i] = sum + dY[i],
+//            the dY rows of the next chunk copied to shared memory (cp.async, each lane its own
+//            slices, two buffers) while a chunk streams.
+constexpr int kStreamRows = 16;  // rows per chunk
+constexpr int kClaim = 4;        // chunks per claim
+
 template <typename T, int D>
-__global__ void __launch_bounds__(256) agg_fwd_rows(const int32_t* __restrict__ ptr, const int32_t* __restrict__ col,
-                                                    const int32_t* __restrict__ cnt, const int32_t* __restrict__ eptr,
-                                                    const int32_t* __restrict__ mlist, const int32_t* __restrict__ nnz_p,
-                                                    const T* __restrict__ H, T* __restrict__ M,
-                                                    const int32_t* __restrict__ chunk_ofs,
-                                                    const float* __restrict__ partials) {
-  using S = AggShape<T, D>;
-  constexpr int G = S::G, CR = StreamShape<T, D>::CR;
-  constexpr int U = 8;
-  const int grp = threadIdx.x / G, lane = threadIdx.x % G;
-  const int gshift = (threadIdx.x & 31) / G * G;
-  const unsigned gmask = G == 32 ? 0xffffffffu : (((1u << G) - 1u) << gshift);
-  const int64_t nrows = *nnz_p;
+struct StreamCfg {
+  static constexpr int kFwdThreads = 256;
+  static constexpr int kBwdThreads = 128;
+  static constexpr int kYBytes = kBwdThreads / 32 * 2 * kStreamRows * D * (int)sizeof(T);  // backward dY buffers
+};
+
+template <typename T, int D, bool kBwd>
+__device__ __forceinline__ void stream_rows(const int32_t* __restrict__ ptr, const int32_t* __restrict__ col,
+                                            const int32_t* __restrict__ cnt, const int32_t* __restrict__ eptr,
+                                            const int32_t* __restrict__ mlist, int64_t nrows,
+                                            const T* __restrict__ src, const T* __restrict__ dY, T* __restrict__ out,
+                                            const int32_t* __restrict__ chunk_ofs, const float* __restrict__ partials,
+                                            int32_t* __restrict__ work, T* __restrict__ ysm) {
+  using SL = Slice<T, D>;
+  constexpr int E = SL::E, CR = kStreamRows, U = 8;
+  constexpr int kSliceBytes = E * (int)sizeof(T);
+  constexpr unsigned kAll = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
   const int64_t nchunks = (nrows + CR - 1) / CR;
-  const int64_t step = (int64_t)gridDim.x * S::kGroups;
-  const T* base = H + lane * S::kVec;
-  // CSR row of chunk ch's row `lane` (-1: none)
+  const T* base = src + lane * E;
+  T* ys = ysm + (size_t)(threadIdx.x >> 5) * 2 * CR * D;  // this warp's two dY buffers (backward)
+  // the warp's chunk sequence: blocks of kClaim chunks claimed from the counter by lane 0; the
+  // following block's claim is in flight while a block is processed
+  int claim_next = 0, j = 0;
+  int claim_cur = 0;
+  if (lane == 0) {
+    claim_cur = atomicAdd(work, 1);
+    claim_next = atomicAdd(work, 1);
+  }
+  int blk = __shfl_sync(kAll, claim_cur, 0);
+  auto take = [&]() -> int64_t {
+    const int64_t r = (int64_t)blk * kClaim + j;
+    if (++j == kClaim) {
+      j = 0;
+      blk = __shfl_sync(kAll, claim_next, 0);
+      if (lane == 0) claim_next = atomicAdd(work, 1);
+    }
+    return r;
+  };
+  // list row of chunk ch's row `lane` (-1: none)
   auto row_of = [&](int64_t ch) -> int {
     const int64_t k = ch * CR + lane;
     if (ch >= nchunks || lane >= CR || k >= nrows) return -1;
-    return __ldg(mlist + k);
+    return kBwd ? (int)k : __ldg(mlist + k);
   };
   auto bounds = [&](int row, int& rb, int& re, float& sc) {
     rb = re = 0;
@@ -374,79 +461,116 @@ __global__ void __launch_bounds__(256) agg_fwd_rows(const int32_t* __restrict__ 
     if (row >= 0) {
       rb = __ldg(ptr + row);
       re = __ldg(ptr + row + 1);
-      sc = __fdiv_rn(1.0f, (float)(__ldg(eptr + row + 1) - __ldg(eptr + row)));
+      if (!kBwd) sc = __fdiv_rn(1.0f, (float)(__ldg(eptr + row + 1) - __ldg(eptr + row)));
     }
   };
-  int64_t ch = (int64_t)blockIdx.x * S::kGroups + grp;
+  // backward: chunk ch's dY rows (this lane's slices) into buffer b; one commit group per call
+  auto stage_y = [&](int64_t ch, int b) {
+    if constexpr (kBwd) {
+      if (ch < nchunks) {
+        const int nr = (int)min((int64_t)CR, nrows - ch * CR);
+        for (int r = 0; r < nr; ++r) {
+          T* d = ys + (b * CR + r) * D + lane * E;
+          const T* g = dY + (ch * CR + r) * D + lane * E;
+          if constexpr (kSliceBytes == 4) {
+            tc::cp_async4(d, g);
+          } else if constexpr (kSliceBytes == 8) {
+            tc::cp_async8(d, g);
+          } else {
+#pragma unroll
+            for (int q = 0; q < kSliceBytes / 16; ++q) tc::cp_async16(d + q * (16 / (int)sizeof(T)), g + q * (16 / (int)sizeof(T)), true);
+          }
+        }
+      }
+      tc::cp_async_commit();
+    }
+  };
+  int64_t ch = take(), nch = take(), nnch = take();
   int row = row_of(ch), rb, re;
   float sc;
   bounds(row, rb, re, sc);
-  int nrow = row_of(ch + step);
-  for (; ch < nchunks; ch += step) {
+  int nrow = row_of(nch);
+  stage_y(ch, 0);
+  for (int it = 0; ch < nchunks; ch = nch, nch = nnch, nnch = take(), ++it) {
     const int64_t k0 = ch * CR;
     const int nr = (int)min((int64_t)CR, nrows - k0);
+    stage_y(nch, (it + 1) & 1);  // the next chunk's dY rows
     // the next chunk's bounds (its rows were loaded a chunk ago) and the rows of the one after
     int nrb, nre;
     float nsc;
     bounds(nrow, nrb, nre, nsc);
-    const int nnrow = row_of(ch + 2 * step);
+    const int nnrow = row_of(nnch);
 
-    const unsigned hubs = (__ballot_sync(gmask, lane < nr && re - rb > kHubDegree) >> gshift) & ((1u << CR) - 1u);
-    const int chunk_end = __shfl_sync(gmask, re, nr - 1, G);
-    int e = __shfl_sync(gmask, rb, 0, G);
-    int cur = 0;                              // row of the chunk being summed
-    int cend = __shfl_sync(gmask, re, 0, G);  // its last run + 1
-    float acc[S::F];
+    const unsigned hubs = __ballot_sync(kAll, lane < nr && re - rb > kHubDegree);
+    const int chunk_end = __shfl_sync(kAll, re, nr - 1);
+    int e = __shfl_sync(kAll, rb, 0);
+    int cur = 0;                          // row of the chunk being summed
+    int cend = __shfl_sync(kAll, re, 0);  // its last run + 1
+    bool ywait = kBwd;                    // this chunk's dY rows not yet waited for
+    const T* yb = ys + (it & 1) * CR * D + lane * E;
+    float acc[E];
 #pragma unroll
-    for (int q = 0; q < S::F; ++q) acc[q] = 0.f;
+    for (int q = 0; q < E; ++q) acc[q] = 0.f;
     // writes row cur and moves to the next row
     auto flush = [&]() {
-      store_row<T, D>(M + (k0 + cur) * D, lane, acc, __shfl_sync(gmask, sc, cur, G));
+      if constexpr (kBwd) {
+        if (ywait) {
+          tc::cp_async_wait<1>();  // all but the next chunk's copies
+          ywait = false;
+        }
+        SL y;
 #pragma unroll
-      for (int q = 0; q < S::F; ++q) acc[q] = 0.f;
+        for (int q = 0; q < SL::kWords; ++q) y.w[q] = reinterpret_cast<const uint32_t*>(yb + cur * D)[q];
+        float f[E];
+        y.to_float(f);
+#pragma unroll
+        for (int q = 0; q < E; ++q) acc[q] += f[q];
+      }
+      SL::store(out + (k0 + cur) * D + lane * E, acc, __shfl_sync(kAll, sc, cur));
+#pragma unroll
+      for (int q = 0; q < E; ++q) acc[q] = 0.f;
       ++cur;
-      if (cur < nr) cend = __shfl_sync(gmask, re, cur, G);
+      if (cur < nr) cend = __shfl_sync(kAll, re, cur);
     };
     while (cur < nr) {
-      if ((hubs >> cur) & 1u) {  // a hub row: the sum of its chunk partials
-        const int hrow = __shfl_sync(gmask, row, cur, G);
-        add_partials<T, D>(partials, chunk_ofs[hrow], chunk_ofs[hrow + 1], lane, acc);
+      if ((hubs >> cur) & 1u) {  // a hub row: the sum of its chunk partials, in chunk-run order
+        const int hrow = __shfl_sync(kAll, row, cur);
+        for (int c = chunk_ofs[hrow]; c < chunk_ofs[hrow + 1]; c += kPartRun) {
+          const float* p = partials + (int64_t)c * D + lane * E;
+#pragma unroll
+          for (int q = 0; q < E; ++q) acc[q] += p[q];
+        }
         e = cend;
         flush();
         continue;
       }
-      if (e >= cend) {  // the row's runs are all added
+      if (e >= cend) {  // the row's runs are all added (or it has none)
         flush();
         continue;
       }
       // up to U runs from e on, stopping at the next hub row (whose runs are not gathered)
       const unsigned later = hubs & ~((2u << cur) - 1u);
-      const int stop = later ? __shfl_sync(gmask, rb, __ffs(later) - 1, G) : chunk_end;
+      const int stop = later ? __shfl_sync(kAll, rb, __ffs(later) - 1) : chunk_end;
       const int nb = min(U, stop - e);
       int c[U];
       float w[U];
 #pragma unroll
       for (int u = 0; u < U; ++u) {
-        c[u] = u < nb ? __ldg(col + e + u) : -1;
+        c[u] = u < nb ? __ldg(col + e + u) : 0;
         w[u] = u < nb ? (float)__ldg(cnt + e + u) : 0.f;
       }
-      uint4 x[U][S::V];
+      SL x[U];
 #pragma unroll
       for (int u = 0; u < U; ++u)
-#pragma unroll
-        for (int v = 0; v < S::V; ++v)
-          x[u][v] = c[u] >= 0 ? ldg16(base + (int64_t)c[u] * D + v * S::G * S::kVec) : make_uint4(0, 0, 0, 0);
+        if (u < nb) x[u].load(base + (int64_t)c[u] * D);
 #pragma unroll
       for (int u = 0; u < U; ++u) {
         if (u >= nb) break;
         while (e + u >= cend) flush();  // run e + u belongs to a later row (not a hub: nb stops before)
+        float f[E];
+        x[u].to_float(f);
 #pragma unroll
-        for (int v = 0; v < S::V; ++v) {
-          float f[S::kVec];
-          unpack(x[u][v], f, T());
-#pragma unroll
-          for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] = fmaf(w[u], f[q], acc[v * S::kVec + q]);
-        }
+        for (int q = 0; q < E; ++q) acc[q] = fmaf(w[u], f[q], acc[q]);
       }
       e += nb;
     }
@@ -456,106 +580,27 @@ __global__ void __launch_bounds__(256) agg_fwd_rows(const int32_t* __restrict__ 
     sc = nsc;
     nrow = nnrow;
   }
+  if constexpr (kBwd) tc::cp_async_wait<0>();  // no copy outlives the kernel
 }
 
-// The backward node kernel runs a two-deep pipeline per group: while node i gathers, the first
-// kFirst runs of node i + step and the bounds of node i + 2 step are in flight, so a short
-// row's gathers are issued without waiting on an index load.  Indices past the row's end, and
-// those of a row that takes the chunk path, are -1.  (The forward row kernel keeps a plain scalar
-// loop over short rows: with the extra registers of the pipeline it ran slower.)
-constexpr int kFirst = 4;  // a node row averages 3-4 runs once parallel edges are coalesced
-
-__device__ __forceinline__ void load_first(const int32_t* __restrict__ col, int beg, int end, int* c) {
-  const bool small = end - beg <= kHubDegree;
-#pragma unroll
-  for (int u = 0; u < kFirst; ++u) c[u] = small && u < end - beg ? __ldg(col + beg + u) : -1;
-}
-
-// acc += the rows of the preloaded first indices c (in order), then the row's edges from
-// beg + kFirst on, so every row is still summed in edge order.
-template <typename T, int D, bool kBatchTail>
-__device__ __forceinline__ void gather_row(const int32_t* __restrict__ col, const int32_t* __restrict__ cnt, int beg,
-                                           int end, const int* c, const T* __restrict__ src, int lane, float* acc) {
-  using S = AggShape<T, D>;
-  const T* base = src + lane * S::kVec;
-  float w[kFirst];  // multiplicities: loaded beside the rows (they depend only on beg)
-#pragma unroll
-  for (int u = 0; u < kFirst; ++u) w[u] = c[u] >= 0 ? (float)__ldg(cnt + beg + u) : 0.f;
-  uint4 x[kFirst][S::V];
-#pragma unroll
-  for (int u = 0; u < kFirst; ++u)
-#pragma unroll
-    for (int v = 0; v < S::V; ++v)
-      x[u][v] = c[u] >= 0 ? ldg16(base + (int64_t)c[u] * D + v * S::G * S::kVec) : make_uint4(0, 0, 0, 0);
-#pragma unroll
-  for (int u = 0; u < kFirst; ++u) {
-    if (c[u] < 0) break;
-#pragma unroll
-    for (int v = 0; v < S::V; ++v) {
-      float f[S::kVec];
-      unpack(x[u][v], f, T());
-#pragma unroll
-      for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] = fmaf(w[u], f[q], acc[v * S::kVec + q]);
-    }
-  }
-  if (end - beg > kFirst) gather_sum<T, D, kBatchTail>(col, cnt, beg + kFirst, end, 1, 0, src, lane, acc);
-}
-
-// Backward nodes: dH[i] = dY[i] + sum of the node's row in the node-major out-edge list (every
-// relation leaving its type, relation by relation, each edge holding the dMs row it reads).
-// Persistent: each group strides over nodes (pipelined as above).
 template <typename T, int D>
-__global__ void __launch_bounds__(256, 4) agg_bwd_nodes(int64_t N, const int32_t* __restrict__ nptr,
-                                                     const int32_t* __restrict__ ncol,
-                                                     const int32_t* __restrict__ ncnt, const T* __restrict__ dMs,
-                                                     const T* __restrict__ dY, T* __restrict__ dH,
-                                                     const int32_t* __restrict__ chunk_ofs,
-                                                     const float* __restrict__ partials) {
-  using S = AggShape<T, D>;
-  const int grp = threadIdx.x / S::G, lane = threadIdx.x % S::G;
-  const int64_t step = (int64_t)gridDim.x * S::kGroups;
-  int64_t node = (int64_t)blockIdx.x * S::kGroups + grp;
-  int beg = 0, end = 0, nbeg = 0, nend = 0;
-  if (node < N) {
-    beg = __ldg(nptr + node);
-    end = __ldg(nptr + node + 1);
-  }
-  if (node + step < N) {
-    nbeg = __ldg(nptr + node + step);
-    nend = __ldg(nptr + node + step + 1);
-  }
-  int c[kFirst];
-  load_first(ncol, beg, end, c);
-  while (node < N) {
-    int cn[kFirst];
-    load_first(ncol, nbeg, nend, cn);
-    const int64_t node2 = node + 2 * step;
-    int b2 = 0, e2 = 0;
-    if (node2 < N) {
-      b2 = __ldg(nptr + node2);
-      e2 = __ldg(nptr + node2 + 1);
-    }
-    float acc[S::F];
-#pragma unroll
-    for (int v = 0; v < S::V; ++v) {
-      float f[S::kVec];
-      unpack(ldg16(dY + node * D + (lane + v * S::G) * S::kVec), f, T());
-#pragma unroll
-      for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] = f[q];
-    }
-    if (end - beg > kHubDegree)
-      add_partials<T, D>(partials, chunk_ofs[node], chunk_ofs[node + 1], lane, acc);
-    else
-      gather_row<T, D, true>(ncol, ncnt, beg, end, c, dMs, lane, acc);
-    store_row<T, D>(dH + node * D, lane, acc, 1.0f);
-    node += step;
-    beg = nbeg;
-    end = nend;
-    nbeg = b2;
-    nend = e2;
-#pragma unroll
-    for (int u = 0; u < kFirst; ++u) c[u] = cn[u];
-  }
+__global__ void __launch_bounds__(StreamCfg<T, D>::kFwdThreads) agg_fwd_rows(
+    const int32_t* __restrict__ ptr, const int32_t* __restrict__ col, const int32_t* __restrict__ cnt,
+    const int32_t* __restrict__ eptr, const int32_t* __restrict__ mlist, const int32_t* __restrict__ nnz_p,
+    const T* __restrict__ H, T* __restrict__ M, const int32_t* __restrict__ chunk_ofs,
+    const float* __restrict__ partials, int32_t* __restrict__ work) {
+  stream_rows<T, D, false>(ptr, col, cnt, eptr, mlist, (int64_t)*nnz_p, H, nullptr, M, chunk_ofs, partials, work,
+                           nullptr);
+}
+
+template <typename T, int D>
+__global__ void __launch_bounds__(StreamCfg<T, D>::kBwdThreads) agg_bwd_nodes(
+    int64_t N, const int32_t* __restrict__ nptr, const int32_t* __restrict__ ncol, const int32_t* __restrict__ ncnt,
+    const T* __restrict__ dMs, const T* __restrict__ dY, T* __restrict__ dH, const int32_t* __restrict__ chunk_ofs,
+    const float* __restrict__ partials, int32_t* __restrict__ work) {
+  extern __shared__ uint4 ysm_raw[];
+  stream_rows<T, D, true>(nptr, ncol, ncnt, nullptr, nullptr, N, dMs, dY, dH, chunk_ofs, partials, work,
+                          reinterpret_cast<T*>(ysm_raw));
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -563,11 +608,11 @@ __global__ void __launch_bounds__(256, 4) agg_bwd_nodes(int64_t N, const int32_t
 // ---------------------------------------------------------------------------------------------
 // Persistent grids: as many 256-thread blocks as are resident at once (occupancy of the kernel).
 template <typename K>
-static hg_status persist_blocks(K kernel, int64_t* blocks, size_t smem = 0) {
+static hg_status persist_blocks(K kernel, int64_t* blocks, size_t smem = 0, int threads = 256) {
   int dev = 0, sms = 0, per_sm = 0;
   HG_CUDA(cudaGetDevice(&dev));
   HG_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
-  HG_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, 256, smem));
+  HG_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, threads, smem));
   *blocks = (int64_t)sms * std::max(1, per_sm);
   return HG_OK;
 }
@@ -587,7 +632,8 @@ static hg_status chunk_blocks(int64_t* blocks) {
 }
 
 template <typename T, int D>
-static hg_status agg_fwd_t(const hg_graph* g, const void* H, void* M, float* partials, cudaStream_t s) {
+static hg_status agg_fwd_t(const hg_graph* g, const void* H, void* M, float* partials, int32_t* work,
+                           cudaStream_t s) {
   using S = AggShape<T, D>;
   int64_t cb = 0;
   HG_TRY((chunk_blocks<T, D>(&cb)));
@@ -597,20 +643,21 @@ static hg_status agg_fwd_t(const hg_graph* g, const void* H, void* M, float* par
                 (const int32_t*)g->agg_chunk_row, (const int32_t*)g->agg_chunk_ofs, g->csr_rows, partials));
   HG_TRY(launch("combine_chunk_partials", combine_chunk_partials<D>, dim3(chunk_grid(g->chunk_cap_csr)), dim3(D), 0, s,
                 (const int32_t*)g->agg_chunk_row, (const int32_t*)g->agg_chunk_ofs, g->csr_rows, partials));
+  constexpr int kT = StreamCfg<T, D>::kFwdThreads;
   static int64_t pb = 0;
-  if (pb == 0) HG_TRY(persist_blocks(agg_fwd_rows<T, D>, &pb));
-  const int64_t groups = ceil_div(g->csr_rows, StreamShape<T, D>::CR);  // chunks (the compact rows are fewer)
+  if (pb == 0) HG_TRY(persist_blocks(agg_fwd_rows<T, D>, &pb, 0, kT));
+  const int64_t chunks = ceil_div(g->csr_rows, kStreamRows);  // a warp per chunk (the compact rows are fewer)
+  HG_CUDA(cudaMemsetAsync(work, 0, sizeof(int32_t), s));
   return launch("agg_fwd_rows", agg_fwd_rows<T, D>,
-                dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(groups, S::kGroups), pb))), dim3(256), 0,
+                dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(chunks, kT / 32), pb))), dim3(kT), 0,
                 s, (const int32_t*)g->agg_ptr, (const int32_t*)g->agg_col, (const int32_t*)g->agg_cnt,
                 (const int32_t*)g->csr_ptr, (const int32_t*)g->mlist, (const int32_t*)(g->mbase + g->meta.num_rels),
-                (const T*)H, (T*)M, (const int32_t*)g->agg_chunk_ofs, (const float*)partials);
+                (const T*)H, (T*)M, (const int32_t*)g->agg_chunk_ofs, (const float*)partials, work);
 }
 
 template <typename T, int D>
 static hg_status agg_bwd_t(const hg_graph* g, const void* dMs, const void* dY, void* dH, float* partials,
-                           cudaStream_t s) {
-  using S = AggShape<T, D>;
+                           int32_t* work, cudaStream_t s) {
   int64_t cb = 0;
   const int64_t N = g->meta.type_off[g->meta.num_types];
   HG_TRY((chunk_blocks<T, D>(&cb)));
@@ -620,12 +667,19 @@ static hg_status agg_bwd_t(const hg_graph* g, const void* dMs, const void* dY, v
                 (const int32_t*)g->bagg_chunk_row, (const int32_t*)g->bagg_chunk_ofs, N, partials));
   HG_TRY(launch("combine_chunk_partials", combine_chunk_partials<D>, dim3(chunk_grid(g->chunk_cap_node)), dim3(D), 0,
                 s, (const int32_t*)g->bagg_chunk_row, (const int32_t*)g->bagg_chunk_ofs, N, partials));
+  constexpr int kT = StreamCfg<T, D>::kBwdThreads, kY = StreamCfg<T, D>::kYBytes;
   static int64_t pb = 0;
-  if (pb == 0) HG_TRY(persist_blocks(agg_bwd_nodes<T, D>, &pb));
+  if (pb == 0) {
+    HG_CUDA(cudaFuncSetAttribute(agg_bwd_nodes<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, kY));
+    HG_TRY(persist_blocks(agg_bwd_nodes<T, D>, &pb, kY, kT));
+  }
+  const int64_t chunks = ceil_div(N, kStreamRows);
+  HG_CUDA(cudaMemsetAsync(work + 1, 0, sizeof(int32_t), s));
   return launch("agg_bwd_nodes", agg_bwd_nodes<T, D>,
-                dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(N, S::kGroups), pb))), dim3(256), 0, s,
+                dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(chunks, kT / 32), pb))), dim3(kT), kY, s,
                 N, (const int32_t*)g->bagg_ptr, (const int32_t*)g->bagg_col, (const int32_t*)g->bagg_cnt,
-                (const T*)dMs, (const T*)dY, (T*)dH, (const int32_t*)g->bagg_chunk_ofs, (const float*)partials);
+                (const T*)dMs, (const T*)dY, (T*)dH, (const int32_t*)g->bagg_chunk_ofs, (const float*)partials,
+                work + 1);
 }
 
 #define HG_DISPATCH_TD(dtype, d, FN, ...)                                                   \
@@ -644,13 +698,13 @@ static hg_status agg_bwd_t(const hg_graph* g, const void* dMs, const void* dY, v
   } while (0)
 
 hg_status aggregate_forward(const hg_graph* g, hg_dtype dt, int d, const void* H, void* M, float* partials,
-                            cudaStream_t s) {
-  HG_DISPATCH_TD(dt, d, agg_fwd_t, g, H, M, partials, s);
+                            int32_t* work, cudaStream_t s) {
+  HG_DISPATCH_TD(dt, d, agg_fwd_t, g, H, M, partials, work, s);
 }
 
 hg_status aggregate_backward(const hg_graph* g, hg_dtype dt, int d, const void* dMs, const void* dY, void* dH,
-                             float* partials, cudaStream_t s) {
-  HG_DISPATCH_TD(dt, d, agg_bwd_t, g, dMs, dY, dH, partials, s);
+                             float* partials, int32_t* work, cudaStream_t s) {
+  HG_DISPATCH_TD(dt, d, agg_bwd_t, g, dMs, dY, dH, partials, work, s);
 }
 
 }  // namespace hg

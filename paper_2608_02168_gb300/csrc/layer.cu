@@ -86,6 +86,7 @@ void carve_layer(const hg_graph* g, int d, hg_dtype dt, void* saved, void* scrat
     L->Vt = s.take<char>(2 * m.num_rels * dd * b);
   }
   L->agg_part = k.take<float>((size_t)std::max(g->chunk_cap_csr, g->chunk_cap_node) * d);
+  L->work = k.take<int32_t>(64);
   L->dY = k.take<char>((size_t)N * d * b);
   L->dU = k.take<char>((size_t)N * d * b);
   if (!tc) L->dZ = k.take<char>((size_t)N * d * b);
@@ -237,7 +238,7 @@ extern "C" hg_status hg_layer_fwd(const hg_graph* graph, const hg_layer_params* 
   const int d = p->d;
   LayerLayout L;
   carve_layer(graph, d, p->dtype, saved, scratch, &L, nullptr, nullptr);
-  HG_TRY(aggregate_forward(graph, p->dtype, d, H_in, L.M, L.agg_part, s));
+  HG_TRY(aggregate_forward(graph, p->dtype, d, H_in, L.M, L.agg_part, L.work, s));
   return project_forward(graph, p, H_in, H_out, L, true, s);
 }
 
@@ -333,7 +334,7 @@ extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* 
   LayerLayout L;
   carve_layer(graph, p->d, p->dtype, const_cast<void*>(saved), scratch, &L, nullptr, nullptr);
   HG_TRY(project_backward(graph, p, H_in, dH_out, grads, L, true, true, s));
-  if (dH_in) HG_TRY(aggregate_backward(graph, p->dtype, p->d, L.dMs, L.dY, dH_in, L.agg_part, s));
+  if (dH_in) HG_TRY(aggregate_backward(graph, p->dtype, p->d, L.dMs, L.dY, dH_in, L.agg_part, L.work, s));
   return HG_OK;
 }
 

@@ -124,9 +124,10 @@ int wgrad_tc_splits(int64_t n, int d);
 int* device_status_ptr();  // device address of the library status word
 
 hg_status aggregate_forward(const hg_graph* g, hg_dtype dt, int d, const void* H, void* M, float* partials,
+                            int32_t* work,
                             cudaStream_t s);
 hg_status aggregate_backward(const hg_graph* g, hg_dtype dt, int d, const void* dMs, const void* dY, void* dH,
-                             float* partials, cudaStream_t s);
+                             float* partials, int32_t* work, cudaStream_t s);
 hg_status proj_forward(hg_dtype dt, int d, const FwdArgs& a, cudaStream_t s);
 hg_status proj_backward(hg_dtype dt, int d, const BwdArgs& a, cudaStream_t s);
 // out = X^T Y over rows [x0, x0 + n) of X and [y0, y0 + n) of Y; with xmap, X row x0 + k is
@@ -158,6 +159,7 @@ struct LayerLayout {
   void* V;        // saved (bf16 only): R x 2 x d x d fused weights W_r W_agg (hi, lo halves)
   void* Vt;       // saved (bf16 only): their transposes (same order)
   float* agg_part;  // scratch: chunk partials
+  int32_t* work;    // scratch: work counter of the forward row kernel (zeroed before each launch)
   void* dY;       // scratch: N x d
   void* dU;
   void* dZ;       // scratch (fp32 storage only)
