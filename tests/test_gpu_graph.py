@@ -143,3 +143,27 @@ def test_node_order_with_eight_relations_into_one_type():
     compare_node_order(hg, G, ref, offs, rels)
     mask = sum((ref[r]["deg"] > 0).astype(np.int64) << r for r in range(8))
     assert len(np.unique(mask)) > 200  # nearly every mask value occurs
+
+
+def test_25_bit_row_keys():
+    # three relations into a 6M-node type: 18M CSR rows and 18M CSC rows (25-bit keys, four radix
+    # passes each, the last on a 1-bit digit), 23-bit node ids; bit-exact against the oracle on 2M
+    # random edges with parallel edges
+    need_gpu()
+    hg = lib()
+    n0 = 6_000_000
+    offs = np.array([0, n0, n0 + 100], np.int64)
+    rels = ((0, 0), (0, 0), (0, 0))
+    rng = np.random.default_rng(21)
+    E = 2_000_000
+    src = rng.integers(0, n0, E)
+    dst = np.minimum((rng.pareto(1.2, E) * 1000).astype(np.int64), n0 - 1)
+    rel = rng.integers(0, 3, E)
+    src[:50_000] = src[50_000:100_000]
+    dst[:50_000] = dst[50_000:100_000]
+    rel[:50_000] = rel[50_000:100_000]
+    G, bad = gpu_csr(hg, src, dst, rel, offs, rels)
+    assert bad == 0
+    ref = oracle.build_csr(src, dst, rel, offs, rels)
+    compare_layout(hg, G, ref, rels)
+    compare_node_order(hg, G, ref, offs, rels)
