@@ -471,19 +471,38 @@ __global__ void run_row_starts(const int32_t* __restrict__ ptr, int64_t rows, in
     if (ptr[r + 1] > ptr[r]) flag[ptr[r]] = 1;
 }
 
-// With u = the exclusive scan of the flags (u[n] = number of runs): run k = u[p] of a flagged
-// position p gets ucol[k] = col[p] (or map[col[p]] when a map is given) and its start upos[k] = p;
-// upos[U] = n.
-__global__ void run_write(const int32_t* __restrict__ flag, const int32_t* __restrict__ u,
-                          const int32_t* __restrict__ col, const int32_t* __restrict__ ptr, int64_t rows,
-                          const int32_t* __restrict__ map, int32_t* __restrict__ ucol, int32_t* __restrict__ upos) {
+// With u = the exclusive scan of the run-start flags (u[n] = number of runs): position p starts a
+// run exactly when u[p + 1] != u[p]; run k = u[p] gets ucol[k] = col[p] (or map[col[p]] when a map
+// is given) and its start upos[k] = p; upos[U] = n.  Four positions per thread, u read as 16-byte
+// vectors (the flags themselves are not read again).
+__global__ void run_write(const int32_t* __restrict__ u, const int32_t* __restrict__ col,
+                          const int32_t* __restrict__ ptr, int64_t rows, const int32_t* __restrict__ map,
+                          int32_t* __restrict__ ucol, int32_t* __restrict__ upos) {
   const int64_t n = ptr[rows];
-  for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p <= n; p += (int64_t)gridDim.x * blockDim.x) {
-    if (p == n) {
-      upos[u[n]] = (int32_t)n;
-    } else if (flag[p]) {
-      ucol[u[p]] = map ? map[col[p]] : col[p];
-      upos[u[p]] = (int32_t)p;
+  const bool vec = (reinterpret_cast<uintptr_t>(u) & 15) == 0;
+  for (int64_t p = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * 4; p <= n;
+       p += (int64_t)gridDim.x * blockDim.x * 4) {
+    int32_t v[5];
+    if (vec && p + 4 <= n) {
+      const int4 w = *reinterpret_cast<const int4*>(u + p);
+      v[0] = w.x;
+      v[1] = w.y;
+      v[2] = w.z;
+      v[3] = w.w;
+      v[4] = u[p + 4];
+    } else {
+#pragma unroll
+      for (int i = 0; i < 5; ++i) v[i] = p + i <= n ? u[p + i] : 0;
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int64_t q = p + i;
+      if (q < n && v[i + 1] != v[i]) {
+        ucol[v[i]] = map ? map[col[q]] : col[q];
+        upos[v[i]] = (int32_t)q;
+      } else if (q == n) {
+        upos[v[i]] = (int32_t)n;
+      }
     }
   }
 }
@@ -813,8 +832,8 @@ static hg_status coalesce_runs(const int32_t* col, const int32_t* ptr, int64_t r
   HG_TRY(launch("run_flags", run_flags, dim3(grid_for(E)), dim3(256), 0, s, col, ptr, rows, E, flag));
   HG_TRY(launch("run_row_starts", run_row_starts, dim3(grid_for(rows)), dim3(256), 0, s, ptr, rows, flag));
   HG_TRY(exclusive_scan(flag, u, E, L.sort.scan_scratch, s));
-  HG_TRY(launch("run_write", run_write, dim3(grid_for(E + 1)), dim3(256), 0, s, (const int32_t*)flag,
-                (const int32_t*)u, col, ptr, rows, map, ucol, upos));
+  HG_TRY(launch("run_write", run_write, dim3(grid_for(E / 4 + 1)), dim3(256), 0, s, (const int32_t*)u, col, ptr, rows,
+                map, ucol, upos));
   return launch("run_finish", run_finish, dim3(grid_for(std::max(E, rows + 1))), dim3(256), 0, s, (const int32_t*)u,
                 (const int32_t*)upos, ptr, rows, ucnt, uptr);
 }
