@@ -2,7 +2,7 @@
 // transpose for the backward pass.
 //
 // Forward:  M_r[j] = (1/deg_r(j)) * sum_{(i -> j) in r} H[i]          (CSR row j of relation r)
-// Backward: dH[i]  = dY[i] + sum_r sum_{(i -> j) in r} dMs_r[j]
+// Backward: dH[i]  = sum_r sum_{(i -> j) in r} dMs_r[j] + dY[i]
 //           where dMs_r[j] = dM_r[j] / deg_r(j) is produced, already scaled, by the projection
 //           backward kernel, and dY[i] is the residual-path gradient of Eq. 11.  The sum runs over
 //           node i's row of the node-major out-edge list (its CSC rows of every relation leaving
@@ -15,15 +15,14 @@
 // neighbour row is gathered once per row and multiplied by its count (deg_r(j) is still the
 // number of edges, the CSR row length).
 //
-// Mapping: a group of G lanes per row, each lane owning 16-byte slices of the feature row
-// (G = d * sizeof(T) / 16, at most 32), gathers with 128-bit loads and eight neighbour rows in
-// flight, fp32 accumulation.  The row kernels are persistent (one wave of blocks): the forward one
-// streams chunks of consecutive compact rows through their contiguous runs, the backward one loads
-// the next node's first indices while the current one gathers.
-// Rows above kHubDegree edges are split into kChunkEdges-edge chunks: a whole CTA reduces one
-// chunk (its groups interleave over the chunk's edges, then combine in group order) into an fp32
-// partial, runs of 64 partials are summed in order, and the row adds the run sums in order.
-// Every sum has a fixed order, so results are bitwise reproducible run to run.
+// Mapping: the row kernels (agg_fwd_rows, agg_bwd_nodes) give a warp chunks of 16 consecutive
+// rows, each lane owning d / 32 columns, and stream through the chunks' contiguous runs with eight
+// gathered rows in flight (fp32 accumulation); chunks are claimed dynamically.  Rows above
+// kHubDegree runs are split into kChunkEdges-run chunks: a whole CTA reduces one chunk (groups of
+// d * sizeof(T) / 16 lanes interleave over the chunk's runs, gathering into shared memory by
+// cp.async, then combine in group order) into an fp32 partial, runs of 64 partials are summed in
+// order, and the row adds the run sums in order.  Every sum has a fixed order, so results are
+// bitwise reproducible run to run.
 #include <algorithm>
 
 #include "layer_kernels.cuh"
@@ -42,129 +41,10 @@ struct AggShape {
   static constexpr int kGroups = kThreads / G;
 };
 
-// acc += sum of cnt[e] * src[col[e] + delta] for e = beg, beg + stride, ... < end, added in run
-// order; eight neighbour rows are loaded before they are added.
-template <typename T, int D, bool kBatchTail = true>
-__device__ __forceinline__ void gather_sum(const int32_t* __restrict__ col, const int32_t* __restrict__ cnt,
-                                           int64_t beg, int64_t end, int stride, int64_t delta,
-                                           const T* __restrict__ src, int lane, float* acc) {
-  using S = AggShape<T, D>;
-  constexpr int U = 8;
-  const T* base = src + delta * D + lane * S::kVec;
-  int64_t e = beg;
-  for (; e + (U - 1) * (int64_t)stride < end; e += U * (int64_t)stride) {
-    int c[U];
-    float w[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      c[u] = __ldg(col + e + u * stride);
-      w[u] = (float)__ldg(cnt + e + u * stride);
-    }
-    uint4 x[U][S::V];
-#pragma unroll
-    for (int u = 0; u < U; ++u)
-#pragma unroll
-      for (int v = 0; v < S::V; ++v) x[u][v] = ldg16(base + (int64_t)c[u] * D + v * S::G * S::kVec);
-#pragma unroll
-    for (int u = 0; u < U; ++u)
-#pragma unroll
-      for (int v = 0; v < S::V; ++v) {
-        float f[S::kVec];
-        unpack(x[u][v], f, T());
-#pragma unroll
-        for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] = fmaf(w[u], f[q], acc[v * S::kVec + q]);
-      }
-  }
-  if (!kBatchTail) {
-    for (; e < end; e += stride) {
-      const int c = __ldg(col + e);
-      const float w = (float)__ldg(cnt + e);
-#pragma unroll
-      for (int v = 0; v < S::V; ++v) {
-        float f[S::kVec];
-        unpack(ldg16(base + (int64_t)c * D + v * S::G * S::kVec), f, T());
-#pragma unroll
-        for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] = fmaf(w, f[q], acc[v * S::kVec + q]);
-      }
-    }
-  } else if (e < end) {  // the last (fewer than U) rows as one predicated batch
-    int c[U];
-    float w[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const bool in = e + u * (int64_t)stride < end;
-      c[u] = in ? __ldg(col + e + u * stride) : -1;
-      w[u] = in ? (float)__ldg(cnt + e + u * stride) : 0.f;
-    }
-    uint4 x[U][S::V];
-#pragma unroll
-    for (int u = 0; u < U; ++u)
-#pragma unroll
-      for (int v = 0; v < S::V; ++v)
-        x[u][v] = c[u] >= 0 ? ldg16(base + (int64_t)c[u] * D + v * S::G * S::kVec) : make_uint4(0, 0, 0, 0);
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      if (c[u] < 0) break;
-#pragma unroll
-      for (int v = 0; v < S::V; ++v) {
-        float f[S::kVec];
-        unpack(x[u][v], f, T());
-#pragma unroll
-        for (int q = 0; q < S::kVec; ++q) acc[v * S::kVec + q] = fmaf(w[u], f[q], acc[v * S::kVec + q]);
-      }
-    }
-  }
-}
-
 // Chunk partials are combined in two fixed-order levels: combine_chunk_partials sums every run of
 // kPartRun consecutive chunks of a row into the run's first slot, and a row then adds its run
 // sums in order (eight loads in flight).
 constexpr int kPartRun = 64;
-
-template <typename T, int D>
-__device__ __forceinline__ void add_partials(const float* __restrict__ partials, int c0, int c1, int lane,
-                                             float* acc) {
-  using S = AggShape<T, D>;
-  constexpr int U = 8;
-  int c = c0;
-  for (; c + (U - 1) * kPartRun < c1; c += U * kPartRun) {
-    float4 x[U][S::V][S::kVec / 4];
-#pragma unroll
-    for (int u = 0; u < U; ++u)
-#pragma unroll
-      for (int v = 0; v < S::V; ++v) {
-        const float4* p = reinterpret_cast<const float4*>(partials + (int64_t)(c + u * kPartRun) * D +
-                                                          (lane + v * S::G) * S::kVec);
-#pragma unroll
-        for (int q = 0; q < S::kVec / 4; ++q) x[u][v][q] = p[q];
-      }
-#pragma unroll
-    for (int u = 0; u < U; ++u)
-#pragma unroll
-      for (int v = 0; v < S::V; ++v)
-#pragma unroll
-        for (int q = 0; q < S::kVec / 4; ++q) {
-          acc[v * S::kVec + 4 * q + 0] += x[u][v][q].x;
-          acc[v * S::kVec + 4 * q + 1] += x[u][v][q].y;
-          acc[v * S::kVec + 4 * q + 2] += x[u][v][q].z;
-          acc[v * S::kVec + 4 * q + 3] += x[u][v][q].w;
-        }
-  }
-  for (; c < c1; c += kPartRun) {
-#pragma unroll
-    for (int v = 0; v < S::V; ++v) {
-      const float4* p = reinterpret_cast<const float4*>(partials + (int64_t)c * D + (lane + v * S::G) * S::kVec);
-#pragma unroll
-      for (int q = 0; q < S::kVec / 4; ++q) {
-        float4 x = p[q];
-        acc[v * S::kVec + 4 * q + 0] += x.x;
-        acc[v * S::kVec + 4 * q + 1] += x.y;
-        acc[v * S::kVec + 4 * q + 2] += x.z;
-        acc[v * S::kVec + 4 * q + 3] += x.w;
-      }
-    }
-  }
-}
 
 // Sums each run of kPartRun consecutive chunk partials of a row, in order, into the run's first
 // slot (one block of d threads per run leader; grid-stride over the chunk list).
@@ -191,18 +71,6 @@ __global__ void __launch_bounds__(D) combine_chunk_partials(const int32_t* __res
     }
     for (; cc < c1; ++cc) s += partials[(int64_t)cc * D + k];
     partials[(int64_t)c * D + k] = s;
-  }
-}
-
-template <typename T, int D>
-__device__ __forceinline__ void store_row(T* __restrict__ dst, int lane, const float* acc, float scale) {
-  using S = AggShape<T, D>;
-#pragma unroll
-  for (int v = 0; v < S::V; ++v) {
-    float f[S::kVec];
-#pragma unroll
-    for (int q = 0; q < S::kVec; ++q) f[q] = acc[v * S::kVec + q] * scale;
-    st16(dst + (lane + v * S::G) * S::kVec, pack(f, T()));
   }
 }
 
