@@ -23,10 +23,12 @@
 // Backward:
 //   ln_act_bwd   (warp per row)  dY = LayerNorm backward, dU = dY act'(U); column partials of the
 //                                bias / gain / shift gradients
-//   proj_bwd_tc  (CTA per 128 rows)  dMs_r = (dU V_r^T) / deg_r   (A = dU by TMA, B = V_r chunks,
-//                                hi and lo halves)
-//   weight gradients: G_r = M_r^T dU (split-K GEMM, MN-major TMA operands), then
-//                     dW_r = G_r W_agg^T and dW_agg[t] = sum_{r -> t} W_r^T G_r (wgrad_finish).
+//   proj_bwd_tc  (persistent, jobs of 128 stored rows)  dMs_r = (dU V_r^T) / deg_r   (A = the rows'
+//                                dU gathered by TMA, B = V_r chunks, hi and lo halves)
+//   weight gradients: G_r = M_r^T dU over a relation's stored rows (wgrad_rows_tc: split-K, MN-major
+//                     operands copied by cp.async; wgrad_tc: the dense variant with TMA operands for
+//                     callers whose rows are all stored), then dW_r = G_r W_agg^T and
+//                     dW_agg[t] = sum_{r -> t} W_r^T G_r (wgrad_finish).
 //
 // Epilogue threads own one accumulator row each (warp w reads TMEM lanes 32 (w % 4) ..); one
 // thread issues the MMAs.  All waits are bounded (tc::kSpinLimit) and report through the library
