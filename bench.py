@@ -671,13 +671,15 @@ def measure_hgt(w: dict, steps: int, warmup: int, dev, with_cpu: bool) -> dict:
     rep = hg.hg_timing_report()
     tot = sum(ms for _, ms in rep.values()) or 1.0
     ms = statistics.median(times)
-    # no-reuse model per layer: the forward and the two backward edge passes each gather a 4-byte
-    # index and two rows per edge (K and V; K and V; Q' and dS), plus the dense rows (K, V, Q', S
-    # written and read, the projection's and the backward products' rows)
+    # no-reuse model per layer: the forward and the two backward edge passes each read a run entry
+    # (8 bytes: column and multiplicity) and gather two rows per run of parallel edges (K and V; K
+    # and V; Q' and dS), plus the dense rows (K, V, Q', S written and read, the projection's and
+    # the backward products' rows)
     b = 4 if sp.dtype == "f32" else 2
     offs = [int(x) for x in g["type_offsets"]]
     RR = sum(offs[t + 1] - offs[t] for _, t in g["rels"])
-    per_layer = 3 * sp.num_edges * (4 + 2 * sp.d * b) + (2 * RR + 10 * sp.num_nodes) * sp.d * b
+    runs = int(torch.unique((g["rel"].long() * N + g["dst"].long()) * N + g["src"].long()).numel())
+    per_layer = 3 * runs * (8 + 2 * sp.d * b) + (2 * RR + 10 * sp.num_nodes) * sp.d * b
     peaks, psrc = load_peaks()
     ach = sp.layers * per_layer / (ms / 1e3) / 1e9
     res = {"workload": workload_desc(sp), "ms": round(ms, 4), "layers": sp.layers, "heads": HGT_HEADS,
@@ -685,7 +687,8 @@ def measure_hgt(w: dict, steps: int, warmup: int, dev, with_cpu: bool) -> dict:
            "roofline": {"bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
                         "peak_source": f"{psrc} hbm_gbs", "frac": round(ach / peaks["hbm_gbs"], 4),
                         "frac_of_nominal": round(ach / NOMINAL_HBM_GBS, 4),
-                        "model": "no-reuse: 3 edge passes x (4 + 2 d b) per edge + (2 csr_rows + 10 N) d b per layer",
+                        "model": "no-reuse: 3 edge passes x (8 + 2 d b) per run of parallel edges + (2 csr_rows + 10 N) d b per layer",
+                        "runs": runs,
                         "algorithmic_bytes_per_call": int(sp.layers * per_layer)},
            "kernel_time_share": {k: round(v / tot, 4) for k, (_, v) in sorted(rep.items(), key=lambda kv: -kv[1][1])},
            "cpu_baseline": None}

@@ -714,7 +714,7 @@ struct GraphLayout {
   int32_t *csr_ptr, *csr_col, *csr_eid, *csc_ptr, *csc_col, *csc_eid;
   float* csc_coef;
   int32_t *node_ptr, *node_col;  // node-major out-edges (dMs rows) for the backward aggregation
-  int32_t *csr_chunk_ofs, *csr_chunk_row, *node_chunk_ofs, *node_chunk_row, *invalid, *cnt;
+  int32_t *invalid, *cnt;
   // parallel edges coalesced: CSR rows and node-major rows as (column, multiplicity) runs
   int32_t *agg_ptr, *agg_col, *agg_cnt, *agg_chunk_ofs, *agg_chunk_row;
   int32_t *bagg_ptr, *bagg_col, *bagg_cnt, *bagg_chunk_ofs, *bagg_chunk_row;
@@ -735,10 +735,6 @@ static size_t carve_graph(void* ws, int64_t E, int64_t rows, int64_t crows, int6
   L->csc_coef = c.take<float>(Ea);
   L->node_ptr = c.take<int32_t>(N + 1);
   L->node_col = c.take<int32_t>(Ea);
-  L->csr_chunk_ofs = c.take<int32_t>(rows + 1);
-  L->csr_chunk_row = c.take<int32_t>(chunk_cap(E));
-  L->node_chunk_ofs = c.take<int32_t>(N + 1);
-  L->node_chunk_row = c.take<int32_t>(chunk_cap(E));
   L->agg_ptr = c.take<int32_t>(rows + 1);
   L->agg_col = c.take<int32_t>(Ea);
   L->agg_cnt = c.take<int32_t>(Ea);
@@ -971,9 +967,7 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
     HG_TRY(launch("order_tiles", order_tiles, dim3((unsigned)ceil_div(tiles * 32, 256)), dim3(256), 0, s,
                   (const int32_t*)L.csr_ptr, tr, n, (const int32_t*)perm, tiles, L.tmask + tile_base[t]));
   }
-  // chunk tables for rows above the hub degree: per edge (attention layer), per run (mean layer)
-  HG_TRY(chunk_table(L.csr_ptr, rows, L.csr_chunk_ofs, L.csr_chunk_row, L, s));
-  HG_TRY(chunk_table(L.node_ptr, N, L.node_chunk_ofs, L.node_chunk_row, L, s));
+  // chunk tables over runs for rows above the hub degree (mean and attention layers)
   HG_TRY(chunk_table(L.agg_ptr, rows, L.agg_chunk_ofs, L.agg_chunk_row, L, s));
   HG_TRY(chunk_table(L.bagg_ptr, N, L.bagg_chunk_ofs, L.bagg_chunk_row, L, s));
 
@@ -992,12 +986,8 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
   gh->csc_col = L.csc_col;
   gh->csc_eid = L.csc_eid;
   gh->csc_coef = L.csc_coef;
-  gh->csr_chunk_ofs = L.csr_chunk_ofs;
-  gh->csr_chunk_row = L.csr_chunk_row;
   gh->node_ptr = L.node_ptr;
   gh->node_col = L.node_col;
-  gh->node_chunk_ofs = L.node_chunk_ofs;
-  gh->node_chunk_row = L.node_chunk_row;
   gh->agg_ptr = L.agg_ptr;
   gh->agg_col = L.agg_col;
   gh->agg_cnt = L.agg_cnt;

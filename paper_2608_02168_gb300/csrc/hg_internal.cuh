@@ -122,15 +122,13 @@ struct hg_graph {
   int32_t* csc_col;
   int32_t* csc_eid;
   float* csc_coef;
-  int32_t* csr_chunk_ofs;  // [csr_rows + 1] exclusive scan of chunks per row (0 for rows <= hub degree)
-  int32_t* csr_chunk_row;  // [chunk_cap_csr] CSR row of each chunk
   int32_t* node_ptr;        // [N + 1] node-major out-edges over all relations (backward aggregation)
   int32_t* node_col;        // [num_edges] dMs row of each out-edge's destination
-  int32_t* node_chunk_ofs;  // [N + 1] chunks per node-major row above the hub degree
-  int32_t* node_chunk_row;
-  // Parallel edges coalesced (the mean layer's aggregation lists): the CSR rows as runs of equal
-  // source ids (agg_col = source, agg_cnt = multiplicity; deg = sum of the counts = CSR row length)
-  // and the node-major rows as runs of equal dMs rows; chunk tables over runs, as above.
+  // Parallel edges coalesced (the aggregation lists of the mean and attention layers): the CSR rows
+  // as runs of equal source ids (agg_col = source, agg_cnt = multiplicity; deg = sum of the counts =
+  // CSR row length) and the node-major rows as runs of equal dMs rows (bagg_col = the compact index
+  // of the target's CSR row); per-row chunk tables over runs for rows above kHubDegree runs
+  // (chunk_ofs: exclusive scan of chunks per row, chunk_row: the row of each chunk).
   int32_t* agg_ptr;         // [csr_rows + 1]
   int32_t* agg_col;         // [runs]
   int32_t* agg_cnt;

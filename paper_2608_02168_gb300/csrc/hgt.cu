@@ -185,14 +185,22 @@ struct HgtArgs {
   int8_t rslot[kMaxTypes][kMaxRels];  // relations into each type in relation order, -1 past the last
   int64_t N, csr_rows;
   int S;
-  const int32_t* csr_ptr;
-  const int32_t* csr_col;
-  const int32_t* csr_chunk_ofs;
-  const int32_t* csr_chunk_row;
-  const int32_t* node_ptr;
-  const int32_t* node_col;
-  const int32_t* node_chunk_ofs;
-  const int32_t* node_chunk_row;
+  // Edges as runs of parallel edges (column, multiplicity): a run's edges share their source, target
+  // and relation, so their scores, weights and gradients are equal and the run is taken once times
+  // its count.  Target side: each CSR row's runs by source (dptr / dcol / dcnt, hub chunks over
+  // runs); source side: each node's out-runs (sptr / scol / scnt), scol naming the target's CSR row
+  // through its compact index (the CSR row is mlist[scol]).
+  const int32_t* dptr;
+  const int32_t* dcol;
+  const int32_t* dcnt;
+  const int32_t* dchunk_ofs;
+  const int32_t* dchunk_row;
+  const int32_t* sptr;
+  const int32_t* scol;
+  const int32_t* scnt;
+  const int32_t* schunk_ofs;
+  const int32_t* schunk_row;
+  const int32_t* mlist;
   const void* KV;    // N x 2d: K then V of each node
   const void* Qp;    // csr_rows x d: relation-scaled queries
   void* Srows;       // csr_rows x d: attention-weighted value sums (forward output, backward input)
@@ -208,11 +216,11 @@ struct HgtArgs {
 constexpr int kBatch = 4;       // edges of a row in flight per warp (node kernels)
 constexpr int kBatchChunk = 4;  // the same for the chunk kernels (eight was slower: registers)
 
-// Online softmax step for one edge (per lane: its head's running maximum m and sum l; the value
-// accumulators are rescaled when the maximum grows).
+// Online softmax step for one run of w parallel edges (per lane: its head's running maximum m and
+// sum l; the value accumulators are rescaled when the maximum grows).
 template <int E, int NACC>
-__device__ __forceinline__ void online_step(float s, const float (&v)[E], float& m, float& l, float (&acc)[NACC][E],
-                                            int slot) {
+__device__ __forceinline__ void online_step(float s, float w, const float (&v)[E], float& m, float& l,
+                                            float (&acc)[NACC][E], int slot) {
   const float mn = fmaxf(m, s);
   if (mn > m) {
     const float so = expf(m - mn);
@@ -223,7 +231,7 @@ __device__ __forceinline__ void online_step(float s, const float (&v)[E], float&
       for (int e = 0; e < E; ++e) acc[k][e] *= so;
     m = mn;
   }
-  const float p = expf(s - m);
+  const float p = w * expf(s - m);  // w edges with this score
   l += p;
 #pragma unroll
   for (int k = 0; k < NACC; ++k)
@@ -241,8 +249,12 @@ __device__ __forceinline__ void fwd_edges(const HgtArgs& a, int64_t beg, int64_t
   const T* KV = (const T*)a.KV;
   for (int64_t e0 = beg; e0 < end; e0 += NB) {
     int src[NB];
+    float w[NB];
 #pragma unroll
-    for (int u = 0; u < NB; ++u) src[u] = e0 + u < end ? __ldg(a.csr_col + e0 + u) : -1;
+    for (int u = 0; u < NB; ++u) {
+      src[u] = e0 + u < end ? __ldg(a.dcol + e0 + u) : -1;
+      w[u] = e0 + u < end ? (float)__ldg(a.dcnt + e0 + u) : 0.f;
+    }
     float k[NB][E], v[NB][E];
 #pragma unroll
     for (int u = 0; u < NB; ++u) {
@@ -258,7 +270,7 @@ __device__ __forceinline__ void fwd_edges(const HgtArgs& a, int64_t beg, int64_t
 #pragma unroll
       for (int e = 0; e < E; ++e) s = fmaf(k[u][e], q[e], s);
       s = head_sum(s, lph);
-      online_step<E, NACC>(s, v[u], m, l, acc, slot);
+      online_step<E, NACC>(s, w[u], v[u], m, l, acc, slot);
     }
   }
 }
@@ -269,12 +281,12 @@ __global__ void __launch_bounds__(256) hgt_fwd_chunks(HgtArgs a) {
   constexpr int E = D / 32;
   const int lane = threadIdx.x & 31, lph = 32 / a.S;
   const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  const int nchunks = a.csr_chunk_ofs[a.csr_rows];
+  const int nchunks = a.dchunk_ofs[a.csr_rows];
   const int stride = 2 * a.S + D;
   for (int64_t c = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; c < nchunks; c += nw) {
-    const int row = a.csr_chunk_row[c];
-    const int64_t beg = (int64_t)a.csr_ptr[row] + (int64_t)(c - a.csr_chunk_ofs[row]) * kChunkEdges;
-    const int64_t end = min((int64_t)a.csr_ptr[row + 1], beg + kChunkEdges);
+    const int row = a.dchunk_row[c];
+    const int64_t beg = (int64_t)a.dptr[row] + (int64_t)(c - a.dchunk_ofs[row]) * kChunkEdges;
+    const int64_t end = min((int64_t)a.dptr[row + 1], beg + kChunkEdges);
     float q[E];
     load_slice<T, E>((const T*)a.Qp + (int64_t)row * D + lane * E, q);
     float m = -INFINITY, l = 0.f, acc[1][E];
@@ -312,10 +324,10 @@ __global__ void __launch_bounds__(256, (D <= 128 && KS <= 4) ? 3 : 1) hgt_fwd_no
     const int r = a.rslot[t][k];
     row[k] = r >= 0 ? a.meta.row_base[r] + jl : -1;
     if (row[k] >= 0) {
-      c0[k] = a.csr_chunk_ofs[row[k]];
-      c1[k] = a.csr_chunk_ofs[row[k] + 1];
-      e0[k] = a.csr_ptr[row[k]];
-      e1[k] = a.csr_ptr[row[k] + 1];
+      c0[k] = a.dchunk_ofs[row[k]];
+      c1[k] = a.dchunk_ofs[row[k] + 1];
+      e0[k] = a.dptr[row[k]];
+      e1[k] = a.dptr[row[k] + 1];
       load_slice<T, E>((const T*)a.Qp + row[k] * D + lane * E, q[k]);
     }
   }
@@ -406,8 +418,12 @@ __device__ __forceinline__ void dst_edges(const HgtArgs& a, int64_t beg, int64_t
   const T* KV = (const T*)a.KV;
   for (int64_t e0 = beg; e0 < end; e0 += NB) {
     int src[NB];
+    float w[NB];
 #pragma unroll
-    for (int u = 0; u < NB; ++u) src[u] = e0 + u < end ? __ldg(a.csr_col + e0 + u) : -1;
+    for (int u = 0; u < NB; ++u) {
+      src[u] = e0 + u < end ? __ldg(a.dcol + e0 + u) : -1;
+      w[u] = e0 + u < end ? (float)__ldg(a.dcnt + e0 + u) : 0.f;
+    }
     float k[NB][E], v[NB][E];
 #pragma unroll
     for (int u = 0; u < NB; ++u) {
@@ -428,7 +444,7 @@ __device__ __forceinline__ void dst_edges(const HgtArgs& a, int64_t beg, int64_t
       s = head_sum(s, lph);
       da = head_sum(da, lph);
       const float alpha = expf(s - m) * inv_l;
-      const float de = alpha * (da - Dh);
+      const float de = w[u] * alpha * (da - Dh);  // the run's w edges
 #pragma unroll
       for (int e = 0; e < E; ++e) acc[e] = fmaf(de, k[u][e], acc[e]);
     }
@@ -440,11 +456,11 @@ __global__ void __launch_bounds__(256) hgt_bwd_dst_chunks(HgtArgs a) {
   constexpr int E = D / 32;
   const int lane = threadIdx.x & 31, lph = 32 / a.S, h = lane / lph;
   const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  const int nchunks = a.csr_chunk_ofs[a.csr_rows];
+  const int nchunks = a.dchunk_ofs[a.csr_rows];
   for (int64_t c = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; c < nchunks; c += nw) {
-    const int row = a.csr_chunk_row[c];
-    const int64_t beg = (int64_t)a.csr_ptr[row] + (int64_t)(c - a.csr_chunk_ofs[row]) * kChunkEdges;
-    const int64_t end = min((int64_t)a.csr_ptr[row + 1], beg + kChunkEdges);
+    const int row = a.dchunk_row[c];
+    const int64_t beg = (int64_t)a.dptr[row] + (int64_t)(c - a.dchunk_ofs[row]) * kChunkEdges;
+    const int64_t end = min((int64_t)a.dptr[row + 1], beg + kChunkEdges);
     const float4 st = a.rstat[(int64_t)row * a.S + h];
     float q[E], g[E], acc[E];
     load_slice<T, E>((const T*)a.Qp + (int64_t)row * D + lane * E, q);
@@ -476,10 +492,10 @@ __global__ void __launch_bounds__(256, (D <= 128 && KS <= 4) ? 3 : 1) hgt_bwd_ds
     const int r = a.rslot[t][k];
     row[k] = r >= 0 ? a.meta.row_base[r] + jl : -1;
     if (row[k] >= 0) {
-      c0[k] = a.csr_chunk_ofs[row[k]];
-      c1[k] = a.csr_chunk_ofs[row[k] + 1];
-      e0[k] = a.csr_ptr[row[k]];
-      e1[k] = a.csr_ptr[row[k] + 1];
+      c0[k] = a.dchunk_ofs[row[k]];
+      c1[k] = a.dchunk_ofs[row[k] + 1];
+      e0[k] = a.dptr[row[k]];
+      e1[k] = a.dptr[row[k] + 1];
       load_slice<T, E>((const T*)a.Qp + row[k] * D + lane * E, q[k]);
       load_slice<T, E>((const T*)a.dS + row[k] * D + lane * E, g[k]);
     }
@@ -512,8 +528,12 @@ __device__ __forceinline__ void src_edges(const HgtArgs& a, int64_t beg, int64_t
   const int lane = threadIdx.x & 31, h = lane / lph;
   for (int64_t e0 = beg; e0 < end; e0 += NB) {
     int row[NB];
+    float w[NB];
 #pragma unroll
-    for (int u = 0; u < NB; ++u) row[u] = e0 + u < end ? __ldg(a.node_col + e0 + u) : -1;
+    for (int u = 0; u < NB; ++u) {
+      row[u] = e0 + u < end ? __ldg(a.mlist + __ldg(a.scol + e0 + u)) : -1;
+      w[u] = e0 + u < end ? (float)__ldg(a.scnt + e0 + u) : 0.f;
+    }
     float q[NB][E], g[NB][E];
     float4 st[NB];
 #pragma unroll
@@ -535,7 +555,7 @@ __device__ __forceinline__ void src_edges(const HgtArgs& a, int64_t beg, int64_t
       }
       s = head_sum(s, lph);
       da = head_sum(da, lph);
-      const float alpha = expf(s - st[u].x) * st[u].y;
+      const float alpha = w[u] * expf(s - st[u].x) * st[u].y;  // the run's w edges
       const float de = alpha * (da - st[u].z);
 #pragma unroll
       for (int e = 0; e < E; ++e) {
@@ -551,12 +571,12 @@ __global__ void __launch_bounds__(256) hgt_bwd_src_chunks(HgtArgs a) {
   constexpr int E = D / 32;
   const int lane = threadIdx.x & 31, lph = 32 / a.S;
   const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  const int nchunks = a.node_chunk_ofs[a.N];
+  const int nchunks = a.schunk_ofs[a.N];
   const T* KV = (const T*)a.KV;
   for (int64_t c = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; c < nchunks; c += nw) {
-    const int i = a.node_chunk_row[c];
-    const int64_t beg = (int64_t)a.node_ptr[i] + (int64_t)(c - a.node_chunk_ofs[i]) * kChunkEdges;
-    const int64_t end = min((int64_t)a.node_ptr[i + 1], beg + kChunkEdges);
+    const int i = a.schunk_row[c];
+    const int64_t beg = (int64_t)a.sptr[i] + (int64_t)(c - a.schunk_ofs[i]) * kChunkEdges;
+    const int64_t end = min((int64_t)a.sptr[i + 1], beg + kChunkEdges);
     float k[E], v[E], ak[E], av[E];
     load_slice<T, E>(KV + (int64_t)i * 2 * D + lane * E, k);
     load_slice<T, E>(KV + (int64_t)i * 2 * D + D + lane * E, v);
@@ -580,7 +600,7 @@ __global__ void __launch_bounds__(256) hgt_bwd_src_nodes(HgtArgs a) {
   float ak[E], av[E];
 #pragma unroll
   for (int e = 0; e < E; ++e) ak[e] = av[e] = 0.f;
-  const int c0 = a.node_chunk_ofs[i], c1 = a.node_chunk_ofs[i + 1];
+  const int c0 = a.schunk_ofs[i], c1 = a.schunk_ofs[i + 1];
   if (c1 > c0) {
     for (int c = c0; c < c1; ++c)
 #pragma unroll
@@ -593,7 +613,7 @@ __global__ void __launch_bounds__(256) hgt_bwd_src_nodes(HgtArgs a) {
     const T* KV = (const T*)a.KV;
     load_slice<T, E>(KV + i * 2 * D + lane * E, k);
     load_slice<T, E>(KV + i * 2 * D + D + lane * E, v);
-    src_edges<T, D>(a, a.node_ptr[i], a.node_ptr[i + 1], k, v, lph, ak, av);
+    src_edges<T, D>(a, a.sptr[i], a.sptr[i + 1], k, v, lph, ak, av);
   }
   store_slice<T, E>((T*)a.dK + i * D + lane * E, ak);
   store_slice<T, E>((T*)a.dV + i * D + lane * E, av);
@@ -730,14 +750,17 @@ HgtArgs edge_args(const hg_graph* g, const hg_hgt_params* p, const HgtLayout& H)
   a.N = g->meta.type_off[g->meta.num_types];
   a.csr_rows = g->csr_rows;
   a.S = p->heads;
-  a.csr_ptr = g->csr_ptr;
-  a.csr_col = g->csr_col;
-  a.csr_chunk_ofs = g->csr_chunk_ofs;
-  a.csr_chunk_row = g->csr_chunk_row;
-  a.node_ptr = g->node_ptr;
-  a.node_col = g->node_col;
-  a.node_chunk_ofs = g->node_chunk_ofs;
-  a.node_chunk_row = g->node_chunk_row;
+  a.dptr = g->agg_ptr;
+  a.dcol = g->agg_col;
+  a.dcnt = g->agg_cnt;
+  a.dchunk_ofs = g->agg_chunk_ofs;
+  a.dchunk_row = g->agg_chunk_row;
+  a.sptr = g->bagg_ptr;
+  a.scol = g->bagg_col;
+  a.scnt = g->bagg_cnt;
+  a.schunk_ofs = g->bagg_chunk_ofs;
+  a.schunk_row = g->bagg_chunk_row;
+  a.mlist = g->mlist;
   a.KV = H.KV;
   a.Qp = H.Qp;
   a.Srows = H.L.M;
