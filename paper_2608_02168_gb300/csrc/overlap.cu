@@ -131,7 +131,8 @@ __global__ void ob_h_small(const int32_t* __restrict__ ofs, const int32_t* __res
   }
 }
 
-// One CTA per node with a list longer than kBigList (grid-stride over all nodes, skipping others).
+// One CTA per node with a list longer than kBigList: the CTAs stride over tiles of kBigThreads
+// nodes, every thread testing one node, and take the tile's long lists one after another.
 // The h-index is the largest h with S(h) = #{degrees >= h} >= h.  Each pass bins the degrees over
 // [lo, hi] into at most kCap bins of width w (degrees above hi in the last bin, below lo dropped);
 // the suffix sums give S at every bin start, the largest bin start still satisfying S >= h brackets
@@ -146,86 +147,99 @@ __global__ void __launch_bounds__(kBigThreads) ob_h_big(const int32_t* __restric
   __shared__ int hist[kCap];
   __shared__ int part[kBigThreads / 32];
   __shared__ int best_s;
+  __shared__ int64_t tile_big[kBigThreads];  // the tile's nodes with long lists
+  __shared__ int tile_nbig;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int64_t v = blockIdx.x; v < N; v += gridDim.x) {
-    const int n = ofs[v + 1] - ofs[v];
-    if (n <= kBigList) continue;
-    const int32_t* nb = nbr + ofs[v];
-    int lo = 0, hi = n;  // S(lo) >= lo holds; the answer lies in [lo, hi]
-    while (true) {
-      const int span = hi - lo + 1;
-      int lw = 0;  // bin width 2^lw, the smallest giving at most kCap bins
-      while (((span + (1 << lw) - 1) >> lw) > kCap) ++lw;
-      const int w = 1 << lw;
-      const int nbins = (span + w - 1) >> lw;
-      for (int i = threadIdx.x; i < nbins; i += blockDim.x) hist[i] = 0;
-      if (threadIdx.x == 0) best_s = 0;
-      __syncthreads();
-      int reg[kRegBins] = {0, 0, 0, 0, 0, 0, 0, 0};
-      auto count = [&](int d) {
-        if (d < lo) return;
-        const int j = min((d - lo) >> lw, nbins - 1);
-        if (j < kRegBins) {
-#pragma unroll
-          for (int q = 0; q < kRegBins; ++q) reg[q] += j == q;
-        } else {
-          atomicAdd(&hist[j], 1);
-        }
-      };
-      int i = threadIdx.x;
-      for (; i + 3 * (int)blockDim.x < n; i += 4 * blockDim.x) {  // four loads in flight
-        const int d0 = nb[i], d1 = nb[i + blockDim.x], d2 = nb[i + 2 * blockDim.x], d3 = nb[i + 3 * blockDim.x];
-        count(d0);
-        count(d1);
-        count(d2);
-        count(d3);
-      }
-      for (; i < n; i += blockDim.x) count(nb[i]);
-#pragma unroll
-      for (int q = 0; q < kRegBins; ++q) {
-        int t = reg[q];
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-        if (lane == 0 && t && q < nbins) atomicAdd(&hist[q], t);
-      }
-      __syncthreads();
-      // suffix sums: thread j owns bins [blo, bhi) counted from the top
-      const int per = (nbins + blockDim.x - 1) / blockDim.x;
-      const int bhi = nbins - threadIdx.x * per, blo = max(0, bhi - per);
-      int own = 0;
-      for (int b = blo; b < bhi; ++b) own += hist[b];
-      int incl = own;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += y;
-      }
-      if (lane == 31) part[warp] = incl;
-      __syncthreads();
-      int run = incl - own;  // entries in higher bins of lower-numbered threads
-#pragma unroll
-      for (int ww = 0; ww < kBigThreads / 32; ++ww) run += ww < warp ? part[ww] : 0;
-      int found = -1;
-      for (int b = bhi - 1; b >= blo; --b) {  // S(lo + b w) from the top of the range down
-        run += hist[b];
-        if (run >= lo + b * w) {
-          found = b;
-          break;
-        }
-      }
-      if (found >= 0) atomicMax(&best_s, found);
-      __syncthreads();
-      const int j = best_s;  // bin 0 always qualifies (S(lo) >= lo)
-      __syncthreads();
-      if (w == 1) {
-        if (threadIdx.x == 0) h[v] = lo + j;
-        break;
-      }
-      const int nlo = lo + j * w;
-      hi = min(hi, nlo + w - 1);
-      lo = nlo;
+  for (int64_t t0 = (int64_t)blockIdx.x * kBigThreads; t0 < N; t0 += (int64_t)gridDim.x * kBigThreads) {
+    if (threadIdx.x == 0) tile_nbig = 0;
+    __syncthreads();
+    {
+      const int64_t u = t0 + threadIdx.x;
+      if (u < N && ofs[u + 1] - ofs[u] > kBigList) tile_big[atomicAdd(&tile_nbig, 1)] = u;
     }
     __syncthreads();
+    const int nbig = tile_nbig;
+    for (int ib = 0; ib < nbig; ++ib) {
+      const int64_t v = tile_big[ib];
+      const int n = ofs[v + 1] - ofs[v];
+      const int32_t* nb = nbr + ofs[v];
+      int lo = 0, hi = n;  // S(lo) >= lo holds; the answer lies in [lo, hi]
+      while (true) {
+        const int span = hi - lo + 1;
+        int lw = 0;  // bin width 2^lw, the smallest giving at most kCap bins
+        while (((span + (1 << lw) - 1) >> lw) > kCap) ++lw;
+        const int w = 1 << lw;
+        const int nbins = (span + w - 1) >> lw;
+        for (int i = threadIdx.x; i < nbins; i += blockDim.x) hist[i] = 0;
+        if (threadIdx.x == 0) best_s = 0;
+        __syncthreads();
+        int reg[kRegBins] = {0, 0, 0, 0, 0, 0, 0, 0};
+        auto count = [&](int d) {
+          if (d < lo) return;
+          const int j = min((d - lo) >> lw, nbins - 1);
+          if (j < kRegBins) {
+  #pragma unroll
+            for (int q = 0; q < kRegBins; ++q) reg[q] += j == q;
+          } else {
+            atomicAdd(&hist[j], 1);
+          }
+        };
+        int i = threadIdx.x;
+        for (; i + 3 * (int)blockDim.x < n; i += 4 * blockDim.x) {  // four loads in flight
+          const int d0 = nb[i], d1 = nb[i + blockDim.x], d2 = nb[i + 2 * blockDim.x], d3 = nb[i + 3 * blockDim.x];
+          count(d0);
+          count(d1);
+          count(d2);
+          count(d3);
+        }
+        for (; i < n; i += blockDim.x) count(nb[i]);
+  #pragma unroll
+        for (int q = 0; q < kRegBins; ++q) {
+          int t = reg[q];
+  #pragma unroll
+          for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+          if (lane == 0 && t && q < nbins) atomicAdd(&hist[q], t);
+        }
+        __syncthreads();
+        // suffix sums: thread j owns bins [blo, bhi) counted from the top
+        const int per = (nbins + blockDim.x - 1) / blockDim.x;
+        const int bhi = nbins - threadIdx.x * per, blo = max(0, bhi - per);
+        int own = 0;
+        for (int b = blo; b < bhi; ++b) own += hist[b];
+        int incl = own;
+  #pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int y = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += y;
+        }
+        if (lane == 31) part[warp] = incl;
+        __syncthreads();
+        int run = incl - own;  // entries in higher bins of lower-numbered threads
+  #pragma unroll
+        for (int ww = 0; ww < kBigThreads / 32; ++ww) run += ww < warp ? part[ww] : 0;
+        int found = -1;
+        for (int b = bhi - 1; b >= blo; --b) {  // S(lo + b w) from the top of the range down
+          run += hist[b];
+          if (run >= lo + b * w) {
+            found = b;
+            break;
+          }
+        }
+        if (found >= 0) atomicMax(&best_s, found);
+        __syncthreads();
+        const int j = best_s;  // bin 0 always qualifies (S(lo) >= lo)
+        __syncthreads();
+        if (w == 1) {
+          if (threadIdx.x == 0) h[v] = lo + j;
+          break;
+        }
+        const int nlo = lo + j * w;
+        hi = min(hi, nlo + w - 1);
+        lo = nlo;
+      }
+      __syncthreads();
+    }
+    __syncthreads();  // tile_big and tile_nbig are rewritten by the next tile
   }
 }
 
