@@ -333,9 +333,12 @@ constexpr size_t kScatterSmem = 3 * kSortTile * sizeof(uint32_t) + kSortWarps * 
 
 // Sorts (key, value, second payload) triples by the low `bits` key bits (at least one pass), stable.
 // The first pass reads keys_src, vals_src (null: the input positions) and vals2_src, which may lie
-// in buffer `start` (it writes buffer start ^ 1 first); returns the buffer index holding the result.
+// in buffer `start` (it writes buffer start ^ 1 first); returns the buffer index holding the sorted
+// keys.  The last pass writes the payloads to vals_final / vals2_final when those are given (the
+// caller's final arrays), else to the sort buffers beside the keys.
 static hg_status radix_sort(SortBuffers& b, int64_t n, int bits, const uint32_t* keys_src, const uint32_t* vals_src,
-                            const uint32_t* vals2_src, int start, cudaStream_t s, int* result) {
+                            const uint32_t* vals2_src, int start, cudaStream_t s, int* result,
+                            uint32_t* vals_final = nullptr, uint32_t* vals2_final = nullptr) {
   static bool attr = false;
   if (!attr) {
     HG_CUDA(cudaFuncSetAttribute(radix_scatter<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kScatterSmem));
@@ -346,15 +349,19 @@ static hg_status radix_sort(SortBuffers& b, int64_t n, int bits, const uint32_t*
   const uint32_t* k = keys_src;
   const uint32_t* v = vals_src;
   const uint32_t* v2 = vals2_src;
-  for (int shift = 0; shift < std::max(bits, 1); shift += 8) {
+  const int nb = std::max(bits, 1);
+  for (int shift = 0; shift < nb; shift += 8) {
+    const bool last = shift + 8 >= nb;
+    uint32_t* vo = last && vals_final ? vals_final : b.vals[cur ^ 1];
+    uint32_t* v2o = last && vals2_final ? vals2_final : b.vals2[cur ^ 1];
     HG_TRY(launch("radix_hist", radix_hist, dim3((unsigned)tiles), dim3(kSortThreads), 0, s, k, n, shift, b.hist,
                   tiles));
     HG_TRY(exclusive_scan(b.hist, b.hist, tiles * kRadix, b.scan_scratch, s));
     HG_TRY(launch("radix_scatter", radix_scatter<true>, dim3((unsigned)tiles), dim3(kSortThreads), kScatterSmem, s, k, v, v2,
-                  b.keys[cur ^ 1], b.vals[cur ^ 1], b.vals2[cur ^ 1], n, shift, (const int32_t*)b.hist, tiles));
+                  b.keys[cur ^ 1], vo, v2o, n, shift, (const int32_t*)b.hist, tiles));
     k = b.keys[cur ^ 1];
-    v = b.vals[cur ^ 1];
-    v2 = b.vals2[cur ^ 1];
+    v = vo;
+    v2 = v2o;
     cur ^= 1;
   }
   *result = cur;
@@ -429,6 +436,19 @@ __global__ void csc_keys_from_csr(const uint32_t* rkey, const uint32_t* __restri
 __global__ void nonempty_flags(const int32_t* __restrict__ ptr, int64_t rows, int32_t* __restrict__ flag) {
   for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < rows; r += (int64_t)gridDim.x * blockDim.x)
     flag[r] = ptr[r + 1] > ptr[r] ? 1 : 0;
+}
+
+// long rows of the fused layer: flag[r] = 1 when CSR row r has more than kFuseRuns runs
+__global__ void long_flags(const int32_t* __restrict__ aptr, int64_t rows, int32_t* __restrict__ flag) {
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < rows; r += (int64_t)gridDim.x * blockDim.x)
+    flag[r] = aptr[r + 1] - aptr[r] > kFuseRuns ? 1 : 0;
+}
+
+// list[ofs[r]] = r for every flagged row r (ofs = the exclusive scan of the flags)
+__global__ void compact_list(const int32_t* __restrict__ flag, const int32_t* __restrict__ ofs, int64_t rows,
+                             int32_t* __restrict__ list) {
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < rows; r += (int64_t)gridDim.x * blockDim.x)
+    if (flag[r]) list[ofs[r]] = (int32_t)r;
 }
 
 // mbase[r] = compact index of relation r's first non-empty row (pos = the scan of the flags, whose
@@ -519,32 +539,20 @@ __global__ void run_finish(const int32_t* __restrict__ u, const int32_t* __restr
 
 // Row pointers from the sorted keys: ptr[k] = first position whose key is >= k, k in [0, rows].
 // Position p owns the rows k with key[p-1] < k <= key[p] (key[-1] = -1, key[n] = rows), so every
-// entry is written exactly once and empty rows get the position of the next non-empty one.
+// entry is written exactly once and empty rows get the position of the next non-empty one.  The
+// owner of k = rows also writes n - ptr[rows] (the positions with keys past the last row) to
+// *invalid when that is given.
 __global__ void row_ptr_from_keys(const uint32_t* __restrict__ keys, int64_t n, int64_t rows,
-                                  int32_t* __restrict__ ptr) {
+                                  int32_t* __restrict__ ptr, int32_t* __restrict__ invalid) {
   for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p <= n;
        p += (int64_t)gridDim.x * blockDim.x) {
     const int64_t lo = p == 0 ? 0 : (int64_t)keys[p - 1] + 1;
     const int64_t hi = p == n ? rows : min((int64_t)keys[p], rows);
     for (int64_t k = lo; k <= hi; ++k) ptr[k] = (int32_t)p;
+    if (invalid && lo <= rows && rows <= hi) *invalid = (int32_t)(n - p);
   }
 }
 
-// CSR arrays from the sorted (row key, edge id, source id) triples.
-__global__ void csr_finish(const uint32_t* __restrict__ eid_sorted, const uint32_t* __restrict__ src_sorted,
-                           const int32_t* __restrict__ ptr, int64_t rows, int64_t E, int32_t* __restrict__ col,
-                           int32_t* __restrict__ eid, int32_t* __restrict__ invalid) {
-  const int64_t nv = ptr[rows];
-  if (blockIdx.x == 0 && threadIdx.x == 0) *invalid = (int32_t)(E - nv);
-  for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < nv;
-       p += (int64_t)gridDim.x * blockDim.x) {
-    eid[p] = (int32_t)eid_sorted[p];
-    col[p] = (int32_t)src_sorted[p];
-  }
-}
-
-// CSC arrays from the sorted (row key, edge id, destination id) triples; the relation is read off
-// the key, 1/deg_r(destination) from the CSR row pointers.
 // Out-degree of every node over all relations leaving its type (the length of its node-major row).
 __global__ void node_out_counts(const int32_t* __restrict__ cptr, GraphMeta m, int32_t* __restrict__ cnt) {
   __shared__ int64_t cbase[kMaxRels];  // CSC row of the type's node 0 in relation r, minus the type offset
@@ -566,14 +574,15 @@ __global__ void node_out_counts(const int32_t* __restrict__ cptr, GraphMeta m, i
   }
 }
 
-// CSC arrays per relation, and the node-major list of out-edges used by the backward aggregation:
-// node i's row holds, relation by relation (ascending) and in CSC order within a relation, the
-// dMs row of each edge's destination (row_base[r] + local destination id).
-__global__ void csc_finish(const uint32_t* __restrict__ key_sorted, const uint32_t* __restrict__ eid_sorted,
-                           const uint32_t* __restrict__ dst_sorted, const int32_t* __restrict__ cptr, int64_t crows,
-                           GraphMeta m, const int32_t* __restrict__ csr_ptr, const int32_t* __restrict__ nptr,
-                           int32_t* __restrict__ ccol, int32_t* __restrict__ ceid, float* __restrict__ coef,
-                           int32_t* __restrict__ ncol) {
+// CSC coefficients and the node-major list of out-edges used by the backward aggregation, from
+// the sorted CSC keys and destination ids (the sort's last pass wrote csc_col and csc_eid): the
+// relation is read off the key, 1/deg_r(destination) from the CSR row pointers.  Node i's row holds,
+// relation by relation (ascending) and in CSC order within a relation, the dMs row of each edge's
+// destination (row_base[r] + local destination id).
+__global__ void csc_finish(const uint32_t* __restrict__ key_sorted, const int32_t* __restrict__ ccol,
+                           const int32_t* __restrict__ cptr, int64_t crows, GraphMeta m,
+                           const int32_t* __restrict__ csr_ptr, const int32_t* __restrict__ nptr,
+                           float* __restrict__ coef, int32_t* __restrict__ ncol) {
   const int64_t nv = cptr[crows];
   for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < nv;
        p += (int64_t)gridDim.x * blockDim.x) {
@@ -582,11 +591,9 @@ __global__ void csc_finish(const uint32_t* __restrict__ key_sorted, const uint32
 #pragma unroll
     for (int k = 1; k < kMaxRels; ++k)
       if (k < m.num_rels && key >= m.csc_base[k]) r = k;
-    const int32_t j = (int32_t)dst_sorted[p];
+    const int32_t j = ccol[p];
     const int64_t row = m.row_base[r] + (j - m.type_off[m.rel_dst[r]]);
     const int deg = csr_ptr[row + 1] - csr_ptr[row];
-    ceid[p] = (int32_t)eid_sorted[p];
-    ccol[p] = j;
     coef[p] = __fdiv_rn(1.0f, (float)deg);
     // node-major position: the node's row start, the edges of its earlier relations, the rank in this one
     const int t = m.rel_src[r];
@@ -709,6 +716,8 @@ static int64_t order_tiles_cap(int64_t N) { return N / kProjTileRows + kMaxTypes
 // Rows above kHubDegree hold sum ceil(deg / kChunkEdges) <= E / kChunkEdges + E / (kHubDegree + 1)
 // chunks (each such row adds at most one partial chunk); +2 covers the integer floors.
 static int64_t chunk_cap(int64_t E) { return E / kChunkEdges + E / (kHubDegree + 1) + 2; }
+// a long row has more than kFuseRuns runs, each of at least one edge
+static int64_t long_cap(int64_t E) { return E / (kFuseRuns + 1) + 1; }
 
 struct GraphLayout {
   int32_t *csr_ptr, *csr_col, *csr_eid, *csc_ptr, *csc_col, *csc_eid;
@@ -720,6 +729,7 @@ struct GraphLayout {
   int32_t *bagg_ptr, *bagg_col, *bagg_cnt, *bagg_chunk_ofs, *bagg_chunk_row;
   int32_t *mrow, *mlist, *mbase;  // non-empty CSR rows: compact index per row, row per index, per relation
   int32_t *nperm, *tmask, *ohist, *oofs;  // node order by relation mask, tile masks, the sort's counts
+  int32_t *long_ofs, *long_list;          // the fused layer's long rows
   SortBuffers sort;
 };
 
@@ -750,6 +760,8 @@ static size_t carve_graph(void* ws, int64_t E, int64_t rows, int64_t crows, int6
   L->mbase = c.take<int32_t>(kMaxRels + 1);
   L->nperm = c.take<int32_t>(std::max<int64_t>(N, 1));
   L->tmask = c.take<int32_t>(order_tiles_cap(N));
+  L->long_ofs = c.take<int32_t>(rows + 1);
+  L->long_list = c.take<int32_t>(long_cap(E));
   L->ohist = c.take<int32_t>(order_hist_cap(N) + 1);
   L->oofs = c.take<int32_t>(order_hist_cap(N) + 1);
   L->invalid = c.take<int32_t>(1);
@@ -908,30 +920,30 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
     int r1 = 0;
     HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)N), (const uint32_t*)L.sort.keys[0], (const uint32_t*)nullptr,
                       (const uint32_t*)L.sort.ckeys, 0, s, &r1));
+    // the last pass writes the edge ids and source ids straight into csr_eid and csr_col
     HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)rows), (const uint32_t*)L.sort.vals2[r1],
-                      (const uint32_t*)L.sort.vals[r1], (const uint32_t*)L.sort.keys[r1], r1, s, &res));
+                      (const uint32_t*)L.sort.vals[r1], (const uint32_t*)L.sort.keys[r1], r1, s, &res,
+                      (uint32_t*)L.csr_eid, (uint32_t*)L.csr_col));
     HG_TRY(launch("row_ptr_from_keys", row_ptr_from_keys, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[res],
-                  E, rows, L.csr_ptr));
-    HG_TRY(launch("csr_finish", csr_finish, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.vals[res],
-                  (const uint32_t*)L.sort.vals2[res], (const int32_t*)L.csr_ptr, rows, E, L.csr_col, L.csr_eid,
-                  L.invalid));
-    // CSC by (source row, destination, edge id): the CSR order sorted stably by source row
+                  E, rows, L.csr_ptr, L.invalid));
+    // CSC by (source row, destination, edge id): the CSR order sorted stably by source row; the last
+    // pass writes the edge ids and destination ids straight into csc_eid and csc_col
     const int r2 = res;
     HG_TRY(launch("csc_keys_from_csr", csc_keys_from_csr, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[r2],
-                  (const uint32_t*)L.sort.vals2[r2], E, (const int32_t*)L.csr_ptr, rows, crows, m, L.sort.ckeys,
+                  (const uint32_t*)L.csr_col, E, (const int32_t*)L.csr_ptr, rows, crows, m, L.sort.ckeys,
                   L.sort.keys[r2]));
     HG_TRY(radix_sort(L.sort, E, bit_width((uint64_t)crows), (const uint32_t*)L.sort.ckeys,
-                      (const uint32_t*)L.sort.vals[r2], (const uint32_t*)L.sort.keys[r2], r2, s, &res));
+                      (const uint32_t*)L.csr_eid, (const uint32_t*)L.sort.keys[r2], r2, s, &res,
+                      (uint32_t*)L.csc_eid, (uint32_t*)L.csc_col));
     HG_TRY(launch("row_ptr_from_keys", row_ptr_from_keys, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[res],
-                  E, crows, L.csc_ptr));
+                  E, crows, L.csc_ptr, (int32_t*)nullptr));
     // node-major rows: out-degree per node over its relations, their scan, then the edges
     HG_TRY(launch("node_out_counts", node_out_counts, dim3(grid_for(N)), dim3(256), 0, s, (const int32_t*)L.csc_ptr,
                   m, L.cnt));
     HG_TRY(exclusive_scan(L.cnt, L.node_ptr, N, L.sort.scan_scratch, s));
     HG_TRY(launch("csc_finish", csc_finish, dim3(g), dim3(256), 0, s, (const uint32_t*)L.sort.keys[res],
-                  (const uint32_t*)L.sort.vals[res], (const uint32_t*)L.sort.vals2[res], (const int32_t*)L.csc_ptr,
-                  crows, m, (const int32_t*)L.csr_ptr, (const int32_t*)L.node_ptr, L.csc_col, L.csc_eid, L.csc_coef,
-                  L.node_col));
+                  (const int32_t*)L.csc_col, (const int32_t*)L.csc_ptr, crows, m, (const int32_t*)L.csr_ptr,
+                  (const int32_t*)L.node_ptr, L.csc_coef, L.node_col));
   }
   // non-empty CSR rows (the rows the mean layer stores) and their compact numbering
   HG_TRY(launch("nonempty_flags", nonempty_flags, dim3(grid_for(rows)), dim3(256), 0, s, (const int32_t*)L.csr_ptr,
@@ -946,6 +958,12 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
     HG_TRY(coalesce_runs(L.csr_col, L.csr_ptr, rows, E, nullptr, L, L.agg_col, L.agg_cnt, L.agg_ptr, s));
     HG_TRY(coalesce_runs(L.node_col, L.node_ptr, N, E, L.mrow, L, L.bagg_col, L.bagg_cnt, L.bagg_ptr, s));
   }
+  // the fused layer's long rows (more than kFuseRuns runs) and their compact slots
+  HG_TRY(launch("long_flags", long_flags, dim3(grid_for(rows)), dim3(256), 0, s, (const int32_t*)L.agg_ptr, rows,
+                L.cnt));
+  HG_TRY(exclusive_scan(L.cnt, L.long_ofs, rows, L.sort.scan_scratch, s));
+  HG_TRY(launch("compact_list", compact_list, dim3(grid_for(rows)), dim3(256), 0, s, (const int32_t*)L.cnt,
+                (const int32_t*)L.long_ofs, rows, L.long_list));
   // node order of the forward projection, per type: sorted by relation mask, and each tile's mask
   int64_t tile_base[kMaxTypes + 1] = {0};
   for (int t = 0; t < m.num_types; ++t) {
@@ -1003,6 +1021,9 @@ extern "C" hg_status hg_build_csr(const int32_t* src, const int32_t* dst, const 
   gh->mbase = L.mbase;
   gh->nperm = L.nperm;
   gh->tmask = L.tmask;
+  gh->long_ofs = L.long_ofs;
+  gh->long_list = L.long_list;
+  gh->long_cap = long_cap(E);
   for (int t = 0; t <= kMaxTypes; ++t) gh->tile_base[t] = tile_base[std::min(t, m.num_types)];
   gh->invalid_count = L.invalid;
   *out = gh;

@@ -22,6 +22,10 @@ constexpr int kProjTileRows = 128;  // output rows per tile of the tensor-core f
 // in chunk order, so the reduction order is fixed (deterministic, atomic-free).
 constexpr int kHubDegree = 512;
 constexpr int kChunkEdges = 512;
+// The fused mean layer (gathers into the projection's operand tiles) sums a CSR row in the
+// projection only up to kFuseRuns runs; the means of longer rows are computed beforehand by the
+// streaming row kernel into a compact buffer, so no row holds the tile's loads for long.
+constexpr int kFuseRuns = 32;
 
 // ---------------------------------------------------------------------------------------------
 // errors
@@ -153,6 +157,12 @@ struct hg_graph {
   int32_t* nperm;           // [N]
   int32_t* tmask;           // [tile_base[num_types]]
   int64_t tile_base[hg::kMaxTypes + 1];
+  // CSR rows with more than kFuseRuns runs (the fused layer's long rows): long_ofs = exclusive scan
+  // of the flags (row is long iff long_ofs[row + 1] > long_ofs[row]; long_ofs[row] is its compact
+  // slot, long_ofs[csr_rows] their number), long_list[k] = the CSR row of slot k.
+  int32_t* long_ofs;        // [csr_rows + 1]
+  int32_t* long_list;       // [long_cap]
+  int64_t long_cap;         // E / (kFuseRuns + 1) + 1: at most that many rows are long
   int32_t* invalid_count;  // device scalar
 };
 
