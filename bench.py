@@ -59,6 +59,7 @@ def parse():
                     help="drive the layers with a synthetic upstream gradient instead of the head and joint loss")
     ap.add_argument("--no-temporal", action="store_true", help="skip the temporal-module measurement")
     ap.add_argument("--no-hgt", action="store_true", help="skip the attention-layer measurement")
+    ap.add_argument("--no-fused", action="store_true", help="skip the fused mean layer's measurement")
     ap.add_argument("--scale", type=int, default=1, help=argparse.SUPPRESS)  # profiling: a 1/k-size instance
     ap.add_argument("--ncu-traffic", default="",
                     help="fold an ncu CSV (--metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum "
@@ -239,6 +240,7 @@ class Clocks:
 # algorithmic bytes / flops per step for each kernel (from the graph's own statistics)
 # ------------------------------------------------------------------------------------------------
 HUB, CHUNK = 512, 512
+FUSE = 32  # the fused mean layer streams rows of at most this many runs in its projection
 
 
 def _graph_of(w):
@@ -261,7 +263,8 @@ def graph_stats(w) -> dict:
     offs = [int(x) for x in g["type_offsets"]]
     N, R = offs[-1], len(g["rels"])
     nz = lambda x: int(torch.count_nonzero(x))  # noqa: E731
-    blank = lambda: dict(E_nh=0, E_h=0, R_nh=0, R_h=0, U_nh=0, U_h=0, chunks=0)  # noqa: E731
+    blank = lambda: dict(E_nh=0, E_h=0, R_nh=0, R_h=0, U_nh=0, U_h=0, chunks=0, R_short=0, U_short=0,  # noqa: E731
+                         rows_long=0)
     st = dict(N=N, E=int(src.shape[0]), RR=0, CC=0, n_ov=n_ov, fwd=blank(), bwd=blank(), types=[], rels=[])
     for t in range(len(offs) - 1):
         st["types"].append(dict(n=offs[t + 1] - offs[t], R=sum(1 for r in g["rels"] if r[1] == t), nnz=0))
@@ -287,7 +290,11 @@ def graph_stats(w) -> dict:
         a["U_nh"] += nz(torch.bincount(u_src[~hub_run], minlength=N))
         hr = runs[runs > HUB]
         a["chunks"] += int(((hr + CHUNK - 1) // CHUNK).sum())
-        del u, u_dst, u_src, runs, hub_run, edges
+        short = runs[u_dst] <= FUSE  # runs the fused projection streams itself
+        a["R_short"] += nz(short)
+        a["U_short"] += nz(torch.bincount(u_src[short], minlength=N))
+        a["rows_long"] += nz(runs > FUSE)
+        del u, u_dst, u_src, runs, hub_run, edges, short
     for r, (_, tt) in enumerate(g["rels"]):
         st["types"][tt]["nnz"] += st["rels"][r]["nnz"]  # stored relation rows (non-empty CSR rows)
     st["NNZ"] = sum(r["nnz"] for r in st["rels"])
@@ -354,6 +361,13 @@ def kernel_models(st: dict, sp) -> dict:
     m["ln_act_bwd"] = (L * lb, 0)
     m["proj_bwd_tc"] = (L * pb, L * pfl)
     m["wgrad_tc"] = (L * (2 * row + 4) * NNZ, L * 2 * d * d * NNZ)  # G_r = M_r^T dU over the stored rows
+    # the fused mean layer: the projection and the weight gradient sum the rows of at most FUSE runs
+    # themselves (run lists, 24 bytes of row metadata per stored row, each distinct source row once)
+    # and read the longer rows' means; M_r is neither written nor read back
+    fuse_in = 8 * f["R_short"] + 24 * NNZ + row * f["U_short"] + row * f["rows_long"]
+    m["proj_fwd_gather_tc"] = (L * (tf - row * NNZ + fuse_in), L * tfl)
+    m["wgrad_gather_tc"] = (L * ((row + 4) * NNZ + fuse_in), L * 2 * d * d * NNZ)
+    m["gathered"].update({"proj_fwd_gather_tc": L * f["R_short"] * (8 + row), "wgrad_gather_tc": L * f["R_short"] * (8 + row)})
     # per 8-bit pass over the keys: read and write of key, edge id and endpoint; three stable sorts
     # (by source id, then CSR row: (row, source, edge id); that order by CSC row)
     passes = lambda rows: max(1, -(-int(rows).bit_length() // 8))  # noqa: E731
@@ -731,7 +745,7 @@ def step_inputs(w: dict, use_head: bool) -> dict:
     return inp
 
 
-def make_path(w: dict, dev, use_head: bool):
+def make_path(w: dict, dev, use_head: bool, fused: bool = False):
     from paper_2608_02168_gb300.step import HotPath
     sp, g = w["spec"], w["graph"]
     return HotPath(g["type_offsets"], g["rels"], int(g["src"].shape[0]), sp.d, sp.dtype, w["params"], view=sp.view_b,
@@ -739,16 +753,29 @@ def make_path(w: dict, dev, use_head: bool):
                    n_gid_a=0 if "gid_a" not in w else int(len(w["gid_a"])),
                    n_gid_b=0 if "gid_b" not in w else int(len(w["gid_b"])), device=dev,
                    head_params=hgsynth.make_head_params(sp) if use_head else None,
-                   n_lab_max=int(len(w["lab_idx"])) if use_head else 0)
+                   n_lab_max=int(len(w["lab_idx"])) if use_head else 0, fused=fused)
 
 
-def run_hot_path(w: dict, dev, steps: int, warmup: int, world: int, use_head: bool, clocks=None, e2e: bool = False) -> dict:
+def path_digest(path) -> dict:
+    """Integer sums of the bit patterns of the path's last step: every layer output, every input
+    gradient and every weight gradient.  Equal digests of two runs mean equal results, bit for bit,
+    in practice."""
+    import torch
+
+    def bits(t):
+        return int(t.view(torch.int16 if t.element_size() == 2 else torch.int32).sum(dtype=torch.int64))
+    return {"H": [bits(t) for stack in path.H for t in stack], "dH": [bits(t) for stack in path.dH for t in stack],
+            "grads": [bits(gd[k]) for stack in path.grads for gd in stack for k in sorted(gd)]}
+
+
+def run_hot_path(w: dict, dev, steps: int, warmup: int, world: int, use_head: bool, clocks=None, e2e: bool = False,
+                 fused: bool = False) -> dict:
     """Times `steps` steps (after `warmup`), then the phases of the step and the per-kernel report;
-    optionally the same steps end to end from pinned host inputs."""
+    optionally the same steps end to end from pinned host inputs.  fused: the fused mean layer."""
     import torch
     from paper_2608_02168_gb300 import hg
     sp = w["spec"]
-    path = make_path(w, dev, use_head)
+    path = make_path(w, dev, use_head, fused)
     devin = step_inputs(w, use_head)
     stream = torch.cuda.current_stream()
 
@@ -806,8 +833,26 @@ def run_hot_path(w: dict, dev, steps: int, warmup: int, world: int, use_head: bo
         res["e2e"] = run_e2e(path, step, devin, dev, steps, world, units, use_head)
     res["loss"] = [float(x) for x in path.loss.cpu()]
     res["head_loss"] = [float(x) for x in path.head_loss.cpu()] if use_head else None
+    res["digest"] = path_digest(path)
+    res["saved_bytes_per_layer"] = int(path.saved[0][0].numel())
     del path
     return res
+
+
+def fused_summary(res: dict, rf: dict) -> dict:
+    """The fused mean layer (M_r never stored) against the plain layer on the same workload."""
+    lay = res["phases_ms"].get("forward", 0) + res["phases_ms"].get("backward", 0)
+    lay_f = rf["phases_ms"].get("forward", 0) + rf["phases_ms"].get("backward", 0)
+    per = lambda rep, k: round(rep[k][1] / rep[k][0], 4) if k in rep and rep[k][0] else None  # noqa: E731
+    kern = {k: {"ms_per_launch": per(rf["report"], k), "launches_per_step": rf["report"][k][0] / max(rf["steps"], 1)}
+            for k in ("proj_fwd_gather_tc", "wgrad_gather_tc", "agg_fwd_long_rows", "agg_fwd_chunks") if k in rf["report"]}
+    return {"ms_per_step": round(rf["ms_per_step"], 4), "phases_ms": rf["phases_ms"],
+            "layers_fwd_bwd_edges_per_s": rf["layers_fwd_bwd_edges_per_s"],
+            "layer_stack_ms": round(lay_f, 4), "plain_layer_stack_ms": round(lay, 4),
+            "bitwise_equal_to_plain": {k: rf["digest"][k] == res["digest"][k] for k in res["digest"]},
+            "saved_bytes_per_layer": rf["saved_bytes_per_layer"],
+            "plain_saved_bytes_per_layer": res["saved_bytes_per_layer"], "kernels": kern,
+            "plain_kernels": {k: per(res["report"], k) for k in ("proj_fwd_tc", "agg_fwd_rows", "wgrad_tc")}}
 
 
 def run_e2e(path, step, devin, dev, steps, world, units, use_head) -> dict:
@@ -1011,6 +1056,15 @@ def run_ours(args, sp, rank, world):
     stats = graph_stats(w)
     stats["n_lab"] = int(len(w["lab_idx"])) if use_head else 0
     models = kernel_models(stats, sp)
+    fused = None
+    if sp.dtype == "bf16" and sp.d == 128 and not args.no_fused:
+        fs = min(args.steps, 5)
+        rfu = run_hot_path(w, dev, fs, min(max(args.warmup, 1), 3), world, use_head, fused=True)
+        rfu["steps"] = fs
+        fused = fused_summary(res, rfu)
+        fused["kernel_rooflines"] = [roofline(rfu["report"], models, fs, peaks, psrc, dom=k)[0]
+                                     for k in ("proj_fwd_gather_tc", "wgrad_gather_tc") if k in rfu["report"]]
+        free_device_memory()
     head = workload_summary(w, res, models, args.steps, peaks, psrc)
     rf, shares = roofline(res["report"], models, args.steps, peaks, psrc)
     top = [k for k in shares if k in models and k != "gathered"][:8]
@@ -1065,7 +1119,7 @@ def run_ours(args, sp, rank, world):
         "layer_stack_roofline": head["layer_stack_roofline"],
         "csr_build_edges_per_s": res["csr_build_edges_per_s"],
         "cpu_baseline": cpu, "e2e": res.get("e2e"), "clocks": res["clocks"], "workloads": extra,
-        "overlap_build": build, "temporal": temporal, "hgt": hgt,
+        "overlap_build": build, "temporal": temporal, "hgt": hgt, "fused_layer": fused,
         "gpu_launches": int(sum(n for n, _ in res["report"].values())),
         "loss": res["loss"], "head_loss": res["head_loss"],
     }

@@ -184,6 +184,12 @@ typedef struct {
   const void* b_agg;
   const void* ln_gamma;
   const void* ln_beta;
+  /* 1: the fused mean layer (bf16, d = 128; else HG_ERR_UNSUPPORTED).  The relation means of rows
+   * with at most 32 runs of parallel edges are summed straight into the projection's operand tiles
+   * and never stored; the backward sums them again for the weight gradient.  Only the means of
+   * longer rows are kept in `saved`, which is then much smaller.  Results are bitwise those of
+   * fused = 0. */
+  int32_t fused;
 } hg_layer_params;
 
 /* Gradients, fp32 device arrays with the shapes of the parameters; OVERWRITTEN by hg_layer_bwd.

@@ -284,7 +284,9 @@ struct StreamCfg {
   static constexpr int kYBytes = kBwdThreads / 32 * 2 * kStreamRows * D * (int)sizeof(T);  // backward dY buffers
 };
 
-template <typename T, int D, bool kBwd>
+// kGapped: the listed rows' runs are not contiguous (a subset of the CSR rows, such as the fused
+// layer's long rows): each row's batches start at its own first run and stop at its last.
+template <typename T, int D, bool kBwd, bool kGapped = false>
 __device__ __forceinline__ void stream_rows(const int32_t* __restrict__ ptr, const int32_t* __restrict__ col,
                                             const int32_t* __restrict__ cnt, const int32_t* __restrict__ eptr,
                                             const int32_t* __restrict__ mlist, int64_t nrows,
@@ -399,6 +401,9 @@ __device__ __forceinline__ void stream_rows(const int32_t* __restrict__ ptr, con
       for (int q = 0; q < E; ++q) acc[q] = 0.f;
       ++cur;
       if (cur < nr) cend = __shfl_sync(kAll, re, cur);
+      if constexpr (kGapped) {
+        if (cur < nr) e = __shfl_sync(kAll, rb, cur);
+      }
     };
     while (cur < nr) {
       if ((hubs >> cur) & 1u) {  // a hub row: the sum of its chunk partials, in chunk-run order
@@ -418,7 +423,7 @@ __device__ __forceinline__ void stream_rows(const int32_t* __restrict__ ptr, con
       }
       // up to U runs from e on, stopping at the next hub row (whose runs are not gathered)
       const unsigned later = hubs & ~((2u << cur) - 1u);
-      const int stop = later ? __shfl_sync(kAll, rb, __ffs(later) - 1) : chunk_end;
+      const int stop = kGapped ? cend : (later ? __shfl_sync(kAll, rb, __ffs(later) - 1) : chunk_end);
       const int nb = min(U, stop - e);
       int c[U];
       float w[U];
@@ -451,13 +456,13 @@ __device__ __forceinline__ void stream_rows(const int32_t* __restrict__ ptr, con
   if constexpr (kBwd) tc::cp_async_wait<0>();  // no copy outlives the kernel
 }
 
-template <typename T, int D>
+template <typename T, int D, bool kGapped = false>
 __global__ void __launch_bounds__(StreamCfg<T, D>::kFwdThreads) agg_fwd_rows(
     const int32_t* __restrict__ ptr, const int32_t* __restrict__ col, const int32_t* __restrict__ cnt,
     const int32_t* __restrict__ eptr, const int32_t* __restrict__ mlist, const int32_t* __restrict__ nnz_p,
     const T* __restrict__ H, T* __restrict__ M, const int32_t* __restrict__ chunk_ofs,
     const float* __restrict__ partials, int32_t* __restrict__ work) {
-  stream_rows<T, D, false>(ptr, col, cnt, eptr, mlist, (int64_t)*nnz_p, H, nullptr, M, chunk_ofs, partials, work,
+  stream_rows<T, D, false, kGapped>(ptr, col, cnt, eptr, mlist, (int64_t)*nnz_p, H, nullptr, M, chunk_ofs, partials, work,
                            nullptr);
 }
 
@@ -499,10 +504,11 @@ static hg_status chunk_blocks(int64_t* blocks) {
   return HG_OK;
 }
 
-template <typename T, int D>
+// The means of the rows listed in mlist (their count at nnz_p, at most cap): the hub rows' chunk
+// partials first, then the streaming row kernel.
+template <typename T, int D, bool kGapped>
 static hg_status agg_fwd_t(const hg_graph* g, const void* H, void* M, float* partials, int32_t* work,
-                           cudaStream_t s) {
-  using S = AggShape<T, D>;
+                           const int32_t* mlist, const int32_t* nnz_p, int64_t cap, cudaStream_t s) {
   int64_t cb = 0;
   HG_TRY((chunk_blocks<T, D>(&cb)));
   HG_TRY(launch("agg_fwd_chunks", agg_chunks<T, D>, dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(g->chunk_cap_csr, cb))), dim3(256),
@@ -513,14 +519,25 @@ static hg_status agg_fwd_t(const hg_graph* g, const void* H, void* M, float* par
                 (const int32_t*)g->agg_chunk_row, (const int32_t*)g->agg_chunk_ofs, g->csr_rows, partials));
   constexpr int kT = StreamCfg<T, D>::kFwdThreads;
   static int64_t pb = 0;
-  if (pb == 0) HG_TRY(persist_blocks(agg_fwd_rows<T, D>, &pb, 0, kT));
-  const int64_t chunks = ceil_div(g->csr_rows, kStreamRows);  // a warp per chunk (the compact rows are fewer)
+  if (pb == 0) HG_TRY(persist_blocks(agg_fwd_rows<T, D, kGapped>, &pb, 0, kT));
+  const int64_t chunks = ceil_div(std::max<int64_t>(cap, 1), kStreamRows);  // a warp per chunk
   HG_CUDA(cudaMemsetAsync(work, 0, sizeof(int32_t), s));
-  return launch("agg_fwd_rows", agg_fwd_rows<T, D>,
+  return launch(kGapped ? "agg_fwd_long_rows" : "agg_fwd_rows", agg_fwd_rows<T, D, kGapped>,
                 dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(chunks, kT / 32), pb))), dim3(kT), 0,
                 s, (const int32_t*)g->agg_ptr, (const int32_t*)g->agg_col, (const int32_t*)g->agg_cnt,
-                (const int32_t*)g->csr_ptr, (const int32_t*)g->mlist, (const int32_t*)(g->mbase + g->meta.num_rels),
-                (const T*)H, (T*)M, (const int32_t*)g->agg_chunk_ofs, (const float*)partials, work);
+                (const int32_t*)g->csr_ptr, mlist, nnz_p, (const T*)H, (T*)M, (const int32_t*)g->agg_chunk_ofs,
+                (const float*)partials, work);
+}
+
+template <typename T, int D>
+static hg_status agg_fwd_dense_t(const hg_graph* g, const void* H, void* M, float* partials, int32_t* work,
+                                 const int32_t* mlist, const int32_t* nnz_p, int64_t cap, cudaStream_t s) {
+  return agg_fwd_t<T, D, false>(g, H, M, partials, work, mlist, nnz_p, cap, s);
+}
+template <typename T, int D>
+static hg_status agg_fwd_gapped_t(const hg_graph* g, const void* H, void* M, float* partials, int32_t* work,
+                                  const int32_t* mlist, const int32_t* nnz_p, int64_t cap, cudaStream_t s) {
+  return agg_fwd_t<T, D, true>(g, H, M, partials, work, mlist, nnz_p, cap, s);
 }
 
 template <typename T, int D>
@@ -567,7 +584,15 @@ static hg_status agg_bwd_t(const hg_graph* g, const void* dMs, const void* dY, v
 
 hg_status aggregate_forward(const hg_graph* g, hg_dtype dt, int d, const void* H, void* M, float* partials,
                             int32_t* work, cudaStream_t s) {
-  HG_DISPATCH_TD(dt, d, agg_fwd_t, g, H, M, partials, work, s);
+  // the non-empty rows, in compact order (at most csr_rows)
+  HG_DISPATCH_TD(dt, d, agg_fwd_dense_t, g, H, M, partials, work, (const int32_t*)g->mlist,
+                 (const int32_t*)(g->mbase + g->meta.num_rels), g->csr_rows, s);
+}
+
+hg_status aggregate_forward_long(const hg_graph* g, int d, const void* H, void* Mlong, float* partials, int32_t* work,
+                                 cudaStream_t s) {
+  HG_DISPATCH_TD(HG_BF16, d, agg_fwd_gapped_t, g, H, Mlong, partials, work, (const int32_t*)g->long_list,
+                 (const int32_t*)(g->long_ofs + g->csr_rows), g->long_cap, s);
 }
 
 hg_status aggregate_backward(const hg_graph* g, hg_dtype dt, int d, const void* dMs, const void* dY, void* dH,

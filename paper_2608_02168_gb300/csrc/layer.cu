@@ -69,7 +69,7 @@ void timing_end(int slot, cudaStream_t s) {
 static size_t elem_size(hg_dtype dt) { return dt == HG_F32 ? 4 : 2; }
 
 void carve_layer(const hg_graph* g, int d, hg_dtype dt, void* saved, void* scratch, LayerLayout* L,
-                 size_t* saved_bytes, size_t* scratch_bytes) {
+                 size_t* saved_bytes, size_t* scratch_bytes, bool fused) {
   const GraphMeta& m = g->meta;
   const int64_t N = m.type_off[m.num_types];
   const size_t b = elem_size(dt);
@@ -77,7 +77,11 @@ void carve_layer(const hg_graph* g, int d, hg_dtype dt, void* saved, void* scrat
   const size_t dd = (size_t)d * d;
   Carve s(saved), k(scratch);
   *L = LayerLayout{};
-  L->M = s.take<char>((size_t)g->csr_rows * d * b);
+  if (fused) {
+    L->Mlong = s.take<char>((size_t)std::max<int64_t>(g->long_cap, 1) * d * b);
+  } else {
+    L->M = s.take<char>((size_t)g->csr_rows * d * b);
+  }
   if (!tc) L->Z = s.take<char>((size_t)N * d * b);
   L->U = s.take<char>((size_t)N * d * b);
   L->stats = s.take<float2>(std::max<int64_t>(N, 1));
@@ -129,6 +133,10 @@ static hg_status check_params(const hg_graph* g, const hg_layer_params* p) {
   HG_REQUIRE(p->W_rel && p->W_agg && p->b_agg, "W_rel, W_agg and b_agg must be non-null");
   HG_REQUIRE(!p->layernorm || (p->ln_gamma && p->ln_beta), "layernorm needs ln_gamma and ln_beta");
   HG_REQUIRE(!p->layernorm || p->ln_eps > 0.f, "ln_eps must be > 0");
+  if (p->fused && !(p->dtype == HG_BF16 && p->d == 128)) {
+    set_error("the fused mean layer needs bf16 and d = 128 (dtype %d, d = %d)", (int)p->dtype, p->d);
+    return HG_ERR_UNSUPPORTED;
+  }
   return HG_OK;
 }
 
@@ -220,7 +228,7 @@ extern "C" hg_status hg_layer_workspace_size(const hg_graph* graph, const hg_lay
   HG_TRY(check_params(graph, params));
   HG_REQUIRE(saved_bytes && scratch_bytes, "saved_bytes and scratch_bytes must be non-null");
   LayerLayout L;
-  carve_layer(graph, params->d, params->dtype, nullptr, nullptr, &L, saved_bytes, scratch_bytes);
+  carve_layer(graph, params->d, params->dtype, nullptr, nullptr, &L, saved_bytes, scratch_bytes, params->fused != 0);
   return HG_OK;
 }
 
@@ -237,8 +245,12 @@ extern "C" hg_status hg_layer_fwd(const hg_graph* graph, const hg_layer_params* 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const int d = p->d;
   LayerLayout L;
-  carve_layer(graph, d, p->dtype, saved, scratch, &L, nullptr, nullptr);
-  HG_TRY(aggregate_forward(graph, p->dtype, d, H_in, L.M, L.agg_part, L.work, s));
+  carve_layer(graph, d, p->dtype, saved, scratch, &L, nullptr, nullptr, p->fused != 0);
+  if (p->fused) {  // only the long rows' means are formed here; the projection sums the others
+    HG_TRY(aggregate_forward_long(graph, d, H_in, L.Mlong, L.agg_part, L.work, s));
+  } else {
+    HG_TRY(aggregate_forward(graph, p->dtype, d, H_in, L.M, L.agg_part, L.work, s));
+  }
   return project_forward(graph, p, H_in, H_out, L, true, s);
 }
 
@@ -280,7 +292,18 @@ hg_status project_forward(const hg_graph* graph, const hg_layer_params* p, const
       a.ln = p->layernorm;
       a.eps = p->ln_eps;
       a.status = device_status_ptr();
-      if (a.n > 0) HG_TRY(tc_proj_forward(d, a, L.M, graph->csr_rows, L.Vt, m.num_rels, s));
+      if (a.n == 0) continue;
+      if (p->fused) {
+        a.agg_ptr = graph->agg_ptr;
+        a.agg_col = graph->agg_col;
+        a.agg_cnt = graph->agg_cnt;
+        a.csr_ptr = graph->csr_ptr;
+        a.long_ofs = graph->long_ofs;
+        a.Mlong = (const __nv_bfloat16*)L.Mlong;
+        HG_TRY(tc_proj_forward_gather(d, a, L.Vt, m.num_rels, s));
+      } else {
+        HG_TRY(tc_proj_forward(d, a, L.M, graph->csr_rows, L.Vt, m.num_rels, s));
+      }
     }
     return HG_OK;
   }
@@ -332,7 +355,7 @@ extern "C" hg_status hg_layer_bwd(const hg_graph* graph, const hg_layer_params* 
   HG_REQUIRE(dH_in != dH_out, "dH_in and dH_out must not alias");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   LayerLayout L;
-  carve_layer(graph, p->d, p->dtype, const_cast<void*>(saved), scratch, &L, nullptr, nullptr);
+  carve_layer(graph, p->d, p->dtype, const_cast<void*>(saved), scratch, &L, nullptr, nullptr, p->fused != 0);
   HG_TRY(project_backward(graph, p, H_in, dH_out, grads, L, true, true, s));
   if (dH_in) HG_TRY(aggregate_backward(graph, p->dtype, p->d, L.dMs, L.dY, dH_in, L.agg_part, L.work, s));
   return HG_OK;
@@ -431,7 +454,14 @@ hg_status project_backward(const hg_graph* graph, const hg_layer_params* p, cons
     if (!tc)
       HG_TRY(weight_grad(p->dtype, d, L.Z, off, L.dU, off, n, L.wpart, grads->dW_agg + (size_t)t * d * d, L.rtmp, s));
   }
-  if (tc && compact) {  // G_r = M_r^T dU over each relation's stored rows (dU rows gathered)
+  if (tc && p->fused) {  // G_r = M_r^T dU, the rows of M_r summed again from H_in
+    for (int r = 0; r < m.num_rels; ++r) {
+      const int t = m.rel_dst[r];
+      HG_TRY(tc_weight_grad_gather(d, graph, H_in, L.Mlong, r, m.row_base[r], L.dU, m.type_off[t],
+                                   m.type_off[t + 1] - m.type_off[t], L.wpart, L.G + (size_t)r * d * d, L.rtmp,
+                                   s));
+    }
+  } else if (tc && compact) {  // G_r = M_r^T dU over each relation's stored rows (dU rows gathered)
     for (int r = 0; r < m.num_rels; ++r) {
       const int t = m.rel_dst[r];
       HG_TRY(tc_weight_grad_rows(d, L.M, graph->csr_rows, graph->mlist, graph->mbase, r, m.row_base[r], L.dU,

@@ -61,6 +61,14 @@ struct TcFwdArgs {
   const __nv_bfloat16* M;     // relation means, [msent][D]
   const int32_t* perm;        // tile position -> local node (the type's nodes by relation mask); null: identity
   const int32_t* tmask;       // per tile, the relations (bit k = rel[k]) with a stored row in it; null: all
+  // the fused mean layer (M unused): the means are summed from H_in over the CSR runs in the
+  // projection; rows above kFuseRuns runs read theirs from Mlong at slot long_ofs[row]
+  const int32_t* agg_ptr;
+  const int32_t* agg_col;
+  const int32_t* agg_cnt;
+  const int32_t* csr_ptr;     // deg = the CSR row length
+  const int32_t* long_ofs;
+  const __nv_bfloat16* Mlong;
   int type;
   const __nv_bfloat16* b;
   const __nv_bfloat16* gamma;
@@ -106,6 +114,9 @@ hg_status tc_fuse_weights(int d, const void* W_rel, const void* W_agg, RelDst rd
                           cudaStream_t s);
 hg_status tc_proj_forward(int d, const TcFwdArgs& a, const void* M, int64_t m_rows, const void* Vt, int num_rels,
                           cudaStream_t s);
+// The fused mean layer's projection (d = 128): the relation means are summed into the operand tiles
+// from a.H_in (a.agg_ptr .. a.Mlong set; a.M unused).
+hg_status tc_proj_forward_gather(int d, const TcFwdArgs& a, const void* Vt, int num_rels, cudaStream_t s);
 hg_status tc_ln_act_backward(int d, const TcBwdArgs& a, int* blocks, cudaStream_t s);
 hg_status tc_proj_backward(int d, const TcBwdArgs& a, const void* V, int num_rels, cudaStream_t s);
 // outs[r] = X[x0[r] .. x0[r]+n)^T Y[y0 .. y0+n) for r < R (R <= wgrad_tc_max_rels(d)); the R
@@ -115,6 +126,11 @@ hg_status tc_proj_backward(int d, const TcBwdArgs& a, const void* V, int num_rel
 hg_status tc_weight_grad_rows(int d, const void* M, int64_t m_rows, const int32_t* mlist, const int32_t* mbase, int rel,
                               int64_t row0, const void* dU, int64_t y0, int64_t n, float* part, float* out, float* tmp,
                               cudaStream_t s);
+// The same with M_r's rows summed from H over the CSR runs (rows above kFuseRuns runs read from Mlong
+// at their long slot): the fused mean layer's backward (d = 128).
+hg_status tc_weight_grad_gather(int d, const hg_graph* g, const void* H, const void* Mlong, int rel, int64_t row0,
+                                const void* dU, int64_t y0, int64_t n, float* part, float* out, float* tmp,
+                                cudaStream_t s);
 hg_status tc_weight_grad(int d, const void* X, const int64_t* x0, int R, const void* Y, int64_t y0, int64_t n,
                          float* part, float* const* outs, float* tmp, cudaStream_t s);
 int wgrad_tc_max_rels(int d);
@@ -126,6 +142,10 @@ int* device_status_ptr();  // device address of the library status word
 hg_status aggregate_forward(const hg_graph* g, hg_dtype dt, int d, const void* H, void* M, float* partials,
                             int32_t* work,
                             cudaStream_t s);
+// The fused mean layer's long rows (more than kFuseRuns runs, bf16): Mlong[k] = the mean of CSR row
+// long_list[k], the same sum as aggregate_forward's.
+hg_status aggregate_forward_long(const hg_graph* g, int d, const void* H, void* Mlong, float* partials, int32_t* work,
+                                 cudaStream_t s);
 hg_status aggregate_backward(const hg_graph* g, hg_dtype dt, int d, const void* dMs, const void* dY, void* dH,
                              float* partials, int32_t* work, cudaStream_t s);
 hg_status proj_forward(hg_dtype dt, int d, const FwdArgs& a, cudaStream_t s);
@@ -153,6 +173,7 @@ hg_status rows_gemm_tc(int d, const void* A, int64_t n, const void* B, const voi
 // Buffers of one layer (saved for the backward, and scratch).
 struct LayerLayout {
   void* M;        // saved: csr_rows x d relation rows (means, or attention-weighted sums)
+  void* Mlong;    // saved (fused mean layer): long_cap x d means of the rows above kFuseRuns runs
   void* Z;        // saved (fp32 storage only): N x d
   void* U;        // saved: N x d pre-activation
   float2* stats;  // saved: N row statistics
@@ -171,8 +192,9 @@ struct LayerLayout {
   void* WrelT;    // scratch (fp32 storage only): R x d x d
   void* WaggT;    // scratch (fp32 storage only): T x d x d
 };
+// fused: the mean layer without stored relation means (L->M null; L->Mlong holds the long rows')
 void carve_layer(const hg_graph* g, int d, hg_dtype dt, void* saved, void* scratch, LayerLayout* L,
-                 size_t* saved_bytes, size_t* scratch_bytes);
+                 size_t* saved_bytes, size_t* scratch_bytes, bool fused = false);
 RelDst rel_dst_of(const GraphMeta& m);
 // Eq. 7 and Eq. 11 from the relation rows in L.M (bias, activation, residual, optional LayerNorm).
 // compact: L.M holds the non-empty CSR rows only, in the graph's compact order (the mean layer);

@@ -54,7 +54,7 @@ constexpr int kATile = kTileRows * 128;  // 128 rows x 64 bf16
 // threads per row (one per column half; eight warps, two per scheduler).  Two TMEM accumulators and
 // two residual tiles let the epilogue of one 128-row tile overlap the loads and MMAs of the next,
 // and every role loads the next tile's metadata (relations, node order, rows of M) ahead of time.
-template <int D>
+template <int D, bool kGather = false>
 struct FwdCfg {
   static constexpr int kStages = D == 256 ? 2 : (D == 128 ? 3 : 4);
   static constexpr int kB = D * 128;  // D rows x 64 bf16 (one half of the weight pair)
@@ -69,12 +69,20 @@ struct FwdCfg {
   static_assert(kSmem <= 227 * 1024, "shared memory of proj_fwd_tc");
   static constexpr int kAccCols = D < 32 ? 32 : D;
   static constexpr int kTmemCols = 2 * kAccCols;
-  static constexpr int kProducers = 64;  // threads; 64 A rows each of a stage's 128 per warp
-  static constexpr int kMmaWarp = 2;
-  static constexpr int kEpiWarp0 = 3;
+  // Roles.  Plain: warps 0-1 copy the stored rows of M (64 A rows each), warp 2 issues the MMAs,
+  // warps 3-10 run the epilogue.  Gather variant (the fused mean layer): sixteen warps whose
+  // registers are split by warpgroup (setmaxnreg): warps 0-3 and 5-7 sum the relation means into
+  // the A stages and warp 4 issues the MMAs, at kLowRegs; warps 8-15 run the epilogue at kHighRegs.
+  static constexpr int kGatherWarps = 7;
+  static constexpr int kProducers = kGather ? 32 * kGatherWarps : 64;  // producer threads (stage arrivals)
+  static constexpr int kMmaWarp = kGather ? 4 : 2;
+  static constexpr int kEpiWarp0 = kGather ? 8 : 3;
   static constexpr int kEpiThreads = 2 * kTileRows;
-  static constexpr int kThreads = 96 + kEpiThreads;
+  static constexpr int kThreads = kGather ? 512 : 96 + kEpiThreads;
   static constexpr int kHalf = D / 2;  // columns per epilogue thread
+  static constexpr int kLowRegs = 88, kHighRegs = 168;
+  // the two register levels use exactly the launch's 128 registers per thread
+  static_assert(!kGather || (256 * (kLowRegs + kHighRegs) == kThreads * 128 && kEpiWarp0 == 8), "register split");
 };
 static_assert(kTileRows == kProjTileRows, "tile of the node order");
 
@@ -104,8 +112,14 @@ __device__ __forceinline__ void store16_bf16(__nv_bfloat16* p, const float* v) {
 
 template <int D>
 __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
-    proj_fwd_tc(const __grid_constant__ CUtensorMap tm_Vt, TcFwdArgs a) {
-  using C = FwdCfg<D>;
+    proj_fwd_tc(const __grid_constant__ CUtensorMap tm_Vt, TcFwdArgs a);
+template <int D>
+__global__ void __launch_bounds__(FwdCfg<D, true>::kThreads, 1)
+    proj_fwd_gather_tc(const __grid_constant__ CUtensorMap tm_Vt, TcFwdArgs a);
+
+template <int D, bool kGather>
+__device__ __forceinline__ void proj_fwd_body(const CUtensorMap& tm_Vt, const TcFwdArgs& a) {
+  using C = FwdCfg<D, kGather>;
   constexpr int S = C::kStages;
   constexpr int KC = D / 64;        // 64-wide K chunks per D
   constexpr uint32_t kLag = S - 1;  // stages a producer thread keeps in flight before releasing one
@@ -136,6 +150,16 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
     if (m >= a.n) return -1;
     return a.perm ? (int64_t)__ldg(a.perm + m) : m;
   };
+  __shared__ int64_t s_row0[kMaxRels];  // gather variant: first CSR row and id of each relation into the type
+  __shared__ int s_rel[kMaxRels];
+  if constexpr (kGather) {
+#pragma unroll
+    for (int r = 0; r < kMaxRels; ++r)
+      if (threadIdx.x == r) {
+        s_row0[r] = a.mrow0[r];
+        s_rel[r] = a.rel[r];
+      }
+  }
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(&full[s], C::kProducers + 1);  // the producer threads and the weight loads' byte count
@@ -155,7 +179,228 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
   fence_after_sync();
   const uint32_t tmem = *tslot;
 
-  if (warp < C::kMmaWarp) {
+  auto gather_role = [&]() {
+    if constexpr (kGather) {
+      // ---- gather producers (the fused mean layer).  The seven warps' fourteen half-warps share
+      // the rows of every relation tile: half h takes rows h, h + 14, ...; lane l of a half owns
+      // 16-byte chunk l of a row (columns 8 l .. 8 l + 7, in K chunk l / 8), so one pass over a
+      // row's runs fills both K chunks' stages (g, g + 1), which are filled together.  Rows above
+      // kFuseRuns runs copy their mean from Mlong; rows without in-edges (or past the type) are
+      // zero; the other rows are streamed: batches of eight runs in row order, crossing row
+      // boundaries (each lane of the batch loads one column or count), and a row is written when
+      // the batch reaches the next one.  A row's runs are added one by one into an fp32 sum that
+      // starts at 0 and the sum is scaled by 1/deg and rounded to bf16: the streaming row
+      // kernel's arithmetic, term for term, so M's rows come out bit for bit.  Thread 0 also
+      // loads the two stages' V_r^T hi / lo chunks by TMA.  A thread arrives on both stage
+      // barriers once its rows are written and fenced for the async proxy.  Lane i < 10 of a half
+      // holds row i's metadata (run bounds, 1/deg, long slot), loaded a relation tile ahead, and
+      // the nodes a relation tile further ahead.
+      static_assert(D == 128 && KC == 2, "gather variant: d = 128");
+      constexpr int kGrp = 2 * C::kGatherWarps;                // half-warps
+      constexpr int kRowsPer = (kTileRows + kGrp - 1) / kGrp;  // rows per half and relation tile
+      static_assert(kRowsPer <= 15, "rows per half fit the 4-bit batch slots");
+      const int half = lane >> 4, hl = lane & 15;
+      const int grp = 2 * (warp < C::kMmaWarp ? warp : warp - 1) + half;
+      const int hb = half << 4;  // first lane of the half
+      const unsigned hmask = 0xffffu << hb;
+      const int myrow = grp + kGrp * hl;  // the row whose metadata this lane holds
+      const bool mine = hl < kRowsPer && myrow < kTileRows;
+      const __nv_bfloat16* Hc = a.H_in + hl * 8;
+      const uint32_t stage_s = smem_u32(stage);
+      bool ok = true;
+      uint32_t g = 0;
+      // The relation tiles of this CTA (warp-uniform): tiles blockIdx.x, + G, ..., each with the
+      // relations of its mask in ascending order (the MMA warp's order).  Lane k holds the mask of
+      // tile wb + G k of a window of 32 tiles.
+      int wb = blockIdx.x;
+      uint32_t wmask = rels_of(wb + G * lane);
+      unsigned wnz = __ballot_sync(0xffffffffu, wmask != 0u);
+      int wnext = 0;
+      uint32_t rem = 0;
+      int ctile = 0;
+      // the next relation tile: its tile and relation (r = -1 past the last)
+      auto next_rt = [&](int& tile, int& r) {
+        r = -1;
+        while (rem == 0u) {
+          const unsigned later = wnext >= 32 ? 0u : (wnz & (0xffffffffu << wnext));
+          if (later == 0u) {
+            wb += 32 * (int)G;
+            if (wb >= ntiles) return;
+            wmask = rels_of(wb + G * lane);
+            wnz = __ballot_sync(0xffffffffu, wmask != 0u);
+            wnext = 0;
+            continue;
+          }
+          const int k = __ffs(later) - 1;
+          wnext = k + 1;
+          ctile = wb + (int)G * k;
+          rem = __shfl_sync(0xffffffffu, wmask, k);
+        }
+        r = __ffs(rem) - 1;
+        rem &= rem - 1u;
+        tile = ctile;
+      };
+      // this lane's node in tile q (-1: none), and its row's metadata under relation r (r < 0: none)
+      auto node_of = [&](int q) -> int { return mine ? (int)node_at((int64_t)q * kTileRows + myrow) : -1; };
+      auto meta_of = [&](int r, int j, int& rb, int& re, int& slot, float& sc) {
+        rb = re = 0;
+        slot = -1;
+        sc = 0.f;
+        if (r >= 0 && j >= 0) {
+          const int64_t row = s_row0[r] + j;
+          rb = __ldg(a.agg_ptr + row);
+          re = __ldg(a.agg_ptr + row + 1);
+          const int l0 = __ldg(a.long_ofs + row), l1 = __ldg(a.long_ofs + row + 1);
+          const int e0 = __ldg(a.csr_ptr + row), e1 = __ldg(a.csr_ptr + row + 1);
+          if (l1 > l0) slot = l0;
+          if (e1 > e0) sc = __fdiv_rn(1.0f, (float)(e1 - e0));
+        }
+      };
+      int tile_c = 0, tile_n = 0, r_c, r_n = -1;
+      next_rt(tile_c, r_c);
+      const int j_c0 = r_c >= 0 ? node_of(tile_c) : -1;
+      if (r_c >= 0) next_rt(tile_n, r_n);
+      int j_n = r_n >= 0 ? (tile_n == tile_c ? j_c0 : node_of(tile_n)) : -1;
+      int m_rb, m_re, m_slot;
+      float m_sc;
+      meta_of(r_c, j_c0, m_rb, m_re, m_slot, m_sc);
+      while (r_c >= 0) {
+        int n_rb, n_re, n_slot;
+        float n_sc;
+        meta_of(r_n, j_n, n_rb, n_re, n_slot, n_sc);  // in flight during this relation tile
+        int tile_nn = 0, r_nn = -1;
+        if (r_n >= 0) next_rt(tile_nn, r_nn);
+        const int j_nn = r_nn >= 0 ? (tile_nn == tile_n ? j_n : node_of(tile_nn)) : -1;
+        // the streamed rows (bit i: row grp + 14 i has runs and is not long)
+        unsigned qrows = (__ballot_sync(hmask, mine && m_slot < 0 && m_rb < m_re) >> hb) & 0xffffu;
+        int qi = 0, qe = 0, qend = 0;  // queue cursor: row qi, its next run qe and end qend
+        // the next eight runs in row order: slot k's row in srow (4 bits each, 15: none); returns the
+        // entry this lane loads for them: lanes 0-7 the source column of slot l, lanes 8-15 the
+        // count of slot l - 8
+        auto fill = [&](uint32_t& srow) -> int {
+          srow = 0xffffffffu;
+          int e = -1;
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            if (qe >= qend && qrows != 0u) {
+              qi = __ffs(qrows) - 1;
+              qrows &= qrows - 1u;
+              qe = __shfl_sync(hmask, m_rb, hb + qi);
+              qend = __shfl_sync(hmask, m_re, hb + qi);
+            }
+            if (qe < qend) {
+              srow = (srow & ~(0xFu << (4 * k))) | ((uint32_t)qi << (4 * k));
+              if ((hl & 7) == k) e = qe;
+              ++qe;
+            }
+          }
+          return e >= 0 ? __ldg((hl < 8 ? a.agg_col : a.agg_cnt) + e) : 0;
+        };
+        uint32_t srow;
+        int v = fill(srow);  // the first batch's run entries, in flight while the stages are awaited
+        // ---- the relation tile's two stages
+        const uint32_t s0 = g % S, s1 = (g + 1) % S;
+        bool w_ok = true;
+        if (g >= (uint32_t)S) w_ok = mbar_wait(&empty[s0], ((g / S) - 1) & 1);
+        if (w_ok && g + 1 >= (uint32_t)S) w_ok = mbar_wait(&empty[s1], (((g + 1) / S) - 1) & 1);
+        ok = __all_sync(0xffffffffu, w_ok);
+        if (!ok) break;
+        if (threadIdx.x == 0) {
+#pragma unroll
+          for (int k = 0; k < 2; ++k) {
+            const uint32_t sk = k ? s1 : s0;
+            uint8_t* Ak = stage + sk * C::kStage;
+            mbar_expect_tx(&full[sk], 2 * C::kB);
+            tma_load_2d(Ak + kATile, &tm_Vt, k * 64, 2 * s_rel[r_c] * D, &full[sk]);                // hi
+            tma_load_2d(Ak + kATile + C::kB, &tm_Vt, k * 64, (2 * s_rel[r_c] + 1) * D, &full[sk]);  // lo
+          }
+        }
+        // this lane's 16 bytes of row rho in its K chunk's stage
+        const uint32_t A = stage_s + ((hl >> 3) ? s1 : s0) * C::kStage;
+        auto put = [&](int rho, uint4 v) {
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(A + sw128_offset(rho, (hl & 7) * 16)),
+                       "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                       : "memory");
+        };
+        // rows without gathers, by cp.async (awaited before the stages are released): a long row's
+        // mean, or zeros
+        uint8_t* Ag = stage + ((hl >> 3) ? s1 : s0) * C::kStage;
+#pragma unroll
+        for (int i = 0; i < kRowsPer; ++i) {
+          const int rho = grp + kGrp * i;
+          if (rho < kTileRows) {  // the same for the whole half
+            const int rb = __shfl_sync(hmask, m_rb, hb + i), re = __shfl_sync(hmask, m_re, hb + i);
+            const int slot = __shfl_sync(hmask, m_slot, hb + i);
+            if (slot >= 0 || rb == re)
+              cp_async16(Ag + sw128_offset(rho, (hl & 7) * 16), a.Mlong + (slot >= 0 ? (int64_t)slot * D + hl * 8 : 0),
+                         slot >= 0);
+          }
+        }
+        cp_async_commit();
+        float acc[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+        int arow = -1;  // the row being summed
+        auto flush = [&]() {
+          const float sc = __shfl_sync(hmask, m_sc, hb + arow);
+          put(grp + kGrp * arow,
+              make_uint4(pack_bf16x2(acc[0] * sc, acc[1] * sc), pack_bf16x2(acc[2] * sc, acc[3] * sc),
+                         pack_bf16x2(acc[4] * sc, acc[5] * sc), pack_bf16x2(acc[6] * sc, acc[7] * sc)));
+#pragma unroll
+          for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+        };
+        while ((srow & 0xFu) != 0xFu) {
+          uint4 x[8];
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const int c = __shfl_sync(hmask, v, hb + k);
+            x[k] = ((srow >> (4 * k)) & 0xFu) != 0xFu ? ldg16(Hc + (int64_t)c * D) : make_uint4(0u, 0u, 0u, 0u);
+          }
+          // the next batch's run entries, in flight while this batch is added
+          uint32_t nsrow;
+          const int vn = fill(nsrow);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const int rk = (int)((srow >> (4 * k)) & 0xFu);
+            if (rk == 0xF) break;
+            if (rk != arow) {
+              if (arow >= 0) flush();
+              arow = rk;
+            }
+            const float w = (float)__shfl_sync(hmask, v, hb + 8 + k);
+            float f[8];
+            unpack(x[k], f, __nv_bfloat16());
+#pragma unroll
+            for (int q = 0; q < 8; ++q) acc[q] = fmaf(w, f[q], acc[q]);
+          }
+          srow = nsrow;
+          v = vn;
+        }
+        if (arow >= 0) flush();
+        cp_async_wait<0>();  // this thread's copies of the long rows and zero rows
+        fence_async_smem();
+        mbar_arrive(&full[s0]);
+        mbar_arrive(&full[s1]);
+        g += 2;
+        __syncwarp();
+        // the next relation tile
+        r_c = r_n;
+        tile_c = tile_n;
+        m_rb = n_rb;
+        m_re = n_re;
+        m_slot = n_slot;
+        m_sc = n_sc;
+        r_n = r_nn;
+        tile_n = tile_nn;
+        j_n = j_nn;
+      }
+      if (!ok) {
+        if (lane == 0) atomicOr(a.status, kErrTimeout);
+        if (threadIdx.x == 0) drain_rounds(full, S, g);
+      }
+    }
+  };
+  auto plain_role = [&]() {
     // ---- producers.  Warp w fills rows 64 w .. 64 w + 63 of every A stage from M with cp.async:
     // one instruction copies four whole 128-byte row chunks (lane l: chunk l % 8 of row 4 k + l / 8),
     // into the 128B-swizzled layout the MMA reads; a row past the type or without a stored relation
@@ -247,7 +492,8 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
       atomicOr(a.status, kErrTimeout);
       if (t == 0) drain_rounds(full, S, g);
     }
-  } else if (warp == C::kMmaWarp) {
+  };
+  auto mma_role = [&]() {
     // ---- MMA issuer: U_tile = sum_r M_r V_r into accumulator (it & 1), over the tile's relations
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16(128, D, false, false);
@@ -295,7 +541,8 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
       }
     }
     __syncwarp();
-  } else {
+  };
+  auto epi_role = [&]() {
     // ---- epilogue: bias, activation, residual, LayerNorm.  Warp w owns TMEM lanes 32 (w % 4) ..;
     // thread (row, half) handles columns kHalf * half .. + kHalf of its row; the two halves of a
     // row add their partial sums through shared memory (a barrier per pair of warps).
@@ -518,10 +765,44 @@ __global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
     }
     if constexpr (C::kHTile) cp_async_wait<0>();  // no residual copy outlives the kernel
     if (!ok) atomicOr(a.status, kErrTimeout);
+  };
+  if constexpr (kGather) {
+    // warpgroups 0-1 (the gather warps and the MMA warp) give registers to 2-3 (the epilogue)
+    if (warp < 8) {
+      setmaxnreg_dec<C::kLowRegs>();
+      if (warp == C::kMmaWarp) {
+        mma_role();
+      } else {
+        gather_role();
+      }
+    } else {
+      setmaxnreg_inc<C::kHighRegs>();
+      epi_role();
+    }
+  } else {
+    if (warp < C::kMmaWarp) {
+      plain_role();
+    } else if (warp == C::kMmaWarp) {
+      mma_role();
+    } else {
+      epi_role();
+    }
   }
   fence_before_sync();
   __syncthreads();
   if (warp == C::kMmaWarp) tmem_dealloc(tmem, C::kTmemCols);
+}
+
+template <int D>
+__global__ void __launch_bounds__(FwdCfg<D>::kThreads, 1)
+    proj_fwd_tc(const __grid_constant__ CUtensorMap tm_Vt, TcFwdArgs a) {
+  proj_fwd_body<D, false>(tm_Vt, a);
+}
+
+template <int D>
+__global__ void __launch_bounds__(FwdCfg<D, true>::kThreads, 1)
+    proj_fwd_gather_tc(const __grid_constant__ CUtensorMap tm_Vt, TcFwdArgs a) {
+  if constexpr (D == 128) proj_fwd_body<D, true>(tm_Vt, a);
 }
 
 // Fused weights V_r = W_r W_agg[t_r] accumulated in fp64 (exact for bf16 factors of these sizes),
@@ -1270,6 +1551,260 @@ __global__ void __launch_bounds__(WgRowsCfg<D>::kThreads, 1)
   if (warp == 4) tmem_dealloc(tmem, D);
 }
 
+// The fused mean layer's weight gradient (d = 128): G_r = M_r^T dU over relation `rel`'s stored rows
+// as wgrad_rows_tc computes it, with each row of M_r summed from H over its CSR runs on the way
+// in instead of read back (a row above kFuseRuns runs reads its mean from Mlong).  Warps 0-15
+// (32 half-warps, two rows of a 64-row chunk each) stream a row's runs as the fused
+// projection does (same terms, same order: the rows come out bit for bit as the forward's) into
+// the MN-major X stage, and copy the rows' dU by cp.async into the Y stage; a stage is released
+// kLag chunks after it was filled (wait_group, proxy fence, arrive).  Warp 16's lane 0 issues the
+// MMAs; warps 0-3 then read the accumulator.  Grid (1, splits) with the plain kernel's split-K
+// partition; part[split][D][D].
+struct WgGatherCfg {
+  static constexpr int kStages = 4;
+  static constexpr int kA = 2 * 8192;  // 64 rows x 128 columns of X
+  static constexpr int kB = 2 * 8192;  // 64 rows x 128 columns of Y
+  static constexpr int kStage = kA + kB;
+  static constexpr int kSmem = kStages * kStage + 256 + 1024;
+  static_assert(kSmem <= 227 * 1024, "shared memory of wgrad_gather_tc");
+  static constexpr int kProdWarps = 16;
+  static constexpr int kRowsPer = 64 / (2 * kProdWarps);  // rows of a chunk per half-warp
+  static constexpr int kThreads = 32 * (kProdWarps + 1);
+};
+
+__global__ void __launch_bounds__(WgGatherCfg::kThreads, 1)
+    wgrad_gather_tc(const __nv_bfloat16* __restrict__ H, const __nv_bfloat16* __restrict__ Mlong,
+                    const int32_t* __restrict__ agg_ptr, const int32_t* __restrict__ agg_col,
+                    const int32_t* __restrict__ agg_cnt, const int32_t* __restrict__ csr_ptr,
+                    const int32_t* __restrict__ long_ofs, const __nv_bfloat16* __restrict__ Y,
+                    const int32_t* __restrict__ mlist, const int32_t* __restrict__ mbase, int rel, int64_t row0,
+                    int64_t ny, float* __restrict__ part, int* __restrict__ status) {
+  constexpr int D = 128;
+  using C = WgGatherCfg;
+  constexpr int S = C::kStages;
+  constexpr uint32_t kLag = S - 1;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S * C::kStage);
+  uint64_t* empty = full + S;
+  uint64_t* accb = empty + S;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(accb + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t base = mbase[rel], count = (int64_t)mbase[rel + 1] - base;
+  const int64_t nchunks = (count + 63) / 64;
+  const int64_t cps = (nchunks + gridDim.y - 1) / gridDim.y;
+  const int64_t c0 = (int64_t)blockIdx.y * cps;
+  const int CT = (int)max((int64_t)0, min(nchunks, c0 + cps) - c0);
+  if (threadIdx.x == 0) {
+    for (int st = 0; st < S; ++st) {
+      mbar_init(&full[st], 32 * C::kProdWarps);
+      mbar_init(&empty[st], 1);
+    }
+    mbar_init(accb, 1);
+    fence_mbar_init();
+  }
+  if (warp == C::kProdWarps) tmem_alloc(tslot, D);
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  const uint32_t tmem = *tslot;
+  if (warp < C::kProdWarps) {
+    // ---- producers: half-warp h takes rows h, h + 32 of every chunk; lane l of the half owns
+    // 16-byte chunk l of a row (64-wide block l / 8).  Lane i < kRowsPer of a half holds row i's
+    // metadata: its dU row (-1: none), run bounds, 1/deg and long slot.
+    constexpr int kHalves = 2 * C::kProdWarps;
+    const int half = lane >> 4, hl = lane & 15;
+    const int grp = 2 * warp + half;
+    const int hb = half << 4;
+    const unsigned hmask = 0xffffu << hb;
+    const __nv_bfloat16* Hc = H + hl * 8;
+    const uint32_t smem_s = smem_u32(smem);
+    bool ok = true;
+    uint32_t done = 0, issued = 0;
+    // the CSR row of this lane's row of chunk q (-1: none)
+    auto row_of = [&](int q) -> int {
+      const int64_t k = (c0 + q) * 64 + grp + kHalves * hl;
+      return hl < C::kRowsPer && q < CT && k < count ? __ldg(mlist + base + k) : -1;
+    };
+    auto meta_of = [&](int row, int& yr, int& rb, int& re, int& slot, float& sc) {
+      yr = -1;
+      rb = re = 0;
+      slot = -1;
+      sc = 0.f;
+      if (row >= 0) {
+        const int64_t y = (int64_t)row - row0;
+        yr = y < ny ? (int)y : -1;
+        rb = __ldg(agg_ptr + row);
+        re = __ldg(agg_ptr + row + 1);
+        const int l0 = __ldg(long_ofs + row), l1 = __ldg(long_ofs + row + 1);
+        const int e0 = __ldg(csr_ptr + row), e1 = __ldg(csr_ptr + row + 1);
+        if (l1 > l0) slot = l0;
+        if (e1 > e0) sc = __fdiv_rn(1.0f, (float)(e1 - e0));
+      }
+    };
+    int m_yr, m_rb, m_re, m_slot;
+    float m_sc;
+    meta_of(row_of(0), m_yr, m_rb, m_re, m_slot, m_sc);
+    int row_n = row_of(1);
+    for (int g = 0; g < CT && ok; ++g) {
+      int n_yr, n_rb, n_re, n_slot;
+      float n_sc;
+      meta_of(row_n, n_yr, n_rb, n_re, n_slot, n_sc);  // the next chunk's rows, in flight
+      const int row_nn = row_of(g + 2);
+      const int st = g % S;
+      if (g >= S) ok = __all_sync(0xffffffffu, mbar_wait(&empty[st], ((g / S) - 1) & 1));
+      if (!ok) break;
+      const uint32_t X = smem_s + st * C::kStage + (hl >> 3) * 8192;  // this lane's 64-wide block of X
+      uint8_t* Xg = smem + st * C::kStage + (hl >> 3) * 8192;
+      uint8_t* Ys = smem + st * C::kStage + C::kA;
+      auto put = [&](int kr, uint4 v) {
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(X + sw128_offset(kr, (hl & 7) * 16)),
+                     "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                     : "memory");
+      };
+      // dU rows (zeros for rows past the relation's count) and the rows without gathers (a long row's
+      // mean, or zeros), by cp.async
+#pragma unroll
+      for (int i = 0; i < C::kRowsPer; ++i) {
+        const int kr = grp + kHalves * i;
+        const int yr = __shfl_sync(hmask, m_yr, hb + i);
+        cp_async16(Ys + (hl >> 3) * 8192 + sw128_offset(kr, (hl & 7) * 16),
+                   Y + (yr >= 0 ? (int64_t)yr * D + hl * 8 : 0), yr >= 0);
+        const int rb = __shfl_sync(hmask, m_rb, hb + i), re = __shfl_sync(hmask, m_re, hb + i);
+        const int slot = __shfl_sync(hmask, m_slot, hb + i);
+        if (slot >= 0 || rb == re)
+          cp_async16(Xg + sw128_offset(kr, (hl & 7) * 16), Mlong + (slot >= 0 ? (int64_t)slot * D + hl * 8 : 0),
+                     slot >= 0);
+      }
+      cp_async_commit();
+      // the streamed rows
+      unsigned qrows = (__ballot_sync(hmask, hl < C::kRowsPer && m_slot < 0 && m_rb < m_re) >> hb) &
+                       ((1u << C::kRowsPer) - 1u);
+      int qi = 0, qe = 0, qend = 0;
+      auto fill = [&](uint32_t& srow) -> int {
+        srow = 0xffffffffu;
+        int e = -1;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          if (qe >= qend && qrows != 0u) {
+            qi = __ffs(qrows) - 1;
+            qrows &= qrows - 1u;
+            qe = __shfl_sync(hmask, m_rb, hb + qi);
+            qend = __shfl_sync(hmask, m_re, hb + qi);
+          }
+          if (qe < qend) {
+            srow = (srow & ~(0xFu << (4 * k))) | ((uint32_t)qi << (4 * k));
+            if ((hl & 7) == k) e = qe;
+            ++qe;
+          }
+        }
+        return e >= 0 ? __ldg((hl < 8 ? agg_col : agg_cnt) + e) : 0;
+      };
+      float acc[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+      int arow = -1;
+      auto flush = [&]() {
+        const float sc = __shfl_sync(hmask, m_sc, hb + arow);
+        put(grp + kHalves * arow,
+            make_uint4(pack_bf16x2(acc[0] * sc, acc[1] * sc), pack_bf16x2(acc[2] * sc, acc[3] * sc),
+                       pack_bf16x2(acc[4] * sc, acc[5] * sc), pack_bf16x2(acc[6] * sc, acc[7] * sc)));
+#pragma unroll
+        for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+      };
+      uint32_t srow;
+      int v = fill(srow);
+      while ((srow & 0xFu) != 0xFu) {
+        uint4 x[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const int c = __shfl_sync(hmask, v, hb + k);
+          x[k] = ((srow >> (4 * k)) & 0xFu) != 0xFu ? ldg16(Hc + (int64_t)c * D) : make_uint4(0u, 0u, 0u, 0u);
+        }
+        uint32_t nsrow;
+        const int vn = fill(nsrow);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const int rk = (int)((srow >> (4 * k)) & 0xFu);
+          if (rk == 0xF) break;
+          if (rk != arow) {
+            if (arow >= 0) flush();
+            arow = rk;
+          }
+          const float w = (float)__shfl_sync(hmask, v, hb + 8 + k);
+          float f[8];
+          unpack(x[k], f, __nv_bfloat16());
+#pragma unroll
+          for (int q = 0; q < 8; ++q) acc[q] = fmaf(w, f[q], acc[q]);
+        }
+        srow = nsrow;
+        v = vn;
+      }
+      if (arow >= 0) flush();
+      ++issued;
+      if (issued - done > kLag) {
+        cp_async_wait<kLag>();
+        fence_async_smem();
+        mbar_arrive(&full[done % S]);
+        ++done;
+      }
+      __syncwarp();
+      m_yr = n_yr;
+      m_rb = n_rb;
+      m_re = n_re;
+      m_slot = n_slot;
+      m_sc = n_sc;
+      row_n = row_nn;
+    }
+    // every chunk filled is released, also on the give-up path (nothing else is in flight)
+    cp_async_wait<0>();
+    fence_async_smem();
+    for (; done < issued; ++done) mbar_arrive(&full[done % S]);
+    if (!ok && lane == 0) atomicOr(status, kErrTimeout);
+  } else if (lane == 0) {  // ---- MMA issuer
+    const uint32_t idesc = idesc_bf16(128, D, true, true);
+    bool ok = true;
+    for (int g = 0; g < CT && ok; ++g) {
+      const int st = g % S;
+      ok = mbar_wait(&full[st], (g / S) & 1);
+      if (!ok) break;
+      fence_after_sync();
+      const uint32_t A0 = smem_u32(smem + st * C::kStage);
+      const uint32_t B = A0 + C::kA;
+#pragma unroll
+      for (int ks = 0; ks < 4; ++ks)
+        mma_bf16(tmem, desc_sw128(A0 + ks * 2048, 8192, 1024), desc_sw128(B + ks * 2048, 8192, 1024), idesc,
+                 (g > 0 || ks > 0) ? 1u : 0u);
+      mma_commit(&empty[st]);
+    }
+    if (!ok) atomicOr(status, kErrTimeout);
+    mma_commit(accb);  // also on the give-up path: the MMAs issued complete before TMEM is released
+  }
+  __syncwarp();
+  if (!mbar_wait(accb, 0)) atomicOr(status, kErrTimeout);
+  fence_after_sync();
+  if (warp < 4) {
+    const int orow = warp * 32 + lane;  // output row i (column of X)
+    float* out = part + (int64_t)blockIdx.y * D * D;
+#pragma unroll 1
+    for (int c = 0; c < D; c += 16) {
+      float v[16];
+      if (CT > 0) {
+        tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + c, v);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = 0.f;
+      }
+#pragma unroll
+      for (int i = 0; i < 16; i += 4)
+        *reinterpret_cast<float4*>(out + (int64_t)orow * D + c + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+    }
+  }
+  fence_before_sync();
+  __syncthreads();
+  if (warp == C::kProdWarps) tmem_dealloc(tmem, D);
+}
+
 // ---------------------------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------------------------
@@ -1311,6 +1846,29 @@ static hg_status tc_fwd_t(const TcFwdArgs& a0, const void* M, int64_t m_rows, co
   const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(a.n, kTileRows), sms));
   return launch("proj_fwd_tc", proj_fwd_tc<D>, dim3(grid), dim3(FwdCfg<D>::kThreads), FwdCfg<D>::kSmem, s, tm_V,
                 a);
+}
+
+template <int D>
+static hg_status tc_fwd_gather_t(const TcFwdArgs& a, const void* Vt, int num_rels, cudaStream_t s) {
+  if constexpr (D != 128) {
+    set_error("the fused mean layer needs d = 128 (d = %d)", D);
+    return HG_ERR_UNSUPPORTED;
+  } else {
+    static bool attr = false;
+    if (!attr) {
+      HG_CUDA(cudaFuncSetAttribute(proj_fwd_gather_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   FwdCfg<D, true>::kSmem));
+      attr = true;
+    }
+    CUtensorMap tm_V;
+    HG_TRY(make_tmap_bf16(&tm_V, Vt, (uint64_t)2 * num_rels * D, D, D));
+    int sms = 0, dev = 0;
+    HG_CUDA(cudaGetDevice(&dev));
+    HG_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(a.n, kTileRows), sms));
+    return launch("proj_fwd_gather_tc", proj_fwd_gather_tc<D>, dim3(grid), dim3(FwdCfg<D, true>::kThreads),
+                  FwdCfg<D, true>::kSmem, s, tm_V, a);
+  }
 }
 
 template <int D>
@@ -1404,6 +1962,35 @@ static hg_status tc_wgrad_rows_t(const void* M, int64_t m_rows, const int32_t* m
 }
 
 template <int D>
+static hg_status tc_wgrad_gather_t(const hg_graph* g, const void* H, const void* Mlong, int rel, int64_t row0,
+                                  const void* dU, int64_t y0, int64_t n, float* part, float* out, float* tmp,
+                                  cudaStream_t s) {
+  if constexpr (D != 128) {
+    set_error("the fused mean layer needs d = 128 (d = %d)", D);
+    return HG_ERR_UNSUPPORTED;
+  } else {
+    static bool attr = false;
+    if (!attr) {
+      HG_CUDA(cudaFuncSetAttribute(wgrad_gather_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, WgGatherCfg::kSmem));
+      attr = true;
+    }
+    if (n == 0) {
+      HG_CUDA(cudaMemsetAsync(out, 0, (size_t)D * D * sizeof(float), s));
+      return HG_OK;
+    }
+    // the split-K partition of the plain kernel (the stored rows, at most n, split on the device),
+    // so that the partial sums and their fixed-order reduction are the same
+    const int splits = wgrad_tc_splits(n, D);
+    HG_TRY(launch("wgrad_gather_tc", wgrad_gather_tc, dim3(1, splits), dim3(WgGatherCfg::kThreads),
+                  (size_t)WgGatherCfg::kSmem, s, (const __nv_bfloat16*)H, (const __nv_bfloat16*)Mlong,
+                  (const int32_t*)g->agg_ptr, (const int32_t*)g->agg_col, (const int32_t*)g->agg_cnt,
+                  (const int32_t*)g->csr_ptr, (const int32_t*)g->long_ofs, (const __nv_bfloat16*)dU + y0 * D,
+                  (const int32_t*)g->mlist, (const int32_t*)g->mbase, rel, row0, n, part, device_status_ptr()));
+    return reduce_partials(part, (int64_t)D * D, splits, (int64_t)D * D, out, tmp, s);
+  }
+}
+
+template <int D>
 static hg_status tc_finish_t(const float* G, const void* W_rel, const void* W_agg, RelDst rd, int num_rels,
                              int num_types, float* dW_rel, float* dW_agg, cudaStream_t s) {
   return launch("wgrad_finish", wgrad_finish<D>, dim3(D / 32, D / 32, num_rels + num_types), dim3(256),
@@ -1428,6 +2015,9 @@ hg_status tc_proj_forward(int d, const TcFwdArgs& a, const void* M, int64_t m_ro
                           cudaStream_t s) {
   HG_TC_DISPATCH(d, tc_fwd_t, a, M, m_rows, Vt, num_rels, s);
 }
+hg_status tc_proj_forward_gather(int d, const TcFwdArgs& a, const void* Vt, int num_rels, cudaStream_t s) {
+  HG_TC_DISPATCH(d, tc_fwd_gather_t, a, Vt, num_rels, s);
+}
 hg_status tc_ln_act_backward(int d, const TcBwdArgs& a, int* blocks, cudaStream_t s) {
   HG_TC_DISPATCH(d, tc_ln_act_t, a, blocks, s);
 }
@@ -1442,6 +2032,11 @@ hg_status tc_weight_grad_rows(int d, const void* M, int64_t m_rows, const int32_
                               int64_t row0, const void* dU, int64_t y0, int64_t n, float* part, float* out, float* tmp,
                               cudaStream_t s) {
   HG_TC_DISPATCH(d, tc_wgrad_rows_t, M, m_rows, mlist, mbase, rel, row0, dU, y0, n, part, out, tmp, s);
+}
+hg_status tc_weight_grad_gather(int d, const hg_graph* g, const void* H, const void* Mlong, int rel, int64_t row0,
+                                const void* dU, int64_t y0, int64_t n, float* part, float* out, float* tmp,
+                                cudaStream_t s) {
+  HG_TC_DISPATCH(d, tc_wgrad_gather_t, g, H, Mlong, rel, row0, dU, y0, n, part, out, tmp, s);
 }
 int wgrad_tc_max_rels(int d) { return d == 64 ? WgCfg<64>::kMaxR : (d == 128 ? WgCfg<128>::kMaxR : WgCfg<256>::kMaxR); }
 hg_status tc_wgrad_finish(int d, const float* G, const void* W_rel, const void* W_agg, RelDst rd, int num_rels,

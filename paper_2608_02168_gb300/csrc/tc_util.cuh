@@ -154,6 +154,18 @@ __device__ __forceinline__ bool bar_and(uint32_t id, uint32_t count, bool p) {
 }
 __device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
+// Register reconfiguration of a warpgroup (all four warps execute it): give registers back to the
+// CTA's pool, or take them from it (waits until the pool has them).  The launch's registers per
+// thread times its threads bound what the warpgroups may hold together.
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_dec() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
+}
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_inc() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
+
 // 16 consecutive fp32 columns of this thread's TMEM lane (warp w reads lanes 32 (w % 4) + 0..31).
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
   uint32_t r[16];

@@ -39,7 +39,7 @@ class hg_node_order(Structure):
 class hg_layer_params(Structure):
     _fields_ = [("d", c_int32), ("dtype", c_int32), ("act", c_int32), ("layernorm", c_int32), ("ln_eps", c_float),
                 ("W_rel", c_void_p), ("W_agg", c_void_p), ("b_agg", c_void_p), ("ln_gamma", c_void_p),
-                ("ln_beta", c_void_p)]
+                ("ln_beta", c_void_p), ("fused", c_int32)]
 
 
 class hg_layer_grads(Structure):
@@ -295,8 +295,9 @@ class LayerParams:
     """Packed device parameters of one layer (see hg_layer_params)."""
 
     def __init__(self, W_rel, W_agg, b_agg, ln_gamma=None, ln_beta=None, act: str = "relu", layernorm: bool = True,
-                 ln_eps: float = 1e-5):
+                 ln_eps: float = 1e-5, fused: bool = False):
         self.W_rel, self.W_agg, self.b_agg = W_rel.contiguous(), W_agg.contiguous(), b_agg.contiguous()
+        self.fused = bool(fused)
         self.ln_gamma = ln_gamma.contiguous() if ln_gamma is not None else None
         self.ln_beta = ln_beta.contiguous() if ln_beta is not None else None
         self.act, self.layernorm, self.ln_eps = act, layernorm, ln_eps
@@ -306,7 +307,7 @@ class LayerParams:
     def c(self) -> hg_layer_params:
         return hg_layer_params(self.d, self.dtype, ACTS[self.act], 1 if self.layernorm else 0, self.ln_eps,
                                _ptr(self.W_rel), _ptr(self.W_agg), _ptr(self.b_agg), _ptr(self.ln_gamma),
-                               _ptr(self.ln_beta))
+                               _ptr(self.ln_beta), 1 if self.fused else 0)
 
 
 def hg_layer_workspace_size(g: Graph, params: LayerParams) -> tuple:

@@ -42,7 +42,8 @@ class HotPath:
 
     def __init__(self, type_offsets, rels, num_edges: int, d: int, dtype: str, layer_params: list,
                  view: str, n_overlap_max: int, n_gid_a: int = 0, n_gid_b: int = 0, act: str = "relu",
-                 layernorm: bool = True, device="cuda", head_params: dict | None = None, n_lab_max: int = 0):
+                 layernorm: bool = True, device="cuda", head_params: dict | None = None, n_lab_max: int = 0,
+                 fused: bool = False):
         self.type_offsets = [int(x) for x in type_offsets]
         self.rels = [tuple(r) for r in rels]
         self.N = self.type_offsets[-1]
@@ -57,7 +58,8 @@ class HotPath:
             self.params.append(hg.LayerParams(
                 torch.as_tensor(p["W_rel"], device=dev).to(td), torch.as_tensor(p["W_agg"], device=dev).to(td),
                 torch.as_tensor(p["b_agg"], device=dev).to(td), torch.as_tensor(p["ln_gamma"], device=dev).to(td),
-                torch.as_tensor(p["ln_beta"], device=dev).to(td), act=act, layernorm=layernorm, ln_eps=LN_EPS))
+                torch.as_tensor(p["ln_beta"], device=dev).to(td), act=act, layernorm=layernorm, ln_eps=LN_EPS,
+                fused=fused))
         self.graph_ws = torch.empty(hg.hg_graph_workspace_size(num_edges, self.type_offsets, self.rels),
                                     dtype=torch.uint8, device=dev)
         saved_b, scratch_b = self._layer_sizes(num_edges)

@@ -46,10 +46,10 @@ def relerr(x, y) -> float:
     return float(np.abs(x - y).max() / max(np.abs(y).max(), 1e-30)) if y.size else 0.0
 
 
-def layer_params(hg, p: dict, dt: str, act="relu", layernorm=True, ln_eps=1e-5):
+def layer_params(hg, p: dict, dt: str, act="relu", layernorm=True, ln_eps=1e-5, fused=False):
     td = tdtype(dt)
     return hg.LayerParams(dev(p["W_rel"], td), dev(p["W_agg"], td), dev(p["b_agg"], td), dev(p["ln_gamma"], td),
-                          dev(p["ln_beta"], td), act=act, layernorm=layernorm, ln_eps=ln_eps)
+                          dev(p["ln_beta"], td), act=act, layernorm=layernorm, ln_eps=ln_eps, fused=fused)
 
 
 def grad_bufs(R, T, d):

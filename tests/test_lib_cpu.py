@@ -164,3 +164,33 @@ def test_device_binding_is_first_come_and_exclusive(hg):
              "assert so.hg_bind_device(1) == 2; assert so.hg_bind_device(-1) == 1; print('ok')")
     r = subprocess.run([sys.executable, "-c", child], capture_output=True, text=True, timeout=120)
     assert r.returncode == 0 and r.stdout.strip() == "ok", r.stdout + r.stderr
+
+
+def test_binding_structs_match_the_header(hg, tmp_path):
+    """Every ctypes struct of the binding has the size and field offsets the C compiler gives the
+    struct of the same name in include/hg.h (the argument structs cross the ABI by pointer)."""
+    import shutil
+    import subprocess
+    if shutil.which("gcc") is None:
+        pytest.skip("no C compiler")
+    structs = [c for c in vars(hg).values()
+               if isinstance(c, type) and issubclass(c, ctypes.Structure) and c.__name__.startswith("hg_")]
+    assert any(c.__name__ == "hg_layer_params" for c in structs)
+    lines = ['#include <stddef.h>', '#include <stdio.h>', '#include "hg.h"', "int main(void) {"]
+    for c in structs:
+        lines.append(f'  printf("{c.__name__} size %zu\\n", sizeof({c.__name__}));')
+        for f in c._fields_:
+            lines.append(f'  printf("{c.__name__} {f[0]} %zu\\n", offsetof({c.__name__}, {f[0]}));')
+    lines.append("  return 0;\n}")
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines))
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-std=c11", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)], check=True)
+    got = {}
+    for line in subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.splitlines():
+        name, field, val = line.split()
+        got[(name, field)] = int(val)
+    for c in structs:
+        assert got[(c.__name__, "size")] == ctypes.sizeof(c), c.__name__
+        for f in c._fields_:
+            assert got[(c.__name__, f[0])] == getattr(c, f[0]).offset, (c.__name__, f[0])
