@@ -66,6 +66,13 @@ def test_graph_stats_follow_the_kernels_rows():
     assert st["bwd"]["U_h"] == len({x for u, h in zip(b_runs, hub) if h for x in u})
     assert st["bwd"]["U_nh"] == len({x for u, h in zip(b_runs, hub) if not h for x in u})
     assert st["E"] == st["fwd"]["E_h"] + st["fwd"]["E_nh"] == st["bwd"]["E_h"] + st["bwd"]["E_nh"]
+    # the fused layer's split: rows of at most FUSE runs are streamed by its kernels, longer rows
+    # are summed beforehand (their means stored)
+    F = bench.FUSE
+    assert any(len(u) > F for _, u, _ in f_small), "the case needs long rows below the hub size"
+    assert st["fwd"]["R_short"] == sum(len(u) for _, u, _ in f_runs if len(u) <= F)
+    assert st["fwd"]["U_short"] == len({(r, x) for r, u, _ in f_runs if len(u) <= F for x in u})
+    assert st["fwd"]["rows_long"] == sum(1 for _, u, _ in f_runs if len(u) > F)
     # runs are far fewer than edges in this recipe (Zipf sources meet Zipf destinations)
     assert st["fwd"]["R_h"] + st["fwd"]["R_nh"] < 0.8 * st["E"]
 
@@ -83,6 +90,14 @@ def test_aggregation_models_are_compulsory_bytes():
                             for r in range(sp.num_rels))
     assert m["agg_fwd_rows"][0] == L * (12 * st["NNZ"] + 8 * f["R_nh"] + row * f["U_nh"] + row * st["NNZ"] +
                                         4 * sp.d * f["chunks"])
+    # the fused layer reads no stored mean for the short rows: the projection's model is the plain
+    # one without the stored rows' read, plus run lists, row metadata and source rows of the short
+    # rows and the long rows' means; the weight gradient's reads dU and the same gather inputs
+    fuse_in = 8 * f["R_short"] + 24 * st["NNZ"] + row * f["U_short"] + row * f["rows_long"]
+    assert m["proj_fwd_gather_tc"][0] == m["proj_fwd_tc"][0] - L * row * st["NNZ"] + L * fuse_in
+    assert m["proj_fwd_gather_tc"][1] == m["proj_fwd_tc"][1]
+    assert m["wgrad_gather_tc"][0] == L * ((row + 4) * st["NNZ"] + fuse_in)
+    assert m["gathered"]["proj_fwd_gather_tc"] == L * f["R_short"] * (8 + row)
     # one gathered row and run entry per run, over both kernels of a direction
     runs_f = st["fwd"]["R_h"] + st["fwd"]["R_nh"]
     assert m["gathered"]["agg_fwd_rows"] + m["gathered"]["agg_fwd_chunks"] == L * runs_f * (8 + row)
