@@ -164,7 +164,7 @@ extern "C" const char* hg_status_string(hg_status s) {
 }
 
 extern "C" const char* hg_last_error(void) { return g_err; }
-extern "C" int32_t hg_abi_version(void) { return 1; }
+extern "C" int32_t hg_abi_version(void) { return 2; }
 
 extern "C" hg_status hg_device_status(int32_t* flags) {
   clear_error();

@@ -34,7 +34,7 @@ def test_every_declared_symbol_is_exported(hg):
 
 def test_status_strings_and_version(hg):
     so = hg.lib()
-    assert so.hg_abi_version() == 1
+    assert so.hg_abi_version() == 2  # hg_layer_params gained `fused`
     assert so.hg_status_string(0) == b"ok"
     assert so.hg_status_string(3) == b"workspace too small"
 
