@@ -120,6 +120,39 @@ def test_full_layer_sampled_rows(full):
         assert relerr(host(grads[k]), v) <= tol, (k, relerr(host(grads[k]), v))
 
 
+def test_full_fused_layer_equals_plain(full):
+    """The fused mean layer (relation means never stored) against the plain layer at full size, bit
+    for bit: outputs, input gradients and every weight gradient (the plain layer is checked against
+    the definition above)."""
+    hg, sp, w, G = full
+    if not (sp.dtype == "bf16" and sp.d == 128):
+        pytest.skip("the fused layer is built for bf16, d = 128")
+    g = w.graph
+    X = dev(w.X, torch.bfloat16)
+    dH_out = dev(w.dH_top, torch.bfloat16)
+    res = []
+    for fused in (False, True):
+        P = layer_params(hg, w.params[0], "bf16", fused=fused)
+        sb, kb = hg.hg_layer_workspace_size(G, P)
+        saved = torch.empty(sb, dtype=torch.uint8, device="cuda")
+        scratch = torch.empty(kb, dtype=torch.uint8, device="cuda")
+        out = torch.empty_like(X)
+        hg.hg_layer_fwd(G, P, X, out, saved, scratch)
+        dH_in = torch.empty_like(X)
+        grads = grad_bufs(len(g["rels"]), 2, sp.d)
+        hg.hg_layer_bwd(G, P, X, saved, dH_out, dH_in, grads, scratch)
+        torch.cuda.synchronize()
+        res.append((out, dH_in, grads, sb))
+        del saved, scratch
+    (o0, d0, g0, s0), (o1, d1, g1, s1) = res
+    assert s1 < s0
+    assert torch.equal(o0.view(torch.int16), o1.view(torch.int16)), "H_out"
+    assert torch.equal(d0.view(torch.int16), d1.view(torch.int16)), "dH_in"
+    for k in g0:
+        assert torch.equal(g0[k], g1[k]), k
+    assert hg.hg_device_status() == 0
+
+
 def test_full_overlap_and_alignment(full):
     hg, sp, w, G = full
     td = tdtype(sp.dtype)
