@@ -38,6 +38,8 @@ class HotPath:
                          (rows found by intersecting the two global-id lists);
           "perturbed" -> the second view is a second live stack run on other input features over the
                          same graph, aligned on the given overlap rows, with gradients into both.
+    fused: run every layer as the fused mean layer (bf16, d = 128; the relation means are not kept
+           between the forward and the backward pass, results unchanged bit for bit).
     """
 
     def __init__(self, type_offsets, rels, num_edges: int, d: int, dtype: str, layer_params: list,
